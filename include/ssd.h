@@ -1,0 +1,218 @@
+/*
+ * ssd.h -- C ABI of the GB300 (sm_103a) self-speculative decoding library.
+ *
+ * Method: FastVLM, "Self-Speculative Decoding for Fast Vision-Language Model
+ * Inference" (arXiv 2510.22641).  Problem statement (Sec. "SSD Setup for
+ * VLMs"): the encoder output z = E(I, T0) and the prompt enter the decoder,
+ * which emits greedy tokens y^{t+1} .. y^T.  The decoder has L layers
+ * x_{l+1} = x_l + f_l(x_l) and an LM head o = g(x_L); greedy decoding takes
+ * argmax softmax(o).  Self-speculative decoding (Sec. 3.1 and Algorithm 1):
+ * the first n layers (here k) plus the imitation network I form the draft
+ * model, which proposes d (here gamma) tokens autoregressively with
+ * argmax g(I(x_k)); the full decoder then verifies them in one
+ * non-autoregressive pass, keeps the longest matching prefix and appends its
+ * own token at the first mismatch.  Draft and full model share one KV cache
+ * (Sec. "Methodology", KV cache).
+ *
+ * Conventions for every entry point:
+ *  - Pointers documented "device" must be CUDA device pointers on the device
+ *    that was current at ssd_create; "host" pointers are ordinary CPU memory.
+ *  - Weights are BORROWED: the caller owns them and must keep them alive and
+ *    unchanged (except resid_scale / in_scale, see below) until ssd_destroy.
+ *    Everything else (KV cache, workspaces, CUDA graphs) is owned by the ctx.
+ *  - A ctx is bound to one CUDA stream and is not thread-safe.  Calls marked
+ *    "async" only enqueue work on that stream; "sync" calls wait for it.
+ *  - No C++ exception crosses this boundary.  Every call returns an
+ *    ssd_status; on failure ssd_last_error(ctx) holds a message.  A device-side
+ *    fault detected by the kernels (bad token id, a bounded wait that ran out)
+ *    sets an error word that the next sync call reports as SSD_ERR_DEVICE or
+ *    SSD_ERR_TIMEOUT.
+ *  - Sizes: d_model, d_ff and in_hidden must be multiples of 64 and
+ *    n_heads*head_dim a multiple of 128; head_dim must be 64 or 128;
+ *    1 <= gamma <= gamma_max <= SSD_MAX_GAMMA.
+ */
+#ifndef SSD_H_
+#define SSD_H_
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SSD_API __attribute__((visibility("default")))
+#else
+#define SSD_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SSD_OK = 0,
+  SSD_ERR_INVALID_ARG = 1,  /* null pointer, bad size, unsupported shape */
+  SSD_ERR_OOM = 2,          /* a device allocation failed */
+  SSD_ERR_CUDA = 3,         /* a CUDA runtime call failed */
+  SSD_ERR_CAPACITY = 4,     /* n_vis + n_prompt + max_new + gamma + 1 > max_seq */
+  SSD_ERR_STATE = 5,        /* call out of order (e.g. verify without a draft) */
+  SSD_ERR_TIMEOUT = 6,      /* a bounded device wait ran out */
+  SSD_ERR_DEVICE = 7,       /* the kernels flagged bad input (e.g. token id >= vocab) */
+  SSD_ERR_UNSUPPORTED = 8   /* no sm_103a device / feature missing */
+} ssd_status;
+
+/* Imitation network variants (Sec. "Methodology", Deep Representation Imitation). */
+enum {
+  SSD_IN_IDENTITY = 0,  /* draft without imitation: g(x_k) ("Draft w/o Im", Table 1) */
+  SSD_IN_MLP2 = 1       /* x + s_in * W2 SiLU(W1 RMSNorm_in(x)): two FC layers + one norm */
+};
+
+#define SSD_MAX_GAMMA 8
+#define SSD_MAX_ROWS 16   /* rows one decode pass may carry (gamma + 1, prefill chunk) */
+
+typedef struct ssd_ctx ssd_ctx;
+
+/* Model shape and decoding limits.  The decoder is a pre-norm LLaMA block stack
+ * (RMSNorm, rotary multi-head attention, SwiGLU MLP). */
+typedef struct {
+  int n_layers;      /* L */
+  int d_model;       /* hidden width */
+  int n_heads;
+  int head_dim;      /* 64 or 128 */
+  int d_ff;          /* SwiGLU width */
+  int vocab;         /* |V| */
+  int draft_exit_k;  /* k (the paper's n): draft = layers 0..k-1, 1 <= k <= L */
+  int in_kind;       /* SSD_IN_* */
+  int in_hidden;     /* width of the imitation network's first FC layer */
+  int gamma_max;     /* largest gamma (the paper's d) any call will use */
+  int max_seq;       /* KV cache capacity in positions */
+  float rms_eps;     /* RMSNorm epsilon */
+  float rope_theta;  /* rotary base, rotate-half pairing (i, i + head_dim/2) */
+  int eos_id;        /* end-of-sequence token, -1 = disabled */
+} ssd_config;
+
+/* Model weights, all device pointers, bf16, nn.Linear layout [out][in], borrowed. */
+typedef struct {
+  const void* embed;       /* [vocab][d_model] */
+  const void* lm_head;     /* [vocab][d_model], shared by draft and full model */
+  const void* final_norm;  /* [d_model], RMSNorm gain inside g(.) */
+  /* host arrays of n_layers device pointers each */
+  const void* const* wq;        /* [n_heads*head_dim][d_model] */
+  const void* const* wk;        /* [n_heads*head_dim][d_model] */
+  const void* const* wv;        /* [n_heads*head_dim][d_model] */
+  const void* const* wo;        /* [d_model][n_heads*head_dim] */
+  const void* const* w_gate;    /* [d_ff][d_model] */
+  const void* const* w_up;      /* [d_ff][d_model] */
+  const void* const* w_down;    /* [d_model][d_ff] */
+  const void* const* attn_norm; /* [d_model] */
+  const void* const* ffn_norm;  /* [d_model] */
+  /* imitation network (ignored for SSD_IN_IDENTITY) */
+  const void* in_norm;     /* [d_model] */
+  const void* in_w1;       /* [in_hidden][d_model] */
+  const void* in_w2;       /* [d_model][in_hidden] */
+  /* fp32 device scalars read at every launch, so they may be changed between
+   * decode calls: s_l scales both residual writes of layer l, s_in the IN's. */
+  const float* resid_scale; /* [n_layers] */
+  const float* in_scale;    /* [1] */
+} ssd_weights;
+
+/* Counters of the last prefill+decode, read back by ssd_get_stats. */
+typedef struct {
+  int64_t steps;          /* verify passes (SSD) or tokens (greedy) after the prefill */
+  int64_t drafted;        /* sum of gamma_eff over steps */
+  int64_t accepted;       /* sum of accepted drafts a over steps */
+  int64_t emitted;        /* tokens emitted, including the prefill's */
+  int64_t accept_hist[SSD_MAX_GAMMA + 1]; /* steps with a = 0 .. SSD_MAX_GAMMA */
+  int64_t kv_len;         /* valid cache length at the end */
+} ssd_stats;
+
+/* Create a context: checks the shape, builds TMA descriptors for the borrowed
+ * weights, allocates the KV cache [L][H][max_seq][head_dim] bf16 (K and V),
+ * activations and workspaces on the current device.  cuda_stream is a
+ * cudaStream_t (NULL = legacy default stream).  sync. */
+SSD_API ssd_status ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, ssd_ctx** out);
+
+/* Free everything the ctx owns (not the weights).  sync.  NULL is accepted. */
+SSD_API ssd_status ssd_destroy(ssd_ctx* ctx);
+
+/* Prefill (Sec. "SSD Setup for VLMs": z is the decoder's input).  Rows
+ * [vis_emb (n_vis rows); embed(prompt)] at positions 0..P-1, P = n_vis + n_prompt,
+ * run through all L layers; K/V of every layer for positions 0..P-1 are
+ * written; the greedy token of the last row is written to first_tok.
+ *   vis_emb:   device bf16 [n_vis][d_model] (may be NULL when n_vis == 0)
+ *   prompt:    device int32 [n_prompt], each in [0, vocab)
+ *   first_tok: device int32 [1] (may be NULL)
+ * Resets the decode state: kv_len = P, one token emitted.  async. */
+SSD_API ssd_status ssd_prefill(ssd_ctx* ctx, const void* vis_emb, int n_vis, const int32_t* prompt,
+                       int n_prompt, int32_t* first_tok);
+
+/* Drafting stage (Sec. 3.1; Algorithm 1, draft loop): gamma tokens
+ * d_j = argmax g(I(x_k)) from the current token, each from layers 0..k-1 and
+ * the imitation network, writing the shallow layers' K/V at positions
+ * kv_len .. kv_len+gamma-1.  draft_tok: device int32 [gamma] (may be NULL).
+ * Needs a prefill first.  async. */
+SSD_API ssd_status ssd_draft(ssd_ctx* ctx, int gamma, int32_t* draft_tok);
+
+/* Verification stage and acceptance (Algorithm 1, verify loop): the full
+ * model runs once over the gamma+1 rows [y, d_1..d_gamma] at positions
+ * kv_len..kv_len+gamma (shallow rows reused from the draft), f_i = argmax
+ * g(x_L) per row; a = longest prefix with d_{i+1} == f_i; emits d_1..d_a and
+ * f_a; kv_len += a + 1 (rollback by length).  gamma must equal the preceding
+ * ssd_draft's.  n_emitted: device int32 [1], emitted: device int32
+ * [gamma + 1] (each may be NULL).  async. */
+SSD_API ssd_status ssd_verify(ssd_ctx* ctx, int gamma, int32_t* n_emitted, int32_t* emitted);
+
+/* Whole SSD decode after ssd_prefill, as one CUDA-graph launch whose loop runs
+ * on the device (a conditional WHILE node): steps of draft + verify + accept
+ * until max_new tokens (counting the prefill's) are out or eos is emitted.
+ * In the last steps gamma_eff = min(gamma, remaining - 1).
+ *   out_tok: device int32 [max_new] (all tokens incl. the prefill's)
+ *   n_out:   device int32 [1]
+ * async. */
+SSD_API ssd_status ssd_decode(ssd_ctx* ctx, int max_new, int gamma, int32_t* out_tok, int32_t* n_out);
+
+/* Baseline: plain greedy decoding with the full model (same kernels, one
+ * token per step, device-side loop).  Same buffers as ssd_decode.  async. */
+SSD_API ssd_status ssd_greedy_decode(ssd_ctx* ctx, int max_new, int32_t* out_tok, int32_t* n_out);
+
+/* End-to-end call with HOST buffers: copies vis_emb (bf16 [n_vis][d_model])
+ * and prompt (int32 [n_prompt]) to the device, prefill, SSD decode, copies the
+ * tokens back.  out: host int32 [max_new]; n_out: host; stats may be NULL.
+ * sync. */
+SSD_API ssd_status ssd_generate(ssd_ctx* ctx, const void* vis_emb, int n_vis, const int32_t* prompt,
+                        int n_prompt, int max_new, int gamma, int32_t* out, int* n_out,
+                        ssd_stats* stats);
+
+/* Same as ssd_generate with greedy decoding of the full model. sync. */
+SSD_API ssd_status ssd_greedy_generate(ssd_ctx* ctx, const void* vis_emb, int n_vis, const int32_t* prompt,
+                               int n_prompt, int max_new, int32_t* out, int* n_out,
+                               ssd_stats* stats);
+
+/* Wait for the ctx stream and report device-side errors.  sync. */
+SSD_API ssd_status ssd_sync(ssd_ctx* ctx);
+
+/* Counters of the last decode (see ssd_stats).  sync. */
+SSD_API ssd_status ssd_get_stats(ssd_ctx* ctx, ssd_stats* stats);
+
+/* Debug capture of the full model's logits: when buf (device fp32
+ * [max_rows][vocab]) is non-NULL, every full-model LM-head row writes its
+ * logits to row (position + 1 - P) -- the index of the token it predicts --
+ * if that index is < max_rows.  Rows of rejected drafts are overwritten by
+ * later steps.  NULL disables.  Takes effect for graphs built afterwards
+ * (the ctx rebuilds them).  sync. */
+SSD_API ssd_status ssd_set_logits_capture(ssd_ctx* ctx, float* buf, int max_rows);
+
+/* Device pointers to the KV cache, layout [L][n_heads][max_seq][head_dim]
+ * bf16, and the current valid length (sync read).  Positions >= kv_len hold
+ * stale rows of rejected drafts. */
+SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v_cache, int* kv_len);
+
+/* Number of kernel launches the last ssd_decode / ssd_greedy_decode /
+ * ssd_prefill performed (from the device step counter).  sync. */
+SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches, int64_t* decode_launches);
+
+SSD_API const char* ssd_status_string(ssd_status s);
+SSD_API const char* ssd_last_error(const ssd_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SSD_H_ */

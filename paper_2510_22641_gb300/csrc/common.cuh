@@ -1,0 +1,142 @@
+// Shared device definitions of the SSD library: device state, PTX wrappers
+// (mbarrier, TMA bulk/tensor copies, programmatic dependent launch) and
+// bounded waits.  sm_103a only.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ssd.h"
+
+namespace ssd {
+
+constexpr int kMaxRows = SSD_MAX_ROWS;
+
+// Device error bits (DevState::error).
+enum : int { DERR_TOKEN = 1, DERR_TIMEOUT = 2, DERR_POS = 4 };
+
+// Decode state kept in device memory so that a captured graph replays the
+// whole draft/verify/accept loop without host round trips.
+struct DevState {
+  int kv_len;      // valid cache length p == position of the current token y
+  int cur_tok;     // y: last emitted token, not yet in the cache
+  int n_out;       // tokens emitted so far (the prefill's first token included)
+  int max_new;     // stop after this many tokens
+  int gamma;       // draft length of the running decode
+  int done;        // 1 once max_new tokens are out or eos was emitted
+  int error;       // DERR_* bits
+  int prompt_len;  // P
+  int steps;       // verify passes / greedy steps since the prefill
+  int drafted;     // sum of gamma_eff
+  int accepted;    // sum of a
+  int last_n;      // tokens emitted by the last accept
+  int eos_id;
+  int pad[3];
+  int hist[SSD_MAX_GAMMA + 1];   // steps per accepted length a
+  int tok_in[kMaxRows];          // verify rows t_0 = y, t_j = d_j
+  int full_tok[kMaxRows];        // f_i = full-model argmax of row i
+  int last_emitted[kMaxRows];
+  unsigned long long am_key[kMaxRows];  // packed argmax accumulators (LM head)
+  unsigned int am_count;                // LM-head row tiles finished
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void fence_mbar_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t globaltimer_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Waits for the phase with the given parity; gives up after ~2 s and returns false.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const uint64_t t0 = globaltimer_ns();
+  for (uint32_t i = 1;; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((i & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) return false;
+  }
+}
+
+// 2D tiled TMA load of one box into shared memory, completing on `bar`.
+__device__ __forceinline__ void tma_load_2d(void* dst, const CUtensorMap* map, uint64_t* bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(smem_u32(dst)), "l"(map), "r"(x), "r"(y), "r"(smem_u32(bar))
+      : "memory");
+}
+
+// Untiled bulk copy global -> shared (16-byte aligned, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(dst)), "l"(src), "r"(bytes), "r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void prefetch_tensormap(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(map) : "memory");
+}
+
+// Programmatic dependent launch: wait for the upstream grid's memory, and let
+// the downstream grid start its prologue early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Named barrier among the first `nthreads` threads (consumer warps only).
+__device__ __forceinline__ void named_bar_sync(int id, int nthreads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(nthreads) : "memory");
+}
+
+__device__ __forceinline__ float2 bf16x2_to_float2(uint32_t w) {
+  return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xFFFF0000u));
+}
+
+__device__ __forceinline__ float silu_f(float v) { return v / (1.0f + expf(-v)); }
+
+// Total order on floats as unsigned keys (larger float -> larger key).
+__device__ __forceinline__ uint32_t orderable(float f) {
+  uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+// Packed (logit, index) key: max picks the largest logit, ties the lowest index.
+__device__ __forceinline__ unsigned long long argmax_key(float logit, uint32_t idx) {
+  return (static_cast<unsigned long long>(orderable(logit)) << 32) | (0xFFFFFFFFu - idx);
+}
+
+__device__ __forceinline__ void set_error(DevState* st, int bits) { atomicOr(&st->error, bits); }
+
+}  // namespace ssd

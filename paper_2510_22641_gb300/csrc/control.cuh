@@ -1,0 +1,214 @@
+// Small kernels around the projections: embedding gather, prefill rows, the
+// greedy acceptance / rollback of Algorithm 1, the greedy baseline's step, and
+// the device-side loop control of the decode graphs.
+#pragma once
+
+#include "common.cuh"
+
+namespace ssd {
+
+// x[m][:] = fp32(E[tok[m]][:]) -- the embedding layer that maps token ids to x_0.
+__global__ void embed_kernel(const __nv_bfloat16* __restrict__ E, const int* tok, float* x, int x_stride, int d,
+                             int vocab, DevState* st) {
+  pdl_trigger();
+  pdl_wait();
+  const int m = blockIdx.x;
+  int t = __ldcg(tok + m);
+  if (t < 0 || t >= vocab) {
+    if (threadIdx.x == 0) set_error(st, DERR_TOKEN);
+    t = 0;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(E + static_cast<size_t>(t) * d);
+  float4* dst = reinterpret_cast<float4*>(x + static_cast<size_t>(m) * x_stride);
+  for (int i = threadIdx.x; i < d / 8; i += blockDim.x) {
+    const uint4 v = __ldg(src + i);
+    const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y), c = bf16x2_to_float2(v.z),
+                 e = bf16x2_to_float2(v.w);
+    dst[2 * i] = make_float4(a.x, a.y, b.x, b.y);
+    dst[2 * i + 1] = make_float4(c.x, c.y, e.x, e.y);
+  }
+}
+
+// Prefill input rows r0 + m of [z (n_vis rows); embed(prompt)] (Sec. "SSD Setup for VLMs": z is fed
+// to the decoder as its first input rows).
+__global__ void prefill_rows_kernel(const __nv_bfloat16* __restrict__ vis, const int* __restrict__ prompt, int n_vis,
+                                    int r0, const __nv_bfloat16* __restrict__ E, int vocab, float* x, int x_stride,
+                                    int d, DevState* st) {
+  pdl_trigger();
+  pdl_wait();
+  const int m = blockIdx.x, r = r0 + m;
+  const __nv_bfloat16* row;
+  if (r < n_vis) {
+    row = vis + static_cast<size_t>(r) * d;
+  } else {
+    int t = __ldg(prompt + (r - n_vis));
+    if (t < 0 || t >= vocab) {
+      if (threadIdx.x == 0) set_error(st, DERR_TOKEN);
+      t = 0;
+    }
+    row = E + static_cast<size_t>(t) * d;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(row);
+  float4* dst = reinterpret_cast<float4*>(x + static_cast<size_t>(m) * x_stride);
+  for (int i = threadIdx.x; i < d / 8; i += blockDim.x) {
+    const uint4 v = __ldg(src + i);
+    const float2 a = bf16x2_to_float2(v.x), b = bf16x2_to_float2(v.y), c = bf16x2_to_float2(v.z),
+                 e = bf16x2_to_float2(v.w);
+    dst[2 * i] = make_float4(a.x, a.y, b.x, b.y);
+    dst[2 * i + 1] = make_float4(c.x, c.y, e.x, e.y);
+  }
+}
+
+__global__ void prefill_begin_kernel(DevState* st, int P, int eos_id) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  st->kv_len = 0;
+  st->prompt_len = P;
+  st->n_out = 0;
+  st->done = 0;
+  st->error = 0;
+  st->eos_id = eos_id;
+  st->steps = st->drafted = st->accepted = 0;
+  for (int i = 0; i <= SSD_MAX_GAMMA; ++i) st->hist[i] = 0;
+  for (int i = 0; i < kMaxRows; ++i) st->am_key[i] = 0ull;
+  st->am_count = 0u;
+}
+
+// The last prompt row's greedy token is the first new token; the cache now holds positions 0..P-1.
+__global__ void prefill_finish_kernel(DevState* st, int* out_tok, int P) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  const int y = st->full_tok[0];
+  st->cur_tok = y;
+  st->tok_in[0] = y;
+  st->kv_len = P;
+  st->n_out = 1;
+  st->max_new = 1 << 30;
+  out_tok[0] = y;
+  st->last_n = 1;
+  st->last_emitted[0] = y;
+  st->done = (st->eos_id >= 0 && y == st->eos_id) ? 1 : 0;
+}
+
+__global__ void decode_setup_kernel(DevState* st, int max_new, int gamma) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  st->max_new = max_new;
+  st->gamma = gamma;
+  st->steps = st->drafted = st->accepted = 0;
+  for (int i = 0; i <= SSD_MAX_GAMMA; ++i) st->hist[i] = 0;
+  if (st->n_out >= max_new || st->error) st->done = 1;
+}
+
+// First node of a decode graph: run the WHILE body only if decoding is not finished.
+__global__ void loop_begin_kernel(DevState* st, cudaGraphConditionalHandle cond) {
+  if (threadIdx.x == 0) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
+}
+
+// Algorithm 1, acceptance: a = longest prefix with d_{i+1} == f_i (i < gamma_eff),
+// emit d_1..d_a and f_a (the correction, or the bonus token when a = gamma_eff),
+// roll the cache back by length: kv_len += a + 1.
+__global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out_cap,
+                                  cudaGraphConditionalHandle cond, int has_cond) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  if (st->done) {
+    st->last_n = 0;
+    if (has_cond) cudaGraphSetConditional(cond, 0u);
+    return;
+  }
+  const int remaining = st->max_new - st->n_out;
+  const int g_eff = min(gamma, remaining - 1);
+  int a = 0;
+  while (a < g_eff && st->tok_in[a + 1] == st->full_tok[a]) ++a;
+  int cnt = a + 1;
+  bool eos = false;
+  for (int i = 0; i < a + 1; ++i) {
+    const int t = (i < a) ? st->tok_in[i + 1] : st->full_tok[a];
+    st->last_emitted[i] = t;
+    const int o = st->n_out + i;
+    if (o < out_cap) out_tok[o] = t;
+    if (st->eos_id >= 0 && t == st->eos_id) {
+      cnt = i + 1;
+      eos = true;
+      break;
+    }
+  }
+  st->last_n = cnt;
+  st->n_out += cnt;
+  st->kv_len += a + 1;
+  const int y = st->full_tok[a];
+  st->cur_tok = y;
+  st->tok_in[0] = y;
+  st->steps += 1;
+  st->drafted += g_eff;
+  st->accepted += a;
+  st->hist[a] += 1;
+  if (eos || st->n_out >= st->max_new || st->error) st->done = 1;
+  if (has_cond) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
+}
+
+// Greedy baseline step: emit f_0 of the single row, advance the cache by one.
+__global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cudaGraphConditionalHandle cond) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  if (st->done) {
+    cudaGraphSetConditional(cond, 0u);
+    return;
+  }
+  const int y = st->full_tok[0];
+  if (st->n_out < out_cap) out_tok[st->n_out] = y;
+  st->n_out += 1;
+  st->kv_len += 1;
+  st->cur_tok = y;
+  st->tok_in[0] = y;
+  st->steps += 1;
+  st->last_n = 1;
+  st->last_emitted[0] = y;
+  if ((st->eos_id >= 0 && y == st->eos_id) || st->n_out >= st->max_new || st->error) st->done = 1;
+  cudaGraphSetConditional(cond, st->done ? 0u : 1u);
+}
+
+__global__ void copy_out_kernel(const DevState* st, const int* out_int, int* user_out, int* user_n, int max_new) {
+  pdl_wait();
+  const int n = min(st->n_out, max_new);
+  for (int i = threadIdx.x; i < n; i += blockDim.x)
+    if (user_out) user_out[i] = out_int[i];
+  if (threadIdx.x == 0 && user_n) *user_n = n;
+}
+
+__global__ void copy_draft_kernel(const DevState* st, int gamma, int* draft_tok) {
+  pdl_wait();
+  if (threadIdx.x < gamma) draft_tok[threadIdx.x] = st->tok_in[threadIdx.x + 1];
+}
+
+__global__ void copy_emitted_kernel(const DevState* st, int* n_emitted, int* emitted) {
+  pdl_wait();
+  const int n = st->last_n;
+  if (threadIdx.x == 0 && n_emitted) *n_emitted = n;
+  if (emitted && threadIdx.x < n) emitted[threadIdx.x] = st->last_emitted[threadIdx.x];
+}
+
+__global__ void first_token_kernel(const DevState* st, int* first_tok) {
+  pdl_wait();
+  if (threadIdx.x == 0) *first_tok = st->cur_tok;
+}
+
+// cos/sin of pos * theta^(-2j/head_dim), computed in fp64 and rounded to fp32.
+__global__ void rope_table_kernel(float2* cs, int max_seq, int head_dim, double theta) {
+  const int half = head_dim / 2;
+  const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+  if (idx >= max_seq * half) return;
+  const int pos = idx / half, j = idx - pos * half;
+  const double ang = static_cast<double>(pos) * pow(theta, -2.0 * j / head_dim);
+  double s, c;
+  sincos(ang, &s, &c);
+  cs[idx] = make_float2(static_cast<float>(c), static_cast<float>(s));
+}
+
+}  // namespace ssd

@@ -1,0 +1,931 @@
+// Host engine and C ABI of the SSD library (see include/ssd.h).
+//
+// One ssd_ctx owns the KV cache, activation rows, workspaces, a private CUDA
+// stream and the CUDA graphs that replay the decode loop.  Every projection is
+// a gemv_kernel launch (stream-K weight streaming), attention is attn_kernel
+// (split-KV, causal over the query block), and the loop control of Algorithm 1
+// runs in small device kernels; a decode is one graph launch whose WHILE node
+// repeats draft + verify + accept on the device until the device state says
+// done.
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <string>
+#include <utility>
+#include <vector>
+
+#include "attention.cuh"
+#include "control.cuh"
+#include "gemv.cuh"
+
+namespace ssd {
+cudaError_t gemv_launch_qkv(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_launch_gate(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_launch_silu(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_launch_resid(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_launch_head(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_attrs_qkv();
+cudaError_t gemv_attrs_gate();
+cudaError_t gemv_attrs_silu();
+cudaError_t gemv_attrs_resid();
+cudaError_t gemv_attrs_head();
+}  // namespace ssd
+
+using namespace ssd;
+
+namespace {
+
+constexpr int kPrefillChunk = 8;  // prefill rows per pass through the layers
+constexpr int kMaxVerifyRows = 9; // gemv / attention instantiations cover M = 1..9
+
+struct Site {  // one projection: up to three weight matrices with a common K
+  CUtensorMap maps[3];
+  int N = 0, K = 0, n_rt = 0, n_kt = 0, units = 0, grid = 0, seg_rows = 0;
+};
+
+struct LayerSites {
+  Site qkv, o, gateup, down;
+};
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+}  // namespace
+
+struct ssd_ctx {
+  ssd_config cfg{};
+  int qdim = 0, num_sms = 0, device = 0;
+  // borrowed weights
+  const __nv_bfloat16 *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
+  std::vector<const __nv_bfloat16*> attn_norm, ffn_norm;
+  const __nv_bfloat16 *in_norm = nullptr;
+  const float *resid_scale = nullptr, *in_scale = nullptr;
+  std::vector<LayerSites> layers;
+  Site in1, in2, head;
+  // owned device memory
+  DevState* st = nullptr;
+  int* out_int = nullptr;  // [max_seq] emitted tokens
+  float *xv = nullptr, *qb = nullptr, *ob = nullptr, *hb = nullptr, *hin = nullptr, *xt = nullptr;
+  __nv_bfloat16 *kc = nullptr, *vc = nullptr;
+  size_t layer_kv = 0;  // elements per layer in kc / vc
+  float2* rope = nullptr;
+  float* partials = nullptr;
+  unsigned* counters = nullptr;
+  int n_counters = 0;
+  float* att_part = nullptr;
+  unsigned* att_cnt = nullptr;
+  int max_chunks = 0;
+  __nv_bfloat16* in_vis = nullptr;
+  int* in_prompt = nullptr;
+  // streams and graphs
+  cudaStream_t us = nullptr, cs = nullptr;
+  cudaEvent_t ev_in = nullptr, ev_out = nullptr;
+  bool use_pdl = true;
+  std::map<int, cudaGraphExec_t> decode_graphs, draft_graphs, verify_graphs;
+  std::map<std::pair<int, int>, cudaGraphExec_t> prefill_graphs;
+  cudaGraphExec_t greedy_graph = nullptr;
+  std::map<int, int64_t> decode_body_launches;
+  std::map<std::pair<int, int>, int64_t> prefill_launch_count;
+  int64_t greedy_body_launches = 0;
+  int64_t launch_counter = 0;
+  // host-side state machine
+  bool prefilled = false;
+  int drafted_gamma = 0;
+  int prompt_len = 0;
+  int64_t kv_upper = 0;  // upper bound on the device kv_len
+  int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy
+  int last_gamma = 0;
+  std::pair<int, int> last_prefill_shape{0, 0};
+  // debug logits capture
+  float* logits_buf = nullptr;
+  int logits_rows = 0;
+  std::string err;
+};
+
+// ------------------------------------------------------------------ helpers
+
+static ssd_status fail(ssd_ctx* c, ssd_status s, const char* fmt, ...) {
+  if (c) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    c->err = buf;
+  }
+  return s;
+}
+
+#define CK(call)                                                                                          \
+  do {                                                                                                    \
+    cudaError_t e_ = (call);                                                                              \
+    if (e_ != cudaSuccess) {                                                                              \
+      return fail(c, e_ == cudaErrorMemoryAllocation ? SSD_ERR_OOM : SSD_ERR_CUDA, "%s failed: %s (%s:%d)", \
+                  #call, cudaGetErrorString(e_), __FILE__, __LINE__);                                     \
+    }                                                                                                     \
+  } while (0)
+
+#define CKS(expr)                      \
+  do {                                 \
+    ssd_status s_ = (expr);            \
+    if (s_ != SSD_OK) return s_;       \
+  } while (0)
+
+template <typename Kern, typename... Args>
+static cudaError_t launch_k(ssd_ctx* c, Kern kern, dim3 grid, dim3 block, size_t smem, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = c->cs;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = c->use_pdl ? 1 : 0;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  ++c->launch_counter;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+static ssd_status encode_map(ssd_ctx* c, CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+                             uint32_t box_rows) {
+  if (reinterpret_cast<uintptr_t>(base) % 16 != 0)
+    return fail(c, SSD_ERR_INVALID_ARG, "weight pointer %p is not 16-byte aligned", base);
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(c, SSD_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
+  return SSD_OK;
+}
+
+// Site over 1..3 matrices [rows_each][K] stacked along N, 128-row tiles.
+static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nmats, int rows_each, int K) {
+  for (int i = 0; i < nmats; ++i) CKS(encode_map(c, &s->maps[i], mats[i], rows_each, K, kTileN));
+  for (int i = nmats; i < 3; ++i) s->maps[i] = s->maps[0];
+  s->N = rows_each * nmats;
+  s->K = K;
+  s->seg_rows = rows_each;
+  s->n_rt = (s->N + kTileN - 1) / kTileN;
+  s->n_kt = K / kTileK;
+  s->units = s->n_rt * s->n_kt;
+  s->grid = s->units < c->num_sms ? s->units : c->num_sms;
+  return SSD_OK;
+}
+
+// gate/up pair: each unit holds 64 gate rows and the same 64 up rows.
+static ssd_status make_pair_site(ssd_ctx* c, Site* s, const void* gate, const void* up, int rows, int K) {
+  CKS(encode_map(c, &s->maps[0], gate, rows, K, kTileN / 2));
+  CKS(encode_map(c, &s->maps[1], up, rows, K, kTileN / 2));
+  s->maps[2] = s->maps[0];
+  s->N = rows;
+  s->K = K;
+  s->seg_rows = rows;
+  s->n_rt = rows / (kTileN / 2);
+  s->n_kt = K / kTileK;
+  s->units = s->n_rt * s->n_kt;
+  s->grid = s->units < c->num_sms ? s->units : c->num_sms;
+  return SSD_OK;
+}
+
+static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
+  p.K = s.K;
+  p.n_kt = s.n_kt;
+  p.n_rt = s.n_rt;
+  p.units = s.units;
+  p.N = s.N;
+  p.seg_rows = s.seg_rows;
+  p.partials = c->partials;
+  p.counters = c->counters;
+  p.st = c->st;
+  p.eps = c->cfg.rms_eps;
+  cudaError_t r;
+  ++c->launch_counter;
+  switch (e) {
+    case Epi::QKV: r = gemv_launch_qkv(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+    case Epi::GATE_SILU: r = gemv_launch_gate(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+    case Epi::SILU: r = gemv_launch_silu(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+    case Epi::RESID: r = gemv_launch_resid(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+    default: r = gemv_launch_head(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+  }
+  CK(r);
+  return SSD_OK;
+}
+
+template <int M>
+static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a) {
+  if (c->cfg.head_dim == 128)
+    return launch_k(c, attn_kernel<M, 128>, dim3(c->num_sms), dim3(kAttnWarps * 32), 0, a);
+  return launch_k(c, attn_kernel<M, 64>, dim3(c->num_sms), dim3(kAttnWarps * 32), 0, a);
+}
+
+static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off) {
+  AttnParams a{};
+  a.q = c->qb;
+  a.q_stride = c->qdim;
+  a.k_cache = c->kc + l * c->layer_kv;
+  a.v_cache = c->vc + l * c->layer_kv;
+  a.o = c->ob;
+  a.o_stride = c->qdim;
+  a.part = c->att_part;
+  a.counters = c->att_cnt;
+  a.st = c->st;
+  a.pos_off = pos_off;
+  a.n_heads = c->cfg.n_heads;
+  a.max_seq = c->cfg.max_seq;
+  a.max_chunks = c->max_chunks;
+  a.scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
+  cudaError_t r;
+  switch (M) {
+    case 1: r = attn_launch_m<1>(c, a); break;
+    case 2: r = attn_launch_m<2>(c, a); break;
+    case 3: r = attn_launch_m<3>(c, a); break;
+    case 4: r = attn_launch_m<4>(c, a); break;
+    case 5: r = attn_launch_m<5>(c, a); break;
+    case 6: r = attn_launch_m<6>(c, a); break;
+    case 7: r = attn_launch_m<7>(c, a); break;
+    case 8: r = attn_launch_m<8>(c, a); break;
+    case 9: r = attn_launch_m<9>(c, a); break;
+    default: return fail(c, SSD_ERR_INVALID_ARG, "attention rows %d out of range", M);
+  }
+  CK(r);
+  return SSD_OK;
+}
+
+// One decoder layer x_{l+1} = x_l + f_l(x_l) on rows row0 .. row0+M-1 of xv at
+// positions kv_len + pos_off + m.
+static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off) {
+  const int d = c->cfg.d_model;
+  float* x = c->xv + static_cast<size_t>(row0) * d;
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = d;
+  p.gain = c->attn_norm[l];
+  p.pos_off = pos_off;
+  p.q_out = c->qb;
+  p.q_stride = c->qdim;
+  p.k_cache = c->kc + l * c->layer_kv;
+  p.v_cache = c->vc + l * c->layer_kv;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  p.rope_cs = c->rope;
+  CKS(gemv(c, Epi::QKV, M, c->layers[l].qkv, p));
+  CKS(attention(c, l, M, pos_off));
+  p = GemvParams{};
+  p.x = c->ob;
+  p.x_stride = c->qdim;
+  p.base = x;
+  p.base_stride = d;
+  p.dst = x;
+  p.dst_stride = d;
+  p.scale = c->resid_scale + l;
+  CKS(gemv(c, Epi::RESID, M, c->layers[l].o, p));
+  p = GemvParams{};
+  p.x = x;
+  p.x_stride = d;
+  p.gain = c->ffn_norm[l];
+  p.h_out = c->hb;
+  p.h_stride = c->cfg.d_ff;
+  CKS(gemv(c, Epi::GATE_SILU, M, c->layers[l].gateup, p));
+  p = GemvParams{};
+  p.x = c->hb;
+  p.x_stride = c->cfg.d_ff;
+  p.base = x;
+  p.base_stride = d;
+  p.dst = x;
+  p.dst_stride = d;
+  p.scale = c->resid_scale + l;
+  CKS(gemv(c, Epi::RESID, M, c->layers[l].down, p));
+  return SSD_OK;
+}
+
+// LM head g(x) = W_lm RMSNorm_f(x) + greedy argmax on M rows of x.
+static ssd_status enqueue_head(ssd_ctx* c, const float* x, int M, int pos_off, int* tok_dst, bool capture) {
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = c->cfg.d_model;
+  p.gain = c->final_norm;
+  p.pos_off = pos_off;
+  p.tok_dst = tok_dst;
+  p.logits = capture ? c->logits_buf : nullptr;
+  p.logits_rows = capture ? c->logits_rows : 0;
+  return gemv(c, Epi::ARGMAX, M, c->head, p);
+}
+
+static int* st_field(ssd_ctx* c, size_t off) {
+  return reinterpret_cast<int*>(reinterpret_cast<char*>(c->st) + off);
+}
+
+// Drafting stage: gamma tokens from layers 0..k-1, the imitation network and g.
+static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
+  const int d = c->cfg.d_model;
+  int* tok_in = st_field(c, offsetof(DevState, tok_in));
+  for (int j = 0; j < gamma; ++j) {
+    float* xj = c->xv + static_cast<size_t>(j) * d;
+    CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + j), xj, d, d,
+                c->cfg.vocab, c->st));
+    for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, j, 1, j));
+    const float* hx = xj;
+    if (c->cfg.in_kind == SSD_IN_MLP2) {
+      GemvParams p{};
+      p.x = xj;
+      p.x_stride = d;
+      p.gain = c->in_norm;
+      p.h_out = c->hin;
+      p.h_stride = c->cfg.in_hidden;
+      CKS(gemv(c, Epi::SILU, 1, c->in1, p));
+      p = GemvParams{};
+      p.x = c->hin;
+      p.x_stride = c->cfg.in_hidden;
+      p.base = xj;
+      p.base_stride = d;
+      p.dst = c->xt;
+      p.dst_stride = d;
+      p.scale = c->in_scale;
+      CKS(gemv(c, Epi::RESID, 1, c->in2, p));
+      hx = c->xt;
+    }
+    CKS(enqueue_head(c, hx, 1, j, tok_in + j + 1, false));
+  }
+  return SSD_OK;
+}
+
+// Verification stage + acceptance: row gamma through the shallow layers (rows
+// 0..gamma-1 hold x_k from the draft), all gamma+1 rows through layers k..L-1,
+// g + argmax per row, then the acceptance kernel.
+static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHandle cond, int has_cond) {
+  const int d = c->cfg.d_model;
+  int* tok_in = st_field(c, offsetof(DevState, tok_in));
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
+              c->xv + static_cast<size_t>(gamma) * d, d, d, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, gamma, 1, gamma));
+  for (int l = c->cfg.draft_exit_k; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, gamma + 1, 0));
+  CKS(enqueue_head(c, c->xv, gamma + 1, 0, full_tok, true));
+  CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, cond,
+              has_cond));
+  return SSD_OK;
+}
+
+static ssd_status enqueue_greedy_step(ssd_ctx* c, cudaGraphConditionalHandle cond) {
+  int* tok_in = st_field(c, offsetof(DevState, tok_in));
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv,
+              c->cfg.d_model, c->cfg.d_model, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
+  CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
+  CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond));
+  return SSD_OK;
+}
+
+static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
+  const int d = c->cfg.d_model, P = n_vis + n_prompt;
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
+  CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(cudaMemsetAsync(c->att_cnt, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
+  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
+  int r0 = 0;
+  for (; r0 < P; r0 += kPrefillChunk) {
+    const int Mc = P - r0 < kPrefillChunk ? P - r0 : kPrefillChunk;
+    CK(launch_k(c, prefill_rows_kernel, dim3(Mc), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+                static_cast<const int*>(c->in_prompt), n_vis, r0, c->embed, c->cfg.vocab, c->xv, d, d, c->st));
+    for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, Mc, r0));
+  }
+  r0 -= kPrefillChunk;
+  CKS(enqueue_head(c, c->xv + static_cast<size_t>(P - 1 - r0) * d, 1, P - 1, full_tok, true));
+  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
+  return SSD_OK;
+}
+
+// ------------------------------------------------------------------ graphs
+
+static ssd_status begin_capture(ssd_ctx* c, cudaGraph_t g) {
+  CK(cudaStreamBeginCaptureToGraph(c->cs, g, nullptr, nullptr, 0, cudaStreamCaptureModeThreadLocal));
+  return SSD_OK;
+}
+
+static ssd_status end_capture(ssd_ctx* c, cudaGraph_t g, ssd_status inner) {
+  cudaGraph_t out = nullptr;
+  cudaError_t e = cudaStreamEndCapture(c->cs, &out);
+  if (inner != SSD_OK) return inner;
+  if (e != cudaSuccess) return fail(c, SSD_ERR_CUDA, "stream capture failed: %s", cudaGetErrorString(e));
+  (void)g;
+  return SSD_OK;
+}
+
+// Graph = [loop_begin] -> WHILE(cond) { body }.  body is draft+verify+accept
+// (gamma > 0) or one greedy step (gamma == 0).
+static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec, int64_t* body_launches) {
+  cudaGraph_t g = nullptr;
+  CK(cudaGraphCreate(&g, 0));
+  cudaGraphConditionalHandle cond;
+  ssd_status s = SSD_OK;
+  cudaError_t e = cudaGraphConditionalHandleCreate(&cond, g, 0, cudaGraphCondAssignDefault);
+  if (e != cudaSuccess) {
+    cudaGraphDestroy(g);
+    CK(e);
+  }
+  s = begin_capture(c, g);
+  if (s == SSD_OK) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(32);
+    cfg.stream = c->cs;
+    e = cudaLaunchKernelEx(&cfg, loop_begin_kernel, c->st, cond);
+    s = end_capture(c, g, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop_begin launch: %s",
+                                                           cudaGetErrorString(e)));
+  }
+  cudaGraphNode_t begin = nullptr;
+  size_t n = 1;
+  if (s == SSD_OK && cudaGraphGetNodes(g, &begin, &n) != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "graph nodes");
+  cudaGraphNodeParams cp = {};
+  cp.type = cudaGraphNodeTypeConditional;
+  cp.conditional.handle = cond;
+  cp.conditional.type = cudaGraphCondTypeWhile;
+  cp.conditional.size = 1;
+  cudaGraphNode_t cnode;
+  if (s == SSD_OK) {
+    e = cudaGraphAddNode(&cnode, g, &begin, nullptr, 1, &cp);
+    if (e != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "conditional node: %s", cudaGetErrorString(e));
+  }
+  if (s == SSD_OK) {
+    cudaGraph_t body = cp.conditional.phGraph_out[0];
+    s = begin_capture(c, body);
+    if (s == SSD_OK) {
+      const int64_t l0 = c->launch_counter;
+      ssd_status inner = gamma > 0 ? enqueue_draft(c, gamma) : SSD_OK;
+      if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify(c, gamma, cond, 1) : enqueue_greedy_step(c, cond);
+      *body_launches = c->launch_counter - l0;
+      s = end_capture(c, body, inner);
+    }
+  }
+  if (s == SSD_OK) {
+    e = cudaGraphInstantiate(exec, g, 0);
+    if (e != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(e));
+  }
+  cudaGraphDestroy(g);
+  return s;
+}
+
+using EnqueueFn = ssd_status (*)(ssd_ctx*, int, int);
+
+static ssd_status build_plain_graph(ssd_ctx* c, EnqueueFn fn, int a0, int a1, cudaGraphExec_t* exec,
+                                    int64_t* launches) {
+  cudaGraph_t g = nullptr;
+  CK(cudaGraphCreate(&g, 0));
+  ssd_status s = begin_capture(c, g);
+  if (s == SSD_OK) {
+    const int64_t l0 = c->launch_counter;
+    ssd_status inner = fn(c, a0, a1);
+    if (launches) *launches = c->launch_counter - l0;
+    s = end_capture(c, g, inner);
+  }
+  if (s == SSD_OK) {
+    cudaError_t e = cudaGraphInstantiate(exec, g, 0);
+    if (e != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(e));
+  }
+  cudaGraphDestroy(g);
+  return s;
+}
+
+static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) { return enqueue_prefill(c, a, b); }
+static ssd_status enq_draft_fn(ssd_ctx* c, int g, int) { return enqueue_draft(c, g); }
+static ssd_status enq_verify_fn(ssd_ctx* c, int g, int) { return enqueue_verify(c, g, 0, 0); }
+
+static void drop_graphs(ssd_ctx* c) {
+  for (auto& kv : c->decode_graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->draft_graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->verify_graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->prefill_graphs) cudaGraphExecDestroy(kv.second);
+  if (c->greedy_graph) cudaGraphExecDestroy(c->greedy_graph);
+  c->decode_graphs.clear();
+  c->draft_graphs.clear();
+  c->verify_graphs.clear();
+  c->prefill_graphs.clear();
+  c->greedy_graph = nullptr;
+}
+
+// Order the private stream after the caller's stream, and back.
+static ssd_status enter(ssd_ctx* c) {
+  CK(cudaEventRecord(c->ev_in, c->us));
+  CK(cudaStreamWaitEvent(c->cs, c->ev_in, 0));
+  return SSD_OK;
+}
+static ssd_status leave(ssd_ctx* c) {
+  CK(cudaEventRecord(c->ev_out, c->cs));
+  CK(cudaStreamWaitEvent(c->us, c->ev_out, 0));
+  return SSD_OK;
+}
+
+static ssd_status read_device_error(ssd_ctx* c) {
+  int errw = 0;
+  CK(cudaMemcpy(&errw, reinterpret_cast<char*>(c->st) + offsetof(DevState, error), sizeof(int),
+                cudaMemcpyDeviceToHost));
+  if (errw & DERR_TIMEOUT) return fail(c, SSD_ERR_TIMEOUT, "a bounded device wait ran out (error word %d)", errw);
+  if (errw) return fail(c, SSD_ERR_DEVICE, "device error word %d (1 = bad token id, 4 = position out of range)", errw);
+  return SSD_OK;
+}
+
+// ------------------------------------------------------------------ C ABI
+
+extern "C" {
+
+const char* ssd_status_string(ssd_status s) {
+  switch (s) {
+    case SSD_OK: return "ok";
+    case SSD_ERR_INVALID_ARG: return "invalid argument";
+    case SSD_ERR_OOM: return "out of device memory";
+    case SSD_ERR_CUDA: return "CUDA error";
+    case SSD_ERR_CAPACITY: return "KV cache capacity exceeded";
+    case SSD_ERR_STATE: return "call out of order";
+    case SSD_ERR_TIMEOUT: return "device wait timed out";
+    case SSD_ERR_DEVICE: return "device-side error";
+    case SSD_ERR_UNSUPPORTED: return "unsupported device";
+  }
+  return "unknown status";
+}
+
+const char* ssd_last_error(const ssd_ctx* c) { return c ? c->err.c_str() : "null context"; }
+
+static ssd_status alloc(ssd_ctx* c, void** p, size_t bytes) {
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e != cudaSuccess) {
+    *p = nullptr;
+    return fail(c, SSD_ERR_OOM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
+  }
+  e = cudaMemset(*p, 0, bytes);
+  if (e != cudaSuccess) return fail(c, SSD_ERR_CUDA, "cudaMemset failed: %s", cudaGetErrorString(e));
+  return SSD_OK;
+}
+
+ssd_status ssd_destroy(ssd_ctx* c) {
+  if (!c) return SSD_OK;
+  if (c->cs) cudaStreamSynchronize(c->cs);
+  drop_graphs(c);
+  void* bufs[] = {c->st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope,
+                  c->partials, c->counters, c->att_part, c->att_cnt, c->in_vis, c->in_prompt};
+  for (void* b : bufs)
+    if (b) cudaFree(b);
+  if (c->ev_in) cudaEventDestroy(c->ev_in);
+  if (c->ev_out) cudaEventDestroy(c->ev_out);
+  if (c->cs) cudaStreamDestroy(c->cs);
+  delete c;
+  return SSD_OK;
+}
+
+static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weights* w) {
+  const ssd_config& k = *cfg;
+  if (k.n_layers < 1 || k.d_model < 64 || k.n_heads < 1 || k.vocab < 2 || k.d_ff < 64)
+    return fail(c, SSD_ERR_INVALID_ARG, "bad model shape");
+  if (k.head_dim != 64 && k.head_dim != 128) return fail(c, SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
+  const int qdim = k.n_heads * k.head_dim;
+  if (k.d_model % kTileK || k.d_ff % kTileK || qdim % kTileN)
+    return fail(c, SSD_ERR_INVALID_ARG, "d_model, d_ff must be multiples of 64 and n_heads*head_dim of 128");
+  if (k.draft_exit_k < 1 || k.draft_exit_k > k.n_layers) return fail(c, SSD_ERR_INVALID_ARG, "draft_exit_k");
+  if (k.in_kind != SSD_IN_IDENTITY && k.in_kind != SSD_IN_MLP2) return fail(c, SSD_ERR_INVALID_ARG, "in_kind");
+  if (k.in_kind == SSD_IN_MLP2 && (k.in_hidden < 64 || k.in_hidden % kTileK))
+    return fail(c, SSD_ERR_INVALID_ARG, "in_hidden must be a positive multiple of 64");
+  if (k.gamma_max < 1 || k.gamma_max > SSD_MAX_GAMMA || k.gamma_max + 1 > kMaxVerifyRows)
+    return fail(c, SSD_ERR_INVALID_ARG, "gamma_max must be in [1, %d]", SSD_MAX_GAMMA);
+  if (k.max_seq < 2) return fail(c, SSD_ERR_INVALID_ARG, "max_seq");
+  if (!w || !w->embed || !w->lm_head || !w->final_norm || !w->wq || !w->wk || !w->wv || !w->wo || !w->w_gate ||
+      !w->w_up || !w->w_down || !w->attn_norm || !w->ffn_norm || !w->resid_scale)
+    return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer");
+  if (k.in_kind == SSD_IN_MLP2 && (!w->in_norm || !w->in_w1 || !w->in_w2 || !w->in_scale))
+    return fail(c, SSD_ERR_INVALID_ARG, "null imitation-network weight pointer");
+  for (int l = 0; l < k.n_layers; ++l)
+    if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->w_gate[l] || !w->w_up[l] || !w->w_down[l] ||
+        !w->attn_norm[l] || !w->ffn_norm[l])
+      return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer in layer %d", l);
+
+  CK(cudaGetDevice(&c->device));
+  cudaDeviceProp prop;
+  CK(cudaGetDeviceProperties(&prop, c->device));
+  if (prop.major != 10) return fail(c, SSD_ERR_UNSUPPORTED, "needs a Blackwell sm_103 device, got sm_%d%d",
+                                    prop.major, prop.minor);
+  c->num_sms = prop.multiProcessorCount;
+  if (!g_encode) {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    CK(cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q));
+    if (q != cudaDriverEntryPointSuccess || !fn) return fail(c, SSD_ERR_UNSUPPORTED, "cuTensorMapEncodeTiled");
+    g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  CK(gemv_attrs_qkv());
+  CK(gemv_attrs_gate());
+  CK(gemv_attrs_silu());
+  CK(gemv_attrs_resid());
+  CK(gemv_attrs_head());
+
+  c->cfg = k;
+  c->qdim = qdim;
+  c->embed = static_cast<const __nv_bfloat16*>(w->embed);
+  c->lm_head = static_cast<const __nv_bfloat16*>(w->lm_head);
+  c->final_norm = static_cast<const __nv_bfloat16*>(w->final_norm);
+  c->in_norm = static_cast<const __nv_bfloat16*>(w->in_norm);
+  c->resid_scale = w->resid_scale;
+  c->in_scale = w->in_scale;
+  c->layers.resize(k.n_layers);
+  for (int l = 0; l < k.n_layers; ++l) {
+    c->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
+    c->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
+    const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
+    CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model));
+    CKS(make_site(c, &c->layers[l].o, &w->wo[l], 1, k.d_model, qdim));
+    CKS(make_pair_site(c, &c->layers[l].gateup, w->w_gate[l], w->w_up[l], k.d_ff, k.d_model));
+    CKS(make_site(c, &c->layers[l].down, &w->w_down[l], 1, k.d_model, k.d_ff));
+  }
+  if (k.in_kind == SSD_IN_MLP2) {
+    CKS(make_site(c, &c->in1, &w->in_w1, 1, k.in_hidden, k.d_model));
+    CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden));
+  }
+  CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model));
+
+  // owned memory
+  const int R = kMaxRows;
+  const size_t d = k.d_model;
+  CKS(alloc(c, reinterpret_cast<void**>(&c->st), sizeof(DevState)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->out_int), sizeof(int) * k.max_seq));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->xv), sizeof(float) * R * d));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->xt), sizeof(float) * R * d));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->qb), sizeof(float) * R * qdim));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->ob), sizeof(float) * R * qdim));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->hb), sizeof(float) * R * k.d_ff));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->hin), sizeof(float) * R * (k.in_hidden > 0 ? k.in_hidden : 64)));
+  c->layer_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
+  CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(__nv_bfloat16) * c->layer_kv * k.n_layers));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(__nv_bfloat16) * c->layer_kv * k.n_layers));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->rope), sizeof(float2) * k.max_seq * (k.head_dim / 2)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->num_sms * R * kTileN));
+  int max_rt = 1;
+  for (const Site* s : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->head,
+                        &c->in1, &c->in2})
+    max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
+  c->n_counters = max_rt;
+  CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
+  c->max_chunks = (k.max_seq + kAttnChunk - 1) / kAttnChunk;
+  CKS(alloc(c, reinterpret_cast<void**>(&c->att_part),
+            sizeof(float) * k.n_heads * c->max_chunks * R * (k.head_dim + 4)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->att_cnt), sizeof(unsigned) * k.n_heads));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * k.max_seq));
+  CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
+  CK(cudaEventCreateWithFlags(&c->ev_in, cudaEventDisableTiming));
+  CK(cudaEventCreateWithFlags(&c->ev_out, cudaEventDisableTiming));
+  const int nrope = k.max_seq * (k.head_dim / 2);
+  rope_table_kernel<<<(nrope + 255) / 256, 256, 0, c->cs>>>(c->rope, k.max_seq, k.head_dim,
+                                                            static_cast<double>(k.rope_theta));
+  CK(cudaGetLastError());
+  CK(cudaStreamSynchronize(c->cs));
+  return SSD_OK;
+}
+
+ssd_status ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, ssd_ctx** out) {
+  if (!cfg || !out) return SSD_ERR_INVALID_ARG;
+  *out = nullptr;
+  ssd_ctx* c = new (std::nothrow) ssd_ctx();
+  if (!c) return SSD_ERR_OOM;
+  c->us = static_cast<cudaStream_t>(cuda_stream);
+  ssd_status s = create_impl(c, cfg, w);
+  if (s != SSD_OK) {
+    fprintf(stderr, "ssd_create: %s\n", c->err.c_str());
+    ssd_destroy(c);
+    return s;
+  }
+  *out = c;
+  return SSD_OK;
+}
+
+static ssd_status prefill_impl(ssd_ctx* c, int n_vis, int n_prompt) {
+  const int P = n_vis + n_prompt;
+  auto key = std::make_pair(n_vis, n_prompt);
+  auto it = c->prefill_graphs.find(key);
+  if (it == c->prefill_graphs.end()) {
+    cudaGraphExec_t ge;
+    int64_t nl = 0;
+    CKS(build_plain_graph(c, enq_prefill_fn, n_vis, n_prompt, &ge, &nl));
+    it = c->prefill_graphs.emplace(key, ge).first;
+    c->prefill_launch_count[key] = nl;
+  }
+  CK(cudaGraphLaunch(it->second, c->cs));
+  c->prefilled = true;
+  c->drafted_gamma = 0;
+  c->prompt_len = P;
+  c->kv_upper = P;
+  c->last_prefill_shape = key;
+  return SSD_OK;
+}
+
+static ssd_status check_prefill_args(ssd_ctx* c, const void* vis, int n_vis, const int32_t* prompt, int n_prompt) {
+  if (n_vis < 0 || n_prompt < 0 || n_vis + n_prompt < 1) return fail(c, SSD_ERR_INVALID_ARG, "empty prompt");
+  if (n_vis > 0 && !vis) return fail(c, SSD_ERR_INVALID_ARG, "vis_emb is null");
+  if (n_prompt > 0 && !prompt) return fail(c, SSD_ERR_INVALID_ARG, "prompt is null");
+  if (n_vis + n_prompt + 1 > c->cfg.max_seq) return fail(c, SSD_ERR_CAPACITY, "prompt longer than max_seq");
+  return SSD_OK;
+}
+
+ssd_status ssd_prefill(ssd_ctx* c, const void* vis, int n_vis, const int32_t* prompt, int n_prompt,
+                       int32_t* first_tok) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CKS(check_prefill_args(c, vis, n_vis, prompt, n_prompt));
+  CKS(enter(c));
+  if (n_vis > 0)
+    CK(cudaMemcpyAsync(c->in_vis, vis, sizeof(__nv_bfloat16) * n_vis * c->cfg.d_model, cudaMemcpyDeviceToDevice,
+                       c->cs));
+  if (n_prompt > 0)
+    CK(cudaMemcpyAsync(c->in_prompt, prompt, sizeof(int) * n_prompt, cudaMemcpyDeviceToDevice, c->cs));
+  CKS(prefill_impl(c, n_vis, n_prompt));
+  if (first_tok) first_token_kernel<<<1, 32, 0, c->cs>>>(c->st, first_tok);
+  CK(cudaGetLastError());
+  return leave(c);
+}
+
+ssd_status ssd_draft(ssd_ctx* c, int gamma, int32_t* draft_tok) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (!c->prefilled) return fail(c, SSD_ERR_STATE, "ssd_draft before ssd_prefill");
+  if (gamma < 1 || gamma > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma %d", gamma);
+  if (c->kv_upper + gamma + 1 > c->cfg.max_seq) return fail(c, SSD_ERR_CAPACITY, "KV cache full");
+  CKS(enter(c));
+  auto it = c->draft_graphs.find(gamma);
+  if (it == c->draft_graphs.end()) {
+    cudaGraphExec_t ge;
+    CKS(build_plain_graph(c, enq_draft_fn, gamma, 0, &ge, nullptr));
+    it = c->draft_graphs.emplace(gamma, ge).first;
+  }
+  CK(cudaGraphLaunch(it->second, c->cs));
+  if (draft_tok) copy_draft_kernel<<<1, 32, 0, c->cs>>>(c->st, gamma, draft_tok);
+  CK(cudaGetLastError());
+  c->drafted_gamma = gamma;
+  return leave(c);
+}
+
+ssd_status ssd_verify(ssd_ctx* c, int gamma, int32_t* n_emitted, int32_t* emitted) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (!c->prefilled || c->drafted_gamma != gamma)
+    return fail(c, SSD_ERR_STATE, "ssd_verify(gamma=%d) needs a preceding ssd_draft with the same gamma", gamma);
+  CKS(enter(c));
+  auto it = c->verify_graphs.find(gamma);
+  if (it == c->verify_graphs.end()) {
+    cudaGraphExec_t ge;
+    CKS(build_plain_graph(c, enq_verify_fn, gamma, 0, &ge, nullptr));
+    it = c->verify_graphs.emplace(gamma, ge).first;
+  }
+  CK(cudaGraphLaunch(it->second, c->cs));
+  if (n_emitted || emitted) copy_emitted_kernel<<<1, 32, 0, c->cs>>>(c->st, n_emitted, emitted);
+  CK(cudaGetLastError());
+  c->drafted_gamma = 0;
+  c->kv_upper += gamma + 1;
+  return leave(c);
+}
+
+static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_tok, int32_t* n_out) {
+  if (!c->prefilled) return fail(c, SSD_ERR_STATE, "decode before ssd_prefill");
+  if (max_new < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_new must be >= 1");
+  if (gamma < 0 || gamma > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma %d", gamma);
+  if (static_cast<int64_t>(c->prompt_len) + max_new + gamma + 1 > c->cfg.max_seq)
+    return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 = %d > max_seq = %d",
+                c->prompt_len + max_new + gamma + 1, c->cfg.max_seq);
+  cudaGraphExec_t ge;
+  if (gamma > 0) {
+    auto it = c->decode_graphs.find(gamma);
+    if (it == c->decode_graphs.end()) {
+      int64_t nb = 0;
+      CKS(build_loop_graph(c, gamma, &ge, &nb));
+      it = c->decode_graphs.emplace(gamma, ge).first;
+      c->decode_body_launches[gamma] = nb;
+    }
+    ge = it->second;
+  } else {
+    if (!c->greedy_graph) CKS(build_loop_graph(c, 0, &c->greedy_graph, &c->greedy_body_launches));
+    ge = c->greedy_graph;
+  }
+  decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
+  CK(cudaGetLastError());
+  CK(cudaGraphLaunch(ge, c->cs));
+  if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+  CK(cudaGetLastError());
+  c->last_decode_kind = gamma > 0 ? 1 : 2;
+  c->last_gamma = gamma;
+  c->drafted_gamma = 0;
+  c->kv_upper = c->prompt_len + max_new + gamma + 1;
+  return SSD_OK;
+}
+
+ssd_status ssd_decode(ssd_ctx* c, int max_new, int gamma, int32_t* out_tok, int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (gamma < 1) return fail(c, SSD_ERR_INVALID_ARG, "gamma must be >= 1");
+  CKS(enter(c));
+  CKS(decode_impl(c, max_new, gamma, out_tok, n_out));
+  return leave(c);
+}
+
+ssd_status ssd_greedy_decode(ssd_ctx* c, int max_new, int32_t* out_tok, int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CKS(enter(c));
+  CKS(decode_impl(c, max_new, 0, out_tok, n_out));
+  return leave(c);
+}
+
+ssd_status ssd_sync(ssd_ctx* c) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->cs));
+  CK(cudaStreamSynchronize(c->us));
+  return read_device_error(c);
+}
+
+ssd_status ssd_get_stats(ssd_ctx* c, ssd_stats* out) {
+  if (!c || !out) return SSD_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->cs));
+  DevState h;
+  CK(cudaMemcpy(&h, c->st, sizeof(DevState), cudaMemcpyDeviceToHost));
+  memset(out, 0, sizeof(*out));
+  out->steps = h.steps;
+  out->drafted = h.drafted;
+  out->accepted = h.accepted;
+  out->emitted = h.n_out;
+  for (int i = 0; i <= SSD_MAX_GAMMA; ++i) out->accept_hist[i] = h.hist[i];
+  out->kv_len = h.kv_len;
+  return SSD_OK;
+}
+
+static ssd_status generate_impl(ssd_ctx* c, const void* vis, int n_vis, const int32_t* prompt, int n_prompt,
+                                int max_new, int gamma, int32_t* out, int* n_out, ssd_stats* stats) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (!out || !n_out) return fail(c, SSD_ERR_INVALID_ARG, "out / n_out is null");
+  CKS(check_prefill_args(c, vis, n_vis, prompt, n_prompt));
+  if (static_cast<int64_t>(n_vis) + n_prompt + max_new + gamma + 1 > c->cfg.max_seq)
+    return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 > max_seq");
+  CKS(enter(c));
+  if (n_vis > 0)
+    CK(cudaMemcpyAsync(c->in_vis, vis, sizeof(__nv_bfloat16) * n_vis * c->cfg.d_model, cudaMemcpyHostToDevice,
+                       c->cs));
+  if (n_prompt > 0) CK(cudaMemcpyAsync(c->in_prompt, prompt, sizeof(int) * n_prompt, cudaMemcpyHostToDevice, c->cs));
+  CKS(prefill_impl(c, n_vis, n_prompt));
+  CKS(decode_impl(c, max_new, gamma, nullptr, nullptr));
+  CK(cudaMemcpyAsync(out, c->out_int, sizeof(int) * max_new, cudaMemcpyDeviceToHost, c->cs));
+  CK(cudaStreamSynchronize(c->cs));
+  CKS(read_device_error(c));
+  DevState h;
+  CK(cudaMemcpy(&h, c->st, sizeof(DevState), cudaMemcpyDeviceToHost));
+  *n_out = h.n_out < max_new ? h.n_out : max_new;
+  if (stats) CKS(ssd_get_stats(c, stats));
+  return leave(c);
+}
+
+ssd_status ssd_generate(ssd_ctx* c, const void* vis, int n_vis, const int32_t* prompt, int n_prompt, int max_new,
+                        int gamma, int32_t* out, int* n_out, ssd_stats* stats) {
+  if (c && gamma < 1) return fail(c, SSD_ERR_INVALID_ARG, "gamma must be >= 1");
+  return generate_impl(c, vis, n_vis, prompt, n_prompt, max_new, gamma, out, n_out, stats);
+}
+
+ssd_status ssd_greedy_generate(ssd_ctx* c, const void* vis, int n_vis, const int32_t* prompt, int n_prompt,
+                               int max_new, int32_t* out, int* n_out, ssd_stats* stats) {
+  return generate_impl(c, vis, n_vis, prompt, n_prompt, max_new, 0, out, n_out, stats);
+}
+
+ssd_status ssd_set_logits_capture(ssd_ctx* c, float* buf, int max_rows) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (buf && max_rows < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_rows");
+  CK(cudaStreamSynchronize(c->cs));
+  drop_graphs(c);
+  c->logits_buf = buf;
+  c->logits_rows = buf ? max_rows : 0;
+  return SSD_OK;
+}
+
+ssd_status ssd_get_kv(ssd_ctx* c, const void** k_cache, const void** v_cache, int* kv_len) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->cs));
+  if (k_cache) *k_cache = c->kc;
+  if (v_cache) *v_cache = c->vc;
+  if (kv_len) CK(cudaMemcpy(kv_len, c->st, sizeof(int), cudaMemcpyDeviceToHost));
+  return SSD_OK;
+}
+
+ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t* decode_launches) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->cs));
+  DevState h;
+  CK(cudaMemcpy(&h, c->st, sizeof(DevState), cudaMemcpyDeviceToHost));
+  if (prefill_launches) {
+    auto it = c->prefill_launch_count.find(c->last_prefill_shape);
+    *prefill_launches = it == c->prefill_launch_count.end() ? 0 : it->second;
+  }
+  if (decode_launches) {
+    int64_t body = 0;
+    if (c->last_decode_kind == 1) body = c->decode_body_launches[c->last_gamma];
+    if (c->last_decode_kind == 2) body = c->greedy_body_launches;
+    // setup + loop_begin + steps x body + copy-out
+    *decode_launches = c->last_decode_kind ? 2 + static_cast<int64_t>(h.steps) * body + 1 : 0;
+  }
+  return SSD_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,152 @@
+"""Python face of the SSD library: owns torch device copies of the weights and
+forwards every call to the C ABI (include/ssd.h).  No computation happens here.
+"""
+from __future__ import annotations
+
+import ctypes
+
+import numpy as np
+import torch
+
+from . import _binding as B
+
+
+def _ptr(t) -> int | None:
+    return None if t is None else t.data_ptr()
+
+
+def bf16_bits_to_device(bits: np.ndarray, device="cuda") -> torch.Tensor:
+    """Upload bf16 bit patterns (numpy uint16) as a torch.bfloat16 device tensor."""
+    t = torch.from_numpy(np.ascontiguousarray(bits).view(np.int16))
+    return t.to(device).view(torch.bfloat16)
+
+
+class _DeviceArray:
+    """Minimal __cuda_array_interface__ holder to view library-owned memory from torch."""
+
+    def __init__(self, ptr: int, shape, typestr: str):
+        self.__cuda_array_interface__ = {"shape": tuple(shape), "typestr": typestr, "data": (ptr, False),
+                                         "version": 3, "strides": None}
+
+
+def _device_view(ptr: int, shape) -> torch.Tensor:
+    return torch.as_tensor(_DeviceArray(ptr, shape, "<i2"), device="cuda").view(torch.bfloat16)
+
+
+class SSDModel:
+    """One library context (ssd_ctx) over borrowed device weights.
+
+    weights: dict with bf16 device tensors "embed", "lm_head", "final_norm",
+    "layers" (list of dicts wq, wk, wv, wo, w_gate, w_up, w_down, attn_norm,
+    ffn_norm) and, for the MLP2 imitation network, "in_norm", "in_w1", "in_w2".
+    resid_scale: fp32 device tensor [n_layers]; in_scale: fp32 device tensor [1].
+    """
+
+    def __init__(self, cfg: dict, weights: dict, resid_scale: torch.Tensor, in_scale: torch.Tensor,
+                 stream: torch.cuda.Stream | None = None):
+        self.lib = B.load()
+        self.cfg = dict(cfg)
+        self.weights = weights            # keep the borrowed tensors alive
+        self.resid_scale = resid_scale
+        self.in_scale = in_scale
+        c = B.SSDConfig(**{k: self.cfg[k] for k, _ in B.SSDConfig._fields_})
+        L = cfg["n_layers"]
+        arrs = {}
+        for name in ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down", "attn_norm", "ffn_norm"):
+            arrs[name] = (ctypes.c_void_p * L)(*[weights["layers"][l][name].data_ptr() for l in range(L)])
+        self._arrs = arrs
+        w = B.SSDWeights(embed=_ptr(weights["embed"]), lm_head=_ptr(weights["lm_head"]),
+                         final_norm=_ptr(weights["final_norm"]),
+                         in_norm=_ptr(weights.get("in_norm")), in_w1=_ptr(weights.get("in_w1")),
+                         in_w2=_ptr(weights.get("in_w2")), resid_scale=_ptr(resid_scale),
+                         in_scale=_ptr(in_scale), **{k: ctypes.cast(v, B._PP) for k, v in arrs.items()})
+        self.stream = stream if stream is not None else torch.cuda.current_stream()
+        ctx = ctypes.c_void_p()
+        self._check(self.lib.ssd_create(ctypes.byref(c), ctypes.byref(w), self.stream.cuda_stream,
+                                        ctypes.byref(ctx)), None)
+        self.ctx = ctx
+
+    # ------------------------------------------------------------------ plumbing
+    def _check(self, status: int, ctx) -> None:
+        if status != 0:
+            msg = self.lib.ssd_last_error(ctx).decode() if ctx else B.STATUS.get(status, "")
+            raise B.SSDError(status, msg)
+
+    def _call(self, name: str, *args) -> None:
+        self._check(getattr(self.lib, name)(self.ctx, *args), self.ctx)
+
+    def close(self) -> None:
+        if getattr(self, "ctx", None):
+            self.lib.ssd_destroy(self.ctx)
+            self.ctx = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # ------------------------------------------------------------------ device-buffer calls (async)
+    def prefill(self, vis: torch.Tensor | None, prompt: torch.Tensor, first_tok: torch.Tensor | None = None):
+        n_vis = 0 if vis is None else vis.shape[0]
+        self._call("ssd_prefill", _ptr(vis), n_vis, _ptr(prompt), prompt.shape[0], _ptr(first_tok))
+
+    def draft(self, gamma: int, draft_tok: torch.Tensor | None = None):
+        self._call("ssd_draft", gamma, _ptr(draft_tok))
+
+    def verify(self, gamma: int, n_emitted: torch.Tensor | None = None, emitted: torch.Tensor | None = None):
+        self._call("ssd_verify", gamma, _ptr(n_emitted), _ptr(emitted))
+
+    def decode(self, max_new: int, gamma: int, out_tok: torch.Tensor | None = None,
+               n_out: torch.Tensor | None = None):
+        self._call("ssd_decode", max_new, gamma, _ptr(out_tok), _ptr(n_out))
+
+    def greedy_decode(self, max_new: int, out_tok: torch.Tensor | None = None, n_out: torch.Tensor | None = None):
+        self._call("ssd_greedy_decode", max_new, _ptr(out_tok), _ptr(n_out))
+
+    # ------------------------------------------------------------------ host-buffer calls (sync)
+    def _generate(self, name, vis: np.ndarray | torch.Tensor | None, prompt, max_new: int, *extra):
+        vis_p, n_vis = None, 0
+        if vis is not None:
+            n_vis = vis.shape[0]
+            vis_p = vis.data_ptr() if isinstance(vis, torch.Tensor) else vis.ctypes.data
+        prompt_arr = prompt if isinstance(prompt, torch.Tensor) else np.ascontiguousarray(prompt, dtype=np.int32)
+        pp = prompt_arr.data_ptr() if isinstance(prompt_arr, torch.Tensor) else prompt_arr.ctypes.data
+        out = np.zeros(max_new, dtype=np.int32)
+        n = ctypes.c_int(0)
+        st = B.SSDStats()
+        self._call(name, vis_p, n_vis, pp, len(prompt_arr), max_new, *extra, out.ctypes.data, ctypes.byref(n),
+                   ctypes.byref(st))
+        return out[:n.value].tolist(), st.as_dict()
+
+    def generate(self, vis, prompt, max_new: int, gamma: int):
+        """ssd_generate: host inputs in, host tokens + stats out."""
+        return self._generate("ssd_generate", vis, prompt, max_new, gamma)
+
+    def greedy_generate(self, vis, prompt, max_new: int):
+        return self._generate("ssd_greedy_generate", vis, prompt, max_new)
+
+    # ------------------------------------------------------------------ inspection
+    def sync(self):
+        self._call("ssd_sync")
+
+    def stats(self) -> dict:
+        st = B.SSDStats()
+        self._call("ssd_get_stats", ctypes.byref(st))
+        return st.as_dict()
+
+    def set_logits_capture(self, buf: torch.Tensor | None):
+        self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
+
+    def kv(self):
+        """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (bf16) of the library's cache."""
+        k, v, n = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_int()
+        self._call("ssd_get_kv", ctypes.byref(k), ctypes.byref(v), ctypes.byref(n))
+        c = self.cfg
+        shape = (c["n_layers"], c["n_heads"], c["max_seq"], c["head_dim"])
+        return _device_view(k.value, shape), _device_view(v.value, shape), n.value
+
+    def launch_counts(self) -> tuple[int, int]:
+        a, b = ctypes.c_int64(), ctypes.c_int64()
+        self._call("ssd_last_launch_count", ctypes.byref(a), ctypes.byref(b))
+        return a.value, b.value

@@ -1,0 +1,36 @@
+"""Builds a library context for a synthetic workload (device weights from synth)."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import paper_2510_22641_gb300 as lib
+import synth
+
+
+def device_weights(bits: dict) -> dict:
+    up = lib.bf16_bits_to_device
+    out = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm")}
+    out["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+    for k in ("in_norm", "in_w1", "in_w2"):
+        if k in bits:
+            out[k] = up(bits[k])
+    return out
+
+
+def make_model(w: synth.Workload, bits: dict | None = None, dev: dict | None = None, gamma_max: int | None = None,
+               max_seq: int | None = None):
+    bits = bits if bits is not None else synth.make_weights(w)
+    dev = dev if dev is not None else device_weights(bits)
+    cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, gamma_max or max(w.gamma, 1),
+                          max_seq or w.max_seq(), w.eos_id)
+    rs = torch.tensor(w.resid_scale(), dtype=torch.float32, device="cuda")
+    ins = torch.tensor([w.in_scale()], dtype=torch.float32, device="cuda")
+    return lib.SSDModel(cfg, dev, rs, ins), bits, dev
+
+
+def device_inputs(w: synth.Workload, seed: int | None = None):
+    vis, prompt = synth.make_inputs(w, seed)
+    v = lib.bf16_bits_to_device(vis) if w.n_vis > 0 else None
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    return vis, prompt, v, p

@@ -1,0 +1,269 @@
+"""CUDA path vs the fp64 oracle on the tiny workload and its edge cases (through the C ABI).
+
+Sizes here finish in seconds in the oracle yet span several 128x64 weight
+units per matrix, several 64-key attention chunks, a ragged prefill chunk and
+a vocabulary tail.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2510_22641_gb300 as lib
+import synth
+from tests.gpu_util import device_inputs, make_model
+from tests.parity import assert_logits_close, common_prefix, steps_before
+
+pytestmark = pytest.mark.gpu
+
+
+def run_oracle(w, bits, gamma=None, greedy=False):
+    m = oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    if greedy:
+        return oracle.greedy_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, max_seq=w.max_seq())
+    return oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma or w.gamma)
+
+
+def gpu_decode(model, w, gamma, capture=True):
+    """prefill + decode through the device-buffer entry points; returns tokens, logits, stats."""
+    _, _, v, p = device_inputs(w)
+    logits = torch.full((w.max_new, w.shape.vocab), float("nan"), device="cuda") if capture else None
+    model.set_logits_capture(logits)
+    out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
+    n = torch.zeros(1, dtype=torch.int32, device="cuda")
+    model.prefill(v, p)
+    if gamma > 0:
+        model.decode(w.max_new, gamma, out, n)
+    else:
+        model.greedy_decode(w.max_new, out, n)
+    model.sync()
+    toks = out[: int(n.item())].cpu().tolist()
+    return toks, (logits.cpu().numpy() if capture else None), model.stats()
+
+
+def check_against_oracle(toks, logits, stats, ref, gamma):
+    agree = common_prefix(toks, ref.tokens, ref.logits)
+    for t in range(min(agree + 1, len(ref.tokens))):
+        assert_logits_close(logits[t], ref.logits[t], f"logits of token {t}")
+    if gamma > 0:
+        k = steps_before(ref.accept_lengths, agree)
+        hist = np.bincount(ref.accept_lengths[:k], minlength=synth.LLAVA7B.gamma + 4)
+        if agree == len(ref.tokens):
+            assert stats["steps"] == len(ref.accept_lengths)
+            assert stats["accepted"] == sum(ref.accept_lengths)
+            assert stats["kv_len"] == ref.kv_len
+            assert stats["accept_hist"][: gamma + 1] == np.bincount(ref.accept_lengths, minlength=gamma + 1).tolist()
+        assert k <= stats["steps"] and hist.sum() == k
+    return agree
+
+
+@pytest.fixture(scope="module")
+def tiny_bits():
+    return synth.make_weights(synth.TINY.replace(norm_gain="perturbed"))
+
+
+@pytest.fixture(scope="module")
+def tiny_model(tiny_bits):
+    w = synth.TINY.replace(norm_gain="perturbed", gamma=8)
+    model, _, dev = make_model(w, tiny_bits, gamma_max=8, max_seq=w.max_seq())
+    yield model, dev
+    model.close()
+
+
+def set_scale(model, w):
+    model.resid_scale.copy_(torch.tensor(w.resid_scale(), device="cuda"))
+    model.in_scale.copy_(torch.tensor([w.in_scale()], device="cuda"))
+
+
+def test_greedy_matches_oracle(tiny_model, tiny_bits):
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=1.0)
+    set_scale(model, w)
+    toks, logits, _ = gpu_decode(model, w, 0)
+    ref = run_oracle(w, tiny_bits, greedy=True)
+    assert check_against_oracle(toks, logits, {}, ref, 0) >= 8
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.2, 4), (1.0, 4), (0.2, 1), (0.05, 8), (0.2, 3)])
+def test_ssd_matches_oracle_and_gpu_greedy(tiny_model, tiny_bits, s, gamma):
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=s)
+    set_scale(model, w)
+    toks, logits, stats = gpu_decode(model, w, gamma)
+    ref = run_oracle(w, tiny_bits, gamma)
+    check_against_oracle(toks, logits, stats, ref, gamma)
+    # batch invariance: the verify pass (gamma+1 rows) reproduces greedy decoding bitwise
+    gtoks, glogits, _ = gpu_decode(model, w, 0)
+    assert toks == gtoks
+    np.testing.assert_array_equal(logits, glogits)
+    assert stats["emitted"] == w.max_new
+    assert sum(a * c for a, c in enumerate(stats["accept_hist"])) == stats["accepted"]
+    assert stats["steps"] + stats["accepted"] + 1 == w.max_new
+
+
+def test_kv_cache_after_rollback_equals_greedy_cache(tiny_model):
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    set_scale(model, w)
+    gpu_decode(model, w, 4, capture=False)
+    k1, v1, n1 = model.kv()
+    k1, v1 = k1[:, :, :n1].clone(), v1[:, :, :n1].clone()
+    gpu_decode(model, w, 0, capture=False)
+    k2, v2, n2 = model.kv()
+    assert n1 == n2 == w.prompt_len + w.max_new - 1
+    assert torch.equal(k1.view(torch.int16), k2[:, :, :n2].view(torch.int16))
+    assert torch.equal(v1.view(torch.int16), v2[:, :, :n2].view(torch.int16))
+
+
+def test_prefill_kv_matches_oracle(tiny_bits):
+    w = synth.TINY.replace(norm_gain="perturbed", max_new=1)
+    model, _, _ = make_model(w, tiny_bits)
+    gpu_decode(model, w, 0, capture=False)
+    k, v, n = model.kv()
+    m = oracle.model_from_bits(w, tiny_bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    cache = oracle.KVCache(m.cfg, w.max_seq())
+    oracle.prefill(m, cache, synth.bf16_to_f64(vis), prompt)
+    P = w.prompt_len
+    assert n == P
+    for got, ref in ((k, cache.k), (v, cache.v)):
+        g = got[:, :, :P].float().cpu().numpy()
+        r = ref[:, :, :P]
+        # bf16 storage (relative 2^-9) plus drift from bf16 K/V in earlier layers
+        rms = float(np.sqrt(np.mean(r * r)))
+        np.testing.assert_allclose(g, r, rtol=2e-2, atol=2e-2 * rms)
+    model.close()
+
+
+def test_draft_exit_at_L_identity_accepts_everything(tiny_bits):
+    w = synth.TINY.replace(norm_gain="perturbed", draft_exit_k=4, in_kind=synth.IN_IDENTITY, gamma=4, max_new=20)
+    model, _, _ = make_model(w, tiny_bits)
+    toks, logits, stats = gpu_decode(model, w, 4)
+    assert stats["accept_hist"][:5] == [0, 0, 0, 1, 3]
+    ref = run_oracle(w, tiny_bits, 4)
+    check_against_oracle(toks, logits, stats, ref, 4)
+    model.close()
+
+
+def test_standalone_draft_and_verify_steps(tiny_model, tiny_bits):
+    """ssd_draft / ssd_verify per step == the oracle's drafts, accepts and emitted tokens."""
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=0.05, max_new=1000)
+    set_scale(model, w)
+    gamma = 4
+    ref = run_oracle(w.replace(max_new=26), tiny_bits, gamma)
+    _, _, v, p = device_inputs(w)
+    model.set_logits_capture(None)
+    first = torch.zeros(1, dtype=torch.int32, device="cuda")
+    model.prefill(v, p, first)
+    d = torch.zeros(gamma, dtype=torch.int32, device="cuda")
+    ne = torch.zeros(1, dtype=torch.int32, device="cuda")
+    em = torch.zeros(gamma + 1, dtype=torch.int32, device="cuda")
+    toks = [int(first.item())]
+    for step in range(4):
+        model.draft(gamma, d)
+        model.verify(gamma, ne, em)
+        model.sync()
+        n = int(ne.item())
+        if toks + em[:n].cpu().tolist() != ref.tokens[: len(toks) + n]:
+            break  # streams parted (allowed only at a low-margin position, checked below)
+        if d.cpu().tolist()[: ref.accept_lengths[step]] != ref.draft_tokens[step][: ref.accept_lengths[step]]:
+            raise AssertionError("accepted drafts differ from the oracle's")
+        assert n == ref.accept_lengths[step] + 1
+        toks += em[:n].cpu().tolist()
+    common_prefix(toks, ref.tokens[: len(toks)], ref.logits)
+    assert len(toks) > 4
+
+
+@pytest.mark.parametrize("case", ["ragged_prefill", "vocab_tail", "no_visual", "head128", "narrow_in",
+                                  "max_new_1", "max_new_2"])
+def test_edge_shapes(case):
+    base = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    w = {
+        "ragged_prefill": base.replace(n_vis=29, n_prompt=14),                 # P = 43, chunks of 8 + 3
+        "vocab_tail": base.replace(shape=synth.ModelShape(4, 256, 4, 64, 1024, 2000)),
+        "no_visual": base.replace(n_vis=0, n_prompt=21),
+        "head128": base.replace(shape=synth.ModelShape(3, 256, 2, 128, 512, 1024), draft_exit_k=1),
+        "narrow_in": base.replace(in_hidden=192),
+        "max_new_1": base.replace(max_new=1),
+        "max_new_2": base.replace(max_new=2),
+    }[case]
+    bits = synth.make_weights(w)
+    model, _, _ = make_model(w, bits)
+    toks, logits, stats = gpu_decode(model, w, w.gamma)
+    ref = run_oracle(w, bits, w.gamma)
+    check_against_oracle(toks, logits, stats, ref, w.gamma)
+    gtoks, _, _ = gpu_decode(model, w, 0)
+    assert toks == gtoks
+    model.close()
+
+
+def test_eos_stops_like_oracle(tiny_bits):
+    w0 = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    ref0 = run_oracle(w0, tiny_bits, greedy=True)
+    eos = ref0.tokens[6]
+    w = w0.replace(eos_id=eos)
+    model, _, _ = make_model(w, tiny_bits)
+    toks, logits, stats = gpu_decode(model, w, w.gamma)
+    ref = run_oracle(w, tiny_bits, w.gamma)
+    assert ref.tokens[-1] == eos and len(ref.tokens) < w.max_new
+    check_against_oracle(toks, logits, stats, ref, w.gamma)
+    model.close()
+
+
+def test_host_buffer_generate_equals_device_decode(tiny_model):
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    set_scale(model, w)
+    toks, _, st = gpu_decode(model, w, 4, capture=False)
+    vis, prompt = synth.make_inputs(w)
+    htoks, hst = model.generate(vis, prompt, w.max_new, 4)
+    assert htoks == toks and hst["accepted"] == st["accepted"]
+    gt, _ = model.greedy_generate(vis, prompt, w.max_new)
+    assert gt == toks
+
+
+def test_abi_errors_on_gpu(tiny_bits):
+    w = synth.TINY.replace(norm_gain="perturbed")
+    model, _, _ = make_model(w, tiny_bits)
+    with pytest.raises(lib.SSDError) as e:
+        model.verify(4)                                   # no prefill / draft
+    assert e.value.status == 5
+    with pytest.raises(lib.SSDError) as e:
+        model.decode(w.max_new, 4)                        # decode before prefill
+    assert e.value.status == 5
+    _, _, v, p = device_inputs(w)
+    model.prefill(v, p)
+    with pytest.raises(lib.SSDError) as e:
+        model.decode(w.max_seq(), 4)                      # capacity
+    assert e.value.status == 4
+    with pytest.raises(lib.SSDError) as e:
+        model.draft(9)                                    # gamma > gamma_max
+    assert e.value.status == 1
+    model.draft(2)
+    with pytest.raises(lib.SSDError) as e:
+        model.verify(3)                                   # gamma differs from the draft's
+    assert e.value.status == 5
+    bad = p.clone()
+    bad[3] = w.shape.vocab + 5                            # token id out of range -> device error word
+    model.prefill(v, bad)
+    with pytest.raises(lib.SSDError) as e:
+        model.sync()
+    assert e.value.status == 7
+    model.prefill(v, p)                                   # the context stays usable
+    model.decode(w.max_new, 4)
+    model.sync()
+    model.close()
+
+
+def test_launch_counts(tiny_model):
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    set_scale(model, w)
+    _, _, st = gpu_decode(model, w, 4, capture=False)
+    pre, dec = model.launch_counts()
+    L, k = w.shape.n_layers, w.draft_exit_k
+    body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
+    assert dec == 3 + st["steps"] * body
+    assert pre == 2 + ((w.prompt_len + 7) // 8) * (1 + 5 * L) + 1
