@@ -1,0 +1,345 @@
+"""Benchmark of greedy self-speculative decoding on the LLaVA-1.5-7B-shaped workload.
+
+One step = one request through the whole hot path with inputs resident in HBM:
+prefill of 576 synthetic visual rows + 64 prompt ids, then 128 new tokens by
+self-speculative decoding (draft = layers 0..7 + imitation network, gamma = 5,
+full-model verification, on-device accept/rollback), batch 1.
+
+Printed as one JSON line (rank 0):
+  value          new tokens / second over whole requests (prefill included)
+  e2e            the same through ssd_generate with pinned host buffers
+                 (host->device inputs and device->host tokens inside the timing)
+  roofline       the dominant kernel (weight-streaming GEMV, gate/up, 1 row)
+                 timed alone with CUDA events, against the measured HBM copy peak
+  per_s          decode tokens/s of SSD and of greedy decoding (same kernels)
+                 and their ratio for s in {0.05, 0.2, 1.0}
+  cpu_baseline   the fp64 oracle on the host cores over a bounded sample
+
+--impl reference times that oracle itself (rank 0 only).
+Multi-GPU (torchrun): independent replicas, one request stream per GPU.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "tokens/s and speedup vs full-model greedy decode (7B shape, bs1); HBM GB/s"
+UNIT = "tokens/s"
+S_VALUES = synth.LLAVA7B_S_VALUES
+
+
+def workload_config(w: synth.Workload) -> dict:
+    sh = w.shape
+    return {"workload": f"{w.name}: L={sh.n_layers} d={sh.d_model} H={sh.n_heads}x{sh.head_dim} "
+                        f"ff={sh.d_ff} V={sh.vocab}, {w.n_vis} visual + {w.n_prompt} prompt, "
+                        f"{w.max_new} new tokens, k={w.draft_exit_k}, gamma={w.gamma}, s={w.s}, bs1",
+            "batch": 1, "prompt_rows": w.prompt_len, "max_new": w.max_new, "draft_exit_k": w.draft_exit_k,
+            "gamma": w.gamma, "s": w.s, "weights": "bf16 N(0,0.02) random-init, seed 0",
+            "inputs": "visual N(0,1) bf16 + prompt ids U[0,V), seeded",
+            "l2": "no flush needed: each step streams 13.5 GB of weights (>> 129 MB L2) dozens of times"}
+
+
+def algorithmic_bytes(w: synth.Workload) -> dict:
+    """Bytes the method must move (bf16 weights; KV per position per layer = 2*H*Dh*2)."""
+    sh = w.shape
+    layer = 2 * (4 * sh.d_model * sh.qdim + 3 * sh.d_model * sh.d_ff)
+    head = 2 * sh.vocab * sh.d_model
+    imit = 2 * 2 * sh.d_model * w.in_hidden if w.in_kind == synth.IN_MLP2 else 0
+    kv_pos = 2 * sh.n_heads * sh.head_dim * 2
+    return {"layer": layer, "head": head, "imit": imit, "kv_pos_layer": kv_pos,
+            "draft_token": w.draft_exit_k * layer + imit + head,
+            "verify": sh.n_layers * layer + head, "greedy_token": sh.n_layers * layer + head}
+
+
+# --------------------------------------------------------------------------- clocks
+
+CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+           "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+           "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, gpu: int):
+        self.p = None
+        try:
+            self.p = subprocess.Popen(["nvidia-smi", f"--query-gpu={CLOCK_Q}", "--format=csv,noheader,nounits",
+                                       "-i", str(gpu), "-lms", "200"], stdout=subprocess.PIPE,
+                                      stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.p = None
+
+    def stop(self) -> dict | None:
+        if self.p is None:
+            return None
+        self.p.terminate()
+        try:
+            out, _ = self.p.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.p.kill()
+            out, _ = self.p.communicate()
+        sm, smax, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = max(smax, float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": smax, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- oracle legs (CPU)
+
+def oracle_sample(w: synth.Workload, bits, vis, prompt, max_steps: int, warm_steps: int = 0) -> dict:
+    """Time the fp64 oracle on this workload: its prefill and `max_steps` SSD steps."""
+    import oracle
+    t0 = time.perf_counter()
+    m = oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    t_conv = time.perf_counter() - t0
+    r = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, w.gamma,
+                            max_steps=warm_steps + max_steps)
+    steps = r.step_s[warm_steps:]
+    acc = r.accept_lengths[warm_steps:]
+    toks_per_step = (sum(acc) + len(acc)) / max(len(acc), 1)
+    step_mean = sum(steps) / max(len(steps), 1)
+    request_s = r.prefill_s + (w.max_new - 1) / toks_per_step * step_mean
+    return {"value": w.max_new / request_s, "prefill_s": r.prefill_s, "step_s": step_mean,
+            "tokens_per_step": toks_per_step, "n_steps": len(steps), "convert_s": t_conv,
+            "cores": os.cpu_count()}
+
+
+def run_reference(args) -> None:
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = synth.LLAVA7B.replace(s=args.s)
+    bits = synth.make_weights(w)
+    vis, prompt = synth.make_inputs(w)
+    r = oracle_sample(w, bits, vis, prompt, max_steps=args.steps, warm_steps=args.warmup)
+    sample = (f"fp64 numpy oracle: one prefill ({w.prompt_len} rows) + {args.warmup} warm-up and "
+              f"{r['n_steps']} timed SSD steps; tokens/s = {w.max_new} / (prefill + {w.max_new - 1} tokens "
+              f"at the sampled tokens per step and step time)")
+    line = {"impl": "reference", "metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["step_s"] * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(w),
+            "cpu_baseline": {"value": r["value"], "unit": UNIT, "cores": r["cores"], "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": r["value"], "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+            "prefill_s": r["prefill_s"], "tokens_per_step": r["tokens_per_step"]}
+    print(json.dumps(line), flush=True)
+
+
+# --------------------------------------------------------------------------- GPU arm
+
+def main() -> None:
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--s", type=float, default=0.2, help="deep-layer residual scale of the headline run")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-steps", type=int, default=3, help="oracle SSD steps in the CPU sample")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+        return
+    assert args.warmup >= 3, "at least 3 warm-up steps"
+
+    import torch
+    import torch.distributed as dist
+
+    import paper_2510_22641_gb300 as lib
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    lib.build()
+    dev_id = torch.cuda.current_device()
+
+    w = synth.LLAVA7B.replace(s=args.s)
+    bits = synth.make_weights(w)
+    up = lib.bf16_bits_to_device
+    dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm", "in_norm", "in_w1", "in_w2")}
+    dev["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+    rs = torch.tensor(w.resid_scale(), device="cuda")
+    ins = torch.tensor([w.in_scale()], device="cuda")
+    cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                          w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1)
+    model = lib.SSDModel(cfg, dev, rs, ins)
+    vis, prompt = synth.make_inputs(w, seed=rank)
+    v = up(vis)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
+    n_out = torch.zeros(1, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def request(gamma: int, ev=None):
+        model.prefill(v, p)
+        if ev is not None:
+            ev.record(stream)
+        if gamma > 0:
+            model.decode(w.max_new, gamma, out, n_out)
+        else:
+            model.greedy_decode(w.max_new, out, n_out)
+
+    for _ in range(args.warmup):
+        request(w.gamma)
+    model.greedy_decode(w.max_new, out, n_out)   # builds the greedy graph outside the timed region
+    model.sync()
+
+    # ---------------- timed region: K requests
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(2 * args.steps + 1)]
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(dev_id)
+    time.sleep(0.3)
+    evs[0].record(stream)
+    for i in range(args.steps):
+        request(w.gamma, evs[2 * i + 1])
+        evs[2 * i + 2].record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    total_ms = evs[0].elapsed_time(evs[-1])
+    prefill_ms = [evs[2 * i].elapsed_time(evs[2 * i + 1]) for i in range(args.steps)]
+    decode_ms = [evs[2 * i + 1].elapsed_time(evs[2 * i + 2]) for i in range(args.steps)]
+    model.sync()
+    assert int(n_out.item()) == w.max_new
+    st = model.stats()
+    pre_l, dec_l = model.launch_counts()
+    if world > 1:
+        t = torch.tensor([total_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    value = world * args.steps * w.max_new / (total_ms / 1e3)
+
+    # ---------------- end to end through ssd_generate with pinned host buffers
+    vis_h = torch.from_numpy(vis.view(np.int16)).pin_memory()
+    prompt_h = torch.from_numpy(prompt.astype(np.int32)).pin_memory()
+    model.generate(vis_h, prompt_h, w.max_new, w.gamma)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(args.steps):
+        toks, _ = model.generate(vis_h, prompt_h, w.max_new, w.gamma)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = e0.elapsed_time(e1)
+    e2e = {"value": args.steps * w.max_new / (e2e_ms / 1e3), "unit": UNIT,
+           "h2d_bytes_per_step": int(vis.nbytes + 4 * prompt.size), "d2h_bytes_per_step": 4 * w.max_new}
+
+    # ---------------- speedup over greedy decoding per acceptance knob s (decode only)
+    per_s = []
+    for s in S_VALUES:
+        ws = w.replace(s=s)
+        rs.copy_(torch.tensor(ws.resid_scale(), device="cuda"))
+        ins.copy_(torch.tensor([ws.in_scale()], device="cuda"))
+        row = {"s": s}
+        for name, gamma in (("ssd", w.gamma), ("greedy", 0)):
+            ts = []
+            for _ in range(2):
+                a, b, c = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+                a.record(stream)
+                request(gamma, b)
+                c.record(stream)
+                torch.cuda.synchronize()
+                ts.append(b.elapsed_time(c))
+            row[f"{name}_decode_tok_s"] = (w.max_new - 1) / (min(ts) / 1e3)
+            if name == "ssd":
+                sst = model.stats()
+                row["mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
+                row["steps"] = sst["steps"]
+        row["speedup"] = row["ssd_decode_tok_s"] / row["greedy_decode_tok_s"]
+        per_s.append(row)
+    rs.copy_(torch.tensor(w.resid_scale(), device="cuda"))
+    ins.copy_(torch.tensor([w.in_scale()], device="cuda"))
+
+    # ---------------- dominant kernel alone: gate/up GEMV, 1 row (the draft's largest projection)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except OSError:
+        pass
+    hbm_peak = float(peaks.get("hbm_gbs", 6800.0))
+    peak_src = "measured" if "hbm_gbs" in peaks else "fallback"
+    reps = 200
+    model.profile_projection("gateup", layer=0, rows=1, reps=10)
+    k0, k1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    k0.record(stream)
+    nbytes = model.profile_projection("gateup", layer=0, rows=1, reps=reps)
+    k1.record(stream)
+    torch.cuda.synchronize()
+    kern_ms = k0.elapsed_time(k1) / reps
+    achieved = nbytes / (kern_ms / 1e3) / 1e9
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                "frac": achieved / hbm_peak, "traffic": None,
+                "kernel": "gemv_kernel<1, GATE_SILU> (layer gate/up, 2x11008x4096 bf16, 1 row)",
+                "bytes_per_launch": nbytes, "launch_us": kern_ms * 1e3,
+                "peak_source": f"{peak_src} HBM copy (burst)"}
+    model.prefill(v, p)   # the profiling launches clobbered the decode state
+    model.sync()
+
+    # decode-phase bandwidth from algorithmic bytes
+    ab = algorithmic_bytes(w)
+    steps_per_req = st["steps"]
+    kv_read = ab["kv_pos_layer"] * (w.prompt_len + w.max_new / 2) * (
+        steps_per_req * (w.gamma * w.draft_exit_k + w.shape.n_layers))
+    dec_bytes = steps_per_req * (w.gamma * ab["draft_token"] + ab["verify"]) + kv_read
+    dec_ms = statistics.median(decode_ms)
+
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {**workload_config(w), "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                       "arithmetic": "fp32 FMA on bf16 weights, bf16 KV cache"},
+            "e2e": e2e, "gpu_launches": int(args.steps * (pre_l + dec_l)),
+            "roofline": roofline, "clocks": clk,
+            "prefill_ms": statistics.median(prefill_ms), "decode_ms": dec_ms,
+            "decode_tokens_per_s": (w.max_new - 1) / (dec_ms / 1e3),
+            "decode_hbm_gbs": dec_bytes / (dec_ms / 1e3) / 1e9,
+            "decode_hbm_frac": dec_bytes / (dec_ms / 1e3) / 1e9 / hbm_peak,
+            "ssd_steps": st["steps"], "accepted": st["accepted"], "drafted": st["drafted"],
+            "accept_hist": st["accept_hist"][: w.gamma + 1], "per_s": per_s}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        r = oracle_sample(w, bits, vis, prompt, max_steps=args.cpu_steps)
+        line["cpu_baseline"] = {"value": r["value"], "unit": UNIT, "cores": r["cores"], "kind": "oracle",
+                                "sample": (f"fp64 numpy oracle on this workload: prefill ({w.prompt_len} rows, "
+                                           f"{r['prefill_s']:.1f} s) + {r['n_steps']} SSD steps "
+                                           f"({r['step_s']:.2f} s each, {r['tokens_per_step']:.2f} tokens/step), "
+                                           f"scaled to {w.max_new} tokens per request")}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    model.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

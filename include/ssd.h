@@ -208,6 +208,16 @@ SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v
  * ssd_prefill performed (from the device step counter).  sync. */
 SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches, int64_t* decode_launches);
 
+/* Diagnostic for timing one kernel alone: enqueue `reps` back-to-back launches
+ * of one weight-streaming projection (the GEMV kernel with its fused
+ * epilogue) over `rows` activation rows, with whatever activations the ctx
+ * holds.  which: 0 QKV, 1 o_proj, 2 gate/up, 3 down (of `layer`), 4 LM head,
+ * 5 imitation FC1, 6 imitation FC2.  *bytes receives the algorithmic bytes one
+ * launch moves (weights + activation rows in + results out).  Clobbers the
+ * decode state (activations, cache rows at kv_len..kv_len+rows-1): call
+ * ssd_prefill before decoding again.  async. */
+SSD_API ssd_status ssd_profile_projection(ssd_ctx* ctx, int which, int layer, int rows, int reps, int64_t* bytes);
+
 SSD_API const char* ssd_status_string(ssd_status s);
 SSD_API const char* ssd_last_error(const ssd_ctx* ctx);
 

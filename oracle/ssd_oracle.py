@@ -42,6 +42,7 @@ decoding agree bitwise here, not only up to rounding.
 from __future__ import annotations
 
 import dataclasses
+import time
 
 import numpy as np
 
@@ -190,9 +191,9 @@ def prefill(m: Model, cache: KVCache, vis: np.ndarray, prompt) -> np.ndarray:
             K[p] = rope(K[p], p, c.rope_theta)
         cache.k[l, :, :P] = K.transpose(1, 0, 2)
         cache.v[l, :, :P] = V.transpose(1, 0, 2)
-        S = np.einsum("ihd,jhd->hij", Q, K) / np.sqrt(Dh)
+        S = np.matmul(Q.transpose(1, 0, 2), K.transpose(1, 2, 0)) / np.sqrt(Dh)     # [H][i][j]
         S = np.where(causal[None], S, -np.inf)
-        O = np.einsum("hij,jhd->ihd", softmax(S), V).reshape(P, H * Dh)
+        O = np.matmul(softmax(S), V.transpose(1, 0, 2)).transpose(1, 0, 2).reshape(P, H * Dh)
         Hh = X + m.s[l] * (O @ lw["wo"].T)
         U = rms_norm(Hh, lw["ffn_norm"], c.rms_eps)
         X = Hh + m.s[l] * ((silu(U @ lw["w_gate"].T) * (U @ lw["w_up"].T)) @ lw["w_down"].T)
@@ -211,6 +212,8 @@ class Result:
     draft_tokens: list = dataclasses.field(default_factory=list)     # per step: d_1..d_gamma_eff
     draft_logits: list = dataclasses.field(default_factory=list)     # per step: g(I(x_k)) rows
     cache: KVCache | None = None
+    prefill_s: float = 0.0                                            # wall time of the prefill
+    step_s: list = dataclasses.field(default_factory=list)            # wall time per decode step
 
 
 def _truncate_eos(tokens: list, eos_id: int) -> tuple[list, bool]:
@@ -239,7 +242,8 @@ def greedy_generate(m: Model, vis: np.ndarray, prompt, max_new: int, max_seq: in
 
 def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                  max_seq: int | None = None, reuse_draft_rows: bool = True,
-                 keep_cache: bool = False, keep_draft_logits: bool = False) -> Result:
+                 keep_cache: bool = False, keep_draft_logits: bool = False,
+                 max_steps: int | None = None) -> Result:
     """Algorithm 1 (greedy self-speculative decoding with the imitation network).
 
     Per step, with y the last emitted token at position p = kv_len:
@@ -249,16 +253,19 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                  (shallow layers reused from the draft when reuse_draft_rows)
       accepting: a = largest i <= gamma_eff with d_1..d_i = f_0..f_{i-1};
                  emit d_1..d_a and f_a; kv_len = p + a + 1; y = f_a.
+    max_steps (timing samples only) stops after that many steps.
     """
     c = m.cfg
     k, L = c.draft_exit_k, c.n_layers
     P = vis.shape[0] + len(prompt)
     cache = KVCache(c, max_seq or (P + max_new + gamma + 1))
+    t0 = time.perf_counter()
     o = prefill(m, cache, vis, prompt)
     y = argmax_lowest(o)
-    res = Result(tokens=[y], logits=[o], kv_len=P)
+    res = Result(tokens=[y], logits=[o], kv_len=P, prefill_s=time.perf_counter() - t0)
     p, done = P, (c.eos_id >= 0 and y == c.eos_id)
-    while len(res.tokens) < max_new and not done:
+    while len(res.tokens) < max_new and not done and (max_steps is None or len(res.step_s) < max_steps):
+        t0 = time.perf_counter()
         remaining = max_new - len(res.tokens)
         g_eff = min(gamma, remaining - 1)
         toks, xk, dlog = [y], [], []
@@ -292,6 +299,7 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
         p += a + 1
         y = f[a]
         res.kv_lens.append(p)
+        res.step_s.append(time.perf_counter() - t0)
     res.kv_len = p
     if keep_cache:
         res.cache = cache

@@ -928,4 +928,84 @@ ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t*
   return SSD_OK;
 }
 
+ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, int reps, int64_t* bytes) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (rows < 1 || rows > kMaxVerifyRows || reps < 1) return fail(c, SSD_ERR_INVALID_ARG, "rows / reps");
+  if (which < 0 || which > 6 || layer < 0 || layer >= c->cfg.n_layers)
+    return fail(c, SSD_ERR_INVALID_ARG, "which / layer");
+  if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))
+    return fail(c, SSD_ERR_INVALID_ARG, "imitation projections need SSD_IN_MLP2 and rows == 1");
+  const int d = c->cfg.d_model;
+  const Site* site = nullptr;
+  Epi e = Epi::RESID;
+  GemvParams p{};
+  p.x = c->xv;
+  p.x_stride = d;
+  switch (which) {
+    case 0:
+      site = &c->layers[layer].qkv;
+      e = Epi::QKV;
+      p.gain = c->attn_norm[layer];
+      p.q_out = c->qb;
+      p.q_stride = c->qdim;
+      p.k_cache = c->kc + layer * c->layer_kv;
+      p.v_cache = c->vc + layer * c->layer_kv;
+      p.head_dim = c->cfg.head_dim;
+      p.max_seq = c->cfg.max_seq;
+      p.rope_cs = c->rope;
+      break;
+    case 1:
+    case 3:
+      site = which == 1 ? &c->layers[layer].o : &c->layers[layer].down;
+      p.x = which == 1 ? c->ob : c->hb;
+      p.x_stride = which == 1 ? c->qdim : c->cfg.d_ff;
+      p.base = c->xt;
+      p.base_stride = d;
+      p.dst = c->xt;
+      p.dst_stride = d;
+      p.scale = c->resid_scale + layer;
+      break;
+    case 2:
+      site = &c->layers[layer].gateup;
+      e = Epi::GATE_SILU;
+      p.gain = c->ffn_norm[layer];
+      p.h_out = c->hb;
+      p.h_stride = c->cfg.d_ff;
+      break;
+    case 4:
+      site = &c->head;
+      e = Epi::ARGMAX;
+      p.gain = c->final_norm;
+      p.tok_dst = st_field(c, offsetof(DevState, full_tok));
+      break;
+    case 5:
+      site = &c->in1;
+      e = Epi::SILU;
+      p.gain = c->in_norm;
+      p.h_out = c->hin;
+      p.h_stride = c->cfg.in_hidden;
+      break;
+    default:
+      site = &c->in2;
+      p.x = c->hin;
+      p.x_stride = c->cfg.in_hidden;
+      p.base = c->xt;
+      p.base_stride = d;
+      p.dst = c->xt;
+      p.dst_stride = d;
+      p.scale = c->in_scale;
+      break;
+  }
+  const int64_t N = site->N * (e == Epi::GATE_SILU ? 2 : 1);
+  const int64_t out_elems = e == Epi::GATE_SILU ? site->N : (e == Epi::ARGMAX ? 1 : site->N);
+  const int64_t out_bytes = e == Epi::QKV ? rows * (c->qdim * 4 + 2 * c->qdim * 2) : rows * out_elems * 4;
+  if (bytes)
+    *bytes = N * site->K * 2 + static_cast<int64_t>(rows) * site->K * 4 + (p.gain ? site->K * 2 : 0) + out_bytes +
+             (e == Epi::RESID ? static_cast<int64_t>(rows) * site->N * 4 : 0);
+  CKS(enter(c));
+  for (int r = 0; r < reps; ++r) CKS(gemv(c, e, rows, *site, p));
+  c->prefilled = false;
+  return leave(c);
+}
+
 }  // extern "C"

@@ -146,6 +146,14 @@ class SSDModel:
         shape = (c["n_layers"], c["n_heads"], c["max_seq"], c["head_dim"])
         return _device_view(k.value, shape), _device_view(v.value, shape), n.value
 
+    PROJECTIONS = {"qkv": 0, "o": 1, "gateup": 2, "down": 3, "head": 4, "in1": 5, "in2": 6}
+
+    def profile_projection(self, which: str, layer: int = 0, rows: int = 1, reps: int = 1) -> int:
+        """Enqueue reps launches of one projection kernel; returns algorithmic bytes per launch."""
+        b = ctypes.c_int64()
+        self._call("ssd_profile_projection", self.PROJECTIONS[which], layer, rows, reps, ctypes.byref(b))
+        return b.value
+
     def launch_counts(self) -> tuple[int, int]:
         a, b = ctypes.c_int64(), ctypes.c_int64()
         self._call("ssd_last_launch_count", ctypes.byref(a), ctypes.byref(b))
