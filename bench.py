@@ -318,7 +318,7 @@ def main() -> None:
             "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
             "config": {**workload_config(w), "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                       "arithmetic": "fp32 FMA on bf16 weights, bf16 KV cache"},
+                       "arithmetic": "fp32 FMA on bf16 weights, fp32 activations and KV cache"},
             "e2e": e2e, "gpu_launches": int(args.steps * (pre_l + dec_l)),
             "roofline": roofline, "clocks": clk,
             "prefill_ms": statistics.median(prefill_ms), "decode_ms": dec_ms,

@@ -19,6 +19,8 @@
  *    that was current at ssd_create; "host" pointers are ordinary CPU memory.
  *  - Weights are BORROWED: the caller owns them and must keep them alive and
  *    unchanged (except resid_scale / in_scale, see below) until ssd_destroy.
+ *    The RMSNorm gain vectors are the exception: ssd_create copies them
+ *    (zero-padded) into library memory.
  *    Everything else (KV cache, workspaces, CUDA graphs) is owned by the ctx.
  *  - A ctx is bound to one CUDA stream and is not thread-safe.  Calls marked
  *    "async" only enqueue work on that stream; "sync" calls wait for it.
@@ -124,7 +126,7 @@ typedef struct {
 } ssd_stats;
 
 /* Create a context: checks the shape, builds TMA descriptors for the borrowed
- * weights, allocates the KV cache [L][H][max_seq][head_dim] bf16 (K and V),
+ * weights, allocates the KV cache [L][H][max_seq][head_dim] fp32 (K and V),
  * activations and workspaces on the current device.  cuda_stream is a
  * cudaStream_t (NULL = legacy default stream).  sync. */
 SSD_API ssd_status ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, ssd_ctx** out);
@@ -200,7 +202,7 @@ SSD_API ssd_status ssd_get_stats(ssd_ctx* ctx, ssd_stats* stats);
 SSD_API ssd_status ssd_set_logits_capture(ssd_ctx* ctx, float* buf, int max_rows);
 
 /* Device pointers to the KV cache, layout [L][n_heads][max_seq][head_dim]
- * bf16, and the current valid length (sync read).  Positions >= kv_len hold
+ * fp32, and the current valid length (sync read).  Positions >= kv_len hold
  * stale rows of rejected drafts. */
 SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v_cache, int* kv_len);
 

@@ -2,190 +2,218 @@
 // M query rows (Sec. "Methodology", KV cache: draft and verify read one cache).
 //
 // Row m sits at position base + m (base = st->kv_len + pos_off) and attends
-// to keys 0 .. base + m.  Keys are cut into fixed 64-key chunks at absolute
-// positions; one warp handles one (head, chunk) item for all M rows, writes a
-// partial (running max, sum of exp, unnormalised output), and the warp that
-// finishes the head's last item combines the partials in chunk order.
-// Chunk boundaries and the combine order do not depend on M, so each row's
-// output equals the single-row (M = 1) result bitwise.
+// to keys 0 .. base + m.  Keys are cut into fixed 32-key chunks at absolute
+// positions.  Each head is served by one thread-block cluster of kAttnSplit
+// CTAs; CTA r of the cluster takes chunks r, r + kAttnSplit, ... in order:
+// thread 0 brings each chunk's K and V rows (contiguous in the [H][max_seq][Dh]
+// fp32 cache) into shared memory with bulk copies, double-buffered, and the
+// CTA folds the chunk into a running softmax state per row (max, sum of exp,
+// unnormalised output).  The cluster then merges its kAttnSplit states through
+// distributed shared memory in rank order.  The chunk grid, the per-CTA chunk
+// order and the merge order depend only on key positions, never on M, so each
+// row's output equals the single-row (M = 1) result bitwise.
 #pragma once
+
+#include <cooperative_groups.h>
 
 #include "common.cuh"
 
 namespace ssd {
 
-constexpr int kAttnChunk = 64;
-constexpr int kAttnWarps = 4;
+constexpr int kAttnChunk = 32;
+constexpr int kAttnThreads = 128;
+constexpr int kAttnSplit = 8;  // CTAs per head (cluster size)
 
 struct AttnParams {
   const float* q;  // [M][q_stride], rotated queries
   int q_stride;
-  const __nv_bfloat16* k_cache;  // this layer's [H][max_seq][Dh]
-  const __nv_bfloat16* v_cache;
+  const float* k_cache;  // this layer's [H][max_seq][Dh], fp32
+  const float* v_cache;
   float* o;  // [M][o_stride]
   int o_stride;
-  float* part;          // [H][max_chunks][kMaxRows][Dh + 4]
-  unsigned* counters;   // [H]
   DevState* st;
   int pos_off;
-  int n_heads, max_seq, max_chunks;
+  int n_heads, max_seq;
   float scale;  // 1/sqrt(Dh)
 };
 
 template <int M, int DH>
-__global__ void __launch_bounds__(kAttnWarps * 32) attn_kernel(const AttnParams p) {
-  constexpr int PER = DH / 32;       // output dims per lane
-  constexpr int PS = DH + 4;         // partial record stride (floats)
-  __shared__ __align__(16) float q_s[kAttnWarps][M][DH];
+struct AttnSmem {
+  static constexpr int kKV = kAttnChunk * DH * 4;         // one K (or V) chunk
+  static constexpr int kQ = 0;                            // q rows [M][DH]
+  static constexpr int kBuf0 = kQ + M * DH * 4;           // two {K, V} buffers
+  static constexpr int kP = kBuf0 + 4 * kKV;              // probabilities [M][32]
+  static constexpr int kCs = kP + M * kAttnChunk * 4;     // chunk max / sum [2][M]
+  static constexpr int kFin = kCs + 2 * kMaxRows * 4;     // final state: mx[M], l[M], o[M][DH]
+  static constexpr int kBar = (kFin + (2 * M + M * DH) * 4 + 7) & ~7;
+  static constexpr int kTotal = kBar + 3 * 8;
+};
+
+template <int M, int DH>
+__global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThreads)
+    attn_kernel(const AttnParams p) {
+  namespace cg = cooperative_groups;
+  using S = AttnSmem<M, DH>;
+  constexpr int GROUPS = kAttnThreads / DH;  // row groups in P.V: 1 (Dh 128) or 2 (Dh 64)
+  constexpr int RPG = (M + GROUPS - 1) / GROUPS;
+  extern __shared__ __align__(128) uint8_t smem[];
+  float* Qs = reinterpret_cast<float*>(smem + S::kQ);
+  float* Ps = reinterpret_cast<float*>(smem + S::kP);
+  float* cs = reinterpret_cast<float*>(smem + S::kCs);
+  float* fin = reinterpret_cast<float*>(smem + S::kFin);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  cg::cluster_group cluster = cg::this_cluster();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int h = blockIdx.y;
+
   pdl_trigger();
+  if (tid == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_init(&bar[2], 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
   pdl_wait();
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (__ldcg(&p.st->error) & DERR_TIMEOUT) return;
-  const int base = __ldcg(&p.st->kv_len) + p.pos_off;
-  const int n_keys = base + M;  // keys 0 .. base+M-1 exist for the last row
-  if (base < 0 || n_keys > p.max_seq) {
-    if (threadIdx.x == 0 && blockIdx.x == 0) set_error(p.st, DERR_POS);
-    return;
+  int base = __ldcg(&p.st->kv_len) + p.pos_off;
+  bool bad = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
+  if (base < 0 || base + M > p.max_seq) {
+    if (tid == 0 && rank == 0 && h == 0) set_error(p.st, DERR_POS);
+    bad = true;
   }
+  const int n_keys = bad ? 0 : base + M;  // keys 0 .. base+M-1 exist for the last row
   const int n_chunks = (n_keys + kAttnChunk - 1) / kAttnChunk;
-  const int items = p.n_heads * n_chunks;
-  const int gw = blockIdx.x * kAttnWarps + warp, nw = gridDim.x * kAttnWarps;
+  const int my_chunks = n_chunks > rank ? (n_chunks - rank + kAttnSplit - 1) / kAttnSplit : 0;
 
-  for (int item = gw; item < items; item += nw) {
-    const int h = item / n_chunks, c = item - h * n_chunks;
+  auto issue = [&](int buf, int c) {
+    const int j0 = c * kAttnChunk, nk = min(kAttnChunk, n_keys - j0);
+    uint8_t* b = smem + S::kBuf0 + buf * 2 * S::kKV;
+    const uint32_t kv_bytes = static_cast<uint32_t>(nk * DH * 4);
+    mbar_arrive_expect_tx(&bar[buf], 2 * kv_bytes);
+    const size_t off = (static_cast<size_t>(h) * p.max_seq + j0) * DH;
+    bulk_load(b, p.k_cache + off, kv_bytes, &bar[buf]);
+    bulk_load(b + S::kKV, p.v_cache + off, kv_bytes, &bar[buf]);
+  };
+  if (tid == 0 && my_chunks > 0) {
+    mbar_arrive_expect_tx(&bar[2], M * DH * 4);
 #pragma unroll
     for (int m = 0; m < M; ++m)
-      for (int d = lane; d < DH; d += 32) q_s[warp][m][d] = __ldcg(p.q + m * p.q_stride + h * DH + d);
-    __syncwarp();
-
-    const int j0 = c * kAttnChunk;
-    const int jA = j0 + lane, jB = j0 + 32 + lane;
-    const bool inA = jA < n_keys, inB = jB < n_keys;
-    const __nv_bfloat16* kbase = p.k_cache + static_cast<size_t>(h) * p.max_seq * DH;
-    const uint4* kA = reinterpret_cast<const uint4*>(kbase + static_cast<size_t>(inA ? jA : 0) * DH);
-    const uint4* kB = reinterpret_cast<const uint4*>(kbase + static_cast<size_t>(inB ? jB : 0) * DH);
-
-    float sA[M], sB[M];
-#pragma unroll
-    for (int m = 0; m < M; ++m) sA[m] = sB[m] = 0.f;
-#pragma unroll 4
-    for (int d8 = 0; d8 < DH / 8; ++d8) {
-      const uint4 ka = inA ? __ldcg(kA + d8) : make_uint4(0, 0, 0, 0);
-      const uint4 kb = inB ? __ldcg(kB + d8) : make_uint4(0, 0, 0, 0);
-      const float2 a0 = bf16x2_to_float2(ka.x), a1 = bf16x2_to_float2(ka.y), a2 = bf16x2_to_float2(ka.z),
-                   a3 = bf16x2_to_float2(ka.w);
-      const float2 b0 = bf16x2_to_float2(kb.x), b1 = bf16x2_to_float2(kb.y), b2 = bf16x2_to_float2(kb.z),
-                   b3 = bf16x2_to_float2(kb.w);
-#pragma unroll
-      for (int m = 0; m < M; ++m) {
-        const float4 q0 = *reinterpret_cast<const float4*>(&q_s[warp][m][d8 * 8]);
-        const float4 q1 = *reinterpret_cast<const float4*>(&q_s[warp][m][d8 * 8 + 4]);
-        float s = sA[m];
-        s = fmaf(a0.x, q0.x, s); s = fmaf(a0.y, q0.y, s); s = fmaf(a1.x, q0.z, s); s = fmaf(a1.y, q0.w, s);
-        s = fmaf(a2.x, q1.x, s); s = fmaf(a2.y, q1.y, s); s = fmaf(a3.x, q1.z, s); s = fmaf(a3.y, q1.w, s);
-        sA[m] = s;
-        float t = sB[m];
-        t = fmaf(b0.x, q0.x, t); t = fmaf(b0.y, q0.y, t); t = fmaf(b1.x, q0.z, t); t = fmaf(b1.y, q0.w, t);
-        t = fmaf(b2.x, q1.x, t); t = fmaf(b2.y, q1.y, t); t = fmaf(b3.x, q1.z, t); t = fmaf(b3.y, q1.w, t);
-        sB[m] = t;
-      }
-    }
-
-    // softmax statistics of this chunk, per row (keys beyond the row's position masked)
-    float pA[M], pB[M], mxv[M], lv[M];
-#pragma unroll
-    for (int m = 0; m < M; ++m) {
-      const bool vA = jA <= base + m, vB = jB <= base + m;
-      const float a = vA ? sA[m] * p.scale : -INFINITY;
-      const float b = vB ? sB[m] * p.scale : -INFINITY;
-      float mx = fmaxf(a, b);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      float ea = 0.f, eb = 0.f;
-      if (mx != -INFINITY) {
-        ea = vA ? expf(a - mx) : 0.f;
-        eb = vB ? expf(b - mx) : 0.f;
-      }
-      float l = ea + eb;
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
-      pA[m] = ea;
-      pB[m] = eb;
-      mxv[m] = mx;
-      lv[m] = l;
-    }
-
-    // unnormalised P.V over the chunk's keys, lane owns dims lane*PER ..
-    float oacc[M][PER];
-#pragma unroll
-    for (int m = 0; m < M; ++m)
-#pragma unroll
-      for (int e = 0; e < PER; ++e) oacc[m][e] = 0.f;
-    const int nk = min(kAttnChunk, n_keys - j0);
-    const __nv_bfloat16* vbase = p.v_cache + (static_cast<size_t>(h) * p.max_seq + j0) * DH + lane * PER;
-#pragma unroll 4
-    for (int t = 0; t < nk; ++t) {
-      float v[PER];
-      if constexpr (PER == 4) {
-        const uint2 raw = __ldcg(reinterpret_cast<const uint2*>(vbase + static_cast<size_t>(t) * DH));
-        const float2 v0 = bf16x2_to_float2(raw.x), v1 = bf16x2_to_float2(raw.y);
-        v[0] = v0.x; v[1] = v0.y; v[2] = v1.x; v[3] = v1.y;
-      } else {
-        const uint32_t raw = __ldcg(reinterpret_cast<const unsigned int*>(vbase + static_cast<size_t>(t) * DH));
-        const float2 v0 = bf16x2_to_float2(raw);
-        v[0] = v0.x; v[1] = v0.y;
-      }
-#pragma unroll
-      for (int m = 0; m < M; ++m) {
-        const float pm = __shfl_sync(0xffffffffu, t < 32 ? pA[m] : pB[m], t & 31);
-#pragma unroll
-        for (int e = 0; e < PER; ++e) oacc[m][e] = fmaf(pm, v[e], oacc[m][e]);
-      }
-    }
-
-    float* rec = p.part + (static_cast<size_t>(h) * p.max_chunks + c) * kMaxRows * PS;
-#pragma unroll
-    for (int m = 0; m < M; ++m) {
-#pragma unroll
-      for (int e = 0; e < PER; ++e) __stcg(rec + m * PS + 4 + lane * PER + e, oacc[m][e]);
-      if (lane == 0) {
-        __stcg(rec + m * PS, mxv[m]);
-        __stcg(rec + m * PS + 1, lv[m]);
-      }
-    }
-    __threadfence();
-    __syncwarp();
-    unsigned prev = 0;
-    if (lane == 0) prev = atomicAdd(&p.counters[h], 1u);
-    prev = __shfl_sync(0xffffffffu, prev, 0);
-    if (prev == static_cast<unsigned>(n_chunks - 1)) {
-      // last item of head h: combine the chunks in order
-      __threadfence();
-      const float* hrec = p.part + static_cast<size_t>(h) * p.max_chunks * kMaxRows * PS;
-#pragma unroll 1
-      for (int m = 0; m < M; ++m) {
-        float mt = -INFINITY;
-        for (int cc = 0; cc < n_chunks; ++cc) mt = fmaxf(mt, __ldcg(hrec + (cc * kMaxRows + m) * PS));
-        float L = 0.f, O[PER];
-#pragma unroll
-        for (int e = 0; e < PER; ++e) O[e] = 0.f;
-        for (int cc = 0; cc < n_chunks; ++cc) {
-          const float* r = hrec + (cc * kMaxRows + m) * PS;
-          const float mc = __ldcg(r);
-          if (mc == -INFINITY) continue;
-          const float w = expf(mc - mt);
-          L = fmaf(w, __ldcg(r + 1), L);
-#pragma unroll
-          for (int e = 0; e < PER; ++e) O[e] = fmaf(w, __ldcg(r + 4 + lane * PER + e), O[e]);
-        }
-        const float inv = 1.0f / L;
-#pragma unroll
-        for (int e = 0; e < PER; ++e) p.o[m * p.o_stride + h * DH + lane * PER + e] = O[e] * inv;
-      }
-      if (lane == 0) p.counters[h] = 0u;
-    }
-    __syncwarp();
+      bulk_load(Qs + m * DH, p.q + static_cast<size_t>(m) * p.q_stride + h * DH, DH * 4, &bar[2]);
+    issue(0, rank);
   }
+
+  // running state: thread (d, g) owns o[m][d] for m = g, g + GROUPS, ...; row stats kept per thread
+  const int d = tid % DH, g = tid / DH;
+  float o_run[RPG], mx_run[RPG], l_run[RPG];
+#pragma unroll
+  for (int r = 0; r < RPG; ++r) {
+    o_run[r] = 0.f;
+    mx_run[r] = -INFINITY;
+    l_run[r] = 0.f;
+  }
+  bool ok = true;
+  if (my_chunks > 0 && !mbar_wait(&bar[2], 0)) ok = false;
+
+  for (int i = 0; ok && i < my_chunks; ++i) {
+    const int c = rank + i * kAttnSplit, buf = i & 1;
+    const int j0 = c * kAttnChunk, nk = min(kAttnChunk, n_keys - j0);
+    if (tid == 0 && i + 1 < my_chunks) issue(buf ^ 1, c + kAttnSplit);
+    if (!mbar_wait(&bar[buf], static_cast<uint32_t>(i >> 1) & 1u)) {
+      ok = false;
+      break;
+    }
+    const float* Ks = reinterpret_cast<const float*>(smem + S::kBuf0 + buf * 2 * S::kKV);
+    const float* Vs = Ks + kAttnChunk * DH;
+
+    // scores of the chunk: warp w, lane j -> key j, rows m = w, w+4, w+8 (columns read in a rotated order)
+    {
+      const int j = lane;
+      const bool have = j < nk;
+      for (int m = warp; m < M; m += 4) {
+        float s = 0.f;
+        if (have) {
+          const float* kr = Ks + j * DH;
+          const float* qr = Qs + m * DH;
+#pragma unroll 8
+          for (int t = 0; t < DH / 4; ++t) {
+            const int c4 = ((t + j) & (DH / 4 - 1)) * 4;
+            const float4 kv = *reinterpret_cast<const float4*>(kr + c4);
+            const float4 qv = *reinterpret_cast<const float4*>(qr + c4);
+            s = fmaf(kv.x, qv.x, s);
+            s = fmaf(kv.y, qv.y, s);
+            s = fmaf(kv.z, qv.z, s);
+            s = fmaf(kv.w, qv.w, s);
+          }
+        }
+        const bool vis = have && (j0 + j <= base + m);
+        const float v = vis ? s * p.scale : -INFINITY;
+        float mx = v;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+        const float e = (vis && mx != -INFINITY) ? expf(v - mx) : 0.f;
+        float l = e;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
+        Ps[m * kAttnChunk + j] = e;
+        if (lane == 0) {
+          cs[m] = mx;
+          cs[kMaxRows + m] = l;
+        }
+      }
+    }
+    __syncthreads();
+    // chunk P.V and merge into the running state (chunks in increasing position)
+#pragma unroll
+    for (int r = 0; r < RPG; ++r) {
+      const int m = g + r * GROUPS;
+      if (m >= M) continue;
+      float acc = 0.f;
+      for (int j = 0; j < nk; ++j) acc = fmaf(Ps[m * kAttnChunk + j], Vs[j * DH + d], acc);
+      const float cmx = cs[m];
+      if (cmx == -INFINITY) continue;  // no visible key of row m in this chunk
+      const float nmx = fmaxf(mx_run[r], cmx);
+      const float so = expf(mx_run[r] - nmx), sc = expf(cmx - nmx);
+      l_run[r] = l_run[r] * so + cs[kMaxRows + m] * sc;
+      o_run[r] = o_run[r] * so + acc * sc;
+      mx_run[r] = nmx;
+    }
+    __syncthreads();  // buffers and Ps/cs are rewritten by the next chunk
+  }
+  if (!ok) set_error(p.st, DERR_TIMEOUT);
+
+  // publish this CTA's state, then rank 0 merges the cluster's states in rank order
+#pragma unroll
+  for (int r = 0; r < RPG; ++r) {
+    const int m = g + r * GROUPS;
+    if (m >= M) continue;
+    fin[2 * M + m * DH + d] = o_run[r];
+    if (d == 0) {
+      fin[m] = mx_run[r];
+      fin[M + m] = l_run[r];
+    }
+  }
+  cluster.sync();
+  if (rank == 0 && !bad) {
+#pragma unroll
+    for (int r = 0; r < RPG; ++r) {
+      const int m = g + r * GROUPS;
+      if (m >= M) continue;
+      float mt = -INFINITY;
+      for (int q = 0; q < kAttnSplit; ++q) mt = fmaxf(mt, cluster.map_shared_rank(fin, q)[m]);
+      float L = 0.f, O = 0.f;
+      for (int q = 0; q < kAttnSplit; ++q) {
+        const float* f = cluster.map_shared_rank(fin, q);
+        const float mq = f[m];
+        if (mq == -INFINITY) continue;
+        const float w = expf(mq - mt);
+        L = fmaf(w, f[M + m], L);
+        O = fmaf(w, f[2 * M + m * DH + d], O);
+      }
+      p.o[m * p.o_stride + h * DH + d] = O / L;
+    }
+  }
+  cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
 }
 
 }  // namespace ssd

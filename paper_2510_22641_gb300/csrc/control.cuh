@@ -153,12 +153,13 @@ __global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out
 }
 
 // Greedy baseline step: emit f_0 of the single row, advance the cache by one.
-__global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cudaGraphConditionalHandle cond) {
+__global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cudaGraphConditionalHandle cond,
+                                     int has_cond) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
   if (st->done) {
-    cudaGraphSetConditional(cond, 0u);
+    if (has_cond) cudaGraphSetConditional(cond, 0u);
     return;
   }
   const int y = st->full_tok[0];
@@ -171,7 +172,7 @@ __global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cu
   st->last_n = 1;
   st->last_emitted[0] = y;
   if ((st->eos_id >= 0 && y == st->eos_id) || st->n_out >= st->max_new || st->error) st->done = 1;
-  cudaGraphSetConditional(cond, st->done ? 0u : 1u);
+  if (has_cond) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
 }
 
 __global__ void copy_out_kernel(const DevState* st, const int* out_int, int* user_out, int* user_n, int max_new) {

@@ -12,6 +12,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <map>
 #include <string>
@@ -58,10 +59,12 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 struct ssd_ctx {
   ssd_config cfg{};
   int qdim = 0, num_sms = 0, device = 0;
+  int dp = 0, qp = 0, fp = 0, ip = 0;  // activation row strides, padded to a multiple of kTileK
   // borrowed weights
   const __nv_bfloat16 *embed = nullptr, *lm_head = nullptr, *final_norm = nullptr;
   std::vector<const __nv_bfloat16*> attn_norm, ffn_norm;
   const __nv_bfloat16 *in_norm = nullptr;
+  __nv_bfloat16* gains = nullptr;  // zero-padded copies of all RMSNorm gains
   const float *resid_scale = nullptr, *in_scale = nullptr;
   std::vector<LayerSites> layers;
   Site in1, in2, head;
@@ -69,22 +72,24 @@ struct ssd_ctx {
   DevState* st = nullptr;
   int* out_int = nullptr;  // [max_seq] emitted tokens
   float *xv = nullptr, *qb = nullptr, *ob = nullptr, *hb = nullptr, *hin = nullptr, *xt = nullptr;
-  __nv_bfloat16 *kc = nullptr, *vc = nullptr;
+  float *kc = nullptr, *vc = nullptr;  // KV cache [L][H][max_seq][Dh], fp32
   size_t layer_kv = 0;  // elements per layer in kc / vc
   float2* rope = nullptr;
   float* partials = nullptr;
   unsigned* counters = nullptr;
   int n_counters = 0;
-  float* att_part = nullptr;
-  unsigned* att_cnt = nullptr;
-  int max_chunks = 0;
   __nv_bfloat16* in_vis = nullptr;
   int* in_prompt = nullptr;
   // streams and graphs
   cudaStream_t us = nullptr, cs = nullptr;
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
   bool use_pdl = true;
-  std::map<int, cudaGraphExec_t> decode_graphs, draft_graphs, verify_graphs;
+  int pf_dist = 0;  // GEMV units prefetched into L2 ahead of the shared-memory ring
+  std::map<int, cudaGraphExec_t> decode_graphs, draft_graphs, verify_graphs, step_graphs;
+  // Diagnostic: drive the decode loop from the host with one plain graph per
+  // step (ncu cannot profile kernels of graphs that hold conditional nodes).
+  bool host_loop = false;
+  int gemv_ctas = 2;  // GEMV CTAs per SM
   std::map<std::pair<int, int>, cudaGraphExec_t> prefill_graphs;
   cudaGraphExec_t greedy_graph = nullptr;
   std::map<int, int64_t> decode_body_launches;
@@ -165,32 +170,36 @@ static ssd_status encode_map(ssd_ctx* c, CUtensorMap* m, const void* base, uint6
   return SSD_OK;
 }
 
-// Site over 1..3 matrices [rows_each][K] stacked along N, 128-row tiles.
-static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nmats, int rows_each, int K) {
-  for (int i = 0; i < nmats; ++i) CKS(encode_map(c, &s->maps[i], mats[i], rows_each, K, kTileN));
+// Site over 1..3 matrices [rows_each][K] stacked along N.  Units are 32 rows x
+// 256 columns; with `paired`, the first two matrices (q, k) are read as two
+// 16-row halves per unit (rows i and i + head_dim/2 of a head).
+static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nmats, int rows_each, int K,
+                            bool paired) {
+  for (int i = 0; i < nmats; ++i)
+    CKS(encode_map(c, &s->maps[i], mats[i], rows_each, K, (paired && i < 2) ? kHalfN : kTileN));
   for (int i = nmats; i < 3; ++i) s->maps[i] = s->maps[0];
   s->N = rows_each * nmats;
   s->K = K;
   s->seg_rows = rows_each;
   s->n_rt = (s->N + kTileN - 1) / kTileN;
-  s->n_kt = K / kTileK;
+  s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
-  s->grid = s->units < c->num_sms ? s->units : c->num_sms;
+  s->grid = s->units < c->num_sms * c->gemv_ctas ? s->units : c->num_sms * c->gemv_ctas;
   return SSD_OK;
 }
 
-// gate/up pair: each unit holds 64 gate rows and the same 64 up rows.
+// gate/up pair: each unit holds 16 gate rows and the same 16 up rows.
 static ssd_status make_pair_site(ssd_ctx* c, Site* s, const void* gate, const void* up, int rows, int K) {
-  CKS(encode_map(c, &s->maps[0], gate, rows, K, kTileN / 2));
-  CKS(encode_map(c, &s->maps[1], up, rows, K, kTileN / 2));
+  CKS(encode_map(c, &s->maps[0], gate, rows, K, kHalfN));
+  CKS(encode_map(c, &s->maps[1], up, rows, K, kHalfN));
   s->maps[2] = s->maps[0];
   s->N = rows;
   s->K = K;
   s->seg_rows = rows;
-  s->n_rt = rows / (kTileN / 2);
-  s->n_kt = K / kTileK;
+  s->n_rt = (rows + kHalfN - 1) / kHalfN;
+  s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
-  s->grid = s->units < c->num_sms ? s->units : c->num_sms;
+  s->grid = s->units < c->num_sms * c->gemv_ctas ? s->units : c->num_sms * c->gemv_ctas;
   return SSD_OK;
 }
 
@@ -205,6 +214,7 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   p.counters = c->counters;
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
+  p.pf_dist = c->pf_dist;
   cudaError_t r;
   ++c->launch_counter;
   switch (e) {
@@ -220,26 +230,46 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
 
 template <int M>
 static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a) {
+  const dim3 grid(kAttnSplit, c->cfg.n_heads);
   if (c->cfg.head_dim == 128)
-    return launch_k(c, attn_kernel<M, 128>, dim3(c->num_sms), dim3(kAttnWarps * 32), 0, a);
-  return launch_k(c, attn_kernel<M, 64>, dim3(c->num_sms), dim3(kAttnWarps * 32), 0, a);
+    return launch_k(c, attn_kernel<M, 128>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
+  return launch_k(c, attn_kernel<M, 64>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
+}
+
+template <int M>
+static cudaError_t attn_attr_m() {
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<M, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       AttnSmem<M, 128>::kTotal);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_kernel<M, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              AttnSmem<M, 64>::kTotal);
+}
+
+static cudaError_t attn_attrs() {
+  cudaError_t e;
+  if ((e = attn_attr_m<1>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<2>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<3>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<4>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<5>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<6>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<7>()) != cudaSuccess) return e;
+  if ((e = attn_attr_m<8>()) != cudaSuccess) return e;
+  return attn_attr_m<9>();
 }
 
 static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off) {
   AttnParams a{};
   a.q = c->qb;
-  a.q_stride = c->qdim;
+  a.q_stride = c->qp;
   a.k_cache = c->kc + l * c->layer_kv;
   a.v_cache = c->vc + l * c->layer_kv;
   a.o = c->ob;
-  a.o_stride = c->qdim;
-  a.part = c->att_part;
-  a.counters = c->att_cnt;
+  a.o_stride = c->qp;
   a.st = c->st;
   a.pos_off = pos_off;
   a.n_heads = c->cfg.n_heads;
   a.max_seq = c->cfg.max_seq;
-  a.max_chunks = c->max_chunks;
   a.scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
   cudaError_t r;
   switch (M) {
@@ -261,7 +291,7 @@ static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off) {
 // One decoder layer x_{l+1} = x_l + f_l(x_l) on rows row0 .. row0+M-1 of xv at
 // positions kv_len + pos_off + m.
 static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off) {
-  const int d = c->cfg.d_model;
+  const int d = c->dp;
   float* x = c->xv + static_cast<size_t>(row0) * d;
   GemvParams p{};
   p.x = x;
@@ -269,7 +299,7 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   p.gain = c->attn_norm[l];
   p.pos_off = pos_off;
   p.q_out = c->qb;
-  p.q_stride = c->qdim;
+  p.q_stride = c->qp;
   p.k_cache = c->kc + l * c->layer_kv;
   p.v_cache = c->vc + l * c->layer_kv;
   p.head_dim = c->cfg.head_dim;
@@ -279,7 +309,7 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   CKS(attention(c, l, M, pos_off));
   p = GemvParams{};
   p.x = c->ob;
-  p.x_stride = c->qdim;
+  p.x_stride = c->qp;
   p.base = x;
   p.base_stride = d;
   p.dst = x;
@@ -291,11 +321,11 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   p.x_stride = d;
   p.gain = c->ffn_norm[l];
   p.h_out = c->hb;
-  p.h_stride = c->cfg.d_ff;
+  p.h_stride = c->fp;
   CKS(gemv(c, Epi::GATE_SILU, M, c->layers[l].gateup, p));
   p = GemvParams{};
   p.x = c->hb;
-  p.x_stride = c->cfg.d_ff;
+  p.x_stride = c->fp;
   p.base = x;
   p.base_stride = d;
   p.dst = x;
@@ -309,7 +339,7 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
 static ssd_status enqueue_head(ssd_ctx* c, const float* x, int M, int pos_off, int* tok_dst, bool capture) {
   GemvParams p{};
   p.x = x;
-  p.x_stride = c->cfg.d_model;
+  p.x_stride = c->dp;
   p.gain = c->final_norm;
   p.pos_off = pos_off;
   p.tok_dst = tok_dst;
@@ -324,12 +354,12 @@ static int* st_field(ssd_ctx* c, size_t off) {
 
 // Drafting stage: gamma tokens from layers 0..k-1, the imitation network and g.
 static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
-  const int d = c->cfg.d_model;
+  const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   for (int j = 0; j < gamma; ++j) {
     float* xj = c->xv + static_cast<size_t>(j) * d;
-    CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + j), xj, d, d,
-                c->cfg.vocab, c->st));
+    CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + j), xj, d,
+                c->cfg.d_model, c->cfg.vocab, c->st));
     for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, j, 1, j));
     const float* hx = xj;
     if (c->cfg.in_kind == SSD_IN_MLP2) {
@@ -338,11 +368,11 @@ static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
       p.x_stride = d;
       p.gain = c->in_norm;
       p.h_out = c->hin;
-      p.h_stride = c->cfg.in_hidden;
+      p.h_stride = c->ip;
       CKS(gemv(c, Epi::SILU, 1, c->in1, p));
       p = GemvParams{};
       p.x = c->hin;
-      p.x_stride = c->cfg.in_hidden;
+      p.x_stride = c->ip;
       p.base = xj;
       p.base_stride = d;
       p.dst = c->xt;
@@ -360,11 +390,11 @@ static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
 // 0..gamma-1 hold x_k from the draft), all gamma+1 rows through layers k..L-1,
 // g + argmax per row, then the acceptance kernel.
 static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHandle cond, int has_cond) {
-  const int d = c->cfg.d_model;
+  const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
-              c->xv + static_cast<size_t>(gamma) * d, d, d, c->cfg.vocab, c->st));
+              c->xv + static_cast<size_t>(gamma) * d, d, c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, gamma, 1, gamma));
   for (int l = c->cfg.draft_exit_k; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, gamma + 1, 0));
   CKS(enqueue_head(c, c->xv, gamma + 1, 0, full_tok, true));
@@ -373,29 +403,28 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
   return SSD_OK;
 }
 
-static ssd_status enqueue_greedy_step(ssd_ctx* c, cudaGraphConditionalHandle cond) {
+static ssd_status enqueue_greedy_step(ssd_ctx* c, cudaGraphConditionalHandle cond, int has_cond) {
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
-  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv,
-              c->cfg.d_model, c->cfg.d_model, c->cfg.vocab, c->st));
+  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv, c->dp,
+              c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
   CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
-  CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond));
+  CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond, has_cond));
   return SSD_OK;
 }
 
 static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
-  const int d = c->cfg.d_model, P = n_vis + n_prompt;
+  const int d = c->dp, P = n_vis + n_prompt;
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
-  CK(cudaMemsetAsync(c->att_cnt, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
   CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
   int r0 = 0;
   for (; r0 < P; r0 += kPrefillChunk) {
     const int Mc = P - r0 < kPrefillChunk ? P - r0 : kPrefillChunk;
     CK(launch_k(c, prefill_rows_kernel, dim3(Mc), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
-                static_cast<const int*>(c->in_prompt), n_vis, r0, c->embed, c->cfg.vocab, c->xv, d, d, c->st));
+                static_cast<const int*>(c->in_prompt), n_vis, r0, c->embed, c->cfg.vocab, c->xv, d, c->cfg.d_model, c->st));
     for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, Mc, r0));
   }
   r0 -= kPrefillChunk;
@@ -461,7 +490,7 @@ static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec,
     if (s == SSD_OK) {
       const int64_t l0 = c->launch_counter;
       ssd_status inner = gamma > 0 ? enqueue_draft(c, gamma) : SSD_OK;
-      if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify(c, gamma, cond, 1) : enqueue_greedy_step(c, cond);
+      if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify(c, gamma, cond, 1) : enqueue_greedy_step(c, cond, 1);
       *body_launches = c->launch_counter - l0;
       s = end_capture(c, body, inner);
     }
@@ -498,11 +527,19 @@ static ssd_status build_plain_graph(ssd_ctx* c, EnqueueFn fn, int a0, int a1, cu
 static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) { return enqueue_prefill(c, a, b); }
 static ssd_status enq_draft_fn(ssd_ctx* c, int g, int) { return enqueue_draft(c, g); }
 static ssd_status enq_verify_fn(ssd_ctx* c, int g, int) { return enqueue_verify(c, g, 0, 0); }
+// One decode step without a conditional node (host-driven loop, used for profiling).
+static ssd_status enq_step_fn(ssd_ctx* c, int g, int) {
+  if (g == 0) return enqueue_greedy_step(c, 0, 0);
+  CKS(enqueue_draft(c, g));
+  return enqueue_verify(c, g, 0, 0);
+}
 
 static void drop_graphs(ssd_ctx* c) {
   for (auto& kv : c->decode_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->draft_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->verify_graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->step_graphs) cudaGraphExecDestroy(kv.second);
+  c->step_graphs.clear();
   for (auto& kv : c->prefill_graphs) cudaGraphExecDestroy(kv.second);
   if (c->greedy_graph) cudaGraphExecDestroy(c->greedy_graph);
   c->decode_graphs.clear();
@@ -569,8 +606,8 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (!c) return SSD_OK;
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
-  void* bufs[] = {c->st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope,
-                  c->partials, c->counters, c->att_part, c->att_cnt, c->in_vis, c->in_prompt};
+  void* bufs[] = {c->st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
+                  c->partials, c->counters, c->in_vis, c->in_prompt};
   for (void* b : bufs)
     if (b) cudaFree(b);
   if (c->ev_in) cudaEventDestroy(c->ev_in);
@@ -586,11 +623,12 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     return fail(c, SSD_ERR_INVALID_ARG, "bad model shape");
   if (k.head_dim != 64 && k.head_dim != 128) return fail(c, SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
   const int qdim = k.n_heads * k.head_dim;
-  if (k.d_model % kTileK || k.d_ff % kTileK || qdim % kTileN)
+  constexpr int kAlign = 64;  // row strides stay 128-byte multiples for TMA
+  if (k.d_model % kAlign || k.d_ff % kAlign || qdim % 128)
     return fail(c, SSD_ERR_INVALID_ARG, "d_model, d_ff must be multiples of 64 and n_heads*head_dim of 128");
   if (k.draft_exit_k < 1 || k.draft_exit_k > k.n_layers) return fail(c, SSD_ERR_INVALID_ARG, "draft_exit_k");
   if (k.in_kind != SSD_IN_IDENTITY && k.in_kind != SSD_IN_MLP2) return fail(c, SSD_ERR_INVALID_ARG, "in_kind");
-  if (k.in_kind == SSD_IN_MLP2 && (k.in_hidden < 64 || k.in_hidden % kTileK))
+  if (k.in_kind == SSD_IN_MLP2 && (k.in_hidden < 64 || k.in_hidden % kAlign))
     return fail(c, SSD_ERR_INVALID_ARG, "in_hidden must be a positive multiple of 64");
   if (k.gamma_max < 1 || k.gamma_max > SSD_MAX_GAMMA || k.gamma_max + 1 > kMaxVerifyRows)
     return fail(c, SSD_ERR_INVALID_ARG, "gamma_max must be in [1, %d]", SSD_MAX_GAMMA);
@@ -611,6 +649,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (prop.major != 10) return fail(c, SSD_ERR_UNSUPPORTED, "needs a Blackwell sm_103 device, got sm_%d%d",
                                     prop.major, prop.minor);
   c->num_sms = prop.multiProcessorCount;
+  if (const char* e = getenv("SSD_GEMV_PREFETCH")) c->pf_dist = atoi(e) < 0 ? 0 : atoi(e);
+  if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
+  if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) == 2 ? 2 : 1;
   if (!g_encode) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;
@@ -623,9 +664,15 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_silu());
   CK(gemv_attrs_resid());
   CK(gemv_attrs_head());
+  CK(attn_attrs());
 
   c->cfg = k;
   c->qdim = qdim;
+  auto pad = [](int v) { return (v + kTileK - 1) / kTileK * kTileK; };
+  c->dp = pad(k.d_model);
+  c->qp = pad(qdim);
+  c->fp = pad(k.d_ff);
+  c->ip = pad(k.in_hidden > 0 ? k.in_hidden : 64);
   c->embed = static_cast<const __nv_bfloat16*>(w->embed);
   c->lm_head = static_cast<const __nv_bfloat16*>(w->lm_head);
   c->final_norm = static_cast<const __nv_bfloat16*>(w->final_norm);
@@ -637,43 +684,57 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     c->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
     c->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
     const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
-    CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model));
-    CKS(make_site(c, &c->layers[l].o, &w->wo[l], 1, k.d_model, qdim));
+    CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model, true));
+    CKS(make_site(c, &c->layers[l].o, &w->wo[l], 1, k.d_model, qdim, false));
     CKS(make_pair_site(c, &c->layers[l].gateup, w->w_gate[l], w->w_up[l], k.d_ff, k.d_model));
-    CKS(make_site(c, &c->layers[l].down, &w->w_down[l], 1, k.d_model, k.d_ff));
+    CKS(make_site(c, &c->layers[l].down, &w->w_down[l], 1, k.d_model, k.d_ff, false));
   }
   if (k.in_kind == SSD_IN_MLP2) {
-    CKS(make_site(c, &c->in1, &w->in_w1, 1, k.in_hidden, k.d_model));
-    CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden));
+    CKS(make_site(c, &c->in1, &w->in_w1, 1, k.in_hidden, k.d_model, false));
+    CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden, false));
   }
-  CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model));
+  CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model, false));
 
   // owned memory
   const int R = kMaxRows;
   const size_t d = k.d_model;
   CKS(alloc(c, reinterpret_cast<void**>(&c->st), sizeof(DevState)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->out_int), sizeof(int) * k.max_seq));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->xv), sizeof(float) * R * d));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->xt), sizeof(float) * R * d));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->qb), sizeof(float) * R * qdim));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->ob), sizeof(float) * R * qdim));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->hb), sizeof(float) * R * k.d_ff));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->hin), sizeof(float) * R * (k.in_hidden > 0 ? k.in_hidden : 64)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->xv), sizeof(float) * R * c->dp));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->xt), sizeof(float) * R * c->dp));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->qb), sizeof(float) * R * c->qp));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->ob), sizeof(float) * R * c->qp));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->hb), sizeof(float) * R * c->fp));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->hin), sizeof(float) * R * c->ip));
+  // RMSNorm gains: zero-padded copies, so 256-column slices never read past a gain vector
+  const int n_gains = 2 * k.n_layers + 2;
+  CKS(alloc(c, reinterpret_cast<void**>(&c->gains), sizeof(__nv_bfloat16) * n_gains * c->dp));
+  auto copy_gain = [&](int slot, const void* src) -> const __nv_bfloat16* {
+    __nv_bfloat16* dst = c->gains + static_cast<size_t>(slot) * c->dp;
+    if (src && cudaMemcpy(dst, src, sizeof(__nv_bfloat16) * k.d_model, cudaMemcpyDeviceToDevice) != cudaSuccess)
+      return nullptr;
+    return dst;
+  };
+  for (int l = 0; l < k.n_layers; ++l) {
+    c->attn_norm[l] = copy_gain(2 * l, w->attn_norm[l]);
+    c->ffn_norm[l] = copy_gain(2 * l + 1, w->ffn_norm[l]);
+    if (!c->attn_norm[l] || !c->ffn_norm[l]) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
+  }
+  c->final_norm = copy_gain(2 * k.n_layers, w->final_norm);
+  c->in_norm = k.in_kind == SSD_IN_MLP2 ? copy_gain(2 * k.n_layers + 1, w->in_norm) : nullptr;
+  if (!c->final_norm || (k.in_kind == SSD_IN_MLP2 && !c->in_norm))
+    return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
   c->layer_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
-  CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(__nv_bfloat16) * c->layer_kv * k.n_layers));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(__nv_bfloat16) * c->layer_kv * k.n_layers));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(float) * c->layer_kv * k.n_layers));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(float) * c->layer_kv * k.n_layers));
   CKS(alloc(c, reinterpret_cast<void**>(&c->rope), sizeof(float2) * k.max_seq * (k.head_dim / 2)));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->num_sms * R * kTileN));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->gemv_ctas * c->num_sms * R * kTileN));
   int max_rt = 1;
   for (const Site* s : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->head,
                         &c->in1, &c->in2})
     max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
-  c->max_chunks = (k.max_seq + kAttnChunk - 1) / kAttnChunk;
-  CKS(alloc(c, reinterpret_cast<void**>(&c->att_part),
-            sizeof(float) * k.n_heads * c->max_chunks * R * (k.head_dim + 4)));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->att_cnt), sizeof(unsigned) * k.n_heads));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * k.max_seq));
   CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
@@ -793,6 +854,31 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
     return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 = %d > max_seq = %d",
                 c->prompt_len + max_new + gamma + 1, c->cfg.max_seq);
   cudaGraphExec_t ge;
+  if (c->host_loop) {
+    auto it = c->step_graphs.find(gamma);
+    if (it == c->step_graphs.end()) {
+      int64_t nb = 0;
+      CKS(build_plain_graph(c, enq_step_fn, gamma, 0, &ge, &nb));
+      it = c->step_graphs.emplace(gamma, ge).first;
+      if (gamma > 0) c->decode_body_launches[gamma] = nb; else c->greedy_body_launches = nb;
+    }
+    decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
+    CK(cudaGetLastError());
+    int done = 0;
+    for (int it2 = 0; it2 < max_new && !done; ++it2) {
+      CK(cudaGraphLaunch(it->second, c->cs));
+      CK(cudaMemcpyAsync(&done, reinterpret_cast<char*>(c->st) + offsetof(DevState, done), sizeof(int),
+                         cudaMemcpyDeviceToHost, c->cs));
+      CK(cudaStreamSynchronize(c->cs));
+    }
+    if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+    CK(cudaGetLastError());
+    c->last_decode_kind = gamma > 0 ? 1 : 2;
+    c->last_gamma = gamma;
+    c->drafted_gamma = 0;
+    c->kv_upper = c->prompt_len + max_new + gamma + 1;
+    return SSD_OK;
+  }
   if (gamma > 0) {
     auto it = c->decode_graphs.find(gamma);
     if (it == c->decode_graphs.end()) {
@@ -935,7 +1021,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     return fail(c, SSD_ERR_INVALID_ARG, "which / layer");
   if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))
     return fail(c, SSD_ERR_INVALID_ARG, "imitation projections need SSD_IN_MLP2 and rows == 1");
-  const int d = c->cfg.d_model;
+  const int d = c->dp;
   const Site* site = nullptr;
   Epi e = Epi::RESID;
   GemvParams p{};
@@ -947,7 +1033,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       e = Epi::QKV;
       p.gain = c->attn_norm[layer];
       p.q_out = c->qb;
-      p.q_stride = c->qdim;
+      p.q_stride = c->qp;
       p.k_cache = c->kc + layer * c->layer_kv;
       p.v_cache = c->vc + layer * c->layer_kv;
       p.head_dim = c->cfg.head_dim;
@@ -958,7 +1044,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     case 3:
       site = which == 1 ? &c->layers[layer].o : &c->layers[layer].down;
       p.x = which == 1 ? c->ob : c->hb;
-      p.x_stride = which == 1 ? c->qdim : c->cfg.d_ff;
+      p.x_stride = which == 1 ? c->qp : c->fp;
       p.base = c->xt;
       p.base_stride = d;
       p.dst = c->xt;
@@ -970,7 +1056,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       e = Epi::GATE_SILU;
       p.gain = c->ffn_norm[layer];
       p.h_out = c->hb;
-      p.h_stride = c->cfg.d_ff;
+      p.h_stride = c->fp;
       break;
     case 4:
       site = &c->head;
@@ -983,12 +1069,12 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       e = Epi::SILU;
       p.gain = c->in_norm;
       p.h_out = c->hin;
-      p.h_stride = c->cfg.in_hidden;
+      p.h_stride = c->ip;
       break;
     default:
       site = &c->in2;
       p.x = c->hin;
-      p.x_stride = c->cfg.in_hidden;
+      p.x_stride = c->ip;
       p.base = c->xt;
       p.base_stride = d;
       p.dst = c->xt;

@@ -30,7 +30,7 @@ class _DeviceArray:
 
 
 def _device_view(ptr: int, shape) -> torch.Tensor:
-    return torch.as_tensor(_DeviceArray(ptr, shape, "<i2"), device="cuda").view(torch.bfloat16)
+    return torch.as_tensor(_DeviceArray(ptr, shape, "<f4"), device="cuda")
 
 
 class SSDModel:
@@ -139,7 +139,7 @@ class SSDModel:
         self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
 
     def kv(self):
-        """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (bf16) of the library's cache."""
+        """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (fp32) of the library's cache."""
         k, v, n = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_int()
         self._call("ssd_get_kv", ctypes.byref(k), ctypes.byref(v), ctypes.byref(n))
         c = self.cfg

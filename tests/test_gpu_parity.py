@@ -112,8 +112,8 @@ def test_kv_cache_after_rollback_equals_greedy_cache(tiny_model):
     gpu_decode(model, w, 0, capture=False)
     k2, v2, n2 = model.kv()
     assert n1 == n2 == w.prompt_len + w.max_new - 1
-    assert torch.equal(k1.view(torch.int16), k2[:, :, :n2].view(torch.int16))
-    assert torch.equal(v1.view(torch.int16), v2[:, :, :n2].view(torch.int16))
+    assert torch.equal(k1.view(torch.int32), k2[:, :, :n2].view(torch.int32))
+    assert torch.equal(v1.view(torch.int32), v2[:, :, :n2].view(torch.int32))
 
 
 def test_prefill_kv_matches_oracle(tiny_bits):
@@ -130,9 +130,9 @@ def test_prefill_kv_matches_oracle(tiny_bits):
     for got, ref in ((k, cache.k), (v, cache.v)):
         g = got[:, :, :P].float().cpu().numpy()
         r = ref[:, :, :P]
-        # bf16 storage (relative 2^-9) plus drift from bf16 K/V in earlier layers
+        # fp32 cache; the remaining difference is fp32 arithmetic on bf16 weights vs fp64
         rms = float(np.sqrt(np.mean(r * r)))
-        np.testing.assert_allclose(g, r, rtol=2e-2, atol=2e-2 * rms)
+        np.testing.assert_allclose(g, r, rtol=1e-3, atol=1e-3 * rms)
     model.close()
 
 
