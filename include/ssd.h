@@ -210,6 +210,16 @@ SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v
  * ssd_prefill performed (from the device step counter).  sync. */
 SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches, int64_t* decode_launches);
 
+/* The LM head alone (Sec. "SSD Setup for VLMs": o = g(x), greedy argmax):
+ * logits = W_lm RMSNorm_f(x) and the argmax of each row (lowest index on ties)
+ * for `rows` caller rows, with this ctx's lm_head / final_norm weights and
+ * workspace.  Does not touch the decode state.
+ *   x:      device fp32 [rows][d_model], 1 <= rows <= 9
+ *   tok:    device int32 [rows]
+ *   logits: device fp32 [rows][vocab], or NULL
+ * async. */
+SSD_API ssd_status ssd_lm_head(ssd_ctx* ctx, const float* x, int rows, int32_t* tok, float* logits);
+
 /* Diagnostic for timing one kernel alone: enqueue `reps` back-to-back launches
  * of one weight-streaming projection (the GEMV kernel with its fused
  * epilogue) over `rows` activation rows, with whatever activations the ctx

@@ -70,6 +70,7 @@ struct ssd_ctx {
   Site in1, in2, head;
   // owned device memory
   DevState* st = nullptr;
+  DevState* op_st = nullptr;  // state of standalone op calls (ssd_lm_head)
   int* out_int = nullptr;  // [max_seq] emitted tokens
   float *xv = nullptr, *qb = nullptr, *ob = nullptr, *hb = nullptr, *hin = nullptr, *xt = nullptr;
   float *kc = nullptr, *vc = nullptr;  // KV cache [L][H][max_seq][Dh], fp32
@@ -606,7 +607,7 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (!c) return SSD_OK;
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
-  void* bufs[] = {c->st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
+  void* bufs[] = {c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
                   c->partials, c->counters, c->in_vis, c->in_prompt};
   for (void* b : bufs)
     if (b) cudaFree(b);
@@ -699,6 +700,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   const int R = kMaxRows;
   const size_t d = k.d_model;
   CKS(alloc(c, reinterpret_cast<void**>(&c->st), sizeof(DevState)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->op_st), sizeof(DevState)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->out_int), sizeof(int) * k.max_seq));
   CKS(alloc(c, reinterpret_cast<void**>(&c->xv), sizeof(float) * R * c->dp));
   CKS(alloc(c, reinterpret_cast<void**>(&c->xt), sizeof(float) * R * c->dp));
@@ -1011,6 +1013,44 @@ ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t*
     // setup + loop_begin + steps x body + copy-out
     *decode_launches = c->last_decode_kind ? 2 + static_cast<int64_t>(h.steps) * body + 1 : 0;
   }
+  return SSD_OK;
+}
+
+ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float* logits) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (!x || !tok || rows < 1 || rows > kMaxVerifyRows) return fail(c, SSD_ERR_INVALID_ARG, "x / tok / rows");
+  CKS(enter(c));
+  // rows go through the ctx's zero-padded staging buffer (256-column slices never leave a row)
+  CK(cudaMemcpy2DAsync(c->xt, sizeof(float) * c->dp, x, sizeof(float) * c->cfg.d_model,
+                       sizeof(float) * c->cfg.d_model, rows, cudaMemcpyDeviceToDevice, c->cs));
+  // op state: kv_len = 0, prompt_len = 1 -> logits row m lands in row m of the capture buffer
+  DevState zero{};
+  zero.prompt_len = 1;
+  CK(cudaMemcpyAsync(c->op_st, &zero, sizeof(DevState), cudaMemcpyHostToDevice, c->cs));
+  GemvParams p{};
+  p.x = c->xt;
+  p.x_stride = c->dp;
+  p.gain = c->final_norm;
+  p.pos_off = 0;
+  p.tok_dst = tok;
+  p.logits = logits;
+  p.logits_rows = logits ? rows : 0;
+  p.K = c->head.K;
+  p.n_kt = c->head.n_kt;
+  p.n_rt = c->head.n_rt;
+  p.units = c->head.units;
+  p.N = c->head.N;
+  p.seg_rows = c->head.seg_rows;
+  p.partials = c->partials;
+  p.counters = c->counters;
+  p.st = c->op_st;
+  p.eps = c->cfg.rms_eps;
+  p.pf_dist = c->pf_dist;
+  ++c->launch_counter;
+  CK(gemv_launch_head(rows, c->head.maps, p, c->head.grid, c->cs, false));
+  CKS(leave(c));
+  // the host-side DevState must outlive the async copy
+  CK(cudaStreamSynchronize(c->cs));
   return SSD_OK;
 }
 

@@ -146,6 +146,10 @@ class SSDModel:
         shape = (c["n_layers"], c["n_heads"], c["max_seq"], c["head_dim"])
         return _device_view(k.value, shape), _device_view(v.value, shape), n.value
 
+    def lm_head(self, x: torch.Tensor, tok: torch.Tensor, logits: torch.Tensor | None = None):
+        """ssd_lm_head: argmax of W_lm RMSNorm_f(x) per row (x fp32 [rows][d_model] on the device)."""
+        self._call("ssd_lm_head", x.data_ptr(), x.shape[0], tok.data_ptr(), _ptr(logits))
+
     PROJECTIONS = {"qkv": 0, "o": 1, "gateup": 2, "down": 3, "head": 4, "in1": 5, "in2": 6}
 
     def profile_projection(self, which: str, layer: int = 0, rows: int = 1, reps: int = 1) -> int:

@@ -267,3 +267,25 @@ def test_launch_counts(tiny_model):
     body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
     assert dec == 3 + st["steps"] * body
     assert pre == 2 + ((w.prompt_len + 7) // 8) * (1 + 5 * L) + 1
+
+
+@pytest.mark.parametrize("rows", [1, 5, 9])
+def test_lm_head_op_matches_oracle(tiny_model, tiny_bits, rows):
+    """ssd_lm_head: logits of W_lm RMSNorm_f(x) within tolerance, argmax exact away from ties."""
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed")
+    m = oracle.model_from_bits(w, tiny_bits, synth.bf16_to_f64)
+    x = synth.normal_f64(11, rows, (rows, w.shape.d_model), std=3.0)
+    xt = torch.from_numpy(x.astype(np.float32)).cuda()
+    tok = torch.zeros(rows, dtype=torch.int32, device="cuda")
+    lg = torch.zeros((rows, w.shape.vocab), device="cuda")
+    model.lm_head(xt, tok, lg)
+    model.sync()
+    for r in range(rows):
+        ref = oracle.lm_head(m, x[r].astype(np.float32).astype(np.float64))
+        assert_logits_close(lg[r].cpu().numpy(), ref, f"lm_head row {r}")
+        if int(tok[r]) != int(np.argmax(ref)):
+            from tests.parity import margin
+            assert margin(ref) < 1e-2
+    # argmax of the returned logits is the returned token (lowest index on ties)
+    assert tok.cpu().tolist() == lg.argmax(dim=1).cpu().int().tolist()
