@@ -220,6 +220,26 @@ SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches
  * async. */
 SSD_API ssd_status ssd_lm_head(ssd_ctx* ctx, const float* x, int rows, int32_t* tok, float* logits);
 
+/* The same LM head + argmax as ssd_lm_head, for callers that cannot allocate
+ * device memory: code running while a stream is captured into a CUDA graph,
+ * serving loops whose device memory is owned by their own allocator, hosts
+ * that must avoid the implicit synchronisation of cudaMalloc/cudaFree.  The
+ * paper has no counterpart; this is a deployment variant.  It needs no ctx and
+ * allocates nothing: its scratch is a fixed ~1.3 MB array in device memory that
+ * every GPU loading the library holds until the process exits.
+ *   lm_head:    device bf16 [vocab][d_model];  final_norm: device bf16 [d_model]
+ *   x:          device fp32 [rows][d_model];  tok: device int32 [rows]
+ *   logits:     device fp32 [rows][vocab] or NULL;  cuda_stream: cudaStream_t
+ * Limits: 1 <= rows <= 9, vocab <= 262144, d_model a multiple of 256, 16-byte
+ * aligned pointers; SSD_ERR_INVALID_ARG otherwise.  The first call on a device
+ * (with that device current) looks up the array's device address and sets
+ * kernel attributes: make it before any stream capture.  All calls share the
+ * one array, so calls that overlap on the GPU (other streams, other threads)
+ * race and must be serialised by the caller.  async. */
+SSD_API ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const float* x, int rows,
+                                      int vocab, int d_model, float rms_eps, int32_t* tok, float* logits,
+                                      void* cuda_stream);
+
 /* Diagnostic for timing one kernel alone: enqueue `reps` back-to-back launches
  * of one weight-streaming projection (the GEMV kernel with its fused
  * epilogue) over `rows` activation rows, with whatever activations the ctx

@@ -22,7 +22,7 @@ STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_C
 
 EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode",
             "ssd_greedy_decode", "ssd_generate", "ssd_greedy_generate", "ssd_sync", "ssd_get_stats",
-            "ssd_set_logits_capture", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_profile_projection",
+            "ssd_set_logits_capture", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
             "ssd_status_string",
             "ssd_last_error")
 
@@ -85,6 +85,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_last_launch_count": [vp, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)],
         "ssd_profile_projection": [vp, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_int64)],
         "ssd_lm_head": [vp, vp, i32, vp, vp],
+        "ssd_lm_head_static": [vp, vp, vp, i32, i32, i32, ctypes.c_float, vp, vp, vp],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
