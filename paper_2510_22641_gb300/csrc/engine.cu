@@ -12,6 +12,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <algorithm>
 #include <cstdlib>
 #include <cstring>
 #include <map>
@@ -22,6 +23,7 @@
 #include "attention.cuh"
 #include "control.cuh"
 #include "gemv.cuh"
+#include "prefill_params.cuh"
 
 namespace ssd {
 cudaError_t gemv_launch_qkv(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
@@ -34,6 +36,14 @@ cudaError_t gemv_attrs_gate();
 cudaError_t gemv_attrs_silu();
 cudaError_t gemv_attrs_resid();
 cudaError_t gemv_attrs_head();
+cudaError_t prefill_attrs();
+cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
+                           cudaStream_t s, bool pdl);
+cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
+                              __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl);
+cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
+                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
+                                cudaStream_t s, bool pdl);
 }  // namespace ssd
 
 using namespace ssd;
@@ -52,6 +62,17 @@ struct LayerSites {
   Site qkv, o, gateup, down;
 };
 
+// Weights of one projection for the prefill GEMM: 128-row (or 2 x 64-row) boxes
+// of 64 columns, 128-byte swizzled.
+struct TcSite {
+  CUtensorMap maps[3];
+  int N = 0, K = 0, tiles_n = 0, seg_rows = 0;
+};
+
+struct TcLayer {
+  TcSite qkv, o, gateup, down;
+};
+
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 }  // namespace
@@ -68,6 +89,12 @@ struct ssd_ctx {
   const float *resid_scale = nullptr, *in_scale = nullptr;
   std::vector<LayerSites> layers;
   Site in1, in2, head;
+  // prefill (tcgen05) state
+  std::vector<TcLayer> tc_layers;
+  CUtensorMap a_maps[3][2];  // activation splits (hi, lo) for K = d_model, n_heads*head_dim, d_ff
+  __nv_bfloat16 *a_hi = nullptr, *a_lo = nullptr;
+  float *x_pre = nullptr, *q_pre = nullptr, *o_pre = nullptr, *h_pre = nullptr;
+  bool prefill_rows = false;  // SSD_PREFILL=rows: prefill through the decode kernels in 8-row chunks
   // owned device memory
   DevState* st = nullptr;
   DevState* op_st = nullptr;  // state of standalone op calls (ssd_lm_head)
@@ -154,6 +181,21 @@ static cudaError_t launch_k(ssd_ctx* c, Kern kern, dim3 grid, dim3 block, size_t
   cfg.numAttrs = 1;
   ++c->launch_counter;
   return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+static ssd_status encode_map_sw128(ssd_ctx* c, CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
+                                   uint32_t box_rows) {
+  if (reinterpret_cast<uintptr_t>(base) % 16 != 0)
+    return fail(c, SSD_ERR_INVALID_ARG, "pointer %p is not 16-byte aligned", base);
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kTcK), box_rows};
+  cuuint32_t es[2] = {1, 1};
+  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return fail(c, SSD_ERR_CUDA, "cuTensorMapEncodeTiled (swizzled) failed (%d)", static_cast<int>(r));
+  return SSD_OK;
 }
 
 static ssd_status encode_map(ssd_ctx* c, CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
@@ -434,6 +476,81 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   return SSD_OK;
 }
 
+// Prefill over all P rows at once: activation splits + tcgen05 GEMMs with the
+// fused epilogues, and causal attention over the prompt.
+static ssd_status tc_gemm(ssd_ctx* c, Epi e, int kidx, const TcSite& site, int P, TcParams p) {
+  p.M = P;
+  p.N = site.N;
+  p.K = site.K;
+  p.tiles_m = (P + kTcM - 1) / kTcM;
+  p.tiles_n = site.tiles_n;
+  p.k_steps = site.K / kTcK;
+  p.seg_rows = site.seg_rows;
+  p.st = c->st;
+  const int tiles = p.tiles_m * p.tiles_n;
+  ++c->launch_counter;
+  CK(tc_gemm_launch(e, c->a_maps[kidx], site.maps, p, tiles < c->num_sms ? tiles : c->num_sms, c->cs, c->use_pdl));
+  return SSD_OK;
+}
+
+static ssd_status split(ssd_ctx* c, const float* x, int x_stride, int K, const __nv_bfloat16* gain, int P) {
+  ++c->launch_counter;
+  CK(split_rows_launch(x, x_stride, K, gain, c->cfg.rms_eps, c->a_hi, c->a_lo, P, c->cs, c->use_pdl));
+  return SSD_OK;
+}
+
+static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
+  const int P = n_vis + n_prompt, dp = c->dp;
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
+  CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+              static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
+              c->st));
+  for (int l = 0; l < c->cfg.n_layers; ++l) {
+    const TcLayer& tl = c->tc_layers[l];
+    TcParams p{};
+    p.pos0 = 0;
+    p.q_out = c->q_pre;
+    p.q_stride = c->qp;
+    p.k_cache = c->kc + l * c->layer_kv;
+    p.v_cache = c->vc + l * c->layer_kv;
+    p.head_dim = c->cfg.head_dim;
+    p.max_seq = c->cfg.max_seq;
+    p.rope_cs = c->rope;
+    CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->attn_norm[l], P));
+    CKS(tc_gemm(c, Epi::QKV, 0, tl.qkv, P, p));
+    ++c->launch_counter;
+    CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, c->kc + l * c->layer_kv, c->vc + l * c->layer_kv,
+                           c->o_pre, c->qp, P, c->cfg.n_heads, c->cfg.max_seq,
+                           1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->cs, c->use_pdl));
+    CKS(split(c, c->o_pre, c->qp, c->qdim, nullptr, P));
+    p = TcParams{};
+    p.base = c->x_pre;
+    p.base_stride = dp;
+    p.dst = c->x_pre;
+    p.dst_stride = dp;
+    p.scale = c->resid_scale + l;
+    CKS(tc_gemm(c, Epi::RESID, 1, tl.o, P, p));
+    CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->ffn_norm[l], P));
+    p = TcParams{};
+    p.h_out = c->h_pre;
+    p.h_stride = c->fp;
+    CKS(tc_gemm(c, Epi::GATE_SILU, 0, tl.gateup, P, p));
+    CKS(split(c, c->h_pre, c->fp, c->cfg.d_ff, nullptr, P));
+    p = TcParams{};
+    p.base = c->x_pre;
+    p.base_stride = dp;
+    p.dst = c->x_pre;
+    p.dst_stride = dp;
+    p.scale = c->resid_scale + l;
+    CKS(tc_gemm(c, Epi::RESID, 2, tl.down, P, p));
+  }
+  CKS(enqueue_head(c, c->x_pre + static_cast<size_t>(P - 1) * dp, 1, P - 1, full_tok, true));
+  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
+  return SSD_OK;
+}
+
 // ------------------------------------------------------------------ graphs
 
 static ssd_status begin_capture(ssd_ctx* c, cudaGraph_t g) {
@@ -525,7 +642,9 @@ static ssd_status build_plain_graph(ssd_ctx* c, EnqueueFn fn, int a0, int a1, cu
   return s;
 }
 
-static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) { return enqueue_prefill(c, a, b); }
+static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) {
+  return c->prefill_rows ? enqueue_prefill(c, a, b) : enqueue_prefill_tc(c, a, b);
+}
 static ssd_status enq_draft_fn(ssd_ctx* c, int g, int) { return enqueue_draft(c, g); }
 static ssd_status enq_verify_fn(ssd_ctx* c, int g, int) { return enqueue_verify(c, g, 0, 0); }
 // One decode step without a conditional node (host-driven loop, used for profiling).
@@ -607,7 +726,7 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (!c) return SSD_OK;
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
-  void* bufs[] = {c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
+  void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
                   c->partials, c->counters, c->in_vis, c->in_prompt};
   for (void* b : bufs)
     if (b) cudaFree(b);
@@ -653,6 +772,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (const char* e = getenv("SSD_GEMV_PREFETCH")) c->pf_dist = atoi(e) < 0 ? 0 : atoi(e);
   if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
   if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) == 2 ? 2 : 1;
+  if (const char* e = getenv("SSD_PREFILL")) c->prefill_rows = strcmp(e, "rows") == 0;
   if (!g_encode) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;
@@ -666,6 +786,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_resid());
   CK(gemv_attrs_head());
   CK(attn_attrs());
+  CK(prefill_attrs());
 
   c->cfg = k;
   c->qdim = qdim;
@@ -695,6 +816,35 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden, false));
   }
   CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model, false));
+  c->tc_layers.resize(k.n_layers);
+  for (int l = 0; l < k.n_layers; ++l) {
+    TcLayer& t = c->tc_layers[l];
+    const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
+    for (int i = 0; i < 3; ++i) CKS(encode_map_sw128(c, &t.qkv.maps[i], qkv[i], qdim, k.d_model, kTcN));
+    t.qkv.N = 3 * qdim;
+    t.qkv.K = k.d_model;
+    t.qkv.seg_rows = qdim;
+    t.qkv.tiles_n = 3 * qdim / kTcN;
+    CKS(encode_map_sw128(c, &t.o.maps[0], w->wo[l], k.d_model, qdim, kTcN));
+    t.o.maps[1] = t.o.maps[2] = t.o.maps[0];
+    t.o.N = k.d_model;
+    t.o.K = qdim;
+    t.o.seg_rows = k.d_model;
+    t.o.tiles_n = (k.d_model + kTcN - 1) / kTcN;
+    CKS(encode_map_sw128(c, &t.gateup.maps[0], w->w_gate[l], k.d_ff, k.d_model, kTcN / 2));
+    CKS(encode_map_sw128(c, &t.gateup.maps[1], w->w_up[l], k.d_ff, k.d_model, kTcN / 2));
+    t.gateup.maps[2] = t.gateup.maps[0];
+    t.gateup.N = k.d_ff;
+    t.gateup.K = k.d_model;
+    t.gateup.seg_rows = k.d_ff;
+    t.gateup.tiles_n = (k.d_ff + kTcN / 2 - 1) / (kTcN / 2);
+    CKS(encode_map_sw128(c, &t.down.maps[0], w->w_down[l], k.d_model, k.d_ff, kTcN));
+    t.down.maps[1] = t.down.maps[2] = t.down.maps[0];
+    t.down.N = k.d_model;
+    t.down.K = k.d_ff;
+    t.down.seg_rows = k.d_model;
+    t.down.tiles_n = (k.d_model + kTcN - 1) / kTcN;
+  }
 
   // owned memory
   const int R = kMaxRows;
@@ -738,6 +888,22 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
+  {
+    const size_t Pm = k.max_seq;
+    const size_t kmax = std::max(std::max(static_cast<size_t>(k.d_model), static_cast<size_t>(qdim)),
+                                 static_cast<size_t>(k.d_ff));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->a_hi), sizeof(__nv_bfloat16) * Pm * kmax));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->a_lo), sizeof(__nv_bfloat16) * Pm * kmax));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->x_pre), sizeof(float) * Pm * c->dp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->q_pre), sizeof(float) * Pm * c->qp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->o_pre), sizeof(float) * Pm * c->qp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->h_pre), sizeof(float) * Pm * c->fp));
+    const int ks[3] = {k.d_model, qdim, k.d_ff};
+    for (int i = 0; i < 3; ++i) {
+      CKS(encode_map_sw128(c, &c->a_maps[i][0], c->a_hi, Pm, ks[i], kTcM));
+      CKS(encode_map_sw128(c, &c->a_maps[i][1], c->a_lo, Pm, ks[i], kTcM));
+    }
+  }
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * k.max_seq));
   CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->ev_in, cudaEventDisableTiming));

@@ -1,0 +1,69 @@
+// Launchers of the prefill kernels (tcgen05 GEMM, activation split, causal attention).
+#include "prefill.cuh"
+
+namespace ssd {
+
+template <typename Kern, typename... Args>
+static cudaError_t launch_pdl(Kern kern, dim3 grid, dim3 block, size_t smem, cudaStream_t s, bool pdl,
+                              Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+cudaError_t prefill_attrs() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
+    return e;
+  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::GATE_SILU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                kTcSmem)))
+    return e;
+  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
+    return e;
+  if ((e = cudaFuncSetAttribute(prefill_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                PaSmem<128>::kTotal)))
+    return e;
+  return cudaFuncSetAttribute(prefill_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              PaSmem<64>::kTotal);
+}
+
+cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
+                           cudaStream_t s, bool pdl) {
+  const dim3 g(grid), blk(kTcThreads);
+  switch (e) {
+    case Epi::QKV:
+      return launch_pdl(tc_gemm_kernel<Epi::QKV>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+    case Epi::GATE_SILU:
+      return launch_pdl(tc_gemm_kernel<Epi::GATE_SILU>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+    case Epi::RESID:
+      return launch_pdl(tc_gemm_kernel<Epi::RESID>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+    default:
+      return cudaErrorInvalidValue;
+  }
+}
+
+cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
+                              __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl) {
+  return launch_pdl(split_rows_kernel, dim3(rows), dim3(256), 0, s, pdl, x, x_stride, K, gain, eps, hi, lo);
+}
+
+cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
+                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
+                                cudaStream_t s, bool pdl) {
+  const dim3 grid((P + kPaQ - 1) / kPaQ, n_heads);
+  if (head_dim == 128)
+    return launch_pdl(prefill_attn_kernel<128>, grid, dim3(256), PaSmem<128>::kTotal, s, pdl, q, q_stride, kc, vc,
+                      o, o_stride, P, max_seq, scale);
+  return launch_pdl(prefill_attn_kernel<64>, grid, dim3(256), PaSmem<64>::kTotal, s, pdl, q, q_stride, kc, vc, o,
+                    o_stride, P, max_seq, scale);
+}
+
+}  // namespace ssd

@@ -1,0 +1,473 @@
+// Prefill kernels: the decoder's projections over all P prompt rows as a dense
+// tensor-core contraction (tcgen05 / TMEM), and causal attention over the rows.
+//
+// Prefill (Sec. "SSD Setup for VLMs": z and the prompt enter the decoder) runs
+// every layer at M = P rows (P = 640 for the LLaVA-1.5 shape), which makes the
+// projections real dense GEMMs.  They run on the 5th-generation tensor cores:
+//   * activations a (fp32) are split into bf16 hi + lo parts (a = hi + lo up to
+//     2^-17 relative), weights are bf16, and each K step issues two
+//     kind::f16 MMAs (hi x W, lo x W) accumulating in fp32 in TMEM -- fp32-class
+//     accuracy at bf16 tensor-core rate;
+//   * 128 x 128 output tiles, K steps of 64 (one 128-byte swizzled row), a
+//     4-stage TMA ring (A hi, A lo, W: 48 KB per stage), a double-buffered TMEM
+//     accumulator (2 x 128 columns);
+//   * warp 0 issues TMA, warp 1 owns TMEM and one thread of it issues the MMAs,
+//     warps 2-5 drain TMEM with tcgen05.ld and apply the same fused epilogues as
+//     the decode path (RoPE + KV write, SiLU(gate)*up, scaled residual).
+#pragma once
+
+#include "common.cuh"
+#include "gemv.cuh"
+
+#include "prefill_params.cuh"
+
+namespace ssd {
+
+// ------------------------------------------------------------------ tcgen05 helpers
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
+// groups 1024 bytes apart (the layout TMA writes with SWIZZLE_128B).
+__device__ __forceinline__ uint64_t tc_smem_desc(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);        // start address
+  d |= static_cast<uint64_t>(1u) << 16;                       // leading byte offset (unused for swizzled K-major)
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;               // stride byte offset: 8 rows x 128 B
+  d |= static_cast<uint64_t>(1u) << 46;                       // descriptor version
+  d |= static_cast<uint64_t>(2u) << 61;                       // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major, M x N.
+__host__ __device__ constexpr uint32_t tc_idesc(int m, int n) {
+  return (1u << 4)                                  // D format: fp32
+         | (1u << 7)                                // A format: bf16
+         | (1u << 10)                               // B format: bf16
+         | (static_cast<uint32_t>(n >> 3) << 17)    // N / 8
+         | (static_cast<uint32_t>(m >> 4) << 24);   // M / 16
+}
+
+__device__ __forceinline__ void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                       uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+
+// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one lane per thread).
+__device__ __forceinline__ void tc_ld32(uint32_t taddr, float* v) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// ------------------------------------------------------------------ activation split
+
+// Row r of `out_hi` / `out_lo` (bf16 [rows][K]) = split of x[r] (fp32), optionally
+// RMSNorm-scaled: v = x * rs * gain with rs = 1/sqrt(mean(x^2) + eps).
+// hi = bf16(v), lo = bf16(v - hi).
+__global__ void __launch_bounds__(256) split_rows_kernel(const float* __restrict__ x, int x_stride, int K,
+                                                         const __nv_bfloat16* __restrict__ gain, float eps,
+                                                         __nv_bfloat16* __restrict__ out_hi,
+                                                         __nv_bfloat16* __restrict__ out_lo) {
+  __shared__ float red[8];
+  __shared__ float rs_s;
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x, tid = threadIdx.x;
+  const float* xr = x + static_cast<size_t>(r) * x_stride;
+  float rs = 1.f;
+  if (gain) {
+    float ss = 0.f;
+    for (int i = tid; i < (K >> 2); i += 256) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(xr) + i);
+      ss = fmaf(v.x, v.x, ss);
+      ss = fmaf(v.y, v.y, ss);
+      ss = fmaf(v.z, v.z, ss);
+      ss = fmaf(v.w, v.w, ss);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    if ((tid & 31) == 0) red[tid >> 5] = ss;
+    __syncthreads();
+    if (tid == 0) {
+      float t = 0.f;
+      for (int w = 0; w < 8; ++w) t += red[w];
+      rs_s = rsqrtf(t / static_cast<float>(K) + eps);
+    }
+    __syncthreads();
+    rs = rs_s;
+  }
+  __nv_bfloat16* hr = out_hi + static_cast<size_t>(r) * K;
+  __nv_bfloat16* lr = out_lo + static_cast<size_t>(r) * K;
+  for (int i = tid; i < K; i += 256) {
+    float v = __ldcg(xr + i);
+    if (gain) v = v * rs * __bfloat162float(gain[i]);
+    const __nv_bfloat16 h = __float2bfloat16_rn(v);
+    hr[i] = h;
+    lr[i] = __float2bfloat16_rn(v - __bfloat162float(h));
+  }
+}
+
+// ------------------------------------------------------------------ tcgen05 GEMM
+
+template <Epi EPI>
+__device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int r, const float* acc) {
+  // acc: the 128 fp32 outputs of token row r in output tile n_t (columns of the tile)
+  const int pos = p.pos0 + r;
+  if constexpr (EPI == Epi::QKV) {
+    const int c0 = n_t * kTcN, mat = c0 / p.seg_rows, local0 = c0 - mat * p.seg_rows;
+    const int Dh = p.head_dim, half = Dh >> 1;
+    if (pos < 0 || pos >= p.max_seq) {
+      set_error(p.st, DERR_POS);
+      return;
+    }
+    if (mat < 2) {
+      for (int hh = 0; hh < kTcN / Dh; ++hh) {
+        const int h = local0 / Dh + hh;
+        float* kr = mat == 1 ? p.k_cache + (static_cast<size_t>(h) * p.max_seq + pos) * Dh : nullptr;
+        float* qr = mat == 0 ? p.q_out + static_cast<size_t>(r) * p.q_stride + h * Dh : nullptr;
+        for (int j = 0; j < half; ++j) {
+          const float a = acc[hh * Dh + j], b = acc[hh * Dh + j + half];
+          const float2 cs = p.rope_cs[static_cast<size_t>(pos) * half + j];
+          const float va = a * cs.x - b * cs.y;
+          const float vb = a * cs.y + b * cs.x;
+          if (mat == 0) {
+            qr[j] = va;
+            qr[j + half] = vb;
+          } else {
+            kr[j] = va;
+            kr[j + half] = vb;
+          }
+        }
+      }
+    } else {
+      for (int c = 0; c < kTcN; ++c) {
+        const int row = local0 + c, h = row / Dh, d = row - h * Dh;
+        p.v_cache[(static_cast<size_t>(h) * p.max_seq + pos) * Dh + d] = acc[c];
+      }
+    }
+  } else if constexpr (EPI == Epi::GATE_SILU) {
+    float* hr = p.h_out + static_cast<size_t>(r) * p.h_stride + n_t * (kTcN / 2);
+    for (int j = 0; j < kTcN / 2; ++j) {
+      if (n_t * (kTcN / 2) + j >= p.N) break;
+      hr[j] = silu_f(acc[j]) * acc[kTcN / 2 + j];
+    }
+  } else {  // RESID
+    const float s = __ldg(p.scale);
+    const float* br = p.base + static_cast<size_t>(r) * p.base_stride + n_t * kTcN;
+    float* dr = p.dst + static_cast<size_t>(r) * p.dst_stride + n_t * kTcN;
+    for (int c = 0; c < kTcN; ++c) {
+      if (n_t * kTcN + c >= p.N) break;
+      dr[c] = br[c] + s * acc[c];
+    }
+  }
+}
+
+template <Epi EPI>
+__global__ void __launch_bounds__(kTcThreads, 1)
+    tc_gemm_kernel(const __grid_constant__ CUtensorMap map_ahi, const __grid_constant__ CUtensorMap map_alo,
+                   const __grid_constant__ CUtensorMap map_b0, const __grid_constant__ CUtensorMap map_b1,
+                   const __grid_constant__ CUtensorMap map_b2, const TcParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  // 1024-byte aligned base for the swizzled tiles
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kTcStages * kTcStage);
+  uint64_t* empty = full + kTcStages;
+  uint64_t* tfull = empty + kTcStages;   // [2]
+  uint64_t* tempty = tfull + 2;          // [2]
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
+  int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int n_tiles = p.tiles_m * p.tiles_n;
+
+  pdl_trigger();
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kTcStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&tfull[b], 1);
+      mbar_init(&tempty[b], 4);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) {  // TMEM: 2 x 128 fp32 columns
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kTcTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      int g = 0;
+      for (int t = blockIdx.x; t < n_tiles && !*reinterpret_cast<volatile int*>(abort_flag); t += gridDim.x) {
+        const int m_t = t % p.tiles_m, n_t = t / p.tiles_m;
+        for (int ks = 0; ks < p.k_steps; ++ks, ++g) {
+          const int s = g % kTcStages;
+          if (!mbar_wait(&empty[s], ((g / kTcStages) & 1) ^ 1)) {
+            set_error(p.st, DERR_TIMEOUT);
+            *reinterpret_cast<volatile int*>(abort_flag) = 1;
+            break;
+          }
+          uint8_t* st = smem + s * kTcStage;
+          mbar_arrive_expect_tx(&full[s], kTcStage);
+          const int kx = ks * kTcK;
+          tma_load_2d(st, &map_ahi, &full[s], kx, m_t * kTcM);
+          tma_load_2d(st + kTcATile, &map_alo, &full[s], kx, m_t * kTcM);
+          uint8_t* bs = st + 2 * kTcATile;
+          if constexpr (EPI == Epi::GATE_SILU) {
+            tma_load_2d(bs, &map_b0, &full[s], kx, n_t * (kTcN / 2));
+            tma_load_2d(bs + kTcBTile / 2, &map_b1, &full[s], kx, n_t * (kTcN / 2));
+          } else if constexpr (EPI == Epi::QKV) {
+            const int r0 = n_t * kTcN, mat = r0 / p.seg_rows;
+            tma_load_2d(bs, mat == 0 ? &map_b0 : (mat == 1 ? &map_b1 : &map_b2), &full[s], kx, r0 - mat * p.seg_rows);
+          } else {
+            tma_load_2d(bs, &map_b0, &full[s], kx, n_t * kTcN);
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = tc_idesc(kTcM, kTcN);
+      int g = 0, it = 0;
+      for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+        const int b = it & 1;
+        if (!mbar_wait(&tempty[b], ((it >> 1) & 1) ^ 1)) {
+          set_error(p.st, DERR_TIMEOUT);
+          *reinterpret_cast<volatile int*>(abort_flag) = 1;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d = tmem + b * kTcN;
+        bool ok = true;
+        for (int ks = 0; ks < p.k_steps; ++ks, ++g) {
+          const int s = g % kTcStages;
+          if (!mbar_wait(&full[s], (g / kTcStages) & 1)) {
+            set_error(p.st, DERR_TIMEOUT);
+            *reinterpret_cast<volatile int*>(abort_flag) = 1;
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t sa = smem_u32(smem + s * kTcStage);
+          const uint64_t ahi = tc_smem_desc(sa), alo = tc_smem_desc(sa + kTcATile),
+                         bw = tc_smem_desc(sa + 2 * kTcATile);
+#pragma unroll
+          for (int kk = 0; kk < kTcK / 16; ++kk) {
+            // +32 bytes per 16-element K slice inside the 128-byte swizzled row
+            tc_mma(d, ahi + 2 * kk, bw + 2 * kk, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+            tc_mma(d, alo + 2 * kk, bw + 2 * kk, idesc, 1u);
+          }
+          tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+        }
+        if (!ok) break;
+        tc_commit(&tfull[b]);    // accumulator b is complete
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue (warps 2..5)
+    const int q = warp & 3;  // TMEM lane quadrant this warp may access
+    int it = 0;
+    for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
+      const int b = it & 1;
+      const int m_t = t % p.tiles_m, n_t = t / p.tiles_m;
+      if (!mbar_wait(&tfull[b], (it >> 1) & 1)) {
+        set_error(p.st, DERR_TIMEOUT);
+        break;
+      }
+      tc_fence_after();
+      float acc[kTcN];
+      const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + b * kTcN;
+#pragma unroll
+      for (int c = 0; c < kTcN / 32; ++c) tc_ld32(base + c * 32, acc + c * 32);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&tempty[b]);  // accumulator b may be overwritten
+      const int r = m_t * kTcM + q * 32 + lane;
+      if (r < p.M) tc_epilogue_row<EPI>(p, n_t, r, acc);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
+  }
+}
+
+}  // namespace ssd
+
+namespace ssd {
+
+// ------------------------------------------------------------------ causal prefill attention
+// One CTA per (64-query block, head): keys in blocks of 64 up to the query
+// block (causal), scores 4 x 4 per thread in fp32, online softmax per row (a
+// row's 64 scores live on 16 consecutive lanes), O += P V with 4 rows x Dh/16
+// dims per thread.  q: [P][q_stride] rotated queries; K, V: the fp32 cache.
+constexpr int kPaQ = 64;
+constexpr int kPaK = 64;
+constexpr int kPaPad = 68;  // transposed tiles: row length 64 + 4 (16-byte aligned, fewer bank conflicts)
+
+template <int DH>
+struct PaSmem {
+  static constexpr int kQt = 0;                                // [DH][kPaPad]
+  static constexpr int kKt = kQt + DH * kPaPad * 4;            // [DH][kPaPad]
+  static constexpr int kV = kKt + DH * kPaPad * 4;             // [64][DH]
+  static constexpr int kP = kV + kPaK * DH * 4;                // [64][kPaPad]
+  static constexpr int kTotal = kP + kPaQ * kPaPad * 4;
+};
+
+template <int DH>
+__global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restrict__ q, int q_stride,
+                                                           const float* __restrict__ k_cache,
+                                                           const float* __restrict__ v_cache, float* __restrict__ o,
+                                                           int o_stride, int P, int max_seq, float scale) {
+  using S = PaSmem<DH>;
+  constexpr int DPT = DH / 16;  // output dims per thread
+  extern __shared__ __align__(128) uint8_t pa_smem[];
+  float* Qt = reinterpret_cast<float*>(pa_smem + S::kQt);
+  float* Kt = reinterpret_cast<float*>(pa_smem + S::kKt);
+  float* Vs = reinterpret_cast<float*>(pa_smem + S::kV);
+  float* Ps = reinterpret_cast<float*>(pa_smem + S::kP);
+  const int qb = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  const int q0 = qb * kPaQ;
+  const int tr = tid >> 4, tc = tid & 15;  // rows 4tr..4tr+3; score keys 4tc..4tc+3; output dims tc*DPT..
+  pdl_trigger();
+  pdl_wait();
+
+  // Q block, transposed: Qt[d][i] = q[q0 + i][h*DH + d] (rows past P read as 0)
+  for (int idx = tid; idx < kPaQ * DH; idx += 256) {
+    const int i = idx / DH, d = idx - i * DH;
+    Qt[d * kPaPad + i] = (q0 + i < P) ? __ldcg(q + static_cast<size_t>(q0 + i) * q_stride + h * DH + d) : 0.f;
+  }
+  float m_run[4], l_run[4], acc[4][DPT];
+#pragma unroll
+  for (int a = 0; a < 4; ++a) {
+    m_run[a] = -INFINITY;
+    l_run[a] = 0.f;
+#pragma unroll
+    for (int e = 0; e < DPT; ++e) acc[a][e] = 0.f;
+  }
+  const float* kh = k_cache + static_cast<size_t>(h) * max_seq * DH;
+  const float* vh = v_cache + static_cast<size_t>(h) * max_seq * DH;
+  const int n_kb = min(qb + 1, (P + kPaK - 1) / kPaK);
+  for (int kb = 0; kb < n_kb; ++kb) {
+    const int j0 = kb * kPaK;
+    __syncthreads();  // previous block's Kt / Vs / Ps fully used
+    for (int idx = tid; idx < kPaK * DH; idx += 256) {
+      const int j = idx / DH, d = idx - j * DH;
+      const bool in = j0 + j < P;
+      Kt[d * kPaPad + j] = in ? __ldcg(kh + static_cast<size_t>(j0 + j) * DH + d) : 0.f;
+      Vs[j * DH + d] = in ? __ldcg(vh + static_cast<size_t>(j0 + j) * DH + d) : 0.f;
+    }
+    __syncthreads();
+    // scores s[a][b] = q_{4tr+a} . k_{4tc+b}
+    float s[4][4];
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+      for (int b = 0; b < 4; ++b) s[a][b] = 0.f;
+#pragma unroll 4
+    for (int d = 0; d < DH; ++d) {
+      const float4 qv = *reinterpret_cast<const float4*>(Qt + d * kPaPad + 4 * tr);
+      const float4 kv = *reinterpret_cast<const float4*>(Kt + d * kPaPad + 4 * tc);
+      const float qa[4] = {qv.x, qv.y, qv.z, qv.w}, kb4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll
+      for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) s[a][b] = fmaf(qa[a], kb4[b], s[a][b]);
+    }
+    // online softmax per row over this key block (16 lanes share a row)
+#pragma unroll
+    for (int a = 0; a < 4; ++a) {
+      const int qi = q0 + 4 * tr + a;
+      float mx = -INFINITY;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const int kj = j0 + 4 * tc + b;
+        s[a][b] = (kj <= qi && kj < P) ? s[a][b] * scale : -INFINITY;
+        mx = fmaxf(mx, s[a][b]);
+      }
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+      const float m_new = fmaxf(m_run[a], mx);
+      float rsum = 0.f;
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        const float e = (m_new == -INFINITY || s[a][b] == -INFINITY) ? 0.f : expf(s[a][b] - m_new);
+        Ps[(4 * tr + a) * kPaPad + 4 * tc + b] = e;
+        rsum += e;
+      }
+#pragma unroll
+      for (int off = 8; off > 0; off >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, off);
+      const float corr = (m_run[a] == -INFINITY) ? 0.f : expf(m_run[a] - m_new);
+      l_run[a] = l_run[a] * corr + rsum;
+#pragma unroll
+      for (int e = 0; e < DPT; ++e) acc[a][e] *= corr;
+      m_run[a] = m_new;
+    }
+    __syncwarp();
+    __syncthreads();
+    // O += P V
+    const int kn = min(kPaK, P - j0);
+    for (int j = 0; j < kn; ++j) {
+      float vv[DPT];
+#pragma unroll
+      for (int e = 0; e < DPT; e += 4) {
+        const float4 t = *reinterpret_cast<const float4*>(Vs + j * DH + tc * DPT + e);
+        vv[e] = t.x;
+        vv[e + 1] = t.y;
+        vv[e + 2] = t.z;
+        vv[e + 3] = t.w;
+      }
+#pragma unroll
+      for (int a = 0; a < 4; ++a) {
+        const float pj = Ps[(4 * tr + a) * kPaPad + j];
+#pragma unroll
+        for (int e = 0; e < DPT; ++e) acc[a][e] = fmaf(pj, vv[e], acc[a][e]);
+      }
+    }
+  }
+#pragma unroll
+  for (int a = 0; a < 4; ++a) {
+    const int qi = q0 + 4 * tr + a;
+    if (qi >= P) continue;
+    const float inv = 1.0f / l_run[a];
+    float* orow = o + static_cast<size_t>(qi) * o_stride + h * DH + tc * DPT;
+#pragma unroll
+    for (int e = 0; e < DPT; ++e) orow[e] = acc[a][e] * inv;
+  }
+}
+
+}  // namespace ssd

@@ -1,0 +1,42 @@
+// Shape constants and parameters of the prefill (tcgen05) GEMM, shared by the
+// kernels and the host engine.
+#pragma once
+
+#include "common.cuh"
+
+namespace ssd {
+
+constexpr int kTcM = 128;
+constexpr int kTcN = 128;
+constexpr int kTcK = 64;
+constexpr int kTcStages = 4;
+constexpr int kTcThreads = 192;
+constexpr uint32_t kTcATile = kTcM * kTcK * 2;             // 16 KB
+constexpr uint32_t kTcBTile = kTcN * kTcK * 2;             // 16 KB
+constexpr uint32_t kTcStage = 2 * kTcATile + kTcBTile;     // 48 KB
+constexpr int kTcTmemCols = 2 * kTcN;                      // double-buffered fp32 accumulator
+constexpr int kTcSmem = kTcStages * kTcStage + 1024 + 256;  // + alignment slack + barriers
+
+struct TcParams {
+  int M, N, K;          // rows (tokens), output columns, reduction
+  int tiles_m, tiles_n, k_steps;
+  int seg_rows;         // QKV: rows per source matrix
+  int pos0;             // position of row 0
+  DevState* st;
+  // epilogues (same meaning as GemvParams)
+  float* q_out;
+  int q_stride;
+  float* k_cache;
+  float* v_cache;
+  int head_dim, max_seq;
+  const float2* rope_cs;
+  float* h_out;
+  int h_stride;
+  const float* base;
+  int base_stride;
+  float* dst;
+  int dst_stride;
+  const float* scale;
+};
+
+}  // namespace ssd

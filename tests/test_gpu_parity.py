@@ -266,7 +266,8 @@ def test_launch_counts(tiny_model):
     L, k = w.shape.n_layers, w.draft_exit_k
     body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
     assert dec == 3 + st["steps"] * body
-    assert pre == 2 + ((w.prompt_len + 7) // 8) * (1 + 5 * L) + 1
+    # prefill: begin + input rows, per layer 4 activation splits + 4 tensor-core GEMMs + attention, head + finish
+    assert pre == 2 + 9 * L + 2
 
 
 @pytest.mark.parametrize("rows", [1, 5, 9])
@@ -289,3 +290,34 @@ def test_lm_head_op_matches_oracle(tiny_model, tiny_bits, rows):
             assert margin(ref) < 1e-2
     # argmax of the returned logits is the returned token (lowest index on ties)
     assert tok.cpu().tolist() == lg.argmax(dim=1).cpu().int().tolist()
+
+
+@pytest.mark.parametrize("case", ["tiny", "ragged"])
+def test_tensor_core_prefill_matches_row_prefill_and_oracle(case, monkeypatch):
+    """The tcgen05 prefill (hi/lo bf16 split, fp32 accumulation) against the row-chunked decode-kernel prefill."""
+    w = synth.TINY.replace(norm_gain="perturbed", max_new=2)
+    if case == "ragged":
+        w = w.replace(n_vis=131, n_prompt=14)              # P = 145: a partial 128-row tile and 64-query block
+    bits = synth.make_weights(w)
+    caches = []
+    for mode in ("rows", "tc"):
+        monkeypatch.setenv("SSD_PREFILL", mode)
+        model, _, _ = make_model(w, bits)
+        toks, _, _ = gpu_decode(model, w, 0, capture=False)
+        k, v, n = model.kv()
+        P = w.prompt_len
+        caches.append((k[:, :, :P].clone(), v[:, :, :P].clone(), toks))
+        model.close()
+    (k1, v1, t1), (k2, v2, t2) = caches
+    for a, b in ((k1, k2), (v1, v2)):
+        rms = float(a.pow(2).mean().sqrt())
+        torch.testing.assert_close(b, a, rtol=1e-4, atol=1e-4 * rms)
+    m = oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    cache = oracle.KVCache(m.cfg, w.max_seq())
+    ref_logits = oracle.prefill(m, cache, synth.bf16_to_f64(vis), prompt)
+    rms = float(np.sqrt(np.mean(cache.k[:, :, :w.prompt_len] ** 2)))
+    np.testing.assert_allclose(k2.cpu().numpy(), cache.k[:, :, :w.prompt_len], rtol=1e-3, atol=1e-3 * rms)
+    if t2[0] != int(np.argmax(ref_logits)):
+        from tests.parity import margin
+        assert margin(ref_logits) < 1e-2
