@@ -225,7 +225,7 @@ SSD_API ssd_status ssd_lm_head(ssd_ctx* ctx, const float* x, int rows, int32_t* 
  * serving loops whose device memory is owned by their own allocator, hosts
  * that must avoid the implicit synchronisation of cudaMalloc/cudaFree.  The
  * paper has no counterpart; this is a deployment variant.  It needs no ctx and
- * allocates nothing: its scratch is a fixed ~1.3 MB array in device memory that
+ * allocates nothing: its scratch is a fixed ~5.3 MB array in device memory that
  * every GPU loading the library holds until the process exits.
  *   lm_head:    device bf16 [vocab][d_model];  final_norm: device bf16 [d_model]
  *   x:          device fp32 [rows][d_model];  tok: device int32 [rows]

@@ -198,28 +198,18 @@ static ssd_status encode_map_sw128(ssd_ctx* c, CUtensorMap* m, const void* base,
   return SSD_OK;
 }
 
+// GEMV weight boxes: box_rows x 64 columns, 128-byte swizzled (the MMA's A operand).
 static ssd_status encode_map(ssd_ctx* c, CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols,
                              uint32_t box_rows) {
-  if (reinterpret_cast<uintptr_t>(base) % 16 != 0)
-    return fail(c, SSD_ERR_INVALID_ARG, "weight pointer %p is not 16-byte aligned", base);
-  cuuint64_t dims[2] = {cols, rows};
-  cuuint64_t strides[1] = {cols * 2};
-  cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), box_rows};
-  cuuint32_t es[2] = {1, 1};
-  CUresult r = g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, es,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) return fail(c, SSD_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", static_cast<int>(r));
-  return SSD_OK;
+  return encode_map_sw128(c, m, base, rows, cols, box_rows);
 }
 
-// Site over 1..3 matrices [rows_each][K] stacked along N.  Units are 32 rows x
-// 256 columns; with `paired`, the first two matrices (q, k) are read as two
-// 16-row halves per unit (rows i and i + head_dim/2 of a head).
+// Site over 1..3 matrices [rows_each][K] stacked along N.  Units are 128 rows x
+// 64 columns (a QKV unit holds whole heads, so RoPE pairs stay in one unit).
 static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nmats, int rows_each, int K,
                             bool paired) {
   for (int i = 0; i < nmats; ++i)
-    CKS(encode_map(c, &s->maps[i], mats[i], rows_each, K, (paired && i < 2) ? kHalfN : kTileN));
+    CKS(encode_map(c, &s->maps[i], mats[i], rows_each, K, kTileN));
   for (int i = nmats; i < 3; ++i) s->maps[i] = s->maps[0];
   s->N = rows_each * nmats;
   s->K = K;
@@ -231,7 +221,7 @@ static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nm
   return SSD_OK;
 }
 
-// gate/up pair: each unit holds 16 gate rows and the same 16 up rows.
+// gate/up pair: each unit holds 64 gate rows and the same 64 up rows.
 static ssd_status make_pair_site(ssd_ctx* c, Site* s, const void* gate, const void* up, int rows, int K) {
   CKS(encode_map(c, &s->maps[0], gate, rows, K, kHalfN));
   CKS(encode_map(c, &s->maps[1], up, rows, K, kHalfN));
@@ -806,7 +796,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     c->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
     c->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
     const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
-    CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model, true));
+    CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model, false));
     CKS(make_site(c, &c->layers[l].o, &w->wo[l], 1, k.d_model, qdim, false));
     CKS(make_pair_site(c, &c->layers[l].gateup, w->w_gate[l], w->w_up[l], k.d_ff, k.d_model));
     CKS(make_site(c, &c->layers[l].down, &w->w_down[l], 1, k.d_model, k.d_ff, false));

@@ -1,65 +1,67 @@
-// Weight-streaming skinny GEMM ("GEMV" for M = 1..9 activation rows).
+// Weight-streaming skinny GEMM ("GEMV" for M = 1..9 activation rows) on the
+// 5th-generation tensor cores.
 //
 //   out[m][n] = sum_k W[n][k] * a[m][k],   W bf16 [N][K] (nn.Linear layout), a fp32
 //
 // Every decode-time projection of the decoder (Sec. "SSD Setup for VLMs",
 // x_{l+1} = x_l + f_l(x_l)), of the imitation network and of the LM head g
 // runs through this kernel; at batch 1 it is bound by HBM bandwidth, since each
-// weight byte is used for M <= 9 rows only.
-//
-// Design (sm_103a):
+// weight byte is used for M <= 9 rows only.  The arithmetic runs on tcgen05 so
+// that issue slots never limit the weight stream:
 //  * persistent grid of min(2 x #SMs, units) CTAs; the weight matrix is cut
-//    into units of 32 rows x 256 columns (16 KB of bf16, 512-byte runs per row)
-//    and CTA c streams the contiguous unit range [c*U/G, (c+1)*U/G) -- stream-K,
-//    so every SM moves the same number of bytes whatever N and K are;
-//  * thread 0 issues 2D TMA loads of the weight units (plus 1D bulk copies of
-//    the matching 256-column slice of each activation row and of the RMSNorm
-//    gain) into a 4-stage shared-memory ring guarded by mbarriers; the first
-//    stages' weights are requested before griddepcontrol.wait, so they overlap
-//    the previous kernel (programmatic dependent launch); a stage is refilled
-//    as soon as its eight warps have released it;
-//  * warp w owns rows 4w..4w+3 of the unit, lane l columns 8l..8l+7; weights
-//    are read with 128-bit shared loads and accumulated in fp32 with packed
-//    FFMA2 (__ffma2_rn); activations stay fp32;
-//  * finished row tiles are parked in shared memory and their epilogues (and
-//    the cross-CTA reduction of row tiles split between CTAs, in fixed CTA
-//    order by the CTA that finishes last -- an atomic ticket, no spinning) run
-//    after the stream, so the weight stream never pauses mid-kernel;
-//  * the fused epilogue applies the RMSNorm scale 1/rms(x) (the gain is folded
-//    into the activations) and then RoPE + KV-cache write (QKV; the cache holds
-//    fp32), SiLU(gate)*up, SiLU, a scaled residual add, or the LM-head argmax.
-//    For QKV and gate/up a unit holds two 16-row halves: rows i and i+Dh/2 of
-//    a head (a RoPE pair), or gate row i and up row i.
+//    into units of 128 rows x 64 columns (16 KB, one 128-byte swizzled row per
+//    weight row) and CTA c streams the contiguous unit range [c*U/G, (c+1)*U/G)
+//    -- stream-K, so every SM moves the same number of bytes;
+//  * warp 0 issues TMA: the weight unit (SWIZZLE_128B), the fp32 slice of each
+//    activation row and of the RMSNorm gain, into a 4-stage mbarrier ring; the
+//    first stages' weights are requested before griddepcontrol.wait, so they
+//    overlap the previous kernel (programmatic dependent launch);
+//  * warps 2-3 turn each activation slice into the MMA's B operand: a = hi + lo
+//    in bf16 (a to 2^-17 relative), rows padded to N = 16 with zeros, written in
+//    the swizzled K-major layout;
+//  * one thread of warp 1 issues tcgen05.mma.kind::f16 with the weight unit as
+//    A (M = 128 weight rows) and the activations as B (N = 16): per unit 4 K
+//    slices x (hi, lo) = 8 MMAs accumulating in fp32 in TMEM; a row tile's
+//    accumulator (128 lanes x 16 columns) is double-buffered;
+//  * warps 4-7 drain finished accumulators with tcgen05.ld while the stream
+//    goes on, reduce row tiles split between CTAs in fixed CTA order (the CTA
+//    that finishes a tile last does it -- an atomic ticket, no spinning), and
+//    apply the fused epilogue: the RMSNorm scale 1/rms(x) (the gain is folded
+//    into the activations), then RoPE + KV-cache write (QKV), SiLU(gate)*up
+//    (a unit holds 64 gate + the same 64 up rows), SiLU, a scaled residual
+//    add, or the LM-head argmax.
 //
-// Batch invariance: the unit partition, the order of FMAs feeding each output
-// and the reduction trees do not depend on M, so row m of an M-row launch is
-// bitwise equal to the same row computed alone.  This makes the verify pass
-// (M = gamma+1) reproduce greedy decoding (M = 1) exactly.
+// Batch invariance: the unit partition, the MMA shape (always N = 16), the K
+// order and the reduction order do not depend on M, and each output element
+// is an independent dot product, so row m of an M-row launch is bitwise equal
+// to the same row computed alone.  This makes the verify pass (M = gamma+1)
+// reproduce greedy decoding (M = 1) exactly.
 #pragma once
 
 #include "common.cuh"
 
 namespace ssd {
 
-constexpr int kTileN = 32;           // weight rows per unit
-constexpr int kHalfN = kTileN / 2;   // rows per half box (paired units)
-constexpr int kTileK = 256;          // weight columns per unit (512 bytes of bf16)
-constexpr int kConsumerWarps = 8;
-constexpr int kConsumerThreads = kConsumerWarps * 32;
-constexpr int kGemvThreads = kConsumerThreads;
+constexpr int kTileN = 128;          // weight rows per unit (the MMA's M)
+constexpr int kHalfN = kTileN / 2;   // gate or up rows of a paired unit
+constexpr int kTileK = 64;           // weight columns per unit (one 128-byte swizzled row)
+constexpr int kNPad = 16;            // activation rows padded to the MMA's N
 constexpr int kStages = 4;
-constexpr int kMaxSeg = 8;           // parked row-tile results before a flush
-constexpr uint32_t kWTileBytes = kTileN * kTileK * 2;
+constexpr int kGemvThreads = 256;
+constexpr int kDrainThreads = 128;   // warps 4..7
+constexpr int kTmemCols = 32;        // two 16-column accumulators
+constexpr uint32_t kWTileBytes = kTileN * kTileK * 2;   // 16 KB
+constexpr uint32_t kBOpBytes = kNPad * kTileK * 2;      // 2 KB (hi or lo)
 
 enum class Epi : int { QKV = 0, GATE_SILU = 1, SILU = 2, RESID = 3, ARGMAX = 4 };
 
 struct GemvParams {
   int K, n_kt, n_rt, units;
-  int N;           // valid output rows (GATE_SILU: d_ff; a unit holds 16 gate + 16 up rows)
+  int N;           // valid output rows (GATE_SILU: d_ff; a unit holds 64 gate + 64 up rows)
   int seg_rows;    // QKV: rows per source matrix (q, k, v)
-  const float* x;  // activations [M][x_stride] (fp32, columns K..x_stride-1 zero)
+  const float* x;  // activations [M][x_stride] (fp32)
   int x_stride;
-  const __nv_bfloat16* gain;  // RMSNorm gain, zero-padded to a multiple of kTileK, or null (no norm)
+  const __nv_bfloat16* gain;  // RMSNorm gain (zero-padded), or null (no norm)
   float eps;
   float* partials;      // [2 * grid][kMaxRows][kTileN]
   unsigned* counters;   // [n_rt]
@@ -91,17 +93,17 @@ struct GemvParams {
 template <int M>
 struct GemvSmem {
   static constexpr int kActBytes = M * kTileK * 4;
-  static constexpr int kW = 0;
-  static constexpr int kA = kW + kStages * kWTileBytes;
-  static constexpr int kG = kA + kStages * kActBytes;
-  static constexpr int kSeg = kG + kStages * kTileK * 2;          // parked tiles [kMaxSeg][M][kTileN]
-  static constexpr int kSegRt = kSeg + kMaxSeg * M * kTileN * 4;  // [kMaxSeg] row tile, [kMaxSeg] whole flag
-  static constexpr int kOut = kSegRt + 2 * kMaxSeg * 4;          // reduction buffer [M][kTileN]
+  static constexpr int kW = 0;                                  // [stages][16 KB] weight units (1024-aligned)
+  static constexpr int kB = kW + kStages * kWTileBytes;         // [stages][hi | lo] B operands (1024-aligned)
+  static constexpr int kA = kB + kStages * 2 * kBOpBytes;       // [stages][M][64] fp32 activation slices
+  static constexpr int kG = kA + kStages * kActBytes;           // [stages][64] bf16 gain slices
+  static constexpr int kOut = kG + kStages * kTileK * 2;        // drained row tile [M][128]
   static constexpr int kRs = kOut + M * kTileN * 4;
-  static constexpr int kRed = kRs + kMaxRows * 4;
-  static constexpr int kFlag = kRed + kConsumerWarps * kMaxRows * 4;
-  static constexpr int kBar = (kFlag + 16 + 7) & ~7;
-  static constexpr int kTotal = kBar + 2 * kStages * 8;
+  static constexpr int kRed = kRs + kMaxRows * 4;               // [4][kMaxRows]
+  static constexpr int kFlag = kRed + 4 * kMaxRows * 4;
+  static constexpr int kBar = (kFlag + 16 + 7) & ~7;            // full, empty, bready [stages]; afull, aempty [2]
+  static constexpr int kTmemSlot = kBar + (3 * kStages + 4) * 8;
+  static constexpr int kTotal = kTmemSlot + 16 + 1024;          // + slack for the 1024-byte alignment
 };
 
 // Which CTA of a G-CTA grid owns unit u (ranges [floor(cU/G), floor((c+1)U/G))).
@@ -112,57 +114,118 @@ __device__ __forceinline__ int unit_begin(int c, int units, int G) {
   return static_cast<int>((static_cast<long long>(c) * units) / G);
 }
 
+// ------------------------------------------------------------------ tcgen05 helpers
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
+// groups 1024 bytes apart (the layout TMA writes with SWIZZLE_128B).
+__device__ __forceinline__ uint64_t umma_desc_sw128(uint32_t saddr) {
+  uint64_t d = 0;
+  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);  // start address
+  d |= static_cast<uint64_t>(1u) << 16;                 // leading byte offset (unused for swizzled K-major)
+  d |= static_cast<uint64_t>(1024u >> 4) << 32;         // stride byte offset: 8 rows x 128 B
+  d |= static_cast<uint64_t>(1u) << 46;                 // descriptor version
+  d |= static_cast<uint64_t>(2u) << 61;                 // swizzle: 128 B
+  return d;
+}
+
+// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major, M x N.
+__host__ __device__ constexpr uint32_t umma_idesc_bf16(int m, int n) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | (static_cast<uint32_t>(n >> 3) << 17) |
+         (static_cast<uint32_t>(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                         uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void umma_commit(uint64_t* bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+               : "memory");
+}
+
+__device__ __forceinline__ void tmem_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tmem_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+
+// 16 consecutive fp32 columns of this warp's 32 TMEM lanes (one lane per thread).
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float* v) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 lo, __nv_bfloat16 hi) {
+  return static_cast<uint32_t>(__bfloat16_as_ushort(lo)) | (static_cast<uint32_t>(__bfloat16_as_ushort(hi)) << 16);
+}
+
 // ------------------------------------------------------------------ epilogues
-// All run on the 256 threads with the finished row tile in out ([M][kTileN],
+// Run on the 128 drain threads with the finished row tile in out ([M][kTileN],
 // fp32, before the RMSNorm scale) and rs[m] (1 if no norm).
+
+__device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
 
 template <int M, Epi EPI>
 __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const float* out, const float* rs,
                                               int tid) {
   if constexpr (EPI == Epi::QKV) {
-    const int tiles_per_mat = p.seg_rows / kTileN;
-    const int mat = rt / tiles_per_mat;  // 0 = q, 1 = k, 2 = v
-    const int rtm = rt - mat * tiles_per_mat;
-    const int Dh = p.head_dim, half = Dh >> 1, tph = half / kHalfN;  // paired tiles per head
+    const int r0 = rt * kTileN;
+    const int mat = r0 / p.seg_rows;  // 0 = q, 1 = k, 2 = v
+    const int local0 = r0 - mat * p.seg_rows;
+    const int Dh = p.head_dim, half = Dh >> 1;
     const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
     if (mat < 2) {
-      const int h = rtm / tph, j0 = (rtm - h * tph) * kHalfN;
-      for (int idx = tid; idx < M * kHalfN; idx += kConsumerThreads) {
-        const int m = idx / kHalfN, i = idx - m * kHalfN;
+      for (int idx = tid; idx < M * (kTileN / 2); idx += kDrainThreads) {
+        const int m = idx / (kTileN / 2), pr = idx - m * (kTileN / 2);
+        const int hh = pr / half, j = pr - hh * half;
+        const int ra = hh * Dh + j, rb = ra + half;
         const int pos = base_pos + m;
         if (pos < 0 || pos >= p.max_seq) {
           set_error(p.st, DERR_POS);
           continue;
         }
-        const int j = j0 + i;  // rotation pair (j, j + half) of head h
-        const float a = out[m * kTileN + i] * rs[m];
-        const float b = out[m * kTileN + kHalfN + i] * rs[m];
+        const float a = out[m * kTileN + ra] * rs[m];
+        const float b = out[m * kTileN + rb] * rs[m];
         const float2 cs = p.rope_cs[static_cast<size_t>(pos) * half + j];
         const float va = a * cs.x - b * cs.y;
         const float vb = a * cs.y + b * cs.x;
         if (mat == 0) {
-          p.q_out[m * p.q_stride + h * Dh + j] = va;
-          p.q_out[m * p.q_stride + h * Dh + j + half] = vb;
+          p.q_out[m * p.q_stride + local0 + ra] = va;
+          p.q_out[m * p.q_stride + local0 + rb] = vb;
         } else {
+          const int h = local0 / Dh + hh;
           float* kr = p.k_cache + (static_cast<size_t>(h) * p.max_seq + pos) * Dh;
           kr[j] = va;
           kr[j + half] = vb;
         }
       }
     } else {
-      for (int idx = tid; idx < M * kTileN; idx += kConsumerThreads) {
+      for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
         const int m = idx / kTileN, i = idx - m * kTileN;
         const int pos = base_pos + m;
         if (pos < 0 || pos >= p.max_seq) {
           set_error(p.st, DERR_POS);
           continue;
         }
-        const int row = rtm * kTileN + i, h = row / Dh, d = row - h * Dh;
+        const int row = local0 + i, h = row / Dh, d = row - h * Dh;
         p.v_cache[(static_cast<size_t>(h) * p.max_seq + pos) * Dh + d] = out[idx] * rs[m];
       }
     }
   } else if constexpr (EPI == Epi::GATE_SILU) {
-    for (int idx = tid; idx < M * kHalfN; idx += kConsumerThreads) {
+    for (int idx = tid; idx < M * kHalfN; idx += kDrainThreads) {
       const int m = idx / kHalfN, j = idx - m * kHalfN;
       const int n = rt * kHalfN + j;
       if (n >= p.N) continue;
@@ -171,7 +234,7 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       p.h_out[m * p.h_stride + n] = silu_f(g) * u;
     }
   } else if constexpr (EPI == Epi::SILU) {
-    for (int idx = tid; idx < M * kTileN; idx += kConsumerThreads) {
+    for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
       const int m = idx / kTileN, i = idx - m * kTileN;
       const int n = rt * kTileN + i;
       if (n >= p.N) continue;
@@ -179,7 +242,7 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     }
   } else if constexpr (EPI == Epi::RESID) {
     const float s = __ldg(p.scale);
-    for (int idx = tid; idx < M * kTileN; idx += kConsumerThreads) {
+    for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
       const int m = idx / kTileN, i = idx - m * kTileN;
       const int n = rt * kTileN + i;
       if (n >= p.N) continue;
@@ -187,13 +250,14 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       p.dst[m * p.dst_stride + n] = b + s * (out[idx] * rs[m]);
     }
   } else {  // ARGMAX (LM head): argmax over the vocabulary, lowest index on ties
-    const int warp = tid >> 5, lane = tid & 31;
+    const int lane = tid & 31;
     const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
     const int P = __ldcg(&p.st->prompt_len);
-    for (int m = warp; m < M; m += kConsumerWarps) {  // warp per row, lane per tile row
-      const int n = rt * kTileN + lane;
-      const bool valid = n < p.N;
-      const float logit = out[m * kTileN + lane] * rs[m];
+    const int n = rt * kTileN + tid;  // thread per tile row
+    const bool valid = n < p.N;
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      const float logit = out[m * kTileN + tid] * rs[m];
       if (p.logits != nullptr && valid) {
         const int row = base_pos + m + 1 - P;
         if (row >= 0 && row < p.logits_rows) p.logits[static_cast<size_t>(row) * p.N + n] = logit;
@@ -207,7 +271,7 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       if (lane == 0) atomicMax(&p.st->am_key[m], key);
     }
     __threadfence();
-    __syncthreads();
+    drain_sync();
     if (tid == 0) {
       const unsigned prev = atomicAdd(&p.st->am_count, 1u);
       if (prev == static_cast<unsigned>(p.n_rt - 1)) {
@@ -225,16 +289,20 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
 // ------------------------------------------------------------------ kernel
 
 template <int M, Epi EPI>
-__global__ void __launch_bounds__(kGemvThreads, (M <= 6 ? 2 : 1))
+__global__ void __launch_bounds__(kGemvThreads, 2)
     gemv_kernel(const __grid_constant__ CUtensorMap map0, const __grid_constant__ CUtensorMap map1,
                 const __grid_constant__ CUtensorMap map2, const GemvParams p) {
+  static_assert(M >= 1 && M <= kNPad, "activation rows");
   using S = GemvSmem<M>;
-  extern __shared__ __align__(128) uint8_t smem[];
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBar);
   uint64_t* empty = full + kStages;
-  float* seg = reinterpret_cast<float*>(smem + S::kSeg);
-  int* seg_rt = reinterpret_cast<int*>(smem + S::kSegRt);
-  int* seg_whole = seg_rt + kMaxSeg;
+  uint64_t* bready = empty + kStages;
+  uint64_t* afull = bready + kStages;
+  uint64_t* aempty = afull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
   float* outb = reinterpret_cast<float*>(smem + S::kOut);
   float* rs = reinterpret_cast<float*>(smem + S::kRs);
   float* red = reinterpret_cast<float*>(smem + S::kRed);
@@ -246,246 +314,262 @@ __global__ void __launch_bounds__(kGemvThreads, (M <= 6 ? 2 : 1))
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t tx = kWTileBytes + S::kActBytes + (p.gain ? kTileK * 2 : 0);
 
-  // ---- producer helpers (thread 0 only)
-  auto weight_box = [&](int u, auto&& op) {
-    const int rt = u / p.n_kt, kt = u - rt * p.n_kt;
-    const int x = kt * kTileK;
-    if constexpr (EPI == Epi::GATE_SILU) {
-      op(&map0, x, rt * kHalfN, 0);
-      op(&map1, x, rt * kHalfN, static_cast<int>(kWTileBytes / 2));
-    } else if constexpr (EPI == Epi::QKV) {
-      const int tiles_per_mat = p.seg_rows / kTileN;
-      const int mat = rt / tiles_per_mat, rtm = rt - mat * tiles_per_mat;
-      if (mat < 2) {
-        const int half = p.head_dim >> 1, tph = half / kHalfN;
-        const int h = rtm / tph, r1 = h * p.head_dim + (rtm - h * tph) * kHalfN;
-        const CUtensorMap* mp = mat == 0 ? &map0 : &map1;
-        op(mp, x, r1, 0);
-        op(mp, x, r1 + half, static_cast<int>(kWTileBytes / 2));
-      } else {
-        op(&map2, x, rtm * kTileN, 0);
-      }
-    } else {
-      op(&map0, x, rt * kTileN, 0);
-    }
-  };
-  auto issue_weights = [&](int s, int u) {
-    uint8_t* wdst = smem + S::kW + s * kWTileBytes;
-    weight_box(u, [&](const CUtensorMap* mp, int x, int y, int off) { tma_load_2d(wdst + off, mp, &full[s], x, y); });
-    if (p.gain) {
-      const int kt = u % p.n_kt;
-      bulk_load(smem + S::kG + s * kTileK * 2, p.gain + kt * kTileK, kTileK * 2, &full[s]);
-    }
-  };
-  auto prefetch_unit = [&](int u) {
-    weight_box(u, [&](const CUtensorMap* mp, int x, int y, int) { tma_prefetch_2d(mp, x, y); });
-  };
-  auto issue_acts = [&](int s, int u) {
-    const int kt = u % p.n_kt;
-    uint8_t* adst = smem + S::kA + s * S::kActBytes;
-#pragma unroll
-    for (int m = 0; m < M; ++m)
-      bulk_load(adst + m * kTileK * 4, p.x + static_cast<size_t>(m) * p.x_stride + kt * kTileK, kTileK * 4,
-                &full[s]);
-  };
-
   pdl_trigger();
   // After a timed-out wait anywhere in the decode, later kernels do nothing
-  // (best-effort read before any copy is issued).
+  // (best-effort read before any copy is issued or TMEM is taken).
   if (*reinterpret_cast<volatile int*>(&p.st->error) & DERR_TIMEOUT) return;
+
+  // zero the B operands once: rows M..15 stay zero for the whole kernel
+  for (int i = tid; i < kStages * 2 * static_cast<int>(kBOpBytes) / 16; i += kGemvThreads)
+    reinterpret_cast<uint4*>(smem + S::kB)[i] = make_uint4(0, 0, 0, 0);
+  fence_proxy_async_smem();
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&full[s], 1);
-      mbar_init(&empty[s], kConsumerWarps);
+      mbar_init(&empty[s], 1);
+      mbar_init(&bready[s], 2);
     }
-    flag[0] = 0;
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&afull[b], 1);
+      mbar_init(&aempty[b], 4);
+    }
     fence_mbar_init();
   }
-  __syncthreads();
-  const int npre = n_units < kStages ? n_units : kStages;
-  if (tid == 0) {
-    prefetch_tensormap(&map0);
-    // weights do not depend on the previous kernel: start streaming before the wait
-    for (int i = 0; i < npre; ++i) {
-      mbar_arrive_expect_tx(&full[i], tx);
-      issue_weights(i, u0 + i);
-    }
-    const int pf_end = min(n_units, npre + p.pf_dist);
-    for (int i = npre; i < pf_end; ++i) prefetch_unit(u0 + i);
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  pdl_wait();  // activations, residuals and state are written by the previous kernel
-  if (tid == 0)
-    for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
+  tmem_fence_before();
+  __syncthreads();
+  tmem_fence_after();
+  const uint32_t tmem = *tmem_slot;
 
-  float2 acc[4][M];
-#pragma unroll
-  for (int j = 0; j < 4; ++j)
-#pragma unroll
-    for (int m = 0; m < M; ++m) acc[j][m] = make_float2(0.f, 0.f);
-
-  const int rt_first = u0 / p.n_kt;
-  int seg_kt0 = u0 - rt_first * p.n_kt;
-  int nseg = 0;
-  bool rs_done = false;
-  const uint8_t* wbase = smem + S::kW + (warp * 4) * (kTileK * 2) + lane * 16;
-
-  // Runs the epilogues / cross-CTA reductions of the parked row tiles (all threads).
-  auto flush = [&]() {
-    __syncthreads();
-    if (!rs_done) {
-      // RMSNorm scale per row: rs[m] = 1/sqrt(mean(x^2) + eps), fixed reduction order
-      if (p.gain) {
-#pragma unroll 1
-        for (int m = 0; m < M; ++m) {
-          const float4* xr = reinterpret_cast<const float4*>(p.x + static_cast<size_t>(m) * p.x_stride);
-          float ss = 0.f;
-          for (int i = tid; i < (p.K >> 2); i += kConsumerThreads) {
-            const float4 v = __ldcg(xr + i);
-            ss = fmaf(v.x, v.x, ss);
-            ss = fmaf(v.y, v.y, ss);
-            ss = fmaf(v.z, v.z, ss);
-            ss = fmaf(v.w, v.w, ss);
-          }
-#pragma unroll
-          for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-          if (lane == 0) red[warp * kMaxRows + m] = ss;
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      auto issue_weights = [&](int s, int u) {
+        const int rt = u / p.n_kt, kt = u - rt * p.n_kt;
+        uint8_t* wdst = smem + S::kW + s * kWTileBytes;
+        const int x = kt * kTileK;
+        if constexpr (EPI == Epi::GATE_SILU) {
+          tma_load_2d(wdst, &map0, &full[s], x, rt * kHalfN);
+          tma_load_2d(wdst + kWTileBytes / 2, &map1, &full[s], x, rt * kHalfN);
+        } else if constexpr (EPI == Epi::QKV) {
+          const int r0 = rt * kTileN, mat = r0 / p.seg_rows;
+          tma_load_2d(wdst, mat == 0 ? &map0 : (mat == 1 ? &map1 : &map2), &full[s], x, r0 - mat * p.seg_rows);
+        } else {
+          tma_load_2d(wdst, &map0, &full[s], x, rt * kTileN);
         }
-        __syncthreads();
-        if (tid < M) {
-          float t = 0.f;
-          for (int w = 0; w < kConsumerWarps; ++w) t += red[w * kMaxRows + tid];
-          rs[tid] = rsqrtf(t / static_cast<float>(p.K) + p.eps);
-        }
-      } else if (tid < M) {
-        rs[tid] = 1.0f;
+        if (p.gain) bulk_load(smem + S::kG + s * kTileK * 2, p.gain + x, kTileK * 2, &full[s]);
+      };
+      auto issue_acts = [&](int s, int u) {
+        const int kt = u % p.n_kt;
+        uint8_t* adst = smem + S::kA + s * S::kActBytes;
+#pragma unroll
+        for (int m = 0; m < M; ++m)
+          bulk_load(adst + m * kTileK * 4, p.x + static_cast<size_t>(m) * p.x_stride + kt * kTileK, kTileK * 4,
+                    &full[s]);
+      };
+      prefetch_tensormap(&map0);
+      const int npre = n_units < kStages ? n_units : kStages;
+      for (int i = 0; i < npre; ++i) {
+        mbar_arrive_expect_tx(&full[i], tx);
+        issue_weights(i, u0 + i);  // weights do not depend on the previous kernel
       }
-      __syncthreads();
-      rs_done = true;
+      pdl_wait();
+      for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
+      for (int i = npre; i < n_units; ++i) {
+        const int s = i % kStages;
+        if (!mbar_wait(&empty[s], static_cast<uint32_t>((i / kStages) - 1) & 1u)) {
+          set_error(p.st, DERR_TIMEOUT);
+          break;
+        }
+        mbar_arrive_expect_tx(&full[s], tx);
+        issue_weights(s, u0 + i);
+        issue_acts(s, u0 + i);
+      }
     }
-    for (int k = 0; k < nseg; ++k) {
-      const int rt = seg_rt[k];
-      const float* so = seg + k * (M * kTileN);
-      if (seg_whole[k]) {
-        gemv_epilogue<M, EPI>(p, rt, so, rs, tid);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma_idesc_bf16(kTileN, kNPad);
+      int sg = 0;
+      bool seg_open = false;
+      uint32_t d = tmem;
+      for (int i = 0; i < n_units; ++i) {
+        const int u = u0 + i, kt = u % p.n_kt, s = i % kStages;
+        if (!seg_open) {  // a new row-tile segment: take a free accumulator
+          const int b = sg & 1;
+          if (!mbar_wait(&aempty[b], static_cast<uint32_t>(((sg >> 1) & 1) ^ 1))) {
+            set_error(p.st, DERR_TIMEOUT);
+            break;
+          }
+          tmem_fence_after();
+          d = tmem + static_cast<uint32_t>(b * kNPad);
+        }
+        if (!mbar_wait(&bready[s], static_cast<uint32_t>(i / kStages) & 1u)) {
+          set_error(p.st, DERR_TIMEOUT);
+          break;
+        }
+        tmem_fence_after();
+        const uint32_t wa = smem_u32(smem + S::kW + s * kWTileBytes);
+        const uint32_t ba = smem_u32(smem + S::kB + s * 2 * kBOpBytes);
+        const uint64_t adesc = umma_desc_sw128(wa), hdesc = umma_desc_sw128(ba), ldesc = umma_desc_sw128(ba + kBOpBytes);
+#pragma unroll
+        for (int kk = 0; kk < kTileK / 16; ++kk) {
+          // +32 bytes (2 descriptor units) per 16-element K slice inside the swizzled row
+          umma_f16(d, adesc + 2 * kk, hdesc + 2 * kk, idesc, (seg_open || kk > 0) ? 1u : 0u);
+          umma_f16(d, adesc + 2 * kk, ldesc + 2 * kk, idesc, 1u);
+          seg_open = true;
+        }
+        umma_commit(&empty[s]);  // stage s may be refilled once these MMAs have read it
+        if (kt == p.n_kt - 1 || i == n_units - 1) {
+          umma_commit(&afull[sg & 1]);  // the row tile's accumulator is complete
+          ++sg;
+          seg_open = false;
+        }
+      }
+    }
+  } else if (warp < 4) {
+    // ---------------------------------------------------------------- B operand: fp32 -> bf16 hi + lo, swizzled
+    const int ct = tid - 64;  // 0..63
+    for (int i = 0; i < n_units; ++i) {
+      const int s = i % kStages;
+      if (!mbar_wait(&full[s], static_cast<uint32_t>(i / kStages) & 1u)) {
+        set_error(p.st, DERR_TIMEOUT);
+        break;
+      }
+      const float* a = reinterpret_cast<const float*>(smem + S::kA + s * S::kActBytes);
+      const __nv_bfloat16* g = reinterpret_cast<const __nv_bfloat16*>(smem + S::kG + s * kTileK * 2);
+      uint8_t* bh = smem + S::kB + s * 2 * kBOpBytes;
+      for (int task = ct; task < M * 8; task += 64) {
+        const int m = task >> 3, ch = task & 7;
+        const float4 a0 = *reinterpret_cast<const float4*>(a + m * kTileK + ch * 8);
+        const float4 a1 = *reinterpret_cast<const float4*>(a + m * kTileK + ch * 8 + 4);
+        float v[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+        if (p.gain) {
+          const uint4 gv = *reinterpret_cast<const uint4*>(g + ch * 8);
+          const float2 g0 = bf16x2_to_float2(gv.x), g1 = bf16x2_to_float2(gv.y), g2 = bf16x2_to_float2(gv.z),
+                       g3 = bf16x2_to_float2(gv.w);
+          v[0] *= g0.x; v[1] *= g0.y; v[2] *= g1.x; v[3] *= g1.y;
+          v[4] *= g2.x; v[5] *= g2.y; v[6] *= g3.x; v[7] *= g3.y;
+        }
+        uint32_t hw[4], lw[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]), h1 = __float2bfloat16_rn(v[2 * e + 1]);
+          const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * e] - __bfloat162float(h0));
+          const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1));
+          hw[e] = pack_bf16x2(h0, h1);
+          lw[e] = pack_bf16x2(l0, l1);
+        }
+        const int off = m * 128 + ((ch ^ (m & 7)) << 4);  // 128-byte swizzle of row m
+        *reinterpret_cast<uint4*>(bh + off) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        *reinterpret_cast<uint4*>(bh + kBOpBytes + off) = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+      }
+      fence_proxy_async_smem();  // make the generic-proxy writes visible to the tensor core
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bready[s]);
+    }
+  } else {
+    // ---------------------------------------------------------------- drain + epilogues (warps 4..7)
+    const int dt = tid - 128;  // 0..127
+    const int q = warp & 3;    // TMEM lane quadrant: tile rows 32q .. 32q+31
+    pdl_wait();
+    // RMSNorm scale per row: rs[m] = 1/sqrt(mean(x^2) + eps), fixed reduction order
+    if (p.gain) {
+#pragma unroll 1
+      for (int m = 0; m < M; ++m) {
+        const float4* xr = reinterpret_cast<const float4*>(p.x + static_cast<size_t>(m) * p.x_stride);
+        float ss = 0.f;
+        for (int i = dt; i < (p.K >> 2); i += kDrainThreads) {
+          const float4 v = __ldcg(xr + i);
+          ss = fmaf(v.x, v.x, ss);
+          ss = fmaf(v.y, v.y, ss);
+          ss = fmaf(v.z, v.z, ss);
+          ss = fmaf(v.w, v.w, ss);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+        if (lane == 0) red[(warp - 4) * kMaxRows + m] = ss;
+      }
+      drain_sync();
+      if (dt < M) {
+        float t = 0.f;
+        for (int w = 0; w < 4; ++w) t += red[w * kMaxRows + dt];
+        rs[dt] = rsqrtf(t / static_cast<float>(p.K) + p.eps);
+      }
+    } else if (dt < M) {
+      rs[dt] = 1.0f;
+    }
+    drain_sync();
+
+    const int rt_first = u0 / p.n_kt;
+    int seg_kt0 = u0 - rt_first * p.n_kt;
+    int sg = 0;
+    for (int i = 0; i < n_units; ++i) {
+      const int u = u0 + i, rt = u / p.n_kt, kt = u - rt * p.n_kt;
+      if (!(kt == p.n_kt - 1 || i == n_units - 1)) continue;
+      const int b = sg & 1;
+      if (!mbar_wait(&afull[b], static_cast<uint32_t>((sg >> 1) & 1))) {
+        set_error(p.st, DERR_TIMEOUT);
+        break;
+      }
+      tmem_fence_after();
+      float v[kNPad];
+      tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kNPad), v);
+      tmem_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&aempty[b]);  // the MMA warp may reuse accumulator b
+#pragma unroll
+      for (int m = 0; m < M; ++m) outb[m * kTileN + q * 32 + lane] = v[m];
+      drain_sync();
+      const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
+      if (whole) {
+        gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
       } else {
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
-        for (int idx = tid; idx < M * kTileN; idx += kConsumerThreads) __stcg(dstp + idx, so[idx]);
+        for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) __stcg(dstp + idx, outb[idx]);
         __threadfence();
-        __syncthreads();
+        drain_sync();
         const int c_first = unit_owner(rt * p.n_kt, p.units, G);
         const int c_last = unit_owner(rt * p.n_kt + p.n_kt - 1, p.units, G);
-        if (tid == 0) {
+        if (dt == 0) {
           const unsigned prev = atomicAdd(&p.counters[rt], 1u);
           flag[0] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
         }
-        __syncthreads();
+        drain_sync();
         if (flag[0]) {
           __threadfence();
-          for (int idx = tid; idx < M * kTileN; idx += kConsumerThreads) {
+          for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) {
             float sum = 0.f;
             for (int cc = c_first; cc <= c_last; ++cc) {
               const int rt_cc = unit_begin(cc, p.units, G) / p.n_kt;
               const int sl = 2 * cc + (rt == rt_cc ? 0 : 1);
-              const float v = __ldcg(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN) + idx);
-              sum = (cc == c_first) ? v : sum + v;
+              const float pv = __ldcg(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN) + idx);
+              sum = (cc == c_first) ? pv : sum + pv;
             }
             outb[idx] = sum;
           }
-          __syncthreads();
-          gemv_epilogue<M, EPI>(p, rt, outb, rs, tid);
-          if (tid == 0) p.counters[rt] = 0u;
+          drain_sync();
+          gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
+          if (dt == 0) p.counters[rt] = 0u;
         }
       }
-      __syncthreads();
+      drain_sync();
+      seg_kt0 = 0;
+      ++sg;
     }
-    nseg = 0;
-  };
-
-  for (int i = 0; i < n_units; ++i) {
-    const int u = u0 + i;
-    const int rt = u / p.n_kt, kt = u - rt * p.n_kt;
-    const int s = i % kStages;
-    const uint32_t par = static_cast<uint32_t>(i / kStages) & 1u;
-    if (!mbar_wait(&full[s], par)) {
-      set_error(p.st, DERR_TIMEOUT);
-      return;  // every warp times out on the same stage
-    }
-    // weights: rows 4w + j (j < 4), columns 8*lane .. 8*lane+7 of the 32 x 256 unit
-    uint4 wv[4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) wv[j] = *reinterpret_cast<const uint4*>(wbase + s * kWTileBytes + j * (kTileK * 2));
-    float2 gs[4];
-    if (p.gain) {
-      const uint4 gv = *reinterpret_cast<const uint4*>(smem + S::kG + s * kTileK * 2 + lane * 16);
-      gs[0] = bf16x2_to_float2(gv.x);
-      gs[1] = bf16x2_to_float2(gv.y);
-      gs[2] = bf16x2_to_float2(gv.z);
-      gs[3] = bf16x2_to_float2(gv.w);
-    }
-    float2 w2[4][4];
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      w2[j][0] = bf16x2_to_float2(wv[j].x);
-      w2[j][1] = bf16x2_to_float2(wv[j].y);
-      w2[j][2] = bf16x2_to_float2(wv[j].z);
-      w2[j][3] = bf16x2_to_float2(wv[j].w);
-    }
-    const float* abase = reinterpret_cast<const float*>(smem + S::kA + s * S::kActBytes) + lane * 8;
-#pragma unroll
-    for (int m = 0; m < M; ++m) {
-      const float4 a0 = *reinterpret_cast<const float4*>(abase + m * kTileK);
-      const float4 a1 = *reinterpret_cast<const float4*>(abase + m * kTileK + 4);
-      float2 x2[4] = {make_float2(a0.x, a0.y), make_float2(a0.z, a0.w), make_float2(a1.x, a1.y),
-                      make_float2(a1.z, a1.w)};
-      if (p.gain) {
-#pragma unroll
-        for (int q = 0; q < 4; ++q) x2[q] = make_float2(x2[q].x * gs[q].x, x2[q].y * gs[q].y);
-      }
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-#pragma unroll
-        for (int q = 0; q < 4; ++q) acc[j][m] = __ffma2_rn(w2[j][q], x2[q], acc[j][m]);
-    }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&empty[s]);
-    if (tid == 0 && i + kStages < n_units) {
-      // refill this stage once every warp has released it
-      if (!mbar_wait(&empty[s], par)) {
-        set_error(p.st, DERR_TIMEOUT);
-      } else {
-        mbar_arrive_expect_tx(&full[s], tx);
-        issue_weights(s, u + kStages);
-        issue_acts(s, u + kStages);
-        if (p.pf_dist > 0 && i + kStages + p.pf_dist < n_units) prefetch_unit(u + kStages + p.pf_dist);
-      }
-    }
-
-    const bool seg_end = (kt == p.n_kt - 1) || (i == n_units - 1);
-    if (!seg_end) continue;
-
-    // ---- park this row-tile segment: reduce over the 32 column lanes (warp-local)
-    float* so = seg + nseg * (M * kTileN);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-#pragma unroll
-      for (int m = 0; m < M; ++m) {
-        float v = acc[j][m].x + acc[j][m].y;
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) v += __shfl_xor_sync(0xffffffffu, v, off);
-        if (lane == 0) so[m * kTileN + warp * 4 + j] = v;
-        acc[j][m] = make_float2(0.f, 0.f);
-      }
-    }
-    if (tid == 0) {
-      seg_rt[nseg] = rt;
-      seg_whole[nseg] = (seg_kt0 == 0) && (kt == p.n_kt - 1);
-    }
-    ++nseg;
-    seg_kt0 = 0;  // the next segment starts at a row-tile boundary
-    if (nseg == kMaxSeg && i + 1 < n_units) flush();
   }
-  flush();
+  tmem_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tmem_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
+  }
 }
 
 }  // namespace ssd

@@ -23,7 +23,7 @@ using namespace ssd;
 
 namespace {
 
-constexpr int kStaticMaxVocab = 262144;                   // vocab limit (8192 row tiles of 32)
+constexpr int kStaticMaxVocab = 262144;                   // vocab limit (2048 row tiles of 128)
 constexpr int kStaticMaxCtas = 320;                       // GEMV CTAs (2 per SM, up to 160 SMs)
 constexpr int kStaticMaxTiles = kStaticMaxVocab / kTileN;
 constexpr int kStaticMaxDevices = 64;
@@ -34,7 +34,7 @@ struct StaticScratch {
   float partials[2 * kStaticMaxCtas * kMaxRows * kTileN];  // partial sums of split row tiles
 };
 
-// About 1.3 MB of device memory per GPU, held from library load until exit.
+// About 5.3 MB of device memory per GPU, held from library load until exit.
 static __device__ __align__(256) StaticScratch g_head_scratch;
 
 struct DeviceSetup {
@@ -78,7 +78,7 @@ ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const
                               int d_model, float rms_eps, int32_t* tok, float* logits, void* cuda_stream) {
   if (!lm_head || !final_norm || !x || !tok) return SSD_ERR_INVALID_ARG;
   if (rows < 1 || rows > 9 || vocab < 1 || vocab > kStaticMaxVocab) return SSD_ERR_INVALID_ARG;
-  if (d_model < kTileK || d_model % kTileK != 0) return SSD_ERR_INVALID_ARG;  // 256-column slices stay in a row
+  if (d_model < kTileK || d_model % kTileK != 0) return SSD_ERR_INVALID_ARG;  // 64-column slices stay in a row
   const uintptr_t al = reinterpret_cast<uintptr_t>(lm_head) | reinterpret_cast<uintptr_t>(final_norm) |
                        reinterpret_cast<uintptr_t>(x);
   if (al % 16 != 0) return SSD_ERR_INVALID_ARG;
@@ -94,7 +94,7 @@ ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kTileK), static_cast<cuuint32_t>(kTileN)};
   cuuint32_t es[2] = {1, 1};
   if (g_encode_static(&maps[0], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(lm_head), dims, strides, box,
-                      es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                      es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                       CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
     return SSD_ERR_CUDA;
   maps[1] = maps[2] = maps[0];
