@@ -118,6 +118,7 @@ struct ssd_ctx {
   // step (ncu cannot profile kernels of graphs that hold conditional nodes).
   bool host_loop = false;
   int gemv_ctas = 2;  // GEMV CTAs per SM
+  int small_site_rt = 0, small_site_ctas = 2;  // sites with fewer row tiles than small_site_rt use small_site_ctas
   std::map<std::pair<int, int>, cudaGraphExec_t> prefill_graphs;
   cudaGraphExec_t greedy_graph = nullptr;
   std::map<int, int64_t> decode_body_launches;
@@ -217,7 +218,9 @@ static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nm
   s->n_rt = (s->N + kTileN - 1) / kTileN;
   s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
-  s->grid = s->units < c->num_sms * c->gemv_ctas ? s->units : c->num_sms * c->gemv_ctas;
+  // few row tiles: each would be split across many CTAs, so use fewer CTAs
+  const int ctas = (s->n_rt < c->small_site_rt) ? c->small_site_ctas : c->gemv_ctas;
+  s->grid = s->units < c->num_sms * ctas ? s->units : c->num_sms * ctas;
   return SSD_OK;
 }
 
@@ -761,8 +764,12 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   c->num_sms = prop.multiProcessorCount;
   if (const char* e = getenv("SSD_GEMV_PREFETCH")) c->pf_dist = atoi(e) < 0 ? 0 : atoi(e);
   if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
-  if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) == 2 ? 2 : 1;
+  if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) < 1 ? 1 : (atoi(e) > 3 ? 3 : atoi(e));
   if (const char* e = getenv("SSD_PREFILL")) c->prefill_rows = strcmp(e, "rows") == 0;
+  if (const char* e = getenv("SSD_GEMV_SMALL")) {  // "<row tiles>,<ctas per SM>"
+    c->small_site_rt = atoi(e);
+    if (const char* comma = strchr(e, ',')) c->small_site_ctas = atoi(comma + 1) < 1 ? 1 : atoi(comma + 1);
+  }
   if (!g_encode) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;

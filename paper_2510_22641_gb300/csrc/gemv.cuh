@@ -544,13 +544,24 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         drain_sync();
         if (flag[0]) {
           __threadfence();
+          // sum the partials in CTA order; the loads of 8 CTAs are issued together
+          const int nsp = c_last - c_first + 1;
           for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) {
             float sum = 0.f;
-            for (int cc = c_first; cc <= c_last; ++cc) {
-              const int rt_cc = unit_begin(cc, p.units, G) / p.n_kt;
-              const int sl = 2 * cc + (rt == rt_cc ? 0 : 1);
-              const float pv = __ldcg(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN) + idx);
-              sum = (cc == c_first) ? pv : sum + pv;
+            for (int b0 = 0; b0 < nsp; b0 += 8) {
+              float pv[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                const int cc = c_first + b0 + j;
+                pv[j] = 0.f;
+                if (b0 + j < nsp) {
+                  const int sl = 2 * cc + (rt == unit_begin(cc, p.units, G) / p.n_kt ? 0 : 1);
+                  pv[j] = __ldcg(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN) + idx);
+                }
+              }
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                if (b0 + j < nsp) sum = (b0 + j == 0) ? pv[j] : sum + pv[j];
             }
             outb[idx] = sum;
           }
