@@ -36,6 +36,10 @@ sys.path.insert(0, ROOT)
 import synth  # noqa: E402
 
 METRIC = "tokens/s and speedup vs full-model greedy decode (7B shape, bs1); HBM GB/s"
+
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up GEMV
+# launch from an ncu capture, valid only for the kernel source it was taken on.
+GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "13ba0173f9a35134", "bytes": 186_566_912}
 UNIT = "tokens/s"
 S_VALUES = synth.LLAVA7B_S_VALUES
 
@@ -61,6 +65,39 @@ def algorithmic_bytes(w: synth.Workload) -> dict:
     return {"layer": layer, "head": head, "imit": imit, "kv_pos_layer": kv_pos,
             "draft_token": w.draft_exit_k * layer + imit + head,
             "verify": sh.n_layers * layer + head, "greedy_token": sh.n_layers * layer + head}
+
+
+def gemv_traffic_bytes():
+    """Measured bytes per launch if gemv.cuh is the captured version, else None."""
+    import hashlib
+    src = os.path.join(ROOT, "paper_2510_22641_gb300", "csrc", "gemv.cuh")
+    try:
+        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    return GEMV_TRAFFIC["bytes"] if digest.startswith(GEMV_TRAFFIC["gemv_cuh_sha256_prefix"]) else None
+
+
+def prefill_flops(w: synth.Workload) -> float:
+    """Tensor-core work of one prefill: 2 flops per weight per row, times 2 for the bf16 hi/lo activation parts."""
+    sh = w.shape
+    params = 4 * sh.d_model * sh.qdim + 3 * sh.d_model * sh.d_ff
+    return 2.0 * 2.0 * w.prompt_len * params * sh.n_layers
+
+
+def reduce_max(value: float, dist=None, device=None) -> float:
+    """Max over ranks (the slowest rank defines the whole job's time)."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return value
+    import torch
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_tokens_per_s(world: int, steps: int, tokens_per_step: int, max_ms: float) -> float:
+    """Weak scaling: every rank generates `steps` requests; the job lasts as long as the slowest rank."""
+    return world * steps * tokens_per_step / (max_ms / 1e3)
 
 
 # --------------------------------------------------------------------------- clocks
@@ -233,11 +270,8 @@ def main() -> None:
     assert int(n_out.item()) == w.max_new
     st = model.stats()
     pre_l, dec_l = model.launch_counts()
-    if world > 1:
-        t = torch.tensor([total_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
-    value = world * args.steps * w.max_new / (total_ms / 1e3)
+    total_ms = reduce_max(total_ms, dist if world > 1 else None, device="cuda")
+    value = whole_job_tokens_per_s(world, args.steps, w.max_new, total_ms)
 
     # ---------------- end to end through ssd_generate with pinned host buffers
     vis_h = torch.from_numpy(vis.view(np.int16)).pin_memory()
@@ -299,7 +333,7 @@ def main() -> None:
     kern_ms = k0.elapsed_time(k1) / reps
     achieved = nbytes / (kern_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
-                "frac": achieved / hbm_peak, "traffic": None,
+                "frac": achieved / hbm_peak, "traffic": gemv_traffic_bytes(),
                 "kernel": "gemv_kernel<1, GATE_SILU> (layer gate/up, 2x11008x4096 bf16, 1 row)",
                 "bytes_per_launch": nbytes, "launch_us": kern_ms * 1e3,
                 "peak_source": f"{peak_src} HBM copy (burst)"}
@@ -322,6 +356,13 @@ def main() -> None:
             "e2e": e2e, "gpu_launches": int(args.steps * (pre_l + dec_l)),
             "roofline": roofline, "clocks": clk,
             "prefill_ms": statistics.median(prefill_ms), "decode_ms": dec_ms,
+            "prefill_roofline": {"bound": "tensor", "kernel": "tc_gemm_kernel (all prefill projections) + prefill attention",
+                                 "achieved": prefill_flops(w) / (statistics.median(prefill_ms) / 1e3) / 1e12,
+                                 "peak": float(peaks.get("bf16_tflops", 1900.0)), "unit": "TFLOP/s",
+                                 "frac": prefill_flops(w) / (statistics.median(prefill_ms) / 1e3) / 1e12
+                                 / float(peaks.get("bf16_tflops", 1900.0)),
+                                 "note": "whole-prefill time incl. attention and activation splits; "
+                                         "flops counted as issued (bf16 hi + lo parts)"},
             "decode_tokens_per_s": (w.max_new - 1) / (dec_ms / 1e3),
             "decode_hbm_gbs": dec_bytes / (dec_ms / 1e3) / 1e9,
             "decode_hbm_frac": dec_bytes / (dec_ms / 1e3) / 1e9 / hbm_peak,
