@@ -190,6 +190,89 @@ def run_reference(args) -> None:
 
 # --------------------------------------------------------------------------- GPU arm
 
+def run_sweep(args) -> None:
+    """Sweep k x gamma x s on the 7B shape (256 new tokens): accept length, tokens/s, speedup
+    over greedy, draft and verify HBM GB/s.  One JSON line per point."""
+    import torch
+
+    import paper_2510_22641_gb300 as lib
+    lib.build()
+    base = synth.LLAVA7B.replace(max_new=256)
+    bits = synth.make_weights(base)
+    up = lib.bf16_bits_to_device
+    dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm", "in_norm", "in_w1", "in_w2")}
+    dev["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+    vis, prompt = synth.make_inputs(base)
+    v = up(vis)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    stream = torch.cuda.current_stream()
+    rs = torch.tensor(base.resid_scale(), device="cuda")
+    ins = torch.tensor([base.in_scale()], device="cuda")
+
+    def ev():
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(stream)
+        return e
+
+    greedy_tok_s = {}
+    for k in (4, 8, 12, 16):
+        w0 = base.replace(draft_exit_k=k)
+        cfg = lib.config_dict(w0.shape, k, w0.in_kind, w0.in_hidden, lib.SSD_MAX_GAMMA,
+                              w0.prompt_len + w0.max_new + lib.SSD_MAX_GAMMA + 1)
+        model = lib.SSDModel(cfg, dev, rs, ins)
+        ab = algorithmic_bytes(w0)
+        for s_val in S_VALUES:
+            w = w0.replace(s=s_val)
+            rs.copy_(torch.tensor(w.resid_scale(), device="cuda"))
+            ins.copy_(torch.tensor([w.in_scale()], device="cuda"))
+            if s_val not in greedy_tok_s:
+                model.prefill(v, p)
+                model.greedy_decode(w.max_new)
+                model.prefill(v, p)
+                a = ev()
+                model.greedy_decode(w.max_new)
+                b = ev()
+                torch.cuda.synchronize()
+                greedy_tok_s[s_val] = (w.max_new - 1) / (a.elapsed_time(b) / 1e3)
+            for gamma in (2, 3, 4, 5, 6, 8):
+                model.prefill(v, p)
+                model.decode(w.max_new, gamma)          # warm-up and graph build
+                model.prefill(v, p)
+                a = ev()
+                model.decode(w.max_new, gamma)
+                b = ev()
+                torch.cuda.synchronize()
+                st = model.stats()
+                dec_ms = a.elapsed_time(b)
+                # draft / verify stages timed separately over a few steps
+                model.prefill(v, p)
+                model.draft(gamma)
+                model.verify(gamma)
+                d_ms, v_ms, n = 0.0, 0.0, 6
+                for _ in range(n):
+                    e0 = ev()
+                    model.draft(gamma)
+                    e1 = ev()
+                    model.verify(gamma)
+                    e2 = ev()
+                    torch.cuda.synchronize()
+                    d_ms += e0.elapsed_time(e1)
+                    v_ms += e1.elapsed_time(e2)
+                S = w.prompt_len + w.max_new // 2
+                draft_bytes = gamma * (ab["draft_token"] + ab["kv_pos_layer"] * k * S)
+                verify_bytes = ab["verify"] + ab["kv_pos_layer"] * w.shape.n_layers * S
+                tok_s = (w.max_new - 1) / (dec_ms / 1e3)
+                print(json.dumps({"k": k, "gamma": gamma, "s": s_val, "steps": st["steps"],
+                                  "mean_accept": st["accepted"] / max(st["steps"], 1),
+                                  "tokens_per_step": (w.max_new - 1) / max(st["steps"], 1),
+                                  "ssd_tok_s": tok_s, "greedy_tok_s": greedy_tok_s[s_val],
+                                  "speedup": tok_s / greedy_tok_s[s_val],
+                                  "draft_ms": d_ms / n, "verify_ms": v_ms / n,
+                                  "draft_gbs": draft_bytes / (d_ms / n / 1e3) / 1e9,
+                                  "verify_gbs": verify_bytes / (v_ms / n / 1e3) / 1e9}), flush=True)
+        model.close()
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -199,7 +282,11 @@ def main() -> None:
     ap.add_argument("--s", type=float, default=0.2, help="deep-layer residual scale of the headline run")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=3, help="oracle SSD steps in the CPU sample")
+    ap.add_argument("--sweep", action="store_true", help="k x gamma x s sweep (one JSON line per point)")
     args = ap.parse_args()
+    if args.sweep:
+        run_sweep(args)
+        return
     if args.impl == "reference":
         run_reference(args)
         return

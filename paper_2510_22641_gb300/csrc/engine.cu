@@ -23,6 +23,7 @@
 #include "attention.cuh"
 #include "control.cuh"
 #include "gemv.cuh"
+#include "fwd_params.cuh"
 #include "prefill_params.cuh"
 
 namespace ssd {
@@ -44,6 +45,9 @@ cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bf
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
                                 float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
                                 cudaStream_t s, bool pdl);
+cudaError_t fwd_attrs();
+cudaError_t fwd_ctas_per_sm(int head_dim, int* n);
+cudaError_t fwd_launch(int head_dim, const FwdParams& p, int grid, cudaStream_t stream, bool cooperative);
 }  // namespace ssd
 
 using namespace ssd;
@@ -76,6 +80,12 @@ struct TcLayer {
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 }  // namespace
+
+// One phase list of the persistent forward kernel, stored in ssd_ctx::fwd_phases.
+struct FwdProg {
+  size_t off = 0;
+  int n_phases = 0, n_flags = 0;
+};
 
 struct ssd_ctx {
   ssd_config cfg{};
@@ -133,6 +143,24 @@ struct ssd_ctx {
   int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy
   int last_gamma = 0;
   std::pair<int, int> last_prefill_shape{0, 0};
+  // persistent forward kernel (decode): phase lists, map table, flags and scratch
+  bool use_fwd = false;  // SSD_DECODE=fwd: one persistent launch per forward pass
+  bool fwd_coop = true;  // cooperative launch (every CTA resident)
+  bool fwd_ready = false;
+  int fwd_grid = 0, fwd_splits = 1;
+  FwdProg fwd_greedy;
+  std::vector<FwdProg> fwd_draft, fwd_verify;  // indexed by gamma
+  FwdPhase* fwd_phases = nullptr;
+  size_t fwd_phases_cap = 0;
+  CUtensorMap* fwd_maps = nullptr;
+  unsigned *fwd_flags = nullptr, *fwd_tickets = nullptr, *fwd_done = nullptr, *fwd_exit = nullptr;
+  int fwd_flags_cap = 0, fwd_done_cap = 0;
+  float *fwd_partials = nullptr, *fwd_attn_part = nullptr;
+  uint8_t* fwd_btiles = nullptr;  // [kFwdBSlots][fwd_bslot] B operands written by producer epilogues
+  long long fwd_bslot = 0;
+  unsigned long long* fwd_trace = nullptr;  // SSD_FWD_TRACE=<file>: timeline of the last launch
+  std::string fwd_trace_path;
+  int fwd_trace_phases = 0;
   // debug logits capture
   float* logits_buf = nullptr;
   int logits_rows = 0;
@@ -388,8 +416,364 @@ static int* st_field(ssd_ctx* c, size_t off) {
   return reinterpret_cast<int*>(reinterpret_cast<char*>(c->st) + off);
 }
 
+// ------------------------------------------------------------------ persistent forward kernel
+
+static ssd_status fwd_alloc(ssd_ctx* c, void** p, size_t bytes) {
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaSuccess) e = cudaMemset(*p, 0, bytes);
+  if (e != cudaSuccess) {
+    *p = nullptr;
+    return fail(c, SSD_ERR_OOM, "forward-kernel scratch (%zu bytes): %s", bytes, cudaGetErrorString(e));
+  }
+  return SSD_OK;
+}
+
+// Map table: layer l -> [7l] q, k, v, [7l+3] o, [7l+4] gate, [7l+5] up, [7l+6] down;
+// then imitation FC1, FC2 and the LM head.
+static int map_in1(const ssd_ctx* c) { return 7 * c->cfg.n_layers; }
+static int map_in2(const ssd_ctx* c) { return 7 * c->cfg.n_layers + 1; }
+static int map_head(const ssd_ctx* c) { return 7 * c->cfg.n_layers + 2; }
+
+struct FwdBuilder {
+  ssd_ctx* c;
+  std::vector<FwdPhase> ph;
+  int flags = 0;
+  int add(FwdPhase f) {
+    f.flags = flags;
+    f.bt_off = -1;
+    f.bt_dst_off = -1;
+    flags += f.n_tiles;
+    ph.push_back(f);
+    return static_cast<int>(ph.size()) - 1;
+  }
+  // columns of phase q's output per tile (what a consumer's 64-column slice maps to)
+  int out_cols(int q) const {
+    if (q < 0) return kTileN;
+    const int k = ph[q].kind;
+    if (k == FK_GATE_SILU) return kHalfN;
+    if (k == FK_ATTN) return c->cfg.head_dim;
+    return kTileN;
+  }
+};
+
+static FwdPhase fwd_gemv(const Site& s, int kind, int M, int map0, int map1, int map2) {
+  FwdPhase f{};
+  f.kind = kind;
+  f.M = M;
+  f.K = s.K;
+  f.N = s.N;
+  f.n_kt = s.n_kt;
+  f.n_rt = s.n_rt;
+  f.units = s.units;
+  f.seg_rows = s.seg_rows;
+  f.map0 = map0;
+  f.map1 = map1;
+  f.map2 = map2;
+  f.n_tiles = s.n_rt;
+  f.dep = f.epi_dep = -1;
+  return f;
+}
+
+// x[row0 .. row0+M-1] = E[tok_src[0 .. M-1]]; tok_src is final once phase tok_dep is complete.
+static int fwd_add_embed(FwdBuilder& b, const int* tok_src, int row0, int M, int tok_dep) {
+  ssd_ctx* c = b.c;
+  FwdPhase f{};
+  f.kind = FK_EMBED;
+  f.M = M;
+  f.tok_src = tok_src;
+  f.dst = c->xv + static_cast<size_t>(row0) * c->dp;
+  f.dst_stride = c->dp;
+  f.n_tiles = (c->dp + kTileN - 1) / kTileN;
+  f.dep = -1;
+  f.epi_dep = tok_dep;
+  return b.add(f);
+}
+
+// Decoder layer l on rows x[0 .. M-1] (stride dp) at positions kv_len + pos_off + m;
+// x is final once phase xdep is complete.  Returns the phase that completes x_{l+1}.
+static int fwd_add_layer(FwdBuilder& b, int l, float* x, int M, int pos_off, int xdep) {
+  ssd_ctx* c = b.c;
+  const LayerSites& L = c->layers[l];
+  const int m0 = 7 * l;
+  FwdPhase f = fwd_gemv(L.qkv, FK_QKV, M, m0, m0 + 1, m0 + 2);
+  f.x = x;
+  f.x_stride = c->dp;
+  f.gain = c->attn_norm[l];
+  f.dep = xdep;
+  f.dep_cols = b.out_cols(xdep);
+  f.epi_dep = xdep;
+  f.pos_off = pos_off;
+  f.q_out = c->qb;
+  f.q_stride = c->qp;
+  f.k_cache = c->kc + l * c->layer_kv;
+  f.v_cache = c->vc + l * c->layer_kv;
+  const int qkv = b.add(f);
+
+  f = FwdPhase{};
+  f.kind = FK_ATTN;
+  f.M = M;
+  f.x = c->qb;
+  f.x_stride = c->qp;
+  f.dst = c->ob;
+  f.dst_stride = c->qp;
+  f.k_cache = c->kc + l * c->layer_kv;
+  f.v_cache = c->vc + l * c->layer_kv;
+  f.pos_off = pos_off;
+  f.dep = qkv;
+  f.epi_dep = -1;
+  f.n_tiles = c->cfg.n_heads;
+  const int attn = b.add(f);
+
+  f = fwd_gemv(L.o, FK_RESID, M, m0 + 3, m0 + 3, m0 + 3);
+  f.x = c->ob;
+  f.x_stride = c->qp;
+  f.dep = attn;
+  f.dep_cols = b.out_cols(attn);
+  f.epi_dep = xdep;  // base rows x
+  f.base = x;
+  f.base_stride = c->dp;
+  f.dst = x;
+  f.dst_stride = c->dp;
+  f.scale = c->resid_scale + l;
+  const int o = b.add(f);
+
+  f = fwd_gemv(L.gateup, FK_GATE_SILU, M, m0 + 4, m0 + 5, m0 + 4);
+  f.x = x;
+  f.x_stride = c->dp;
+  f.gain = c->ffn_norm[l];
+  f.dep = o;
+  f.dep_cols = b.out_cols(o);
+  f.epi_dep = o;
+  f.h_out = c->hb;
+  f.h_stride = c->fp;
+  const int gu = b.add(f);
+
+  f = fwd_gemv(L.down, FK_RESID, M, m0 + 6, m0 + 6, m0 + 6);
+  f.x = c->hb;
+  f.x_stride = c->fp;
+  f.dep = gu;
+  f.dep_cols = b.out_cols(gu);
+  f.epi_dep = o;  // base rows x
+  f.base = x;
+  f.base_stride = c->dp;
+  f.dst = x;
+  f.dst_stride = c->dp;
+  f.scale = c->resid_scale + l;
+  return b.add(f);
+}
+
+// g(x) = W_lm RMSNorm_f(x) + argmax on rows x[0 .. M-1].
+static int fwd_add_head(FwdBuilder& b, const float* x, int M, int pos_off, int* tok_dst, bool capture, int xdep) {
+  ssd_ctx* c = b.c;
+  FwdPhase f = fwd_gemv(c->head, FK_ARGMAX, M, map_head(c), map_head(c), map_head(c));
+  f.x = x;
+  f.x_stride = c->dp;
+  f.gain = c->final_norm;
+  f.dep = xdep;
+  f.dep_cols = b.out_cols(xdep);
+  f.epi_dep = xdep;
+  f.pos_off = pos_off;
+  f.tok_dst = tok_dst;
+  f.logits = capture ? c->logits_buf : nullptr;
+  f.logits_rows = capture ? c->logits_rows : 0;
+  return b.add(f);
+}
+
+// Imitation network on row x (M = 1): xt = x + s_in * W2 SiLU(W1 RMSNorm_in(x)).
+static int fwd_add_in(FwdBuilder& b, float* x, int xdep) {
+  ssd_ctx* c = b.c;
+  FwdPhase f = fwd_gemv(c->in1, FK_SILU, 1, map_in1(c), map_in1(c), map_in1(c));
+  f.x = x;
+  f.x_stride = c->dp;
+  f.gain = c->in_norm;
+  f.dep = xdep;
+  f.dep_cols = b.out_cols(xdep);
+  f.epi_dep = xdep;
+  f.h_out = c->hin;
+  f.h_stride = c->ip;
+  const int s1 = b.add(f);
+  f = fwd_gemv(c->in2, FK_RESID, 1, map_in2(c), map_in2(c), map_in2(c));
+  f.x = c->hin;
+  f.x_stride = c->ip;
+  f.dep = s1;
+  f.dep_cols = b.out_cols(s1);
+  f.epi_dep = xdep;  // base row x
+  f.base = x;
+  f.base_stride = c->dp;
+  f.dst = c->xt;
+  f.dst_stride = c->dp;
+  f.scale = c->in_scale;
+  return b.add(f);
+}
+
+// The projection q reads the B operands of its 64-column slices from slot q mod kFwdBSlots
+// of the B-operand ring; its producer -- always phase q - 1, so that the drain warps'
+// wait on phase q - 1 - window keeps a slot from being rewritten while it is read --
+// writes them in its epilogue.
+static bool fwd_link_operands(ssd_ctx* c, FwdBuilder& b) {
+  auto out_ptr = [](const FwdPhase& f) -> const float* {
+    return (f.kind == FK_GATE_SILU || f.kind == FK_SILU) ? f.h_out : f.dst;
+  };
+  for (int q = 0; q < static_cast<int>(b.ph.size()); ++q) {
+    FwdPhase& f = b.ph[q];
+    if (f.kind > FK_ARGMAX) continue;
+    const int pq = f.dep;
+    if (pq != q - 1) return false;
+    FwdPhase& pr = b.ph[pq];
+    if (pr.bt_dst_off >= 0 || pr.kind == FK_QKV || pr.kind == FK_ARGMAX) return false;
+    const ptrdiff_t d = out_ptr(pr) - f.x;
+    if (d < 0 || d % f.x_stride != 0) return false;
+    const int row0 = static_cast<int>(d / f.x_stride);
+    if (row0 + pr.M > f.M) return false;
+    f.bt_off = static_cast<long long>(q % kFwdBSlots) * c->fwd_bslot;
+    pr.bt_dst_off = f.bt_off;
+    pr.bt_x = f.x;
+    pr.bt_x_stride = f.x_stride;
+    pr.bt_M = f.M;
+    pr.bt_nkt = f.n_kt;
+    pr.bt_row0 = row0;
+    pr.bt_gain = f.gain;
+  }
+  return true;
+}
+
+static FwdProg fwd_commit(FwdBuilder& b, std::vector<FwdPhase>& all) {
+  if (!fwd_link_operands(b.c, b)) {
+    FwdProg bad;
+    bad.n_phases = -1;
+    return bad;
+  }
+  FwdProg pr;
+  pr.off = all.size();
+  pr.n_phases = static_cast<int>(b.ph.size());
+  pr.n_flags = b.flags;
+  all.insert(all.end(), b.ph.begin(), b.ph.end());
+  return pr;
+}
+
+static int* st_field_early(ssd_ctx* c, size_t off) {
+  return reinterpret_cast<int*>(reinterpret_cast<char*>(c->st) + off);
+}
+
+// Phase lists of the greedy step and, per gamma, of the drafting and verification stages.
+static ssd_status fwd_build_programs(ssd_ctx* c) {
+  const int K = c->cfg.draft_exit_k, Lc = c->cfg.n_layers, d = c->dp;
+  int* tok_in = st_field_early(c, offsetof(DevState, tok_in));
+  int* full_tok = st_field_early(c, offsetof(DevState, full_tok));
+  std::vector<FwdPhase> all;
+  {
+    FwdBuilder b{c};
+    int last = fwd_add_embed(b, tok_in, 0, 1, -1);
+    for (int l = 0; l < Lc; ++l) last = fwd_add_layer(b, l, c->xv, 1, 0, last);
+    fwd_add_head(b, c->xv, 1, 0, full_tok, true, last);
+    c->fwd_greedy = fwd_commit(b, all);
+  }
+  c->fwd_draft.assign(c->cfg.gamma_max + 1, FwdProg{});
+  c->fwd_verify.assign(c->cfg.gamma_max + 1, FwdProg{});
+  for (int g = 1; g <= c->cfg.gamma_max; ++g) {
+    FwdBuilder b{c};
+    int head = -1;
+    for (int j = 0; j < g; ++j) {
+      float* xj = c->xv + static_cast<size_t>(j) * d;
+      int last = fwd_add_embed(b, tok_in + j, j, 1, head);
+      for (int l = 0; l < K; ++l) last = fwd_add_layer(b, l, xj, 1, j, last);
+      const float* hx = xj;
+      if (c->cfg.in_kind == SSD_IN_MLP2) {
+        last = fwd_add_in(b, xj, last);
+        hx = c->xt;
+      }
+      head = fwd_add_head(b, hx, 1, j, tok_in + j + 1, false, last);
+    }
+    c->fwd_draft[g] = fwd_commit(b, all);
+    FwdBuilder v{c};
+    int last = fwd_add_embed(v, tok_in + g, g, 1, -1);
+    float* xg = c->xv + static_cast<size_t>(g) * d;
+    for (int l = 0; l < K; ++l) last = fwd_add_layer(v, l, xg, 1, g, last);
+    for (int l = K; l < Lc; ++l) last = fwd_add_layer(v, l, c->xv, g + 1, 0, last);
+    fwd_add_head(v, c->xv, g + 1, 0, full_tok, true, last);
+    c->fwd_verify[g] = fwd_commit(v, all);
+  }
+  bool linked = c->fwd_greedy.n_phases > 0;
+  for (int g = 1; g <= c->cfg.gamma_max; ++g) linked = linked && c->fwd_draft[g].n_phases > 0 && c->fwd_verify[g].n_phases > 0;
+  if (!linked) return fail(c, SSD_ERR_STATE, "forward-kernel phase list: a projection does not read its predecessor");
+  int max_flags = std::max(1, c->fwd_greedy.n_flags), max_phases = std::max(1, c->fwd_greedy.n_phases);
+  for (int g = 1; g <= c->cfg.gamma_max; ++g)
+    for (const FwdProg* pr : {&c->fwd_draft[g], &c->fwd_verify[g]}) {
+      max_flags = std::max(max_flags, pr->n_flags);
+      max_phases = std::max(max_phases, pr->n_phases);
+    }
+  if (all.size() > c->fwd_phases_cap) {
+    if (c->fwd_phases) cudaFree(c->fwd_phases);
+    c->fwd_phases = nullptr;
+    c->fwd_phases_cap = 0;
+    CK(cudaMalloc(&c->fwd_phases, sizeof(FwdPhase) * all.size()));
+    c->fwd_phases_cap = all.size();
+  }
+  CK(cudaMemcpy(c->fwd_phases, all.data(), sizeof(FwdPhase) * all.size(), cudaMemcpyHostToDevice));
+  if (max_flags > c->fwd_flags_cap) {
+    for (unsigned** b : {&c->fwd_flags, &c->fwd_tickets}) {
+      if (*b) cudaFree(*b);
+      *b = nullptr;
+    }
+    c->fwd_flags_cap = 0;
+    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_flags), sizeof(unsigned) * max_flags));
+    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_tickets), sizeof(unsigned) * max_flags));
+    c->fwd_flags_cap = max_flags;
+  }
+  if (max_phases > c->fwd_done_cap) {
+    if (c->fwd_done) cudaFree(c->fwd_done);
+    c->fwd_done = nullptr;
+    c->fwd_done_cap = 0;
+    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_done), sizeof(unsigned) * max_phases));
+    c->fwd_done_cap = max_phases;
+  }
+  if (!c->fwd_trace_path.empty() && !c->fwd_trace) {
+    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_trace),
+                  sizeof(unsigned long long) * (c->fwd_grid * (max_phases + 1) * 16 + 4 * 8192 * 4)));
+  }
+  c->fwd_ready = true;
+  return SSD_OK;
+}
+
+static ssd_status fwd_run(ssd_ctx* c, const FwdProg& pr) {
+  FwdParams p{};
+  p.phases = c->fwd_phases + pr.off;
+  p.n_phases = pr.n_phases;
+  p.maps = c->fwd_maps;
+  p.st = c->st;
+  p.flags = c->fwd_flags;
+  p.tickets = c->fwd_tickets;
+  p.done = c->fwd_done;
+  p.exit_count = c->fwd_exit;
+  p.btiles = c->fwd_btiles;
+  p.n_flags = pr.n_flags;
+  p.partials = c->fwd_partials;
+  p.attn_part = c->fwd_attn_part;
+  p.n_heads = c->cfg.n_heads;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  p.splits = c->fwd_splits;
+  p.attn_scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
+  p.eps = c->cfg.rms_eps;
+  p.rope = c->rope;
+  p.embed = c->embed;
+  p.vocab = c->cfg.vocab;
+  p.d_model = c->cfg.d_model;
+  p.trace = c->fwd_trace;
+  c->fwd_trace_phases = pr.n_phases;
+  ++c->launch_counter;
+  CK(fwd_launch(c->cfg.head_dim, p, c->fwd_grid, c->cs, c->fwd_coop));
+  return SSD_OK;
+}
+
+static ssd_status fwd_ensure(ssd_ctx* c) {
+  if (!c->use_fwd || c->fwd_ready) return SSD_OK;
+  return fwd_build_programs(c);
+}
+
 // Drafting stage: gamma tokens from layers 0..k-1, the imitation network and g.
 static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
+  if (c->use_fwd) return fwd_run(c, c->fwd_draft[gamma]);
   const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   for (int j = 0; j < gamma; ++j) {
@@ -429,6 +813,12 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
   const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  if (c->use_fwd) {
+    CKS(fwd_run(c, c->fwd_verify[gamma]));
+    CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, cond,
+                has_cond));
+    return SSD_OK;
+  }
   CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
               c->xv + static_cast<size_t>(gamma) * d, d, c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, gamma, 1, gamma));
@@ -442,6 +832,12 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
 static ssd_status enqueue_greedy_step(ssd_ctx* c, cudaGraphConditionalHandle cond, int has_cond) {
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  if (c->use_fwd) {
+    CKS(fwd_run(c, c->fwd_greedy));
+    CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond,
+                has_cond));
+    return SSD_OK;
+  }
   CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv, c->dp,
               c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
@@ -648,6 +1044,7 @@ static ssd_status enq_step_fn(ssd_ctx* c, int g, int) {
 }
 
 static void drop_graphs(ssd_ctx* c) {
+  c->fwd_ready = false;  // phase lists hold the logits-capture pointer
   for (auto& kv : c->decode_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->draft_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->verify_graphs) cudaGraphExecDestroy(kv.second);
@@ -720,7 +1117,8 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
   void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
-                  c->partials, c->counters, c->in_vis, c->in_prompt};
+                  c->partials, c->counters, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
+                  c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles};
   for (void* b : bufs)
     if (b) cudaFree(b);
   if (c->ev_in) cudaEventDestroy(c->ev_in);
@@ -766,6 +1164,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
   if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) < 1 ? 1 : (atoi(e) > 3 ? 3 : atoi(e));
   if (const char* e = getenv("SSD_PREFILL")) c->prefill_rows = strcmp(e, "rows") == 0;
+  if (const char* e = getenv("SSD_DECODE")) c->use_fwd = strcmp(e, "fwd") == 0;
+  if (const char* e = getenv("SSD_FWD_COOP")) c->fwd_coop = atoi(e) != 0;
+  if (const char* e = getenv("SSD_FWD_TRACE")) c->fwd_trace_path = e;
   if (const char* e = getenv("SSD_GEMV_SMALL")) {  // "<row tiles>,<ctas per SM>"
     c->small_site_rt = atoi(e);
     if (const char* comma = strchr(e, ',')) c->small_site_ctas = atoi(comma + 1) < 1 ? 1 : atoi(comma + 1);
@@ -784,6 +1185,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_head());
   CK(attn_attrs());
   CK(prefill_attrs());
+  CK(fwd_attrs());
 
   c->cfg = k;
   c->qdim = qdim;
@@ -902,6 +1304,39 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     }
   }
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * k.max_seq));
+  {
+    // persistent forward kernel: one CTA per SM, the weight maps of every projection in one table
+    int per_sm = 0;
+    CK(fwd_ctas_per_sm(k.head_dim, &per_sm));
+    if (per_sm < 1) return fail(c, SSD_ERR_UNSUPPORTED, "forward kernel does not fit on an SM");
+    c->fwd_grid = c->num_sms;
+    c->fwd_splits = std::max(1, std::min(kFwdMaxSplits, c->fwd_grid / k.n_heads));
+    std::vector<CUtensorMap> maps;
+    for (int l = 0; l < k.n_layers; ++l) {
+      const LayerSites& L = c->layers[l];
+      for (int i = 0; i < 3; ++i) maps.push_back(L.qkv.maps[i]);
+      maps.push_back(L.o.maps[0]);
+      maps.push_back(L.gateup.maps[0]);
+      maps.push_back(L.gateup.maps[1]);
+      maps.push_back(L.down.maps[0]);
+    }
+    maps.push_back(c->in1.maps[0]);
+    maps.push_back(c->in2.maps[0]);
+    maps.push_back(c->head.maps[0]);
+    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_maps), sizeof(CUtensorMap) * maps.size()));
+    CK(cudaMemcpy(c->fwd_maps, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_exit), sizeof(unsigned)));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_partials),
+              sizeof(float) * kFwdWindow * 2 * c->fwd_grid * kFwdRows * kTileN));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_attn_part),
+              sizeof(float) * kFwdWindow * k.n_heads * c->fwd_splits * kFwdRows * (k.head_dim + 2)));
+    int max_kt = c->head.n_kt;
+    for (const Site* st : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->in1,
+                           &c->in2})
+      max_kt = std::max(max_kt, st->n_kt);
+    c->fwd_bslot = static_cast<long long>(max_kt) * kFwdBTile;
+    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_btiles), static_cast<size_t>(kFwdBSlots) * c->fwd_bslot));
+  }
   CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->ev_in, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&c->ev_out, cudaEventDisableTiming));
@@ -978,6 +1413,7 @@ ssd_status ssd_draft(ssd_ctx* c, int gamma, int32_t* draft_tok) {
   if (!c->prefilled) return fail(c, SSD_ERR_STATE, "ssd_draft before ssd_prefill");
   if (gamma < 1 || gamma > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma %d", gamma);
   if (c->kv_upper + gamma + 1 > c->cfg.max_seq) return fail(c, SSD_ERR_CAPACITY, "KV cache full");
+  CKS(fwd_ensure(c));
   CKS(enter(c));
   auto it = c->draft_graphs.find(gamma);
   if (it == c->draft_graphs.end()) {
@@ -996,6 +1432,7 @@ ssd_status ssd_verify(ssd_ctx* c, int gamma, int32_t* n_emitted, int32_t* emitte
   if (!c) return SSD_ERR_INVALID_ARG;
   if (!c->prefilled || c->drafted_gamma != gamma)
     return fail(c, SSD_ERR_STATE, "ssd_verify(gamma=%d) needs a preceding ssd_draft with the same gamma", gamma);
+  CKS(fwd_ensure(c));
   CKS(enter(c));
   auto it = c->verify_graphs.find(gamma);
   if (it == c->verify_graphs.end()) {
@@ -1018,6 +1455,7 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
   if (static_cast<int64_t>(c->prompt_len) + max_new + gamma + 1 > c->cfg.max_seq)
     return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 = %d > max_seq = %d",
                 c->prompt_len + max_new + gamma + 1, c->cfg.max_seq);
+  CKS(fwd_ensure(c));
   cudaGraphExec_t ge;
   if (c->host_loop) {
     auto it = c->step_graphs.find(gamma);
@@ -1088,6 +1526,17 @@ ssd_status ssd_sync(ssd_ctx* c) {
   if (!c) return SSD_ERR_INVALID_ARG;
   CK(cudaStreamSynchronize(c->cs));
   CK(cudaStreamSynchronize(c->us));
+  if (c->fwd_trace && c->fwd_trace_phases > 0) {  // diagnostic timeline of the last forward launch
+    const size_t n = static_cast<size_t>(c->fwd_grid) * (c->fwd_trace_phases + 1) * 16 + 4 * 8192 * 4;
+    std::vector<unsigned long long> h(n);
+    CK(cudaMemcpy(h.data(), c->fwd_trace, sizeof(unsigned long long) * n, cudaMemcpyDeviceToHost));
+    if (FILE* f = fopen(c->fwd_trace_path.c_str(), "wb")) {
+      const int hdr[2] = {c->fwd_grid, c->fwd_trace_phases};
+      fwrite(hdr, sizeof(int), 2, f);
+      fwrite(h.data(), sizeof(unsigned long long), n, f);
+      fclose(f);
+    }
+  }
   return read_device_error(c);
 }
 
