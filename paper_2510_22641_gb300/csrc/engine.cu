@@ -1327,9 +1327,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     CK(cudaMemcpy(c->fwd_maps, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
     CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_exit), sizeof(unsigned)));
     CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_partials),
-              sizeof(float) * kFwdWindow * 2 * c->fwd_grid * kFwdRows * kTileN));
+              sizeof(float) * kFwdWindow * c->fwd_grid * kFwdRows * kTileN));
     CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_attn_part),
-              sizeof(float) * kFwdWindow * k.n_heads * c->fwd_splits * kFwdRows * (k.head_dim + 2)));
+              sizeof(float) * kFwdWindow * k.n_heads * 4 * c->fwd_splits * kFwdRows * (k.head_dim + 2)));
     int max_kt = c->head.n_kt;
     for (const Site* st : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->in1,
                            &c->in2})

@@ -67,8 +67,8 @@ struct FwdSmem {
   static constexpr int kOut = kB + kFwdStages * kFwdBTile;                 // [rows][128] drained / final row tile
   static constexpr int kQ = kOut + kFwdRows * kTileN * 4;                   // [rows][DH] queries
   static constexpr int kS = kQ + kFwdRows * DH * 4;                         // [rows][KPC] scores / probabilities
-  static constexpr int kGen = kS + kFwdRows * kKPC * 4;                     // one K or V chunk read with plain loads
-  static constexpr int kRs = kGen + static_cast<int>(kFwdStageBytes);       // [16] RMSNorm scales
+  static constexpr int kGen = kS + kFwdRows * kKPC * 4;                     // K and V of one chunk read with plain loads
+  static constexpr int kRs = kGen + 2 * static_cast<int>(kFwdStageBytes);   // [16] RMSNorm scales
   static constexpr int kCs = kRs + 16 * 4;                                  // [2][16] chunk max / sum
   static constexpr int kRed = kCs + 32 * 4;                                 // [4][16]
   static constexpr int kFlag = kRed + 64 * 4;                               // [4] ints
@@ -361,15 +361,30 @@ __device__ __forceinline__ void fwd_epilogue(const FwdParams& P, const FwdPhase*
 // values just written), the projection's other rows from its input rows in global
 // memory; each value times the projection's RMSNorm gain, split into bf16 hi (row
 // m) + lo (row 16 + m), rows beyond the projection's M zero, 128-byte swizzled.
+// Gain slices of the (at most two) 8-column chunks thread dt writes, loaded ahead.
+__device__ __forceinline__ void fwd_btile_gains(const FwdPhase* ph, int c0, int nc, int dt, uint4* g) {
+  const int nch = nc >> 3, kmax = ph->bt_nkt * kTileK;
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    const int task = dt + t * kDrainThreads;
+    const int col = c0 + (task % nch) * 8;
+    g[t] = (task < kNPad * nch && col < kmax) ? __ldg(reinterpret_cast<const uint4*>(ph->bt_gain + col))
+                                              : make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
 __device__ __forceinline__ void fwd_btile_write(const FwdParams& P, const FwdPhase* ph, const float* fin, int c0,
-                                                int nc, int dt) {
+                                                int nc, int dt, const uint4* gpre = nullptr) {
   uint8_t* bt = P.btiles + ph->bt_dst_off;
   const float* xc = ph->bt_x;
   const int xs = ph->bt_x_stride, Mc = ph->bt_M, r0 = ph->bt_row0, Mown = ph->M;
   const __nv_bfloat16* gain = ph->bt_gain;
   const int kmax = ph->bt_nkt * kTileK;
-  const int nch = nc >> 3;  // 8-column chunks
-  for (int task = dt; task < kNPad * nch; task += kDrainThreads) {
+  const int nch = nc >> 3;  // 8-column chunks (nc <= 128: at most two per thread)
+#pragma unroll
+  for (int t = 0; t < 2; ++t) {
+    const int task = dt + t * kDrainThreads;
+    if (task >= kNPad * nch) break;
     const int m = task / nch, c8 = task - m * nch;
     const int col = c0 + c8 * 8;
     if (col >= kmax) continue;
@@ -387,7 +402,7 @@ __device__ __forceinline__ void fwd_btile_write(const FwdParams& P, const FwdPha
         v[4] = a1.x; v[5] = a1.y; v[6] = a1.z; v[7] = a1.w;
       }
       if (gain) {
-        const uint4 gv = __ldg(reinterpret_cast<const uint4*>(gain + col));
+        const uint4 gv = gpre ? gpre[t] : __ldg(reinterpret_cast<const uint4*>(gain + col));
         const float2 g0 = bf16x2_to_float2(gv.x), g1 = bf16x2_to_float2(gv.y), g2 = bf16x2_to_float2(gv.z),
                      g3 = bf16x2_to_float2(gv.w);
         v[0] *= g0.x; v[1] *= g0.y; v[2] *= g1.x; v[3] *= g1.y;
@@ -411,105 +426,100 @@ __device__ __forceinline__ void fwd_btile_write(const FwdParams& P, const FwdPha
 
 // ------------------------------------------------------------------ attention pieces (128 drain threads)
 
-// Scores of one chunk: thread -> (key j, quarter/half of the head dimension); the
-// partial dot products are summed across the key's threads with a fixed xor tree.
+// Attention state of one drain warp for the rows of one work item.  Within every
+// chunk the warp owns a fixed quarter of the keys (8 of 32 for head_dim 128, 16 of
+// 64 for 64): scores with TPK lanes per key (32 dimensions each, summed with a
+// fixed xor tree), an online softmax over the warp's keys, and P.V with each lane
+// holding DH/32 output dimensions.  The key -> (split, warp) assignment depends on
+// key positions only, so every row's result is independent of the number of rows.
 template <int DH>
-__device__ __forceinline__ void attn_scores(const float* Ks, const float* Qs, float* Ss, int M, int j0, int nk,
-                                            int base, float scale, int dt) {
-  constexpr int KPC = FwdSmem<DH>::kKPC, TPK = kDrainThreads / KPC, EPT = DH / TPK;
-  static_assert(EPT == 32, "32 elements per thread");
-  const int j = dt / TPK, part = dt - j * TPK, rot = dt & 7;
-  const float* kr = Ks + j * DH + part * EPT;
-  float kv[EPT];
+struct AttnWarp {
+  static constexpr int KPC = FwdSmem<DH>::kKPC;  // keys per chunk
+  static constexpr int KPW = KPC / 4;            // keys per warp
+  static constexpr int TPK = 32 / KPW;           // lanes per key (4 or 2)
+  static constexpr int DPL = DH / 32;            // output dimensions per lane (4 or 2)
+  float mx[kFwdRows], l[kFwdRows], o[kFwdRows][DPL];
+
+  __device__ __forceinline__ void init() {
 #pragma unroll
-  for (int e = 0; e < 8; ++e) {
-    const float4 t = *reinterpret_cast<const float4*>(kr + ((e + rot) & 7) * 4);
-    kv[4 * e] = t.x;
-    kv[4 * e + 1] = t.y;
-    kv[4 * e + 2] = t.z;
-    kv[4 * e + 3] = t.w;
+    for (int m = 0; m < kFwdRows; ++m) {
+      mx[m] = -INFINITY;
+      l[m] = 0.f;
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) o[m][e] = 0.f;
+    }
   }
-#pragma unroll 1
-  for (int m = 0; m < M; ++m) {
-    const float* qr = Qs + m * DH + part * EPT;
-    float s = 0.f;
+
+  // Fold the warp's keys of one chunk (K rows Ks, V rows Vs, keys j0 .. j0+nk-1 valid) into the state.
+  __device__ __forceinline__ void chunk(const float* Ks, const float* Vs, const float* Qs, int M, int j0, int nk,
+                                        int base, float scale, int w, int lane) {
+    const int kk = lane / TPK, part = lane - kk * TPK, rot = lane & 7;
+    const int j = w * KPW + kk;  // this lane's key within the chunk
+    const float* kr = Ks + j * DH + part * 32;
+    float kv[32];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      const float4 q = *reinterpret_cast<const float4*>(qr + ((e + rot) & 7) * 4);
-      s = fmaf(kv[4 * e], q.x, s);
-      s = fmaf(kv[4 * e + 1], q.y, s);
-      s = fmaf(kv[4 * e + 2], q.z, s);
-      s = fmaf(kv[4 * e + 3], q.w, s);
+      const float4 t = *reinterpret_cast<const float4*>(kr + ((e + rot) & 7) * 4);
+      kv[4 * e] = t.x;
+      kv[4 * e + 1] = t.y;
+      kv[4 * e + 2] = t.z;
+      kv[4 * e + 3] = t.w;
     }
+    const int d0 = lane * DPL;
 #pragma unroll
-    for (int off = 1; off < TPK; off <<= 1) s += __shfl_xor_sync(0xffffffffu, s, off);
-    if (part == 0) {
+    for (int m = 0; m < kFwdRows; ++m) {
+      if (m >= M) break;
+      const float* qr = Qs + m * DH + part * 32;
+      float sc = 0.f;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const float4 q = *reinterpret_cast<const float4*>(qr + ((e + rot) & 7) * 4);
+        sc = fmaf(kv[4 * e], q.x, sc);
+        sc = fmaf(kv[4 * e + 1], q.y, sc);
+        sc = fmaf(kv[4 * e + 2], q.z, sc);
+        sc = fmaf(kv[4 * e + 3], q.w, sc);
+      }
+#pragma unroll
+      for (int off = 1; off < TPK; off <<= 1) sc += __shfl_xor_sync(0xffffffffu, sc, off);
       const bool vis = j < nk && j0 + j <= base + m;
-      Ss[m * KPC + j] = vis ? s * scale : -INFINITY;
+      const float v = vis ? sc * scale : -INFINITY;
+      float cmx = v;
+#pragma unroll
+      for (int off = TPK; off < 32; off <<= 1) cmx = fmaxf(cmx, __shfl_xor_sync(0xffffffffu, cmx, off));
+      if (cmx == -INFINITY) continue;  // no visible key of row m among this warp's keys
+      const float pj = vis ? expf(v - cmx) : 0.f;
+      float csum = part == 0 ? pj : 0.f;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
+      float acc[DPL];
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) acc[e] = 0.f;
+#pragma unroll
+      for (int t = 0; t < KPW; ++t) {
+        const float pt = __shfl_sync(0xffffffffu, pj, t * TPK);
+        if (w * KPW + t >= nk) break;  // rows past the chunk's keys hold stale shared memory
+        const float* vr = Vs + (w * KPW + t) * DH + d0;
+        if constexpr (DPL == 4) {
+          const float4 vv = *reinterpret_cast<const float4*>(vr);
+          acc[0] = fmaf(pt, vv.x, acc[0]);
+          acc[1] = fmaf(pt, vv.y, acc[1]);
+          acc[2] = fmaf(pt, vv.z, acc[2]);
+          acc[3] = fmaf(pt, vv.w, acc[3]);
+        } else {
+          const float2 vv = *reinterpret_cast<const float2*>(vr);
+          acc[0] = fmaf(pt, vv.x, acc[0]);
+          acc[1] = fmaf(pt, vv.y, acc[1]);
+        }
+      }
+      const float nmx = fmaxf(mx[m], cmx);
+      const float so = expf(mx[m] - nmx), sn = expf(cmx - nmx);
+      l[m] = l[m] * so + csum * sn;
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) o[m][e] = o[m][e] * so + acc[e] * sn;
+      mx[m] = nmx;
     }
   }
-}
-
-// Row softmax pieces of one chunk: probabilities in place, chunk max and sum per row.
-template <int DH>
-__device__ __forceinline__ void attn_softmax(float* Ss, float* cs, int M, int w4, int lane) {
-  constexpr int KPC = FwdSmem<DH>::kKPC;
-  for (int m = w4; m < M; m += 4) {
-    float v[KPC / 32];
-    float mx = -INFINITY;
-#pragma unroll
-    for (int t = 0; t < KPC / 32; ++t) {
-      v[t] = Ss[m * KPC + t * 32 + lane];
-      mx = fmaxf(mx, v[t]);
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-    float l = 0.f;
-#pragma unroll
-    for (int t = 0; t < KPC / 32; ++t) {
-      const float e = (mx != -INFINITY && v[t] != -INFINITY) ? expf(v[t] - mx) : 0.f;
-      Ss[m * KPC + t * 32 + lane] = e;
-      l += e;
-    }
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) l += __shfl_xor_sync(0xffffffffu, l, off);
-    if (lane == 0) {
-      cs[m] = mx;
-      cs[16 + m] = l;
-    }
-  }
-}
-
-// P.V of one chunk folded into the running state of thread (d, g): rows g, g + GROUPS, ...
-template <int DH>
-__device__ __forceinline__ void attn_pv(const float* Vs, const float* Ss, const float* cs, int M, int nk, int dt,
-                                        float* o_run, float* mx_run, float* l_run) {
-  constexpr int KPC = FwdSmem<DH>::kKPC, GROUPS = kDrainThreads / DH, RPG = (kFwdRows + GROUPS - 1) / GROUPS;
-  const int d = dt % DH, g = dt / DH;
-  float acc[RPG];
-#pragma unroll
-  for (int r = 0; r < RPG; ++r) acc[r] = 0.f;
-  for (int j = 0; j < nk; ++j) {
-    const float v = Vs[j * DH + d];
-#pragma unroll
-    for (int r = 0; r < RPG; ++r) {
-      const int m = g + r * GROUPS;
-      if (m < M) acc[r] = fmaf(Ss[m * KPC + j], v, acc[r]);
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < RPG; ++r) {
-    const int m = g + r * GROUPS;
-    if (m >= M) continue;
-    const float cmx = cs[m];
-    if (cmx == -INFINITY) continue;  // no visible key of row m in this chunk
-    const float nmx = fmaxf(mx_run[r], cmx);
-    const float so = expf(mx_run[r] - nmx), sc = expf(cmx - nmx);
-    l_run[r] = l_run[r] * so + cs[16 + m] * sc;
-    o_run[r] = o_run[r] * so + acc[r] * sc;
-    mx_run[r] = nmx;
-  }
-}
+};
 
 // Plain loads of one chunk's K or V rows (keys j0 .. j0+nk-1) into shared memory.
 template <int DH>
@@ -523,11 +533,12 @@ __device__ __forceinline__ void attn_load_chunk(float* dst, const float* src, in
 template <int DH>
 __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int c, int G, int kv_len, uint32_t& i,
                               uint8_t* smem, uint64_t* full, uint64_t* empty, int dt, const FwdCtl& k) {
-  float* fin = reinterpret_cast<float*>(smem + FwdSmem<DH>::kOut);
   using S = FwdSmem<DH>;
-  constexpr int KPC = S::kKPC, GROUPS = kDrainThreads / DH, RPG = (kFwdRows + GROUPS - 1) / GROUPS;
+  using AW = AttnWarp<DH>;
+  constexpr int KPC = S::kKPC, DPL = AW::DPL;
+  float* fin = reinterpret_cast<float*>(smem + S::kOut);
   const AttnGeom ag = attn_geom(ph, kv_len, P.max_seq, KPC);
-  const int M = ph->M, splits = P.splits, I = P.n_heads * splits;
+  const int M = ph->M, splits = P.splits, I = P.n_heads * splits, nsub = 4 * splits;
   const int it0 = unit_begin(c, I, G), it1 = unit_begin(c + 1, I, G);
   if (ag.bad && dt == 0 && it0 < it1) set_error(P.st, DERR_POS);
   const FwdPhase* qk = P.phases + ph->dep;  // the QKV phase of this layer
@@ -540,13 +551,12 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
   float* o = ph->dst;
   const int o_stride = ph->dst_stride;
   float* Qs = reinterpret_cast<float*>(smem + S::kQ);
-  float* Ss = reinterpret_cast<float*>(smem + S::kS);
-  float* cs = reinterpret_cast<float*>(smem + S::kCs);
-  float* Gb = reinterpret_cast<float*>(smem + S::kGen);
+  float* Gk = reinterpret_cast<float*>(smem + S::kGen);
+  float* Gv = Gk + kFwdStageBytes / 4;
   volatile int* bflag = reinterpret_cast<volatile int*>(smem + S::kFlag) + 1;
-  float* part = P.attn_part + static_cast<size_t>(p % kFwdWindow) * P.n_heads * splits * kFwdRows * (DH + 2);
-  const int w4 = (dt >> 5), lane = dt & 31;
-  const int d = dt % DH, g = dt / DH;
+  constexpr int kEnt = DH + 2;  // o[DH], max, sum
+  float* part = P.attn_part + static_cast<size_t>(p % kFwdWindow) * P.n_heads * nsub * kFwdRows * kEnt;
+  const int w = dt >> 5, lane = dt & 31;
 
   for (int it = it0; it < it1; ++it) {
     const int h = it / splits, r = it - h * splits;
@@ -561,13 +571,8 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
       const int m = idx / DH, e = idx - m * DH;
       Qs[idx] = __ldcg(qsrc + static_cast<size_t>(m) * q_stride + h * DH + e);
     }
-    float o_run[RPG], mx_run[RPG], l_run[RPG];
-#pragma unroll
-    for (int q = 0; q < RPG; ++q) {
-      o_run[q] = 0.f;
-      mx_run[q] = -INFINITY;
-      l_run[q] = 0.f;
-    }
+    AW st;
+    st.init();
     drain_sync();
     const int nr = ring_chunks_of(ag.n_ring, r, splits);
     for (int q = 0; q < nr; ++q) {
@@ -576,14 +581,10 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
       ok = fwd_mbar_wait(&full[sK], (i / kFwdStages) & 1u, k) &&
            fwd_mbar_wait(&full[sV], ((i + 1) / kFwdStages) & 1u, k);
       if (!drain_all(ok)) return false;
-      const float* Ks = reinterpret_cast<const float*>(smem + S::kW + sK * kFwdStageBytes);
-      const float* Vs = reinterpret_cast<const float*>(smem + S::kW + sV * kFwdStageBytes);
-      attn_scores<DH>(Ks, Qs, Ss, M, ck * KPC, KPC, ag.base, P.attn_scale, dt);
-      drain_sync();
-      attn_softmax<DH>(Ss, cs, M, w4, lane);
-      drain_sync();
-      attn_pv<DH>(Vs, Ss, cs, M, KPC, dt, o_run, mx_run, l_run);
-      drain_sync();
+      st.chunk(reinterpret_cast<const float*>(smem + S::kW + sK * kFwdStageBytes),
+               reinterpret_cast<const float*>(smem + S::kW + sV * kFwdStageBytes), Qs, M, ck * KPC, KPC, ag.base,
+               P.attn_scale, w, lane);
+      drain_sync();  // every warp is done with both stages
       if (dt == 0) {
         mbar_arrive(&empty[sK]);
         mbar_arrive(&empty[sV]);
@@ -593,26 +594,23 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
     for (int ck = r + nr * splits; ck < ag.n_chunks; ck += splits) {
       const int j0 = ck * KPC, nk = min(KPC, ag.n_keys - j0);
       const size_t off = (static_cast<size_t>(h) * P.max_seq + j0) * DH;
-      attn_load_chunk<DH>(Gb, kc + off, nk, dt);
+      attn_load_chunk<DH>(Gk, kc + off, nk, dt);
+      attn_load_chunk<DH>(Gv, vc + off, nk, dt);
       drain_sync();
-      attn_scores<DH>(Gb, Qs, Ss, M, j0, nk, ag.base, P.attn_scale, dt);
-      drain_sync();
-      attn_softmax<DH>(Ss, cs, M, w4, lane);
-      attn_load_chunk<DH>(Gb, vc + off, nk, dt);
-      drain_sync();
-      attn_pv<DH>(Gb, Ss, cs, M, nk, dt, o_run, mx_run, l_run);
+      st.chunk(Gk, Gv, Qs, M, j0, nk, ag.base, P.attn_scale, w, lane);
       drain_sync();
     }
-    // publish this split's state; the last split of the head merges all of them in split order
+    // publish this warp's state as sub-split 4 r + w; the last split of the head merges
+    // all 4 * splits states in order
 #pragma unroll
-    for (int q = 0; q < RPG; ++q) {
-      const int m = g + q * GROUPS;
-      if (m >= M) continue;
-      float* e = part + ((static_cast<size_t>(h) * splits + r) * kFwdRows + m) * (DH + 2);
-      __stcg(e + d, o_run[q]);
-      if (d == 0) {
-        __stcg(e + DH, mx_run[q]);
-        __stcg(e + DH + 1, l_run[q]);
+    for (int m = 0; m < kFwdRows; ++m) {
+      if (m >= M) break;
+      float* e = part + ((static_cast<size_t>(h) * nsub + 4 * r + w) * kFwdRows + m) * kEnt;
+#pragma unroll
+      for (int d = 0; d < DPL; ++d) __stcg(e + lane * DPL + d, st.o[m][d]);
+      if (lane == 0) {
+        __stcg(e + DH, st.mx[m]);
+        __stcg(e + DH + 1, st.l[m]);
       }
     }
     __threadfence();
@@ -621,21 +619,37 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
     drain_sync();
     if (*bflag) {
       __threadfence();
+      for (int idx = dt; idx < M * DH; idx += kDrainThreads) {
+        const int m = idx / DH, d = idx - m * DH;
+        const float* e0 = part + (static_cast<size_t>(h) * nsub * kFwdRows + m) * kEnt;
+        const size_t sstride = static_cast<size_t>(kFwdRows) * kEnt;
+        // sub-splits in groups of 16, each group's loads issued together (one round for 4 splits);
+        // a running maximum carries the groups, in a fixed order
+        float mt = -INFINITY, L = 0.f, O = 0.f;
+        for (int q0 = 0; q0 < nsub; q0 += 16) {
+          float mq[16], lq[16], oq[16];
 #pragma unroll
-      for (int q = 0; q < RPG; ++q) {
-        const int m = g + q * GROUPS;
-        if (m >= M) continue;
-        const float* e0 = part + (static_cast<size_t>(h) * splits * kFwdRows + m) * (DH + 2);
-        const size_t rstride = static_cast<size_t>(kFwdRows) * (DH + 2);
-        float mt = -INFINITY;
-        for (int rr = 0; rr < splits; ++rr) mt = fmaxf(mt, __ldcg(e0 + rr * rstride + DH));
-        float L = 0.f, O = 0.f;
-        for (int rr = 0; rr < splits; ++rr) {
-          const float mq = __ldcg(e0 + rr * rstride + DH);
-          if (mq == -INFINITY) continue;
-          const float w = expf(mq - mt);
-          L = fmaf(w, __ldcg(e0 + rr * rstride + DH + 1), L);
-          O = fmaf(w, __ldcg(e0 + rr * rstride + d), O);
+          for (int q = 0; q < 16; ++q) {
+            const bool in = q0 + q < nsub;
+            mq[q] = in ? __ldcg(e0 + (q0 + q) * sstride + DH) : -INFINITY;
+            lq[q] = in ? __ldcg(e0 + (q0 + q) * sstride + DH + 1) : 0.f;
+            oq[q] = in ? __ldcg(e0 + (q0 + q) * sstride + d) : 0.f;
+          }
+          float gm = mt;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) gm = fmaxf(gm, mq[q]);
+          if (gm == -INFINITY) continue;
+          const float so = expf(mt - gm);  // 0 for the first group with a visible key
+          L *= so;
+          O *= so;
+#pragma unroll
+          for (int q = 0; q < 16; ++q) {
+            if (mq[q] == -INFINITY) continue;
+            const float wq = expf(mq[q] - gm);
+            L = fmaf(wq, lq[q], L);
+            O = fmaf(wq, oq[q], O);
+          }
+          mt = gm;
         }
         const float ov = L > 0.f ? O / L : 0.f;
         o[m * o_stride + h * DH + d] = ov;
@@ -1026,12 +1040,32 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_kernel(const __grid_consta
       }
       drain_sync();
 
-      float* part = P.partials + static_cast<size_t>(p % kFwdWindow) * (2 * G * kFwdRows * kTileN);
-      const int rt_first = u0 / n_kt;
-      int seg_kt0 = u0 - rt_first * n_kt;
+      // Split row tiles: the CTA holding a tile's first K slices (the end of its unit
+      // range, so it reaches the tile last) sums its own accumulator and the other
+      // holders' partials -- which they wrote at the start of their ranges -- in CTA
+      // order, and runs the epilogue; the others write a partial and count a ticket.
+      float* part = P.partials + static_cast<size_t>(p % kFwdWindow) * (G * kFwdRows * kTileN);
+      const bool resid = kind == FK_RESID;
+      const bool want_b = ph->bt_dst_off >= 0;
+      const float rscale = resid ? __ldg(ph->scale) : 0.f;
+      int seg_kt0 = u0 % n_kt;
       for (int u = u0; u < u1; ++u) {
         const int rt = u / n_kt, kt = u - rt * n_kt;
         if (!(kt == n_kt - 1 || u == u1 - 1)) continue;
+        const bool whole = (seg_kt0 == 0) && (kt == n_kt - 1);
+        const int c_first = unit_owner(rt * n_kt, units, ge);
+        const int c_last = unit_owner(rt * n_kt + n_kt - 1, units, ge);
+        const bool owner = whole || c == c_first;
+        // epilogue inputs that do not depend on the accumulator, loaded before it is ready
+        float bpre[kFwdRows];
+        uint4 gpre[2];
+        const int ncol = rt * kTileN + dt;
+        if (owner && resid) {
+#pragma unroll
+          for (int m = 0; m < kFwdRows; ++m)
+            bpre[m] = (m < M && ncol < ph->N) ? __ldcg(ph->base + m * ph->base_stride + ncol) : 0.f;
+        }
+        if (owner && want_b && ph->bt_gain) fwd_btile_gains(ph, rt * tcols, tcols, dt, gpre);
         const uint32_t b = sg % kFwdAcc;
         if (!drain_all(fwd_mbar_wait(&accf[b], (sg / kFwdAcc) & 1u, k))) {
           ok = false;
@@ -1049,66 +1083,58 @@ __global__ void __launch_bounds__(kFwdThreads, 1) fwd_kernel(const __grid_consta
         for (int m = 0; m < kFwdRows; ++m)
           if (m < M) outb[m * kTileN + q4 * 32 + lane] = vh[m] + vl[m];  // W a = W hi + W lo
         drain_sync();
-        const bool whole = (seg_kt0 == 0) && (kt == n_kt - 1);
-        if (whole) {
-          fwd_epilogue(P, ph, rt, outb, rs, dt, kv_len);
-          if (ph->bt_dst_off >= 0) {
-            drain_sync();
-            fwd_btile_write(P, ph, outb, rt * tcols, tcols, dt);
+        if (owner && !whole) {  // own accumulator, then the others' partials in CTA order
+          const int nsp = c_last - c_first + 1;
+          if (!drain_all(fwd_flag_wait(P.tickets + ph->flags + rt, static_cast<unsigned>(nsp - 1), k))) {
+            ok = false;
+            break;
           }
-          fwd_release(P, ph, p, rt, dt);
-        } else {
-          const int slot = 2 * c + (rt == rt_first ? 0 : 1);
-          float* dstp = part + static_cast<size_t>(slot) * (kFwdRows * kTileN);
+          for (int f = dt; f < M * (kTileN / 4); f += kDrainThreads) {
+            float4 sum = reinterpret_cast<const float4*>(outb)[f];
+            for (int b0 = 1; b0 < nsp; b0 += 8) {
+              float4 pv[8];
+#pragma unroll
+              for (int j = 0; j < 8; ++j)
+                pv[j] = (b0 + j < nsp) ? __ldcg(reinterpret_cast<const float4*>(
+                                             part + static_cast<size_t>(c_first + b0 + j) * (kFwdRows * kTileN)) + f)
+                                       : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+              for (int j = 0; j < 8; ++j) {
+                if (b0 + j >= nsp) continue;
+                sum.x += pv[j].x;
+                sum.y += pv[j].y;
+                sum.z += pv[j].z;
+                sum.w += pv[j].w;
+              }
+            }
+            reinterpret_cast<float4*>(outb)[f] = sum;
+          }
+          if (dt == 0) P.tickets[ph->flags + rt] = 0u;
+          drain_sync();
+        }
+        if (!owner) {
+          float* dstp = part + static_cast<size_t>(c) * (kFwdRows * kTileN);
           for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) __stcg(dstp + idx, outb[idx]);
           __threadfence();
           drain_sync();
-          const int c_first = unit_owner(rt * n_kt, units, ge);
-          const int c_last = unit_owner(rt * n_kt + n_kt - 1, units, ge);
-          if (dt == 0)
-            sflag[1] = (atomicAdd(P.tickets + ph->flags + rt, 1u) == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
-          drain_sync();
-          if (sflag[1]) {
-            __threadfence();
-            // sum the partials in CTA order; the loads of 8 CTAs are issued together
-            const int nsp = c_last - c_first + 1;
-            for (int f = dt; f < M * (kTileN / 4); f += kDrainThreads) {
-              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-              for (int b0 = 0; b0 < nsp; b0 += 8) {
-                float4 pv[8];
+          if (dt == 0) red_relaxed_add(P.tickets + ph->flags + rt, 1u);
+        } else {
+          if (resid) {  // dst = base + s * (W a), with the base loaded ahead
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  const int cc = c_first + b0 + j;
-                  pv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-                  if (b0 + j < nsp) {
-                    const int sl = 2 * cc + (rt == unit_begin(cc, units, ge) / n_kt ? 0 : 1);
-                    pv[j] = __ldcg(reinterpret_cast<const float4*>(part + static_cast<size_t>(sl) * (kFwdRows * kTileN)) + f);
-                  }
-                }
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  if (b0 + j >= nsp) continue;
-                  if (b0 + j == 0) {
-                    sum = pv[j];
-                  } else {
-                    sum.x += pv[j].x;
-                    sum.y += pv[j].y;
-                    sum.z += pv[j].z;
-                    sum.w += pv[j].w;
-                  }
-                }
-              }
-              reinterpret_cast<float4*>(outb)[f] = sum;
+            for (int m = 0; m < kFwdRows; ++m) {
+              if (m >= M || ncol >= ph->N) continue;
+              const float y = bpre[m] + rscale * (outb[m * kTileN + dt] * rs[m]);
+              ph->dst[m * ph->dst_stride + ncol] = y;
+              outb[m * kTileN + dt] = y;
             }
-            drain_sync();
+          } else {
             fwd_epilogue(P, ph, rt, outb, rs, dt, kv_len);
-            if (dt == 0) P.tickets[ph->flags + rt] = 0u;
-            if (ph->bt_dst_off >= 0) {
-              drain_sync();
-              fwd_btile_write(P, ph, outb, rt * tcols, tcols, dt);
-            }
-            fwd_release(P, ph, p, rt, dt);
           }
+          if (want_b) {
+            drain_sync();
+            fwd_btile_write(P, ph, outb, rt * tcols, tcols, dt, ph->bt_gain ? gpre : nullptr);
+          }
+          fwd_release(P, ph, p, rt, dt);
         }
         drain_sync();
         seg_kt0 = 0;

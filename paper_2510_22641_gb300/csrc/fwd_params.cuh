@@ -84,8 +84,8 @@ struct FwdParams {
   unsigned* exit_count;  // CTAs that have left
   uint8_t* btiles;       // [kFwdBSlots][max n_kt][kFwdBTile] B operands, written by producer epilogues
   int n_flags;
-  float* partials;       // [kFwdWindow][2 * grid][kFwdRows][128]
-  float* attn_part;      // [kFwdWindow][n_heads][splits][kFwdRows][head_dim + 2]
+  float* partials;       // [kFwdWindow][grid][kFwdRows][128]
+  float* attn_part;      // [kFwdWindow][n_heads][4 * splits][kFwdRows][head_dim + 2] (one state per drain warp)
   int n_heads, head_dim, max_seq, splits;
   float attn_scale, eps;
   const float2* rope;    // [max_seq][head_dim / 2] (cos, sin)
