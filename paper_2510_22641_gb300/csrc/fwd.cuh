@@ -99,6 +99,13 @@ __device__ __forceinline__ void red_relaxed_add(unsigned* p, unsigned v) {
 
 __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
+// 16-byte asynchronous global -> shared copies (completion: cp_async_wait_all).
+__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
 // AND of `ok` over the 128 drain threads (named barrier 1).
 __device__ __forceinline__ bool drain_all(bool ok) {
   uint32_t r;
@@ -146,15 +153,14 @@ __device__ __forceinline__ bool fwd_mbar_wait(uint64_t* bar, uint32_t parity, co
   }
 }
 
-// Waits until *f >= target; false once stopped or after ~2 s.  Polls with
-// relaxed loads (back-to-back for the first 20 us, then with a short sleep) and
-// ends with one acquire load (an acquire also drops the SM's L1 lines, which the
-// other roles keep hot).
+// Waits until *f >= target; false once stopped or after ~2 s.  One acquire load
+// when the flag is already set (the common case: one L2 round trip); otherwise
+// relaxed polls (back-to-back for the first 20 us, then with a short sleep) and a
+// final acquire load (an acquire also drops the SM's L1 lines, which the other
+// roles keep hot, so it is not used for polling; a fence.acq_rel instead would also
+// wait for the thread's bulk copies in flight).
 __device__ __forceinline__ bool fwd_flag_wait(const unsigned* f, unsigned target, const FwdCtl& k) {
-  if (ld_relaxed_u32(f) >= target) {
-    ld_acquire_u32(f);
-    return true;
-  }
+  if (ld_acquire_u32(f) >= target) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (ld_relaxed_u32(f) >= target) {
@@ -542,8 +548,6 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
   const int it0 = unit_begin(c, I, G), it1 = unit_begin(c + 1, I, G);
   if (ag.bad && dt == 0 && it0 < it1) set_error(P.st, DERR_POS);
   const FwdPhase* qk = P.phases + ph->dep;  // the QKV phase of this layer
-  const int seg = qk->seg_rows;
-  const unsigned* qflags = P.flags + qk->flags;
   const float* qsrc = ph->x;
   const int q_stride = ph->x_stride;
   const float* kc = ph->k_cache;
@@ -553,28 +557,39 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
   float* Qs = reinterpret_cast<float*>(smem + S::kQ);
   float* Gk = reinterpret_cast<float*>(smem + S::kGen);
   float* Gv = Gk + kFwdStageBytes / 4;
-  volatile int* bflag = reinterpret_cast<volatile int*>(smem + S::kFlag) + 1;
   constexpr int kEnt = DH + 2;  // o[DH], max, sum
   float* part = P.attn_part + static_cast<size_t>(p % kFwdWindow) * P.n_heads * nsub * kFwdRows * kEnt;
   const int w = dt >> 5, lane = dt & 31;
 
   for (int it = it0; it < it1; ++it) {
     const int h = it / splits, r = it - h * splits;
+    // q, k and v of every head come from one QKV phase whose row tiles finish within a
+    // microsecond of each other: one wait on the phase instead of three flag round trips
     bool ok = true;
-    if (!ag.bad) {
-      ok = fwd_flag_wait(qflags + (h * DH) / kTileN, 1u, k) &&
-           fwd_flag_wait(qflags + (seg + h * DH) / kTileN, 1u, k) &&
-           fwd_flag_wait(qflags + (2 * seg + h * DH) / kTileN, 1u, k);
-    }
+    if (!ag.bad) ok = fwd_flag_wait(P.done + ph->dep, static_cast<unsigned>(qk->n_tiles), k);
     if (!drain_all(ok)) return false;
+    if (dt == 0) fwd_stamp(P, c, p, 8);
     for (int idx = dt; idx < M * DH; idx += kDrainThreads) {
       const int m = idx / DH, e = idx - m * DH;
       Qs[idx] = __ldcg(qsrc + static_cast<size_t>(m) * q_stride + h * DH + e);
     }
     AW st;
     st.init();
-    drain_sync();
+    // the first chunk holding keys at or above kv_len (written this launch) is fetched now,
+    // behind the ring chunks
     const int nr = ring_chunks_of(ag.n_ring, r, splits);
+    const int ck_gen = r + nr * splits;
+    if (ck_gen < ag.n_chunks) {
+      const int j0 = ck_gen * KPC, nk = min(KPC, ag.n_keys - j0);
+      const size_t off = (static_cast<size_t>(h) * P.max_seq + j0) * DH;
+      for (int e = dt; e < nk * DH / 4; e += kDrainThreads) {
+        cp_async16(Gk + 4 * e, kc + off + 4 * e);
+        cp_async16(Gv + 4 * e, vc + off + 4 * e);
+      }
+      cp_async_commit();
+    }
+    drain_sync();
+    if (dt == 0) fwd_stamp(P, c, p, 9);
     for (int q = 0; q < nr; ++q) {
       const int ck = r + q * splits;
       const int sK = static_cast<int>(i % kFwdStages), sV = static_cast<int>((i + 1) % kFwdStages);
@@ -591,15 +606,21 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
       }
       i += 2;
     }
-    for (int ck = r + nr * splits; ck < ag.n_chunks; ck += splits) {
+    if (dt == 0) fwd_stamp(P, c, p, 10);
+    for (int ck = ck_gen; ck < ag.n_chunks; ck += splits) {
       const int j0 = ck * KPC, nk = min(KPC, ag.n_keys - j0);
-      const size_t off = (static_cast<size_t>(h) * P.max_seq + j0) * DH;
-      attn_load_chunk<DH>(Gk, kc + off, nk, dt);
-      attn_load_chunk<DH>(Gv, vc + off, nk, dt);
+      if (ck == ck_gen) {
+        cp_async_wait_all();
+      } else {
+        const size_t off = (static_cast<size_t>(h) * P.max_seq + j0) * DH;
+        attn_load_chunk<DH>(Gk, kc + off, nk, dt);
+        attn_load_chunk<DH>(Gv, vc + off, nk, dt);
+      }
       drain_sync();
       st.chunk(Gk, Gv, Qs, M, j0, nk, ag.base, P.attn_scale, w, lane);
       drain_sync();
     }
+    if (dt == 0) fwd_stamp(P, c, p, 11);
     // publish this warp's state as sub-split 4 r + w; the last split of the head merges
     // all 4 * splits states in order
 #pragma unroll
@@ -613,12 +634,20 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
         __stcg(e + DH + 1, st.l[m]);
       }
     }
-    __threadfence();
-    drain_sync();
-    if (dt == 0) *bflag = (atomicAdd(P.tickets + ph->flags + h, 1u) == static_cast<unsigned>(splits - 1)) ? 1 : 0;
-    drain_sync();
-    if (*bflag) {
+    // The split holding the newest chunk (always the one with the most work) merges: it
+    // waits for the other splits' tickets and reads its own states without a fence.
+    const int r_merge = ag.n_chunks > 0 ? (ag.n_chunks - 1) % splits : 0;
+    const bool merger = r == r_merge;
+    if (!merger) {
       __threadfence();
+      drain_sync();
+      if (dt == 0) red_relaxed_add(P.tickets + ph->flags + h, 1u);
+    } else {
+      drain_sync();
+      if (!drain_all(fwd_flag_wait(P.tickets + ph->flags + h, static_cast<unsigned>(splits - 1), k))) return false;
+    }
+    if (dt == 0) fwd_stamp(P, c, p, 12);
+    if (merger) {
       for (int idx = dt; idx < M * DH; idx += kDrainThreads) {
         const int m = idx / DH, d = idx - m * DH;
         const float* e0 = part + (static_cast<size_t>(h) * nsub * kFwdRows + m) * kEnt;
@@ -661,6 +690,7 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
         fwd_btile_write(P, ph, fin, h * DH, DH, dt);
       }
       fwd_release(P, ph, p, h, dt);
+      if (dt == 0) fwd_stamp(P, c, p, 13);
     }
     drain_sync();
   }
