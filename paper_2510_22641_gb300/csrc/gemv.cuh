@@ -241,13 +241,17 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       p.h_out[m * p.h_stride + n] = silu_f(out[idx] * rs[m]);
     }
   } else if constexpr (EPI == Epi::RESID) {
+    // thread tid owns column tid of every row; the base rows are loaded before any store
+    // (dst may alias base, so the stores would otherwise serialize the loads)
+    static_assert(kDrainThreads == kTileN, "one thread per tile column");
     const float s = __ldg(p.scale);
-    for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
-      const int m = idx / kTileN, i = idx - m * kTileN;
-      const int n = rt * kTileN + i;
-      if (n >= p.N) continue;
-      const float b = __ldcg(p.base + m * p.base_stride + n);
-      p.dst[m * p.dst_stride + n] = b + s * (out[idx] * rs[m]);
+    const int n = rt * kTileN + tid;
+    if (n < p.N) {
+      float bv[M];
+#pragma unroll
+      for (int m = 0; m < M; ++m) bv[m] = __ldcg(p.base + m * p.base_stride + n);
+#pragma unroll
+      for (int m = 0; m < M; ++m) p.dst[m * p.dst_stride + n] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
     }
   } else {  // ARGMAX (LM head): argmax over the vocabulary, lowest index on ties
     const int lane = tid & 31;
@@ -544,26 +548,36 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         drain_sync();
         if (flag[0]) {
           __threadfence();
-          // sum the partials in CTA order; the loads of 8 CTAs are issued together
+          // sum the partials in CTA order; 16-byte loads of 8 CTAs are issued together,
+          // all rows at once
           const int nsp = c_last - c_first + 1;
-          for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) {
-            float sum = 0.f;
+          for (int f = dt; f < M * (kTileN / 4); f += kDrainThreads) {
+            float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
             for (int b0 = 0; b0 < nsp; b0 += 8) {
-              float pv[8];
+              float4 pv[8];
 #pragma unroll
               for (int j = 0; j < 8; ++j) {
                 const int cc = c_first + b0 + j;
-                pv[j] = 0.f;
+                pv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (b0 + j < nsp) {
                   const int sl = 2 * cc + (rt == unit_begin(cc, p.units, G) / p.n_kt ? 0 : 1);
-                  pv[j] = __ldcg(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN) + idx);
+                  pv[j] = __ldcg(reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN)) + f);
                 }
               }
 #pragma unroll
-              for (int j = 0; j < 8; ++j)
-                if (b0 + j < nsp) sum = (b0 + j == 0) ? pv[j] : sum + pv[j];
+              for (int j = 0; j < 8; ++j) {
+                if (b0 + j >= nsp) continue;
+                if (b0 + j == 0) {
+                  sum = pv[j];
+                } else {
+                  sum.x += pv[j].x;
+                  sum.y += pv[j].y;
+                  sum.z += pv[j].z;
+                  sum.w += pv[j].w;
+                }
+              }
             }
-            outb[idx] = sum;
+            reinterpret_cast<float4*>(outb)[f] = sum;
           }
           drain_sync();
           gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
