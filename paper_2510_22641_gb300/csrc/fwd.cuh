@@ -54,6 +54,7 @@
 #pragma once
 
 #include "common.cuh"
+#include "attn_warp.cuh"
 #include "fwd_params.cuh"
 #include "gemv.cuh"
 
@@ -77,6 +78,7 @@ struct FwdSmem {
   static constexpr int kTmemSlot = kBar + kNBar * 8;
   static constexpr int kTotal = kTmemSlot + 16 + 1024;  // + slack for the 1024-byte alignment
   static_assert(kB % 1024 == 0 && kOut % 16 == 0 && kGen % 16 == 0 && kBar % 8 == 0, "shared-memory alignment");
+  static_assert(kKPC == AttnWarp<DH>::KPC && kFwdRows == kAttnMaxRows, "attention chunk shape");
 };
 
 // ------------------------------------------------------------------ synchronisation helpers
@@ -432,101 +434,6 @@ __device__ __forceinline__ void fwd_btile_write(const FwdParams& P, const FwdPha
 
 // ------------------------------------------------------------------ attention pieces (128 drain threads)
 
-// Attention state of one drain warp for the rows of one work item.  Within every
-// chunk the warp owns a fixed quarter of the keys (8 of 32 for head_dim 128, 16 of
-// 64 for 64): scores with TPK lanes per key (32 dimensions each, summed with a
-// fixed xor tree), an online softmax over the warp's keys, and P.V with each lane
-// holding DH/32 output dimensions.  The key -> (split, warp) assignment depends on
-// key positions only, so every row's result is independent of the number of rows.
-template <int DH>
-struct AttnWarp {
-  static constexpr int KPC = FwdSmem<DH>::kKPC;  // keys per chunk
-  static constexpr int KPW = KPC / 4;            // keys per warp
-  static constexpr int TPK = 32 / KPW;           // lanes per key (4 or 2)
-  static constexpr int DPL = DH / 32;            // output dimensions per lane (4 or 2)
-  float mx[kFwdRows], l[kFwdRows], o[kFwdRows][DPL];
-
-  __device__ __forceinline__ void init() {
-#pragma unroll
-    for (int m = 0; m < kFwdRows; ++m) {
-      mx[m] = -INFINITY;
-      l[m] = 0.f;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) o[m][e] = 0.f;
-    }
-  }
-
-  // Fold the warp's keys of one chunk (K rows Ks, V rows Vs, keys j0 .. j0+nk-1 valid) into the state.
-  __device__ __forceinline__ void chunk(const float* Ks, const float* Vs, const float* Qs, int M, int j0, int nk,
-                                        int base, float scale, int w, int lane) {
-    const int kk = lane / TPK, part = lane - kk * TPK, rot = lane & 7;
-    const int j = w * KPW + kk;  // this lane's key within the chunk
-    const float* kr = Ks + j * DH + part * 32;
-    float kv[32];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-      const float4 t = *reinterpret_cast<const float4*>(kr + ((e + rot) & 7) * 4);
-      kv[4 * e] = t.x;
-      kv[4 * e + 1] = t.y;
-      kv[4 * e + 2] = t.z;
-      kv[4 * e + 3] = t.w;
-    }
-    const int d0 = lane * DPL;
-#pragma unroll
-    for (int m = 0; m < kFwdRows; ++m) {
-      if (m >= M) break;
-      const float* qr = Qs + m * DH + part * 32;
-      float sc = 0.f;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const float4 q = *reinterpret_cast<const float4*>(qr + ((e + rot) & 7) * 4);
-        sc = fmaf(kv[4 * e], q.x, sc);
-        sc = fmaf(kv[4 * e + 1], q.y, sc);
-        sc = fmaf(kv[4 * e + 2], q.z, sc);
-        sc = fmaf(kv[4 * e + 3], q.w, sc);
-      }
-#pragma unroll
-      for (int off = 1; off < TPK; off <<= 1) sc += __shfl_xor_sync(0xffffffffu, sc, off);
-      const bool vis = j < nk && j0 + j <= base + m;
-      const float v = vis ? sc * scale : -INFINITY;
-      float cmx = v;
-#pragma unroll
-      for (int off = TPK; off < 32; off <<= 1) cmx = fmaxf(cmx, __shfl_xor_sync(0xffffffffu, cmx, off));
-      if (cmx == -INFINITY) continue;  // no visible key of row m among this warp's keys
-      const float pj = vis ? expf(v - cmx) : 0.f;
-      float csum = part == 0 ? pj : 0.f;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) csum += __shfl_xor_sync(0xffffffffu, csum, off);
-      float acc[DPL];
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) acc[e] = 0.f;
-#pragma unroll
-      for (int t = 0; t < KPW; ++t) {
-        const float pt = __shfl_sync(0xffffffffu, pj, t * TPK);
-        if (w * KPW + t >= nk) break;  // rows past the chunk's keys hold stale shared memory
-        const float* vr = Vs + (w * KPW + t) * DH + d0;
-        if constexpr (DPL == 4) {
-          const float4 vv = *reinterpret_cast<const float4*>(vr);
-          acc[0] = fmaf(pt, vv.x, acc[0]);
-          acc[1] = fmaf(pt, vv.y, acc[1]);
-          acc[2] = fmaf(pt, vv.z, acc[2]);
-          acc[3] = fmaf(pt, vv.w, acc[3]);
-        } else {
-          const float2 vv = *reinterpret_cast<const float2*>(vr);
-          acc[0] = fmaf(pt, vv.x, acc[0]);
-          acc[1] = fmaf(pt, vv.y, acc[1]);
-        }
-      }
-      const float nmx = fmaxf(mx[m], cmx);
-      const float so = expf(mx[m] - nmx), sn = expf(cmx - nmx);
-      l[m] = l[m] * so + csum * sn;
-#pragma unroll
-      for (int e = 0; e < DPL; ++e) o[m][e] = o[m][e] * so + acc[e] * sn;
-      mx[m] = nmx;
-    }
-  }
-};
-
 // Plain loads of one chunk's K or V rows (keys j0 .. j0+nk-1) into shared memory.
 template <int DH>
 __device__ __forceinline__ void attn_load_chunk(float* dst, const float* src, int nk, int dt) {
@@ -596,9 +503,9 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
       ok = fwd_mbar_wait(&full[sK], (i / kFwdStages) & 1u, k) &&
            fwd_mbar_wait(&full[sV], ((i + 1) / kFwdStages) & 1u, k);
       if (!drain_all(ok)) return false;
-      st.chunk(reinterpret_cast<const float*>(smem + S::kW + sK * kFwdStageBytes),
-               reinterpret_cast<const float*>(smem + S::kW + sV * kFwdStageBytes), Qs, M, ck * KPC, KPC, ag.base,
-               P.attn_scale, w, lane);
+      st.chunk_rows(reinterpret_cast<const float*>(smem + S::kW + sK * kFwdStageBytes),
+                    reinterpret_cast<const float*>(smem + S::kW + sV * kFwdStageBytes), Qs, M, ck * KPC, KPC, ag.base,
+                    P.attn_scale, w, lane);
       drain_sync();  // every warp is done with both stages
       if (dt == 0) {
         mbar_arrive(&empty[sK]);
@@ -617,7 +524,7 @@ __device__ bool fwd_attention(const FwdParams& P, const FwdPhase* ph, int p, int
         attn_load_chunk<DH>(Gv, vc + off, nk, dt);
       }
       drain_sync();
-      st.chunk(Gk, Gv, Qs, M, j0, nk, ag.base, P.attn_scale, w, lane);
+      st.chunk_rows(Gk, Gv, Qs, M, j0, nk, ag.base, P.attn_scale, w, lane);
       drain_sync();
     }
     if (dt == 0) fwd_stamp(P, c, p, 11);

@@ -3,6 +3,7 @@ cudaProfilerStart/Stop window (use `ncu --profile-from-start off`).
 
   python -m paper_2510_22641_gb300.profile_run --layers 32 --phase greedy --tokens 8
   python -m paper_2510_22641_gb300.profile_run --layers 2 --phase greedy --tokens 1
+  python -m paper_2510_22641_gb300.profile_run --layers 1 --phase proj --proj gateup --rows 1
 
 --layers keeps the 7B layer shape (d=4096, ff=11008, 32x128 heads, V=32000)
 but fewer layers, so full metric sets can be captured with a few GB on the
@@ -25,7 +26,9 @@ if ROOT not in sys.path:
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--layers", type=int, default=32)
-    ap.add_argument("--phase", choices=["greedy", "ssd", "prefill"], default="greedy")
+    ap.add_argument("--phase", choices=["greedy", "ssd", "prefill", "proj"], default="greedy")
+    ap.add_argument("--proj", default="gateup", help="--phase proj: qkv, o, gateup, down or head")
+    ap.add_argument("--rows", type=int, default=1, help="--phase proj: activation rows")
     ap.add_argument("--tokens", type=int, default=8)
     ap.add_argument("--s", type=float, default=0.2)
     args = ap.parse_args()
@@ -58,6 +61,16 @@ def main() -> None:
         elif args.phase == "ssd":
             model.decode(1 + args.tokens, w.gamma)
 
+    if args.phase == "proj":  # isolated launches of one projection kernel
+        model.profile_projection(args.proj, 0, args.rows, 3)
+        model.sync()
+        torch.cuda.profiler.start()
+        model.profile_projection(args.proj, 0, args.rows, 3)
+        model.sync()
+        torch.cuda.profiler.stop()
+        print("profile_run done", args.proj, args.rows)
+        model.close()
+        return
     run()                       # builds the graphs, warms up
     model.sync()
     if args.phase != "prefill":
