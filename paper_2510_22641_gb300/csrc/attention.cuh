@@ -10,8 +10,8 @@
 // copies, double-buffered.  Within a chunk, each of the 4 warps owns a fixed
 // quarter of the keys and folds them into its own running softmax state per row
 // (max, sum of exp, unnormalised output), so a chunk costs one CTA barrier.  The
-// cluster's rank 0 then merges the 4 x kAttnSplit states in (CTA, warp) order
-// through distributed shared memory.  The chunk grid, the key -> (CTA, warp)
+// cluster then merges the 4 x kAttnSplit states through distributed shared
+// memory, each CTA a slice of the output columns, in (CTA, warp) order.  The chunk grid, the key -> (CTA, warp)
 // assignment and the merge order depend only on key positions, never on M, so
 // each row's output equals the single-row (M = 1) result bitwise.
 #pragma once
@@ -45,7 +45,8 @@ struct AttnSmem {
   static constexpr int kBuf0 = (kQ + M * DH * 4 + 15) & ~15;        // two {K, V} buffers
   static constexpr int kFin = kBuf0 + 4 * kKV;                      // warp states [4][M][DH + 2]
   static constexpr int kPw = kFin + 4 * M * (DH + 2) * 4;           // per-warp probabilities [4][rows][KPW]
-  static constexpr int kBar = (kPw + 4 * kAttnMaxRows * (AttnWarp<DH>::KPW) * 4 + 7) & ~7;
+  static constexpr int kWq = kPw + 4 * kAttnMaxRows * (AttnWarp<DH>::KPW) * 4;  // merge weights [M][32], sums [M]
+  static constexpr int kBar = (kWq + M * 33 * 4 + 7) & ~7;
   static constexpr int kTotal = kBar + 3 * 8;
 };
 
@@ -121,7 +122,10 @@ __global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThread
   }
   if (!ok) set_error(p.st, DERR_TIMEOUT);
 
-  // publish the warps' states, then rank 0 merges the cluster's 4 x kAttnSplit states in order
+  // publish the warps' states; the cluster then merges the 4 x kAttnSplit states of each row.
+  // State s = 4 * CTA + warp.  Per row, one warp forms the weights exp(mx_s - max) and their sum
+  // with fixed shuffle trees; then CTA r combines columns [r * DH / kAttnSplit, (r + 1) * DH /
+  // kAttnSplit) of all rows, summing the states in s order.  None of it depends on M.
 #pragma unroll
   for (int m = 0; m < M; ++m) {
     float* e = fin + (w * M + m) * (DH + 2);
@@ -133,28 +137,36 @@ __global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThread
     }
   }
   cluster.sync();
-  if (rank == 0 && !bad) {
-    for (int idx = tid; idx < M * DH; idx += kAttnThreads) {
-      const int m = idx / DH, d = idx - m * DH;
-      float mt = -INFINITY;
-      for (int q = 0; q < kAttnSplit; ++q) {
-        const float* f = cluster.map_shared_rank(fin, q);
+  static_assert(4 * kAttnSplit == 32, "one merge lane per state");
+  if (!bad) {
+    float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][32]
+    float* ls = wq + M * 32;                              // [M]
+    const float* fs = cluster.map_shared_rank(fin, lane >> 2);
+    for (int m = w; m < M; m += 4) {
+      const float* e = fs + ((lane & 3) * M + m) * (DH + 2);
+      const float mq = e[DH], lq = e[DH + 1];
+      float mt = mq;
 #pragma unroll
-        for (int ww = 0; ww < 4; ++ww) mt = fmaxf(mt, f[(ww * M + m) * (DH + 2) + DH]);
-      }
-      float L = 0.f, O = 0.f;
-      for (int q = 0; q < kAttnSplit; ++q) {
-        const float* f = cluster.map_shared_rank(fin, q);
+      for (int o = 16; o; o >>= 1) mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+      const float g = mq == -INFINITY ? 0.f : expf(mq - mt);
+      float L = g * lq;
 #pragma unroll
-        for (int ww = 0; ww < 4; ++ww) {
-          const float* e = f + (ww * M + m) * (DH + 2);
-          const float mq = e[DH];
-          if (mq == -INFINITY) continue;
-          const float wq = expf(mq - mt);
-          L = fmaf(wq, e[DH + 1], L);
-          O = fmaf(wq, e[d], O);
-        }
-      }
+      for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
+      wq[m * 32 + lane] = g;
+      if (lane == 0) ls[m] = L;
+    }
+    __syncthreads();
+    constexpr int DS = DH / kAttnSplit;
+    for (int idx = tid; idx < M * DS; idx += kAttnThreads) {
+      const int m = idx / DS, d = rank * DS + (idx - m * DS);
+      float v[32];
+#pragma unroll
+      for (int s = 0; s < 32; ++s)
+        v[s] = cluster.map_shared_rank(fin, s >> 2)[((s & 3) * M + m) * (DH + 2) + d];
+      float O = 0.f;
+#pragma unroll
+      for (int s = 0; s < 32; ++s) O = fmaf(wq[m * 32 + s], v[s], O);
+      const float L = ls[m];
       p.o[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
     }
   }
