@@ -67,6 +67,46 @@ def algorithmic_bytes(w: synth.Workload) -> dict:
             "verify": sh.n_layers * layer + head, "greedy_token": sh.n_layers * layer + head}
 
 
+KERNEL_ROWS = (("qkv", "gemv_kernel<M, QKV> (q/k/v + RoPE + KV write)"),
+               ("o", "gemv_kernel<M, RESID> (o_proj)"),
+               ("gateup", "gemv_kernel<M, GATE_SILU> (gate/up)"),
+               ("down", "gemv_kernel<M, RESID> (down)"),
+               ("attn", "attn_kernel<M, 128> (split-KV, cache after prefill)"),
+               ("head", "gemv_kernel<M, ARGMAX> (LM head)"),
+               ("in1", "gemv_kernel<1, SILU> (imitation FC1)"),
+               ("in2", "gemv_kernel<1, RESID> (imitation FC2)"))
+
+
+def kernel_table(model, w, v, p, stream, hbm_peak, reps=50):
+    """Every decode kernel timed alone (CUDA events, `reps` back-to-back launches) at the draft's
+    1 row and the verification's gamma + 1 rows, against the HBM copy peak.  `layer_m*` sums one
+    decoder layer's kernels (bytes / time), the fraction a layer would reach with no launch gaps."""
+    import torch
+    rows_out, layer = [], {}
+    for rows in (1, w.gamma + 1):
+        for name, label in KERNEL_ROWS:
+            if name in ("in1", "in2") and rows != 1:
+                continue
+            model.prefill(v, p)
+            model.profile_projection(name, layer=0, rows=rows, reps=3)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            a.record(stream)
+            nbytes = model.profile_projection(name, layer=0, rows=rows, reps=reps)
+            b.record(stream)
+            torch.cuda.synchronize()
+            us = a.elapsed_time(b) / reps * 1e3
+            gbs = nbytes / us / 1e3
+            rows_out.append({"kernel": label.replace("<M,", f"<{rows},"), "rows": rows, "bytes": nbytes,
+                             "us": round(us, 2), "gbs": round(gbs, 1), "frac": round(gbs / hbm_peak, 3)})
+            if name in ("qkv", "o", "gateup", "down", "attn"):
+                lb, lt = layer.get(rows, (0, 0.0))
+                layer[rows] = (lb + nbytes, lt + us)
+    summary = {f"layer_m{r}": {"us": round(t, 1), "gbs": round(b_ / t / 1e3, 1), "frac": round(b_ / t / 1e3 / hbm_peak, 3)}
+               for r, (b_, t) in layer.items()}
+    return {"peak_gbs": hbm_peak, "launches": rows_out, **summary}
+
+
 def gemv_traffic_bytes():
     """Measured bytes per launch if gemv.cuh is the captured version, else None."""
     import hashlib
@@ -424,6 +464,7 @@ def main() -> None:
                 "kernel": "gemv_kernel<1, GATE_SILU> (layer gate/up, 2x11008x4096 bf16, 1 row)",
                 "bytes_per_launch": nbytes, "launch_us": kern_ms * 1e3,
                 "peak_source": f"{peak_src} HBM copy (burst)"}
+    kernels = kernel_table(model, w, v, p, stream, hbm_peak)
     model.prefill(v, p)   # the profiling launches clobbered the decode state
     model.sync()
 
@@ -441,7 +482,7 @@ def main() -> None:
             "config": {**workload_config(w), "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                        "arithmetic": "fp32 FMA on bf16 weights, fp32 activations and KV cache"},
             "e2e": e2e, "gpu_launches": int(args.steps * (pre_l + dec_l)),
-            "roofline": roofline, "clocks": clk,
+            "roofline": roofline, "kernels": kernels, "clocks": clk,
             "prefill_ms": statistics.median(prefill_ms), "decode_ms": dec_ms,
             "prefill_roofline": {"bound": "tensor", "kernel": "tc_gemm_kernel (all prefill projections) + prefill attention",
                                  "achieved": prefill_flops(w) / (statistics.median(prefill_ms) / 1e3) / 1e12,

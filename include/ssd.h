@@ -244,8 +244,10 @@ SSD_API ssd_status ssd_lm_head_static(const void* lm_head, const void* final_nor
  * of one weight-streaming projection (the GEMV kernel with its fused
  * epilogue) over `rows` activation rows, with whatever activations the ctx
  * holds.  which: 0 QKV, 1 o_proj, 2 gate/up, 3 down (of `layer`), 4 LM head,
- * 5 imitation FC1, 6 imitation FC2.  *bytes receives the algorithmic bytes one
- * launch moves (weights + activation rows in + results out).  Clobbers the
+ * 5 imitation FC1, 6 imitation FC2, 7 the split-KV attention of `layer` for
+ * query rows kv_len .. kv_len+rows-1 over the cache as it stands (waits for
+ * the stream once to read kv_len).  *bytes receives the algorithmic bytes one
+ * launch moves (weights or K/V + activation rows in + results out).  Clobbers the
  * decode state (activations, cache rows at kv_len..kv_len+rows-1): call
  * ssd_prefill before decoding again.  async. */
 SSD_API ssd_status ssd_profile_projection(ssd_ctx* ctx, int which, int layer, int rows, int reps, int64_t* bytes);

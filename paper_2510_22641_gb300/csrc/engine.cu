@@ -122,7 +122,6 @@ struct ssd_ctx {
   cudaStream_t us = nullptr, cs = nullptr;
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
   bool use_pdl = true;
-  int pf_dist = 0;  // GEMV units prefetched into L2 ahead of the shared-memory ring
   std::map<int, cudaGraphExec_t> decode_graphs, draft_graphs, verify_graphs, step_graphs;
   // Diagnostic: drive the decode loop from the host with one plain graph per
   // step (ncu cannot profile kernels of graphs that hold conditional nodes).
@@ -278,7 +277,6 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   p.counters = c->counters;
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
-  p.pf_dist = c->pf_dist;
   cudaError_t r;
   ++c->launch_counter;
   switch (e) {
@@ -1160,7 +1158,6 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (prop.major != 10) return fail(c, SSD_ERR_UNSUPPORTED, "needs a Blackwell sm_103 device, got sm_%d%d",
                                     prop.major, prop.minor);
   c->num_sms = prop.multiProcessorCount;
-  if (const char* e = getenv("SSD_GEMV_PREFETCH")) c->pf_dist = atoi(e) < 0 ? 0 : atoi(e);
   if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
   if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) < 1 ? 1 : (atoi(e) > 3 ? 3 : atoi(e));
   if (const char* e = getenv("SSD_PREFILL")) c->prefill_rows = strcmp(e, "rows") == 0;
@@ -1657,7 +1654,6 @@ ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float
   p.counters = c->counters;
   p.st = c->op_st;
   p.eps = c->cfg.rms_eps;
-  p.pf_dist = c->pf_dist;
   ++c->launch_counter;
   CK(gemv_launch_head(rows, c->head.maps, p, c->head.grid, c->cs, false));
   CKS(leave(c));
@@ -1669,8 +1665,21 @@ ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float
 ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, int reps, int64_t* bytes) {
   if (!c) return SSD_ERR_INVALID_ARG;
   if (rows < 1 || rows > kMaxVerifyRows || reps < 1) return fail(c, SSD_ERR_INVALID_ARG, "rows / reps");
-  if (which < 0 || which > 6 || layer < 0 || layer >= c->cfg.n_layers)
+  if (which < 0 || which > 7 || layer < 0 || layer >= c->cfg.n_layers)
     return fail(c, SSD_ERR_INVALID_ARG, "which / layer");
+  if (which == 7) {  // split-KV attention of `layer` for rows kv_len .. kv_len+rows-1
+    CK(cudaStreamSynchronize(c->cs));
+    int kv = 0;
+    CK(cudaMemcpy(&kv, reinterpret_cast<char*>(c->st) + offsetof(DevState, kv_len), sizeof(int),
+                  cudaMemcpyDeviceToHost));
+    if (kv < 0 || kv + rows > c->cfg.max_seq) return fail(c, SSD_ERR_INVALID_ARG, "kv_len %d + rows past max_seq", kv);
+    const int64_t qd = static_cast<int64_t>(c->cfg.n_heads) * c->cfg.head_dim;
+    if (bytes) *bytes = 2 * (kv + rows) * qd * 4 + 2 * static_cast<int64_t>(rows) * qd * 4;  // K, V; q in, o out
+    CKS(enter(c));
+    for (int r = 0; r < reps; ++r) CKS(attention(c, layer, rows, 0));
+    c->prefilled = false;
+    return leave(c);
+  }
   if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))
     return fail(c, SSD_ERR_INVALID_ARG, "imitation projections need SSD_IN_MLP2 and rows == 1");
   const int d = c->dp;

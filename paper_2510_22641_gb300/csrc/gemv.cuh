@@ -67,7 +67,6 @@ struct GemvParams {
   unsigned* counters;   // [n_rt]
   DevState* st;
   int pos_off;          // row m sits at position st->kv_len + pos_off + m
-  int pf_dist;          // units prefetched into L2 ahead of the shared-memory ring
   // QKV
   float* q_out;
   int q_stride;

@@ -150,7 +150,7 @@ class SSDModel:
         """ssd_lm_head: argmax of W_lm RMSNorm_f(x) per row (x fp32 [rows][d_model] on the device)."""
         self._call("ssd_lm_head", x.data_ptr(), x.shape[0], tok.data_ptr(), _ptr(logits))
 
-    PROJECTIONS = {"qkv": 0, "o": 1, "gateup": 2, "down": 3, "head": 4, "in1": 5, "in2": 6}
+    PROJECTIONS = {"qkv": 0, "o": 1, "gateup": 2, "down": 3, "head": 4, "in1": 5, "in2": 6, "attn": 7}
 
     def profile_projection(self, which: str, layer: int = 0, rows: int = 1, reps: int = 1) -> int:
         """Enqueue reps launches of one projection kernel; returns algorithmic bytes per launch."""

@@ -329,3 +329,36 @@ def test_tensor_core_prefill_matches_row_prefill_and_oracle(case, monkeypatch):
     if t2[0] != int(np.argmax(ref_logits)):
         from tests.parity import margin
         assert margin(ref_logits) < 1e-2
+
+
+def test_profile_projection_bytes_and_state_recovery(tiny_model):
+    """The single-kernel timing entry point reports each kernel's algorithmic bytes, raises no
+    device error, and a prefill afterwards restores the decode exactly."""
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=0.2)
+    set_scale(model, w)
+    before, _, _ = gpu_decode(model, w, 4, capture=False)
+    sh = w.shape
+    d, qd, ff, V = sh.d_model, sh.n_heads * sh.head_dim, sh.d_ff, sh.vocab
+    kv = w.prompt_len
+    for rows in (1, 5):
+        expect = {
+            "qkv": 3 * qd * d * 2 + rows * d * 4 + d * 2 + rows * (qd * 4 + 2 * qd * 2),
+            "o": d * qd * 2 + rows * qd * 4 + 2 * rows * d * 4,
+            "gateup": 2 * ff * d * 2 + rows * d * 4 + d * 2 + rows * ff * 4,
+            "down": d * ff * 2 + rows * ff * 4 + 2 * rows * d * 4,
+            "head": V * d * 2 + rows * d * 4 + d * 2 + rows * 4,
+            "attn": 2 * (kv + rows) * qd * 4 + 2 * rows * qd * 4,
+        }
+        if rows == 1:
+            h = w.in_hidden
+            expect["in1"] = h * d * 2 + d * 4 + d * 2 + h * 4
+            expect["in2"] = d * h * 2 + h * 4 + 2 * d * 4
+        for name, b in expect.items():
+            model.prefill(*device_inputs(w)[2:])
+            assert model.profile_projection(name, layer=sh.n_layers - 1, rows=rows, reps=2) == b, (name, rows)
+            model.sync()
+    with pytest.raises(RuntimeError):
+        model.profile_projection("in1", rows=2)
+    after, _, _ = gpu_decode(model, w, 4, capture=False)
+    assert after == before
