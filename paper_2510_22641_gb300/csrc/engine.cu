@@ -158,6 +158,7 @@ struct ssd_ctx {
   uint8_t* fwd_btiles = nullptr;  // [kFwdBSlots][fwd_bslot] B operands written by producer epilogues
   long long fwd_bslot = 0;
   unsigned long long* fwd_trace = nullptr;  // SSD_FWD_TRACE=<file>: timeline of the last launch
+  std::string gemv_trace_path;  // SSD_GEMV_TRACE=<file>: per-CTA timeline of ssd_profile_projection's last launch
   std::string fwd_trace_path;
   int fwd_trace_phases = 0;
   // debug logits capture
@@ -1164,6 +1165,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (const char* e = getenv("SSD_DECODE")) c->use_fwd = strcmp(e, "fwd") == 0;
   if (const char* e = getenv("SSD_FWD_COOP")) c->fwd_coop = atoi(e) != 0;
   if (const char* e = getenv("SSD_FWD_TRACE")) c->fwd_trace_path = e;
+  if (const char* e = getenv("SSD_GEMV_TRACE")) c->gemv_trace_path = e;
   if (const char* e = getenv("SSD_GEMV_SMALL")) {  // "<row tiles>,<ctas per SM>"
     c->small_site_rt = atoi(e);
     if (const char* comma = strchr(e, ',')) c->small_site_ctas = atoi(comma + 1) < 1 ? 1 : atoi(comma + 1);
@@ -1750,8 +1752,28 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     *bytes = N * site->K * 2 + static_cast<int64_t>(rows) * site->K * 4 + (p.gain ? site->K * 2 : 0) + out_bytes +
              (e == Epi::RESID ? static_cast<int64_t>(rows) * site->N * 4 : 0);
   CKS(enter(c));
-  for (int r = 0; r < reps; ++r) CKS(gemv(c, e, rows, *site, p));
+  unsigned long long* tr = nullptr;
+  if (!c->gemv_trace_path.empty()) {  // diagnostic: timeline of the last launch, written here
+    CK(cudaMalloc(&tr, sizeof(unsigned long long) * kGemvTrace * site->grid));
+    CK(cudaMemsetAsync(tr, 0, sizeof(unsigned long long) * kGemvTrace * site->grid, c->cs));
+  }
+  for (int r = 0; r < reps; ++r) {
+    p.trace = r == reps - 1 ? tr : nullptr;
+    CKS(gemv(c, e, rows, *site, p));
+  }
   c->prefilled = false;
+  if (tr) {
+    std::vector<unsigned long long> h(kGemvTrace * static_cast<size_t>(site->grid));
+    CK(cudaStreamSynchronize(c->cs));
+    CK(cudaMemcpy(h.data(), tr, sizeof(unsigned long long) * h.size(), cudaMemcpyDeviceToHost));
+    CK(cudaFree(tr));
+    if (FILE* f = fopen(c->gemv_trace_path.c_str(), "ab")) {
+      const int hdr[4] = {which, rows, site->grid, kGemvTrace};
+      fwrite(hdr, sizeof(int), 4, f);
+      fwrite(h.data(), sizeof(unsigned long long), h.size(), f);
+      fclose(f);
+    }
+  }
   return leave(c);
 }
 

@@ -47,6 +47,7 @@ constexpr int kHalfN = kTileN / 2;   // gate or up rows of a paired unit
 constexpr int kTileK = 64;           // weight columns per unit (one 128-byte swizzled row)
 constexpr int kNPad = 16;            // activation rows padded to the MMA's N
 constexpr int kStages = 4;
+constexpr int kGemvTrace = 12;  // timeline stamps per CTA
 constexpr int kGemvThreads = 256;
 constexpr int kDrainThreads = 128;   // warps 4..7
 constexpr int kTmemCols = 32;        // two 16-column accumulators
@@ -87,6 +88,12 @@ struct GemvParams {
   int* tok_dst;        // tok_dst[m] = argmax of row m
   float* logits;       // optional [logits_rows][N] capture
   int logits_rows;
+  // optional timeline, [grid][kGemvTrace] %globaltimer stamps per CTA: 0 entry, 1 first weight
+  // copies issued, 2 upstream grid complete, 3 first unit landed, 4 last MMA issued, 5 first
+  // accumulator drained, 6 epilogues done, 7 exit; for the last split tile this CTA owned:
+  // 8 ticket taken, 9 partials summed, 10 its epilogue done, 11 split tiles owned.  Null when
+  // not tracing.
+  unsigned long long* trace;
 };
 
 template <int M>
@@ -318,6 +325,8 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
   const uint32_t tx = kWTileBytes + S::kActBytes + (p.gain ? kTileK * 2 : 0);
 
   pdl_trigger();
+  unsigned long long* tr = p.trace ? p.trace + static_cast<size_t>(c) * kGemvTrace : nullptr;
+  if (tr && tid == 0) tr[0] = globaltimer_ns();
   // After a timed-out wait anywhere in the decode, later kernels do nothing
   // (best-effort read before any copy is issued or TMEM is taken).
   if (*reinterpret_cast<volatile int*>(&p.st->error) & DERR_TIMEOUT) return;
@@ -381,7 +390,9 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         mbar_arrive_expect_tx(&full[i], tx);
         issue_weights(i, u0 + i);  // weights do not depend on the previous kernel
       }
+      if (tr) tr[1] = globaltimer_ns();
       pdl_wait();
+      if (tr) tr[2] = globaltimer_ns();
       for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
       for (int i = npre; i < n_units; ++i) {
         const int s = i % kStages;
@@ -428,6 +439,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
           seg_open = true;
         }
         umma_commit(&empty[s]);  // stage s may be refilled once these MMAs have read it
+        if (tr && i == n_units - 1) tr[4] = globaltimer_ns();
         if (kt == p.n_kt - 1 || i == n_units - 1) {
           umma_commit(&afull[sg & 1]);  // the row tile's accumulator is complete
           ++sg;
@@ -444,6 +456,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         set_error(p.st, DERR_TIMEOUT);
         break;
       }
+      if (tr && i == 0 && ct == 0) tr[3] = globaltimer_ns();
       const float* a = reinterpret_cast<const float*>(smem + S::kA + s * S::kActBytes);
       const __nv_bfloat16* g = reinterpret_cast<const __nv_bfloat16*>(smem + S::kG + s * kTileK * 2);
       uint8_t* bh = smem + S::kB + s * 2 * kBOpBytes;
@@ -521,6 +534,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         break;
       }
       tmem_fence_after();
+      if (tr && sg == 0 && dt == 0) tr[5] = globaltimer_ns();
       float v[kNPad];
       tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kNPad), v);
       tmem_fence_before();
@@ -536,35 +550,41 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
         for (int idx = dt; idx < M * kTileN; idx += kDrainThreads) __stcg(dstp + idx, outb[idx]);
-        __threadfence();
+        // Release / acquire through the tile's ticket: the CTA barrier orders every drain thread's
+        // partial stores before thread 0's acq_rel atomic, and the barrier after it orders the
+        // owner's loads after its acquire (no per-thread fences).
         drain_sync();
         const int c_first = unit_owner(rt * p.n_kt, p.units, G);
         const int c_last = unit_owner(rt * p.n_kt + p.n_kt - 1, p.units, G);
         if (dt == 0) {
-          const unsigned prev = atomicAdd(&p.counters[rt], 1u);
+          const unsigned prev = atom_add_acq_rel_gpu(&p.counters[rt], 1u);
           flag[0] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
         }
         drain_sync();
         if (flag[0]) {
-          __threadfence();
-          // sum the partials in CTA order; 16-byte loads of 8 CTAs are issued together,
-          // all rows at once
+          if (tr && dt == 0) {
+            tr[8] = globaltimer_ns();
+            tr[11] += 1;
+          }
+          // Sum the partials in CTA order, all rows at once, 16 CTAs' 16-byte loads in flight.
+          // Every CTA after c_first starts its range inside this tile (slot 2 cc); c_first's slot
+          // depends on whether the tile is its first one.
           const int nsp = c_last - c_first + 1;
+          const int slot0 = 2 * c_first + (unit_begin(c_first, p.units, G) / p.n_kt == rt ? 0 : 1);
+          const float4* part = reinterpret_cast<const float4*>(p.partials);
+          constexpr int kSlotF4 = kMaxRows * kTileN / 4;
           for (int f = dt; f < M * (kTileN / 4); f += kDrainThreads) {
             float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int b0 = 0; b0 < nsp; b0 += 8) {
-              float4 pv[8];
+            for (int b0 = 0; b0 < nsp; b0 += 16) {
+              float4 pv[16];
 #pragma unroll
-              for (int j = 0; j < 8; ++j) {
-                const int cc = c_first + b0 + j;
-                pv[j] = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (b0 + j < nsp) {
-                  const int sl = 2 * cc + (rt == unit_begin(cc, p.units, G) / p.n_kt ? 0 : 1);
-                  pv[j] = __ldcg(reinterpret_cast<const float4*>(p.partials + static_cast<size_t>(sl) * (kMaxRows * kTileN)) + f);
-                }
+              for (int j = 0; j < 16; ++j) {
+                const int k = b0 + j;
+                const int sl = k == 0 ? slot0 : 2 * (c_first + k);
+                pv[j] = k < nsp ? __ldcg(part + static_cast<size_t>(sl) * kSlotF4 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
               }
 #pragma unroll
-              for (int j = 0; j < 8; ++j) {
+              for (int j = 0; j < 16; ++j) {
                 if (b0 + j >= nsp) continue;
                 if (b0 + j == 0) {
                   sum = pv[j];
@@ -579,17 +599,24 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
             reinterpret_cast<float4*>(outb)[f] = sum;
           }
           drain_sync();
+          if (tr && dt == 0) tr[9] = globaltimer_ns();
           gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
           if (dt == 0) p.counters[rt] = 0u;
+          if (tr) {
+            drain_sync();
+            if (dt == 0) tr[10] = globaltimer_ns();
+          }
         }
       }
       drain_sync();
       seg_kt0 = 0;
       ++sg;
     }
+    if (tr && dt == 0) tr[6] = globaltimer_ns();
   }
   tmem_fence_before();
   __syncthreads();
+  if (tr && tid == 0) tr[7] = globaltimer_ns();
   if (warp == 1) {
     tmem_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");
