@@ -5,15 +5,27 @@
 // to keys 0 .. base + m.  Keys are cut into fixed 16 KB chunks at absolute
 // positions (32 keys for head_dim 128, 64 for 64).  Each head is served by one
 // thread-block cluster of kAttnSplit CTAs; CTA r of the cluster takes chunks r,
-// r + kAttnSplit, ... in order: thread 0 brings each chunk's K and V rows
-// (contiguous in the [H][max_seq][Dh] fp32 cache) into shared memory with bulk
-// copies, double-buffered.  Within a chunk, each of the 4 warps owns a fixed
-// quarter of the keys and folds them into its own running softmax state per row
-// (max, sum of exp, unnormalised output), so a chunk costs one CTA barrier.  The
-// cluster then merges the 4 x kAttnSplit states through distributed shared
-// memory, each CTA a slice of the output columns, in (CTA, warp) order.  The chunk grid, the key -> (CTA, warp)
-// assignment and the merge order depend only on key positions, never on M, so
-// each row's output equals the single-row (M = 1) result bitwise.
+// r + kAttnSplit, ... in order, in groups of kAttnBufs chunks: thread 0 brings a
+// group's K and V rows (contiguous in the [H][max_seq][Dh] fp32 cache) into
+// shared memory with bulk copies.  Per group the CTA
+//   1. scores every key of the group for every row (warp w owns a fixed 1/8 of
+//      each chunk's keys, TPK lanes per key with a fixed xor tree),
+//   2. updates each row's running max and sum once for the whole group (one warp
+//      per row; exponentials written back in place of the scores),
+//   3. folds P.V into the warps' output accumulators, rescaled by the row's
+//      running-max change.
+// All warps share one running max per row, so the CTA's state is the warps'
+// accumulators summed in warp order.  The cluster then merges the kAttnSplit CTA
+// states through distributed shared memory in CTA order, each CTA a slice of the
+// output columns.  The chunk grid, the grouping, the key -> (CTA, warp)
+// assignment and every summation order depend only on key positions, never on
+// M, so each row's output equals the single-row (M = 1) result bitwise.
+//
+// With prefetch_old set, the launch before this one triggered its dependents
+// only after its own upstream grid had completed, so everything older than that
+// launch is complete here: the chunks holding only keys below base (written by
+// earlier launches) are fetched before the wait on the upstream grid, and only
+// q and the chunk with this step's keys after it.
 #pragma once
 
 #include <cooperative_groups.h>
@@ -22,8 +34,10 @@
 
 namespace ssd {
 
-constexpr int kAttnThreads = 128;
+constexpr int kAttnWarps = 8;
+constexpr int kAttnThreads = 32 * kAttnWarps;
 constexpr int kAttnSplit = 8;  // CTAs per head (cluster size)
+constexpr int kAttnBufs = 3;   // chunks per group = {K, V} buffers per CTA
 
 struct AttnParams {
   const float* q;  // [M][q_stride], rotated queries
@@ -35,57 +49,87 @@ struct AttnParams {
   DevState* st;
   int pos_off;
   int n_heads, max_seq;
-  float scale;  // 1/sqrt(Dh)
+  float scale;       // 1/sqrt(Dh)
+  int prefetch_old;  // the previous launch triggered after its own upstream completed (see above)
+  // optional timeline, [n_heads * kAttnSplit][8] %globaltimer stamps per CTA: 0 entry, 1 upstream
+  // grid complete, 2 first chunk landed, 3 last chunk folded, 4 states published (cluster barrier
+  // passed), 5 merge done, 6 exit, 7 chunks taken.  Null when not tracing.
+  unsigned long long* trace;
+};
+
+template <int DH>
+struct AttnGeo {
+  static constexpr int KPC = kAttnChunkBytes / (DH * 4);  // keys per chunk (32 or 64)
+  static constexpr int KPW = KPC / kAttnWarps;            // keys per warp and chunk (4 or 8)
+  static constexpr int TPK = 32 / KPW;                    // lanes per key (8 or 4)
+  static constexpr int DPP = DH / TPK;                    // key dimensions per lane in the scores
+  static constexpr int NF = DPP / 4;                      // 16-byte loads per lane and row
+  static constexpr int DPL = DH / 32;                     // output dimensions per lane (4 or 2)
+  static constexpr int GK = kAttnBufs * KPC;              // keys per group
+  static constexpr int KPL = GK / 32;                     // keys per lane in the row statistics
+  static_assert(NF == 4 && KPW % 4 == 0 && KPW * kAttnWarps == KPC && GK % 32 == 0, "chunk split");
 };
 
 template <int M, int DH>
 struct AttnSmem {
-  static constexpr int kKV = kAttnChunkBytes;                       // one K (or V) chunk
-  static constexpr int kQ = 0;                                      // q rows [M][DH]
-  static constexpr int kBuf0 = (kQ + M * DH * 4 + 15) & ~15;        // two {K, V} buffers
-  static constexpr int kFin = kBuf0 + 4 * kKV;                      // warp states [4][M][DH + 2]
-  static constexpr int kPw = kFin + 4 * M * (DH + 2) * 4;           // per-warp probabilities [4][rows][KPW]
-  static constexpr int kWq = kPw + 4 * kAttnMaxRows * (AttnWarp<DH>::KPW) * 4;  // merge weights [M][32], sums [M]
-  static constexpr int kBar = (kWq + M * 33 * 4 + 7) & ~7;
-  static constexpr int kTotal = kBar + 3 * 8;
+  using G = AttnGeo<DH>;
+  static constexpr int kKV = kAttnChunkBytes;                    // one K (or V) chunk
+  static constexpr int kQ = 0;                                   // q rows [M][DH]
+  static constexpr int kBuf0 = (kQ + M * DH * 4 + 127) & ~127;   // kAttnBufs {K, V} buffers
+  static constexpr int kWs = kBuf0;  // warp accumulators [kAttnWarps][M][DH], over the buffers after the last group
+  static_assert(kAttnWarps * M * DH * 4 <= kAttnBufs * 2 * kKV, "warp accumulators fit the chunk buffers");
+  static constexpr int kS = kBuf0 + kAttnBufs * 2 * kKV;         // scores, then probabilities [M][GK]
+  static constexpr int kRow = kS + M * G::GK * 4;                // per row: running max, sum, rescale, - [M][4]
+  static constexpr int kCs = kRow + M * 4 * 4;                   // CTA state [M][DH + 2] (read by the cluster)
+  static constexpr int kMg = kCs + M * (DH + 2) * 4;             // merge: [M][kAttnSplit] (max, sum)
+  static constexpr int kWq = kMg + M * kAttnSplit * 2 * 4;       // merge weights [M][kAttnSplit], totals [M]
+  static constexpr int kBar = (kWq + M * (kAttnSplit + 1) * 4 + 7) & ~7;
+  static constexpr int kTotal = kBar + (kAttnBufs + 1) * 8;
 };
 
 template <int M, int DH>
-__global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThreads)
+__global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThreads, 2)
     attn_kernel(const AttnParams p) {
   namespace cg = cooperative_groups;
   using S = AttnSmem<M, DH>;
-  using AW = AttnWarp<DH>;
-  constexpr int KPC = AW::KPC, DPL = AW::DPL;
+  using G = AttnGeo<DH>;
+  constexpr int KPC = G::KPC, KPW = G::KPW, TPK = G::TPK, DPP = G::DPP, NF = G::NF, DPL = G::DPL;
+  constexpr int GK = G::GK, E = DH + 2;
   static_assert(M <= kAttnMaxRows, "query rows");
   extern __shared__ __align__(128) uint8_t smem[];
   float* Qs = reinterpret_cast<float*>(smem + S::kQ);
-  float* fin = reinterpret_cast<float*>(smem + S::kFin);
-  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  float* ss = reinterpret_cast<float*>(smem + S::kS);
+  float* rowst = reinterpret_cast<float*>(smem + S::kRow);
+  float* ws = reinterpret_cast<float*>(smem + S::kWs);
+  float* cst = reinterpret_cast<float*>(smem + S::kCs);
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem + S::kBar);  // [kAttnBufs] chunks, then q
   cg::cluster_group cluster = cg::this_cluster();
   const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
   const int rank = static_cast<int>(cluster.block_rank());
   const int h = blockIdx.y;
 
   pdl_trigger();
+  unsigned long long* tr = p.trace ? p.trace + (static_cast<size_t>(h) * kAttnSplit + rank) * 8 : nullptr;
+  if (tr && tid == 0) tr[0] = globaltimer_ns();
   if (tid == 0) {
-    mbar_init(&bar[0], 1);
-    mbar_init(&bar[1], 1);
-    mbar_init(&bar[2], 1);
+    for (int b = 0; b <= kAttnBufs; ++b) mbar_init(&bar[b], 1);
     fence_mbar_init();
   }
-  __syncthreads();
-  pdl_wait();
-  int base = __ldcg(&p.st->kv_len) + p.pos_off;
-  bool bad = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
-  if (base < 0 || base + M > p.max_seq) {
-    if (tid == 0 && rank == 0 && h == 0) set_error(p.st, DERR_POS);
-    bad = true;
+  if (tid < M) {
+    rowst[4 * tid] = -INFINITY;
+    rowst[4 * tid + 1] = 0.f;
   }
-  const int n_keys = bad ? 0 : base + M;  // keys 0 .. base+M-1 exist for the last row
-  const int n_chunks = (n_keys + KPC - 1) / KPC;
-  const int my_chunks = n_chunks > rank ? (n_chunks - rank + kAttnSplit - 1) / kAttnSplit : 0;
+  __syncthreads();
 
+  int base = 0, n_keys = 0, my_chunks = 0;
+  bool bad = false;
+  auto geometry = [&]() {
+    base = __ldcg(&p.st->kv_len) + p.pos_off;
+    bad = base < 0 || base + M > p.max_seq;
+    n_keys = bad ? 0 : base + M;  // keys 0 .. base+M-1 exist for the last row
+    const int n_chunks = (n_keys + KPC - 1) / KPC;
+    my_chunks = n_chunks > rank ? (n_chunks - rank + kAttnSplit - 1) / kAttnSplit : 0;
+  };
   auto issue = [&](int buf, int c) {
     const int j0 = c * KPC, nk = min(KPC, n_keys - j0);
     uint8_t* b = smem + S::kBuf0 + buf * 2 * S::kKV;
@@ -95,82 +139,246 @@ __global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThread
     bulk_load(b, p.k_cache + off, kv_bytes, &bar[buf]);
     bulk_load(b + S::kKV, p.v_cache + off, kv_bytes, &bar[buf]);
   };
+  int issued = 0;  // thread 0: chunks of the first group already requested
+  if (p.prefetch_old) {
+    geometry();
+    if (tid == 0)
+      for (; issued < kAttnBufs && issued < my_chunks; ++issued) {
+        const int c = rank + issued * kAttnSplit;
+        if ((c + 1) * KPC > base) break;  // holds keys the upstream grid writes
+        issue(issued, c);
+      }
+  }
+  pdl_wait();
+  if (tr && tid == 0) tr[1] = globaltimer_ns();
+  if (!p.prefetch_old) geometry();
+  if (bad && tid == 0 && rank == 0 && h == 0) set_error(p.st, DERR_POS);
+  const bool timed_out = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
   if (tid == 0 && my_chunks > 0) {
-    mbar_arrive_expect_tx(&bar[2], M * DH * 4);
+    mbar_arrive_expect_tx(&bar[kAttnBufs], M * DH * 4);
 #pragma unroll
     for (int m = 0; m < M; ++m)
-      bulk_load(Qs + m * DH, p.q + static_cast<size_t>(m) * p.q_stride + h * DH, DH * 4, &bar[2]);
-    issue(0, rank);
+      bulk_load(Qs + m * DH, p.q + static_cast<size_t>(m) * p.q_stride + h * DH, DH * 4, &bar[kAttnBufs]);
+    for (; issued < kAttnBufs && issued < my_chunks; ++issued) issue(issued, rank + issued * kAttnSplit);
   }
 
-  AW st;
-  st.init();
+  const int kk = lane / TPK, part = lane - kk * TPK, rot = ((lane & 7) >> 1) & 3;
+  const int jw = w * KPW + kk;  // this lane's key within a chunk (scores)
+  float acc[M][DPL];
+#pragma unroll
+  for (int m = 0; m < M; ++m)
+#pragma unroll
+    for (int e = 0; e < DPL; ++e) acc[m][e] = 0.f;
   bool ok = true;
-  if (my_chunks > 0 && !mbar_wait(&bar[2], 0)) ok = false;
-  for (int i = 0; ok && i < my_chunks; ++i) {
-    const int c = rank + i * kAttnSplit, buf = i & 1;
-    const int j0 = c * KPC, nk = min(KPC, n_keys - j0);
-    if (tid == 0 && i + 1 < my_chunks) issue(buf ^ 1, c + kAttnSplit);
-    if (!mbar_wait(&bar[buf], static_cast<uint32_t>(i >> 1) & 1u)) {
-      ok = false;
-      break;
+  if (my_chunks > 0 && !mbar_wait(&bar[kAttnBufs], 0)) ok = false;
+  for (int g0 = 0; ok && g0 < my_chunks; g0 += kAttnBufs) {
+    const int gn = min(kAttnBufs, my_chunks - g0);
+    const uint32_t parity = static_cast<uint32_t>(g0 / kAttnBufs) & 1u;
+    // 1. scores of the group's keys for every row (-inf where masked): the lane's key slices of
+    // all the group's chunks are held in registers, so each q row is read once per group
+    float kv[kAttnBufs][DPP];
+    int nkc[kAttnBufs], j0c[kAttnBufs];
+#pragma unroll
+    for (int i = 0; i < kAttnBufs; ++i) {
+      j0c[i] = (rank + (g0 + i) * kAttnSplit) * KPC;
+      nkc[i] = i < gn ? min(KPC, n_keys - j0c[i]) : 0;
+      if (i >= gn) continue;
+      if (!mbar_wait(&bar[i], parity)) {
+        ok = false;
+        continue;
+      }
+      if (tr && tid == 0 && g0 == 0 && i == 0) tr[2] = globaltimer_ns();
+      const float* kr = reinterpret_cast<const float*>(smem + S::kBuf0 + i * 2 * S::kKV) + jw * DH + part * DPP;
+#pragma unroll
+      for (int e = 0; e < NF; ++e) {
+        const float4 t = *reinterpret_cast<const float4*>(kr + ((e + rot) & (NF - 1)) * 4);
+        kv[i][4 * e] = t.x;
+        kv[i][4 * e + 1] = t.y;
+        kv[i][4 * e + 2] = t.z;
+        kv[i][4 * e + 3] = t.w;
+      }
     }
-    const float* Ks = reinterpret_cast<const float*>(smem + S::kBuf0 + buf * 2 * S::kKV);
-    st.chunk(Ks, Ks + KPC * DH, Qs, M, j0, nk, base, p.scale, w, lane,
-             reinterpret_cast<float*>(smem + S::kPw) + w * kAttnMaxRows * AW::KPW);
-    __syncthreads();  // buffer buf is refilled by the next iteration's copy
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      const float* qr = Qs + m * DH + part * DPP;
+      float4 q4[NF];
+#pragma unroll
+      for (int e = 0; e < NF; ++e) q4[e] = *reinterpret_cast<const float4*>(qr + ((e + rot) & (NF - 1)) * 4);
+#pragma unroll
+      for (int i = 0; i < kAttnBufs; ++i) {
+        if (i >= gn) break;
+        float a = 0.f;
+#pragma unroll
+        for (int e = 0; e < NF; ++e) {
+          a = fmaf(kv[i][4 * e], q4[e].x, a);
+          a = fmaf(kv[i][4 * e + 1], q4[e].y, a);
+          a = fmaf(kv[i][4 * e + 2], q4[e].z, a);
+          a = fmaf(kv[i][4 * e + 3], q4[e].w, a);
+        }
+#pragma unroll
+        for (int off = 1; off < TPK; off <<= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
+        if (part == 0) {
+          const bool vis = jw < nkc[i] && j0c[i] + jw <= base + m;
+          ss[m * GK + i * KPC + jw] = vis ? a * p.scale : -INFINITY;
+        }
+      }
+    }
+    __syncthreads();
+    if (!ok) break;
+    // 2. per row (one warp each): running max and sum over the group, exponentials in place
+    for (int m = w; m < M; m += kAttnWarps) {
+      float* sr = ss + m * GK;
+      const int nkg = gn * KPC;
+      float v[G::KPL];
+      float gm = -INFINITY;
+#pragma unroll
+      for (int t = 0; t < G::KPL; ++t) {
+        const int idx = lane + 32 * t;
+        v[t] = idx < nkg ? sr[idx] : -INFINITY;
+        gm = fmaxf(gm, v[t]);
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) gm = fmaxf(gm, __shfl_xor_sync(0xffffffffu, gm, off));
+      const float rm = rowst[4 * m], nm = fmaxf(rm, gm);
+      float ls = 0.f;
+#pragma unroll
+      for (int t = 0; t < G::KPL; ++t) {
+        const int idx = lane + 32 * t;
+        const float pj = v[t] == -INFINITY ? 0.f : expf(v[t] - nm);
+        if (idx < nkg) sr[idx] = pj;
+        ls += pj;
+      }
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) ls += __shfl_xor_sync(0xffffffffu, ls, off);
+      if (lane == 0) {
+        const float so = rm == -INFINITY ? 0.f : expf(rm - nm);
+        rowst[4 * m] = nm;
+        rowst[4 * m + 1] = rowst[4 * m + 1] * so + ls;
+        rowst[4 * m + 2] = so;
+      }
+    }
+    __syncthreads();
+    // 3. P.V over this warp's keys of the group, onto the rescaled accumulators
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+      const float so = rowst[4 * m + 2];
+#pragma unroll
+      for (int e = 0; e < DPL; ++e) acc[m][e] *= so;
+    }
+    for (int i = 0; i < gn; ++i) {
+      const int nk = nkc[i];
+      const float* vs = reinterpret_cast<const float*>(smem + S::kBuf0 + i * 2 * S::kKV + S::kKV);
+      float pt[M][KPW];  // this warp's probabilities of the chunk, 16-byte broadcasts
+#pragma unroll
+      for (int m = 0; m < M; ++m)
+#pragma unroll
+        for (int t = 0; t < KPW; t += 4) {
+          const float4 p4 = *reinterpret_cast<const float4*>(ss + m * GK + i * KPC + w * KPW + t);
+          pt[m][t] = p4.x;
+          pt[m][t + 1] = p4.y;
+          pt[m][t + 2] = p4.z;
+          pt[m][t + 3] = p4.w;
+        }
+#pragma unroll
+      for (int t = 0; t < KPW; ++t) {
+        const int jj = w * KPW + t;
+        if (jj >= nk) break;  // rows past the chunk's keys hold stale shared memory
+        const float* vr = vs + jj * DH + lane * DPL;
+        float vv[DPL];
+        if constexpr (DPL == 4) {
+          const float4 v4 = *reinterpret_cast<const float4*>(vr);
+          vv[0] = v4.x;
+          vv[1] = v4.y;
+          vv[2] = v4.z;
+          vv[3] = v4.w;
+        } else {
+          const float2 v2 = *reinterpret_cast<const float2*>(vr);
+          vv[0] = v2.x;
+          vv[1] = v2.y;
+        }
+#pragma unroll
+        for (int m = 0; m < M; ++m)
+#pragma unroll
+          for (int e = 0; e < DPL; ++e) acc[m][e] = fmaf(pt[m][t], vv[e], acc[m][e]);
+      }
+    }
+    __syncthreads();  // buffers and scores are free again
+    if (tid == 0)
+      for (int i = 0; i < kAttnBufs && g0 + kAttnBufs + i < my_chunks; ++i)
+        issue(i, rank + (g0 + kAttnBufs + i) * kAttnSplit);
   }
   if (!ok) set_error(p.st, DERR_TIMEOUT);
+  if (tr && tid == 0) {
+    tr[3] = globaltimer_ns();
+    tr[7] = static_cast<unsigned long long>(my_chunks);
+  }
 
-  // publish the warps' states; the cluster then merges the 4 x kAttnSplit states of each row.
-  // State s = 4 * CTA + warp.  Per row, one warp forms the weights exp(mx_s - max) and their sum
-  // with fixed shuffle trees; then CTA r combines columns [r * DH / kAttnSplit, (r + 1) * DH /
-  // kAttnSplit) of all rows, summing the states in s order.  None of it depends on M.
+  // this CTA's state per row: the warps' accumulators summed in warp order (the chunk buffers
+  // are free: every chunk was waited for and folded before the last barrier)
 #pragma unroll
-  for (int m = 0; m < M; ++m) {
-    float* e = fin + (w * M + m) * (DH + 2);
+  for (int m = 0; m < M; ++m)
 #pragma unroll
-    for (int d = 0; d < DPL; ++d) e[lane * DPL + d] = st.o[m][d];
-    if (lane == 0) {
-      e[DH] = st.mx[m];
-      e[DH + 1] = st.l[m];
+    for (int e = 0; e < DPL; ++e) ws[(w * M + m) * DH + lane * DPL + e] = acc[m][e];
+  __syncthreads();
+  for (int idx = tid; idx < M * DH; idx += kAttnThreads) {
+    const int m = idx / DH, d = idx - m * DH;
+    float O = 0.f;
+#pragma unroll
+    for (int q = 0; q < kAttnWarps; ++q) O += ws[(q * M + m) * DH + d];
+    cst[m * E + d] = O;
+    if (d == 0) {
+      cst[m * E + DH] = rowst[4 * m];
+      cst[m * E + DH + 1] = rowst[4 * m + 1];
     }
   }
   cluster.sync();
-  static_assert(4 * kAttnSplit == 32, "one merge lane per state");
-  if (!bad) {
-    float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][32]
-    float* ls = wq + M * 32;                              // [M]
-    const float* fs = cluster.map_shared_rank(fin, lane >> 2);
-    for (int m = w; m < M; m += 4) {
-      const float* e = fs + ((lane & 3) * M + m) * (DH + 2);
-      const float mq = e[DH], lq = e[DH + 1];
-      float mt = mq;
+  if (tr && tid == 0) tr[4] = globaltimer_ns();
+
+  // the cluster's CTA states combined in CTA order; CTA r writes columns [r * DS, (r + 1) * DS)
+  if (!bad && !timed_out) {
+    float* mg = reinterpret_cast<float*>(smem + S::kMg);  // [M][kAttnSplit][2] (max, sum)
+    float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][kAttnSplit] weights, then [M] totals
+    if (tid < M * kAttnSplit) {
+      const int m = tid / kAttnSplit, q = tid - m * kAttnSplit;
+      const float* e = cluster.map_shared_rank(cst, q) + m * E;
+      mg[2 * tid] = e[DH];
+      mg[2 * tid + 1] = e[DH + 1];
+    }
+    __syncthreads();
+    if (tid < M) {
+      const float* g = mg + tid * kAttnSplit * 2;
+      float mt = -INFINITY;
 #pragma unroll
-      for (int o = 16; o; o >>= 1) mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
-      const float g = mq == -INFINITY ? 0.f : expf(mq - mt);
-      float L = g * lq;
+      for (int q = 0; q < kAttnSplit; ++q) mt = fmaxf(mt, g[2 * q]);
+      float L = 0.f;
 #pragma unroll
-      for (int o = 16; o; o >>= 1) L += __shfl_xor_sync(0xffffffffu, L, o);
-      wq[m * 32 + lane] = g;
-      if (lane == 0) ls[m] = L;
+      for (int q = 0; q < kAttnSplit; ++q) {
+        const float gq = g[2 * q] == -INFINITY ? 0.f : expf(g[2 * q] - mt);
+        wq[tid * kAttnSplit + q] = gq;
+        L = fmaf(gq, g[2 * q + 1], L);
+      }
+      wq[M * kAttnSplit + tid] = L;
     }
     __syncthreads();
     constexpr int DS = DH / kAttnSplit;
     for (int idx = tid; idx < M * DS; idx += kAttnThreads) {
       const int m = idx / DS, d = rank * DS + (idx - m * DS);
-      float v[32];
+      float v[kAttnSplit];
 #pragma unroll
-      for (int s = 0; s < 32; ++s)
-        v[s] = cluster.map_shared_rank(fin, s >> 2)[((s & 3) * M + m) * (DH + 2) + d];
+      for (int q = 0; q < kAttnSplit; ++q) v[q] = cluster.map_shared_rank(cst, q)[m * E + d];
       float O = 0.f;
 #pragma unroll
-      for (int s = 0; s < 32; ++s) O = fmaf(wq[m * 32 + s], v[s], O);
-      const float L = ls[m];
+      for (int q = 0; q < kAttnSplit; ++q) O = fmaf(wq[m * kAttnSplit + q], v[q], O);
+      const float L = wq[M * kAttnSplit + m];
       p.o[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
     }
   }
-  cluster.sync();  // keep every CTA's shared memory alive until rank 0 has read it
+  if (tr) {
+    __syncthreads();
+    if (tid == 0) tr[5] = globaltimer_ns();
+  }
+  cluster.sync();  // keep every CTA's shared memory alive until the others have read it
+  if (tr && tid == 0) tr[6] = globaltimer_ns();
 }
 
 }  // namespace ssd

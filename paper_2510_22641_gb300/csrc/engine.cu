@@ -158,7 +158,7 @@ struct ssd_ctx {
   uint8_t* fwd_btiles = nullptr;  // [kFwdBSlots][fwd_bslot] B operands written by producer epilogues
   long long fwd_bslot = 0;
   unsigned long long* fwd_trace = nullptr;  // SSD_FWD_TRACE=<file>: timeline of the last launch
-  std::string gemv_trace_path;  // SSD_GEMV_TRACE=<file>: per-CTA timeline of ssd_profile_projection's last launch
+  std::string gemv_trace_path;  // SSD_GEMV_TRACE=<file>: per-CTA timeline of ssd_profile_projection's last launch (GEMV or attention)
   std::string fwd_trace_path;
   int fwd_trace_phases = 0;
   // debug logits capture
@@ -321,8 +321,12 @@ static cudaError_t attn_attrs() {
   return attn_attr_m<9>();
 }
 
-static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off) {
+// prefetch_old: the launch before is the layer's QKV projection with a late trigger.
+static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch_old,
+                            unsigned long long* trace = nullptr) {
   AttnParams a{};
+  a.trace = trace;
+  a.prefetch_old = prefetch_old ? 1 : 0;
   a.q = c->qb;
   a.q_stride = c->qp;
   a.k_cache = c->kc + l * c->layer_kv;
@@ -368,8 +372,9 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   p.head_dim = c->cfg.head_dim;
   p.max_seq = c->cfg.max_seq;
   p.rope_cs = c->rope;
+  p.late_trigger = 1;
   CKS(gemv(c, Epi::QKV, M, c->layers[l].qkv, p));
-  CKS(attention(c, l, M, pos_off));
+  CKS(attention(c, l, M, pos_off, true));
   p = GemvParams{};
   p.x = c->ob;
   p.x_stride = c->qp;
@@ -1678,8 +1683,26 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     const int64_t qd = static_cast<int64_t>(c->cfg.n_heads) * c->cfg.head_dim;
     if (bytes) *bytes = 2 * (kv + rows) * qd * 4 + 2 * static_cast<int64_t>(rows) * qd * 4;  // K, V; q in, o out
     CKS(enter(c));
-    for (int r = 0; r < reps; ++r) CKS(attention(c, layer, rows, 0));
+    const size_t ntr = static_cast<size_t>(8) * kAttnSplit * c->cfg.n_heads;
+    unsigned long long* tr = nullptr;
+    if (!c->gemv_trace_path.empty()) {  // diagnostic: timeline of the last launch, written here
+      CK(cudaMalloc(&tr, sizeof(unsigned long long) * ntr));
+      CK(cudaMemsetAsync(tr, 0, sizeof(unsigned long long) * ntr, c->cs));
+    }
+    for (int r = 0; r < reps; ++r) CKS(attention(c, layer, rows, 0, false, r == reps - 1 ? tr : nullptr));
     c->prefilled = false;
+    if (tr) {
+      std::vector<unsigned long long> h(ntr);
+      CK(cudaStreamSynchronize(c->cs));
+      CK(cudaMemcpy(h.data(), tr, sizeof(unsigned long long) * ntr, cudaMemcpyDeviceToHost));
+      CK(cudaFree(tr));
+      if (FILE* f = fopen(c->gemv_trace_path.c_str(), "ab")) {
+        const int hdr[4] = {which, rows, kAttnSplit * c->cfg.n_heads, 8};
+        fwrite(hdr, sizeof(int), 4, f);
+        fwrite(h.data(), sizeof(unsigned long long), ntr, f);
+        fclose(f);
+      }
+    }
     return leave(c);
   }
   if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))

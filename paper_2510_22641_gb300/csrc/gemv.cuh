@@ -94,6 +94,11 @@ struct GemvParams {
   // 8 ticket taken, 9 partials summed, 10 its epilogue done, 11 split tiles owned.  Null when
   // not tracing.
   unsigned long long* trace;
+  // Trigger the dependent launch only once the upstream grid has completed (from the weight
+  // producer, after its wait), so that everything older than this launch is complete when the
+  // dependent grid starts: the split-KV attention after the QKV projection reads older cache rows
+  // before its own wait.
+  int late_trigger;
 };
 
 template <int M>
@@ -324,7 +329,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const uint32_t tx = kWTileBytes + S::kActBytes + (p.gain ? kTileK * 2 : 0);
 
-  pdl_trigger();
+  if (!p.late_trigger) pdl_trigger();
   unsigned long long* tr = p.trace ? p.trace + static_cast<size_t>(c) * kGemvTrace : nullptr;
   if (tr && tid == 0) tr[0] = globaltimer_ns();
   // After a timed-out wait anywhere in the decode, later kernels do nothing
@@ -392,6 +397,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       }
       if (tr) tr[1] = globaltimer_ns();
       pdl_wait();
+      if (p.late_trigger) pdl_trigger();
       if (tr) tr[2] = globaltimer_ns();
       for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
       for (int i = npre; i < n_units; ++i) {
