@@ -109,7 +109,8 @@ struct GemvSmem {
   static constexpr int kA = kB + kStages * 2 * kBOpBytes;       // [stages][M][64] fp32 activation slices
   static constexpr int kG = kA + kStages * kActBytes;           // [stages][64] bf16 gain slices
   static constexpr int kOut = kG + kStages * kTileK * 2;        // drained row tile [M][128]
-  static constexpr int kRs = kOut + M * kTileN * 4;
+  static constexpr int kPre = kOut + M * kTileN * 4;             // epilogue inputs fetched early: [2][M][128] fp32
+  static constexpr int kRs = kPre + 2 * M * kTileN * 4;
   static constexpr int kRed = kRs + kMaxRows * 4;               // [4][kMaxRows]
   static constexpr int kFlag = kRed + 4 * kMaxRows * 4;
   static constexpr int kBar = (kFlag + 16 + 7) & ~7;            // full, empty, bready [stages]; afull, aempty [2]
@@ -185,19 +186,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 lo, __nv_bfloat16 
 
 // ------------------------------------------------------------------ epilogues
 // Run on the 128 drain threads with the finished row tile in out ([M][kTileN],
-// fp32, before the RMSNorm scale) and rs[m] (1 if no norm).
+// fp32, before the RMSNorm scale) and rs[m] (1 if no norm).  pre: inputs fetched
+// into shared memory after the upstream wait, or null -- QKV: the rotation table
+// rows of the M positions ([M][head_dim / 2] float2); RESID: the tile's base rows
+// ([M][kTileN]).  base_pos: position of row 0 (st->kv_len + pos_off, read once per CTA).
 
 __device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
 
 template <int M, Epi EPI>
 __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const float* out, const float* rs,
-                                              int tid) {
+                                              const float* pre, int base_pos, int tid) {
   if constexpr (EPI == Epi::QKV) {
     const int r0 = rt * kTileN;
     const int mat = r0 / p.seg_rows;  // 0 = q, 1 = k, 2 = v
     const int local0 = r0 - mat * p.seg_rows;
     const int Dh = p.head_dim, half = Dh >> 1;
-    const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
     if (mat < 2) {
       for (int idx = tid; idx < M * (kTileN / 2); idx += kDrainThreads) {
         const int m = idx / (kTileN / 2), pr = idx - m * (kTileN / 2);
@@ -210,7 +213,8 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
         }
         const float a = out[m * kTileN + ra] * rs[m];
         const float b = out[m * kTileN + rb] * rs[m];
-        const float2 cs = p.rope_cs[static_cast<size_t>(pos) * half + j];
+        const float2 cs = pre ? reinterpret_cast<const float2*>(pre)[m * half + j]
+                              : p.rope_cs[static_cast<size_t>(pos) * half + j];
         const float va = a * cs.x - b * cs.y;
         const float vb = a * cs.y + b * cs.x;
         if (mat == 0) {
@@ -260,14 +264,13 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     if (n < p.N) {
       float bv[M];
 #pragma unroll
-      for (int m = 0; m < M; ++m) bv[m] = __ldcg(p.base + m * p.base_stride + n);
+      for (int m = 0; m < M; ++m) bv[m] = pre ? pre[m * kTileN + tid] : __ldcg(p.base + m * p.base_stride + n);
 #pragma unroll
       for (int m = 0; m < M; ++m) p.dst[m * p.dst_stride + n] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
     }
   } else {  // ARGMAX (LM head): argmax over the vocabulary, lowest index on ties
     const int lane = tid & 31;
-    const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
-    const int P = __ldcg(&p.st->prompt_len);
+    const int P = p.logits != nullptr ? __ldcg(&p.st->prompt_len) : 0;
     const int n = rt * kTileN + tid;  // thread per tile row
     const bool valid = n < p.N;
 #pragma unroll
@@ -285,18 +288,18 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       }
       if (lane == 0) atomicMax(&p.st->am_key[m], key);
     }
-    __threadfence();
+    // the tile's maxima are released by one acq_rel ticket after the CTA barrier; the tile
+    // that completes the count reads and resets the M keys, one thread per row
+    __shared__ int am_last;
     drain_sync();
-    if (tid == 0) {
-      const unsigned prev = atomicAdd(&p.st->am_count, 1u);
-      if (prev == static_cast<unsigned>(p.n_rt - 1)) {
-        __threadfence();
-        for (int m = 0; m < M; ++m) {
-          const unsigned long long key = atomicExch(&p.st->am_key[m], 0ull);
-          p.tok_dst[m] = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
-        }
-        atomicExch(&p.st->am_count, 0u);
+    if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(p.n_rt - 1);
+    drain_sync();
+    if (am_last) {
+      if (tid < M) {
+        const unsigned long long key = atomicExch(&p.st->am_key[tid], 0ull);
+        p.tok_dst[tid] = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
       }
+      if (tid == 0) atomicExch(&p.st->am_count, 0u);
     }
   }
 }
@@ -526,9 +529,39 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
     } else if (dt < M) {
       rs[dt] = 1.0f;
     }
+    // epilogue inputs fetched now, off the tail: the rotation rows of the M positions (QKV),
+    // the base rows of this CTA's first and last row tiles (RESID; every contributor of a split
+    // tile fetches them, whichever ends up owning it, before its ticket)
+    const int rt_first = u0 / p.n_kt, rt_last = (u1 - 1) / p.n_kt;
+    const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
+    float* pre = reinterpret_cast<float*>(smem + S::kPre);
+    bool pre_rope = false;
+    if constexpr (EPI == Epi::QKV) {
+      const int half = p.head_dim >> 1;
+      pre_rope = base_pos >= 0 && base_pos + M <= p.max_seq && half <= kTileN;
+      if (pre_rope)
+        for (int idx = dt; idx < M * half; idx += kDrainThreads) {
+          const int m = idx / half, j = idx - m * half;
+          reinterpret_cast<float2*>(pre)[idx] = p.rope_cs[static_cast<size_t>(base_pos + m) * half + j];
+        }
+    } else if constexpr (EPI == Epi::RESID) {
+      const int nb = rt_last == rt_first ? 1 : 2;
+      for (int idx = dt; idx < nb * M * kTileN; idx += kDrainThreads) {
+        const int b = idx / (M * kTileN), r = idx - b * (M * kTileN), m = r / kTileN, i = r - m * kTileN;
+        const int n = (b == 0 ? rt_first : rt_last) * kTileN + i;
+        pre[idx] = n < p.N ? __ldcg(p.base + m * p.base_stride + n) : 0.f;
+      }
+    }
     drain_sync();
+    auto pre_of = [&](int rt) -> const float* {
+      if constexpr (EPI == Epi::QKV) return pre_rope ? pre : nullptr;
+      if constexpr (EPI == Epi::RESID) {
+        if (rt == rt_first) return pre;
+        if (rt == rt_last) return pre + M * kTileN;
+      }
+      return nullptr;
+    };
 
-    const int rt_first = u0 / p.n_kt;
     int seg_kt0 = u0 - rt_first * p.n_kt;
     int sg = 0;
     for (int i = 0; i < n_units; ++i) {
@@ -551,7 +584,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       drain_sync();
       const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
       if (whole) {
-        gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
+        gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, dt);
       } else {
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
@@ -606,7 +639,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
           }
           drain_sync();
           if (tr && dt == 0) tr[9] = globaltimer_ns();
-          gemv_epilogue<M, EPI>(p, rt, outb, rs, dt);
+          gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, dt);
           if (dt == 0) p.counters[rt] = 0u;
           if (tr) {
             drain_sync();
