@@ -3,9 +3,9 @@
 //
 // Row m sits at position base + m (base = st->kv_len + pos_off) and attends
 // to keys 0 .. base + m.  Keys are cut into fixed 16 KB chunks at absolute
-// positions (32 keys for head_dim 128, 64 for 64).  Each head is served by one
-// thread-block cluster of kAttnSplit CTAs; CTA r of the cluster takes chunks r,
-// r + kAttnSplit, ... in order, in groups of kAttnBufs chunks: thread 0 brings a
+// positions (32 keys for head_dim 128, 64 for 64).  Each head is served by
+// kAttnSplit CTAs; CTA r of the head takes chunks r, r + kAttnSplit, ... in
+// order, in groups of kAttnBufs chunks: thread 0 brings a
 // group's K and V rows (contiguous in the [H][max_seq][Dh] fp32 cache) into
 // shared memory with bulk copies.  Per group the CTA
 //   1. scores every key of the group for every row (warp w owns a fixed 1/8 of
@@ -15,9 +15,11 @@
 //   3. folds P.V into the warps' output accumulators, rescaled by the row's
 //      running-max change.
 // All warps share one running max per row, so the CTA's state is the warps'
-// accumulators summed in warp order.  The cluster then merges the kAttnSplit CTA
-// states through distributed shared memory in CTA order, each CTA a slice of the
-// output columns.  The chunk grid, the grouping, the key -> (CTA, warp)
+// accumulators summed in warp order.  Each CTA stores its state and takes the
+// head's ticket (one acq_rel atomic after a CTA barrier); the CTA that completes
+// the count merges the kAttnSplit states in CTA order and writes the head's
+// output, so the other CTAs leave without waiting for each other.  The chunk
+// grid, the grouping, the key -> (CTA, warp)
 // assignment and every summation order depend only on key positions, never on
 // M, so each row's output equals the single-row (M = 1) result bitwise.
 //
@@ -28,15 +30,13 @@
 // q and the chunk with this step's keys after it.
 #pragma once
 
-#include <cooperative_groups.h>
-
 #include "attn_warp.cuh"
 
 namespace ssd {
 
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = 32 * kAttnWarps;
-constexpr int kAttnSplit = 8;  // CTAs per head (cluster size)
+constexpr int kAttnSplit = 8;  // CTAs per head
 constexpr int kAttnBufs = 3;   // chunks per group = {K, V} buffers per CTA
 
 struct AttnParams {
@@ -51,9 +51,11 @@ struct AttnParams {
   int n_heads, max_seq;
   float scale;       // 1/sqrt(Dh)
   int prefetch_old;  // the previous launch triggered after its own upstream completed (see above)
+  float* part;        // [n_heads][kAttnSplit][kAttnMaxRows][Dh + 2] CTA states (output, max, sum)
+  unsigned* tickets;  // [n_heads], zero between launches
   // optional timeline, [n_heads * kAttnSplit][8] %globaltimer stamps per CTA: 0 entry, 1 upstream
-  // grid complete, 2 first chunk landed, 3 last chunk folded, 4 states published (cluster barrier
-  // passed), 5 merge done, 6 exit, 7 chunks taken.  Null when not tracing.
+  // grid complete, 2 first chunk landed, 3 last chunk folded, 4 state stored and ticket taken,
+  // 5 merge done (the head's last CTA), 6 exit, 7 chunks taken.  Null when not tracing.
   unsigned long long* trace;
 };
 
@@ -80,17 +82,14 @@ struct AttnSmem {
   static_assert(kAttnWarps * M * DH * 4 <= kAttnBufs * 2 * kKV, "warp accumulators fit the chunk buffers");
   static constexpr int kS = kBuf0 + kAttnBufs * 2 * kKV;         // scores, then probabilities [M][GK]
   static constexpr int kRow = kS + M * G::GK * 4;                // per row: running max, sum, rescale, - [M][4]
-  static constexpr int kCs = kRow + M * 4 * 4;                   // CTA state [M][DH + 2] (read by the cluster)
-  static constexpr int kMg = kCs + M * (DH + 2) * 4;             // merge: [M][kAttnSplit] (max, sum)
-  static constexpr int kWq = kMg + M * kAttnSplit * 2 * 4;       // merge weights [M][kAttnSplit], totals [M]
-  static constexpr int kBar = (kWq + M * (kAttnSplit + 1) * 4 + 7) & ~7;
+  static constexpr int kWq = kRow + M * 4 * 4;                   // merge weights [M][kAttnSplit], totals [M]
+  static constexpr int kFlag = kWq + M * (kAttnSplit + 1) * 4;   // last-CTA flag
+  static constexpr int kBar = (kFlag + 4 + 7) & ~7;
   static constexpr int kTotal = kBar + (kAttnBufs + 1) * 8;
 };
 
 template <int M, int DH>
-__global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThreads, 2)
-    attn_kernel(const AttnParams p) {
-  namespace cg = cooperative_groups;
+__global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams p) {
   using S = AttnSmem<M, DH>;
   using G = AttnGeo<DH>;
   constexpr int KPC = G::KPC, KPW = G::KPW, TPK = G::TPK, DPP = G::DPP, NF = G::NF, DPL = G::DPL;
@@ -101,11 +100,9 @@ __global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThread
   float* ss = reinterpret_cast<float*>(smem + S::kS);
   float* rowst = reinterpret_cast<float*>(smem + S::kRow);
   float* ws = reinterpret_cast<float*>(smem + S::kWs);
-  float* cst = reinterpret_cast<float*>(smem + S::kCs);
   uint64_t* bar = reinterpret_cast<uint64_t*>(smem + S::kBar);  // [kAttnBufs] chunks, then q
-  cg::cluster_group cluster = cg::this_cluster();
   const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
-  const int rank = static_cast<int>(cluster.block_rank());
+  const int rank = blockIdx.x;
   const int h = blockIdx.y;
 
   pdl_trigger();
@@ -313,71 +310,81 @@ __global__ void __cluster_dims__(kAttnSplit, 1, 1) __launch_bounds__(kAttnThread
     tr[7] = static_cast<unsigned long long>(my_chunks);
   }
 
-  // this CTA's state per row: the warps' accumulators summed in warp order (the chunk buffers
-  // are free: every chunk was waited for and folded before the last barrier)
+  // this CTA's state per row -- the warps' accumulators summed in warp order (the chunk buffers
+  // are free: every chunk was waited for and folded before the last barrier) -- goes to part;
+  // the CTA completing the head's ticket merges the kAttnSplit states in CTA order
 #pragma unroll
   for (int m = 0; m < M; ++m)
 #pragma unroll
     for (int e = 0; e < DPL; ++e) ws[(w * M + m) * DH + lane * DPL + e] = acc[m][e];
   __syncthreads();
+  constexpr int kSlot = kAttnMaxRows * E;  // one CTA state in part
+  float* head_part = p.part + static_cast<size_t>(h) * kAttnSplit * kSlot;
+  float* mine = head_part + rank * kSlot;
   for (int idx = tid; idx < M * DH; idx += kAttnThreads) {
     const int m = idx / DH, d = idx - m * DH;
     float O = 0.f;
 #pragma unroll
     for (int q = 0; q < kAttnWarps; ++q) O += ws[(q * M + m) * DH + d];
-    cst[m * E + d] = O;
-    if (d == 0) {
-      cst[m * E + DH] = rowst[4 * m];
-      cst[m * E + DH + 1] = rowst[4 * m + 1];
-    }
+    __stcg(mine + m * E + d, O);
   }
-  cluster.sync();
+  if (tid < M) {
+    __stcg(mine + tid * E + DH, rowst[4 * tid]);
+    __stcg(mine + tid * E + DH + 1, rowst[4 * tid + 1]);
+  }
+  int* last = reinterpret_cast<int*>(smem + S::kFlag);
+  __syncthreads();
+  if (tid == 0) *last = atom_add_acq_rel_gpu(&p.tickets[h], 1u) == static_cast<unsigned>(kAttnSplit - 1);
+  __syncthreads();
   if (tr && tid == 0) tr[4] = globaltimer_ns();
-
-  // the cluster's CTA states combined in CTA order; CTA r writes columns [r * DS, (r + 1) * DS)
-  if (!bad && !timed_out) {
-    float* mg = reinterpret_cast<float*>(smem + S::kMg);  // [M][kAttnSplit][2] (max, sum)
-    float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][kAttnSplit] weights, then [M] totals
-    if (tid < M * kAttnSplit) {
-      const int m = tid / kAttnSplit, q = tid - m * kAttnSplit;
-      const float* e = cluster.map_shared_rank(cst, q) + m * E;
-      mg[2 * tid] = e[DH];
-      mg[2 * tid + 1] = e[DH + 1];
-    }
-    __syncthreads();
-    if (tid < M) {
-      const float* g = mg + tid * kAttnSplit * 2;
-      float mt = -INFINITY;
+  if (*last) {
+    if (!bad && !timed_out) {
+      float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][kAttnSplit] weights, then [M] totals
+      constexpr int NE = (M * DH + kAttnThreads - 1) / kAttnThreads;
+      float v[NE][kAttnSplit];  // the states' outputs, loaded before the weights are known
 #pragma unroll
-      for (int q = 0; q < kAttnSplit; ++q) mt = fmaxf(mt, g[2 * q]);
-      float L = 0.f;
+      for (int e = 0; e < NE; ++e) {
+        const int idx = tid + e * kAttnThreads;
+        if (idx >= M * DH) break;
+        const int m = idx / DH, d = idx - m * DH;
 #pragma unroll
-      for (int q = 0; q < kAttnSplit; ++q) {
-        const float gq = g[2 * q] == -INFINITY ? 0.f : expf(g[2 * q] - mt);
-        wq[tid * kAttnSplit + q] = gq;
-        L = fmaf(gq, g[2 * q + 1], L);
+        for (int q = 0; q < kAttnSplit; ++q) v[e][q] = __ldcg(head_part + q * kSlot + m * E + d);
       }
-      wq[M * kAttnSplit + tid] = L;
-    }
-    __syncthreads();
-    constexpr int DS = DH / kAttnSplit;
-    for (int idx = tid; idx < M * DS; idx += kAttnThreads) {
-      const int m = idx / DS, d = rank * DS + (idx - m * DS);
-      float v[kAttnSplit];
+      if (tid < M) {
+        float mq[kAttnSplit], lq[kAttnSplit];
 #pragma unroll
-      for (int q = 0; q < kAttnSplit; ++q) v[q] = cluster.map_shared_rank(cst, q)[m * E + d];
-      float O = 0.f;
+        for (int q = 0; q < kAttnSplit; ++q) {
+          mq[q] = __ldcg(head_part + q * kSlot + tid * E + DH);
+          lq[q] = __ldcg(head_part + q * kSlot + tid * E + DH + 1);
+        }
+        float mt = -INFINITY;
 #pragma unroll
-      for (int q = 0; q < kAttnSplit; ++q) O = fmaf(wq[m * kAttnSplit + q], v[q], O);
-      const float L = wq[M * kAttnSplit + m];
-      p.o[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
+        for (int q = 0; q < kAttnSplit; ++q) mt = fmaxf(mt, mq[q]);
+        float L = 0.f;
+#pragma unroll
+        for (int q = 0; q < kAttnSplit; ++q) {
+          const float gq = mq[q] == -INFINITY ? 0.f : expf(mq[q] - mt);
+          wq[tid * kAttnSplit + q] = gq;
+          L = fmaf(gq, lq[q], L);
+        }
+        wq[M * kAttnSplit + tid] = L;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int e = 0; e < NE; ++e) {
+        const int idx = tid + e * kAttnThreads;
+        if (idx >= M * DH) break;
+        const int m = idx / DH, d = idx - m * DH;
+        float O = 0.f;
+#pragma unroll
+        for (int q = 0; q < kAttnSplit; ++q) O = fmaf(wq[m * kAttnSplit + q], v[e][q], O);
+        const float L = wq[M * kAttnSplit + m];
+        p.o[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
+      }
     }
+    if (tid == 0) p.tickets[h] = 0u;
+    if (tr && tid == 0) tr[5] = globaltimer_ns();
   }
-  if (tr) {
-    __syncthreads();
-    if (tid == 0) tr[5] = globaltimer_ns();
-  }
-  cluster.sync();  // keep every CTA's shared memory alive until the others have read it
   if (tr && tid == 0) tr[6] = globaltimer_ns();
 }
 

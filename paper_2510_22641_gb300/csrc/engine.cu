@@ -116,6 +116,8 @@ struct ssd_ctx {
   float* partials = nullptr;
   unsigned* counters = nullptr;
   int n_counters = 0;
+  float* attn_part = nullptr;       // split-KV attention: CTA states [H][kAttnSplit][kAttnMaxRows][Dh + 2]
+  unsigned* attn_tickets = nullptr;  // [H]
   __nv_bfloat16* in_vis = nullptr;
   int* in_prompt = nullptr;
   // streams and graphs
@@ -327,6 +329,8 @@ static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch
   AttnParams a{};
   a.trace = trace;
   a.prefetch_old = prefetch_old ? 1 : 0;
+  a.part = c->attn_part;
+  a.tickets = c->attn_tickets;
   a.q = c->qb;
   a.q_stride = c->qp;
   a.k_cache = c->kc + l * c->layer_kv;
@@ -855,6 +859,7 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
   CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
   int r0 = 0;
   for (; r0 < P; r0 += kPrefillChunk) {
@@ -896,6 +901,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   const int P = n_vis + n_prompt, dp = c->dp;
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
   CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
   CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
@@ -1121,7 +1127,7 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
   void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
-                  c->partials, c->counters, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
+                  c->partials, c->counters, c->attn_part, c->attn_tickets, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
                   c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles};
   for (void* b : bufs)
     if (b) cudaFree(b);
@@ -1290,6 +1296,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->attn_part),
+            sizeof(float) * k.n_heads * kAttnSplit * kAttnMaxRows * (k.head_dim + 2)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * k.n_heads));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
   {
     const size_t Pm = k.max_seq;
