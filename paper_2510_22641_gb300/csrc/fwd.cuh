@@ -101,13 +101,6 @@ __device__ __forceinline__ void red_relaxed_add(unsigned* p, unsigned v) {
 
 __device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
 
-// 16-byte asynchronous global -> shared copies (completion: cp_async_wait_all).
-__device__ __forceinline__ void cp_async16(void* dst, const void* src) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(smem_u32(dst)), "l"(src) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
-
 // AND of `ok` over the 128 drain threads (named barrier 1).
 __device__ __forceinline__ bool drain_all(bool ok) {
   uint32_t r;

@@ -331,20 +331,25 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 namespace ssd {
 
 // ------------------------------------------------------------------ causal prefill attention
-// One CTA per (64-query block, head): keys in blocks of 64 up to the query
-// block (causal), scores 4 x 4 per thread in fp32, online softmax per row (a
-// row's 64 scores live on 16 consecutive lanes), O += P V with 4 rows x Dh/16
-// dims per thread.  q: [P][q_stride] rotated queries; K, V: the fp32 cache.
+// One CTA per (64-query block, head), the blocks with the most key blocks launched
+// first: keys in blocks of 64 up to the query block (causal), brought into shared
+// memory with 16-byte asynchronous copies, double-buffered (block kb + 1 loads while
+// block kb is computed).  Scores 4 rows x 4 keys per thread in fp32 (keys tc, tc + 16,
+// tc + 32, tc + 48: with K rows padded to Dh + 4 floats, the 16-byte K reads of a
+// quarter warp hit 8 different bank groups), online softmax per row (a row's 64
+// scores live on 16 consecutive lanes), O += P V with 4 rows x Dh/16 dims per thread.
+// q: [P][q_stride] rotated queries; K, V: the fp32 cache.
 constexpr int kPaQ = 64;
 constexpr int kPaK = 64;
-constexpr int kPaPad = 68;  // transposed tiles: row length 64 + 4 (16-byte aligned, fewer bank conflicts)
+constexpr int kPaPad = 68;  // Q^T and P rows: 64 + 4 floats
 
 template <int DH>
 struct PaSmem {
-  static constexpr int kQt = 0;                                // [DH][kPaPad]
-  static constexpr int kKt = kQt + DH * kPaPad * 4;            // [DH][kPaPad]
-  static constexpr int kV = kKt + DH * kPaPad * 4;             // [64][DH]
-  static constexpr int kP = kV + kPaK * DH * 4;                // [64][kPaPad]
+  static constexpr int kKs = DH + 4;                            // padded K row
+  static constexpr int kQt = 0;                                 // [DH][kPaPad]
+  static constexpr int kK = kQt + DH * kPaPad * 4;              // [2][64][DH + 4]
+  static constexpr int kV = kK + 2 * kPaK * kKs * 4;            // [2][64][DH]
+  static constexpr int kP = kV + 2 * kPaK * DH * 4;             // [64][kPaPad]
   static constexpr int kTotal = kP + kPaQ * kPaPad * 4;
 };
 
@@ -355,16 +360,37 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
                                                            int o_stride, int P, int max_seq, float scale) {
   using S = PaSmem<DH>;
   constexpr int DPT = DH / 16;  // output dims per thread
+  constexpr int KS = S::kKs;
   extern __shared__ __align__(128) uint8_t pa_smem[];
   float* Qt = reinterpret_cast<float*>(pa_smem + S::kQt);
-  float* Kt = reinterpret_cast<float*>(pa_smem + S::kKt);
-  float* Vs = reinterpret_cast<float*>(pa_smem + S::kV);
+  float* Kb = reinterpret_cast<float*>(pa_smem + S::kK);
+  float* Vb = reinterpret_cast<float*>(pa_smem + S::kV);
   float* Ps = reinterpret_cast<float*>(pa_smem + S::kP);
-  const int qb = blockIdx.x, h = blockIdx.y, tid = threadIdx.x;
+  const int nqb = gridDim.x, qb = nqb - 1 - static_cast<int>(blockIdx.x), h = blockIdx.y, tid = threadIdx.x;
   const int q0 = qb * kPaQ;
-  const int tr = tid >> 4, tc = tid & 15;  // rows 4tr..4tr+3; score keys 4tc..4tc+3; output dims tc*DPT..
+  const int tr = tid >> 4, tc = tid & 15;  // rows 4tr..4tr+3; score keys tc + 16b; output dims tc*DPT..
+  const float* kh = k_cache + static_cast<size_t>(h) * max_seq * DH;
+  const float* vh = v_cache + static_cast<size_t>(h) * max_seq * DH;
+  const int n_kb = min(qb + 1, (P + kPaK - 1) / kPaK);
+  // key block kb -> buffer kb & 1; rows at or past P are zero-filled (nothing read)
+  auto issue = [&](int kb) {
+    const int j0 = kb * kPaK;
+    float* kd = Kb + (kb & 1) * kPaK * KS;
+    float* vd = Vb + (kb & 1) * kPaK * DH;
+    for (int c = tid; c < kPaK * (DH / 4); c += 256) {
+      const int j = c / (DH / 4), d4 = (c - j * (DH / 4)) * 4;
+      const bool in = j0 + j < P;
+      const size_t off = in ? static_cast<size_t>(j0 + j) * DH + d4 : 0;
+      cp_async16_fill(kd + j * KS + d4, kh + off, in ? 16u : 0u);
+      cp_async16_fill(vd + j * DH + d4, vh + off, in ? 16u : 0u);
+    }
+    cp_async_commit();
+  };
   pdl_trigger();
   pdl_wait();
+  issue(0);
+  if (n_kb > 1) issue(1);
+  else cp_async_commit();  // keep one group per block for the waits below
 
   // Q block, transposed: Qt[d][i] = q[q0 + i][h*DH + d] (rows past P read as 0)
   for (int idx = tid; idx < kPaQ * DH; idx += 256) {
@@ -379,34 +405,44 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
 #pragma unroll
     for (int e = 0; e < DPT; ++e) acc[a][e] = 0.f;
   }
-  const float* kh = k_cache + static_cast<size_t>(h) * max_seq * DH;
-  const float* vh = v_cache + static_cast<size_t>(h) * max_seq * DH;
-  const int n_kb = min(qb + 1, (P + kPaK - 1) / kPaK);
   for (int kb = 0; kb < n_kb; ++kb) {
     const int j0 = kb * kPaK;
-    __syncthreads();  // previous block's Kt / Vs / Ps fully used
-    for (int idx = tid; idx < kPaK * DH; idx += 256) {
-      const int j = idx / DH, d = idx - j * DH;
-      const bool in = j0 + j < P;
-      Kt[d * kPaPad + j] = in ? __ldcg(kh + static_cast<size_t>(j0 + j) * DH + d) : 0.f;
-      Vs[j * DH + d] = in ? __ldcg(vh + static_cast<size_t>(j0 + j) * DH + d) : 0.f;
-    }
+    const float* Ks = Kb + (kb & 1) * kPaK * KS;
+    const float* Vs = Vb + (kb & 1) * kPaK * DH;
+    cp_async_wait_group<1>();  // block kb has landed (block kb + 1 may still be in flight)
     __syncthreads();
-    // scores s[a][b] = q_{4tr+a} . k_{4tc+b}
+    // scores s[a][b] = q_{4tr+a} . k_{tc+16b}
     float s[4][4];
 #pragma unroll
     for (int a = 0; a < 4; ++a)
 #pragma unroll
       for (int b = 0; b < 4; ++b) s[a][b] = 0.f;
-#pragma unroll 4
-    for (int d = 0; d < DH; ++d) {
-      const float4 qv = *reinterpret_cast<const float4*>(Qt + d * kPaPad + 4 * tr);
-      const float4 kv = *reinterpret_cast<const float4*>(Kt + d * kPaPad + 4 * tc);
-      const float qa[4] = {qv.x, qv.y, qv.z, qv.w}, kb4[4] = {kv.x, kv.y, kv.z, kv.w};
+#pragma unroll 2
+    for (int d = 0; d < DH; d += 4) {
+      float4 qv[4], kv[4];
 #pragma unroll
-      for (int a = 0; a < 4; ++a)
+      for (int e = 0; e < 4; ++e) qv[e] = *reinterpret_cast<const float4*>(Qt + (d + e) * kPaPad + 4 * tr);
 #pragma unroll
-        for (int b = 0; b < 4; ++b) s[a][b] = fmaf(qa[a], kb4[b], s[a][b]);
+      for (int b = 0; b < 4; ++b) kv[b] = *reinterpret_cast<const float4*>(Ks + (tc + 16 * b) * KS + d);
+#pragma unroll
+      for (int b = 0; b < 4; ++b) {
+        s[0][b] = fmaf(qv[0].x, kv[b].x, s[0][b]);
+        s[1][b] = fmaf(qv[0].y, kv[b].x, s[1][b]);
+        s[2][b] = fmaf(qv[0].z, kv[b].x, s[2][b]);
+        s[3][b] = fmaf(qv[0].w, kv[b].x, s[3][b]);
+        s[0][b] = fmaf(qv[1].x, kv[b].y, s[0][b]);
+        s[1][b] = fmaf(qv[1].y, kv[b].y, s[1][b]);
+        s[2][b] = fmaf(qv[1].z, kv[b].y, s[2][b]);
+        s[3][b] = fmaf(qv[1].w, kv[b].y, s[3][b]);
+        s[0][b] = fmaf(qv[2].x, kv[b].z, s[0][b]);
+        s[1][b] = fmaf(qv[2].y, kv[b].z, s[1][b]);
+        s[2][b] = fmaf(qv[2].z, kv[b].z, s[2][b]);
+        s[3][b] = fmaf(qv[2].w, kv[b].z, s[3][b]);
+        s[0][b] = fmaf(qv[3].x, kv[b].w, s[0][b]);
+        s[1][b] = fmaf(qv[3].y, kv[b].w, s[1][b]);
+        s[2][b] = fmaf(qv[3].z, kv[b].w, s[2][b]);
+        s[3][b] = fmaf(qv[3].w, kv[b].w, s[3][b]);
+      }
     }
     // online softmax per row over this key block (16 lanes share a row)
 #pragma unroll
@@ -415,7 +451,7 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
       float mx = -INFINITY;
 #pragma unroll
       for (int b = 0; b < 4; ++b) {
-        const int kj = j0 + 4 * tc + b;
+        const int kj = j0 + tc + 16 * b;
         s[a][b] = (kj <= qi && kj < P) ? s[a][b] * scale : -INFINITY;
         mx = fmaxf(mx, s[a][b]);
       }
@@ -426,7 +462,7 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
 #pragma unroll
       for (int b = 0; b < 4; ++b) {
         const float e = (m_new == -INFINITY || s[a][b] == -INFINITY) ? 0.f : expf(s[a][b] - m_new);
-        Ps[(4 * tr + a) * kPaPad + 4 * tc + b] = e;
+        Ps[(4 * tr + a) * kPaPad + tc + 16 * b] = e;
         rsum += e;
       }
 #pragma unroll
@@ -437,7 +473,6 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
       for (int e = 0; e < DPT; ++e) acc[a][e] *= corr;
       m_run[a] = m_new;
     }
-    __syncwarp();
     __syncthreads();
     // O += P V
     const int kn = min(kPaK, P - j0);
@@ -458,7 +493,11 @@ __global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restri
         for (int e = 0; e < DPT; ++e) acc[a][e] = fmaf(pj, vv[e], acc[a][e]);
       }
     }
+    __syncthreads();  // buffer kb & 1 and Ps are free again
+    if (kb + 2 < n_kb) issue(kb + 2);
+    else cp_async_commit();
   }
+  cp_async_wait_all();
 #pragma unroll
   for (int a = 0; a < 4; ++a) {
     const int qi = q0 + 4 * tr + a;
