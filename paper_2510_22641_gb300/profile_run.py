@@ -27,7 +27,7 @@ def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--layers", type=int, default=32)
     ap.add_argument("--phase", choices=["greedy", "ssd", "prefill", "proj"], default="greedy")
-    ap.add_argument("--proj", default="gateup", help="--phase proj: qkv, o, gateup, down or head")
+    ap.add_argument("--proj", default="gateup", help="--phase proj: qkv, o, gateup, down, head, in1, in2 or attn")
     ap.add_argument("--rows", type=int, default=1, help="--phase proj: activation rows")
     ap.add_argument("--tokens", type=int, default=8)
     ap.add_argument("--s", type=float, default=0.2)
@@ -61,8 +61,10 @@ def main() -> None:
         elif args.phase == "ssd":
             model.decode(1 + args.tokens, w.gamma)
 
-    if args.phase == "proj":  # isolated launches of one projection kernel
+    if args.phase == "proj":  # isolated launches of one projection kernel (attention: over the prompt's cache)
+        model.prefill(v, p)
         model.profile_projection(args.proj, 0, args.rows, 3)
+        model.prefill(v, p)
         model.sync()
         torch.cuda.profiler.start()
         model.profile_projection(args.proj, 0, args.rows, 3)
