@@ -605,37 +605,63 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
             tr[8] = globaltimer_ns();
             tr[11] += 1;
           }
-          // Sum the partials in CTA order, all rows at once, 16 CTAs' 16-byte loads in flight.
-          // Every CTA after c_first starts its range inside this tile (slot 2 cc); c_first's slot
-          // depends on whether the tile is its first one.
+          // Sum the partials in CTA order, all rows at once.  Every CTA after c_first starts its
+          // range inside this tile (slot 2 cc); c_first's slot depends on whether the tile is its
+          // first one.  When this is the CTA's last segment its weight ring is idle (every MMA
+          // has completed), so all partials land there with one round of 16-byte asynchronous
+          // copies; otherwise 16 CTAs' 16-byte loads are kept in flight per round.
           const int nsp = c_last - c_first + 1;
           const int slot0 = 2 * c_first + (unit_begin(c_first, p.units, G) / p.n_kt == rt ? 0 : 1);
           const float4* part = reinterpret_cast<const float4*>(p.partials);
           constexpr int kSlotF4 = kMaxRows * kTileN / 4;
-          for (int f = dt; f < M * (kTileN / 4); f += kDrainThreads) {
-            float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int b0 = 0; b0 < nsp; b0 += 16) {
-              float4 pv[16];
-#pragma unroll
-              for (int j = 0; j < 16; ++j) {
-                const int k = b0 + j;
-                const int sl = k == 0 ? slot0 : 2 * (c_first + k);
-                pv[j] = k < nsp ? __ldcg(part + static_cast<size_t>(sl) * kSlotF4 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+          constexpr int kF4 = M * (kTileN / 4);  // float4s of one partial
+          if (i == n_units - 1 && nsp * kF4 * 16 <= kStages * static_cast<int>(kWTileBytes)) {
+            float4* land = reinterpret_cast<float4*>(smem + S::kW);  // [nsp][kF4]
+            for (int t = dt; t < nsp * kF4; t += kDrainThreads) {
+              const int k = t / kF4, f = t - k * kF4;
+              const int sl = k == 0 ? slot0 : 2 * (c_first + k);
+              cp_async16(land + t, part + static_cast<size_t>(sl) * kSlotF4 + f);
+            }
+            cp_async_commit();
+            cp_async_wait_all();
+            drain_sync();
+            for (int f = dt; f < kF4; f += kDrainThreads) {
+              float4 sum = land[f];
+              for (int k = 1; k < nsp; ++k) {
+                const float4 v = land[k * kF4 + f];
+                sum.x += v.x;
+                sum.y += v.y;
+                sum.z += v.z;
+                sum.w += v.w;
               }
+              reinterpret_cast<float4*>(outb)[f] = sum;
+            }
+          } else {
+            for (int f = dt; f < kF4; f += kDrainThreads) {
+              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+              for (int b0 = 0; b0 < nsp; b0 += 16) {
+                float4 pv[16];
 #pragma unroll
-              for (int j = 0; j < 16; ++j) {
-                if (b0 + j >= nsp) continue;
-                if (b0 + j == 0) {
-                  sum = pv[j];
-                } else {
-                  sum.x += pv[j].x;
-                  sum.y += pv[j].y;
-                  sum.z += pv[j].z;
-                  sum.w += pv[j].w;
+                for (int j = 0; j < 16; ++j) {
+                  const int k = b0 + j;
+                  const int sl = k == 0 ? slot0 : 2 * (c_first + k);
+                  pv[j] = k < nsp ? __ldcg(part + static_cast<size_t>(sl) * kSlotF4 + f) : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                  if (b0 + j >= nsp) continue;
+                  if (b0 + j == 0) {
+                    sum = pv[j];
+                  } else {
+                    sum.x += pv[j].x;
+                    sum.y += pv[j].y;
+                    sum.z += pv[j].z;
+                    sum.w += pv[j].w;
+                  }
                 }
               }
+              reinterpret_cast<float4*>(outb)[f] = sum;
             }
-            reinterpret_cast<float4*>(outb)[f] = sum;
           }
           drain_sync();
           if (tr && dt == 0) tr[9] = globaltimer_ns();
