@@ -11,7 +11,8 @@ Printed as one JSON line (rank 0):
                  (host->device inputs and device->host tokens inside the timing)
   roofline       the dominant kernel (weight-streaming GEMV, gate/up, 1 row)
                  timed alone with CUDA events, against the measured HBM copy peak
-  per_s          decode tokens/s of SSD and of greedy decoding (same kernels)
+  per_s          decode tokens/s of SSD and of greedy decoding (same kernels), and of SSD with the
+                 dynamic draft length d(t) (d0 = 5, N = the context's max_seq, capped at gamma_max)
                  and their ratio for s in {0.05, 0.2, 1.0}
   cpu_baseline   the fp64 oracle on the host cores over a bounded sample
 
@@ -363,11 +364,15 @@ def main() -> None:
     n_out = torch.zeros(1, dtype=torch.int32, device="cuda")
     stream = torch.cuda.current_stream()
 
+    dyn_n = w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1   # N of d(t): the longest sequence of this context
+
     def request(gamma: int, ev=None):
         model.prefill(v, p)
         if ev is not None:
             ev.record(stream)
-        if gamma > 0:
+        if gamma < 0:   # dynamic draft length d(t), d0 = 5, capped at gamma_max
+            model.decode_dynamic(w.max_new, 5, dyn_n, lib.SSD_MAX_GAMMA, out, n_out)
+        elif gamma > 0:
             model.decode(w.max_new, gamma, out, n_out)
         else:
             model.greedy_decode(w.max_new, out, n_out)
@@ -422,7 +427,7 @@ def main() -> None:
         rs.copy_(torch.tensor(ws.resid_scale(), device="cuda"))
         ins.copy_(torch.tensor([ws.in_scale()], device="cuda"))
         row = {"s": s}
-        for name, gamma in (("ssd", w.gamma), ("greedy", 0)):
+        for name, gamma in (("ssd", w.gamma), ("greedy", 0), ("ssd_dynamic", -1)):
             ts = []
             for _ in range(2):
                 a, b, c = (torch.cuda.Event(enable_timing=True) for _ in range(3))
@@ -436,7 +441,12 @@ def main() -> None:
                 sst = model.stats()
                 row["mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
                 row["steps"] = sst["steps"]
+            if name == "ssd_dynamic":
+                sst = model.stats()
+                row["dynamic_mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
+                row["dynamic_mean_gamma"] = sst["drafted"] / max(sst["steps"], 1)
         row["speedup"] = row["ssd_decode_tok_s"] / row["greedy_decode_tok_s"]
+        row["dynamic_speedup"] = row["ssd_dynamic_decode_tok_s"] / row["greedy_decode_tok_s"]
         per_s.append(row)
     rs.copy_(torch.tensor(w.resid_scale(), device="cuda"))
     ins.copy_(torch.tensor([w.in_scale()], device="cuda"))

@@ -170,6 +170,23 @@ SSD_API ssd_status ssd_verify(ssd_ctx* ctx, int gamma, int32_t* n_emitted, int32
  * async. */
 SSD_API ssd_status ssd_decode(ssd_ctx* ctx, int max_new, int gamma, int32_t* out_tok, int32_t* n_out);
 
+/* SSD decode with the dynamic draft length of Sec. "Choice of d":
+ *   d(t) = d0 + floor(10 / (1 + exp(-0.01 (t - n_max / 2))))   (fp64, host)
+ * where the t-th token is generated from t - 1 tokens of context, so a step
+ * whose last emitted token sits at position kv_len uses t = kv_len + 2.  Each
+ * step drafts min(d(t), gamma_cap) tokens (gamma_cap <= gamma_max; the paper's
+ * range is d0 .. d0 + 10) and, in the last steps, accepts at most remaining - 1.
+ * One CUDA-graph launch: a WHILE node whose body selects the step's branch of a
+ * SWITCH node (one draft + verify + accept branch per gamma) from a device
+ * table of d(kv_len + 2).  Same buffers, capacity rule (with gamma_cap) and
+ * errors as ssd_decode.  async. */
+SSD_API ssd_status ssd_decode_dynamic(ssd_ctx* ctx, int max_new, int d0, int n_max, int gamma_cap,
+                                      int32_t* out_tok, int32_t* n_out);
+
+/* d(t) of Sec. "Choice of d", the value ssd_decode_dynamic tabulates (host
+ * function; no context, no GPU). */
+SSD_API int ssd_draft_length(int t, int d0, int n_max);
+
 /* Baseline: plain greedy decoding with the full model (same kernels, one
  * token per step, device-side loop).  Same buffers as ssd_decode.  async. */
 SSD_API ssd_status ssd_greedy_decode(ssd_ctx* ctx, int max_new, int32_t* out_tok, int32_t* n_out);

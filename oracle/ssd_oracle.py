@@ -28,12 +28,18 @@ here; d = draft tokens per step, written gamma):
   the full model; rows of rejected positions are simply overwritten later
   (rollback by length).
 
-Readings where the paper is silent or garbled (each is listed in the design doc):
+Readings where the paper is silent or garbled:
 gamma drafts per step (the printed draft loop runs one index too far); the
 bonus token is taken after the verify loop; the loop stops after max_new
 tokens or after an eos; in the last steps gamma_eff = min(gamma, remaining-1);
 argmax ties go to the lowest index; rotate-half RoPE with theta = 10000;
 RMSNorm eps = 1e-5.
+
+Dynamic draft length (Sec. "Choice of d"): d(t) = d(0) + floor(10 / (1 + exp(-0.01
+(t - N/2)))), evaluated in fp64, where the t-th token is generated from t - 1
+tokens of context (so t = kv_len + 2 at a step whose last emitted token y sits at
+position kv_len) and N is the longest sequence the model is run with; each step
+drafts min(d(t), gamma_cap, remaining - 1) tokens.
 
 Decode rows are always processed one at a time by the same function, so a
 row's result does not depend on how many rows a step holds: SSD and greedy
@@ -222,6 +228,16 @@ def _truncate_eos(tokens: list, eos_id: int) -> tuple[list, bool]:
     return tokens, False
 
 
+def draft_length(t: int, d0: int, n_max: int) -> int:
+    """Sec. "Choice of d", the equation for d(t): d0 + floor(10 * sigmoid(0.01 (t - N/2))) in fp64.
+
+    The sigmoid is written as 1 / (1 + exp(-z)); for t far above N/2 it rounds to 1 and d reaches
+    d0 + 10, the paper's stated upper end {5, ..., 15} for d0 = 5.
+    """
+    z = -0.01 * (float(t) - float(n_max) / 2.0)
+    return d0 + int(np.floor(10.0 / (1.0 + np.exp(z))))
+
+
 def greedy_generate(m: Model, vis: np.ndarray, prompt, max_new: int, max_seq: int | None = None,
                     keep_cache: bool = False) -> Result:
     """Plain autoregressive greedy decoding of the full model (the speedup baseline)."""
@@ -243,7 +259,7 @@ def greedy_generate(m: Model, vis: np.ndarray, prompt, max_new: int, max_seq: in
 def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                  max_seq: int | None = None, reuse_draft_rows: bool = True,
                  keep_cache: bool = False, keep_draft_logits: bool = False,
-                 max_steps: int | None = None) -> Result:
+                 max_steps: int | None = None, dynamic: tuple[int, int] | None = None) -> Result:
     """Algorithm 1 (greedy self-speculative decoding with the imitation network).
 
     Per step, with y the last emitted token at position p = kv_len:
@@ -254,6 +270,8 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
       accepting: a = largest i <= gamma_eff with d_1..d_i = f_0..f_{i-1};
                  emit d_1..d_a and f_a; kv_len = p + a + 1; y = f_a.
     max_steps (timing samples only) stops after that many steps.
+    dynamic = (d0, N): each step drafts min(d(t), gamma, remaining - 1) tokens with
+    t = kv_len + 2 (Sec. "Choice of d"); gamma is then the cap.
     """
     c = m.cfg
     k, L = c.draft_exit_k, c.n_layers
@@ -267,7 +285,8 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
     while len(res.tokens) < max_new and not done and (max_steps is None or len(res.step_s) < max_steps):
         t0 = time.perf_counter()
         remaining = max_new - len(res.tokens)
-        g_eff = min(gamma, remaining - 1)
+        g_step = gamma if dynamic is None else min(gamma, draft_length(p + 2, dynamic[0], dynamic[1]))
+        g_eff = min(g_step, remaining - 1)
         toks, xk, dlog = [y], [], []
         for j in range(g_eff):                                   # drafting stage
             x = forward_row(m, embed(m, toks[j]), p + j, cache, range(k))

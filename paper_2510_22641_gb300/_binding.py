@@ -20,7 +20,8 @@ SSD_IN_MLP2 = 1
 STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_CUDA", 4: "SSD_ERR_CAPACITY",
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
 
-EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode",
+EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode", "ssd_decode_dynamic",
+            "ssd_draft_length",
             "ssd_greedy_decode", "ssd_generate", "ssd_greedy_generate", "ssd_sync", "ssd_get_stats",
             "ssd_set_logits_capture", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
             "ssd_status_string",
@@ -75,6 +76,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_draft": [vp, i32, pi32],
         "ssd_verify": [vp, i32, pi32, pi32],
         "ssd_decode": [vp, i32, i32, pi32, pi32],
+        "ssd_decode_dynamic": [vp, i32, i32, i32, i32, pi32, pi32],
         "ssd_greedy_decode": [vp, i32, pi32, pi32],
         "ssd_generate": [vp, vp, i32, vp, i32, i32, i32, vp, ctypes.POINTER(i32), ctypes.POINTER(SSDStats)],
         "ssd_greedy_generate": [vp, vp, i32, vp, i32, i32, vp, ctypes.POINTER(i32), ctypes.POINTER(SSDStats)],
@@ -91,6 +93,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         f = getattr(lib, name)
         f.argtypes = args
         f.restype = ctypes.c_int
+    lib.ssd_draft_length.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int]
+    lib.ssd_draft_length.restype = ctypes.c_int
     lib.ssd_status_string.argtypes = [ctypes.c_int]
     lib.ssd_status_string.restype = ctypes.c_char_p
     lib.ssd_last_error.argtypes = [vp]

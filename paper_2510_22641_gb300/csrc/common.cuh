@@ -33,7 +33,8 @@ struct DevState {
   int accepted;    // sum of a
   int last_n;      // tokens emitted by the last accept
   int eos_id;
-  int pad[3];
+  int dyn_launches;  // kernel launches of the running dynamic-length decode's steps
+  int pad[2];
   int hist[SSD_MAX_GAMMA + 1];   // steps per accepted length a
   int tok_in[kMaxRows];          // verify rows t_0 = y, t_j = d_j
   int full_tok[kMaxRows];        // f_i = full-model argmax of row i

@@ -99,8 +99,31 @@ __global__ void decode_setup_kernel(DevState* st, int max_new, int gamma) {
   st->max_new = max_new;
   st->gamma = gamma;
   st->steps = st->drafted = st->accepted = 0;
+  st->dyn_launches = 0;
   for (int i = 0; i <= SSD_MAX_GAMMA; ++i) st->hist[i] = 0;
   if (st->n_out >= max_new || st->error) st->done = 1;
+}
+
+// Dynamic draft length (Sec. "Choice of d"): this step drafts gamma = table[kv_len] tokens,
+// clamped to [1, cap] (table[p] = d(p + 2), evaluated on the host in fp64); the step's branch
+// of the SWITCH node is gamma - 1.  launches[gamma - 1]: kernel launches of that branch.
+__global__ void dyn_select_kernel(DevState* st, const int* table, const int* launches, int cap,
+                                  cudaGraphConditionalHandle sw) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x != 0) return;
+  int g = table[st->kv_len];
+  g = g < 1 ? 1 : (g > cap ? cap : g);
+  st->gamma = g;
+  st->dyn_launches += launches[g - 1] + 2;  // + this kernel and the loop test
+  cudaGraphSetConditional(sw, static_cast<unsigned>(g - 1));
+}
+
+// Loop test after a dynamic-length step: run the WHILE body again unless decoding is finished.
+__global__ void loop_continue_kernel(DevState* st, cudaGraphConditionalHandle cond) {
+  pdl_trigger();
+  pdl_wait();
+  if (threadIdx.x == 0) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
 }
 
 // First node of a decode graph: run the WHILE body only if decoding is not finished.

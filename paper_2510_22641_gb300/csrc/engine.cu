@@ -125,6 +125,13 @@ struct ssd_ctx {
   cudaEvent_t ev_in = nullptr, ev_out = nullptr;
   bool use_pdl = true;
   std::map<int, cudaGraphExec_t> decode_graphs, draft_graphs, verify_graphs, step_graphs;
+  // dynamic draft length (Sec. "Choice of d"): d(p + 2) per kv_len p, step graphs by cap
+  int* dyn_table = nullptr;   // device [max_seq + 1]
+  int* dyn_launch = nullptr;  // device [SSD_MAX_GAMMA]: kernel launches of the step branch for gamma
+  std::vector<int> dyn_table_h;
+  int dyn_d0 = -1, dyn_n = -1;
+  std::map<int, cudaGraphExec_t> dyn_graphs;
+  int64_t dyn_host_launches = 0;
   // Diagnostic: drive the decode loop from the host with one plain graph per
   // step (ncu cannot profile kernels of graphs that hold conditional nodes).
   bool host_loop = false;
@@ -141,7 +148,7 @@ struct ssd_ctx {
   int drafted_gamma = 0;
   int prompt_len = 0;
   int64_t kv_upper = 0;  // upper bound on the device kv_len
-  int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy
+  int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy, 3 ssd with the dynamic draft length
   int last_gamma = 0;
   std::pair<int, int> last_prefill_shape{0, 0};
   // persistent forward kernel (decode): phase lists, map table, flags and scratch
@@ -1041,6 +1048,105 @@ static ssd_status build_plain_graph(ssd_ctx* c, EnqueueFn fn, int a0, int a1, cu
   return s;
 }
 
+// d(t) of Sec. "Choice of d" in fp64: d0 + floor(10 / (1 + exp(-0.01 (t - N/2)))).
+static int draft_length_fp64(int t, int d0, int n_max) {
+  const double z = -0.01 * (static_cast<double>(t) - static_cast<double>(n_max) / 2.0);
+  return d0 + static_cast<int>(std::floor(10.0 / (1.0 + std::exp(z))));
+}
+
+// Kernel launch without the programmatic-serialization attribute (graph nodes whose upstream is
+// a conditional node, or that have none).
+template <typename Kern, typename... Args>
+static cudaError_t launch_plain(ssd_ctx* c, Kern kern, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(1);
+  cfg.blockDim = dim3(32);
+  cfg.stream = c->cs;
+  ++c->launch_counter;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+// Dynamic-length SSD graph = [loop_begin] -> WHILE(cond) { select -> SWITCH(sw) { branch g - 1:
+// draft g + verify g + accept, g = 1..cap } -> loop test }.  The select kernel picks the branch
+// from the d(t) table; the loop test (in the WHILE body itself) sets cond.
+static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
+  cudaGraph_t g = nullptr;
+  CK(cudaGraphCreate(&g, 0));
+  cudaGraphConditionalHandle cond;
+  cudaError_t e = cudaGraphConditionalHandleCreate(&cond, g, 0, cudaGraphCondAssignDefault);
+  if (e != cudaSuccess) {
+    cudaGraphDestroy(g);
+    CK(e);
+  }
+  ssd_status s = begin_capture(c, g);
+  if (s == SSD_OK) {
+    e = launch_plain(c, loop_begin_kernel, c->st, cond);
+    s = end_capture(c, g, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop_begin: %s", cudaGetErrorString(e)));
+  }
+  cudaGraphNode_t begin = nullptr;
+  size_t n = 1;
+  if (s == SSD_OK && cudaGraphGetNodes(g, &begin, &n) != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "graph nodes");
+  cudaGraphNodeParams wp = {};
+  wp.type = cudaGraphNodeTypeConditional;
+  wp.conditional.handle = cond;
+  wp.conditional.type = cudaGraphCondTypeWhile;
+  wp.conditional.size = 1;
+  cudaGraphNode_t wnode;
+  if (s == SSD_OK && (e = cudaGraphAddNode(&wnode, g, &begin, nullptr, 1, &wp)) != cudaSuccess)
+    s = fail(c, SSD_ERR_CUDA, "WHILE node: %s", cudaGetErrorString(e));
+  std::vector<int> launches(cap, 0);
+  if (s == SSD_OK) {
+    cudaGraph_t body = wp.conditional.phGraph_out[0];
+    cudaGraphConditionalHandle sw;
+    if ((e = cudaGraphConditionalHandleCreate(&sw, body, 0, 0)) != cudaSuccess)
+      s = fail(c, SSD_ERR_CUDA, "switch handle: %s", cudaGetErrorString(e));
+    if (s == SSD_OK) s = begin_capture(c, body);
+    if (s == SSD_OK) {
+      e = launch_plain(c, dyn_select_kernel, c->st, static_cast<const int*>(c->dyn_table),
+                       static_cast<const int*>(c->dyn_launch), cap, sw);
+      s = end_capture(c, body, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "select: %s", cudaGetErrorString(e)));
+    }
+    cudaGraphNode_t sel = nullptr;
+    size_t nb = 1;
+    if (s == SSD_OK && cudaGraphGetNodes(body, &sel, &nb) != cudaSuccess) s = fail(c, SSD_ERR_CUDA, "body nodes");
+    cudaGraphNodeParams sp = {};
+    sp.type = cudaGraphNodeTypeConditional;
+    sp.conditional.handle = sw;
+    sp.conditional.type = cudaGraphCondTypeSwitch;
+    sp.conditional.size = static_cast<unsigned>(cap);
+    cudaGraphNode_t snode;
+    if (s == SSD_OK && (e = cudaGraphAddNode(&snode, body, &sel, nullptr, 1, &sp)) != cudaSuccess)
+      s = fail(c, SSD_ERR_CUDA, "SWITCH node: %s", cudaGetErrorString(e));
+    for (int i = 0; s == SSD_OK && i < cap; ++i) {
+      cudaGraph_t br = sp.conditional.phGraph_out[i];
+      s = begin_capture(c, br);
+      if (s == SSD_OK) {
+        const int64_t l0 = c->launch_counter;
+        ssd_status inner = enqueue_draft(c, i + 1);
+        if (inner == SSD_OK) inner = enqueue_verify(c, i + 1, 0, 0);
+        launches[i] = static_cast<int>(c->launch_counter - l0);
+        s = end_capture(c, br, inner);
+      }
+    }
+    if (s == SSD_OK) {
+      if ((e = cudaStreamBeginCaptureToGraph(c->cs, body, &snode, nullptr, 1, cudaStreamCaptureModeThreadLocal)) !=
+          cudaSuccess)
+        s = fail(c, SSD_ERR_CUDA, "capture after SWITCH: %s", cudaGetErrorString(e));
+      if (s == SSD_OK) {
+        e = launch_plain(c, loop_continue_kernel, c->st, cond);
+        s = end_capture(c, body, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop test: %s", cudaGetErrorString(e)));
+      }
+    }
+  }
+  if (s == SSD_OK && (e = cudaMemcpy(c->dyn_launch, launches.data(), sizeof(int) * cap, cudaMemcpyHostToDevice)) !=
+                         cudaSuccess)
+    s = fail(c, SSD_ERR_CUDA, "launch counts: %s", cudaGetErrorString(e));
+  if (s == SSD_OK && (e = cudaGraphInstantiate(exec, g, 0)) != cudaSuccess)
+    s = fail(c, SSD_ERR_CUDA, "graph instantiate: %s", cudaGetErrorString(e));
+  cudaGraphDestroy(g);
+  return s;
+}
+
 static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) {
   return c->prefill_rows ? enqueue_prefill(c, a, b) : enqueue_prefill_tc(c, a, b);
 }
@@ -1061,6 +1167,8 @@ static void drop_graphs(ssd_ctx* c) {
   for (auto& kv : c->step_graphs) cudaGraphExecDestroy(kv.second);
   c->step_graphs.clear();
   for (auto& kv : c->prefill_graphs) cudaGraphExecDestroy(kv.second);
+  for (auto& kv : c->dyn_graphs) cudaGraphExecDestroy(kv.second);
+  c->dyn_graphs.clear();
   if (c->greedy_graph) cudaGraphExecDestroy(c->greedy_graph);
   c->decode_graphs.clear();
   c->draft_graphs.clear();
@@ -1127,7 +1235,7 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
   void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
-                  c->partials, c->counters, c->attn_part, c->attn_tickets, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
+                  c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
                   c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles};
   for (void* b : bufs)
     if (b) cudaFree(b);
@@ -1299,6 +1407,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_part),
             sizeof(float) * k.n_heads * kAttnSplit * kAttnMaxRows * (k.head_dim + 2)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * k.n_heads));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_table), sizeof(int) * (k.max_seq + 1)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_launch), sizeof(int) * SSD_MAX_GAMMA));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
   {
     const size_t Pm = k.max_seq;
@@ -1520,6 +1630,73 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
   return SSD_OK;
 }
 
+static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, int cap, int32_t* out_tok,
+                                  int32_t* n_out) {
+  if (!c->prefilled) return fail(c, SSD_ERR_STATE, "decode before ssd_prefill");
+  if (max_new < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_new must be >= 1");
+  if (cap < 1 || cap > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma cap %d", cap);
+  if (d0 < 1 || n_max < 1) return fail(c, SSD_ERR_INVALID_ARG, "d0 %d, n_max %d", d0, n_max);
+  if (static_cast<int64_t>(c->prompt_len) + max_new + cap + 1 > c->cfg.max_seq)
+    return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + cap + 1 = %d > max_seq = %d",
+                c->prompt_len + max_new + cap + 1, c->cfg.max_seq);
+  CKS(fwd_ensure(c));
+  if (d0 != c->dyn_d0 || n_max != c->dyn_n) {  // the table of the previous schedule may still be read
+    CK(cudaStreamSynchronize(c->cs));
+    c->dyn_table_h.resize(c->cfg.max_seq + 1);
+    for (int p = 0; p <= c->cfg.max_seq; ++p) c->dyn_table_h[p] = draft_length_fp64(p + 2, d0, n_max);
+    CK(cudaMemcpy(c->dyn_table, c->dyn_table_h.data(), sizeof(int) * (c->cfg.max_seq + 1), cudaMemcpyHostToDevice));
+    c->dyn_d0 = d0;
+    c->dyn_n = n_max;
+  }
+  decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, cap);
+  CK(cudaGetLastError());
+  if (c->host_loop) {  // one plain graph per step; the host reads kv_len and picks the step's gamma
+    c->dyn_host_launches = 0;
+    for (int it = 0; it < max_new; ++it) {
+      DevState h;
+      CK(cudaMemcpyAsync(&h, c->st, sizeof(int) * 8, cudaMemcpyDeviceToHost, c->cs));
+      CK(cudaStreamSynchronize(c->cs));
+      if (h.done) break;
+      const int g = std::max(1, std::min(cap, c->dyn_table_h[h.kv_len]));
+      auto sg = c->step_graphs.find(g);
+      if (sg == c->step_graphs.end()) {
+        cudaGraphExec_t ge;
+        int64_t nb = 0;
+        CKS(build_plain_graph(c, enq_step_fn, g, 0, &ge, &nb));
+        sg = c->step_graphs.emplace(g, ge).first;
+        c->decode_body_launches[g] = nb;
+      }
+      CK(cudaGraphLaunch(sg->second, c->cs));
+      c->dyn_host_launches += c->decode_body_launches[g];
+    }
+  } else {
+    auto it = c->dyn_graphs.find(cap);
+    if (it == c->dyn_graphs.end()) {
+      cudaGraphExec_t ge;
+      CKS(build_dyn_graph(c, cap, &ge));
+      it = c->dyn_graphs.emplace(cap, ge).first;
+    }
+    CK(cudaGraphLaunch(it->second, c->cs));
+  }
+  if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+  CK(cudaGetLastError());
+  c->last_decode_kind = 3;
+  c->last_gamma = cap;
+  c->drafted_gamma = 0;
+  c->kv_upper = c->prompt_len + max_new + cap + 1;
+  return SSD_OK;
+}
+
+int ssd_draft_length(int t, int d0, int n_max) { return draft_length_fp64(t, d0, n_max); }
+
+ssd_status ssd_decode_dynamic(ssd_ctx* c, int max_new, int d0, int n_max, int gamma_cap, int32_t* out_tok,
+                              int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CKS(enter(c));
+  CKS(decode_dyn_impl(c, max_new, d0, n_max, gamma_cap, out_tok, n_out));
+  return leave(c);
+}
+
 ssd_status ssd_decode(ssd_ctx* c, int max_new, int gamma, int32_t* out_tok, int32_t* n_out) {
   if (!c) return SSD_ERR_INVALID_ARG;
   if (gamma < 1) return fail(c, SSD_ERR_INVALID_ARG, "gamma must be >= 1");
@@ -1637,6 +1814,10 @@ ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t*
     if (c->last_decode_kind == 2) body = c->greedy_body_launches;
     // setup + loop_begin + steps x body + copy-out
     *decode_launches = c->last_decode_kind ? 2 + static_cast<int64_t>(h.steps) * body + 1 : 0;
+    // dynamic draft length: setup + loop_begin + per step (select + branch + loop test) + copy-out,
+    // or, host-driven, setup + the step graphs + copy-out
+    if (c->last_decode_kind == 3)
+      *decode_launches = c->host_loop ? 2 + c->dyn_host_launches : 3 + static_cast<int64_t>(h.dyn_launches);
   }
   return SSD_OK;
 }

@@ -101,6 +101,11 @@ class SSDModel:
                n_out: torch.Tensor | None = None):
         self._call("ssd_decode", max_new, gamma, _ptr(out_tok), _ptr(n_out))
 
+    def decode_dynamic(self, max_new: int, d0: int, n_max: int, gamma_cap: int, out_tok: torch.Tensor | None = None,
+                       n_out: torch.Tensor | None = None):
+        """SSD with the dynamic draft length d(t) (Sec. "Choice of d"), capped at gamma_cap."""
+        self._call("ssd_decode_dynamic", max_new, d0, n_max, gamma_cap, _ptr(out_tok), _ptr(n_out))
+
     def greedy_decode(self, max_new: int, out_tok: torch.Tensor | None = None, n_out: torch.Tensor | None = None):
         self._call("ssd_greedy_decode", max_new, _ptr(out_tok), _ptr(n_out))
 

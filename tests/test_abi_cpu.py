@@ -56,3 +56,12 @@ def test_create_rejects_bad_arguments_before_touching_the_device(so):
     w = _binding.SSDWeights()
     assert l.ssd_create(ctypes.byref(cfg), ctypes.byref(w), None, ctypes.byref(ctx)) == 1  # d_model % 64
     assert not ctx.value
+
+
+def test_draft_length_matches_the_oracle(so):
+    """The library's d(t) table (Sec. "Choice of d") equals the oracle's, point by point."""
+    import oracle
+    l = _binding.load()
+    for d0, n_max in [(5, 777), (5, 1000), (5, 4096), (3, 120)]:
+        for t in range(0, 2 * n_max + 50):
+            assert l.ssd_draft_length(t, d0, n_max) == oracle.draft_length(t, d0, n_max), (t, d0, n_max)

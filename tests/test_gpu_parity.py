@@ -104,6 +104,44 @@ def test_ssd_matches_oracle_and_gpu_greedy(tiny_model, tiny_bits, s, gamma):
     assert stats["steps"] + stats["accepted"] + 1 == w.max_new
 
 
+@pytest.mark.parametrize("s,cap,n_max", [(0.05, 8, 120), (0.2, 6, 90), (1.0, 8, 40)])
+def test_dynamic_draft_length_matches_oracle(tiny_model, tiny_bits, s, cap, n_max):
+    """Sec. "Choice of d": each step drafts min(d(kv_len + 2), cap) tokens; tokens, logits, steps,
+    accept lengths and kv_len match the oracle's dynamic run, and the tokens equal greedy decoding."""
+    model, _ = tiny_model
+    w = synth.TINY.replace(norm_gain="perturbed", s=s)
+    set_scale(model, w)
+    _, _, v, p = device_inputs(w)
+    logits = torch.full((w.max_new, w.shape.vocab), float("nan"), device="cuda")
+    model.set_logits_capture(logits)
+    out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
+    n = torch.zeros(1, dtype=torch.int32, device="cuda")
+    model.prefill(v, p)
+    model.decode_dynamic(w.max_new, 5, n_max, cap, out, n)
+    model.sync()
+    toks, stats = out[: int(n.item())].cpu().tolist(), model.stats()
+    m = oracle.model_from_bits(w, tiny_bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, cap, dynamic=(5, n_max))
+    _, dec = model.launch_counts()
+    check_against_oracle(toks, logits.cpu().numpy(), stats, ref, cap)
+    assert stats["drafted"] == sum(len(d) for d in ref.draft_tokens)
+    gtoks, _, _ = gpu_decode(model, w, 0, capture=False)
+    assert toks == gtoks
+    # launches: setup, loop test at entry, copy-out; per step the branch for gamma_t plus its
+    # selection (and, in the device loop, the loop test)
+    L, k = w.shape.n_layers, w.draft_exit_k
+    fwd = os.environ.get("SSD_DECODE") == "fwd"
+    host = os.environ.get("SSD_HOST_LOOP", "0") not in ("", "0")
+    body = lambda g: 3 if fwd else g * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
+    p_, expect = w.prompt_len, 0
+    for kv in ref.kv_lens:
+        g_t = min(oracle.draft_length(p_ + 2, 5, n_max), cap)
+        expect += body(g_t) + (0 if host else 2)
+        p_ = kv
+    assert dec == expect + (2 if host else 3)
+
+
 def test_kv_cache_after_rollback_equals_greedy_cache(tiny_model):
     model, _ = tiny_model
     w = synth.TINY.replace(norm_gain="perturbed", s=0.2)

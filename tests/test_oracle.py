@@ -280,3 +280,41 @@ def test_prefill_rows_equal_sequential_decode(tiny_bits):
         x = oracle.forward_row(m, x, p, c2, range(m.cfg.n_layers))
     np.testing.assert_allclose(oracle.lm_head(m, x), o1, rtol=1e-10, atol=1e-10)
     np.testing.assert_allclose(c2.k[:, :, :len(rows)], c1.k[:, :, :len(rows)], rtol=1e-10, atol=1e-12)
+
+
+# --------------------------------------------------------------------------- dynamic draft length d(t)
+
+def test_draft_length_closed_form_pins():
+    """Sec. "Choice of d": d(t) = d0 + floor(10 sigmoid(0.01 (t - N/2))).  Pinned by the sigmoid's
+    inverse: 10 sigmoid(z) = k exactly at z = ln(k / (10 - k)), so d steps from d0 + k - 1 to d0 + k
+    between t = floor and ceil of N/2 + 100 ln(k / (10 - k))."""
+    for d0, n_max in [(5, 1000), (5, 4096), (3, 777)]:
+        assert oracle.draft_length(n_max // 2, d0, n_max) == d0 + 5 if n_max % 2 == 0 else True
+        for k in range(1, 10):
+            tk = n_max / 2 + 100.0 * math.log(k / (10 - k))
+            lo, hi = math.floor(tk), math.ceil(tk)
+            if lo == hi or lo < 0:
+                continue
+            assert oracle.draft_length(lo, d0, n_max) == d0 + k - 1, (d0, n_max, k)
+            assert oracle.draft_length(hi, d0, n_max) == d0 + k, (d0, n_max, k)
+        ds = [oracle.draft_length(t, d0, n_max) for t in range(0, 4 * n_max)]
+        assert all(b >= a for a, b in zip(ds, ds[1:]))          # non-decreasing in t
+        assert min(ds) >= d0 and max(ds) <= d0 + 10
+    assert oracle.draft_length(0, 5, 4096) == 5                  # sigmoid(-20.48) * 10 < 1
+    assert oracle.draft_length(10**6, 5, 4096) == 15             # sigmoid rounds to 1 in fp64
+
+
+@pytest.mark.parametrize("s,cap,n_max", [(0.05, 8, 120), (0.2, 6, 90), (1.0, 8, 40)])
+def test_ssd_dynamic_draft_length_equals_greedy(tiny_bits, s, cap, n_max):
+    w = tiny(s=s, gamma=cap)
+    m, vis, prompt = build(w, tiny_bits)
+    g = oracle.greedy_generate(m, vis, prompt, w.max_new)
+    r = oracle.ssd_generate(m, vis, prompt, w.max_new, cap, dynamic=(5, n_max))
+    assert r.tokens == g.tokens
+    # per step: gamma_t = min(d(kv_len + 2), cap, remaining - 1) drafts, 0 <= a <= gamma_t
+    p, n = w.prompt_len, 1
+    for drafts, a, kv in zip(r.draft_tokens, r.accept_lengths, r.kv_lens):
+        g_t = min(oracle.draft_length(p + 2, 5, n_max), cap, w.max_new - n - 1)
+        assert len(drafts) == g_t and 0 <= a <= g_t
+        p, n = kv, n + a + 1
+    assert p == r.kv_len == g.kv_len
