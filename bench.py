@@ -40,7 +40,7 @@ METRIC = "tokens/s and speedup vs full-model greedy decode (7B shape, bs1); HBM 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up GEMV
 # launch from an ncu capture, valid only for the kernel source it was taken on.
-GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "3d9257d3f5d7f4b7", "bytes": 182_902_016}
+GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "8dbe91b28c5a66ff", "bytes": 182_967_552}
 UNIT = "tokens/s"
 S_VALUES = synth.LLAVA7B_S_VALUES
 
