@@ -195,6 +195,9 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
         kv[i][4 * e + 3] = t.w;
       }
     }
+    // all (row, chunk) partial dots first, then the xor trees level by level, then the stores:
+    // no shared-memory store sits between one row's q loads and the next's
+    float a[M][kAttnBufs];
 #pragma unroll
     for (int m = 0; m < M; ++m) {
       const float* qr = Qs + m * DH + part * DPP;
@@ -203,22 +206,32 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
       for (int e = 0; e < NF; ++e) q4[e] = *reinterpret_cast<const float4*>(qr + ((e + rot) & (NF - 1)) * 4);
 #pragma unroll
       for (int i = 0; i < kAttnBufs; ++i) {
-        if (i >= gn) break;
-        float a = 0.f;
+        float t = 0.f;
 #pragma unroll
         for (int e = 0; e < NF; ++e) {
-          a = fmaf(kv[i][4 * e], q4[e].x, a);
-          a = fmaf(kv[i][4 * e + 1], q4[e].y, a);
-          a = fmaf(kv[i][4 * e + 2], q4[e].z, a);
-          a = fmaf(kv[i][4 * e + 3], q4[e].w, a);
+          t = fmaf(kv[i][4 * e], q4[e].x, t);
+          t = fmaf(kv[i][4 * e + 1], q4[e].y, t);
+          t = fmaf(kv[i][4 * e + 2], q4[e].z, t);
+          t = fmaf(kv[i][4 * e + 3], q4[e].w, t);
         }
-#pragma unroll
-        for (int off = 1; off < TPK; off <<= 1) a += __shfl_xor_sync(0xffffffffu, a, off);
-        if (part == 0) {
-          const bool vis = jw < nkc[i] && j0c[i] + jw <= base + m;
-          ss[m * GK + i * KPC + jw] = vis ? a * p.scale : -INFINITY;
-        }
+        a[m][i] = t;
       }
+    }
+#pragma unroll
+    for (int off = 1; off < TPK; off <<= 1)
+#pragma unroll
+      for (int m = 0; m < M; ++m)
+#pragma unroll
+        for (int i = 0; i < kAttnBufs; ++i) a[m][i] += __shfl_xor_sync(0xffffffffu, a[m][i], off);
+    if (part == 0) {
+#pragma unroll
+      for (int m = 0; m < M; ++m)
+#pragma unroll
+        for (int i = 0; i < kAttnBufs; ++i) {
+          if (i >= gn) break;
+          const bool vis = jw < nkc[i] && j0c[i] + jw <= base + m;
+          ss[m * GK + i * KPC + jw] = vis ? a[m][i] * p.scale : -INFINITY;
+        }
     }
     __syncthreads();
     if (!ok) break;
