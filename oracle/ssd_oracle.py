@@ -19,7 +19,13 @@ here; d = draft tokens per step, written gamma):
 * Imitation network I (Sec. "Methodology", "Deep Representation Imitation";
   Sec. "Experiments", Training: two fully connected layers and one layer norm):
   I(x) = x + s_in W2 SiLU(W1 RMSNorm_in(x)), hidden width = model width by
-  default.  IN_IDENTITY gives "Draft w/o Im" (Table 1).
+  default.  IN_IDENTITY gives "Draft w/o Im" (Table 1).  IN_BLOCK reads the
+  module as one decoder block of the model's shape (the NAS space of Sec.
+  "Choice of n" holds such blocks): x + f_I(x) with its own weights, residual
+  scale s_in and its own KV cache.  Its cache rows hold, for every position
+  below kv_len, the block's K/V of that token's x_k: the prefill fills them for
+  the prompt rows, each drafting step for its row, and the verification pass
+  for row gamma (whose x_k only the verification computes).
 * Algorithm 1 (greedy SSD with imitation): draft gamma tokens with
   argmax g(I(x_k)), verify them with the full model in one pass over the
   gamma+1 rows, accept the longest matching prefix, append the full model's
@@ -54,6 +60,7 @@ import numpy as np
 
 IN_IDENTITY = 0
 IN_MLP2 = 1
+IN_BLOCK = 2
 
 
 # --------------------------------------------------------------------------- building blocks
@@ -114,7 +121,8 @@ class Model:
 
     ``weights`` holds fp64 arrays in nn.Linear layout [out][in]:
     embed [V][d], lm_head [V][d], final_norm [d], layers[l] = {wq, wk, wv, wo,
-    w_gate, w_up, w_down, attn_norm, ffn_norm}, in_norm/in_w1/in_w2 for IN_MLP2.
+    w_gate, w_up, w_down, attn_norm, ffn_norm}, in_norm/in_w1/in_w2 for IN_MLP2,
+    in_block = {the same keys as a layer} for IN_BLOCK.
     ``resid_scale`` = s_l per layer, ``in_scale`` = s_in.
     """
 
@@ -126,10 +134,11 @@ class Model:
 
 
 class KVCache:
-    """One cache for the draft and the full model: K, V [L][n_heads][S_max][head_dim]."""
+    """One cache for the draft and the full model: K, V [L][n_heads][S_max][head_dim]
+    (slot L: the IN_BLOCK imitation block)."""
 
     def __init__(self, cfg: OracleConfig, max_seq: int):
-        shp = (cfg.n_layers, cfg.n_heads, max_seq, cfg.head_dim)
+        shp = (cfg.n_layers + (1 if cfg.in_kind == IN_BLOCK else 0), cfg.n_heads, max_seq, cfg.head_dim)
         self.k = np.zeros(shp)
         self.v = np.zeros(shp)
 
@@ -138,22 +147,36 @@ def embed(m: Model, token: int) -> np.ndarray:
     return m.w["embed"][token].copy()
 
 
-def layer_row(m: Model, l: int, x: np.ndarray, pos: int, cache: KVCache) -> np.ndarray:
-    """x_{l+1} = x_l + f_l(x_l) for one row at position ``pos``; writes K/V[l][:, pos]."""
-    c, lw = m.cfg, m.w["layers"][l]
+def block_row(m: Model, lw: dict, s: float, slot: int, x: np.ndarray, pos: int, cache: KVCache) -> np.ndarray:
+    """x + f(x) for one pre-norm block (weights lw, residual scale s) and one row at position
+    ``pos``; writes K/V[slot][:, pos] and attends over K/V[slot][:, 0..pos]."""
+    c = m.cfg
     H, Dh = c.n_heads, c.head_dim
     n = rms_norm(x, lw["attn_norm"], c.rms_eps)
     q = rope((lw["wq"] @ n).reshape(H, Dh), pos, c.rope_theta)
     k = rope((lw["wk"] @ n).reshape(H, Dh), pos, c.rope_theta)
     v = (lw["wv"] @ n).reshape(H, Dh)
-    cache.k[l, :, pos] = k
-    cache.v[l, :, pos] = v
-    keys, vals = cache.k[l, :, :pos + 1], cache.v[l, :, :pos + 1]      # causal: keys 0..pos
+    cache.k[slot, :, pos] = k
+    cache.v[slot, :, pos] = v
+    keys, vals = cache.k[slot, :, :pos + 1], cache.v[slot, :, :pos + 1]      # causal: keys 0..pos
     scores = np.einsum("hd,hjd->hj", q, keys) / np.sqrt(Dh)
     o = np.einsum("hj,hjd->hd", softmax(scores), vals).reshape(H * Dh)
-    h = x + m.s[l] * (lw["wo"] @ o)
+    h = x + s * (lw["wo"] @ o)
     u = rms_norm(h, lw["ffn_norm"], c.rms_eps)
-    return h + m.s[l] * (lw["w_down"] @ (silu(lw["w_gate"] @ u) * (lw["w_up"] @ u)))
+    return h + s * (lw["w_down"] @ (silu(lw["w_gate"] @ u) * (lw["w_up"] @ u)))
+
+
+def layer_row(m: Model, l: int, x: np.ndarray, pos: int, cache: KVCache) -> np.ndarray:
+    """x_{l+1} = x_l + f_l(x_l) for one row at position ``pos``; writes K/V[l][:, pos]."""
+    return block_row(m, m.w["layers"][l], m.s[l], l, x, pos, cache)
+
+
+def block_kv(m: Model, x: np.ndarray, pos: int, cache: KVCache) -> None:
+    """The IN_BLOCK block's K/V of x (a row's x_k) at ``pos``, without the rest of the block."""
+    c, lw, slot = m.cfg, m.w["in_block"], m.cfg.n_layers
+    n = rms_norm(x, lw["attn_norm"], c.rms_eps)
+    cache.k[slot, :, pos] = rope((lw["wk"] @ n).reshape(c.n_heads, c.head_dim), pos, c.rope_theta)
+    cache.v[slot, :, pos] = (lw["wv"] @ n).reshape(c.n_heads, c.head_dim)
 
 
 def forward_row(m: Model, x: np.ndarray, pos: int, cache: KVCache, layers) -> np.ndarray:
@@ -167,10 +190,13 @@ def lm_head(m: Model, x: np.ndarray) -> np.ndarray:
     return m.w["lm_head"] @ rms_norm(x, m.w["final_norm"], m.cfg.rms_eps)
 
 
-def imitation(m: Model, x: np.ndarray) -> np.ndarray:
-    """x_I = I(x_k): identity, or x + s_in W2 SiLU(W1 RMSNorm_in(x))."""
+def imitation(m: Model, x: np.ndarray, pos: int | None = None, cache: KVCache | None = None) -> np.ndarray:
+    """x_I = I(x_k): identity, x + s_in W2 SiLU(W1 RMSNorm_in(x)), or (IN_BLOCK) the imitation
+    block at position ``pos`` over its own cache slot."""
     if m.cfg.in_kind == IN_IDENTITY:
         return x
+    if m.cfg.in_kind == IN_BLOCK:
+        return block_row(m, m.w["in_block"], m.s_in, m.cfg.n_layers, x, pos, cache)
     n = rms_norm(x, m.w["in_norm"], m.cfg.rms_eps)
     return x + m.s_in * (m.w["in_w2"] @ silu(m.w["in_w1"] @ n))
 
@@ -186,7 +212,19 @@ def prefill(m: Model, cache: KVCache, vis: np.ndarray, prompt) -> np.ndarray:
     H, Dh, P = c.n_heads, c.head_dim, vis.shape[0] + len(prompt)
     X = np.concatenate([vis, m.w["embed"][np.asarray(prompt, dtype=np.int64)]], axis=0)
     causal = np.tril(np.ones((P, P), dtype=bool))
+
+    def block_kv_rows(X):                                        # the imitation block's K/V of every x_k row
+        lw = m.w["in_block"]
+        N = rms_norm(X, lw["attn_norm"], c.rms_eps)
+        K = (N @ lw["wk"].T).reshape(P, H, Dh)
+        for p in range(P):
+            K[p] = rope(K[p], p, c.rope_theta)
+        cache.k[c.n_layers, :, :P] = K.transpose(1, 0, 2)
+        cache.v[c.n_layers, :, :P] = (N @ lw["wv"].T).reshape(P, H, Dh).transpose(1, 0, 2)
+
     for l in range(c.n_layers):
+        if l == c.draft_exit_k and c.in_kind == IN_BLOCK:
+            block_kv_rows(X)
         lw = m.w["layers"][l]
         N = rms_norm(X, lw["attn_norm"], c.rms_eps)
         Q = (N @ lw["wq"].T).reshape(P, H, Dh)
@@ -203,6 +241,8 @@ def prefill(m: Model, cache: KVCache, vis: np.ndarray, prompt) -> np.ndarray:
         Hh = X + m.s[l] * (O @ lw["wo"].T)
         U = rms_norm(Hh, lw["ffn_norm"], c.rms_eps)
         X = Hh + m.s[l] * ((silu(U @ lw["w_gate"].T) * (U @ lw["w_up"].T)) @ lw["w_down"].T)
+    if c.draft_exit_k == c.n_layers and c.in_kind == IN_BLOCK:
+        block_kv_rows(X)
     return lm_head(m, X[-1])
 
 
@@ -291,7 +331,7 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
         for j in range(g_eff):                                   # drafting stage
             x = forward_row(m, embed(m, toks[j]), p + j, cache, range(k))
             xk.append(x)
-            od = lm_head(m, imitation(m, x))
+            od = lm_head(m, imitation(m, x, p + j, cache))
             dlog.append(od)
             toks.append(argmax_lowest(od))
         f, flog = [], []
@@ -300,6 +340,8 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                 x = xk[i]
             else:
                 x = forward_row(m, embed(m, toks[i]), p + i, cache, range(k))
+                if c.in_kind == IN_BLOCK:                        # the block's K/V of this row's x_k
+                    block_kv(m, x, p + i, cache)
             x = forward_row(m, x, p + i, cache, range(k, L))
             of = lm_head(m, x)
             flog.append(of)
@@ -343,4 +385,6 @@ def model_from_bits(w, bits: dict, to_f64) -> Model:
     for n in ("in_norm", "in_w1", "in_w2"):
         if n in bits:
             f[n] = to_f64(bits[n])
+    if "in_block" in bits:
+        f["in_block"] = {n: to_f64(a) for n, a in bits["in_block"].items()}
     return Model(config_from_workload(w), f, w.resid_scale().astype(np.float64), w.in_scale())

@@ -103,6 +103,8 @@ def f32_to_bf16(x: np.ndarray) -> np.ndarray:
 
 IN_IDENTITY = 0   # draft without imitation: g(x_k) directly
 IN_MLP2 = 1       # x + s_in * W2 SiLU(W1 RMSNorm(x)): two FC layers and one norm
+IN_BLOCK = 2      # one decoder block of the model's shape, with its own KV cache
+IN_BLOCK_LAYER = 0xFFFF   # stream index of the block's weights (no decoder layer uses it)
 
 
 @dataclasses.dataclass(frozen=True)
@@ -173,6 +175,10 @@ LLAVA13B_SHAPE = ModelShape(n_layers=40, d_model=5120, n_heads=40, head_dim=128,
 TINY = Workload(name="tiny_L4_d256", shape=TINY_SHAPE, draft_exit_k=2, in_kind=IN_MLP2,
                 in_hidden=1024, gamma=4, n_vis=32, n_prompt=16, max_new=32, s=1.0)
 
+# The same tiny model with the imitation module read literally as one decoder block of the model's
+# shape (its own attention over its own KV cache, SwiGLU MLP, two RMSNorms).
+TINY_BLOCK = TINY.replace(name="tiny_L4_d256_inblock", in_kind=IN_BLOCK)
+
 # LLaVA-1.5-7B-shaped decoder: 576 visual rows (24x24 grid) + 64 prompt ids, k=8, gamma=5.
 LLAVA7B = Workload(name="llava15_7b_shape", shape=LLAVA7B_SHAPE, draft_exit_k=8, in_kind=IN_MLP2,
                    in_hidden=4096, gamma=5, n_vis=576, n_prompt=64, max_new=128, s=0.2)
@@ -212,7 +218,8 @@ def make_weights(w: Workload) -> dict:
     """All weights of the workload as bf16 bit arrays, nn.Linear layout [out][in].
 
     Returns {"embed", "lm_head", "final_norm", "layers": [ {wq, ...}, ... ],
-             "in_norm", "in_w1", "in_w2"} (IN entries absent for IN_IDENTITY).
+             "in_norm", "in_w1", "in_w2"} (IN_MLP2) or "in_block": {wq, ...} (IN_BLOCK);
+    no IN entries for IN_IDENTITY.
     """
     sh = w.shape
     d, V = sh.d_model, sh.vocab
@@ -223,14 +230,19 @@ def make_weights(w: Workload) -> dict:
         "final_norm": _gain(w, "final_norm", 0, d),
         "layers": [],
     }
-    for l in range(sh.n_layers):
+    def block(l: int) -> dict:
         lw = {}
         for name, shp in layer_shapes(sh).items():
             if name.endswith("norm"):
                 lw[name] = _gain(w, name, l, shp[0])
             else:
                 lw[name] = normal_bf16(w.weight_seed, stream_id(name, l), shp, std=std)
-        out["layers"].append(lw)
+        return lw
+
+    for l in range(sh.n_layers):
+        out["layers"].append(block(l))
+    if w.in_kind == IN_BLOCK:
+        out["in_block"] = block(IN_BLOCK_LAYER)
     if w.in_kind == IN_MLP2:
         out["in_norm"] = _gain(w, "in_norm", 0, d)
         out["in_w1"] = normal_bf16(w.weight_seed, stream_id("in_w1"), (w.in_hidden, d), std=std)

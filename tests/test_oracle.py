@@ -318,3 +318,67 @@ def test_ssd_dynamic_draft_length_equals_greedy(tiny_bits, s, cap, n_max):
         assert len(drafts) == g_t and 0 <= a <= g_t
         p, n = kv, n + a + 1
     assert p == r.kv_len == g.kv_len
+
+
+# --------------------------------------------------------------------------- IN_BLOCK imitation (one decoder block)
+
+def torch_block_rows(m: oracle.Model, vis: np.ndarray, tokens):
+    """No-cache torch forward of rows [z; embed(tokens)] through layers 0..k-1 (x_k of every row),
+    then the imitation block applied causally over those rows: returns (X_k, block K, block V,
+    block output) in fp64."""
+    c, W = m.cfg, m.w
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    H, Dh, half = c.n_heads, c.head_dim, c.head_dim // 2
+    X = torch.cat([t(vis), t(W["embed"])[torch.as_tensor(np.asarray(tokens, dtype=np.int64))]], 0)
+    P = X.shape[0]
+    inv = c.rope_theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / Dh)
+    rot = torch.polar(torch.ones(P, half, dtype=torch.float64), torch.arange(P, dtype=torch.float64)[:, None] * inv)
+
+    def rope_c(Z):
+        z = torch.complex(Z[..., :half], Z[..., half:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], -1)
+
+    def block(X, lw, s):
+        N = F.rms_norm(X, (c.d_model,), lw["attn_norm"], c.rms_eps)
+        Q = rope_c((N @ lw["wq"].T).view(P, H, Dh))
+        K = rope_c((N @ lw["wk"].T).view(P, H, Dh))
+        V = (N @ lw["wv"].T).view(P, H, Dh)
+        O = F.scaled_dot_product_attention(Q.transpose(0, 1)[None], K.transpose(0, 1)[None], V.transpose(0, 1)[None],
+                                           is_causal=True)[0]
+        Y = X + s * (O.transpose(0, 1).reshape(P, H * Dh) @ lw["wo"].T)
+        U = F.rms_norm(Y, (c.d_model,), lw["ffn_norm"], c.rms_eps)
+        return Y + s * ((F.silu(U @ lw["w_gate"].T) * (U @ lw["w_up"].T)) @ lw["w_down"].T), K, V
+
+    for l in range(c.draft_exit_k):
+        X, _, _ = block(X, {k: t(v) for k, v in W["layers"][l].items()}, m.s[l])
+    out, K, V = block(X, {k: t(v) for k, v in W["in_block"].items()}, m.s_in)
+    return X.numpy(), K.numpy(), V.numpy(), out.numpy()
+
+
+def test_in_block_first_draft_matches_torch_no_cache_forward():
+    """The first draft token's logits g(I(x_k)) with I one decoder block over its own cache (filled by
+    the prefill for the prompt rows) equal a no-cache torch forward of the whole sequence."""
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=0.2, max_new=3)
+    m, vis, prompt = build(w)
+    r = oracle.ssd_generate(m, vis, prompt, w.max_new, 2, keep_draft_logits=True)
+    y = r.tokens[0]
+    _, _, _, out = torch_block_rows(m, vis, list(prompt) + [y])
+    ref = m.w["lm_head"] @ oracle.rms_norm(out[-1], m.w["final_norm"], m.cfg.rms_eps)
+    np.testing.assert_allclose(r.draft_logits[0][0], ref, rtol=1e-9, atol=1e-9)
+
+
+@pytest.mark.parametrize("s,gamma,k", [(0.05, 4, 2), (0.2, 4, 2), (1.0, 3, 1), (0.05, 6, 4)])
+def test_in_block_ssd_equals_greedy_and_block_cache_matches(s, gamma, k):
+    """SSD with the block imitation equals greedy decoding; afterwards the block's cache rows at
+    every position below kv_len hold the block K/V of that token's x_k (no-cache torch forward):
+    prompt rows from the prefill, drafted rows from the drafts, row gamma from the verification."""
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=s, gamma=gamma, draft_exit_k=k)
+    m, vis, prompt = build(w)
+    g = oracle.greedy_generate(m, vis, prompt, w.max_new)
+    r = oracle.ssd_generate(m, vis, prompt, w.max_new, gamma, keep_cache=True)
+    assert r.tokens == g.tokens
+    _, K, V, _ = torch_block_rows(m, vis, list(prompt) + r.tokens[:-1])
+    n = r.kv_len
+    L = m.cfg.n_layers
+    np.testing.assert_allclose(r.cache.k[L, :, :n], K.transpose(1, 0, 2)[:, :n], rtol=1e-9, atol=1e-9)
+    np.testing.assert_allclose(r.cache.v[L, :, :n], V.transpose(1, 0, 2)[:, :n], rtol=1e-9, atol=1e-9)
