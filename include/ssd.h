@@ -63,7 +63,9 @@ typedef enum {
 /* Imitation network variants (Sec. "Methodology", Deep Representation Imitation). */
 enum {
   SSD_IN_IDENTITY = 0,  /* draft without imitation: g(x_k) ("Draft w/o Im", Table 1) */
-  SSD_IN_MLP2 = 1       /* x + s_in * W2 SiLU(W1 RMSNorm_in(x)): two FC layers + one norm */
+  SSD_IN_MLP2 = 1,      /* x + s_in * W2 SiLU(W1 RMSNorm_in(x)): two FC layers + one norm */
+  SSD_IN_BLOCK = 2      /* one decoder block of the model's shape with its own KV cache, residual
+                         * writes scaled by s_in (the module read as a block; Sec. "Choice of n") */
 };
 
 #define SSD_MAX_GAMMA 8
@@ -113,6 +115,12 @@ typedef struct {
    * decode calls: s_l scales both residual writes of layer l, s_in the IN's. */
   const float* resid_scale; /* [n_layers] */
   const float* in_scale;    /* [1] */
+  /* SSD_IN_BLOCK: host array of 9 device pointers, the block's wq, wk, wv, wo,
+   * w_gate, w_up, w_down, attn_norm, ffn_norm (layouts as above); NULL otherwise.
+   * Its cache rows hold the block's K/V of every position's x_k: the prefill
+   * fills the prompt rows, each drafting step its row, the verification pass
+   * row gamma. */
+  const void* const* in_block;
 } ssd_weights;
 
 /* Counters of the last prefill+decode, read back by ssd_get_stats. */
@@ -219,8 +227,9 @@ SSD_API ssd_status ssd_get_stats(ssd_ctx* ctx, ssd_stats* stats);
 SSD_API ssd_status ssd_set_logits_capture(ssd_ctx* ctx, float* buf, int max_rows);
 
 /* Device pointers to the KV cache, layout [L][n_heads][max_seq][head_dim]
- * fp32, and the current valid length (sync read).  Positions >= kv_len hold
- * stale rows of rejected drafts. */
+ * fp32 (with SSD_IN_BLOCK, [L + 1]: slot L is the imitation block's), and the
+ * current valid length (sync read).  Positions >= kv_len hold stale rows of
+ * rejected drafts. */
 SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v_cache, int* kv_len);
 
 /* Number of kernel launches the last ssd_decode / ssd_greedy_decode /

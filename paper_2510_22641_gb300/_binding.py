@@ -16,6 +16,7 @@ SSD_MAX_GAMMA = 8
 SSD_MAX_ROWS = 16
 SSD_IN_IDENTITY = 0
 SSD_IN_MLP2 = 1
+SSD_IN_BLOCK = 2
 
 STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_CUDA", 4: "SSD_ERR_CAPACITY",
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
@@ -44,7 +45,7 @@ class SSDWeights(ctypes.Structure):
                 ("wq", _PP), ("wk", _PP), ("wv", _PP), ("wo", _PP), ("w_gate", _PP), ("w_up", _PP),
                 ("w_down", _PP), ("attn_norm", _PP), ("ffn_norm", _PP),
                 ("in_norm", ctypes.c_void_p), ("in_w1", ctypes.c_void_p), ("in_w2", ctypes.c_void_p),
-                ("resid_scale", ctypes.c_void_p), ("in_scale", ctypes.c_void_p)]
+                ("resid_scale", ctypes.c_void_p), ("in_scale", ctypes.c_void_p), ("in_block", _PP)]
 
 
 class SSDStats(ctypes.Structure):

@@ -368,9 +368,38 @@ static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch
 
 // One decoder layer x_{l+1} = x_l + f_l(x_l) on rows row0 .. row0+M-1 of xv at
 // positions kv_len + pos_off + m.
+// s_l of layer l; for l == n_layers (the IN_BLOCK imitation block) s_in.
+static const float* resid_scale_of(const ssd_ctx* c, int l) {
+  return l < c->cfg.n_layers ? c->resid_scale + l : c->in_scale;
+}
+
+// The QKV projection of block l on M rows x alone (RoPE + K/V writes at kv_len + pos_off + m):
+// the IN_BLOCK block's cache rows of x_k rows whose block output is not needed.
+static ssd_status enqueue_qkv_only(ssd_ctx* c, int l, const float* x, int M, int pos_off) {
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = c->dp;
+  p.gain = c->attn_norm[l];
+  p.pos_off = pos_off;
+  p.q_out = c->qb;
+  p.q_stride = c->qp;
+  p.k_cache = c->kc + l * c->layer_kv;
+  p.v_cache = c->vc + l * c->layer_kv;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  p.rope_cs = c->rope;
+  return gemv(c, Epi::QKV, M, c->layers[l].qkv, p);
+}
+
+static ssd_status enqueue_layer_x(ssd_ctx* c, int l, float* x, int M, int pos_off);
+
 static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off) {
+  return enqueue_layer_x(c, l, c->xv + static_cast<size_t>(row0) * c->dp, M, pos_off);
+}
+
+// Block l (a decoder layer, or the IN_BLOCK block for l == n_layers) on M rows x, in place.
+static ssd_status enqueue_layer_x(ssd_ctx* c, int l, float* x, int M, int pos_off) {
   const int d = c->dp;
-  float* x = c->xv + static_cast<size_t>(row0) * d;
   GemvParams p{};
   p.x = x;
   p.x_stride = d;
@@ -393,7 +422,7 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   p.base_stride = d;
   p.dst = x;
   p.dst_stride = d;
-  p.scale = c->resid_scale + l;
+  p.scale = resid_scale_of(c, l);
   CKS(gemv(c, Epi::RESID, M, c->layers[l].o, p));
   p = GemvParams{};
   p.x = x;
@@ -409,7 +438,7 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   p.base_stride = d;
   p.dst = x;
   p.dst_stride = d;
-  p.scale = c->resid_scale + l;
+  p.scale = resid_scale_of(c, l);
   CKS(gemv(c, Epi::RESID, M, c->layers[l].down, p));
   return SSD_OK;
 }
@@ -783,6 +812,8 @@ static ssd_status fwd_run(ssd_ctx* c, const FwdProg& pr) {
 
 static ssd_status fwd_ensure(ssd_ctx* c) {
   if (!c->use_fwd || c->fwd_ready) return SSD_OK;
+  if (c->cfg.in_kind == SSD_IN_BLOCK)
+    return fail(c, SSD_ERR_UNSUPPORTED, "the persistent forward kernel has no imitation-block program");
   return fwd_build_programs(c);
 }
 
@@ -797,6 +828,11 @@ static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
                 c->cfg.d_model, c->cfg.vocab, c->st));
     for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, j, 1, j));
     const float* hx = xj;
+    if (c->cfg.in_kind == SSD_IN_BLOCK) {  // I(x_k): the imitation block on a copy (x_k stays for verification)
+      CK(cudaMemcpyAsync(c->xt, xj, sizeof(float) * d, cudaMemcpyDeviceToDevice, c->cs));
+      CKS(enqueue_layer_x(c, c->cfg.n_layers, c->xt, 1, j));
+      hx = c->xt;
+    }
     if (c->cfg.in_kind == SSD_IN_MLP2) {
       GemvParams p{};
       p.x = xj;
@@ -837,6 +873,8 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
   CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
               c->xv + static_cast<size_t>(gamma) * d, d, c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, gamma, 1, gamma));
+  if (c->cfg.in_kind == SSD_IN_BLOCK)  // the imitation block's cache row of d_gamma's x_k
+    CKS(enqueue_qkv_only(c, c->cfg.n_layers, c->xv + static_cast<size_t>(gamma) * d, 1, gamma));
   for (int l = c->cfg.draft_exit_k; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, gamma + 1, 0));
   CKS(enqueue_head(c, c->xv, gamma + 1, 0, full_tok, true));
   CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, cond,
@@ -873,7 +911,13 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
     const int Mc = P - r0 < kPrefillChunk ? P - r0 : kPrefillChunk;
     CK(launch_k(c, prefill_rows_kernel, dim3(Mc), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
                 static_cast<const int*>(c->in_prompt), n_vis, r0, c->embed, c->cfg.vocab, c->xv, d, c->cfg.d_model, c->st));
-    for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, Mc, r0));
+    for (int l = 0; l < c->cfg.n_layers; ++l) {
+      if (l == c->cfg.draft_exit_k && c->cfg.in_kind == SSD_IN_BLOCK)  // the block's cache rows of x_k
+        CKS(enqueue_qkv_only(c, c->cfg.n_layers, c->xv, Mc, r0));
+      CKS(enqueue_layer(c, l, 0, Mc, r0));
+    }
+    if (c->cfg.draft_exit_k == c->cfg.n_layers && c->cfg.in_kind == SSD_IN_BLOCK)
+      CKS(enqueue_qkv_only(c, c->cfg.n_layers, c->xv, Mc, r0));
   }
   r0 -= kPrefillChunk;
   CKS(enqueue_head(c, c->xv + static_cast<size_t>(P - 1 - r0) * d, 1, P - 1, full_tok, true));
@@ -913,7 +957,23 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
               c->st));
+  // the IN_BLOCK block's cache rows of every prompt row's x_k: its QKV GEMM alone
+  auto block_kv = [&]() -> ssd_status {
+    const int b = c->cfg.n_layers;
+    TcParams p{};
+    p.pos0 = 0;
+    p.q_out = c->q_pre;
+    p.q_stride = c->qp;
+    p.k_cache = c->kc + b * c->layer_kv;
+    p.v_cache = c->vc + b * c->layer_kv;
+    p.head_dim = c->cfg.head_dim;
+    p.max_seq = c->cfg.max_seq;
+    p.rope_cs = c->rope;
+    CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->attn_norm[b], P));
+    return tc_gemm(c, Epi::QKV, 0, c->tc_layers[b].qkv, P, p);
+  };
   for (int l = 0; l < c->cfg.n_layers; ++l) {
+    if (l == c->cfg.draft_exit_k && c->cfg.in_kind == SSD_IN_BLOCK) CKS(block_kv());
     const TcLayer& tl = c->tc_layers[l];
     TcParams p{};
     p.pos0 = 0;
@@ -936,7 +996,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     p.base_stride = dp;
     p.dst = c->x_pre;
     p.dst_stride = dp;
-    p.scale = c->resid_scale + l;
+    p.scale = resid_scale_of(c, l);
     CKS(tc_gemm(c, Epi::RESID, 1, tl.o, P, p));
     CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->ffn_norm[l], P));
     p = TcParams{};
@@ -949,9 +1009,10 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     p.base_stride = dp;
     p.dst = c->x_pre;
     p.dst_stride = dp;
-    p.scale = c->resid_scale + l;
+    p.scale = resid_scale_of(c, l);
     CKS(tc_gemm(c, Epi::RESID, 2, tl.down, P, p));
   }
+  if (c->cfg.draft_exit_k == c->cfg.n_layers && c->cfg.in_kind == SSD_IN_BLOCK) CKS(block_kv());
   CKS(enqueue_head(c, c->x_pre + static_cast<size_t>(P - 1) * dp, 1, P - 1, full_tok, true));
   CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
   return SSD_OK;
@@ -1256,7 +1317,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (k.d_model % kAlign || k.d_ff % kAlign || qdim % 128)
     return fail(c, SSD_ERR_INVALID_ARG, "d_model, d_ff must be multiples of 64 and n_heads*head_dim of 128");
   if (k.draft_exit_k < 1 || k.draft_exit_k > k.n_layers) return fail(c, SSD_ERR_INVALID_ARG, "draft_exit_k");
-  if (k.in_kind != SSD_IN_IDENTITY && k.in_kind != SSD_IN_MLP2) return fail(c, SSD_ERR_INVALID_ARG, "in_kind");
+  if (k.in_kind != SSD_IN_IDENTITY && k.in_kind != SSD_IN_MLP2 && k.in_kind != SSD_IN_BLOCK)
+    return fail(c, SSD_ERR_INVALID_ARG, "in_kind");
   if (k.in_kind == SSD_IN_MLP2 && (k.in_hidden < 64 || k.in_hidden % kAlign))
     return fail(c, SSD_ERR_INVALID_ARG, "in_hidden must be a positive multiple of 64");
   if (k.gamma_max < 1 || k.gamma_max > SSD_MAX_GAMMA || k.gamma_max + 1 > kMaxVerifyRows)
@@ -1267,6 +1329,11 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer");
   if (k.in_kind == SSD_IN_MLP2 && (!w->in_norm || !w->in_w1 || !w->in_w2 || !w->in_scale))
     return fail(c, SSD_ERR_INVALID_ARG, "null imitation-network weight pointer");
+  if (k.in_kind == SSD_IN_BLOCK) {
+    if (!w->in_block || !w->in_scale) return fail(c, SSD_ERR_INVALID_ARG, "null imitation-block weight pointer");
+    for (int i = 0; i < 9; ++i)
+      if (!w->in_block[i]) return fail(c, SSD_ERR_INVALID_ARG, "null imitation-block weight pointer %d", i);
+  }
   for (int l = 0; l < k.n_layers; ++l)
     if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->w_gate[l] || !w->w_up[l] || !w->w_down[l] ||
         !w->attn_norm[l] || !w->ffn_norm[l])
@@ -1318,44 +1385,53 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   c->in_norm = static_cast<const __nv_bfloat16*>(w->in_norm);
   c->resid_scale = w->resid_scale;
   c->in_scale = w->in_scale;
-  c->layers.resize(k.n_layers);
-  for (int l = 0; l < k.n_layers; ++l) {
-    c->attn_norm.push_back(static_cast<const __nv_bfloat16*>(w->attn_norm[l]));
-    c->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(w->ffn_norm[l]));
-    const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
+  // layer l's weights; l == n_layers: the IN_BLOCK imitation block
+  const int n_blocks = k.n_layers + (k.in_kind == SSD_IN_BLOCK ? 1 : 0);
+  auto wt = [&](int l, int i) -> const void* {
+    if (l == k.n_layers) return w->in_block[i];
+    const void* const* a[9] = {w->wq, w->wk, w->wv, w->wo, w->w_gate, w->w_up, w->w_down, w->attn_norm, w->ffn_norm};
+    return a[i][l];
+  };
+  c->layers.resize(n_blocks);
+  for (int l = 0; l < n_blocks; ++l) {
+    c->attn_norm.push_back(static_cast<const __nv_bfloat16*>(wt(l, 7)));
+    c->ffn_norm.push_back(static_cast<const __nv_bfloat16*>(wt(l, 8)));
+    const void* qkv[3] = {wt(l, 0), wt(l, 1), wt(l, 2)};
+    const void* wo_l = wt(l, 3);
+    const void* wd_l = wt(l, 6);
     CKS(make_site(c, &c->layers[l].qkv, qkv, 3, qdim, k.d_model, false));
-    CKS(make_site(c, &c->layers[l].o, &w->wo[l], 1, k.d_model, qdim, false));
-    CKS(make_pair_site(c, &c->layers[l].gateup, w->w_gate[l], w->w_up[l], k.d_ff, k.d_model));
-    CKS(make_site(c, &c->layers[l].down, &w->w_down[l], 1, k.d_model, k.d_ff, false));
+    CKS(make_site(c, &c->layers[l].o, &wo_l, 1, k.d_model, qdim, false));
+    CKS(make_pair_site(c, &c->layers[l].gateup, wt(l, 4), wt(l, 5), k.d_ff, k.d_model));
+    CKS(make_site(c, &c->layers[l].down, &wd_l, 1, k.d_model, k.d_ff, false));
   }
   if (k.in_kind == SSD_IN_MLP2) {
     CKS(make_site(c, &c->in1, &w->in_w1, 1, k.in_hidden, k.d_model, false));
     CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden, false));
   }
   CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model, false));
-  c->tc_layers.resize(k.n_layers);
-  for (int l = 0; l < k.n_layers; ++l) {
+  c->tc_layers.resize(n_blocks);
+  for (int l = 0; l < n_blocks; ++l) {
     TcLayer& t = c->tc_layers[l];
-    const void* qkv[3] = {w->wq[l], w->wk[l], w->wv[l]};
+    const void* qkv[3] = {wt(l, 0), wt(l, 1), wt(l, 2)};
     for (int i = 0; i < 3; ++i) CKS(encode_map_sw128(c, &t.qkv.maps[i], qkv[i], qdim, k.d_model, kTcN));
     t.qkv.N = 3 * qdim;
     t.qkv.K = k.d_model;
     t.qkv.seg_rows = qdim;
     t.qkv.tiles_n = 3 * qdim / kTcN;
-    CKS(encode_map_sw128(c, &t.o.maps[0], w->wo[l], k.d_model, qdim, kTcN));
+    CKS(encode_map_sw128(c, &t.o.maps[0], wt(l, 3), k.d_model, qdim, kTcN));
     t.o.maps[1] = t.o.maps[2] = t.o.maps[0];
     t.o.N = k.d_model;
     t.o.K = qdim;
     t.o.seg_rows = k.d_model;
     t.o.tiles_n = (k.d_model + kTcN - 1) / kTcN;
-    CKS(encode_map_sw128(c, &t.gateup.maps[0], w->w_gate[l], k.d_ff, k.d_model, kTcN / 2));
-    CKS(encode_map_sw128(c, &t.gateup.maps[1], w->w_up[l], k.d_ff, k.d_model, kTcN / 2));
+    CKS(encode_map_sw128(c, &t.gateup.maps[0], wt(l, 4), k.d_ff, k.d_model, kTcN / 2));
+    CKS(encode_map_sw128(c, &t.gateup.maps[1], wt(l, 5), k.d_ff, k.d_model, kTcN / 2));
     t.gateup.maps[2] = t.gateup.maps[0];
     t.gateup.N = k.d_ff;
     t.gateup.K = k.d_model;
     t.gateup.seg_rows = k.d_ff;
     t.gateup.tiles_n = (k.d_ff + kTcN / 2 - 1) / (kTcN / 2);
-    CKS(encode_map_sw128(c, &t.down.maps[0], w->w_down[l], k.d_model, k.d_ff, kTcN));
+    CKS(encode_map_sw128(c, &t.down.maps[0], wt(l, 6), k.d_model, k.d_ff, kTcN));
     t.down.maps[1] = t.down.maps[2] = t.down.maps[0];
     t.down.N = k.d_model;
     t.down.K = k.d_ff;
@@ -1376,7 +1452,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CKS(alloc(c, reinterpret_cast<void**>(&c->hb), sizeof(float) * R * c->fp));
   CKS(alloc(c, reinterpret_cast<void**>(&c->hin), sizeof(float) * R * c->ip));
   // RMSNorm gains: zero-padded copies, so 256-column slices never read past a gain vector
-  const int n_gains = 2 * k.n_layers + 2;
+  const int n_gains = 2 * n_blocks + 2;
   CKS(alloc(c, reinterpret_cast<void**>(&c->gains), sizeof(__nv_bfloat16) * n_gains * c->dp));
   auto copy_gain = [&](int slot, const void* src) -> const __nv_bfloat16* {
     __nv_bfloat16* dst = c->gains + static_cast<size_t>(slot) * c->dp;
@@ -1384,18 +1460,18 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
       return nullptr;
     return dst;
   };
-  for (int l = 0; l < k.n_layers; ++l) {
-    c->attn_norm[l] = copy_gain(2 * l, w->attn_norm[l]);
-    c->ffn_norm[l] = copy_gain(2 * l + 1, w->ffn_norm[l]);
+  for (int l = 0; l < n_blocks; ++l) {
+    c->attn_norm[l] = copy_gain(2 * l, wt(l, 7));
+    c->ffn_norm[l] = copy_gain(2 * l + 1, wt(l, 8));
     if (!c->attn_norm[l] || !c->ffn_norm[l]) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
   }
-  c->final_norm = copy_gain(2 * k.n_layers, w->final_norm);
-  c->in_norm = k.in_kind == SSD_IN_MLP2 ? copy_gain(2 * k.n_layers + 1, w->in_norm) : nullptr;
+  c->final_norm = copy_gain(2 * n_blocks, w->final_norm);
+  c->in_norm = k.in_kind == SSD_IN_MLP2 ? copy_gain(2 * n_blocks + 1, w->in_norm) : nullptr;
   if (!c->final_norm || (k.in_kind == SSD_IN_MLP2 && !c->in_norm))
     return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
   c->layer_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
-  CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(float) * c->layer_kv * k.n_layers));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(float) * c->layer_kv * k.n_layers));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(float) * c->layer_kv * n_blocks));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(float) * c->layer_kv * n_blocks));
   CKS(alloc(c, reinterpret_cast<void**>(&c->rope), sizeof(float2) * k.max_seq * (k.head_dim / 2)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->gemv_ctas * c->num_sms * R * kTileN));
   int max_rt = 1;

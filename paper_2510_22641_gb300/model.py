@@ -38,7 +38,8 @@ class SSDModel:
 
     weights: dict with bf16 device tensors "embed", "lm_head", "final_norm",
     "layers" (list of dicts wq, wk, wv, wo, w_gate, w_up, w_down, attn_norm,
-    ffn_norm) and, for the MLP2 imitation network, "in_norm", "in_w1", "in_w2".
+    ffn_norm) and, for the MLP2 imitation network, "in_norm", "in_w1", "in_w2"; for the block
+    imitation network "in_block" (a dict like a layer's).
     resid_scale: fp32 device tensor [n_layers]; in_scale: fp32 device tensor [1].
     """
 
@@ -54,6 +55,9 @@ class SSDModel:
         arrs = {}
         for name in ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down", "attn_norm", "ffn_norm"):
             arrs[name] = (ctypes.c_void_p * L)(*[weights["layers"][l][name].data_ptr() for l in range(L)])
+        if "in_block" in weights:
+            names = ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down", "attn_norm", "ffn_norm")
+            arrs["in_block"] = (ctypes.c_void_p * 9)(*[weights["in_block"][n].data_ptr() for n in names])
         self._arrs = arrs
         w = B.SSDWeights(embed=_ptr(weights["embed"]), lm_head=_ptr(weights["lm_head"]),
                          final_norm=_ptr(weights["final_norm"]),
@@ -144,11 +148,13 @@ class SSDModel:
         self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
 
     def kv(self):
-        """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (fp32) of the library's cache."""
+        """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (fp32) of the library's cache
+        ([L + 1] with the block imitation network, whose rows are slot L)."""
         k, v, n = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_int()
         self._call("ssd_get_kv", ctypes.byref(k), ctypes.byref(v), ctypes.byref(n))
         c = self.cfg
-        shape = (c["n_layers"], c["n_heads"], c["max_seq"], c["head_dim"])
+        slots = c["n_layers"] + (1 if c["in_kind"] == B.SSD_IN_BLOCK else 0)
+        shape = (slots, c["n_heads"], c["max_seq"], c["head_dim"])
         return _device_view(k.value, shape), _device_view(v.value, shape), n.value
 
     def lm_head(self, x: torch.Tensor, tok: torch.Tensor, logits: torch.Tensor | None = None):

@@ -12,6 +12,8 @@ def device_weights(bits: dict) -> dict:
     up = lib.bf16_bits_to_device
     out = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm")}
     out["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+    if "in_block" in bits:
+        out["in_block"] = {n: up(a) for n, a in bits["in_block"].items()}
     for k in ("in_norm", "in_w1", "in_w2"):
         if k in bits:
             out[k] = up(bits[k])

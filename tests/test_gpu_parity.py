@@ -400,3 +400,45 @@ def test_profile_projection_bytes_and_state_recovery(tiny_model):
         model.profile_projection("in1", rows=2)
     after, _, _ = gpu_decode(model, w, 4, capture=False)
     assert after == before
+
+
+# --------------------------------------------------------------------------- IN_BLOCK imitation (one decoder block)
+
+@pytest.fixture(scope="module")
+def block_bits():
+    return synth.make_weights(synth.TINY_BLOCK.replace(norm_gain="perturbed"))
+
+
+@pytest.fixture(scope="module")
+def block_model(block_bits):
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", gamma=8)
+    model, _, dev = make_model(w, block_bits, gamma_max=8, max_seq=w.max_seq())
+    yield model
+    model.close()
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.2, 4), (1.0, 3)])
+def test_in_block_imitation_matches_oracle(block_model, block_bits, s, gamma):
+    """The imitation module as one decoder block with its own KV cache: tokens, logits, steps, accept
+    lengths and kv_len match the oracle; the block's cache rows (prompt rows from the prefill, drafted
+    rows, and row gamma from the verification) match the oracle's; SSD equals GPU greedy decoding."""
+    model = block_model
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=s)
+    set_scale(model, w)
+    if os.environ.get("SSD_DECODE") == "fwd":
+        with pytest.raises(lib.SSDError, match="UNSUPPORTED"):
+            gpu_decode(model, w, gamma)
+        return
+    toks, logits, stats = gpu_decode(model, w, gamma)
+    m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma, keep_cache=True)
+    agree = check_against_oracle(toks, logits, stats, ref, gamma)
+    K, V, n = model.kv()
+    L = w.shape.n_layers
+    upto = min(n, w.prompt_len + agree - 1)
+    np.testing.assert_allclose(K[L, :, :upto].cpu().numpy(), ref.cache.k[L, :, :upto], rtol=2e-3, atol=2e-4)
+    np.testing.assert_allclose(V[L, :, :upto].cpu().numpy(), ref.cache.v[L, :, :upto], rtol=2e-3, atol=2e-4)
+    gtoks, glogits, _ = gpu_decode(model, w, 0)
+    assert toks == gtoks
+    np.testing.assert_array_equal(logits, glogits)
