@@ -231,6 +231,72 @@ def run_reference(args) -> None:
 
 # --------------------------------------------------------------------------- GPU arm
 
+def run_in_block(args) -> None:
+    """The configs[1] workload (7B shape, k = 8, gamma = 5, 128 new tokens) with the imitation module
+    read as one decoder block with its own KV cache (IN_BLOCK): decode tokens/s of SSD and greedy,
+    speedup, accept length and the drafting stage's HBM GB/s, per s.  One JSON line."""
+    import torch
+
+    import paper_2510_22641_gb300 as lib
+    lib.build()
+    w = synth.LLAVA7B.replace(in_kind=synth.IN_BLOCK)
+    bits = synth.make_weights(w)
+    up = lib.bf16_bits_to_device
+    dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm")}
+    dev["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+    dev["in_block"] = {n: up(a) for n, a in bits["in_block"].items()}
+    vis, prompt = synth.make_inputs(w)
+    v = up(vis)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    stream = torch.cuda.current_stream()
+    rs = torch.tensor(w.resid_scale(), device="cuda")
+    ins = torch.tensor([w.in_scale()], device="cuda")
+    cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                          w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1)
+    model = lib.SSDModel(cfg, dev, rs, ins)
+    ab = algorithmic_bytes(w)
+    draft_bytes = w.draft_exit_k * ab["layer"] + ab["layer"] + ab["head"]   # shallow layers + the block + g
+
+    def timed(fn):
+        model.prefill(v, p)
+        fn()
+        model.prefill(v, p)
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    rows = []
+    for s_val in S_VALUES:
+        ws = w.replace(s=s_val)
+        rs.copy_(torch.tensor(ws.resid_scale(), device="cuda"))
+        ins.copy_(torch.tensor([ws.in_scale()], device="cuda"))
+        g_ms = timed(lambda: model.greedy_decode(w.max_new))
+        s_ms = timed(lambda: model.decode(w.max_new, w.gamma))
+        st = model.stats()
+        model.prefill(v, p)
+        model.draft(w.gamma)
+        model.verify(w.gamma)
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        model.draft(w.gamma)
+        b.record(stream)
+        torch.cuda.synchronize()
+        d_ms = a.elapsed_time(b)
+        rows.append({"s": s_val, "ssd_decode_tok_s": (w.max_new - 1) / (s_ms / 1e3),
+                     "greedy_decode_tok_s": (w.max_new - 1) / (g_ms / 1e3), "speedup": g_ms / s_ms,
+                     "mean_accept": st["accepted"] / max(st["steps"], 1), "draft_ms": d_ms,
+                     "draft_gbs": w.gamma * draft_bytes / (d_ms / 1e3) / 1e9})
+    model.close()
+    print(json.dumps({"workload": workload_config(w)["workload"] + ", imitation = one decoder block (IN_BLOCK)",
+                      "per_s": rows}), flush=True)
+
+
 def run_sweep(args) -> None:
     """Sweep k x gamma x s on the 7B shape (256 new tokens): accept length, tokens/s, speedup
     over greedy, draft and verify HBM GB/s.  One JSON line per point."""
@@ -324,9 +390,14 @@ def main() -> None:
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-steps", type=int, default=3, help="oracle SSD steps in the CPU sample")
     ap.add_argument("--sweep", action="store_true", help="k x gamma x s sweep (one JSON line per point)")
+    ap.add_argument("--in-block", action="store_true",
+                    help="the 7B workload with the imitation module as one decoder block (one JSON line)")
     args = ap.parse_args()
     if args.sweep:
         run_sweep(args)
+        return
+    if args.in_block:
+        run_in_block(args)
         return
     if args.impl == "reference":
         run_reference(args)
