@@ -442,3 +442,47 @@ def test_in_block_imitation_matches_oracle(block_model, block_bits, s, gamma):
     gtoks, glogits, _ = gpu_decode(model, w, 0)
     assert toks == gtoks
     np.testing.assert_array_equal(logits, glogits)
+
+
+def test_in_block_with_dynamic_draft_length_matches_oracle(block_model, block_bits):
+    """IN_BLOCK and the dynamic draft length d(t) together: tokens, steps, accept lengths, kv_len."""
+    model = block_model
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=0.05)
+    set_scale(model, w)
+    _, _, v, p = device_inputs(w)
+    out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
+    n = torch.zeros(1, dtype=torch.int32, device="cuda")
+    model.set_logits_capture(None)
+    model.prefill(v, p)
+    if os.environ.get("SSD_DECODE") == "fwd":
+        with pytest.raises(lib.SSDError, match="UNSUPPORTED"):
+            model.decode_dynamic(w.max_new, 5, 120, 8, out, n)
+        return
+    model.decode_dynamic(w.max_new, 5, 120, 8, out, n)
+    model.sync()
+    toks, stats = out[: int(n.item())].cpu().tolist(), model.stats()
+    m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 8, dynamic=(5, 120))
+    agree = common_prefix(toks, ref.tokens, ref.logits)
+    if agree == len(ref.tokens):
+        assert stats["steps"] == len(ref.accept_lengths)
+        assert stats["accepted"] == sum(ref.accept_lengths)
+        assert stats["kv_len"] == ref.kv_len
+
+
+def test_in_block_draft_exit_at_last_layer(block_bits):
+    """k = L: the block's prompt rows come from the final x_L rows (after the last layer), and the
+    verification pass has no deep layers; tokens and stats match the oracle."""
+    if os.environ.get("SSD_DECODE") == "fwd":
+        pytest.skip("the persistent forward kernel path has no imitation-block program")
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=0.2, draft_exit_k=4, gamma=4)
+    model, _, _ = make_model(w, block_bits, gamma_max=4, max_seq=w.max_seq())
+    try:
+        toks, logits, stats = gpu_decode(model, w, 4)
+        m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
+        vis, prompt = synth.make_inputs(w)
+        ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 4)
+        check_against_oracle(toks, logits, stats, ref, 4)
+    finally:
+        model.close()
