@@ -256,3 +256,168 @@ def make_inputs(w: Workload, seed: int | None = None) -> tuple[np.ndarray, np.nd
     vis = normal_bf16(seed, stream_id("vis"), (w.n_vis, w.shape.d_model), std=w.vis_std)
     prompt = uniform_i32(seed, stream_id("prompt"), (w.n_prompt,), 0, w.shape.vocab)
     return vis, prompt
+
+
+# --------------------------------------------------------------------------- encoder-decoder (FlanT5-shaped)
+
+@dataclasses.dataclass(frozen=True)
+class T5Shape:
+    """T5 v1.1 shape: pre-norm blocks, gated-GELU MLP, relative-position bias, untied LM head."""
+    n_enc: int
+    n_dec: int
+    d_model: int
+    n_heads: int
+    head_dim: int
+    d_ff: int
+    vocab: int
+    rel_buckets: int = 32
+    rel_max_distance: int = 128
+
+    @property
+    def qdim(self) -> int:
+        return self.n_heads * self.head_dim
+
+    def dec_layer_bytes_bf16(self) -> int:
+        """Weights one decode row streams per decoder layer (self q/k/v/o, cross q/o, MLP, 3 norms);
+        the cross-attention K/V projections run once per request, over the encoder output."""
+        d, q, f = self.d_model, self.qdim, self.d_ff
+        return 2 * (4 * q * d + 2 * q * d + 3 * f * d) + 2 * 3 * d
+
+
+@dataclasses.dataclass(frozen=True)
+class T5Workload:
+    """One synthetic encoder-decoder self-speculative decoding workload (bs1).
+
+    The encoder reads n_query synthetic query embeddings (the image-grounded queries, N(0, vis_std))
+    followed by n_prompt prompt ids; the decoder starts from token 0 and drafts with decoder layers
+    0..k-1 plus the imitation network.
+    """
+    name: str
+    shape: T5Shape
+    draft_exit_k: int
+    in_kind: int
+    in_hidden: int
+    gamma: int
+    n_query: int
+    n_prompt: int
+    max_new: int
+    s: float = 1.0
+    weight_std: float = 0.02
+    embed_std: float = 1.0
+    rel_std: float = 0.5
+    vis_std: float = 1.0
+    norm_gain: str = "ones"
+    eos_id: int = -1
+    weight_seed: int = 0
+    input_seed: int = 0
+
+    def replace(self, **kw) -> "T5Workload":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def enc_len(self) -> int:
+        return self.n_query + self.n_prompt
+
+    def max_dec(self) -> int:
+        return self.max_new + self.gamma + 1
+
+    def dec_scale(self) -> np.ndarray:
+        """s_l of the decoder: 1 for layers 0..k-1, s for k..L-1 (fp32)."""
+        sc = np.ones(self.shape.n_dec, dtype=np.float32)
+        sc[self.draft_exit_k:] = np.float32(self.s)
+        return sc
+
+    def in_scale(self) -> float:
+        return float(np.float32(self.s))
+
+
+T5_TINY_SHAPE = T5Shape(n_enc=2, n_dec=4, d_model=256, n_heads=4, head_dim=64, d_ff=512, vocab=2048)
+FLANT5XL_SHAPE = T5Shape(n_enc=24, n_dec=24, d_model=2048, n_heads=32, head_dim=64, d_ff=5120, vocab=32128)
+
+# Tiny encoder-decoder parity workload: 2 encoder + 4 decoder layers, draft = decoder layers 0-1 + imitation.
+T5_TINY = T5Workload(name="t5_tiny_e2_d4_d256", shape=T5_TINY_SHAPE, draft_exit_k=2, in_kind=IN_MLP2,
+                     in_hidden=512, gamma=4, n_query=32, n_prompt=16, max_new=24, s=1.0)
+
+# BLIP-2 FlanT5-xl-shaped language model: 32 queries + 16 prompt ids, draft = decoder layers 0-5, gamma=4.
+FLANT5XL = T5Workload(name="blip2_flant5xl_shape", shape=FLANT5XL_SHAPE, draft_exit_k=6, in_kind=IN_MLP2,
+                      in_hidden=2048, gamma=4, n_query=32, n_prompt=16, max_new=30, s=0.2)
+
+_T5_KIND = {
+    "t5_embed": 60, "t5_lm_head": 61, "enc_final": 62, "dec_final": 63, "enc_rel": 64, "dec_rel": 65,
+    "attn_norm": 66, "self_norm": 67, "cross_norm": 68, "ffn_norm": 69,
+    "wq": 70, "wk": 71, "wv": 72, "wo": 73, "cq": 74, "ck": 75, "cv": 76, "co": 77,
+    "wi0": 78, "wi1": 79, "wff": 80, "in_norm": 81, "in_w1": 82, "in_w2": 83,
+    "query": 84, "t5_prompt": 85,
+}
+_T5_DEC = 0x100   # stream-layer offset of decoder layers
+
+
+def t5_stream_id(kind: str, layer: int = 0) -> int:
+    return (_T5_KIND[kind] << 16) | layer
+
+
+def t5_layer_shapes(shape: T5Shape, decoder: bool) -> dict:
+    d, q, f = shape.d_model, shape.qdim, shape.d_ff
+    out = {"wq": (q, d), "wk": (q, d), "wv": (q, d), "wo": (d, q)}
+    if decoder:
+        out.update({"cq": (q, d), "ck": (q, d), "cv": (q, d), "co": (d, q),
+                    "self_norm": (d,), "cross_norm": (d,)})
+    else:
+        out["attn_norm"] = (d,)
+    out.update({"wi0": (f, d), "wi1": (f, d), "wff": (d, f), "ffn_norm": (d,)})
+    return out
+
+
+def make_t5_weights(w: T5Workload) -> dict:
+    """All weights as bf16 bit arrays ([out][in] layouts).
+
+    {"embed" [V][d], "lm_head" [V][d], "enc_final", "dec_final" [d], "enc_rel", "dec_rel" [buckets][H],
+     "enc": [{wq, wk, wv, wo, attn_norm, wi0, wi1, wff, ffn_norm}], "dec": [{... + cq, ck, cv, co,
+     self_norm, cross_norm}], "in_norm", "in_w1", "in_w2" (IN_MLP2)}.
+    Query projections (wq, cq) are drawn with std weight_std / sqrt(head_dim): T5 computes attention
+    logits without a 1/sqrt(head_dim) factor and folds it into the query projection's scale instead.
+    """
+    sh = w.shape
+    d, V, std = sh.d_model, sh.vocab, w.weight_std
+    sd = w.weight_seed
+
+    def gain(kind, layer, n):
+        if w.norm_gain == "ones":
+            return np.full(n, 0x3F80, dtype=np.uint16)
+        return normal_bf16(sd, t5_stream_id(kind, layer), (n,), mean=1.0, std=0.1)
+
+    def block(layer, decoder):
+        lw = {}
+        for name, shp in t5_layer_shapes(sh, decoder).items():
+            if name.endswith("norm"):
+                lw[name] = gain(name, layer, shp[0])
+            else:
+                s = std / np.sqrt(sh.head_dim) if name in ("wq", "cq") else std
+                lw[name] = normal_bf16(sd, t5_stream_id(name, layer), shp, std=s)
+        return lw
+
+    out = {
+        "embed": normal_bf16(sd, t5_stream_id("t5_embed"), (V, d), std=w.embed_std),
+        "lm_head": normal_bf16(sd, t5_stream_id("t5_lm_head"), (V, d), std=std),
+        "enc_final": gain("enc_final", 0, d),
+        "dec_final": gain("dec_final", 0, d),
+        "enc_rel": normal_bf16(sd, t5_stream_id("enc_rel"), (sh.rel_buckets, sh.n_heads), std=w.rel_std),
+        "dec_rel": normal_bf16(sd, t5_stream_id("dec_rel"), (sh.rel_buckets, sh.n_heads), std=w.rel_std),
+        "enc": [block(l, False) for l in range(sh.n_enc)],
+        "dec": [block(_T5_DEC + l, True) for l in range(sh.n_dec)],
+    }
+    if w.in_kind == IN_MLP2:
+        out["in_norm"] = gain("in_norm", 0, d)
+        out["in_w1"] = normal_bf16(sd, t5_stream_id("in_w1"), (w.in_hidden, d), std=std)
+        out["in_w2"] = normal_bf16(sd, t5_stream_id("in_w2"), (d, w.in_hidden), std=std)
+    elif w.in_kind != IN_IDENTITY:
+        raise ValueError("encoder-decoder workloads take IN_IDENTITY or IN_MLP2")
+    return out
+
+
+def make_t5_inputs(w: T5Workload, seed: int | None = None) -> tuple[np.ndarray, np.ndarray]:
+    """Synthetic query embeddings (bf16 bits [n_query][d], N(0, vis_std)) and prompt ids U[0, V)."""
+    seed = w.input_seed if seed is None else seed
+    q = normal_bf16(seed, t5_stream_id("query"), (w.n_query, w.shape.d_model), std=w.vis_std)
+    prompt = uniform_i32(seed, t5_stream_id("t5_prompt"), (w.n_prompt,), 0, w.shape.vocab)
+    return q, prompt
