@@ -297,6 +297,101 @@ def run_in_block(args) -> None:
                       "per_s": rows}), flush=True)
 
 
+def run_encdec(args) -> None:
+    """The BLIP-2 FlanT5-xl-shaped encoder-decoder workload (24 + 24 layers, d = 2048, 32 x 64 heads,
+    gated-GELU 5120, V = 32128; 32 query embeddings + 16 prompt ids; draft = decoder layers 0-5 + the
+    imitation network; gamma = 4; 30 new tokens): decode tokens/s of SSD and of greedy decoding with
+    the same kernels, speedup, accept length, the drafting stage's and the greedy decoder's HBM GB/s
+    (of measured), and the encoder prefill time, per s.  One JSON line."""
+    import torch
+
+    import paper_2510_22641_gb300 as lib
+    lib.build()
+    w = synth.FLANT5XL
+    sh = w.shape
+    bits = synth.make_t5_weights(w)
+    up = lib.bf16_bits_to_device
+    ren = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
+           "ffn_norm": "ffn_norm"}
+
+    def stack(lw, norm):
+        d = {ren[n]: up(a) for n, a in lw.items() if n in ren}
+        d["attn_norm"] = up(lw[norm])
+        return d
+
+    dev = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
+           "layers": [stack(lw, "self_norm") for lw in bits["dec"]],
+           "in_norm": up(bits["in_norm"]), "in_w1": up(bits["in_w1"]), "in_w2": up(bits["in_w2"]),
+           "encdec": {"cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
+                      "enc": [stack(lw, "attn_norm") for lw in bits["enc"]], "enc_final": up(bits["enc_final"]),
+                      "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}}
+    q, prompt = synth.make_t5_inputs(w)
+    v = up(q)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    stream = torch.cuda.current_stream()
+    rs = torch.tensor(w.dec_scale(), device="cuda")
+    ins = torch.tensor([w.in_scale()], device="cuda")
+    cfg = lib.t5_config_dict(sh, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                             w.max_new + lib.SSD_MAX_GAMMA + 2, w.enc_len, w.eos_id)
+    model = lib.SSDModel(cfg, dev, rs, ins)
+    # algorithmic bytes per decode row: a decoder layer's weights (self q/k/v/o, cross q/o, MLP, norms)
+    # plus the cross-attention K/V it reads (fp32); the imitation network; the LM head
+    layer = sh.dec_layer_bytes_bf16() + 2 * sh.n_heads * w.enc_len * sh.head_dim * 4
+    in_bytes = 2 * 2 * w.in_hidden * sh.d_model + 2 * sh.d_model
+    head = 2 * sh.vocab * sh.d_model + 2 * sh.d_model
+    draft_bytes = w.draft_exit_k * layer + in_bytes + head
+    greedy_bytes = sh.n_dec * layer + head
+    try:
+        peak = float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["hbm_gbs"])
+    except (OSError, KeyError, ValueError):
+        peak = None
+
+    def ev_ms(fn):
+        torch.cuda.synchronize()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b)
+
+    def timed(fn):
+        model.prefill(v, p)
+        fn()
+        model.prefill(v, p)
+        return ev_ms(fn)
+
+    model.prefill(v, p)
+    prefill_ms = min(ev_ms(lambda: model.prefill(v, p)) for _ in range(3))
+    rows = []
+    for s_val in S_VALUES:
+        ws = w.replace(s=s_val)
+        rs.copy_(torch.tensor(ws.dec_scale(), device="cuda"))
+        ins.copy_(torch.tensor([ws.in_scale()], device="cuda"))
+        g_ms = min(timed(lambda: model.greedy_decode(w.max_new)) for _ in range(3))
+        s_ms = min(timed(lambda: model.decode(w.max_new, w.gamma)) for _ in range(3))
+        st = model.stats()
+        model.prefill(v, p)
+        model.draft(w.gamma)
+        model.verify(w.gamma)
+        d_ms = ev_ms(lambda: model.draft(w.gamma))
+        g_gbs = (w.max_new - 1) * greedy_bytes / (g_ms / 1e3) / 1e9
+        d_gbs = w.gamma * draft_bytes / (d_ms / 1e3) / 1e9
+        rows.append({"s": s_val, "ssd_decode_tok_s": (w.max_new - 1) / (s_ms / 1e3),
+                     "greedy_decode_tok_s": (w.max_new - 1) / (g_ms / 1e3), "speedup": g_ms / s_ms,
+                     "mean_accept": st["accepted"] / max(st["steps"], 1), "steps": st["steps"],
+                     "draft_ms": d_ms, "draft_gbs": d_gbs, "greedy_gbs": g_gbs,
+                     "draft_frac": d_gbs / peak if peak else None, "greedy_frac": g_gbs / peak if peak else None})
+    model.close()
+    print(json.dumps({"workload": f"{w.name}: {sh.n_enc}+{sh.n_dec} layers, d={sh.d_model}, {sh.n_heads}x"
+                                  f"{sh.head_dim} heads, gated-GELU {sh.d_ff}, V={sh.vocab}; {w.n_query} queries + "
+                                  f"{w.n_prompt} prompt ids; k={w.draft_exit_k}, gamma={w.gamma}, "
+                                  f"{w.max_new} new tokens; bs1",
+                      "prefill_ms": prefill_ms, "peak_hbm_gbs": peak, "bytes_per_token":
+                          {"draft": draft_bytes, "greedy": greedy_bytes}, "per_s": rows}), flush=True)
+
+
 def run_sweep(args) -> None:
     """Sweep k x gamma x s on the 7B shape (256 new tokens): accept length, tokens/s, speedup
     over greedy, draft and verify HBM GB/s.  One JSON line per point."""
@@ -392,7 +487,12 @@ def main() -> None:
     ap.add_argument("--sweep", action="store_true", help="k x gamma x s sweep (one JSON line per point)")
     ap.add_argument("--in-block", action="store_true",
                     help="the 7B workload with the imitation module as one decoder block (one JSON line)")
+    ap.add_argument("--encdec", action="store_true",
+                    help="the BLIP-2 FlanT5-xl-shaped encoder-decoder workload (one JSON line)")
     args = ap.parse_args()
+    if args.encdec:
+        run_encdec(args)
+        return
     if args.sweep:
         run_sweep(args)
         return

@@ -53,7 +53,7 @@ typedef enum {
   SSD_ERR_INVALID_ARG = 1,  /* null pointer, bad size, unsupported shape */
   SSD_ERR_OOM = 2,          /* a device allocation failed */
   SSD_ERR_CUDA = 3,         /* a CUDA runtime call failed */
-  SSD_ERR_CAPACITY = 4,     /* n_vis + n_prompt + max_new + gamma + 1 > max_seq */
+  SSD_ERR_CAPACITY = 4,     /* n_vis + n_prompt + max_new + gamma + 1 > max_seq (T5: encoder rows > max_enc) */
   SSD_ERR_STATE = 5,        /* call out of order (e.g. verify without a draft) */
   SSD_ERR_TIMEOUT = 6,      /* a bounded device wait ran out */
   SSD_ERR_DEVICE = 7,       /* the kernels flagged bad input (e.g. token id >= vocab) */
@@ -68,13 +68,25 @@ enum {
                          * writes scaled by s_in (the module read as a block; Sec. "Choice of n") */
 };
 
+/* Model families. */
+enum {
+  SSD_ARCH_LLAMA = 0,  /* decoder-only pre-norm LLaMA stack (LLaVA-1.5): RMSNorm, rotary attention, SwiGLU */
+  SSD_ARCH_T5 = 1      /* encoder-decoder T5 v1.1 stack (BLIP-2 FlanT5-xl, Sec. "Experiments"): the encoder reads
+                        * [vis_emb; embed(prompt)] once; the decoder, which drafts and verifies, starts
+                        * from start_token at position 0 and has, per layer, self-attention with a
+                        * learned relative-position bias and no 1/sqrt(head_dim) factor, cross-attention
+                        * to the encoder's normed output, and a gated-GELU (tanh form) MLP; no RoPE */
+};
+
 #define SSD_MAX_GAMMA 8
 #define SSD_MAX_ROWS 16   /* rows one decode pass may carry (gamma + 1, prefill chunk) */
 
 typedef struct ssd_ctx ssd_ctx;
 
 /* Model shape and decoding limits.  The decoder is a pre-norm LLaMA block stack
- * (RMSNorm, rotary multi-head attention, SwiGLU MLP). */
+ * (RMSNorm, rotary multi-head attention, SwiGLU MLP), or with arch = SSD_ARCH_T5
+ * the decoder of a T5 v1.1 encoder-decoder.  Fields after eos_id are read only
+ * for SSD_ARCH_T5 (zero them otherwise). */
 typedef struct {
   int n_layers;      /* L */
   int d_model;       /* hidden width */
@@ -90,7 +102,40 @@ typedef struct {
   float rms_eps;     /* RMSNorm epsilon */
   float rope_theta;  /* rotary base, rotate-half pairing (i, i + head_dim/2) */
   int eos_id;        /* end-of-sequence token, -1 = disabled */
+  int arch;          /* SSD_ARCH_* (0 = LLaMA) */
+  int n_enc_layers;  /* T5: encoder depth */
+  int max_enc;       /* T5: encoder rows capacity, >= n_vis + n_prompt of every prefill */
+  int rel_buckets;   /* T5: relative-position buckets (even, >= 4) */
+  int rel_max_distance; /* T5: offsets at or beyond this share the last bucket */
+  int start_token;   /* T5: the decoder's first input id */
 } ssd_config;
+
+/* Extra weights of SSD_ARCH_T5, device bf16, [out][in], borrowed.  The
+ * ssd_weights layer arrays hold the DECODER: wq/wk/wv/wo its self-attention,
+ * w_gate/w_up/w_down the gated-GELU MLP (wi_0, wi_1, wo), attn_norm the
+ * self-attention norm, ffn_norm the MLP norm, final_norm the decoder's final
+ * norm; resid_scale[l] scales all three residual writes of decoder layer l. */
+typedef struct {
+  /* host arrays of n_layers device pointers: cross-attention of decoder layer l */
+  const void* const* cq;          /* [n_heads*head_dim][d_model], applied to RMSNorm_cross(x) */
+  const void* const* ck;          /* [n_heads*head_dim][d_model], applied to the encoder output */
+  const void* const* cv;          /* [n_heads*head_dim][d_model] */
+  const void* const* co;          /* [d_model][n_heads*head_dim] */
+  const void* const* cross_norm;  /* [d_model] */
+  /* host arrays of n_enc_layers device pointers: the encoder (bidirectional attention) */
+  const void* const* enc_wq;
+  const void* const* enc_wk;
+  const void* const* enc_wv;
+  const void* const* enc_wo;
+  const void* const* enc_wi0;     /* [d_ff][d_model] gate */
+  const void* const* enc_wi1;     /* [d_ff][d_model] up */
+  const void* const* enc_wff;     /* [d_model][d_ff] */
+  const void* const* enc_attn_norm;
+  const void* const* enc_ffn_norm;
+  const void* enc_final;          /* [d_model] the encoder's final norm */
+  const void* enc_rel;            /* [rel_buckets][n_heads] encoder bias (bidirectional buckets) */
+  const void* dec_rel;            /* [rel_buckets][n_heads] decoder self-attention bias (past-only buckets) */
+} ssd_encdec_weights;
 
 /* Model weights, all device pointers, bf16, nn.Linear layout [out][in], borrowed. */
 typedef struct {
@@ -121,6 +166,8 @@ typedef struct {
    * fills the prompt rows, each drafting step its row, the verification pass
    * row gamma. */
   const void* const* in_block;
+  /* SSD_ARCH_T5: the encoder and cross-attention weights; NULL otherwise. */
+  const ssd_encdec_weights* encdec;
 } ssd_weights;
 
 /* Counters of the last prefill+decode, read back by ssd_get_stats. */
@@ -146,6 +193,11 @@ SSD_API ssd_status ssd_destroy(ssd_ctx* ctx);
  * [vis_emb (n_vis rows); embed(prompt)] at positions 0..P-1, P = n_vis + n_prompt,
  * run through all L layers; K/V of every layer for positions 0..P-1 are
  * written; the greedy token of the last row is written to first_tok.
+ * SSD_ARCH_T5: the P rows are the ENCODER's input (P <= max_enc); the encoder
+ * runs, every decoder layer's cross-attention K/V of its output are written,
+ * and the decoder runs once on start_token at position 0, whose greedy token
+ * is the first new token (kv_len = 1 afterwards; decoder positions count from
+ * 0, so the capacity rule below reads 1 + max_new + gamma + 1 <= max_seq).
  *   vis_emb:   device bf16 [n_vis][d_model] (may be NULL when n_vis == 0)
  *   prompt:    device int32 [n_prompt], each in [0, vocab)
  *   first_tok: device int32 [1] (may be NULL)

@@ -1,5 +1,5 @@
 """Plain fp64 CPU oracle for greedy self-speculative decoding on an encoder-decoder VLM
-(the paper's BLIP-2 + FlanT5-xl setting; FastVLM, arXiv 2510.22641).
+(the BLIP-2 + FlanT5-xl setting of Sec. "Experiments"; FastVLM, arXiv 2510.22641).
 
 TEST INFRASTRUCTURE ONLY.  Only ``tests/`` (and, later, ``bench.py``'s CPU baseline) may
 import or run this module.  It shares no code with any CUDA path; its inputs come from
@@ -105,7 +105,10 @@ def rel_bucket(delta: int, bidirectional: bool, n_buckets: int, max_distance: in
     keys after it.  Past-only: every bucket is for keys at or before the query (later keys share
     bucket 0; the decoder masks them anyway).  Within a half, offsets below n/2 get one bucket
     each and larger offsets share logarithmically spaced buckets up to max_distance, beyond which
-    they share the last one.  The logarithm is evaluated in fp64 and truncated.
+    they share the last one.  The logarithmic index is evaluated in fp64 and floored after adding
+    1e-9: at exact powers (offset 16 of the bidirectional half, for one) the exact index is an integer
+    that fp64 rounding could otherwise put one bucket short, and the guard makes the decision
+    independent of the platform's log.
     """
     n = n_buckets
     base = 0
@@ -119,7 +122,7 @@ def rel_bucket(delta: int, bidirectional: bool, n_buckets: int, max_distance: in
     exact = n // 2
     if dist < exact:
         return base + dist
-    far = exact + int(math.log(dist / exact) / math.log(max_distance / exact) * (n - exact))
+    far = exact + int(math.log(dist / exact) / math.log(max_distance / exact) * (n - exact) + 1e-9)
     return base + min(far, n - 1)
 
 
@@ -252,15 +255,16 @@ def greedy_generate(m: T5Model, z: np.ndarray, prompt, max_new: int) -> T5Result
 
 
 def ssd_generate(m: T5Model, z: np.ndarray, prompt, max_new: int, gamma: int,
-                 reuse_draft_rows: bool = True) -> T5Result:
-    """Algorithm 1 on the decoder (see the module docstring); kv_len counts decoder positions."""
+                 reuse_draft_rows: bool = True, max_steps: int | None = None) -> T5Result:
+    """Algorithm 1 on the decoder (see the module docstring); kv_len counts decoder positions.
+    max_steps: stop after that many draft + verify steps (a sampled prefix of a long run)."""
     c = m.cfg
     k, L = c.draft_exit_k, c.n_dec
     cache, o = _first(m, z, prompt, max_new + gamma + 1)
     y = argmax_lowest(o)
     res = T5Result(tokens=[y], logits=[o], kv_len=1)
     p, done = 1, (c.eos_id >= 0 and y == c.eos_id)
-    while len(res.tokens) < max_new and not done:
+    while len(res.tokens) < max_new and not done and (max_steps is None or len(res.accept_lengths) < max_steps):
         g_eff = min(gamma, max_new - len(res.tokens) - 1)
         toks, xk = [y], []
         for j in range(g_eff):                                   # drafting stage

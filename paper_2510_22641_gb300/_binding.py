@@ -17,6 +17,8 @@ SSD_MAX_ROWS = 16
 SSD_IN_IDENTITY = 0
 SSD_IN_MLP2 = 1
 SSD_IN_BLOCK = 2
+SSD_ARCH_LLAMA = 0
+SSD_ARCH_T5 = 1
 
 STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_CUDA", 4: "SSD_ERR_CAPACITY",
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
@@ -34,10 +36,20 @@ class SSDConfig(ctypes.Structure):
                 ("head_dim", ctypes.c_int), ("d_ff", ctypes.c_int), ("vocab", ctypes.c_int),
                 ("draft_exit_k", ctypes.c_int), ("in_kind", ctypes.c_int), ("in_hidden", ctypes.c_int),
                 ("gamma_max", ctypes.c_int), ("max_seq", ctypes.c_int), ("rms_eps", ctypes.c_float),
-                ("rope_theta", ctypes.c_float), ("eos_id", ctypes.c_int)]
+                ("rope_theta", ctypes.c_float), ("eos_id", ctypes.c_int), ("arch", ctypes.c_int),
+                ("n_enc_layers", ctypes.c_int), ("max_enc", ctypes.c_int), ("rel_buckets", ctypes.c_int),
+                ("rel_max_distance", ctypes.c_int), ("start_token", ctypes.c_int)]
 
 
 _PP = ctypes.POINTER(ctypes.c_void_p)
+
+ENCDEC_ARRAYS = ("cq", "ck", "cv", "co", "cross_norm", "enc_wq", "enc_wk", "enc_wv", "enc_wo", "enc_wi0", "enc_wi1",
+                 "enc_wff", "enc_attn_norm", "enc_ffn_norm")
+
+
+class SSDEncDecWeights(ctypes.Structure):
+    _fields_ = [(n, _PP) for n in ENCDEC_ARRAYS] + [("enc_final", ctypes.c_void_p), ("enc_rel", ctypes.c_void_p),
+                                                    ("dec_rel", ctypes.c_void_p)]
 
 
 class SSDWeights(ctypes.Structure):
@@ -45,7 +57,8 @@ class SSDWeights(ctypes.Structure):
                 ("wq", _PP), ("wk", _PP), ("wv", _PP), ("wo", _PP), ("w_gate", _PP), ("w_up", _PP),
                 ("w_down", _PP), ("attn_norm", _PP), ("ffn_norm", _PP),
                 ("in_norm", ctypes.c_void_p), ("in_w1", ctypes.c_void_p), ("in_w2", ctypes.c_void_p),
-                ("resid_scale", ctypes.c_void_p), ("in_scale", ctypes.c_void_p), ("in_block", _PP)]
+                ("resid_scale", ctypes.c_void_p), ("in_scale", ctypes.c_void_p), ("in_block", _PP),
+                ("encdec", ctypes.POINTER(SSDEncDecWeights))]
 
 
 class SSDStats(ctypes.Structure):

@@ -57,6 +57,13 @@ struct AttnParams {
   // grid complete, 2 first chunk landed, 3 last chunk folded, 4 state stored and ticket taken,
   // 5 merge done (the head's last CTA), 6 exit, 7 chunks taken.  Null when not tracing.
   unsigned long long* trace;
+  // Non-causal key sets and relative-position bias (encoder-decoder models; read only by the EXT
+  // instantiations, so the causal kernels compile without them):
+  int fixed_keys;     // 1: keys 0 .. st->enc_len - 1, every one visible to every row (cross-attention,
+                      // bidirectional encoder self-attention); 0: causal over the cache (above)
+  int abs_pos;        // row m sits at position pos_off + m (st->kv_len ignored): the encoder's rows
+  const float* bias;  // null, or [n_heads][bias_stride]: score(row at i, key j) += bias[h][j - i + bias_zero]
+  int bias_stride, bias_zero;
 };
 
 template <int DH>
@@ -88,7 +95,7 @@ struct AttnSmem {
   static constexpr int kTotal = kBar + (kAttnBufs + 1) * 8;
 };
 
-template <int M, int DH>
+template <int M, int DH, bool EXT>
 __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams p) {
   using S = AttnSmem<M, DH>;
   using G = AttnGeo<DH>;
@@ -121,9 +128,15 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
   int base = 0, n_keys = 0, my_chunks = 0;
   bool bad = false;
   auto geometry = [&]() {
-    base = __ldcg(&p.st->kv_len) + p.pos_off;
-    bad = base < 0 || base + M > p.max_seq;
-    n_keys = bad ? 0 : base + M;  // keys 0 .. base+M-1 exist for the last row
+    base = ((EXT && p.abs_pos) ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
+    if (EXT && p.fixed_keys) {
+      const int ne = __ldcg(&p.st->enc_len);
+      bad = base < 0 || ne < 1 || ne > p.max_seq;
+      n_keys = bad ? 0 : ne;
+    } else {
+      bad = base < 0 || base + M > p.max_seq;
+      n_keys = bad ? 0 : base + M;  // keys 0 .. base+M-1 exist for the last row
+    }
     const int n_chunks = (n_keys + KPC - 1) / KPC;
     my_chunks = n_chunks > rank ? (n_chunks - rank + kAttnSplit - 1) / kAttnSplit : 0;
   };
@@ -142,7 +155,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
     if (tid == 0)
       for (; issued < kAttnBufs && issued < my_chunks; ++issued) {
         const int c = rank + issued * kAttnSplit;
-        if ((c + 1) * KPC > base) break;  // holds keys the upstream grid writes
+        if ((EXT && p.fixed_keys) || (c + 1) * KPC > base) break;  // holds keys the upstream grid writes
         issue(issued, c);
       }
   }
@@ -229,8 +242,16 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
 #pragma unroll
         for (int i = 0; i < kAttnBufs; ++i) {
           if (i >= gn) break;
-          const bool vis = jw < nkc[i] && j0c[i] + jw <= base + m;
-          ss[m * GK + i * KPC + jw] = vis ? a[m][i] * p.scale : -INFINITY;
+          const int j = j0c[i] + jw;
+          const bool vis = jw < nkc[i] && ((EXT && p.fixed_keys) || j <= base + m);
+          float sv = a[m][i] * p.scale;
+          if constexpr (EXT) {
+            if (vis && p.bias) {
+              const int bi = min(max(j - (base + m) + p.bias_zero, 0), p.bias_stride - 1);
+              sv += __ldg(p.bias + static_cast<size_t>(h) * p.bias_stride + bi);
+            }
+          }
+          ss[m * GK + i * KPC + jw] = vis ? sv : -INFINITY;
         }
     }
     __syncthreads();

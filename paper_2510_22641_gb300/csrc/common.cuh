@@ -34,7 +34,8 @@ struct DevState {
   int last_n;      // tokens emitted by the last accept
   int eos_id;
   int dyn_launches;  // kernel launches of the running dynamic-length decode's steps
-  int pad[2];
+  int enc_len;     // encoder rows = cross-attention keys (encoder-decoder model), else 0
+  int pad1;
   int hist[SSD_MAX_GAMMA + 1];   // steps per accepted length a
   int tok_in[kMaxRows];          // verify rows t_0 = y, t_j = d_j
   int full_tok[kMaxRows];        // f_i = full-model argmax of row i
@@ -153,6 +154,10 @@ __device__ __forceinline__ float2 bf16x2_to_float2(uint32_t w) {
 }
 
 __device__ __forceinline__ float silu_f(float v) { return v / (1.0f + expf(-v)); }
+// GELU in its tanh form, 0.5 v (1 + tanh(sqrt(2/pi) (v + 0.044715 v^3))) (the gated-GELU MLP of T5 v1.1).
+__device__ __forceinline__ float gelu_tanh_f(float v) {
+  return 0.5f * v * (1.0f + tanhf(0.7978845608028654f * (v + 0.044715f * v * v * v)));
+}
 
 // Total order on floats as unsigned keys (larger float -> larger key).
 __device__ __forceinline__ uint32_t orderable(float f) {

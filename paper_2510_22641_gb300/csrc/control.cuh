@@ -59,12 +59,15 @@ __global__ void prefill_rows_kernel(const __nv_bfloat16* __restrict__ vis, const
   }
 }
 
-__global__ void prefill_begin_kernel(DevState* st, int P, int eos_id) {
+// P: decoder rows of the prompt (the position of the first new token + 1); enc_len: encoder rows
+// (encoder-decoder model; 0 otherwise).
+__global__ void prefill_begin_kernel(DevState* st, int P, int eos_id, int enc_len) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
   st->kv_len = 0;
   st->prompt_len = P;
+  st->enc_len = enc_len;
   st->n_out = 0;
   st->done = 0;
   st->error = 0;
@@ -233,6 +236,16 @@ __global__ void rope_table_kernel(float2* cs, int max_seq, int head_dim, double 
   double s, c;
   sincos(ang, &s, &c);
   cs[idx] = make_float2(static_cast<float>(c), static_cast<float>(s));
+}
+
+// Relative-position bias table out[h][j] = rel[bucket[j]][h] (rel: the learned [buckets][n_heads]
+// bf16 table of a T5-style stack; bucket[j]: the bucket of offset j - zero, decided on the host).
+__global__ void bias_table_kernel(const __nv_bfloat16* __restrict__ rel, const int* __restrict__ bucket, int n,
+                                  int n_heads, float* out) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n * n_heads) return;
+  const int h = i / n, j = i - h * n;
+  out[i] = __bfloat162float(rel[static_cast<size_t>(bucket[j]) * n_heads + h]);
 }
 
 }  // namespace ssd

@@ -170,6 +170,20 @@ struct ssd_ctx {
   std::string gemv_trace_path;  // SSD_GEMV_TRACE=<file>: per-CTA timeline of ssd_profile_projection's last launch (GEMV or attention)
   std::string fwd_trace_path;
   int fwd_trace_phases = 0;
+  // encoder-decoder model (SSD_ARCH_T5)
+  bool t5 = false;
+  int max_enc = 0;
+  std::vector<LayerSites> enc_layers;
+  std::vector<const __nv_bfloat16*> enc_attn_norm, enc_ffn_norm, cross_norm;
+  const __nv_bfloat16* enc_final = nullptr;
+  std::vector<Site> cross_q, cross_o, cross_kv;      // per decoder layer: cq, co, [ck; cv]
+  float *x_enc = nullptr, *enc_q = nullptr, *enc_o = nullptr;  // encoder rows [max_enc][dp or qp]
+  float *enc_k = nullptr, *enc_v = nullptr;          // one encoder layer's K/V [H][max_enc][Dh]
+  float *ckc = nullptr, *cvc = nullptr;              // cross-attention K/V [L][H][max_enc][Dh]
+  size_t cross_layer_kv = 0;
+  float *dec_bias = nullptr, *enc_bias = nullptr;    // [H][max_seq] and [H][2 max_enc - 1]
+  float* one = nullptr;                              // device 1.0f: the encoder's residual scale
+  int* start_tok = nullptr;                          // device copy of cfg.start_token
   // debug logits capture
   float* logits_buf = nullptr;
   int logits_rows = 0;
@@ -300,21 +314,32 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   return SSD_OK;
 }
 
+// EXT: fixed key sets / absolute positions / relative-position bias (the encoder-decoder model).
 template <int M>
 static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a) {
   const dim3 grid(kAttnSplit, c->cfg.n_heads);
+  const bool ext = a.fixed_keys || a.abs_pos || a.bias;
   if (c->cfg.head_dim == 128)
-    return launch_k(c, attn_kernel<M, 128>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
-  return launch_k(c, attn_kernel<M, 64>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
+    return ext ? launch_k(c, attn_kernel<M, 128, true>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a)
+               : launch_k(c, attn_kernel<M, 128, false>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
+  return ext ? launch_k(c, attn_kernel<M, 64, true>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a)
+             : launch_k(c, attn_kernel<M, 64, false>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
+}
+
+template <int M, int DH>
+static cudaError_t attn_attr_md() {
+  cudaError_t e = cudaFuncSetAttribute(attn_kernel<M, DH, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       AttnSmem<M, DH>::kTotal);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(attn_kernel<M, DH, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              AttnSmem<M, DH>::kTotal);
 }
 
 template <int M>
 static cudaError_t attn_attr_m() {
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<M, 128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       AttnSmem<M, 128>::kTotal);
+  cudaError_t e = attn_attr_md<M, 128>();
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_kernel<M, 64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              AttnSmem<M, 64>::kTotal);
+  return attn_attr_md<M, 64>();
 }
 
 static cudaError_t attn_attrs() {
@@ -330,25 +355,12 @@ static cudaError_t attn_attrs() {
   return attn_attr_m<9>();
 }
 
-// prefetch_old: the launch before is the layer's QKV projection with a late trigger.
-static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch_old,
-                            unsigned long long* trace = nullptr) {
-  AttnParams a{};
-  a.trace = trace;
-  a.prefetch_old = prefetch_old ? 1 : 0;
+// One split-KV attention launch over M query rows (the ctx's scratch, state and head count filled in).
+static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a) {
   a.part = c->attn_part;
   a.tickets = c->attn_tickets;
-  a.q = c->qb;
-  a.q_stride = c->qp;
-  a.k_cache = c->kc + l * c->layer_kv;
-  a.v_cache = c->vc + l * c->layer_kv;
-  a.o = c->ob;
-  a.o_stride = c->qp;
   a.st = c->st;
-  a.pos_off = pos_off;
   a.n_heads = c->cfg.n_heads;
-  a.max_seq = c->cfg.max_seq;
-  a.scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
   cudaError_t r;
   switch (M) {
     case 1: r = attn_launch_m<1>(c, a); break;
@@ -364,6 +376,45 @@ static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch
   }
   CK(r);
   return SSD_OK;
+}
+
+// Causal self-attention of layer l over the KV cache for the M rows at kv_len + pos_off + m.  The
+// encoder-decoder model's decoder adds its relative-position bias and has no 1/sqrt(head_dim) factor.
+// prefetch_old: the launch before is the layer's QKV projection with a late trigger.
+static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch_old,
+                            unsigned long long* trace = nullptr) {
+  AttnParams a{};
+  a.trace = trace;
+  a.prefetch_old = prefetch_old ? 1 : 0;
+  a.q = c->qb;
+  a.q_stride = c->qp;
+  a.k_cache = c->kc + l * c->layer_kv;
+  a.v_cache = c->vc + l * c->layer_kv;
+  a.o = c->ob;
+  a.o_stride = c->qp;
+  a.pos_off = pos_off;
+  a.max_seq = c->cfg.max_seq;
+  a.scale = c->t5 ? 1.0f : 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
+  if (c->t5) {
+    a.bias = c->dec_bias;
+    a.bias_stride = c->cfg.max_seq;
+    a.bias_zero = c->cfg.max_seq - 1;
+  }
+  return attn_run(c, M, a);
+}
+
+// x = x + (*scale) * W in, on M rows (x: activation rows of stride dp).
+static ssd_status resid_gemv(ssd_ctx* c, int M, const Site& s, const float* in, int in_stride, float* x,
+                             const float* scale) {
+  GemvParams p{};
+  p.x = in;
+  p.x_stride = in_stride;
+  p.base = x;
+  p.base_stride = c->dp;
+  p.dst = x;
+  p.dst_stride = c->dp;
+  p.scale = scale;
+  return gemv(c, Epi::RESID, M, s, p);
 }
 
 // One decoder layer x_{l+1} = x_l + f_l(x_l) on rows row0 .. row0+M-1 of xv at
@@ -397,8 +448,65 @@ static ssd_status enqueue_layer(ssd_ctx* c, int l, int row0, int M, int pos_off)
   return enqueue_layer_x(c, l, c->xv + static_cast<size_t>(row0) * c->dp, M, pos_off);
 }
 
+// Decoder layer l of the encoder-decoder model on M rows x (positions kv_len + pos_off + m), in place:
+//   x += s_l W_o Attn(RMSNorm_self(x))       causal, relative-position bias, no 1/sqrt(head_dim), no RoPE
+//   x += s_l W_co CrossAttn(RMSNorm_cross(x))  over the encoder output's K/V (all st->enc_len keys)
+//   x += s_l W_ff (GELU_tanh(W_i0 u) * W_i1 u), u = RMSNorm_ffn(x)
+static ssd_status enqueue_t5_layer(ssd_ctx* c, int l, float* x, int M, int pos_off) {
+  const int d = c->dp;
+  const float* s_l = c->resid_scale + l;
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = d;
+  p.gain = c->attn_norm[l];
+  p.pos_off = pos_off;
+  p.q_out = c->qb;
+  p.q_stride = c->qp;
+  p.k_cache = c->kc + l * c->layer_kv;
+  p.v_cache = c->vc + l * c->layer_kv;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  p.late_trigger = 1;
+  CKS(gemv(c, Epi::QKV, M, c->layers[l].qkv, p));
+  CKS(attention(c, l, M, pos_off, true));
+  CKS(resid_gemv(c, M, c->layers[l].o, c->ob, c->qp, x, s_l));
+  p = GemvParams{};
+  p.x = x;
+  p.x_stride = d;
+  p.gain = c->cross_norm[l];
+  p.pos_off = pos_off;
+  p.q_out = c->qb;
+  p.q_stride = c->qp;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  CKS(gemv(c, Epi::QKV, M, c->cross_q[l], p));  // a one-matrix site: q only
+  AttnParams a{};
+  a.q = c->qb;
+  a.q_stride = c->qp;
+  a.k_cache = c->ckc + l * c->cross_layer_kv;
+  a.v_cache = c->cvc + l * c->cross_layer_kv;
+  a.o = c->ob;
+  a.o_stride = c->qp;
+  a.pos_off = pos_off;
+  a.max_seq = c->max_enc;
+  a.scale = 1.0f;
+  a.fixed_keys = 1;
+  CKS(attn_run(c, M, a));
+  CKS(resid_gemv(c, M, c->cross_o[l], c->ob, c->qp, x, s_l));
+  p = GemvParams{};
+  p.x = x;
+  p.x_stride = d;
+  p.gain = c->ffn_norm[l];
+  p.h_out = c->hb;
+  p.h_stride = c->fp;
+  p.act = 1;
+  CKS(gemv(c, Epi::GATE_SILU, M, c->layers[l].gateup, p));
+  return resid_gemv(c, M, c->layers[l].down, c->hb, c->fp, x, s_l);
+}
+
 // Block l (a decoder layer, or the IN_BLOCK block for l == n_layers) on M rows x, in place.
 static ssd_status enqueue_layer_x(ssd_ctx* c, int l, float* x, int M, int pos_off) {
+  if (c->t5) return enqueue_t5_layer(c, l, x, M, pos_off);
   const int d = c->dp;
   GemvParams p{};
   p.x = x;
@@ -814,6 +922,7 @@ static ssd_status fwd_ensure(ssd_ctx* c) {
   if (!c->use_fwd || c->fwd_ready) return SSD_OK;
   if (c->cfg.in_kind == SSD_IN_BLOCK)
     return fail(c, SSD_ERR_UNSUPPORTED, "the persistent forward kernel has no imitation-block program");
+  if (c->t5) return fail(c, SSD_ERR_UNSUPPORTED, "the persistent forward kernel has no encoder-decoder program");
   return fwd_build_programs(c);
 }
 
@@ -905,7 +1014,7 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
   CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
-  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
+  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
   int r0 = 0;
   for (; r0 < P; r0 += kPrefillChunk) {
     const int Mc = P - r0 < kPrefillChunk ? P - r0 : kPrefillChunk;
@@ -922,6 +1031,96 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   r0 -= kPrefillChunk;
   CKS(enqueue_head(c, c->xv + static_cast<size_t>(P - 1 - r0) * d, 1, P - 1, full_tok, true));
   CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
+  return SSD_OK;
+}
+
+// Prefill of the encoder-decoder model (Sec. "SSD Setup for VLMs" with the BLIP-2 FlanT5 language
+// model): the encoder over the P rows [z; embed(prompt)] in chunks of kPrefillChunk rows through the
+// decode kernels (bidirectional attention: every row sees all P keys, with the encoder's
+// relative-position bias), the cross-attention K/V of every decoder layer from the encoder's normed
+// output, then the decoder on start_token at position 0, whose greedy token is the first new token.
+static ssd_status enqueue_prefill_t5(ssd_ctx* c, int n_vis, int n_prompt) {
+  const int P = n_vis + n_prompt, dp = c->dp, qp = c->qp;
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
+  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 1, c->cfg.eos_id, P));
+  CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+              static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_enc, dp, c->cfg.d_model,
+              c->st));
+  for (int e = 0; e < c->cfg.n_enc_layers; ++e) {
+    const LayerSites& S = c->enc_layers[e];
+    for (int r0 = 0; r0 < P; r0 += kPrefillChunk) {
+      const int Mc = std::min(kPrefillChunk, P - r0);
+      GemvParams p{};
+      p.x = c->x_enc + static_cast<size_t>(r0) * dp;
+      p.x_stride = dp;
+      p.gain = c->enc_attn_norm[e];
+      p.pos_off = r0;
+      p.abs_pos = 1;
+      p.q_out = c->enc_q + static_cast<size_t>(r0) * qp;
+      p.q_stride = qp;
+      p.k_cache = c->enc_k;
+      p.v_cache = c->enc_v;
+      p.head_dim = c->cfg.head_dim;
+      p.max_seq = c->max_enc;
+      CKS(gemv(c, Epi::QKV, Mc, S.qkv, p));
+    }
+    for (int r0 = 0; r0 < P; r0 += kPrefillChunk) {
+      const int Mc = std::min(kPrefillChunk, P - r0);
+      AttnParams a{};
+      a.q = c->enc_q + static_cast<size_t>(r0) * qp;
+      a.q_stride = qp;
+      a.k_cache = c->enc_k;
+      a.v_cache = c->enc_v;
+      a.o = c->enc_o + static_cast<size_t>(r0) * qp;
+      a.o_stride = qp;
+      a.pos_off = r0;
+      a.abs_pos = 1;
+      a.fixed_keys = 1;
+      a.max_seq = c->max_enc;
+      a.scale = 1.0f;
+      a.bias = c->enc_bias;
+      a.bias_stride = 2 * c->max_enc - 1;
+      a.bias_zero = c->max_enc - 1;
+      CKS(attn_run(c, Mc, a));
+    }
+    for (int r0 = 0; r0 < P; r0 += kPrefillChunk) {
+      const int Mc = std::min(kPrefillChunk, P - r0);
+      float* xr = c->x_enc + static_cast<size_t>(r0) * dp;
+      CKS(resid_gemv(c, Mc, S.o, c->enc_o + static_cast<size_t>(r0) * qp, qp, xr, c->one));
+      GemvParams p{};
+      p.x = xr;
+      p.x_stride = dp;
+      p.gain = c->enc_ffn_norm[e];
+      p.h_out = c->hb;
+      p.h_stride = c->fp;
+      p.act = 1;
+      CKS(gemv(c, Epi::GATE_SILU, Mc, S.gateup, p));
+      CKS(resid_gemv(c, Mc, S.down, c->hb, c->fp, xr, c->one));
+    }
+  }
+  for (int l = 0; l < c->cfg.n_layers; ++l)
+    for (int r0 = 0; r0 < P; r0 += kPrefillChunk) {
+      const int Mc = std::min(kPrefillChunk, P - r0);
+      GemvParams p{};
+      p.x = c->x_enc + static_cast<size_t>(r0) * dp;
+      p.x_stride = dp;
+      p.gain = c->enc_final;  // cross K/V read the encoder's normed output
+      p.pos_off = r0;
+      p.abs_pos = 1;
+      p.seg_base = 1;  // the [ck; cv] site's segments are k and v
+      p.k_cache = c->ckc + l * c->cross_layer_kv;
+      p.v_cache = c->cvc + l * c->cross_layer_kv;
+      p.head_dim = c->cfg.head_dim;
+      p.max_seq = c->max_enc;
+      CKS(gemv(c, Epi::QKV, Mc, c->cross_kv[l], p));
+    }
+  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(c->start_tok), c->xv, dp,
+              c->cfg.d_model, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
+  CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
+  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, 1));
   return SSD_OK;
 }
 
@@ -953,7 +1152,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
   CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
-  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id));
+  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
   CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
               c->st));
@@ -1209,6 +1408,7 @@ static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
 }
 
 static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) {
+  if (c->t5) return enqueue_prefill_t5(c, a, b);
   return c->prefill_rows ? enqueue_prefill(c, a, b) : enqueue_prefill_tc(c, a, b);
 }
 static ssd_status enq_draft_fn(ssd_ctx* c, int g, int) { return enqueue_draft(c, g); }
@@ -1297,7 +1497,9 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   drop_graphs(c);
   void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
                   c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
-                  c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles};
+                  c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles,
+                  c->x_enc, c->enc_q, c->enc_o, c->enc_k, c->enc_v, c->ckc, c->cvc, c->dec_bias, c->enc_bias, c->one,
+                  c->start_tok};
   for (void* b : bufs)
     if (b) cudaFree(b);
   if (c->ev_in) cudaEventDestroy(c->ev_in);
@@ -1307,8 +1509,52 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   return SSD_OK;
 }
 
+// Relative-position bucket of the key-minus-query offset delta (T5 v1.1): bidirectional stacks split
+// the buckets between earlier (and equal) and later keys, past-only stacks give all of them to
+// earlier keys (later keys share bucket 0); within a half, offsets below n/2 get one bucket each and
+// larger ones logarithmically spaced buckets up to max_distance, beyond which they share the last.
+// The logarithmic index is computed in fp64 and floored after adding 1e-9, so that exact powers land
+// on their bucket whatever the platform's log rounds to.
+static int rel_bucket_host(int delta, bool bidirectional, int n_buckets, int max_distance) {
+  int n = n_buckets, base = 0, dist;
+  if (bidirectional) {
+    n /= 2;
+    if (delta > 0) base = n;
+    dist = delta < 0 ? -delta : delta;
+  } else {
+    dist = delta < 0 ? -delta : 0;
+  }
+  const int exact = n / 2;
+  if (dist < exact) return base + dist;
+  const double f = std::log(static_cast<double>(dist) / exact) / std::log(static_cast<double>(max_distance) / exact) *
+                       (n - exact) + 1e-9;
+  const int far = exact + static_cast<int>(f);
+  return base + (far < n - 1 ? far : n - 1);
+}
+
+// out[h][j] = rel[bucket(j - zero)][h] for j < n, on the ctx stream (bucket decided on the host).
+static ssd_status build_bias_table(ssd_ctx* c, const void* rel, float* out, int n, int zero, bool bidirectional) {
+  std::vector<int> b(n);
+  for (int j = 0; j < n; ++j)
+    b[j] = rel_bucket_host(j - zero, bidirectional, c->cfg.rel_buckets, c->cfg.rel_max_distance);
+  int* db = nullptr;
+  CK(cudaMalloc(&db, sizeof(int) * n));
+  cudaError_t e = cudaMemcpy(db, b.data(), sizeof(int) * n, cudaMemcpyHostToDevice);
+  const int H = c->cfg.n_heads;
+  if (e == cudaSuccess) {
+    bias_table_kernel<<<(n * H + 255) / 256, 256, 0, c->cs>>>(static_cast<const __nv_bfloat16*>(rel), db, n, H, out);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->cs);
+  cudaFree(db);
+  CK(e);
+  return SSD_OK;
+}
+
 static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weights* w) {
   const ssd_config& k = *cfg;
+  const bool t5 = k.arch == SSD_ARCH_T5;
+  if (k.arch != SSD_ARCH_LLAMA && !t5) return fail(c, SSD_ERR_INVALID_ARG, "arch %d", k.arch);
   if (k.n_layers < 1 || k.d_model < 64 || k.n_heads < 1 || k.vocab < 2 || k.d_ff < 64)
     return fail(c, SSD_ERR_INVALID_ARG, "bad model shape");
   if (k.head_dim != 64 && k.head_dim != 128) return fail(c, SSD_ERR_INVALID_ARG, "head_dim must be 64 or 128");
@@ -1338,6 +1584,26 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     if (!w->wq[l] || !w->wk[l] || !w->wv[l] || !w->wo[l] || !w->w_gate[l] || !w->w_up[l] || !w->w_down[l] ||
         !w->attn_norm[l] || !w->ffn_norm[l])
       return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer in layer %d", l);
+  const ssd_encdec_weights* ed = t5 ? w->encdec : nullptr;
+  if (t5) {
+    if (k.in_kind == SSD_IN_BLOCK)
+      return fail(c, SSD_ERR_INVALID_ARG, "the encoder-decoder model takes SSD_IN_IDENTITY or SSD_IN_MLP2");
+    if (k.n_enc_layers < 1 || k.max_enc < 1) return fail(c, SSD_ERR_INVALID_ARG, "n_enc_layers / max_enc");
+    if (k.rel_buckets < 4 || k.rel_buckets % 2 || k.rel_max_distance <= k.rel_buckets / 2)
+      return fail(c, SSD_ERR_INVALID_ARG, "rel_buckets must be even and >= 4, rel_max_distance > rel_buckets / 2");
+    if (k.start_token < 0 || k.start_token >= k.vocab) return fail(c, SSD_ERR_INVALID_ARG, "start_token");
+    if (!ed || !ed->cq || !ed->ck || !ed->cv || !ed->co || !ed->cross_norm || !ed->enc_wq || !ed->enc_wk ||
+        !ed->enc_wv || !ed->enc_wo || !ed->enc_wi0 || !ed->enc_wi1 || !ed->enc_wff || !ed->enc_attn_norm ||
+        !ed->enc_ffn_norm || !ed->enc_final || !ed->enc_rel || !ed->dec_rel)
+      return fail(c, SSD_ERR_INVALID_ARG, "null encoder-decoder weight pointer");
+    for (int l = 0; l < k.n_layers; ++l)
+      if (!ed->cq[l] || !ed->ck[l] || !ed->cv[l] || !ed->co[l] || !ed->cross_norm[l])
+        return fail(c, SSD_ERR_INVALID_ARG, "null cross-attention weight pointer in layer %d", l);
+    for (int e = 0; e < k.n_enc_layers; ++e)
+      if (!ed->enc_wq[e] || !ed->enc_wk[e] || !ed->enc_wv[e] || !ed->enc_wo[e] || !ed->enc_wi0[e] ||
+          !ed->enc_wi1[e] || !ed->enc_wff[e] || !ed->enc_attn_norm[e] || !ed->enc_ffn_norm[e])
+        return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer in encoder layer %d", e);
+  }
 
   CK(cudaGetDevice(&c->device));
   cudaDeviceProp prop;
@@ -1374,6 +1640,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
 
   c->cfg = k;
   c->qdim = qdim;
+  c->t5 = t5;
+  c->max_enc = t5 ? k.max_enc : 0;
   auto pad = [](int v) { return (v + kTileK - 1) / kTileK * kTileK; };
   c->dp = pad(k.d_model);
   c->qp = pad(qdim);
@@ -1409,6 +1677,26 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     CKS(make_site(c, &c->in2, &w->in_w2, 1, k.d_model, k.in_hidden, false));
   }
   CKS(make_site(c, &c->head, &w->lm_head, 1, k.vocab, k.d_model, false));
+  if (t5) {
+    c->cross_q.resize(k.n_layers);
+    c->cross_o.resize(k.n_layers);
+    c->cross_kv.resize(k.n_layers);
+    for (int l = 0; l < k.n_layers; ++l) {
+      const void* kv[2] = {ed->ck[l], ed->cv[l]};
+      CKS(make_site(c, &c->cross_q[l], &ed->cq[l], 1, qdim, k.d_model, false));
+      CKS(make_site(c, &c->cross_o[l], &ed->co[l], 1, k.d_model, qdim, false));
+      CKS(make_site(c, &c->cross_kv[l], kv, 2, qdim, k.d_model, false));
+    }
+    c->enc_layers.resize(k.n_enc_layers);
+    for (int e = 0; e < k.n_enc_layers; ++e) {
+      LayerSites& S = c->enc_layers[e];
+      const void* qkv[3] = {ed->enc_wq[e], ed->enc_wk[e], ed->enc_wv[e]};
+      CKS(make_site(c, &S.qkv, qkv, 3, qdim, k.d_model, false));
+      CKS(make_site(c, &S.o, &ed->enc_wo[e], 1, k.d_model, qdim, false));
+      CKS(make_pair_site(c, &S.gateup, ed->enc_wi0[e], ed->enc_wi1[e], k.d_ff, k.d_model));
+      CKS(make_site(c, &S.down, &ed->enc_wff[e], 1, k.d_model, k.d_ff, false));
+    }
+  }
   c->tc_layers.resize(n_blocks);
   for (int l = 0; l < n_blocks; ++l) {
     TcLayer& t = c->tc_layers[l];
@@ -1452,7 +1740,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CKS(alloc(c, reinterpret_cast<void**>(&c->hb), sizeof(float) * R * c->fp));
   CKS(alloc(c, reinterpret_cast<void**>(&c->hin), sizeof(float) * R * c->ip));
   // RMSNorm gains: zero-padded copies, so 256-column slices never read past a gain vector
-  const int n_gains = 2 * n_blocks + 2;
+  const int n_gains = 2 * n_blocks + 2 + (t5 ? 2 * k.n_enc_layers + k.n_layers + 1 : 0);
   CKS(alloc(c, reinterpret_cast<void**>(&c->gains), sizeof(__nv_bfloat16) * n_gains * c->dp));
   auto copy_gain = [&](int slot, const void* src) -> const __nv_bfloat16* {
     __nv_bfloat16* dst = c->gains + static_cast<size_t>(slot) * c->dp;
@@ -1469,15 +1757,51 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   c->in_norm = k.in_kind == SSD_IN_MLP2 ? copy_gain(2 * n_blocks + 1, w->in_norm) : nullptr;
   if (!c->final_norm || (k.in_kind == SSD_IN_MLP2 && !c->in_norm))
     return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
+  if (t5) {
+    int slot = 2 * n_blocks + 2;
+    for (int e = 0; e < k.n_enc_layers; ++e) {
+      c->enc_attn_norm.push_back(copy_gain(slot++, ed->enc_attn_norm[e]));
+      c->enc_ffn_norm.push_back(copy_gain(slot++, ed->enc_ffn_norm[e]));
+      if (!c->enc_attn_norm.back() || !c->enc_ffn_norm.back()) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
+    }
+    for (int l = 0; l < k.n_layers; ++l) {
+      c->cross_norm.push_back(copy_gain(slot++, ed->cross_norm[l]));
+      if (!c->cross_norm.back()) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
+    }
+    c->enc_final = copy_gain(slot++, ed->enc_final);
+    if (!c->enc_final) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
+  }
   c->layer_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
   CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(float) * c->layer_kv * n_blocks));
   CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(float) * c->layer_kv * n_blocks));
   CKS(alloc(c, reinterpret_cast<void**>(&c->rope), sizeof(float2) * k.max_seq * (k.head_dim / 2)));
+  if (t5) {
+    const size_t E = k.max_enc;
+    c->cross_layer_kv = static_cast<size_t>(k.n_heads) * E * k.head_dim;
+    CKS(alloc(c, reinterpret_cast<void**>(&c->x_enc), sizeof(float) * E * c->dp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->enc_q), sizeof(float) * E * c->qp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->enc_o), sizeof(float) * E * c->qp));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->enc_k), sizeof(float) * c->cross_layer_kv));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->enc_v), sizeof(float) * c->cross_layer_kv));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->ckc), sizeof(float) * c->cross_layer_kv * k.n_layers));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->cvc), sizeof(float) * c->cross_layer_kv * k.n_layers));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->dec_bias), sizeof(float) * k.n_heads * k.max_seq));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->enc_bias), sizeof(float) * k.n_heads * (2 * E - 1)));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->one), sizeof(float)));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->start_tok), sizeof(int)));
+    const float one = 1.0f;
+    CK(cudaMemcpy(c->one, &one, sizeof(float), cudaMemcpyHostToDevice));
+    CK(cudaMemcpy(c->start_tok, &k.start_token, sizeof(int), cudaMemcpyHostToDevice));
+  }
   CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->gemv_ctas * c->num_sms * R * kTileN));
   int max_rt = 1;
   for (const Site* s : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->head,
                         &c->in1, &c->in2})
     max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
+  if (t5)
+    for (const Site* s : {&c->cross_q[0], &c->cross_o[0], &c->cross_kv[0], &c->enc_layers[0].qkv, &c->enc_layers[0].o,
+                          &c->enc_layers[0].gateup, &c->enc_layers[0].down})
+      max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_part),
@@ -1485,7 +1809,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * k.n_heads));
   CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_table), sizeof(int) * (k.max_seq + 1)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_launch), sizeof(int) * SSD_MAX_GAMMA));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * k.max_seq * d));
+  const size_t in_rows = std::max(static_cast<size_t>(k.max_seq), static_cast<size_t>(c->max_enc));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * in_rows * d));
   {
     const size_t Pm = k.max_seq;
     const size_t kmax = std::max(std::max(static_cast<size_t>(k.d_model), static_cast<size_t>(qdim)),
@@ -1502,7 +1827,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
       CKS(encode_map_sw128(c, &c->a_maps[i][1], c->a_lo, Pm, ks[i], kTcM));
     }
   }
-  CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * k.max_seq));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * in_rows));
   {
     // persistent forward kernel: one CTA per SM, the weight maps of every projection in one table
     int per_sm = 0;
@@ -1539,11 +1864,17 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->ev_in, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&c->ev_out, cudaEventDisableTiming));
-  const int nrope = k.max_seq * (k.head_dim / 2);
-  rope_table_kernel<<<(nrope + 255) / 256, 256, 0, c->cs>>>(c->rope, k.max_seq, k.head_dim,
-                                                            static_cast<double>(k.rope_theta));
-  CK(cudaGetLastError());
+  if (!t5) {  // the encoder-decoder model has no rotary embedding
+    const int nrope = k.max_seq * (k.head_dim / 2);
+    rope_table_kernel<<<(nrope + 255) / 256, 256, 0, c->cs>>>(c->rope, k.max_seq, k.head_dim,
+                                                              static_cast<double>(k.rope_theta));
+    CK(cudaGetLastError());
+  }
   CK(cudaStreamSynchronize(c->cs));
+  if (t5) {
+    CKS(build_bias_table(c, ed->dec_rel, c->dec_bias, k.max_seq, k.max_seq - 1, false));
+    CKS(build_bias_table(c, ed->enc_rel, c->enc_bias, 2 * k.max_enc - 1, k.max_enc - 1, true));
+  }
   return SSD_OK;
 }
 
@@ -1577,8 +1908,8 @@ static ssd_status prefill_impl(ssd_ctx* c, int n_vis, int n_prompt) {
   CK(cudaGraphLaunch(it->second, c->cs));
   c->prefilled = true;
   c->drafted_gamma = 0;
-  c->prompt_len = P;
-  c->kv_upper = P;
+  c->prompt_len = c->t5 ? 1 : P;  // decoder positions before the first new token
+  c->kv_upper = c->prompt_len;
   c->last_prefill_shape = key;
   return SSD_OK;
 }
@@ -1587,7 +1918,12 @@ static ssd_status check_prefill_args(ssd_ctx* c, const void* vis, int n_vis, con
   if (n_vis < 0 || n_prompt < 0 || n_vis + n_prompt < 1) return fail(c, SSD_ERR_INVALID_ARG, "empty prompt");
   if (n_vis > 0 && !vis) return fail(c, SSD_ERR_INVALID_ARG, "vis_emb is null");
   if (n_prompt > 0 && !prompt) return fail(c, SSD_ERR_INVALID_ARG, "prompt is null");
-  if (n_vis + n_prompt + 1 > c->cfg.max_seq) return fail(c, SSD_ERR_CAPACITY, "prompt longer than max_seq");
+  if (c->t5) {
+    if (n_vis + n_prompt > c->max_enc) return fail(c, SSD_ERR_CAPACITY, "encoder rows %d > max_enc %d",
+                                                   n_vis + n_prompt, c->max_enc);
+  } else if (n_vis + n_prompt + 1 > c->cfg.max_seq) {
+    return fail(c, SSD_ERR_CAPACITY, "prompt longer than max_seq");
+  }
   return SSD_OK;
 }
 
@@ -1826,8 +2162,9 @@ static ssd_status generate_impl(ssd_ctx* c, const void* vis, int n_vis, const in
   if (!c) return SSD_ERR_INVALID_ARG;
   if (!out || !n_out) return fail(c, SSD_ERR_INVALID_ARG, "out / n_out is null");
   CKS(check_prefill_args(c, vis, n_vis, prompt, n_prompt));
-  if (static_cast<int64_t>(n_vis) + n_prompt + max_new + gamma + 1 > c->cfg.max_seq)
-    return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 > max_seq");
+  const int64_t dec_prompt = c->t5 ? 1 : static_cast<int64_t>(n_vis) + n_prompt;
+  if (dec_prompt + max_new + gamma + 1 > c->cfg.max_seq)
+    return fail(c, SSD_ERR_CAPACITY, "decoder prompt rows + max_new + gamma + 1 > max_seq");
   CKS(enter(c));
   if (n_vis > 0)
     CK(cudaMemcpyAsync(c->in_vis, vis, sizeof(__nv_bfloat16) * n_vis * c->cfg.d_model, cudaMemcpyHostToDevice,

@@ -99,6 +99,9 @@ struct GemvParams {
   // dependent grid starts: the split-KV attention after the QKV projection reads older cache rows
   // before its own wait.
   int late_trigger;
+  int seg_base;  // QKV: segment of the site's first matrix (0 = q; 1 = k, for a [k; v] site)
+  int abs_pos;   // row m sits at position pos_off + m, st->kv_len ignored (the encoder's rows)
+  int act;       // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up (gated GELU)
 };
 
 template <int M>
@@ -189,7 +192,8 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 lo, __nv_bfloat16 
 // fp32, before the RMSNorm scale) and rs[m] (1 if no norm).  pre: inputs fetched
 // into shared memory after the upstream wait, or null -- QKV: the rotation table
 // rows of the M positions ([M][head_dim / 2] float2); RESID: the tile's base rows
-// ([M][kTileN]).  base_pos: position of row 0 (st->kv_len + pos_off, read once per CTA).
+// ([M][kTileN]).  base_pos: position of row 0 (st->kv_len + pos_off, or pos_off with abs_pos; read
+// once per CTA).
 
 __device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
 
@@ -198,8 +202,9 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
                                               const float* pre, int base_pos, int tid) {
   if constexpr (EPI == Epi::QKV) {
     const int r0 = rt * kTileN;
-    const int mat = r0 / p.seg_rows;  // 0 = q, 1 = k, 2 = v
-    const int local0 = r0 - mat * p.seg_rows;
+    const int seg = r0 / p.seg_rows;       // source matrix of this row tile within the site
+    const int mat = seg + p.seg_base;      // 0 = q, 1 = k, 2 = v
+    const int local0 = r0 - seg * p.seg_rows;
     const int Dh = p.head_dim, half = Dh >> 1;
     if (mat < 2) {
       for (int idx = tid; idx < M * (kTileN / 2); idx += kDrainThreads) {
@@ -213,10 +218,13 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
         }
         const float a = out[m * kTileN + ra] * rs[m];
         const float b = out[m * kTileN + rb] * rs[m];
-        const float2 cs = pre ? reinterpret_cast<const float2*>(pre)[m * half + j]
-                              : p.rope_cs[static_cast<size_t>(pos) * half + j];
-        const float va = a * cs.x - b * cs.y;
-        const float vb = a * cs.y + b * cs.x;
+        float va = a, vb = b;  // no rotation without a table (relative-position-bias models)
+        if (p.rope_cs) {
+          const float2 cs = pre ? reinterpret_cast<const float2*>(pre)[m * half + j]
+                                : p.rope_cs[static_cast<size_t>(pos) * half + j];
+          va = a * cs.x - b * cs.y;
+          vb = a * cs.y + b * cs.x;
+        }
         if (mat == 0) {
           p.q_out[m * p.q_stride + local0 + ra] = va;
           p.q_out[m * p.q_stride + local0 + rb] = vb;
@@ -246,7 +254,7 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       if (n >= p.N) continue;
       const float g = out[m * kTileN + j] * rs[m];
       const float u = out[m * kTileN + kHalfN + j] * rs[m];
-      p.h_out[m * p.h_stride + n] = silu_f(g) * u;
+      p.h_out[m * p.h_stride + n] = (p.act ? gelu_tanh_f(g) : silu_f(g)) * u;
     }
   } else if constexpr (EPI == Epi::SILU) {
     for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
@@ -533,12 +541,12 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
     // the base rows of this CTA's first and last row tiles (RESID; every contributor of a split
     // tile fetches them, whichever ends up owning it, before its ticket)
     const int rt_first = u0 / p.n_kt, rt_last = (u1 - 1) / p.n_kt;
-    const int base_pos = __ldcg(&p.st->kv_len) + p.pos_off;
+    const int base_pos = (p.abs_pos ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
     float* pre = reinterpret_cast<float*>(smem + S::kPre);
     bool pre_rope = false;
     if constexpr (EPI == Epi::QKV) {
       const int half = p.head_dim >> 1;
-      pre_rope = base_pos >= 0 && base_pos + M <= p.max_seq && half <= kTileN;
+      pre_rope = p.rope_cs != nullptr && base_pos >= 0 && base_pos + M <= p.max_seq && half <= kTileN;
       if (pre_rope)
         for (int idx = dt; idx < M * half; idx += kDrainThreads) {
           const int m = idx / half, j = idx - m * half;

@@ -41,6 +41,10 @@ class SSDModel:
     ffn_norm) and, for the MLP2 imitation network, "in_norm", "in_w1", "in_w2"; for the block
     imitation network "in_block" (a dict like a layer's).
     resid_scale: fp32 device tensor [n_layers]; in_scale: fp32 device tensor [1].
+    Encoder-decoder model (cfg["arch"] == SSD_ARCH_T5): "layers" and "final_norm" are the decoder's
+    (w_gate / w_up / w_down = wi_0 / wi_1 / wo of its gated-GELU MLP), and weights["encdec"] holds
+    "cross" (list of dicts cq, ck, cv, co, cross_norm per decoder layer), "enc" (list of dicts like a
+    layer's), "enc_final", "enc_rel", "dec_rel".
     """
 
     def __init__(self, cfg: dict, weights: dict, resid_scale: torch.Tensor, in_scale: torch.Tensor,
@@ -50,7 +54,7 @@ class SSDModel:
         self.weights = weights            # keep the borrowed tensors alive
         self.resid_scale = resid_scale
         self.in_scale = in_scale
-        c = B.SSDConfig(**{k: self.cfg[k] for k, _ in B.SSDConfig._fields_})
+        c = B.SSDConfig(**{k: self.cfg.get(k, 0) for k, _ in B.SSDConfig._fields_})
         L = cfg["n_layers"]
         arrs = {}
         for name in ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down", "attn_norm", "ffn_norm"):
@@ -58,12 +62,29 @@ class SSDModel:
         if "in_block" in weights:
             names = ("wq", "wk", "wv", "wo", "w_gate", "w_up", "w_down", "attn_norm", "ffn_norm")
             arrs["in_block"] = (ctypes.c_void_p * 9)(*[weights["in_block"][n].data_ptr() for n in names])
+        encdec = None
+        if self.cfg.get("arch", 0) == B.SSD_ARCH_T5:
+            ed = weights["encdec"]
+            E = cfg["n_enc_layers"]
+            for n in ("cq", "ck", "cv", "co", "cross_norm"):
+                arrs["x_" + n] = (ctypes.c_void_p * L)(*[ed["cross"][l][n].data_ptr() for l in range(L)])
+            enc_names = {"enc_wq": "wq", "enc_wk": "wk", "enc_wv": "wv", "enc_wo": "wo", "enc_wi0": "w_gate",
+                         "enc_wi1": "w_up", "enc_wff": "w_down", "enc_attn_norm": "attn_norm",
+                         "enc_ffn_norm": "ffn_norm"}
+            for cn, n in enc_names.items():
+                arrs["x_" + cn] = (ctypes.c_void_p * E)(*[ed["enc"][e][n].data_ptr() for e in range(E)])
+            encdec = B.SSDEncDecWeights(enc_final=_ptr(ed["enc_final"]), enc_rel=_ptr(ed["enc_rel"]),
+                                        dec_rel=_ptr(ed["dec_rel"]),
+                                        **{n: ctypes.cast(arrs["x_" + n], B._PP) for n in B.ENCDEC_ARRAYS})
+            self._encdec = encdec
         self._arrs = arrs
         w = B.SSDWeights(embed=_ptr(weights["embed"]), lm_head=_ptr(weights["lm_head"]),
                          final_norm=_ptr(weights["final_norm"]),
                          in_norm=_ptr(weights.get("in_norm")), in_w1=_ptr(weights.get("in_w1")),
                          in_w2=_ptr(weights.get("in_w2")), resid_scale=_ptr(resid_scale),
-                         in_scale=_ptr(in_scale), **{k: ctypes.cast(v, B._PP) for k, v in arrs.items()})
+                         in_scale=_ptr(in_scale),
+                         encdec=ctypes.pointer(encdec) if encdec is not None else None,
+                         **{k: ctypes.cast(v, B._PP) for k, v in arrs.items() if not k.startswith("x_")})
         self.stream = stream if stream is not None else torch.cuda.current_stream()
         ctx = ctypes.c_void_p()
         self._check(self.lib.ssd_create(ctypes.byref(c), ctypes.byref(w), self.stream.cuda_stream,

@@ -36,3 +36,46 @@ def device_inputs(w: synth.Workload, seed: int | None = None):
     v = lib.bf16_bits_to_device(vis) if w.n_vis > 0 else None
     p = torch.from_numpy(prompt.astype(np.int32)).cuda()
     return vis, prompt, v, p
+
+
+_T5_RENAME = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
+              "ffn_norm": "ffn_norm"}
+
+
+def t5_device_weights(bits: dict) -> dict:
+    """Device copies of a synth encoder-decoder workload in the layout lib.SSDModel takes."""
+    up = lib.bf16_bits_to_device
+
+    def stack(lw, norm):
+        d = {_T5_RENAME[n]: up(a) for n, a in lw.items() if n in _T5_RENAME}
+        d["attn_norm"] = up(lw[norm])
+        return d
+
+    out = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
+           "layers": [stack(lw, "self_norm") for lw in bits["dec"]]}
+    out["encdec"] = {
+        "cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
+        "enc": [stack(lw, "attn_norm") for lw in bits["enc"]],
+        "enc_final": up(bits["enc_final"]), "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}
+    for k in ("in_norm", "in_w1", "in_w2"):
+        if k in bits:
+            out[k] = up(bits[k])
+    return out
+
+
+def make_t5_model(w: synth.T5Workload, bits: dict | None = None, dev: dict | None = None,
+                  gamma_max: int | None = None, max_seq: int | None = None, max_enc: int | None = None):
+    bits = bits if bits is not None else synth.make_t5_weights(w)
+    dev = dev if dev is not None else t5_device_weights(bits)
+    cfg = lib.t5_config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, gamma_max or max(w.gamma, 1),
+                             max_seq or (w.max_dec() + 1), max_enc or w.enc_len, w.eos_id)
+    rs = torch.tensor(w.dec_scale(), dtype=torch.float32, device="cuda")
+    ins = torch.tensor([w.in_scale()], dtype=torch.float32, device="cuda")
+    return lib.SSDModel(cfg, dev, rs, ins), bits, dev
+
+
+def t5_device_inputs(w: synth.T5Workload, seed: int | None = None):
+    q, prompt = synth.make_t5_inputs(w, seed)
+    v = lib.bf16_bits_to_device(q) if w.n_query > 0 else None
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    return q, prompt, v, p
