@@ -78,14 +78,24 @@ KERNEL_ROWS = (("qkv", "gemv_kernel<M, QKV> (q/k/v + RoPE + KV write)"),
                ("in2", "gemv_kernel<1, RESID> (imitation FC2)"))
 
 
-def kernel_table(model, w, v, p, stream, hbm_peak, reps=50):
+ENCDEC_KERNEL_ROWS = (("qkv", "gemv_kernel<M, QKV> (self q/k/v + KV write, no RoPE)"),
+                      ("o", "gemv_kernel<M, RESID> (self o; cross q / cross o have this shape)"),
+                      ("gateup", "gemv_kernel<M, GATE_SILU> (wi_0/wi_1, gated GELU)"),
+                      ("down", "gemv_kernel<M, RESID> (wo of the MLP)"),
+                      ("attn", "attn_kernel<M, 64, EXT> (self-attention, relative-position bias)"),
+                      ("head", "gemv_kernel<M, ARGMAX> (LM head)"),
+                      ("in1", "gemv_kernel<1, SILU> (imitation FC1)"),
+                      ("in2", "gemv_kernel<1, RESID> (imitation FC2)"))
+
+
+def kernel_table(model, w, v, p, stream, hbm_peak, reps=50, rows_table=KERNEL_ROWS, layer_sum=True):
     """Every decode kernel timed alone (CUDA events, `reps` back-to-back launches) at the draft's
     1 row and the verification's gamma + 1 rows, against the HBM copy peak.  `layer_m*` sums one
     decoder layer's kernels (bytes / time), the fraction a layer would reach with no launch gaps."""
     import torch
     rows_out, layer = [], {}
     for rows in (1, w.gamma + 1):
-        for name, label in KERNEL_ROWS:
+        for name, label in rows_table:
             if name in ("in1", "in2") and rows != 1:
                 continue
             model.prefill(v, p)
@@ -100,7 +110,7 @@ def kernel_table(model, w, v, p, stream, hbm_peak, reps=50):
             gbs = nbytes / us / 1e3
             rows_out.append({"kernel": label.replace("<M,", f"<{rows},"), "rows": rows, "bytes": nbytes,
                              "us": round(us, 2), "gbs": round(gbs, 1), "frac": round(gbs / hbm_peak, 3)})
-            if name in ("qkv", "o", "gateup", "down", "attn"):
+            if layer_sum and name in ("qkv", "o", "gateup", "down", "attn"):
                 lb, lt = layer.get(rows, (0, 0.0))
                 layer[rows] = (lb + nbytes, lt + us)
     summary = {f"layer_m{r}": {"us": round(t, 1), "gbs": round(b_ / t / 1e3, 1), "frac": round(b_ / t / 1e3 / hbm_peak, 3)}
@@ -364,6 +374,7 @@ def run_encdec(args) -> None:
 
     model.prefill(v, p)
     prefill_ms = min(ev_ms(lambda: model.prefill(v, p)) for _ in range(3))
+    kernels = kernel_table(model, w, v, p, stream, peak or 6800.0, rows_table=ENCDEC_KERNEL_ROWS, layer_sum=False)
     rows = []
     for s_val in S_VALUES:
         ws = w.replace(s=s_val)
@@ -389,7 +400,8 @@ def run_encdec(args) -> None:
                                   f"{w.n_prompt} prompt ids; k={w.draft_exit_k}, gamma={w.gamma}, "
                                   f"{w.max_new} new tokens; bs1",
                       "prefill_ms": prefill_ms, "peak_hbm_gbs": peak, "bytes_per_token":
-                          {"draft": draft_bytes, "greedy": greedy_bytes}, "per_s": rows}), flush=True)
+                          {"draft": draft_bytes, "greedy": greedy_bytes}, "per_s": rows, "kernels": kernels}),
+          flush=True)
 
 
 def run_sweep(args) -> None:

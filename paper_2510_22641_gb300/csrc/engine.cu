@@ -2327,7 +2327,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       p.v_cache = c->vc + layer * c->layer_kv;
       p.head_dim = c->cfg.head_dim;
       p.max_seq = c->cfg.max_seq;
-      p.rope_cs = c->rope;
+      p.rope_cs = c->t5 ? nullptr : c->rope;
       break;
     case 1:
     case 3:

@@ -9,6 +9,11 @@ cudaProfilerStart/Stop window (use `ncu --profile-from-start off`).
 but fewer layers, so full metric sets can be captured with a few GB on the
 device; every weight matrix is still larger or comparable to what one kernel
 streams at full size.
+
+  python -m paper_2510_22641_gb300.profile_run --encdec --layers 24 --phase greedy --tokens 2
+
+--encdec runs the BLIP-2 FlanT5-xl-shaped encoder-decoder instead (d=2048, 32x64 heads,
+gated-GELU 5120, V=32128; --layers encoder and decoder layers each, 24 at full size).
 """
 from __future__ import annotations
 
@@ -31,12 +36,17 @@ def main() -> None:
     ap.add_argument("--rows", type=int, default=1, help="--phase proj: activation rows")
     ap.add_argument("--tokens", type=int, default=8)
     ap.add_argument("--s", type=float, default=0.2)
+    ap.add_argument("--encdec", action="store_true", help="the FlanT5-xl-shaped encoder-decoder model")
     args = ap.parse_args()
 
     import torch
 
     import paper_2510_22641_gb300 as lib
     import synth
+
+    if args.encdec:
+        encdec(args, lib, synth, torch)
+        return
 
     base = synth.LLAVA7B
     shape = synth.ModelShape(args.layers, 4096, 32, 128, 11008, 32000)
@@ -90,6 +100,54 @@ def main() -> None:
         model.prefill(v, p)
         model.sync()
         torch.cuda.profiler.stop()
+    print("profile_run done", model.stats())
+    model.close()
+
+
+def encdec(args, lib, synth, torch) -> None:
+    """Prefill (encoder + cross K/V + first decoder step) and one decode phase of the FlanT5-xl shape."""
+    base = synth.FLANT5XL
+    shape = synth.T5Shape(args.layers, args.layers, 2048, 32, 64, 5120, 32128)
+    w = base.replace(shape=shape, draft_exit_k=min(base.draft_exit_k, args.layers), s=args.s)
+    lib.build()
+    bits = synth.make_t5_weights(w)
+    up = lib.bf16_bits_to_device
+    ren = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
+           "ffn_norm": "ffn_norm"}
+
+    def stack(lw, norm):
+        d = {ren[n]: up(a) for n, a in lw.items() if n in ren}
+        d["attn_norm"] = up(lw[norm])
+        return d
+
+    dev = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
+           "layers": [stack(lw, "self_norm") for lw in bits["dec"]],
+           "in_norm": up(bits["in_norm"]), "in_w1": up(bits["in_w1"]), "in_w2": up(bits["in_w2"]),
+           "encdec": {"cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
+                      "enc": [stack(lw, "attn_norm") for lw in bits["enc"]], "enc_final": up(bits["enc_final"]),
+                      "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}}
+    cfg = lib.t5_config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                             w.max_new + lib.SSD_MAX_GAMMA + 2, w.enc_len)
+    model = lib.SSDModel(cfg, dev, torch.tensor(w.dec_scale(), device="cuda"),
+                         torch.tensor([w.in_scale()], device="cuda"))
+    q, prompt = synth.make_t5_inputs(w)
+    v = up(q)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    n = 1 + args.tokens
+    model.prefill(v, p)
+    model.greedy_decode(n) if args.phase == "greedy" else model.decode(n, w.gamma)
+    if args.phase != "prefill":
+        model.prefill(v, p)
+    model.sync()
+    torch.cuda.profiler.start()
+    if args.phase == "greedy":
+        model.greedy_decode(n)
+    elif args.phase == "ssd":
+        model.decode(n, w.gamma)
+    else:
+        model.prefill(v, p)
+    model.sync()
+    torch.cuda.profiler.stop()
     print("profile_run done", model.stats())
     model.close()
 
