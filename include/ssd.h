@@ -247,6 +247,17 @@ SSD_API ssd_status ssd_decode_dynamic(ssd_ctx* ctx, int max_new, int d0, int n_m
  * function; no context, no GPU). */
 SSD_API int ssd_draft_length(int t, int d0, int n_max);
 
+/* Relative-position bucket of the key-minus-query offset `delta` that the
+ * SSD_ARCH_T5 model's bias tables use (host function; no context, no GPU):
+ * bidirectional != 0 splits the n_buckets between earlier (and equal) and later
+ * keys (the encoder), otherwise all go to earlier keys and later keys share
+ * bucket 0 (the decoder's self-attention).  Within a half, offsets below n/2
+ * get one bucket each and larger ones logarithmically spaced buckets up to
+ * max_distance, past which they share the last.  The logarithmic index is
+ * floored in fp64 after adding 1e-9.  Returns -1 for n_buckets < 4, odd
+ * n_buckets or max_distance <= n_buckets / 2. */
+SSD_API int ssd_rel_bucket(int delta, int bidirectional, int n_buckets, int max_distance);
+
 /* Baseline: plain greedy decoding with the full model (same kernels, one
  * token per step, device-side loop).  Same buffers as ssd_decode.  async. */
 SSD_API ssd_status ssd_greedy_decode(ssd_ctx* ctx, int max_new, int32_t* out_tok, int32_t* n_out);

@@ -24,7 +24,7 @@ STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_C
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
 
 EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode", "ssd_decode_dynamic",
-            "ssd_draft_length",
+            "ssd_draft_length", "ssd_rel_bucket",
             "ssd_greedy_decode", "ssd_generate", "ssd_greedy_generate", "ssd_sync", "ssd_get_stats",
             "ssd_set_logits_capture", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
             "ssd_status_string",
@@ -109,6 +109,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         f.restype = ctypes.c_int
     lib.ssd_draft_length.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int]
     lib.ssd_draft_length.restype = ctypes.c_int
+    lib.ssd_rel_bucket.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int]
+    lib.ssd_rel_bucket.restype = ctypes.c_int
     lib.ssd_status_string.argtypes = [ctypes.c_int]
     lib.ssd_status_string.restype = ctypes.c_char_p
     lib.ssd_last_error.argtypes = [vp]

@@ -2101,6 +2101,11 @@ static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, in
 
 int ssd_draft_length(int t, int d0, int n_max) { return draft_length_fp64(t, d0, n_max); }
 
+int ssd_rel_bucket(int delta, int bidirectional, int n_buckets, int max_distance) {
+  if (n_buckets < 4 || n_buckets % 2 || max_distance <= n_buckets / 2) return -1;
+  return rel_bucket_host(delta, bidirectional != 0, n_buckets, max_distance);
+}
+
 ssd_status ssd_decode_dynamic(ssd_ctx* c, int max_new, int d0, int n_max, int gamma_cap, int32_t* out_tok,
                               int32_t* n_out) {
   if (!c) return SSD_ERR_INVALID_ARG;
