@@ -8,12 +8,13 @@ from ._binding import SSD_ARCH_LLAMA, SSD_ARCH_T5, SSD_IN_IDENTITY, SSD_IN_MLP2,
 from .build import build
 
 __all__ = ["build", "load", "SSDError", "SSD_ARCH_LLAMA", "SSD_ARCH_T5", "SSD_IN_IDENTITY", "SSD_IN_MLP2",
-           "SSD_MAX_GAMMA", "SSDModel", "bf16_bits_to_device", "config_dict", "t5_config_dict"]
+           "SSD_MAX_GAMMA", "SSDModel", "bf16_bits_to_device", "encdec_device_weights", "config_dict",
+           "t5_config_dict"]
 
 
 def __getattr__(name):
     # torch is only needed for the model wrapper; the ABI loader works without it.
-    if name in ("SSDModel", "bf16_bits_to_device"):
+    if name in ("SSDModel", "bf16_bits_to_device", "encdec_device_weights"):
         from . import model
         return getattr(model, name)
     raise AttributeError(name)

@@ -21,6 +21,33 @@ def bf16_bits_to_device(bits: np.ndarray, device="cuda") -> torch.Tensor:
     return t.to(device).view(torch.bfloat16)
 
 
+_ENCDEC_RENAME = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
+                  "ffn_norm": "ffn_norm"}
+
+
+def encdec_device_weights(bits: dict, device="cuda") -> dict:
+    """Upload an encoder-decoder model given as bf16 bit arrays in T5 naming -- {"embed", "lm_head",
+    "enc_final", "dec_final", "enc_rel", "dec_rel", "enc": [{wq, wk, wv, wo, attn_norm, wi0, wi1, wff,
+    ffn_norm}], "dec": [{... + self_norm, cq, ck, cv, co, cross_norm}], optional "in_norm", "in_w1",
+    "in_w2"} -- into the weights dict SSDModel takes for SSD_ARCH_T5."""
+    up = lambda a: bf16_bits_to_device(a, device)
+
+    def stack(lw, norm):
+        d = {_ENCDEC_RENAME[n]: up(a) for n, a in lw.items() if n in _ENCDEC_RENAME}
+        d["attn_norm"] = up(lw[norm])
+        return d
+
+    out = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
+           "layers": [stack(lw, "self_norm") for lw in bits["dec"]],
+           "encdec": {"cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
+                      "enc": [stack(lw, "attn_norm") for lw in bits["enc"]], "enc_final": up(bits["enc_final"]),
+                      "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}}
+    for k in ("in_norm", "in_w1", "in_w2"):
+        if k in bits:
+            out[k] = up(bits[k])
+    return out
+
+
 class _DeviceArray:
     """Minimal __cuda_array_interface__ holder to view library-owned memory from torch."""
 

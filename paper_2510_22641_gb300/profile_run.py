@@ -112,20 +112,7 @@ def encdec(args, lib, synth, torch) -> None:
     lib.build()
     bits = synth.make_t5_weights(w)
     up = lib.bf16_bits_to_device
-    ren = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
-           "ffn_norm": "ffn_norm"}
-
-    def stack(lw, norm):
-        d = {ren[n]: up(a) for n, a in lw.items() if n in ren}
-        d["attn_norm"] = up(lw[norm])
-        return d
-
-    dev = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
-           "layers": [stack(lw, "self_norm") for lw in bits["dec"]],
-           "in_norm": up(bits["in_norm"]), "in_w1": up(bits["in_w1"]), "in_w2": up(bits["in_w2"]),
-           "encdec": {"cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
-                      "enc": [stack(lw, "attn_norm") for lw in bits["enc"]], "enc_final": up(bits["enc_final"]),
-                      "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}}
+    dev = lib.encdec_device_weights(bits)
     cfg = lib.t5_config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
                              w.max_new + lib.SSD_MAX_GAMMA + 2, w.enc_len)
     model = lib.SSDModel(cfg, dev, torch.tensor(w.dec_scale(), device="cuda"),

@@ -38,29 +38,9 @@ def device_inputs(w: synth.Workload, seed: int | None = None):
     return vis, prompt, v, p
 
 
-_T5_RENAME = {"wq": "wq", "wk": "wk", "wv": "wv", "wo": "wo", "wi0": "w_gate", "wi1": "w_up", "wff": "w_down",
-              "ffn_norm": "ffn_norm"}
-
-
 def t5_device_weights(bits: dict) -> dict:
     """Device copies of a synth encoder-decoder workload in the layout lib.SSDModel takes."""
-    up = lib.bf16_bits_to_device
-
-    def stack(lw, norm):
-        d = {_T5_RENAME[n]: up(a) for n, a in lw.items() if n in _T5_RENAME}
-        d["attn_norm"] = up(lw[norm])
-        return d
-
-    out = {"embed": up(bits["embed"]), "lm_head": up(bits["lm_head"]), "final_norm": up(bits["dec_final"]),
-           "layers": [stack(lw, "self_norm") for lw in bits["dec"]]}
-    out["encdec"] = {
-        "cross": [{n: up(lw[n]) for n in ("cq", "ck", "cv", "co", "cross_norm")} for lw in bits["dec"]],
-        "enc": [stack(lw, "attn_norm") for lw in bits["enc"]],
-        "enc_final": up(bits["enc_final"]), "enc_rel": up(bits["enc_rel"]), "dec_rel": up(bits["dec_rel"])}
-    for k in ("in_norm", "in_w1", "in_w2"):
-        if k in bits:
-            out[k] = up(bits[k])
-    return out
+    return lib.encdec_device_weights(bits)
 
 
 def make_t5_model(w: synth.T5Workload, bits: dict | None = None, dev: dict | None = None,
