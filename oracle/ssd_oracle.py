@@ -47,6 +47,10 @@ tokens of context (so t = kv_len + 2 at a step whose last emitted token y sits a
 position kv_len) and N is the longest sequence the model is run with; each step
 drafts min(d(t), gamma_cap, remaining - 1) tokens.
 
+Batches of requests (the serving form): ssd_generate_batch runs Algorithm 1 on
+independent requests with ragged prompts in lockstep; each request keeps its own
+cache, positions and accept lengths, so batching changes no request's result.
+
 Decode rows are always processed one at a time by the same function, so a
 row's result does not depend on how many rows a step holds: SSD and greedy
 decoding agree bitwise here, not only up to rounding.
@@ -296,6 +300,75 @@ def greedy_generate(m: Model, vis: np.ndarray, prompt, max_new: int, max_seq: in
     return Result(tokens=tokens, logits=logits, kv_len=pos, cache=cache if keep_cache else None)
 
 
+class _SSDRun:
+    """One request under Algorithm 1: the prefill at construction, then one draft + verify + accept
+    step per call to step() (see ssd_generate)."""
+
+    def __init__(self, m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int, max_seq: int | None,
+                 reuse_draft_rows: bool, keep_draft_logits: bool, dynamic: tuple[int, int] | None):
+        c = m.cfg
+        self.m, self.max_new, self.gamma = m, max_new, gamma
+        self.reuse, self.keep_dlog, self.dynamic = reuse_draft_rows, keep_draft_logits, dynamic
+        P = vis.shape[0] + len(prompt)
+        self.cache = KVCache(c, max_seq or (P + max_new + gamma + 1))
+        t0 = time.perf_counter()
+        o = prefill(m, self.cache, vis, prompt)
+        self.y = argmax_lowest(o)
+        self.res = Result(tokens=[self.y], logits=[o], kv_len=P, prefill_s=time.perf_counter() - t0)
+        self.p, self.done = P, (c.eos_id >= 0 and self.y == c.eos_id)
+
+    @property
+    def finished(self) -> bool:
+        return self.done or len(self.res.tokens) >= self.max_new
+
+    def gamma_eff(self) -> int:
+        """Drafts of the next step: min(gamma or d(t), remaining - 1)."""
+        remaining = self.max_new - len(self.res.tokens)
+        g_step = self.gamma if self.dynamic is None else min(self.gamma, draft_length(self.p + 2, *self.dynamic))
+        return min(g_step, remaining - 1)
+
+    def step(self) -> None:
+        m, c, res = self.m, self.m.cfg, self.res
+        k, L, p, cache = c.draft_exit_k, c.n_layers, self.p, self.cache
+        t0 = time.perf_counter()
+        g_eff = self.gamma_eff()
+        toks, xk, dlog = [self.y], [], []
+        for j in range(g_eff):                                   # drafting stage
+            x = forward_row(m, embed(m, toks[j]), p + j, cache, range(k))
+            xk.append(x)
+            od = lm_head(m, imitation(m, x, p + j, cache))
+            dlog.append(od)
+            toks.append(argmax_lowest(od))
+        f, flog = [], []
+        for i in range(g_eff + 1):                               # verification stage
+            if self.reuse and i < g_eff:
+                x = xk[i]
+            else:
+                x = forward_row(m, embed(m, toks[i]), p + i, cache, range(k))
+                if c.in_kind == IN_BLOCK:                        # the block's K/V of this row's x_k
+                    block_kv(m, x, p + i, cache)
+            x = forward_row(m, x, p + i, cache, range(k, L))
+            of = lm_head(m, x)
+            flog.append(of)
+            f.append(argmax_lowest(of))
+        a = 0                                                    # acceptance
+        while a < g_eff and toks[a + 1] == f[a]:
+            a += 1
+        emitted = toks[1:a + 1] + [f[a]]
+        emitted, self.done = _truncate_eos(emitted, c.eos_id)
+        res.tokens += emitted
+        res.logits += flog[:len(emitted)]
+        res.accept_lengths.append(a)
+        res.draft_tokens.append(toks[1:])
+        if self.keep_dlog:
+            res.draft_logits.append(dlog)
+        self.p = p + a + 1
+        self.y = f[a]
+        res.kv_lens.append(self.p)
+        res.kv_len = self.p
+        res.step_s.append(time.perf_counter() - t0)
+
+
 def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                  max_seq: int | None = None, reuse_draft_rows: bool = True,
                  keep_cache: bool = False, keep_draft_logits: bool = False,
@@ -313,58 +386,40 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
     dynamic = (d0, N): each step drafts min(d(t), gamma, remaining - 1) tokens with
     t = kv_len + 2 (Sec. "Choice of d"); gamma is then the cap.
     """
-    c = m.cfg
-    k, L = c.draft_exit_k, c.n_layers
-    P = vis.shape[0] + len(prompt)
-    cache = KVCache(c, max_seq or (P + max_new + gamma + 1))
-    t0 = time.perf_counter()
-    o = prefill(m, cache, vis, prompt)
-    y = argmax_lowest(o)
-    res = Result(tokens=[y], logits=[o], kv_len=P, prefill_s=time.perf_counter() - t0)
-    p, done = P, (c.eos_id >= 0 and y == c.eos_id)
-    while len(res.tokens) < max_new and not done and (max_steps is None or len(res.step_s) < max_steps):
-        t0 = time.perf_counter()
-        remaining = max_new - len(res.tokens)
-        g_step = gamma if dynamic is None else min(gamma, draft_length(p + 2, dynamic[0], dynamic[1]))
-        g_eff = min(g_step, remaining - 1)
-        toks, xk, dlog = [y], [], []
-        for j in range(g_eff):                                   # drafting stage
-            x = forward_row(m, embed(m, toks[j]), p + j, cache, range(k))
-            xk.append(x)
-            od = lm_head(m, imitation(m, x, p + j, cache))
-            dlog.append(od)
-            toks.append(argmax_lowest(od))
-        f, flog = [], []
-        for i in range(g_eff + 1):                               # verification stage
-            if reuse_draft_rows and i < g_eff:
-                x = xk[i]
-            else:
-                x = forward_row(m, embed(m, toks[i]), p + i, cache, range(k))
-                if c.in_kind == IN_BLOCK:                        # the block's K/V of this row's x_k
-                    block_kv(m, x, p + i, cache)
-            x = forward_row(m, x, p + i, cache, range(k, L))
-            of = lm_head(m, x)
-            flog.append(of)
-            f.append(argmax_lowest(of))
-        a = 0                                                    # acceptance
-        while a < g_eff and toks[a + 1] == f[a]:
-            a += 1
-        emitted = toks[1:a + 1] + [f[a]]
-        emitted, done = _truncate_eos(emitted, c.eos_id)
-        res.tokens += emitted
-        res.logits += flog[:len(emitted)]
-        res.accept_lengths.append(a)
-        res.draft_tokens.append(toks[1:])
-        if keep_draft_logits:
-            res.draft_logits.append(dlog)
-        p += a + 1
-        y = f[a]
-        res.kv_lens.append(p)
-        res.step_s.append(time.perf_counter() - t0)
-    res.kv_len = p
+    run = _SSDRun(m, vis, prompt, max_new, gamma, max_seq, reuse_draft_rows, keep_draft_logits, dynamic)
+    while not run.finished and (max_steps is None or len(run.res.step_s) < max_steps):
+        run.step()
     if keep_cache:
-        res.cache = cache
-    return res
+        run.res.cache = run.cache
+    return run.res
+
+
+@dataclasses.dataclass
+class BatchResult:
+    results: list    # per request: Result
+    active: list     # per batched step: indices of the requests that stepped
+    rows: list       # per batched step: verification rows, the sum of gamma_eff + 1 over the active requests
+
+
+def ssd_generate_batch(m: Model, requests, max_new: int, gamma: int, max_seq: int | None = None) -> BatchResult:
+    """Algorithm 1 on a batch of independent requests in lockstep (the serving form of the method).
+
+    requests: list of (vis, prompt) with prompts of different lengths (ragged).  Each request has its
+    own cache, kv_len and accept lengths; in every batched step each unfinished request drafts
+    gamma_eff = min(gamma, remaining - 1) tokens at its own positions, the verification covers the
+    rows of all active requests at once, and each request accepts and rolls back on its own.  A
+    finished request (max_new tokens out, or eos) takes no further rows.  Every request's tokens,
+    logits and accept lengths are those of ssd_generate on it alone.
+    """
+    runs = [_SSDRun(m, vis, prompt, max_new, gamma, max_seq, True, False, None) for vis, prompt in requests]
+    out = BatchResult(results=[r.res for r in runs], active=[], rows=[])
+    while not all(r.finished for r in runs):
+        act = [b for b, r in enumerate(runs) if not r.finished]
+        out.rows.append(sum(runs[b].gamma_eff() + 1 for b in act))
+        out.active.append(act)
+        for b in act:
+            runs[b].step()
+    return out
 
 
 # --------------------------------------------------------------------------- construction helpers

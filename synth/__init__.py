@@ -185,6 +185,37 @@ LLAVA7B = Workload(name="llava15_7b_shape", shape=LLAVA7B_SHAPE, draft_exit_k=8,
 
 LLAVA7B_S_VALUES = (0.05, 0.2, 1.0)
 
+# LLaVA-1.5-13B-shaped decoder: 576 visual rows + up to 256 prompt ids, k=10, gamma=6, 256 new tokens.
+LLAVA13B = Workload(name="llava15_13b_shape", shape=LLAVA13B_SHAPE, draft_exit_k=10, in_kind=IN_MLP2,
+                    in_hidden=5120, gamma=6, n_vis=576, n_prompt=256, max_new=256, s=0.2)
+
+
+@dataclasses.dataclass(frozen=True)
+class BatchWorkload:
+    """A batch of independent requests on one model (the serving form of the method): every request
+    has the base workload's visual rows and a prompt of length U[prompt_min, prompt_max] (ragged)."""
+    base: Workload
+    batch: int
+    prompt_min: int
+    prompt_max: int
+
+    def replace(self, **kw) -> "BatchWorkload":
+        return dataclasses.replace(self, **kw)
+
+    def prompt_lengths(self, seed: int | None = None) -> np.ndarray:
+        seed = self.base.input_seed if seed is None else seed
+        return uniform_i32(seed, stream_id("prompt_len"), (self.batch,), self.prompt_min, self.prompt_max + 1)
+
+    def max_seq(self) -> int:
+        b = self.base
+        return b.n_vis + self.prompt_max + b.max_new + b.gamma + 1
+
+
+# configs[4]: 16 requests on the 13B shape, prompts U[32, 256] after the 576 visual rows, s = 0.2.
+LLAVA13B_B16 = BatchWorkload(base=LLAVA13B, batch=16, prompt_min=32, prompt_max=256)
+# Its tiny stand-in for parity: 4 requests on the tiny model, prompts U[4, 24].
+TINY_B4 = BatchWorkload(base=TINY, batch=4, prompt_min=4, prompt_max=24)
+
 
 # --------------------------------------------------------------------------- weights and inputs
 
@@ -193,7 +224,7 @@ _KIND = {
     "wq": 10, "wk": 11, "wv": 12, "wo": 13, "w_gate": 14, "w_up": 15, "w_down": 16,
     "attn_norm": 17, "ffn_norm": 18,
     "in_norm": 20, "in_w1": 21, "in_w2": 22,
-    "vis": 40, "prompt": 41,
+    "vis": 40, "prompt": 41, "prompt_len": 42,
 }
 
 
@@ -421,3 +452,16 @@ def make_t5_inputs(w: T5Workload, seed: int | None = None) -> tuple[np.ndarray, 
     q = normal_bf16(seed, t5_stream_id("query"), (w.n_query, w.shape.d_model), std=w.vis_std)
     prompt = uniform_i32(seed, t5_stream_id("t5_prompt"), (w.n_prompt,), 0, w.shape.vocab)
     return q, prompt
+
+
+def make_batch_inputs(bw: BatchWorkload, seed: int | None = None) -> list:
+    """Per request b: synthetic encoder output (bf16 bits [n_vis][d], N(0, vis_std)) and prompt ids
+    U[0, V) of the request's ragged length; request b draws from streams of its own (layer field b + 1)."""
+    seed = bw.base.input_seed if seed is None else seed
+    w = bw.base
+    out = []
+    for b, n in enumerate(bw.prompt_lengths(seed)):
+        vis = normal_bf16(seed, stream_id("vis", b + 1), (w.n_vis, w.shape.d_model), std=w.vis_std)
+        prompt = uniform_i32(seed, stream_id("prompt", b + 1), (int(n),), 0, w.shape.vocab)
+        out.append((vis, prompt))
+    return out

@@ -382,3 +382,42 @@ def test_in_block_ssd_equals_greedy_and_block_cache_matches(s, gamma, k):
     L = m.cfg.n_layers
     np.testing.assert_allclose(r.cache.k[L, :, :n], K.transpose(1, 0, 2)[:, :n], rtol=1e-9, atol=1e-9)
     np.testing.assert_allclose(r.cache.v[L, :, :n], V.transpose(1, 0, 2)[:, :n], rtol=1e-9, atol=1e-9)
+
+
+# --------------------------------------------------------------------------- batch of ragged requests
+
+def test_batch_prompt_lengths_are_ragged_and_in_range():
+    for bw in (synth.LLAVA13B_B16, synth.TINY_B4):
+        n = bw.prompt_lengths()
+        assert len(n) == bw.batch and n.min() >= bw.prompt_min and n.max() <= bw.prompt_max
+        assert len(set(n.tolist())) > 1
+    ins = synth.make_batch_inputs(synth.TINY_B4)
+    assert [len(p) for _, p in ins] == synth.TINY_B4.prompt_lengths().tolist()
+    assert not np.array_equal(ins[0][0], ins[1][0])      # every request has its own visual rows
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.3, 6), (1.0, 2)])
+def test_batch_ssd_equals_each_request_alone_and_greedy(tiny_bits, s, gamma):
+    """Lockstep batching changes no request's result: tokens, logits, accept lengths and kv_len equal
+    ssd_generate on the request alone and its greedy decoding; positions start at the request's own P;
+    the batch runs as many steps as its slowest request, each request's rows summing its gamma_eff + 1."""
+    bw = synth.TINY_B4.replace(base=tiny(s=s, gamma=gamma, max_new=20))
+    m, _, _ = build(bw.base, tiny_bits)
+    reqs = [(synth.bf16_to_f64(v), p) for v, p in synth.make_batch_inputs(bw)]
+    br = oracle.ssd_generate_batch(m, reqs, bw.base.max_new, gamma)
+    assert len(br.results) == bw.batch
+    for b, ((vis, prompt), r) in enumerate(zip(reqs, br.results)):
+        alone = oracle.ssd_generate(m, vis, prompt, bw.base.max_new, gamma)
+        greedy = oracle.greedy_generate(m, vis, prompt, bw.base.max_new)
+        assert r.tokens == alone.tokens == greedy.tokens
+        assert r.accept_lengths == alone.accept_lengths and r.kv_lens == alone.kv_lens
+        for a, g in zip(r.logits, greedy.logits):
+            np.testing.assert_array_equal(a, g)
+        P = vis.shape[0] + len(prompt)
+        assert r.kv_lens[0] == P + r.accept_lengths[0] + 1 and r.kv_len == P + bw.base.max_new - 1
+        assert sum(1 for act in br.active if b in act) == len(r.accept_lengths)
+    assert len(br.active) == max(len(r.accept_lengths) for r in br.results)
+    # rows per batched step: each active request's drafted tokens + 1
+    for t, act in enumerate(br.active):
+        drafted = sum(len(br.results[b].draft_tokens[sum(1 for u in br.active[:t] if b in u)]) for b in act)
+        assert br.rows[t] == drafted + len(act)
