@@ -217,6 +217,19 @@ def oracle_sample(w: synth.Workload, bits, vis, prompt, max_steps: int, warm_ste
             "cores": os.cpu_count()}
 
 
+def oracle_sample_encdec(w: synth.T5Workload, bits, query, prompt, max_steps: int) -> dict:
+    """Time the fp64 encoder-decoder oracle: its encoder + first decoder step and `max_steps` SSD steps."""
+    from oracle import t5_oracle
+    m = t5_oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    r = t5_oracle.ssd_generate(m, synth.bf16_to_f64(query), prompt, w.max_new, w.gamma, max_steps=max_steps)
+    acc = r.accept_lengths
+    toks_per_step = (sum(acc) + len(acc)) / max(len(acc), 1)
+    step_mean = sum(r.step_s) / max(len(r.step_s), 1)
+    return {"decode_tok_s": toks_per_step / step_mean if step_mean > 0 else None, "prefill_s": r.prefill_s,
+            "step_s": step_mean, "tokens_per_step": toks_per_step, "n_steps": len(r.step_s),
+            "cores": os.cpu_count()}
+
+
 def run_reference(args) -> None:
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -382,12 +395,20 @@ def run_encdec(args) -> None:
                      "draft_ms": d_ms, "draft_gbs": d_gbs, "greedy_gbs": g_gbs,
                      "draft_frac": d_gbs / peak if peak else None, "greedy_frac": g_gbs / peak if peak else None})
     model.close()
+    cpu = None
+    if not args.no_cpu_baseline:
+        r = oracle_sample_encdec(w, bits, q, prompt, max_steps=args.cpu_steps)
+        cpu = {"value": r["decode_tok_s"], "unit": UNIT, "cores": r["cores"], "kind": "oracle",
+               "sample": f"fp64 numpy encoder-decoder oracle at s = {w.s}: encoder + first decoder step "
+                         f"({r['prefill_s']:.1f} s) and {r['n_steps']} SSD steps ({r['step_s']:.2f} s each, "
+                         f"{r['tokens_per_step']:.2f} tokens/step); value = decode tokens/s"}
     print(json.dumps({"workload": f"{w.name}: {sh.n_enc}+{sh.n_dec} layers, d={sh.d_model}, {sh.n_heads}x"
                                   f"{sh.head_dim} heads, gated-GELU {sh.d_ff}, V={sh.vocab}; {w.n_query} queries + "
                                   f"{w.n_prompt} prompt ids; k={w.draft_exit_k}, gamma={w.gamma}, "
                                   f"{w.max_new} new tokens; bs1",
                       "prefill_ms": prefill_ms, "peak_hbm_gbs": peak, "bytes_per_token":
-                          {"draft": draft_bytes, "greedy": greedy_bytes}, "per_s": rows, "kernels": kernels}),
+                          {"draft": draft_bytes, "greedy": greedy_bytes}, "per_s": rows, "kernels": kernels,
+                      "cpu_baseline": cpu}),
           flush=True)
 
 

@@ -33,6 +33,7 @@ from __future__ import annotations
 
 import dataclasses
 import math
+import time
 
 import numpy as np
 
@@ -227,6 +228,8 @@ class T5Result:
     accept_lengths: list = dataclasses.field(default_factory=list)
     kv_lens: list = dataclasses.field(default_factory=list)
     draft_tokens: list = dataclasses.field(default_factory=list)
+    prefill_s: float = 0.0                                  # wall time of the encoder + first decoder step
+    step_s: list = dataclasses.field(default_factory=list)  # wall time per SSD step
 
 
 def _first(m: T5Model, z, prompt, max_seq: int):
@@ -260,11 +263,13 @@ def ssd_generate(m: T5Model, z: np.ndarray, prompt, max_new: int, gamma: int,
     max_steps: stop after that many draft + verify steps (a sampled prefix of a long run)."""
     c = m.cfg
     k, L = c.draft_exit_k, c.n_dec
+    t0 = time.perf_counter()
     cache, o = _first(m, z, prompt, max_new + gamma + 1)
     y = argmax_lowest(o)
-    res = T5Result(tokens=[y], logits=[o], kv_len=1)
+    res = T5Result(tokens=[y], logits=[o], kv_len=1, prefill_s=time.perf_counter() - t0)
     p, done = 1, (c.eos_id >= 0 and y == c.eos_id)
     while len(res.tokens) < max_new and not done and (max_steps is None or len(res.accept_lengths) < max_steps):
+        t0 = time.perf_counter()
         g_eff = min(gamma, max_new - len(res.tokens) - 1)
         toks, xk = [y], []
         for j in range(g_eff):                                   # drafting stage
@@ -292,6 +297,7 @@ def ssd_generate(m: T5Model, z: np.ndarray, prompt, max_new: int, gamma: int,
         p += a + 1
         y = f[a]
         res.kv_lens.append(p)
+        res.step_s.append(time.perf_counter() - t0)
     res.kv_len = p
     return res
 

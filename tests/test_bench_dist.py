@@ -41,3 +41,15 @@ def test_replicas_take_the_slowest_rank_and_count_all_tokens():
 def test_single_process_needs_no_process_group():
     assert bench.reduce_max(12.5) == 12.5
     assert bench.whole_job_tokens_per_s(1, 10, 128, 2000.0) == pytest.approx(640.0)
+
+
+def test_encoder_decoder_oracle_sample_on_the_tiny_model():
+    """bench.py --encdec's CPU leg: the encoder-decoder oracle timed over a bounded number of steps."""
+    import synth
+    w = synth.T5_TINY.replace(s=0.3)
+    bits = synth.make_t5_weights(w)
+    q, prompt = synth.make_t5_inputs(w)
+    r = bench.oracle_sample_encdec(w, bits, q, prompt, max_steps=3)
+    assert r["n_steps"] == 3 and r["prefill_s"] > 0 and r["step_s"] > 0
+    assert 1.0 <= r["tokens_per_step"] <= w.gamma + 1
+    assert r["decode_tok_s"] == pytest.approx(r["tokens_per_step"] / r["step_s"])
