@@ -1,8 +1,8 @@
 """Plain fp64 CPU oracle for greedy self-speculative decoding on an encoder-decoder VLM
 (the BLIP-2 + FlanT5-xl setting of Sec. "Experiments"; FastVLM, arXiv 2510.22641).
 
-TEST INFRASTRUCTURE ONLY.  Only ``tests/`` (and, later, ``bench.py``'s CPU baseline) may
-import or run this module.  It shares no code with any CUDA path; its inputs come from
+TEST INFRASTRUCTURE ONLY.  Only ``tests/`` and the ``cpu_baseline`` leg of ``bench.py --encdec``
+may import or run this module.  It shares no code with any CUDA path; its inputs come from
 ``synth`` (seeded generators).
 
 What it computes:
@@ -36,6 +36,8 @@ import math
 import time
 
 import numpy as np
+
+from .ssd_oracle import draft_length
 
 IN_IDENTITY = 0
 IN_MLP2 = 1
@@ -258,9 +260,12 @@ def greedy_generate(m: T5Model, z: np.ndarray, prompt, max_new: int) -> T5Result
 
 
 def ssd_generate(m: T5Model, z: np.ndarray, prompt, max_new: int, gamma: int,
-                 reuse_draft_rows: bool = True, max_steps: int | None = None) -> T5Result:
+                 reuse_draft_rows: bool = True, max_steps: int | None = None,
+                 dynamic: tuple[int, int] | None = None) -> T5Result:
     """Algorithm 1 on the decoder (see the module docstring); kv_len counts decoder positions.
-    max_steps: stop after that many draft + verify steps (a sampled prefix of a long run)."""
+    max_steps: stop after that many draft + verify steps (a sampled prefix of a long run).
+    dynamic = (d0, N): each step drafts min(d(t), gamma, remaining - 1) tokens with t = kv_len + 2
+    (Sec. "Choice of d", the decoder-only oracle's draft_length); gamma is then the cap."""
     c = m.cfg
     k, L = c.draft_exit_k, c.n_dec
     t0 = time.perf_counter()
@@ -270,7 +275,8 @@ def ssd_generate(m: T5Model, z: np.ndarray, prompt, max_new: int, gamma: int,
     p, done = 1, (c.eos_id >= 0 and y == c.eos_id)
     while len(res.tokens) < max_new and not done and (max_steps is None or len(res.accept_lengths) < max_steps):
         t0 = time.perf_counter()
-        g_eff = min(gamma, max_new - len(res.tokens) - 1)
+        g_step = gamma if dynamic is None else min(gamma, draft_length(p + 2, dynamic[0], dynamic[1]))
+        g_eff = min(g_step, max_new - len(res.tokens) - 1)
         toks, xk = [y], []
         for j in range(g_eff):                                   # drafting stage
             x = dec_forward_row(m, m.w["embed"][toks[j]].copy(), p + j, cache, range(k))

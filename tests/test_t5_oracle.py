@@ -247,3 +247,19 @@ def test_torch_forward_catches(monkeypatch, name, tiny_model):
     for pos, y in enumerate([m.cfg.start_token] + toks):
         got.append(T.lm_head(m, T.dec_forward_row(m, m.w["embed"][y].copy(), pos, cache, range(m.cfg.n_dec))))
     assert not np.allclose(np.stack(got), ref, rtol=1e-6, atol=1e-6)
+
+
+@pytest.mark.parametrize("s,cap,n_max", [(0.05, 8, 60), (0.3, 6, 200)])
+def test_ssd_dynamic_draft_length_equals_greedy(s, cap, n_max):
+    """Sec. "Choice of d" on the decoder: each step drafts min(d(kv_len + 2), cap, remaining - 1) tokens
+    and the output is still greedy decoding."""
+    w = tiny(s=s, max_new=40)
+    m, z, prompt = build(w)
+    r = T.ssd_generate(m, z, prompt, w.max_new, cap, dynamic=(5, n_max))
+    assert r.tokens == T.greedy_generate(m, z, prompt, w.max_new).tokens
+    p, n = 1, 1
+    for step, a in enumerate(r.accept_lengths):
+        g = min(cap, 5 + int(np.floor(10.0 / (1.0 + np.exp(-0.01 * ((p + 2) - n_max / 2.0))))), w.max_new - n - 1)
+        assert len(r.draft_tokens[step]) == g and 0 <= a <= g
+        p += a + 1
+        n += a + 1
