@@ -71,6 +71,8 @@ class T5Model:
     """
 
     def __init__(self, cfg: T5Config, w: dict, dec_scale, in_scale: float):
+        if cfg.rel_buckets < 4 or cfg.rel_buckets % 2 or cfg.rel_max_distance <= cfg.rel_buckets // 2:
+            raise ValueError("rel_buckets must be even and >= 4, rel_max_distance > rel_buckets / 2")
         self.cfg = cfg
         self.w = w
         self.s = [float(v) for v in dec_scale]

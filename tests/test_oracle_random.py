@@ -85,7 +85,7 @@ def t5_case(draw):
                 ff=draw(st.sampled_from([8, 24])), V=draw(st.sampled_from([16, 41])), k=draw(st.integers(1, n_dec)),
                 in_kind=draw(st.sampled_from([T.IN_IDENTITY, T.IN_MLP2])), gamma=draw(st.integers(1, 4)),
                 s=draw(st.sampled_from([0.05, 0.3, 1.0])), buckets=draw(st.sampled_from([8, 32])),
-                maxd=draw(st.sampled_from([12, 128])), n_q=draw(st.integers(1, 6)), n_p=draw(st.integers(0, 5)),
+                maxd=draw(st.sampled_from([20, 128])), n_q=draw(st.integers(1, 6)), n_p=draw(st.integers(0, 5)),
                 seed=draw(st.integers(0, 2 ** 20)))
 
 
