@@ -255,7 +255,7 @@ def run_reference(args) -> None:
 # --------------------------------------------------------------------------- GPU arm
 
 def run_in_block(args) -> None:
-    """The configs[1] workload (7B shape, k = 8, gamma = 5, 128 new tokens) with the imitation module
+    """The LLaVA-1.5-7B-shaped workload (k = 8, gamma = 5, 128 new tokens) with the imitation module
     read as one decoder block with its own KV cache (IN_BLOCK): decode tokens/s of SSD and greedy,
     speedup, accept length and the drafting stage's HBM GB/s, per s.  One JSON line."""
     import torch

@@ -211,7 +211,7 @@ class BatchWorkload:
         return b.n_vis + self.prompt_max + b.max_new + b.gamma + 1
 
 
-# configs[4]: 16 requests on the 13B shape, prompts U[32, 256] after the 576 visual rows, s = 0.2.
+# 16 requests on the 13B shape, prompts U[32, 256] after the 576 visual rows, s = 0.2.
 LLAVA13B_B16 = BatchWorkload(base=LLAVA13B, batch=16, prompt_min=32, prompt_max=256)
 # Its tiny stand-in for parity: 4 requests on the tiny model, prompts U[4, 24].
 TINY_B4 = BatchWorkload(base=TINY, batch=4, prompt_min=4, prompt_max=24)
