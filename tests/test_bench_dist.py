@@ -53,3 +53,16 @@ def test_encoder_decoder_oracle_sample_on_the_tiny_model():
     assert r["n_steps"] == 3 and r["prefill_s"] > 0 and r["step_s"] > 0
     assert 1.0 <= r["tokens_per_step"] <= w.gamma + 1
     assert r["decode_tok_s"] == pytest.approx(r["tokens_per_step"] / r["step_s"])
+
+
+def test_decoder_oracle_sample_on_the_tiny_model():
+    """bench.py's cpu_baseline / --impl reference leg: prefill plus bounded SSD steps of the oracle."""
+    import synth
+    w = synth.TINY.replace(s=0.3)
+    bits = synth.make_weights(w)
+    vis, prompt = synth.make_inputs(w)
+    r = bench.oracle_sample(w, bits, vis, prompt, max_steps=3, warm_steps=1)
+    assert r["n_steps"] == 3 and r["prefill_s"] > 0 and r["step_s"] > 0
+    assert 1.0 <= r["tokens_per_step"] <= w.gamma + 1
+    request_s = r["prefill_s"] + (w.max_new - 1) / r["tokens_per_step"] * r["step_s"]
+    assert r["value"] == pytest.approx(w.max_new / request_s)
