@@ -1,8 +1,9 @@
 """Planted mistakes in the oracle (on the CPU) must be caught by its pins.
 
 Each case monkeypatches one oracle building block with a plausible bug (a
-wrong sign, a dropped term, an off-by-one, a transposed operand) and checks
-that the independent torch forward or an Algorithm 1 property disagrees.
+wrong sign, a dropped term, an off-by-one, a transposed operand, a skipped
+cache write, a shared cache, a missing norm) and checks that the independent
+torch forward or an Algorithm 1 property disagrees.
 """
 import numpy as np
 import pytest
@@ -77,3 +78,52 @@ def test_accept_rule_off_by_one_is_caught(monkeypatch):
     monkeypatch.setattr(so, "argmax_lowest", lying_argmax)
     r = so.ssd_generate(m, vis, prompt, w.max_new, w.gamma)
     assert r.tokens != g.tokens
+
+
+# --------------------------------------------------------------------------- newer features
+
+def test_in_block_catch_up_row_skipped_is_caught(monkeypatch):
+    """Dropping the verification pass's catch-up (the block's cache row of d_gamma's x_k) leaves stale
+    block rows that the no-cache torch forward of the block exposes."""
+    from tests.test_oracle import torch_block_rows
+    w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=1.0, gamma=4)
+    m, vis, prompt = build(w)
+    monkeypatch.setattr(so, "block_kv", lambda *a, **k: None)
+    r = so.ssd_generate(m, vis, prompt, w.max_new, w.gamma, keep_cache=True)
+    _, K, _, _ = torch_block_rows(m, vis, list(prompt) + r.tokens[:-1])
+    n, L = r.kv_len, m.cfg.n_layers
+    assert not np.allclose(r.cache.k[L, :, :n], K.transpose(1, 0, 2)[:, :n], rtol=1e-6, atol=1e-6)
+
+
+def test_batch_sharing_one_cache_is_caught(monkeypatch):
+    """Requests that share one KV cache (a missing per-request cache) no longer reproduce their runs alone."""
+    w = tiny(s=0.3, max_new=12)
+    m, _, _ = build(w)
+    bw = synth.TINY_B4.replace(base=w)
+    reqs = [(synth.bf16_to_f64(v), p) for v, p in synth.make_batch_inputs(bw)]
+    alone = [so.ssd_generate(m, v, p, w.max_new, w.gamma) for v, p in reqs]
+    shared = so.KVCache(m.cfg, bw.max_seq())
+    monkeypatch.setattr(so, "KVCache", lambda cfg, max_seq: shared)
+    br = so.ssd_generate_batch(m, reqs, w.max_new, w.gamma)
+    assert any(b.logits[-1].tolist() != a.logits[-1].tolist() for a, b in zip(alone, br.results))
+
+
+def test_encoder_decoder_cross_cache_from_unnormed_output_is_caught(monkeypatch):
+    """Cross-attention K/V taken from the encoder's residual stream instead of its normed output fails
+    the torch forward."""
+    from oracle import t5_oracle as T
+    from tests.test_t5_oracle import build as t5_build, tiny as t5_tiny, torch_forward
+    m, z, prompt = t5_build(t5_tiny())
+    toks = [5, 9, 2, 6, 5, 3]
+    ref = torch_forward(m, z, prompt, toks)
+    orig = T.rms_norm
+
+    def skip_final_norm(x, gain, eps):       # the encoder's final norm is its last rms_norm call on [P][d]
+        if x.ndim == 2 and gain is m.w["enc_final"]:
+            return x
+        return orig(x, gain, eps)
+    monkeypatch.setattr(T, "rms_norm", skip_final_norm)
+    cache = T.DecCache(m, T.encode(m, z, prompt), len(toks) + 1)
+    got = [T.lm_head(m, T.dec_forward_row(m, m.w["embed"][y].copy(), pos, cache, range(m.cfg.n_dec)))
+           for pos, y in enumerate([m.cfg.start_token] + toks)]
+    assert not np.allclose(np.stack(got), ref, rtol=1e-6, atol=1e-6)
