@@ -18,6 +18,10 @@ Printed as one JSON line (rank 0):
 
 --impl reference times that oracle itself (rank 0 only).
 Multi-GPU (torchrun): independent replicas, one request stream per GPU.
+
+Other workloads, one JSON line each: --sweep (k x gamma x s on the 7B shape), --in-block (the
+imitation module as one decoder block), --encdec (the BLIP-2 FlanT5-xl-shaped encoder-decoder:
+decode tokens/s per s, per-kernel table, encoder prefill, and its oracle on the host cores).
 """
 from __future__ import annotations
 
