@@ -19,6 +19,7 @@ Printed as one JSON line (rank 0):
 --impl reference times that oracle itself (rank 0 only).
 Multi-GPU (torchrun): independent replicas, one request stream per GPU.
 
+--profile PHASE opens a profiler window around one phase for ncu (no JSON line).
 Other workloads, one JSON line each: --sweep (k x gamma x s on the 7B shape), --in-block (the
 imitation module as one decoder block), --encdec (the BLIP-2 FlanT5-xl-shaped encoder-decoder:
 decode tokens/s per s, per-kernel table, encoder prefill, and its oracle on the host cores).
@@ -72,24 +73,24 @@ def algorithmic_bytes(w: synth.Workload) -> dict:
             "verify": sh.n_layers * layer + head, "greedy_token": sh.n_layers * layer + head}
 
 
-KERNEL_ROWS = (("qkv", "gemv_kernel<M, QKV> (q/k/v + RoPE + KV write)"),
-               ("o", "gemv_kernel<M, RESID> (o_proj)"),
-               ("gateup", "gemv_kernel<M, GATE_SILU> (gate/up)"),
-               ("down", "gemv_kernel<M, RESID> (down)"),
-               ("attn", "attn_kernel<M, 128> (split-KV, cache after prefill)"),
-               ("head", "gemv_kernel<M, ARGMAX> (LM head)"),
-               ("in1", "gemv_kernel<1, SILU> (imitation FC1)"),
-               ("in2", "gemv_kernel<1, RESID> (imitation FC2)"))
+KERNEL_ROWS = (("qkv", "ssd_wstream_kernel<M, QKV> (q/k/v + RoPE + KV write)"),
+               ("o", "ssd_wstream_kernel<M, RESID> (o_proj)"),
+               ("gateup", "ssd_wstream_kernel<M, GATE_SILU> (gate/up)"),
+               ("down", "ssd_wstream_kernel<M, RESID> (down)"),
+               ("attn", "ssd_splitkv_attn_kernel<M, 128> (split-KV, cache after prefill)"),
+               ("head", "ssd_wstream_kernel<M, ARGMAX> (LM head)"),
+               ("in1", "ssd_wstream_kernel<1, SILU> (imitation FC1)"),
+               ("in2", "ssd_wstream_kernel<1, RESID> (imitation FC2)"))
 
 
-ENCDEC_KERNEL_ROWS = (("qkv", "gemv_kernel<M, QKV> (self q/k/v + KV write, no RoPE)"),
-                      ("o", "gemv_kernel<M, RESID> (self o; cross q / cross o have this shape)"),
-                      ("gateup", "gemv_kernel<M, GATE_SILU> (wi_0/wi_1, gated GELU)"),
-                      ("down", "gemv_kernel<M, RESID> (wo of the MLP)"),
-                      ("attn", "attn_kernel<M, 64, EXT> (self-attention, relative-position bias)"),
-                      ("head", "gemv_kernel<M, ARGMAX> (LM head)"),
-                      ("in1", "gemv_kernel<1, SILU> (imitation FC1)"),
-                      ("in2", "gemv_kernel<1, RESID> (imitation FC2)"))
+ENCDEC_KERNEL_ROWS = (("qkv", "ssd_wstream_kernel<M, QKV> (self q/k/v + KV write, no RoPE)"),
+                      ("o", "ssd_wstream_kernel<M, RESID> (self o; cross q / cross o have this shape)"),
+                      ("gateup", "ssd_wstream_kernel<M, GATE_SILU> (wi_0/wi_1, gated GELU)"),
+                      ("down", "ssd_wstream_kernel<M, RESID> (wo of the MLP)"),
+                      ("attn", "ssd_splitkv_attn_kernel<M, 64, EXT> (self-attention, relative-position bias)"),
+                      ("head", "ssd_wstream_kernel<M, ARGMAX> (LM head)"),
+                      ("in1", "ssd_wstream_kernel<1, SILU> (imitation FC1)"),
+                      ("in2", "ssd_wstream_kernel<1, RESID> (imitation FC2)"))
 
 
 def kernel_table(model, w, v, p, stream, hbm_peak, reps=50, rows_table=KERNEL_ROWS, layer_sum=True):
@@ -499,6 +500,67 @@ def run_sweep(args) -> None:
         model.close()
 
 
+def run_profile(args) -> None:
+    """A profiler window around one phase (run under `ncu --profile-from-start off`): the 7B layer
+    shape with --layers layers (fewer layers keep a capture to a few GB on the device while every
+    weight matrix keeps its full size), or with --encdec the FlanT5-xl layer shape.  Decode phases
+    run the host-driven loop (SSD_OPT_HOST_LOOP), since profilers do not see kernels inside
+    conditional graph nodes.  Phases: greedy / ssd (--tokens new tokens), prefill, proj (reps
+    launches of one kernel alone: --proj qkv, o, gateup, down, head, in1, in2 or attn at --rows)."""
+    import torch
+
+    import paper_2510_22641_gb300 as lib
+
+    lib.build()
+    up = lib.bf16_bits_to_device
+    if args.encdec:
+        base = synth.FLANT5XL
+        shape = synth.T5Shape(args.layers, args.layers, 2048, 32, 64, 5120, 32128)
+        w = base.replace(shape=shape, draft_exit_k=min(base.draft_exit_k, args.layers), s=args.s)
+        bits = synth.make_t5_weights(w)
+        dev = lib.encdec_device_weights(bits)
+        cfg = lib.t5_config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                                 w.max_new + lib.SSD_MAX_GAMMA + 2, w.enc_len, options=lib.SSD_OPT_HOST_LOOP)
+        rs = torch.tensor(w.dec_scale(), device="cuda")
+        vis, prompt = synth.make_t5_inputs(w)
+    else:
+        base = synth.LLAVA7B
+        shape = synth.ModelShape(args.layers, 4096, 32, 128, 11008, 32000)
+        w = base.replace(shape=shape, draft_exit_k=min(base.draft_exit_k, args.layers), s=args.s)
+        bits = synth.make_weights(w)
+        dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm", "in_norm", "in_w1", "in_w2")}
+        dev["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+        cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
+                              w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1, options=lib.SSD_OPT_HOST_LOOP)
+        rs = torch.tensor(w.resid_scale(), device="cuda")
+        vis, prompt = synth.make_inputs(w)
+    model = lib.SSDModel(cfg, dev, rs, torch.tensor([w.in_scale()], device="cuda"))
+    v = up(vis)
+    p = torch.from_numpy(prompt.astype(np.int32)).cuda()
+    n = 1 + args.tokens
+
+    def phase():
+        if args.profile == "greedy":
+            model.greedy_decode(n)
+        elif args.profile == "ssd":
+            model.decode(n, w.gamma)
+        elif args.profile == "proj":
+            model.profile_projection(args.proj, 0, args.rows, 3)
+        else:
+            model.prefill(v, p)
+
+    model.prefill(v, p)
+    phase()                     # builds the graphs, warms up
+    model.prefill(v, p)
+    model.sync()
+    torch.cuda.profiler.start()
+    phase()
+    model.sync()
+    torch.cuda.profiler.stop()
+    print("profile done", args.profile, model.stats(), flush=True)
+    model.close()
+
+
 def main() -> None:
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -513,7 +575,18 @@ def main() -> None:
                     help="the 7B workload with the imitation module as one decoder block (one JSON line)")
     ap.add_argument("--encdec", action="store_true",
                     help="the BLIP-2 FlanT5-xl-shaped encoder-decoder workload (one JSON line)")
+    ap.add_argument("--profile", choices=["greedy", "ssd", "prefill", "proj"],
+                    help="a profiler window around one phase instead of the bench (see run_profile)")
+    ap.add_argument("--layers", type=int, default=32, help="--profile: layers of the model")
+    ap.add_argument("--tokens", type=int, default=4, help="--profile greedy/ssd: new tokens")
+    ap.add_argument("--proj", default="gateup", help="--profile proj: the kernel")
+    ap.add_argument("--rows", type=int, default=1, help="--profile proj: activation rows")
+    ap.add_argument("--host-loop", action="store_true",
+                    help="drive the decode loop from the host (same kernels and results; lets ncu list them)")
     args = ap.parse_args()
+    if args.profile:
+        run_profile(args)
+        return
     if args.encdec:
         run_encdec(args)
         return
@@ -550,7 +623,8 @@ def main() -> None:
     rs = torch.tensor(w.resid_scale(), device="cuda")
     ins = torch.tensor([w.in_scale()], device="cuda")
     cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, lib.SSD_MAX_GAMMA,
-                          w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1)
+                          w.prompt_len + w.max_new + lib.SSD_MAX_GAMMA + 1,
+                          options=lib.SSD_OPT_HOST_LOOP if args.host_loop else 0)
     model = lib.SSDModel(cfg, dev, rs, ins)
     vis, prompt = synth.make_inputs(w, seed=rank)
     v = up(vis)
@@ -666,7 +740,7 @@ def main() -> None:
     achieved = nbytes / (kern_ms / 1e3) / 1e9
     roofline = {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                 "frac": achieved / hbm_peak, "traffic": gemv_traffic_bytes(),
-                "kernel": "gemv_kernel<1, GATE_SILU> (layer gate/up, 2x11008x4096 bf16, 1 row)",
+                "kernel": "ssd_wstream_kernel<1, GATE_SILU> (layer gate/up, 2x11008x4096 bf16, 1 row)",
                 "bytes_per_launch": nbytes, "launch_us": kern_ms * 1e3,
                 "peak_source": f"{peak_src} HBM copy (burst)"}
     kernels = kernel_table(model, w, v, p, stream, hbm_peak)
@@ -689,7 +763,7 @@ def main() -> None:
             "e2e": e2e, "gpu_launches": int(args.steps * (pre_l + dec_l)),
             "roofline": roofline, "kernels": kernels, "clocks": clk,
             "prefill_ms": statistics.median(prefill_ms), "decode_ms": dec_ms,
-            "prefill_roofline": {"bound": "tensor", "kernel": "tc_gemm_kernel (all prefill projections) + prefill attention",
+            "prefill_roofline": {"bound": "tensor", "kernel": "ssd_prefill_tc_kernel (all prefill projections) + prefill attention",
                                  "achieved": prefill_flops(w) / (statistics.median(prefill_ms) / 1e3) / 1e12,
                                  "peak": float(peaks.get("bf16_tflops", 1900.0)), "unit": "TFLOP/s",
                                  "frac": prefill_flops(w) / (statistics.median(prefill_ms) / 1e3) / 1e12

@@ -78,6 +78,13 @@ enum {
                         * to the encoder's normed output, and a gated-GELU (tanh form) MLP; no RoPE */
 };
 
+/* ssd_config.options: alternative execution paths with identical results (diagnostics and
+ * cross-checks; 0 selects the default path).  Unknown bits are SSD_ERR_INVALID_ARG. */
+#define SSD_OPT_HOST_LOOP 1     /* decode loops driven from the host, one plain CUDA graph per step
+                                 * (kernel profilers do not see kernels inside conditional graph nodes) */
+#define SSD_OPT_PREFILL_ROWS 2  /* prefill through the decode kernels in 8-row chunks instead of the
+                                 * tensor-core GEMMs */
+
 #define SSD_MAX_GAMMA 8
 #define SSD_MAX_ROWS 16   /* rows one decode pass may carry (gamma + 1, prefill chunk) */
 
@@ -85,8 +92,8 @@ typedef struct ssd_ctx ssd_ctx;
 
 /* Model shape and decoding limits.  The decoder is a pre-norm LLaMA block stack
  * (RMSNorm, rotary multi-head attention, SwiGLU MLP), or with arch = SSD_ARCH_T5
- * the decoder of a T5 v1.1 encoder-decoder.  Fields after eos_id are read only
- * for SSD_ARCH_T5 (zero them otherwise). */
+ * the decoder of a T5 v1.1 encoder-decoder.  The fields n_enc_layers ..
+ * start_token are read only for SSD_ARCH_T5 (zero them otherwise). */
 typedef struct {
   int n_layers;      /* L */
   int d_model;       /* hidden width */
@@ -108,6 +115,7 @@ typedef struct {
   int rel_buckets;   /* T5: relative-position buckets (even, >= 4) */
   int rel_max_distance; /* T5: offsets at or beyond this share the last bucket */
   int start_token;   /* T5: the decoder's first input id */
+  int options;       /* SSD_OPT_* bits, 0 = the default path */
 } ssd_config;
 
 /* Extra weights of SSD_ARCH_T5, device bf16, [out][in], borrowed.  The
@@ -289,6 +297,19 @@ SSD_API ssd_status ssd_get_stats(ssd_ctx* ctx, ssd_stats* stats);
  * (the ctx rebuilds them).  sync. */
 SSD_API ssd_status ssd_set_logits_capture(ssd_ctx* ctx, float* buf, int max_rows);
 
+/* Debug capture of the drafting stage's logits g(I(x_k)) (Algorithm 1, draft loop): when buf
+ * (device fp32 [max_steps][gamma_max][vocab]) is non-NULL, the LM-head row of draft j in step s
+ * (steps counted from the last prefill; every step drafts gamma rows, of which the first
+ * gamma_eff are used) writes its logits to buf[s][j] while s < max_steps.  NULL disables.  Takes
+ * effect for graphs built afterwards (the ctx rebuilds them).  sync. */
+SSD_API ssd_status ssd_set_draft_logits_capture(ssd_ctx* ctx, float* buf, int max_steps);
+
+/* Per-step record of the last decode (Algorithm 1, acceptance): for each step s since the last
+ * prefill, accepted[s] = a (drafts kept) and drafted[s] = gamma_eff (drafts that could be kept);
+ * greedy steps record (0, 0).  Fills min(steps, cap) entries of the host arrays (either may be
+ * NULL) and sets *n_steps to the number of steps.  sync. */
+SSD_API ssd_status ssd_get_step_log(ssd_ctx* ctx, int32_t* accepted, int32_t* drafted, int cap, int* n_steps);
+
 /* Device pointers to the KV cache, layout [L][n_heads][max_seq][head_dim]
  * fp32 (with SSD_IN_BLOCK, [L + 1]: slot L is the imitation block's), and the
  * current valid length (sync read).  Positions >= kv_len hold stale rows of
@@ -319,12 +340,15 @@ SSD_API ssd_status ssd_lm_head(ssd_ctx* ctx, const float* x, int rows, int32_t* 
  *   lm_head:    device bf16 [vocab][d_model];  final_norm: device bf16 [d_model]
  *   x:          device fp32 [rows][d_model];  tok: device int32 [rows]
  *   logits:     device fp32 [rows][vocab] or NULL;  cuda_stream: cudaStream_t
- * Limits: 1 <= rows <= 9, vocab <= 262144, d_model a multiple of 256, 16-byte
- * aligned pointers; SSD_ERR_INVALID_ARG otherwise.  The first call on a device
- * (with that device current) looks up the array's device address and sets
- * kernel attributes: make it before any stream capture.  All calls share the
- * one array, so calls that overlap on the GPU (other streams, other threads)
- * race and must be serialised by the caller.  async. */
+ * Limits: 1 <= rows <= 9, vocab <= 262144, d_model a multiple of 64, 16-byte
+ * aligned pointers, and cuda_stream (when not NULL) a stream of the current
+ * device; SSD_ERR_INVALID_ARG otherwise.  The first call on a device (with that
+ * device current) looks up the array's device address and sets kernel
+ * attributes: make it before any stream capture (a failed first call is retried
+ * by the next one).  tok is set to -1 before the kernel runs and stays -1 if a
+ * bounded device wait gives up, so -1 marks a call that did not complete.  All
+ * calls share the one array, so calls that overlap on the GPU (other streams,
+ * other threads) race and must be serialised by the caller.  async. */
 SSD_API ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const float* x, int rows,
                                       int vocab, int d_model, float rms_eps, int32_t* tok, float* logits,
                                       void* cuda_stream);

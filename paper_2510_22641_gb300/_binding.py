@@ -19,6 +19,8 @@ SSD_IN_MLP2 = 1
 SSD_IN_BLOCK = 2
 SSD_ARCH_LLAMA = 0
 SSD_ARCH_T5 = 1
+SSD_OPT_HOST_LOOP = 1
+SSD_OPT_PREFILL_ROWS = 2
 
 STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_CUDA", 4: "SSD_ERR_CAPACITY",
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
@@ -26,7 +28,7 @@ STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_C
 EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode", "ssd_decode_dynamic",
             "ssd_draft_length", "ssd_rel_bucket",
             "ssd_greedy_decode", "ssd_generate", "ssd_greedy_generate", "ssd_sync", "ssd_get_stats",
-            "ssd_set_logits_capture", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
+            "ssd_set_logits_capture", "ssd_set_draft_logits_capture", "ssd_get_step_log", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
             "ssd_status_string",
             "ssd_last_error")
 
@@ -38,7 +40,7 @@ class SSDConfig(ctypes.Structure):
                 ("gamma_max", ctypes.c_int), ("max_seq", ctypes.c_int), ("rms_eps", ctypes.c_float),
                 ("rope_theta", ctypes.c_float), ("eos_id", ctypes.c_int), ("arch", ctypes.c_int),
                 ("n_enc_layers", ctypes.c_int), ("max_enc", ctypes.c_int), ("rel_buckets", ctypes.c_int),
-                ("rel_max_distance", ctypes.c_int), ("start_token", ctypes.c_int)]
+                ("rel_max_distance", ctypes.c_int), ("start_token", ctypes.c_int), ("options", ctypes.c_int)]
 
 
 _PP = ctypes.POINTER(ctypes.c_void_p)
@@ -97,6 +99,8 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_sync": [vp],
         "ssd_get_stats": [vp, ctypes.POINTER(SSDStats)],
         "ssd_set_logits_capture": [vp, vp, i32],
+        "ssd_set_draft_logits_capture": [vp, vp, i32],
+        "ssd_get_step_log": [vp, vp, vp, i32, ctypes.POINTER(i32)],
         "ssd_get_kv": [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(i32)],
         "ssd_last_launch_count": [vp, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)],
         "ssd_profile_projection": [vp, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_int64)],

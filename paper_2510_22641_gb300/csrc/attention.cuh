@@ -30,10 +30,12 @@
 // q and the chunk with this step's keys after it.
 #pragma once
 
-#include "attn_warp.cuh"
+#include "common.cuh"
 
 namespace ssd {
 
+constexpr int kAttnMaxRows = 9;           // query rows of one call (gamma_max + 1)
+constexpr int kAttnChunkBytes = 16384;    // one K (or V) chunk: 32 keys of head_dim 128, 64 of 64
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = 32 * kAttnWarps;
 constexpr int kAttnSplit = 8;  // CTAs per head
@@ -53,10 +55,6 @@ struct AttnParams {
   int prefetch_old;  // the previous launch triggered after its own upstream completed (see above)
   float* part;        // [n_heads][kAttnSplit][kAttnMaxRows][Dh + 2] CTA states (output, max, sum)
   unsigned* tickets;  // [n_heads], zero between launches
-  // optional timeline, [n_heads * kAttnSplit][8] %globaltimer stamps per CTA: 0 entry, 1 upstream
-  // grid complete, 2 first chunk landed, 3 last chunk folded, 4 state stored and ticket taken,
-  // 5 merge done (the head's last CTA), 6 exit, 7 chunks taken.  Null when not tracing.
-  unsigned long long* trace;
   // Non-causal key sets and relative-position bias (encoder-decoder models; read only by the EXT
   // instantiations, so the causal kernels compile without them):
   int fixed_keys;     // 1: keys 0 .. st->enc_len - 1, every one visible to every row (cross-attention,
@@ -96,7 +94,7 @@ struct AttnSmem {
 };
 
 template <int M, int DH, bool EXT>
-__global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const AttnParams p) {
   using S = AttnSmem<M, DH>;
   using G = AttnGeo<DH>;
   constexpr int KPC = G::KPC, KPW = G::KPW, TPK = G::TPK, DPP = G::DPP, NF = G::NF, DPL = G::DPL;
@@ -113,8 +111,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
   const int h = blockIdx.y;
 
   pdl_trigger();
-  unsigned long long* tr = p.trace ? p.trace + (static_cast<size_t>(h) * kAttnSplit + rank) * 8 : nullptr;
-  if (tr && tid == 0) tr[0] = globaltimer_ns();
   if (tid == 0) {
     for (int b = 0; b <= kAttnBufs; ++b) mbar_init(&bar[b], 1);
     fence_mbar_init();
@@ -160,7 +156,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
       }
   }
   pdl_wait();
-  if (tr && tid == 0) tr[1] = globaltimer_ns();
   if (!p.prefetch_old) geometry();
   if (bad && tid == 0 && rank == 0 && h == 0) set_error(p.st, DERR_POS);
   const bool timed_out = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
@@ -197,7 +192,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
         ok = false;
         continue;
       }
-      if (tr && tid == 0 && g0 == 0 && i == 0) tr[2] = globaltimer_ns();
       const float* kr = reinterpret_cast<const float*>(smem + S::kBuf0 + i * 2 * S::kKV) + jw * DH + part * DPP;
 #pragma unroll
       for (int e = 0; e < NF; ++e) {
@@ -339,10 +333,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
         issue(i, rank + (g0 + kAttnBufs + i) * kAttnSplit);
   }
   if (!ok) set_error(p.st, DERR_TIMEOUT);
-  if (tr && tid == 0) {
-    tr[3] = globaltimer_ns();
-    tr[7] = static_cast<unsigned long long>(my_chunks);
-  }
 
   // this CTA's state per row -- the warps' accumulators summed in warp order (the chunk buffers
   // are free: every chunk was waited for and folded before the last barrier) -- goes to part;
@@ -370,7 +360,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
   __syncthreads();
   if (tid == 0) *last = atom_add_acq_rel_gpu(&p.tickets[h], 1u) == static_cast<unsigned>(kAttnSplit - 1);
   __syncthreads();
-  if (tr && tid == 0) tr[4] = globaltimer_ns();
   if (*last) {
     if (!bad && !timed_out) {
       float* wq = reinterpret_cast<float*>(smem + S::kWq);  // [M][kAttnSplit] weights, then [M] totals
@@ -417,9 +406,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) attn_kernel(const AttnParams 
       }
     }
     if (tid == 0) p.tickets[h] = 0u;
-    if (tr && tid == 0) tr[5] = globaltimer_ns();
   }
-  if (tr && tid == 0) tr[6] = globaltimer_ns();
 }
 
 }  // namespace ssd

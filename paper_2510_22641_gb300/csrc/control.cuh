@@ -8,7 +8,7 @@
 namespace ssd {
 
 // x[m][:] = fp32(E[tok[m]][:]) -- the embedding layer that maps token ids to x_0.
-__global__ void embed_kernel(const __nv_bfloat16* __restrict__ E, const int* tok, float* x, int x_stride, int d,
+__global__ void ssd_embed_kernel(const __nv_bfloat16* __restrict__ E, const int* tok, float* x, int x_stride, int d,
                              int vocab, DevState* st) {
   pdl_trigger();
   pdl_wait();
@@ -31,7 +31,7 @@ __global__ void embed_kernel(const __nv_bfloat16* __restrict__ E, const int* tok
 
 // Prefill input rows r0 + m of [z (n_vis rows); embed(prompt)] (Sec. "SSD Setup for VLMs": z is fed
 // to the decoder as its first input rows).
-__global__ void prefill_rows_kernel(const __nv_bfloat16* __restrict__ vis, const int* __restrict__ prompt, int n_vis,
+__global__ void ssd_prefill_rows_kernel(const __nv_bfloat16* __restrict__ vis, const int* __restrict__ prompt, int n_vis,
                                     int r0, const __nv_bfloat16* __restrict__ E, int vocab, float* x, int x_stride,
                                     int d, DevState* st) {
   pdl_trigger();
@@ -61,7 +61,7 @@ __global__ void prefill_rows_kernel(const __nv_bfloat16* __restrict__ vis, const
 
 // P: decoder rows of the prompt (the position of the first new token + 1); enc_len: encoder rows
 // (encoder-decoder model; 0 otherwise).
-__global__ void prefill_begin_kernel(DevState* st, int P, int eos_id, int enc_len) {
+__global__ void ssd_prefill_begin_kernel(DevState* st, int P, int eos_id, int enc_len) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
@@ -79,7 +79,7 @@ __global__ void prefill_begin_kernel(DevState* st, int P, int eos_id, int enc_le
 }
 
 // The last prompt row's greedy token is the first new token; the cache now holds positions 0..P-1.
-__global__ void prefill_finish_kernel(DevState* st, int* out_tok, int P) {
+__global__ void ssd_prefill_finish_kernel(DevState* st, int* out_tok, int P) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
@@ -95,7 +95,7 @@ __global__ void prefill_finish_kernel(DevState* st, int* out_tok, int P) {
   st->done = (st->eos_id >= 0 && y == st->eos_id) ? 1 : 0;
 }
 
-__global__ void decode_setup_kernel(DevState* st, int max_new, int gamma) {
+__global__ void ssd_decode_setup_kernel(DevState* st, int max_new, int gamma) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
@@ -110,7 +110,7 @@ __global__ void decode_setup_kernel(DevState* st, int max_new, int gamma) {
 // Dynamic draft length (Sec. "Choice of d"): this step drafts gamma = table[kv_len] tokens,
 // clamped to [1, cap] (table[p] = d(p + 2), evaluated on the host in fp64); the step's branch
 // of the SWITCH node is gamma - 1.  launches[gamma - 1]: kernel launches of that branch.
-__global__ void dyn_select_kernel(DevState* st, const int* table, const int* launches, int cap,
+__global__ void ssd_dyn_select_kernel(DevState* st, const int* table, const int* launches, int cap,
                                   cudaGraphConditionalHandle sw) {
   pdl_trigger();
   pdl_wait();
@@ -123,21 +123,22 @@ __global__ void dyn_select_kernel(DevState* st, const int* table, const int* lau
 }
 
 // Loop test after a dynamic-length step: run the WHILE body again unless decoding is finished.
-__global__ void loop_continue_kernel(DevState* st, cudaGraphConditionalHandle cond) {
+__global__ void ssd_loop_continue_kernel(DevState* st, cudaGraphConditionalHandle cond) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x == 0) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
 }
 
 // First node of a decode graph: run the WHILE body only if decoding is not finished.
-__global__ void loop_begin_kernel(DevState* st, cudaGraphConditionalHandle cond) {
+__global__ void ssd_loop_begin_kernel(DevState* st, cudaGraphConditionalHandle cond) {
   if (threadIdx.x == 0) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
 }
 
 // Algorithm 1, acceptance: a = longest prefix with d_{i+1} == f_i (i < gamma_eff),
 // emit d_1..d_a and f_a (the correction, or the bonus token when a = gamma_eff),
-// roll the cache back by length: kv_len += a + 1.
-__global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out_cap,
+// roll the cache back by length: kv_len += a + 1.  step_log[steps] = (a, gamma_eff) while
+// steps < log_cap.
+__global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out_cap, int2* step_log, int log_cap,
                                   cudaGraphConditionalHandle cond, int has_cond) {
   pdl_trigger();
   pdl_wait();
@@ -167,6 +168,7 @@ __global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out
   st->last_n = cnt;
   st->n_out += cnt;
   st->kv_len += a + 1;
+  if (st->steps < log_cap) step_log[st->steps] = make_int2(a, g_eff);
   const int y = st->full_tok[a];
   st->cur_tok = y;
   st->tok_in[0] = y;
@@ -179,8 +181,8 @@ __global__ void ssd_accept_kernel(DevState* st, int gamma, int* out_tok, int out
 }
 
 // Greedy baseline step: emit f_0 of the single row, advance the cache by one.
-__global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cudaGraphConditionalHandle cond,
-                                     int has_cond) {
+__global__ void ssd_greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, int2* step_log, int log_cap,
+                                         cudaGraphConditionalHandle cond, int has_cond) {
   pdl_trigger();
   pdl_wait();
   if (threadIdx.x != 0) return;
@@ -194,6 +196,7 @@ __global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cu
   st->kv_len += 1;
   st->cur_tok = y;
   st->tok_in[0] = y;
+  if (st->steps < log_cap) step_log[st->steps] = make_int2(0, 0);
   st->steps += 1;
   st->last_n = 1;
   st->last_emitted[0] = y;
@@ -201,7 +204,7 @@ __global__ void greedy_accept_kernel(DevState* st, int* out_tok, int out_cap, cu
   if (has_cond) cudaGraphSetConditional(cond, st->done ? 0u : 1u);
 }
 
-__global__ void copy_out_kernel(const DevState* st, const int* out_int, int* user_out, int* user_n, int max_new) {
+__global__ void ssd_copy_out_kernel(const DevState* st, const int* out_int, int* user_out, int* user_n, int max_new) {
   pdl_wait();
   const int n = min(st->n_out, max_new);
   for (int i = threadIdx.x; i < n; i += blockDim.x)
@@ -209,25 +212,25 @@ __global__ void copy_out_kernel(const DevState* st, const int* out_int, int* use
   if (threadIdx.x == 0 && user_n) *user_n = n;
 }
 
-__global__ void copy_draft_kernel(const DevState* st, int gamma, int* draft_tok) {
+__global__ void ssd_copy_draft_kernel(const DevState* st, int gamma, int* draft_tok) {
   pdl_wait();
   if (threadIdx.x < gamma) draft_tok[threadIdx.x] = st->tok_in[threadIdx.x + 1];
 }
 
-__global__ void copy_emitted_kernel(const DevState* st, int* n_emitted, int* emitted) {
+__global__ void ssd_copy_emitted_kernel(const DevState* st, int* n_emitted, int* emitted) {
   pdl_wait();
   const int n = st->last_n;
   if (threadIdx.x == 0 && n_emitted) *n_emitted = n;
   if (emitted && threadIdx.x < n) emitted[threadIdx.x] = st->last_emitted[threadIdx.x];
 }
 
-__global__ void first_token_kernel(const DevState* st, int* first_tok) {
+__global__ void ssd_first_token_kernel(const DevState* st, int* first_tok) {
   pdl_wait();
   if (threadIdx.x == 0) *first_tok = st->cur_tok;
 }
 
 // cos/sin of pos * theta^(-2j/head_dim), computed in fp64 and rounded to fp32.
-__global__ void rope_table_kernel(float2* cs, int max_seq, int head_dim, double theta) {
+__global__ void ssd_rope_table_kernel(float2* cs, int max_seq, int head_dim, double theta) {
   const int half = head_dim / 2;
   const int idx = blockIdx.x * blockDim.x + threadIdx.x;
   if (idx >= max_seq * half) return;
@@ -240,7 +243,7 @@ __global__ void rope_table_kernel(float2* cs, int max_seq, int head_dim, double 
 
 // Relative-position bias table out[h][j] = rel[bucket[j]][h] (rel: the learned [buckets][n_heads]
 // bf16 table of a T5-style stack; bucket[j]: the bucket of offset j - zero, decided on the host).
-__global__ void bias_table_kernel(const __nv_bfloat16* __restrict__ rel, const int* __restrict__ bucket, int n,
+__global__ void ssd_bias_table_kernel(const __nv_bfloat16* __restrict__ rel, const int* __restrict__ bucket, int n,
                                   int n_heads, float* out) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n * n_heads) return;

@@ -2,7 +2,7 @@
 //
 // One ssd_ctx owns the KV cache, activation rows, workspaces, a private CUDA
 // stream and the CUDA graphs that replay the decode loop.  Every projection is
-// a gemv_kernel launch (stream-K weight streaming), attention is attn_kernel
+// a ssd_wstream_kernel launch (stream-K weight streaming), attention is ssd_splitkv_attn_kernel
 // (split-KV, causal over the query block), and the loop control of Algorithm 1
 // runs in small device kernels; a decode is one graph launch whose WHILE node
 // repeats draft + verify + accept on the device until the device state says
@@ -23,7 +23,6 @@
 #include "attention.cuh"
 #include "control.cuh"
 #include "gemv.cuh"
-#include "fwd_params.cuh"
 #include "prefill_params.cuh"
 
 namespace ssd {
@@ -45,9 +44,6 @@ cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bf
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
                                 float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
                                 cudaStream_t s, bool pdl);
-cudaError_t fwd_attrs();
-cudaError_t fwd_ctas_per_sm(int head_dim, int* n);
-cudaError_t fwd_launch(int head_dim, const FwdParams& p, int grid, cudaStream_t stream, bool cooperative);
 }  // namespace ssd
 
 using namespace ssd;
@@ -81,12 +77,6 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 
 }  // namespace
 
-// One phase list of the persistent forward kernel, stored in ssd_ctx::fwd_phases.
-struct FwdProg {
-  size_t off = 0;
-  int n_phases = 0, n_flags = 0;
-};
-
 struct ssd_ctx {
   ssd_config cfg{};
   int qdim = 0, num_sms = 0, device = 0;
@@ -104,11 +94,12 @@ struct ssd_ctx {
   CUtensorMap a_maps[3][2];  // activation splits (hi, lo) for K = d_model, n_heads*head_dim, d_ff
   __nv_bfloat16 *a_hi = nullptr, *a_lo = nullptr;
   float *x_pre = nullptr, *q_pre = nullptr, *o_pre = nullptr, *h_pre = nullptr;
-  bool prefill_rows = false;  // SSD_PREFILL=rows: prefill through the decode kernels in 8-row chunks
+  bool prefill_rows = false;  // SSD_OPT_PREFILL_ROWS: prefill through the decode kernels in 8-row chunks
   // owned device memory
   DevState* st = nullptr;
   DevState* op_st = nullptr;  // state of standalone op calls (ssd_lm_head)
   int* out_int = nullptr;  // [max_seq] emitted tokens
+  int2* step_log = nullptr;  // [max_seq] (accepted drafts a, gamma_eff) per step since the prefill
   float *xv = nullptr, *qb = nullptr, *ob = nullptr, *hb = nullptr, *hin = nullptr, *xt = nullptr;
   float *kc = nullptr, *vc = nullptr;  // KV cache [L][H][max_seq][Dh], fp32
   size_t layer_kv = 0;  // elements per layer in kc / vc
@@ -135,8 +126,6 @@ struct ssd_ctx {
   // Diagnostic: drive the decode loop from the host with one plain graph per
   // step (ncu cannot profile kernels of graphs that hold conditional nodes).
   bool host_loop = false;
-  int gemv_ctas = 2;  // GEMV CTAs per SM
-  int small_site_rt = 0, small_site_ctas = 2;  // sites with fewer row tiles than small_site_rt use small_site_ctas
   std::map<std::pair<int, int>, cudaGraphExec_t> prefill_graphs;
   cudaGraphExec_t greedy_graph = nullptr;
   std::map<int, int64_t> decode_body_launches;
@@ -151,25 +140,6 @@ struct ssd_ctx {
   int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy, 3 ssd with the dynamic draft length
   int last_gamma = 0;
   std::pair<int, int> last_prefill_shape{0, 0};
-  // persistent forward kernel (decode): phase lists, map table, flags and scratch
-  bool use_fwd = false;  // SSD_DECODE=fwd: one persistent launch per forward pass
-  bool fwd_coop = true;  // cooperative launch (every CTA resident)
-  bool fwd_ready = false;
-  int fwd_grid = 0, fwd_splits = 1;
-  FwdProg fwd_greedy;
-  std::vector<FwdProg> fwd_draft, fwd_verify;  // indexed by gamma
-  FwdPhase* fwd_phases = nullptr;
-  size_t fwd_phases_cap = 0;
-  CUtensorMap* fwd_maps = nullptr;
-  unsigned *fwd_flags = nullptr, *fwd_tickets = nullptr, *fwd_done = nullptr, *fwd_exit = nullptr;
-  int fwd_flags_cap = 0, fwd_done_cap = 0;
-  float *fwd_partials = nullptr, *fwd_attn_part = nullptr;
-  uint8_t* fwd_btiles = nullptr;  // [kFwdBSlots][fwd_bslot] B operands written by producer epilogues
-  long long fwd_bslot = 0;
-  unsigned long long* fwd_trace = nullptr;  // SSD_FWD_TRACE=<file>: timeline of the last launch
-  std::string gemv_trace_path;  // SSD_GEMV_TRACE=<file>: per-CTA timeline of ssd_profile_projection's last launch (GEMV or attention)
-  std::string fwd_trace_path;
-  int fwd_trace_phases = 0;
   // encoder-decoder model (SSD_ARCH_T5)
   bool t5 = false;
   int max_enc = 0;
@@ -184,9 +154,11 @@ struct ssd_ctx {
   float *dec_bias = nullptr, *enc_bias = nullptr;    // [H][max_seq] and [H][2 max_enc - 1]
   float* one = nullptr;                              // device 1.0f: the encoder's residual scale
   int* start_tok = nullptr;                          // device copy of cfg.start_token
-  // debug logits capture
+  // debug logits capture: full-model rows by predicted token index, draft rows by (step, j)
   float* logits_buf = nullptr;
   int logits_rows = 0;
+  float* draft_logits_buf = nullptr;
+  int draft_logits_steps = 0;
   std::string err;
 };
 
@@ -269,9 +241,7 @@ static ssd_status make_site(ssd_ctx* c, Site* s, const void* const* mats, int nm
   s->n_rt = (s->N + kTileN - 1) / kTileN;
   s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
-  // few row tiles: each would be split across many CTAs, so use fewer CTAs
-  const int ctas = (s->n_rt < c->small_site_rt) ? c->small_site_ctas : c->gemv_ctas;
-  s->grid = s->units < c->num_sms * ctas ? s->units : c->num_sms * ctas;
+  s->grid = s->units < c->num_sms * kGemvCtasPerSm ? s->units : c->num_sms * kGemvCtasPerSm;
   return SSD_OK;
 }
 
@@ -286,7 +256,7 @@ static ssd_status make_pair_site(ssd_ctx* c, Site* s, const void* gate, const vo
   s->n_rt = (rows + kHalfN - 1) / kHalfN;
   s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
-  s->grid = s->units < c->num_sms * c->gemv_ctas ? s->units : c->num_sms * c->gemv_ctas;
+  s->grid = s->units < c->num_sms * kGemvCtasPerSm ? s->units : c->num_sms * kGemvCtasPerSm;
   return SSD_OK;
 }
 
@@ -320,18 +290,18 @@ static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a) {
   const dim3 grid(kAttnSplit, c->cfg.n_heads);
   const bool ext = a.fixed_keys || a.abs_pos || a.bias;
   if (c->cfg.head_dim == 128)
-    return ext ? launch_k(c, attn_kernel<M, 128, true>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a)
-               : launch_k(c, attn_kernel<M, 128, false>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
-  return ext ? launch_k(c, attn_kernel<M, 64, true>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a)
-             : launch_k(c, attn_kernel<M, 64, false>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
+    return ext ? launch_k(c, ssd_splitkv_attn_kernel<M, 128, true>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a)
+               : launch_k(c, ssd_splitkv_attn_kernel<M, 128, false>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
+  return ext ? launch_k(c, ssd_splitkv_attn_kernel<M, 64, true>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a)
+             : launch_k(c, ssd_splitkv_attn_kernel<M, 64, false>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
 }
 
 template <int M, int DH>
 static cudaError_t attn_attr_md() {
-  cudaError_t e = cudaFuncSetAttribute(attn_kernel<M, DH, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(ssd_splitkv_attn_kernel<M, DH, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        AttnSmem<M, DH>::kTotal);
   if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(attn_kernel<M, DH, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(ssd_splitkv_attn_kernel<M, DH, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               AttnSmem<M, DH>::kTotal);
 }
 
@@ -381,10 +351,8 @@ static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a) {
 // Causal self-attention of layer l over the KV cache for the M rows at kv_len + pos_off + m.  The
 // encoder-decoder model's decoder adds its relative-position bias and has no 1/sqrt(head_dim) factor.
 // prefetch_old: the launch before is the layer's QKV projection with a late trigger.
-static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch_old,
-                            unsigned long long* trace = nullptr) {
+static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch_old) {
   AttnParams a{};
-  a.trace = trace;
   a.prefetch_old = prefetch_old ? 1 : 0;
   a.q = c->qb;
   a.q_stride = c->qp;
@@ -564,376 +532,32 @@ static ssd_status enqueue_head(ssd_ctx* c, const float* x, int M, int pos_off, i
   return gemv(c, Epi::ARGMAX, M, c->head, p);
 }
 
+// LM head + argmax of draft row j (the token d_{j+1}); with a draft capture buffer its logits go
+// to row st->steps * gamma_max + j.
+static ssd_status enqueue_draft_head(ssd_ctx* c, const float* x, int j, int* tok_dst) {
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = c->dp;
+  p.gain = c->final_norm;
+  p.pos_off = j;
+  p.tok_dst = tok_dst;
+  p.logits = c->draft_logits_buf;
+  p.logits_rows = c->draft_logits_buf ? c->draft_logits_steps * c->cfg.gamma_max : 0;
+  p.logits_step_rows = c->cfg.gamma_max;
+  return gemv(c, Epi::ARGMAX, 1, c->head, p);
+}
+
 static int* st_field(ssd_ctx* c, size_t off) {
   return reinterpret_cast<int*>(reinterpret_cast<char*>(c->st) + off);
 }
 
-// ------------------------------------------------------------------ persistent forward kernel
-
-static ssd_status fwd_alloc(ssd_ctx* c, void** p, size_t bytes) {
-  cudaError_t e = cudaMalloc(p, bytes);
-  if (e == cudaSuccess) e = cudaMemset(*p, 0, bytes);
-  if (e != cudaSuccess) {
-    *p = nullptr;
-    return fail(c, SSD_ERR_OOM, "forward-kernel scratch (%zu bytes): %s", bytes, cudaGetErrorString(e));
-  }
-  return SSD_OK;
-}
-
-// Map table: layer l -> [7l] q, k, v, [7l+3] o, [7l+4] gate, [7l+5] up, [7l+6] down;
-// then imitation FC1, FC2 and the LM head.
-static int map_in1(const ssd_ctx* c) { return 7 * c->cfg.n_layers; }
-static int map_in2(const ssd_ctx* c) { return 7 * c->cfg.n_layers + 1; }
-static int map_head(const ssd_ctx* c) { return 7 * c->cfg.n_layers + 2; }
-
-struct FwdBuilder {
-  ssd_ctx* c;
-  std::vector<FwdPhase> ph;
-  int flags = 0;
-  int add(FwdPhase f) {
-    f.flags = flags;
-    f.bt_off = -1;
-    f.bt_dst_off = -1;
-    flags += f.n_tiles;
-    ph.push_back(f);
-    return static_cast<int>(ph.size()) - 1;
-  }
-  // columns of phase q's output per tile (what a consumer's 64-column slice maps to)
-  int out_cols(int q) const {
-    if (q < 0) return kTileN;
-    const int k = ph[q].kind;
-    if (k == FK_GATE_SILU) return kHalfN;
-    if (k == FK_ATTN) return c->cfg.head_dim;
-    return kTileN;
-  }
-};
-
-static FwdPhase fwd_gemv(const Site& s, int kind, int M, int map0, int map1, int map2) {
-  FwdPhase f{};
-  f.kind = kind;
-  f.M = M;
-  f.K = s.K;
-  f.N = s.N;
-  f.n_kt = s.n_kt;
-  f.n_rt = s.n_rt;
-  f.units = s.units;
-  f.seg_rows = s.seg_rows;
-  f.map0 = map0;
-  f.map1 = map1;
-  f.map2 = map2;
-  f.n_tiles = s.n_rt;
-  f.dep = f.epi_dep = -1;
-  return f;
-}
-
-// x[row0 .. row0+M-1] = E[tok_src[0 .. M-1]]; tok_src is final once phase tok_dep is complete.
-static int fwd_add_embed(FwdBuilder& b, const int* tok_src, int row0, int M, int tok_dep) {
-  ssd_ctx* c = b.c;
-  FwdPhase f{};
-  f.kind = FK_EMBED;
-  f.M = M;
-  f.tok_src = tok_src;
-  f.dst = c->xv + static_cast<size_t>(row0) * c->dp;
-  f.dst_stride = c->dp;
-  f.n_tiles = (c->dp + kTileN - 1) / kTileN;
-  f.dep = -1;
-  f.epi_dep = tok_dep;
-  return b.add(f);
-}
-
-// Decoder layer l on rows x[0 .. M-1] (stride dp) at positions kv_len + pos_off + m;
-// x is final once phase xdep is complete.  Returns the phase that completes x_{l+1}.
-static int fwd_add_layer(FwdBuilder& b, int l, float* x, int M, int pos_off, int xdep) {
-  ssd_ctx* c = b.c;
-  const LayerSites& L = c->layers[l];
-  const int m0 = 7 * l;
-  FwdPhase f = fwd_gemv(L.qkv, FK_QKV, M, m0, m0 + 1, m0 + 2);
-  f.x = x;
-  f.x_stride = c->dp;
-  f.gain = c->attn_norm[l];
-  f.dep = xdep;
-  f.dep_cols = b.out_cols(xdep);
-  f.epi_dep = xdep;
-  f.pos_off = pos_off;
-  f.q_out = c->qb;
-  f.q_stride = c->qp;
-  f.k_cache = c->kc + l * c->layer_kv;
-  f.v_cache = c->vc + l * c->layer_kv;
-  const int qkv = b.add(f);
-
-  f = FwdPhase{};
-  f.kind = FK_ATTN;
-  f.M = M;
-  f.x = c->qb;
-  f.x_stride = c->qp;
-  f.dst = c->ob;
-  f.dst_stride = c->qp;
-  f.k_cache = c->kc + l * c->layer_kv;
-  f.v_cache = c->vc + l * c->layer_kv;
-  f.pos_off = pos_off;
-  f.dep = qkv;
-  f.epi_dep = -1;
-  f.n_tiles = c->cfg.n_heads;
-  const int attn = b.add(f);
-
-  f = fwd_gemv(L.o, FK_RESID, M, m0 + 3, m0 + 3, m0 + 3);
-  f.x = c->ob;
-  f.x_stride = c->qp;
-  f.dep = attn;
-  f.dep_cols = b.out_cols(attn);
-  f.epi_dep = xdep;  // base rows x
-  f.base = x;
-  f.base_stride = c->dp;
-  f.dst = x;
-  f.dst_stride = c->dp;
-  f.scale = c->resid_scale + l;
-  const int o = b.add(f);
-
-  f = fwd_gemv(L.gateup, FK_GATE_SILU, M, m0 + 4, m0 + 5, m0 + 4);
-  f.x = x;
-  f.x_stride = c->dp;
-  f.gain = c->ffn_norm[l];
-  f.dep = o;
-  f.dep_cols = b.out_cols(o);
-  f.epi_dep = o;
-  f.h_out = c->hb;
-  f.h_stride = c->fp;
-  const int gu = b.add(f);
-
-  f = fwd_gemv(L.down, FK_RESID, M, m0 + 6, m0 + 6, m0 + 6);
-  f.x = c->hb;
-  f.x_stride = c->fp;
-  f.dep = gu;
-  f.dep_cols = b.out_cols(gu);
-  f.epi_dep = o;  // base rows x
-  f.base = x;
-  f.base_stride = c->dp;
-  f.dst = x;
-  f.dst_stride = c->dp;
-  f.scale = c->resid_scale + l;
-  return b.add(f);
-}
-
-// g(x) = W_lm RMSNorm_f(x) + argmax on rows x[0 .. M-1].
-static int fwd_add_head(FwdBuilder& b, const float* x, int M, int pos_off, int* tok_dst, bool capture, int xdep) {
-  ssd_ctx* c = b.c;
-  FwdPhase f = fwd_gemv(c->head, FK_ARGMAX, M, map_head(c), map_head(c), map_head(c));
-  f.x = x;
-  f.x_stride = c->dp;
-  f.gain = c->final_norm;
-  f.dep = xdep;
-  f.dep_cols = b.out_cols(xdep);
-  f.epi_dep = xdep;
-  f.pos_off = pos_off;
-  f.tok_dst = tok_dst;
-  f.logits = capture ? c->logits_buf : nullptr;
-  f.logits_rows = capture ? c->logits_rows : 0;
-  return b.add(f);
-}
-
-// Imitation network on row x (M = 1): xt = x + s_in * W2 SiLU(W1 RMSNorm_in(x)).
-static int fwd_add_in(FwdBuilder& b, float* x, int xdep) {
-  ssd_ctx* c = b.c;
-  FwdPhase f = fwd_gemv(c->in1, FK_SILU, 1, map_in1(c), map_in1(c), map_in1(c));
-  f.x = x;
-  f.x_stride = c->dp;
-  f.gain = c->in_norm;
-  f.dep = xdep;
-  f.dep_cols = b.out_cols(xdep);
-  f.epi_dep = xdep;
-  f.h_out = c->hin;
-  f.h_stride = c->ip;
-  const int s1 = b.add(f);
-  f = fwd_gemv(c->in2, FK_RESID, 1, map_in2(c), map_in2(c), map_in2(c));
-  f.x = c->hin;
-  f.x_stride = c->ip;
-  f.dep = s1;
-  f.dep_cols = b.out_cols(s1);
-  f.epi_dep = xdep;  // base row x
-  f.base = x;
-  f.base_stride = c->dp;
-  f.dst = c->xt;
-  f.dst_stride = c->dp;
-  f.scale = c->in_scale;
-  return b.add(f);
-}
-
-// The projection q reads the B operands of its 64-column slices from slot q mod kFwdBSlots
-// of the B-operand ring; its producer -- always phase q - 1, so that the drain warps'
-// wait on phase q - 1 - window keeps a slot from being rewritten while it is read --
-// writes them in its epilogue.
-static bool fwd_link_operands(ssd_ctx* c, FwdBuilder& b) {
-  auto out_ptr = [](const FwdPhase& f) -> const float* {
-    return (f.kind == FK_GATE_SILU || f.kind == FK_SILU) ? f.h_out : f.dst;
-  };
-  for (int q = 0; q < static_cast<int>(b.ph.size()); ++q) {
-    FwdPhase& f = b.ph[q];
-    if (f.kind > FK_ARGMAX) continue;
-    const int pq = f.dep;
-    if (pq != q - 1) return false;
-    FwdPhase& pr = b.ph[pq];
-    if (pr.bt_dst_off >= 0 || pr.kind == FK_QKV || pr.kind == FK_ARGMAX) return false;
-    const ptrdiff_t d = out_ptr(pr) - f.x;
-    if (d < 0 || d % f.x_stride != 0) return false;
-    const int row0 = static_cast<int>(d / f.x_stride);
-    if (row0 + pr.M > f.M) return false;
-    f.bt_off = static_cast<long long>(q % kFwdBSlots) * c->fwd_bslot;
-    pr.bt_dst_off = f.bt_off;
-    pr.bt_x = f.x;
-    pr.bt_x_stride = f.x_stride;
-    pr.bt_M = f.M;
-    pr.bt_nkt = f.n_kt;
-    pr.bt_row0 = row0;
-    pr.bt_gain = f.gain;
-  }
-  return true;
-}
-
-static FwdProg fwd_commit(FwdBuilder& b, std::vector<FwdPhase>& all) {
-  if (!fwd_link_operands(b.c, b)) {
-    FwdProg bad;
-    bad.n_phases = -1;
-    return bad;
-  }
-  FwdProg pr;
-  pr.off = all.size();
-  pr.n_phases = static_cast<int>(b.ph.size());
-  pr.n_flags = b.flags;
-  all.insert(all.end(), b.ph.begin(), b.ph.end());
-  return pr;
-}
-
-static int* st_field_early(ssd_ctx* c, size_t off) {
-  return reinterpret_cast<int*>(reinterpret_cast<char*>(c->st) + off);
-}
-
-// Phase lists of the greedy step and, per gamma, of the drafting and verification stages.
-static ssd_status fwd_build_programs(ssd_ctx* c) {
-  const int K = c->cfg.draft_exit_k, Lc = c->cfg.n_layers, d = c->dp;
-  int* tok_in = st_field_early(c, offsetof(DevState, tok_in));
-  int* full_tok = st_field_early(c, offsetof(DevState, full_tok));
-  std::vector<FwdPhase> all;
-  {
-    FwdBuilder b{c};
-    int last = fwd_add_embed(b, tok_in, 0, 1, -1);
-    for (int l = 0; l < Lc; ++l) last = fwd_add_layer(b, l, c->xv, 1, 0, last);
-    fwd_add_head(b, c->xv, 1, 0, full_tok, true, last);
-    c->fwd_greedy = fwd_commit(b, all);
-  }
-  c->fwd_draft.assign(c->cfg.gamma_max + 1, FwdProg{});
-  c->fwd_verify.assign(c->cfg.gamma_max + 1, FwdProg{});
-  for (int g = 1; g <= c->cfg.gamma_max; ++g) {
-    FwdBuilder b{c};
-    int head = -1;
-    for (int j = 0; j < g; ++j) {
-      float* xj = c->xv + static_cast<size_t>(j) * d;
-      int last = fwd_add_embed(b, tok_in + j, j, 1, head);
-      for (int l = 0; l < K; ++l) last = fwd_add_layer(b, l, xj, 1, j, last);
-      const float* hx = xj;
-      if (c->cfg.in_kind == SSD_IN_MLP2) {
-        last = fwd_add_in(b, xj, last);
-        hx = c->xt;
-      }
-      head = fwd_add_head(b, hx, 1, j, tok_in + j + 1, false, last);
-    }
-    c->fwd_draft[g] = fwd_commit(b, all);
-    FwdBuilder v{c};
-    int last = fwd_add_embed(v, tok_in + g, g, 1, -1);
-    float* xg = c->xv + static_cast<size_t>(g) * d;
-    for (int l = 0; l < K; ++l) last = fwd_add_layer(v, l, xg, 1, g, last);
-    for (int l = K; l < Lc; ++l) last = fwd_add_layer(v, l, c->xv, g + 1, 0, last);
-    fwd_add_head(v, c->xv, g + 1, 0, full_tok, true, last);
-    c->fwd_verify[g] = fwd_commit(v, all);
-  }
-  bool linked = c->fwd_greedy.n_phases > 0;
-  for (int g = 1; g <= c->cfg.gamma_max; ++g) linked = linked && c->fwd_draft[g].n_phases > 0 && c->fwd_verify[g].n_phases > 0;
-  if (!linked) return fail(c, SSD_ERR_STATE, "forward-kernel phase list: a projection does not read its predecessor");
-  int max_flags = std::max(1, c->fwd_greedy.n_flags), max_phases = std::max(1, c->fwd_greedy.n_phases);
-  for (int g = 1; g <= c->cfg.gamma_max; ++g)
-    for (const FwdProg* pr : {&c->fwd_draft[g], &c->fwd_verify[g]}) {
-      max_flags = std::max(max_flags, pr->n_flags);
-      max_phases = std::max(max_phases, pr->n_phases);
-    }
-  if (all.size() > c->fwd_phases_cap) {
-    if (c->fwd_phases) cudaFree(c->fwd_phases);
-    c->fwd_phases = nullptr;
-    c->fwd_phases_cap = 0;
-    CK(cudaMalloc(&c->fwd_phases, sizeof(FwdPhase) * all.size()));
-    c->fwd_phases_cap = all.size();
-  }
-  CK(cudaMemcpy(c->fwd_phases, all.data(), sizeof(FwdPhase) * all.size(), cudaMemcpyHostToDevice));
-  if (max_flags > c->fwd_flags_cap) {
-    for (unsigned** b : {&c->fwd_flags, &c->fwd_tickets}) {
-      if (*b) cudaFree(*b);
-      *b = nullptr;
-    }
-    c->fwd_flags_cap = 0;
-    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_flags), sizeof(unsigned) * max_flags));
-    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_tickets), sizeof(unsigned) * max_flags));
-    c->fwd_flags_cap = max_flags;
-  }
-  if (max_phases > c->fwd_done_cap) {
-    if (c->fwd_done) cudaFree(c->fwd_done);
-    c->fwd_done = nullptr;
-    c->fwd_done_cap = 0;
-    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_done), sizeof(unsigned) * max_phases));
-    c->fwd_done_cap = max_phases;
-  }
-  if (!c->fwd_trace_path.empty() && !c->fwd_trace) {
-    CKS(fwd_alloc(c, reinterpret_cast<void**>(&c->fwd_trace),
-                  sizeof(unsigned long long) * (c->fwd_grid * (max_phases + 1) * 16 + 4 * 8192 * 4)));
-  }
-  c->fwd_ready = true;
-  return SSD_OK;
-}
-
-static ssd_status fwd_run(ssd_ctx* c, const FwdProg& pr) {
-  FwdParams p{};
-  p.phases = c->fwd_phases + pr.off;
-  p.n_phases = pr.n_phases;
-  p.maps = c->fwd_maps;
-  p.st = c->st;
-  p.flags = c->fwd_flags;
-  p.tickets = c->fwd_tickets;
-  p.done = c->fwd_done;
-  p.exit_count = c->fwd_exit;
-  p.btiles = c->fwd_btiles;
-  p.n_flags = pr.n_flags;
-  p.partials = c->fwd_partials;
-  p.attn_part = c->fwd_attn_part;
-  p.n_heads = c->cfg.n_heads;
-  p.head_dim = c->cfg.head_dim;
-  p.max_seq = c->cfg.max_seq;
-  p.splits = c->fwd_splits;
-  p.attn_scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
-  p.eps = c->cfg.rms_eps;
-  p.rope = c->rope;
-  p.embed = c->embed;
-  p.vocab = c->cfg.vocab;
-  p.d_model = c->cfg.d_model;
-  p.trace = c->fwd_trace;
-  c->fwd_trace_phases = pr.n_phases;
-  ++c->launch_counter;
-  CK(fwd_launch(c->cfg.head_dim, p, c->fwd_grid, c->cs, c->fwd_coop));
-  return SSD_OK;
-}
-
-static ssd_status fwd_ensure(ssd_ctx* c) {
-  if (!c->use_fwd || c->fwd_ready) return SSD_OK;
-  if (c->cfg.in_kind == SSD_IN_BLOCK)
-    return fail(c, SSD_ERR_UNSUPPORTED, "the persistent forward kernel has no imitation-block program");
-  if (c->t5) return fail(c, SSD_ERR_UNSUPPORTED, "the persistent forward kernel has no encoder-decoder program");
-  return fwd_build_programs(c);
-}
-
 // Drafting stage: gamma tokens from layers 0..k-1, the imitation network and g.
 static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
-  if (c->use_fwd) return fwd_run(c, c->fwd_draft[gamma]);
   const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   for (int j = 0; j < gamma; ++j) {
     float* xj = c->xv + static_cast<size_t>(j) * d;
-    CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + j), xj, d,
+    CK(launch_k(c, ssd_embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + j), xj, d,
                 c->cfg.d_model, c->cfg.vocab, c->st));
     for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, j, 1, j));
     const float* hx = xj;
@@ -961,7 +585,7 @@ static ssd_status enqueue_draft(ssd_ctx* c, int gamma) {
       CKS(gemv(c, Epi::RESID, 1, c->in2, p));
       hx = c->xt;
     }
-    CKS(enqueue_head(c, hx, 1, j, tok_in + j + 1, false));
+    CKS(enqueue_draft_head(c, hx, j, tok_in + j + 1));
   }
   return SSD_OK;
 }
@@ -973,20 +597,15 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
   const int d = c->dp;
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
-  if (c->use_fwd) {
-    CKS(fwd_run(c, c->fwd_verify[gamma]));
-    CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, cond,
-                has_cond));
-    return SSD_OK;
-  }
-  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
+  CK(launch_k(c, ssd_embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in + gamma),
               c->xv + static_cast<size_t>(gamma) * d, d, c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer(c, l, gamma, 1, gamma));
   if (c->cfg.in_kind == SSD_IN_BLOCK)  // the imitation block's cache row of d_gamma's x_k
     CKS(enqueue_qkv_only(c, c->cfg.n_layers, c->xv + static_cast<size_t>(gamma) * d, 1, gamma));
   for (int l = c->cfg.draft_exit_k; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, gamma + 1, 0));
   CKS(enqueue_head(c, c->xv, gamma + 1, 0, full_tok, true));
-  CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, cond,
+  CK(launch_k(c, ssd_accept_kernel, dim3(1), dim3(32), 0, c->st, gamma, c->out_int, c->cfg.max_seq, c->step_log,
+              c->cfg.max_seq, cond,
               has_cond));
   return SSD_OK;
 }
@@ -994,17 +613,12 @@ static ssd_status enqueue_verify(ssd_ctx* c, int gamma, cudaGraphConditionalHand
 static ssd_status enqueue_greedy_step(ssd_ctx* c, cudaGraphConditionalHandle cond, int has_cond) {
   int* tok_in = st_field(c, offsetof(DevState, tok_in));
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
-  if (c->use_fwd) {
-    CKS(fwd_run(c, c->fwd_greedy));
-    CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond,
-                has_cond));
-    return SSD_OK;
-  }
-  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv, c->dp,
+  CK(launch_k(c, ssd_embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(tok_in), c->xv, c->dp,
               c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
   CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
-  CK(launch_k(c, greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, cond, has_cond));
+  CK(launch_k(c, ssd_greedy_accept_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, c->cfg.max_seq, c->step_log,
+              c->cfg.max_seq, cond, has_cond));
   return SSD_OK;
 }
 
@@ -1014,11 +628,11 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
   CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
-  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
+  CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
   int r0 = 0;
   for (; r0 < P; r0 += kPrefillChunk) {
     const int Mc = P - r0 < kPrefillChunk ? P - r0 : kPrefillChunk;
-    CK(launch_k(c, prefill_rows_kernel, dim3(Mc), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+    CK(launch_k(c, ssd_prefill_rows_kernel, dim3(Mc), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
                 static_cast<const int*>(c->in_prompt), n_vis, r0, c->embed, c->cfg.vocab, c->xv, d, c->cfg.d_model, c->st));
     for (int l = 0; l < c->cfg.n_layers; ++l) {
       if (l == c->cfg.draft_exit_k && c->cfg.in_kind == SSD_IN_BLOCK)  // the block's cache rows of x_k
@@ -1030,7 +644,7 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   }
   r0 -= kPrefillChunk;
   CKS(enqueue_head(c, c->xv + static_cast<size_t>(P - 1 - r0) * d, 1, P - 1, full_tok, true));
-  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
+  CK(launch_k(c, ssd_prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
   return SSD_OK;
 }
 
@@ -1044,8 +658,8 @@ static ssd_status enqueue_prefill_t5(ssd_ctx* c, int n_vis, int n_prompt) {
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
   CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
-  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 1, c->cfg.eos_id, P));
-  CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+  CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 1, c->cfg.eos_id, P));
+  CK(launch_k(c, ssd_prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_enc, dp, c->cfg.d_model,
               c->st));
   for (int e = 0; e < c->cfg.n_enc_layers; ++e) {
@@ -1116,11 +730,11 @@ static ssd_status enqueue_prefill_t5(ssd_ctx* c, int n_vis, int n_prompt) {
       p.max_seq = c->max_enc;
       CKS(gemv(c, Epi::QKV, Mc, c->cross_kv[l], p));
     }
-  CK(launch_k(c, embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(c->start_tok), c->xv, dp,
+  CK(launch_k(c, ssd_embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(c->start_tok), c->xv, dp,
               c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
   CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
-  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, 1));
+  CK(launch_k(c, ssd_prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, 1));
   return SSD_OK;
 }
 
@@ -1152,8 +766,8 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
   CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
-  CK(launch_k(c, prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
-  CK(launch_k(c, prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+  CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
+  CK(launch_k(c, ssd_prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
               c->st));
   // the IN_BLOCK block's cache rows of every prompt row's x_k: its QKV GEMM alone
@@ -1213,7 +827,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   }
   if (c->cfg.draft_exit_k == c->cfg.n_layers && c->cfg.in_kind == SSD_IN_BLOCK) CKS(block_kv());
   CKS(enqueue_head(c, c->x_pre + static_cast<size_t>(P - 1) * dp, 1, P - 1, full_tok, true));
-  CK(launch_k(c, prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
+  CK(launch_k(c, ssd_prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, P));
   return SSD_OK;
 }
 
@@ -1251,7 +865,7 @@ static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec,
     cfg.gridDim = dim3(1);
     cfg.blockDim = dim3(32);
     cfg.stream = c->cs;
-    e = cudaLaunchKernelEx(&cfg, loop_begin_kernel, c->st, cond);
+    e = cudaLaunchKernelEx(&cfg, ssd_loop_begin_kernel, c->st, cond);
     s = end_capture(c, g, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop_begin launch: %s",
                                                            cudaGetErrorString(e)));
   }
@@ -1340,7 +954,7 @@ static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
   }
   ssd_status s = begin_capture(c, g);
   if (s == SSD_OK) {
-    e = launch_plain(c, loop_begin_kernel, c->st, cond);
+    e = launch_plain(c, ssd_loop_begin_kernel, c->st, cond);
     s = end_capture(c, g, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop_begin: %s", cudaGetErrorString(e)));
   }
   cudaGraphNode_t begin = nullptr;
@@ -1362,7 +976,7 @@ static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
       s = fail(c, SSD_ERR_CUDA, "switch handle: %s", cudaGetErrorString(e));
     if (s == SSD_OK) s = begin_capture(c, body);
     if (s == SSD_OK) {
-      e = launch_plain(c, dyn_select_kernel, c->st, static_cast<const int*>(c->dyn_table),
+      e = launch_plain(c, ssd_dyn_select_kernel, c->st, static_cast<const int*>(c->dyn_table),
                        static_cast<const int*>(c->dyn_launch), cap, sw);
       s = end_capture(c, body, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "select: %s", cudaGetErrorString(e)));
     }
@@ -1393,7 +1007,7 @@ static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
           cudaSuccess)
         s = fail(c, SSD_ERR_CUDA, "capture after SWITCH: %s", cudaGetErrorString(e));
       if (s == SSD_OK) {
-        e = launch_plain(c, loop_continue_kernel, c->st, cond);
+        e = launch_plain(c, ssd_loop_continue_kernel, c->st, cond);
         s = end_capture(c, body, e == cudaSuccess ? SSD_OK : fail(c, SSD_ERR_CUDA, "loop test: %s", cudaGetErrorString(e)));
       }
     }
@@ -1421,7 +1035,6 @@ static ssd_status enq_step_fn(ssd_ctx* c, int g, int) {
 }
 
 static void drop_graphs(ssd_ctx* c) {
-  c->fwd_ready = false;  // phase lists hold the logits-capture pointer
   for (auto& kv : c->decode_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->draft_graphs) cudaGraphExecDestroy(kv.second);
   for (auto& kv : c->verify_graphs) cudaGraphExecDestroy(kv.second);
@@ -1495,9 +1108,8 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (!c) return SSD_OK;
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
-  void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
-                  c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt, c->fwd_phases, c->fwd_maps, c->fwd_flags,
-                  c->fwd_tickets, c->fwd_done, c->fwd_exit, c->fwd_partials, c->fwd_attn_part, c->fwd_trace, c->fwd_btiles,
+  void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->step_log, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
+                  c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt,
                   c->x_enc, c->enc_q, c->enc_o, c->enc_k, c->enc_v, c->ckc, c->cvc, c->dec_bias, c->enc_bias, c->one,
                   c->start_tok};
   for (void* b : bufs)
@@ -1542,7 +1154,7 @@ static ssd_status build_bias_table(ssd_ctx* c, const void* rel, float* out, int 
   cudaError_t e = cudaMemcpy(db, b.data(), sizeof(int) * n, cudaMemcpyHostToDevice);
   const int H = c->cfg.n_heads;
   if (e == cudaSuccess) {
-    bias_table_kernel<<<(n * H + 255) / 256, 256, 0, c->cs>>>(static_cast<const __nv_bfloat16*>(rel), db, n, H, out);
+    ssd_bias_table_kernel<<<(n * H + 255) / 256, 256, 0, c->cs>>>(static_cast<const __nv_bfloat16*>(rel), db, n, H, out);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->cs);
@@ -1611,17 +1223,10 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (prop.major != 10) return fail(c, SSD_ERR_UNSUPPORTED, "needs a Blackwell sm_103 device, got sm_%d%d",
                                     prop.major, prop.minor);
   c->num_sms = prop.multiProcessorCount;
-  if (const char* e = getenv("SSD_HOST_LOOP")) c->host_loop = atoi(e) != 0;
-  if (const char* e = getenv("SSD_GEMV_CTAS")) c->gemv_ctas = atoi(e) < 1 ? 1 : (atoi(e) > 3 ? 3 : atoi(e));
-  if (const char* e = getenv("SSD_PREFILL")) c->prefill_rows = strcmp(e, "rows") == 0;
-  if (const char* e = getenv("SSD_DECODE")) c->use_fwd = strcmp(e, "fwd") == 0;
-  if (const char* e = getenv("SSD_FWD_COOP")) c->fwd_coop = atoi(e) != 0;
-  if (const char* e = getenv("SSD_FWD_TRACE")) c->fwd_trace_path = e;
-  if (const char* e = getenv("SSD_GEMV_TRACE")) c->gemv_trace_path = e;
-  if (const char* e = getenv("SSD_GEMV_SMALL")) {  // "<row tiles>,<ctas per SM>"
-    c->small_site_rt = atoi(e);
-    if (const char* comma = strchr(e, ',')) c->small_site_ctas = atoi(comma + 1) < 1 ? 1 : atoi(comma + 1);
-  }
+  if (k.options & ~(SSD_OPT_HOST_LOOP | SSD_OPT_PREFILL_ROWS))
+    return fail(c, SSD_ERR_INVALID_ARG, "unknown option bits 0x%x", k.options);
+  c->host_loop = (k.options & SSD_OPT_HOST_LOOP) != 0;
+  c->prefill_rows = (k.options & SSD_OPT_PREFILL_ROWS) != 0;
   if (!g_encode) {
     cudaDriverEntryPointQueryResult q;
     void* fn = nullptr;
@@ -1636,7 +1241,6 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_head());
   CK(attn_attrs());
   CK(prefill_attrs());
-  CK(fwd_attrs());
 
   c->cfg = k;
   c->qdim = qdim;
@@ -1733,6 +1337,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CKS(alloc(c, reinterpret_cast<void**>(&c->st), sizeof(DevState)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->op_st), sizeof(DevState)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->out_int), sizeof(int) * k.max_seq));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->step_log), sizeof(int2) * k.max_seq));
   CKS(alloc(c, reinterpret_cast<void**>(&c->xv), sizeof(float) * R * c->dp));
   CKS(alloc(c, reinterpret_cast<void**>(&c->xt), sizeof(float) * R * c->dp));
   CKS(alloc(c, reinterpret_cast<void**>(&c->qb), sizeof(float) * R * c->qp));
@@ -1793,7 +1398,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     CK(cudaMemcpy(c->one, &one, sizeof(float), cudaMemcpyHostToDevice));
     CK(cudaMemcpy(c->start_tok, &k.start_token, sizeof(int), cudaMemcpyHostToDevice));
   }
-  CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * c->gemv_ctas * c->num_sms * R * kTileN));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->partials), sizeof(float) * 2 * kGemvCtasPerSm * c->num_sms * R * kTileN));
   int max_rt = 1;
   for (const Site* s : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->head,
                         &c->in1, &c->in2})
@@ -1828,45 +1433,12 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     }
   }
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * in_rows));
-  {
-    // persistent forward kernel: one CTA per SM, the weight maps of every projection in one table
-    int per_sm = 0;
-    CK(fwd_ctas_per_sm(k.head_dim, &per_sm));
-    if (per_sm < 1) return fail(c, SSD_ERR_UNSUPPORTED, "forward kernel does not fit on an SM");
-    c->fwd_grid = c->num_sms;
-    c->fwd_splits = std::max(1, std::min(kFwdMaxSplits, c->fwd_grid / k.n_heads));
-    std::vector<CUtensorMap> maps;
-    for (int l = 0; l < k.n_layers; ++l) {
-      const LayerSites& L = c->layers[l];
-      for (int i = 0; i < 3; ++i) maps.push_back(L.qkv.maps[i]);
-      maps.push_back(L.o.maps[0]);
-      maps.push_back(L.gateup.maps[0]);
-      maps.push_back(L.gateup.maps[1]);
-      maps.push_back(L.down.maps[0]);
-    }
-    maps.push_back(c->in1.maps[0]);
-    maps.push_back(c->in2.maps[0]);
-    maps.push_back(c->head.maps[0]);
-    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_maps), sizeof(CUtensorMap) * maps.size()));
-    CK(cudaMemcpy(c->fwd_maps, maps.data(), sizeof(CUtensorMap) * maps.size(), cudaMemcpyHostToDevice));
-    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_exit), sizeof(unsigned)));
-    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_partials),
-              sizeof(float) * kFwdWindow * c->fwd_grid * kFwdRows * kTileN));
-    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_attn_part),
-              sizeof(float) * kFwdWindow * k.n_heads * 4 * c->fwd_splits * kFwdRows * (k.head_dim + 2)));
-    int max_kt = c->head.n_kt;
-    for (const Site* st : {&c->layers[0].qkv, &c->layers[0].o, &c->layers[0].gateup, &c->layers[0].down, &c->in1,
-                           &c->in2})
-      max_kt = std::max(max_kt, st->n_kt);
-    c->fwd_bslot = static_cast<long long>(max_kt) * kFwdBTile;
-    CKS(alloc(c, reinterpret_cast<void**>(&c->fwd_btiles), static_cast<size_t>(kFwdBSlots) * c->fwd_bslot));
-  }
   CK(cudaStreamCreateWithFlags(&c->cs, cudaStreamNonBlocking));
   CK(cudaEventCreateWithFlags(&c->ev_in, cudaEventDisableTiming));
   CK(cudaEventCreateWithFlags(&c->ev_out, cudaEventDisableTiming));
   if (!t5) {  // the encoder-decoder model has no rotary embedding
     const int nrope = k.max_seq * (k.head_dim / 2);
-    rope_table_kernel<<<(nrope + 255) / 256, 256, 0, c->cs>>>(c->rope, k.max_seq, k.head_dim,
+    ssd_rope_table_kernel<<<(nrope + 255) / 256, 256, 0, c->cs>>>(c->rope, k.max_seq, k.head_dim,
                                                               static_cast<double>(k.rope_theta));
     CK(cudaGetLastError());
   }
@@ -1938,7 +1510,7 @@ ssd_status ssd_prefill(ssd_ctx* c, const void* vis, int n_vis, const int32_t* pr
   if (n_prompt > 0)
     CK(cudaMemcpyAsync(c->in_prompt, prompt, sizeof(int) * n_prompt, cudaMemcpyDeviceToDevice, c->cs));
   CKS(prefill_impl(c, n_vis, n_prompt));
-  if (first_tok) first_token_kernel<<<1, 32, 0, c->cs>>>(c->st, first_tok);
+  if (first_tok) ssd_first_token_kernel<<<1, 32, 0, c->cs>>>(c->st, first_tok);
   CK(cudaGetLastError());
   return leave(c);
 }
@@ -1948,7 +1520,6 @@ ssd_status ssd_draft(ssd_ctx* c, int gamma, int32_t* draft_tok) {
   if (!c->prefilled) return fail(c, SSD_ERR_STATE, "ssd_draft before ssd_prefill");
   if (gamma < 1 || gamma > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma %d", gamma);
   if (c->kv_upper + gamma + 1 > c->cfg.max_seq) return fail(c, SSD_ERR_CAPACITY, "KV cache full");
-  CKS(fwd_ensure(c));
   CKS(enter(c));
   auto it = c->draft_graphs.find(gamma);
   if (it == c->draft_graphs.end()) {
@@ -1957,7 +1528,7 @@ ssd_status ssd_draft(ssd_ctx* c, int gamma, int32_t* draft_tok) {
     it = c->draft_graphs.emplace(gamma, ge).first;
   }
   CK(cudaGraphLaunch(it->second, c->cs));
-  if (draft_tok) copy_draft_kernel<<<1, 32, 0, c->cs>>>(c->st, gamma, draft_tok);
+  if (draft_tok) ssd_copy_draft_kernel<<<1, 32, 0, c->cs>>>(c->st, gamma, draft_tok);
   CK(cudaGetLastError());
   c->drafted_gamma = gamma;
   return leave(c);
@@ -1967,7 +1538,6 @@ ssd_status ssd_verify(ssd_ctx* c, int gamma, int32_t* n_emitted, int32_t* emitte
   if (!c) return SSD_ERR_INVALID_ARG;
   if (!c->prefilled || c->drafted_gamma != gamma)
     return fail(c, SSD_ERR_STATE, "ssd_verify(gamma=%d) needs a preceding ssd_draft with the same gamma", gamma);
-  CKS(fwd_ensure(c));
   CKS(enter(c));
   auto it = c->verify_graphs.find(gamma);
   if (it == c->verify_graphs.end()) {
@@ -1976,7 +1546,7 @@ ssd_status ssd_verify(ssd_ctx* c, int gamma, int32_t* n_emitted, int32_t* emitte
     it = c->verify_graphs.emplace(gamma, ge).first;
   }
   CK(cudaGraphLaunch(it->second, c->cs));
-  if (n_emitted || emitted) copy_emitted_kernel<<<1, 32, 0, c->cs>>>(c->st, n_emitted, emitted);
+  if (n_emitted || emitted) ssd_copy_emitted_kernel<<<1, 32, 0, c->cs>>>(c->st, n_emitted, emitted);
   CK(cudaGetLastError());
   c->drafted_gamma = 0;
   c->kv_upper += gamma + 1;
@@ -1990,7 +1560,6 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
   if (static_cast<int64_t>(c->prompt_len) + max_new + gamma + 1 > c->cfg.max_seq)
     return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + gamma + 1 = %d > max_seq = %d",
                 c->prompt_len + max_new + gamma + 1, c->cfg.max_seq);
-  CKS(fwd_ensure(c));
   cudaGraphExec_t ge;
   if (c->host_loop) {
     auto it = c->step_graphs.find(gamma);
@@ -2000,7 +1569,7 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
       it = c->step_graphs.emplace(gamma, ge).first;
       if (gamma > 0) c->decode_body_launches[gamma] = nb; else c->greedy_body_launches = nb;
     }
-    decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
+    ssd_decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
     CK(cudaGetLastError());
     int done = 0;
     for (int it2 = 0; it2 < max_new && !done; ++it2) {
@@ -2009,7 +1578,7 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
                          cudaMemcpyDeviceToHost, c->cs));
       CK(cudaStreamSynchronize(c->cs));
     }
-    if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+    if (out_tok || n_out) ssd_copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
     CK(cudaGetLastError());
     c->last_decode_kind = gamma > 0 ? 1 : 2;
     c->last_gamma = gamma;
@@ -2030,10 +1599,10 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
     if (!c->greedy_graph) CKS(build_loop_graph(c, 0, &c->greedy_graph, &c->greedy_body_launches));
     ge = c->greedy_graph;
   }
-  decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
+  ssd_decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, gamma);
   CK(cudaGetLastError());
   CK(cudaGraphLaunch(ge, c->cs));
-  if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+  if (out_tok || n_out) ssd_copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
   CK(cudaGetLastError());
   c->last_decode_kind = gamma > 0 ? 1 : 2;
   c->last_gamma = gamma;
@@ -2051,7 +1620,6 @@ static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, in
   if (static_cast<int64_t>(c->prompt_len) + max_new + cap + 1 > c->cfg.max_seq)
     return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + cap + 1 = %d > max_seq = %d",
                 c->prompt_len + max_new + cap + 1, c->cfg.max_seq);
-  CKS(fwd_ensure(c));
   if (d0 != c->dyn_d0 || n_max != c->dyn_n) {  // the table of the previous schedule may still be read
     CK(cudaStreamSynchronize(c->cs));
     c->dyn_table_h.resize(c->cfg.max_seq + 1);
@@ -2060,7 +1628,7 @@ static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, in
     c->dyn_d0 = d0;
     c->dyn_n = n_max;
   }
-  decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, cap);
+  ssd_decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, cap);
   CK(cudaGetLastError());
   if (c->host_loop) {  // one plain graph per step; the host reads kv_len and picks the step's gamma
     c->dyn_host_launches = 0;
@@ -2090,7 +1658,7 @@ static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, in
     }
     CK(cudaGraphLaunch(it->second, c->cs));
   }
-  if (out_tok || n_out) copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
+  if (out_tok || n_out) ssd_copy_out_kernel<<<1, 256, 0, c->cs>>>(c->st, c->out_int, out_tok, n_out, max_new);
   CK(cudaGetLastError());
   c->last_decode_kind = 3;
   c->last_gamma = cap;
@@ -2133,17 +1701,6 @@ ssd_status ssd_sync(ssd_ctx* c) {
   if (!c) return SSD_ERR_INVALID_ARG;
   CK(cudaStreamSynchronize(c->cs));
   CK(cudaStreamSynchronize(c->us));
-  if (c->fwd_trace && c->fwd_trace_phases > 0) {  // diagnostic timeline of the last forward launch
-    const size_t n = static_cast<size_t>(c->fwd_grid) * (c->fwd_trace_phases + 1) * 16 + 4 * 8192 * 4;
-    std::vector<unsigned long long> h(n);
-    CK(cudaMemcpy(h.data(), c->fwd_trace, sizeof(unsigned long long) * n, cudaMemcpyDeviceToHost));
-    if (FILE* f = fopen(c->fwd_trace_path.c_str(), "wb")) {
-      const int hdr[2] = {c->fwd_grid, c->fwd_trace_phases};
-      fwrite(hdr, sizeof(int), 2, f);
-      fwrite(h.data(), sizeof(unsigned long long), n, f);
-      fclose(f);
-    }
-  }
   return read_device_error(c);
 }
 
@@ -2205,6 +1762,36 @@ ssd_status ssd_set_logits_capture(ssd_ctx* c, float* buf, int max_rows) {
   drop_graphs(c);
   c->logits_buf = buf;
   c->logits_rows = buf ? max_rows : 0;
+  return SSD_OK;
+}
+
+ssd_status ssd_set_draft_logits_capture(ssd_ctx* c, float* buf, int max_steps) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (buf && max_steps < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_steps %d", max_steps);
+  CK(cudaStreamSynchronize(c->cs));
+  drop_graphs(c);
+  c->draft_logits_buf = buf;
+  c->draft_logits_steps = buf ? max_steps : 0;
+  return SSD_OK;
+}
+
+ssd_status ssd_get_step_log(ssd_ctx* c, int32_t* accepted, int32_t* drafted, int cap, int* n_steps) {
+  if (!c || !n_steps || cap < 0 || (cap > 0 && !accepted && !drafted)) return SSD_ERR_INVALID_ARG;
+  CK(cudaStreamSynchronize(c->cs));
+  int steps = 0;
+  CK(cudaMemcpy(&steps, reinterpret_cast<char*>(c->st) + offsetof(DevState, steps), sizeof(int),
+                cudaMemcpyDeviceToHost));
+  steps = std::min(steps, c->cfg.max_seq);
+  const int n = std::min(steps, cap);
+  if (n > 0) {
+    std::vector<int2> h(n);
+    CK(cudaMemcpy(h.data(), c->step_log, sizeof(int2) * n, cudaMemcpyDeviceToHost));
+    for (int i = 0; i < n; ++i) {
+      if (accepted) accepted[i] = h[i].x;
+      if (drafted) drafted[i] = h[i].y;
+    }
+  }
+  *n_steps = steps;
   return SSD_OK;
 }
 
@@ -2291,26 +1878,8 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     const int64_t qd = static_cast<int64_t>(c->cfg.n_heads) * c->cfg.head_dim;
     if (bytes) *bytes = 2 * (kv + rows) * qd * 4 + 2 * static_cast<int64_t>(rows) * qd * 4;  // K, V; q in, o out
     CKS(enter(c));
-    const size_t ntr = static_cast<size_t>(8) * kAttnSplit * c->cfg.n_heads;
-    unsigned long long* tr = nullptr;
-    if (!c->gemv_trace_path.empty()) {  // diagnostic: timeline of the last launch, written here
-      CK(cudaMalloc(&tr, sizeof(unsigned long long) * ntr));
-      CK(cudaMemsetAsync(tr, 0, sizeof(unsigned long long) * ntr, c->cs));
-    }
-    for (int r = 0; r < reps; ++r) CKS(attention(c, layer, rows, 0, false, r == reps - 1 ? tr : nullptr));
+    for (int r = 0; r < reps; ++r) CKS(attention(c, layer, rows, 0, false));
     c->prefilled = false;
-    if (tr) {
-      std::vector<unsigned long long> h(ntr);
-      CK(cudaStreamSynchronize(c->cs));
-      CK(cudaMemcpy(h.data(), tr, sizeof(unsigned long long) * ntr, cudaMemcpyDeviceToHost));
-      CK(cudaFree(tr));
-      if (FILE* f = fopen(c->gemv_trace_path.c_str(), "ab")) {
-        const int hdr[4] = {which, rows, kAttnSplit * c->cfg.n_heads, 8};
-        fwrite(hdr, sizeof(int), 4, f);
-        fwrite(h.data(), sizeof(unsigned long long), ntr, f);
-        fclose(f);
-      }
-    }
     return leave(c);
   }
   if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))
@@ -2383,28 +1952,8 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     *bytes = N * site->K * 2 + static_cast<int64_t>(rows) * site->K * 4 + (p.gain ? site->K * 2 : 0) + out_bytes +
              (e == Epi::RESID ? static_cast<int64_t>(rows) * site->N * 4 : 0);
   CKS(enter(c));
-  unsigned long long* tr = nullptr;
-  if (!c->gemv_trace_path.empty()) {  // diagnostic: timeline of the last launch, written here
-    CK(cudaMalloc(&tr, sizeof(unsigned long long) * kGemvTrace * site->grid));
-    CK(cudaMemsetAsync(tr, 0, sizeof(unsigned long long) * kGemvTrace * site->grid, c->cs));
-  }
-  for (int r = 0; r < reps; ++r) {
-    p.trace = r == reps - 1 ? tr : nullptr;
-    CKS(gemv(c, e, rows, *site, p));
-  }
+  for (int r = 0; r < reps; ++r) CKS(gemv(c, e, rows, *site, p));
   c->prefilled = false;
-  if (tr) {
-    std::vector<unsigned long long> h(kGemvTrace * static_cast<size_t>(site->grid));
-    CK(cudaStreamSynchronize(c->cs));
-    CK(cudaMemcpy(h.data(), tr, sizeof(unsigned long long) * h.size(), cudaMemcpyDeviceToHost));
-    CK(cudaFree(tr));
-    if (FILE* f = fopen(c->gemv_trace_path.c_str(), "ab")) {
-      const int hdr[4] = {which, rows, site->grid, kGemvTrace};
-      fwrite(hdr, sizeof(int), 4, f);
-      fwrite(h.data(), sizeof(unsigned long long), h.size(), f);
-      fclose(f);
-    }
-  }
   return leave(c);
 }
 

@@ -47,8 +47,8 @@ constexpr int kHalfN = kTileN / 2;   // gate or up rows of a paired unit
 constexpr int kTileK = 64;           // weight columns per unit (one 128-byte swizzled row)
 constexpr int kNPad = 16;            // activation rows padded to the MMA's N
 constexpr int kStages = 4;
-constexpr int kGemvTrace = 12;  // timeline stamps per CTA
 constexpr int kGemvThreads = 256;
+constexpr int kGemvCtasPerSm = 2;   // persistent grid: min(units, 2 x #SMs) CTAs
 constexpr int kDrainThreads = 128;   // warps 4..7
 constexpr int kTmemCols = 32;        // two 16-column accumulators
 constexpr uint32_t kWTileBytes = kTileN * kTileK * 2;   // 16 KB
@@ -86,14 +86,11 @@ struct GemvParams {
   const float* scale;
   // ARGMAX
   int* tok_dst;        // tok_dst[m] = argmax of row m
-  float* logits;       // optional [logits_rows][N] capture
+  float* logits;       // optional [logits_rows][N] capture: row m's logits go to row position + 1 - P
+                       // (the index of the token it predicts), or with logits_step_rows > 0 to row
+                       // st->steps * logits_step_rows + pos_off + m (draft rows by step)
   int logits_rows;
-  // optional timeline, [grid][kGemvTrace] %globaltimer stamps per CTA: 0 entry, 1 first weight
-  // copies issued, 2 upstream grid complete, 3 first unit landed, 4 last MMA issued, 5 first
-  // accumulator drained, 6 epilogues done, 7 exit; for the last split tile this CTA owned:
-  // 8 ticket taken, 9 partials summed, 10 its epilogue done, 11 split tiles owned.  Null when
-  // not tracing.
-  unsigned long long* trace;
+  int logits_step_rows;
   // Trigger the dependent launch only once the upstream grid has completed (from the weight
   // producer, after its wait), so that everything older than this launch is complete when the
   // dependent grid starts: the split-KV attention after the QKV projection reads older cache rows
@@ -278,14 +275,16 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     }
   } else {  // ARGMAX (LM head): argmax over the vocabulary, lowest index on ties
     const int lane = tid & 31;
-    const int P = p.logits != nullptr ? __ldcg(&p.st->prompt_len) : 0;
+    const int row0 = p.logits == nullptr ? 0
+                     : p.logits_step_rows > 0 ? __ldcg(&p.st->steps) * p.logits_step_rows + p.pos_off
+                                              : base_pos + 1 - __ldcg(&p.st->prompt_len);
     const int n = rt * kTileN + tid;  // thread per tile row
     const bool valid = n < p.N;
 #pragma unroll
     for (int m = 0; m < M; ++m) {
       const float logit = out[m * kTileN + tid] * rs[m];
       if (p.logits != nullptr && valid) {
-        const int row = base_pos + m + 1 - P;
+        const int row = row0 + m;
         if (row >= 0 && row < p.logits_rows) p.logits[static_cast<size_t>(row) * p.N + n] = logit;
       }
       unsigned long long key = valid ? argmax_key(logit, static_cast<uint32_t>(n)) : 0ull;
@@ -303,9 +302,10 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(p.n_rt - 1);
     drain_sync();
     if (am_last) {
-      if (tid < M) {
+      if (tid < M) {  // -1 once a bounded wait anywhere has given up: the keys may miss tiles
         const unsigned long long key = atomicExch(&p.st->am_key[tid], 0ull);
-        p.tok_dst[tid] = static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
+        const bool stopped = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
+        p.tok_dst[tid] = stopped ? -1 : static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
       }
       if (tid == 0) atomicExch(&p.st->am_count, 0u);
     }
@@ -316,7 +316,7 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
 
 template <int M, Epi EPI>
 __global__ void __launch_bounds__(kGemvThreads, 2)
-    gemv_kernel(const __grid_constant__ CUtensorMap map0, const __grid_constant__ CUtensorMap map1,
+    ssd_wstream_kernel(const __grid_constant__ CUtensorMap map0, const __grid_constant__ CUtensorMap map1,
                 const __grid_constant__ CUtensorMap map2, const GemvParams p) {
   static_assert(M >= 1 && M <= kNPad, "activation rows");
   using S = GemvSmem<M>;
@@ -341,8 +341,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
   const uint32_t tx = kWTileBytes + S::kActBytes + (p.gain ? kTileK * 2 : 0);
 
   if (!p.late_trigger) pdl_trigger();
-  unsigned long long* tr = p.trace ? p.trace + static_cast<size_t>(c) * kGemvTrace : nullptr;
-  if (tr && tid == 0) tr[0] = globaltimer_ns();
   // After a timed-out wait anywhere in the decode, later kernels do nothing
   // (best-effort read before any copy is issued or TMEM is taken).
   if (*reinterpret_cast<volatile int*>(&p.st->error) & DERR_TIMEOUT) return;
@@ -406,10 +404,8 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         mbar_arrive_expect_tx(&full[i], tx);
         issue_weights(i, u0 + i);  // weights do not depend on the previous kernel
       }
-      if (tr) tr[1] = globaltimer_ns();
       pdl_wait();
       if (p.late_trigger) pdl_trigger();
-      if (tr) tr[2] = globaltimer_ns();
       for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
       for (int i = npre; i < n_units; ++i) {
         const int s = i % kStages;
@@ -456,7 +452,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
           seg_open = true;
         }
         umma_commit(&empty[s]);  // stage s may be refilled once these MMAs have read it
-        if (tr && i == n_units - 1) tr[4] = globaltimer_ns();
         if (kt == p.n_kt - 1 || i == n_units - 1) {
           umma_commit(&afull[sg & 1]);  // the row tile's accumulator is complete
           ++sg;
@@ -473,7 +468,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         set_error(p.st, DERR_TIMEOUT);
         break;
       }
-      if (tr && i == 0 && ct == 0) tr[3] = globaltimer_ns();
       const float* a = reinterpret_cast<const float*>(smem + S::kA + s * S::kActBytes);
       const __nv_bfloat16* g = reinterpret_cast<const __nv_bfloat16*>(smem + S::kG + s * kTileK * 2);
       uint8_t* bh = smem + S::kB + s * 2 * kBOpBytes;
@@ -581,7 +575,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         break;
       }
       tmem_fence_after();
-      if (tr && sg == 0 && dt == 0) tr[5] = globaltimer_ns();
       float v[kNPad];
       tmem_ld16(tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kNPad), v);
       tmem_fence_before();
@@ -609,10 +602,6 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         }
         drain_sync();
         if (flag[0]) {
-          if (tr && dt == 0) {
-            tr[8] = globaltimer_ns();
-            tr[11] += 1;
-          }
           // Sum the partials in CTA order, all rows at once.  Every CTA after c_first starts its
           // range inside this tile (slot 2 cc); c_first's slot depends on whether the tile is its
           // first one.  When this is the CTA's last segment its weight ring is idle (every MMA
@@ -672,24 +661,17 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
             }
           }
           drain_sync();
-          if (tr && dt == 0) tr[9] = globaltimer_ns();
           gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, dt);
           if (dt == 0) p.counters[rt] = 0u;
-          if (tr) {
-            drain_sync();
-            if (dt == 0) tr[10] = globaltimer_ns();
-          }
         }
       }
       drain_sync();
       seg_kt0 = 0;
       ++sg;
     }
-    if (tr && dt == 0) tr[6] = globaltimer_ns();
   }
   tmem_fence_before();
   __syncthreads();
-  if (tr && tid == 0) tr[7] = globaltimer_ns();
   if (warp == 1) {
     tmem_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols) : "memory");

@@ -1,4 +1,4 @@
-// Host-side launch helpers for gemv_kernel instantiations (one translation
+// Host-side launch helpers for ssd_wstream_kernel instantiations (one translation
 // unit per epilogue kind keeps compile times parallel).
 #pragma once
 
@@ -18,12 +18,12 @@ cudaError_t gemv_launch_m(const CUtensorMap* maps, const GemvParams& p, int grid
   at[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, gemv_kernel<M, EPI>, maps[0], maps[1], maps[2], p);
+  return cudaLaunchKernelEx(&cfg, ssd_wstream_kernel<M, EPI>, maps[0], maps[1], maps[2], p);
 }
 
 template <int M, Epi EPI>
 cudaError_t gemv_attr_m() {
-  return cudaFuncSetAttribute(gemv_kernel<M, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(ssd_wstream_kernel<M, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               GemvSmem<M>::kTotal);
 }
 

@@ -21,17 +21,17 @@ static cudaError_t launch_pdl(Kern kern, dim3 grid, dim3 block, size_t smem, cud
 
 cudaError_t prefill_attrs() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
+  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
     return e;
-  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::GATE_SILU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::GATE_SILU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 kTcSmem)))
     return e;
-  if ((e = cudaFuncSetAttribute(tc_gemm_kernel<Epi::RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
+  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
     return e;
-  if ((e = cudaFuncSetAttribute(prefill_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if ((e = cudaFuncSetAttribute(ssd_prefill_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 PaSmem<128>::kTotal)))
     return e;
-  return cudaFuncSetAttribute(prefill_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  return cudaFuncSetAttribute(ssd_prefill_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                               PaSmem<64>::kTotal);
 }
 
@@ -40,11 +40,11 @@ cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, co
   const dim3 g(grid), blk(kTcThreads);
   switch (e) {
     case Epi::QKV:
-      return launch_pdl(tc_gemm_kernel<Epi::QKV>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return launch_pdl(ssd_prefill_tc_kernel<Epi::QKV>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
     case Epi::GATE_SILU:
-      return launch_pdl(tc_gemm_kernel<Epi::GATE_SILU>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return launch_pdl(ssd_prefill_tc_kernel<Epi::GATE_SILU>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
     case Epi::RESID:
-      return launch_pdl(tc_gemm_kernel<Epi::RESID>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return launch_pdl(ssd_prefill_tc_kernel<Epi::RESID>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
     default:
       return cudaErrorInvalidValue;
   }
@@ -52,7 +52,7 @@ cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, co
 
 cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                               __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl) {
-  return launch_pdl(split_rows_kernel, dim3(rows), dim3(256), 0, s, pdl, x, x_stride, K, gain, eps, hi, lo);
+  return launch_pdl(ssd_split_rows_kernel, dim3(rows), dim3(256), 0, s, pdl, x, x_stride, K, gain, eps, hi, lo);
 }
 
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
@@ -60,9 +60,9 @@ cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, cons
                                 cudaStream_t s, bool pdl) {
   const dim3 grid((P + kPaQ - 1) / kPaQ, n_heads);
   if (head_dim == 128)
-    return launch_pdl(prefill_attn_kernel<128>, grid, dim3(256), PaSmem<128>::kTotal, s, pdl, q, q_stride, kc, vc,
+    return launch_pdl(ssd_prefill_attn_kernel<128>, grid, dim3(256), PaSmem<128>::kTotal, s, pdl, q, q_stride, kc, vc,
                       o, o_stride, P, max_seq, scale);
-  return launch_pdl(prefill_attn_kernel<64>, grid, dim3(256), PaSmem<64>::kTotal, s, pdl, q, q_stride, kc, vc, o,
+  return launch_pdl(ssd_prefill_attn_kernel<64>, grid, dim3(256), PaSmem<64>::kTotal, s, pdl, q, q_stride, kc, vc, o,
                     o_stride, P, max_seq, scale);
 }
 

@@ -84,7 +84,7 @@ __device__ __forceinline__ void tc_ld32(uint32_t taddr, float* v) {
 // Row r of `out_hi` / `out_lo` (bf16 [rows][K]) = split of x[r] (fp32), optionally
 // RMSNorm-scaled: v = x * rs * gain with rs = 1/sqrt(mean(x^2) + eps).
 // hi = bf16(v), lo = bf16(v - hi).
-__global__ void __launch_bounds__(256) split_rows_kernel(const float* __restrict__ x, int x_stride, int K,
+__global__ void __launch_bounds__(256) ssd_split_rows_kernel(const float* __restrict__ x, int x_stride, int K,
                                                          const __nv_bfloat16* __restrict__ gain, float eps,
                                                          __nv_bfloat16* __restrict__ out_hi,
                                                          __nv_bfloat16* __restrict__ out_lo) {
@@ -184,7 +184,7 @@ __device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int 
 
 template <Epi EPI>
 __global__ void __launch_bounds__(kTcThreads, 1)
-    tc_gemm_kernel(const __grid_constant__ CUtensorMap map_ahi, const __grid_constant__ CUtensorMap map_alo,
+    ssd_prefill_tc_kernel(const __grid_constant__ CUtensorMap map_ahi, const __grid_constant__ CUtensorMap map_alo,
                    const __grid_constant__ CUtensorMap map_b0, const __grid_constant__ CUtensorMap map_b1,
                    const __grid_constant__ CUtensorMap map_b2, const TcParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -354,7 +354,7 @@ struct PaSmem {
 };
 
 template <int DH>
-__global__ void __launch_bounds__(256) prefill_attn_kernel(const float* __restrict__ q, int q_stride,
+__global__ void __launch_bounds__(256) ssd_prefill_attn_kernel(const float* __restrict__ q, int q_stride,
                                                            const float* __restrict__ k_cache,
                                                            const float* __restrict__ v_cache, float* __restrict__ o,
                                                            int o_stride, int P, int max_seq, float scale) {

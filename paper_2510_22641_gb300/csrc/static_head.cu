@@ -39,7 +39,6 @@ static __device__ __align__(256) StaticScratch g_head_scratch;
 
 struct DeviceSetup {
   bool done = false;
-  cudaError_t status = cudaSuccess;
   StaticScratch* scratch = nullptr;  // device address of g_head_scratch on this device
   int num_sms = 0;
 };
@@ -53,21 +52,21 @@ PFN_cuTensorMapEncodeTiled_v12000 g_encode_static = nullptr;
 cudaError_t setup_device(int dev, DeviceSetup** out) {
   std::lock_guard<std::mutex> lk(g_setup_mu);
   DeviceSetup& s = g_setup[dev];
-  if (!s.done) {
-    s.done = true;
-    s.status = cudaGetSymbolAddress(reinterpret_cast<void**>(&s.scratch), g_head_scratch);
-    if (s.status == cudaSuccess) s.status = cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (s.status == cudaSuccess) s.status = gemv_attrs_head();
-    if (s.status == cudaSuccess && !g_encode_static) {
-      cudaDriverEntryPointQueryResult q;
-      void* fn = nullptr;
-      s.status = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
-      if (s.status == cudaSuccess && (q != cudaDriverEntryPointSuccess || !fn)) s.status = cudaErrorNotSupported;
-      if (s.status == cudaSuccess) g_encode_static = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    }
-  }
   *out = &s;
-  return s.status;
+  if (s.done) return cudaSuccess;
+  // a failed set-up is not cached: the next call on this device tries again
+  cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void**>(&s.scratch), g_head_scratch);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&s.num_sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = gemv_attrs_head();
+  if (e == cudaSuccess && !g_encode_static) {
+    cudaDriverEntryPointQueryResult q;
+    void* fn = nullptr;
+    e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+    if (e == cudaSuccess && (q != cudaDriverEntryPointSuccess || !fn)) e = cudaErrorNotSupported;
+    if (e == cudaSuccess) g_encode_static = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+  }
+  s.done = e == cudaSuccess;
+  return e;
 }
 
 }  // namespace
@@ -84,9 +83,14 @@ ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const
   if (al % 16 != 0) return SSD_ERR_INVALID_ARG;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kStaticMaxDevices) return SSD_ERR_CUDA;
+  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
+  if (stream) {  // the array's address below is the current device's: the stream must belong to it
+    int sdev = -1;
+    if (cudaStreamGetDevice(stream, &sdev) != cudaSuccess) return SSD_ERR_CUDA;
+    if (sdev != dev) return SSD_ERR_INVALID_ARG;
+  }
   DeviceSetup* ds = nullptr;
   if (setup_device(dev, &ds) != cudaSuccess) return SSD_ERR_CUDA;
-  cudaStream_t stream = static_cast<cudaStream_t>(cuda_stream);
 
   CUtensorMap maps[3];
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(d_model), static_cast<cuuint64_t>(vocab)};
@@ -124,7 +128,9 @@ ssd_status ssd_lm_head_static(const void* lm_head, const void* final_norm, const
 
   // The array keeps the previous call's contents: clear the state and the
   // tickets this call uses (the kernel leaves them at zero, but a call that
-  // stopped early might not have).
+  // stopped early might not have).  tok starts at -1, which a call whose
+  // kernel gave up on a bounded wait leaves in place.
+  if (cudaMemsetAsync(tok, 0xFF, sizeof(int32_t) * rows, stream) != cudaSuccess) return SSD_ERR_CUDA;
   if (cudaMemsetAsync(&sc->st, 0, sizeof(DevState), stream) != cudaSuccess) return SSD_ERR_CUDA;
   if (cudaMemsetAsync(sc->counters, 0, sizeof(unsigned) * p.n_rt, stream) != cudaSuccess) return SSD_ERR_CUDA;
   if (gemv_launch_head(rows, maps, p, grid, stream, false) != cudaSuccess) return SSD_ERR_CUDA;

@@ -195,6 +195,19 @@ class SSDModel:
     def set_logits_capture(self, buf: torch.Tensor | None):
         self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
 
+    def set_draft_logits_capture(self, buf: torch.Tensor | None):
+        """buf: device fp32 [max_steps][gamma_max][vocab]; draft j of step s writes buf[s][j]."""
+        self._call("ssd_set_draft_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
+
+    def step_log(self, cap: int = 4096) -> tuple[list, list]:
+        """(accepted a, drafted gamma_eff) of every step since the last prefill."""
+        acc = np.zeros(cap, dtype=np.int32)
+        dr = np.zeros(cap, dtype=np.int32)
+        n = ctypes.c_int(0)
+        self._call("ssd_get_step_log", acc.ctypes.data, dr.ctypes.data, cap, ctypes.byref(n))
+        m = min(n.value, cap)
+        return acc[:m].tolist(), dr[:m].tolist()
+
     def kv(self):
         """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (fp32) of the library's cache
         ([L + 1] with the block imitation network, whose rows are slot L)."""

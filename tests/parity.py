@@ -4,7 +4,9 @@ Tolerances (stated for a bf16-weight, fp32-activation path against fp64):
   logits:  |gpu - ref| <= 3e-2 + 2e-2 * |ref|   (3e-2 absolute / 2e-2 relative)
   tokens:  identical, except that once the oracle's top-1/top-2 logit margin
            at a position is below 1e-2 the two streams may part from there on;
-  accept lengths and KV lengths: bit-exact over the steps before the streams part.
+  accept lengths and KV lengths: bit-exact over the steps before the streams part;
+  draft logits g(I(x_k)): the same logit tolerance for every draft row of those steps up to the
+           first draft whose token differs, which must sit at an oracle draft margin below 1e-2.
 """
 from __future__ import annotations
 
@@ -53,3 +55,33 @@ def steps_before(accept_lengths, n_tokens_agreeing: int) -> int:
         pos += a + 1
         k += 1
     return k
+
+
+def assert_step_log(accepted, drafted, ref, n_tokens_agreeing: int) -> int:
+    """The device's per-step (a, gamma_eff) record equals the oracle's accept lengths and draft
+    counts over every step before the streams part (all steps when they never part)."""
+    k = steps_before(ref.accept_lengths, n_tokens_agreeing)
+    if n_tokens_agreeing == len(ref.tokens):
+        k = len(ref.accept_lengths)
+        assert len(accepted) == k, (len(accepted), k)
+    assert list(accepted[:k]) == list(ref.accept_lengths[:k]), (accepted[:k], ref.accept_lengths[:k])
+    assert list(drafted[:k]) == [len(d) for d in ref.draft_tokens[:k]]
+    return k
+
+
+def assert_draft_logits(draft_logits: np.ndarray, ref, n_steps: int) -> int:
+    """draft_logits[s][j]: the GPU's g(I(x_k)) of draft j in step s.  For the first n_steps steps,
+    every draft row the oracle computed is compared at the logit tolerance until the first draft
+    token that differs (argmax of the GPU row vs the oracle's d_{j+1}); that one must be a near-tie
+    of the oracle's draft logits, after which the step's later drafts see other inputs.  Returns
+    the number of rows compared."""
+    rows = 0
+    for s in range(n_steps):
+        for j, ref_row in enumerate(ref.draft_logits[s]):
+            assert_logits_close(draft_logits[s][j], ref_row, f"draft logits of step {s} row {j}")
+            rows += 1
+            if int(np.argmax(draft_logits[s][j])) != ref.draft_tokens[s][j]:
+                m = margin(ref_row)
+                assert m < MARGIN, f"draft {j} of step {s} differs at oracle margin {m:.4g}"
+                break
+    return rows

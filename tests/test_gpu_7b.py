@@ -16,7 +16,7 @@ import oracle
 import paper_2510_22641_gb300 as lib
 import synth
 from tests.gpu_util import device_weights
-from tests.parity import assert_logits_close, common_prefix, steps_before
+from tests.parity import assert_draft_logits, assert_logits_close, common_prefix, steps_before
 
 pytestmark = pytest.mark.gpu
 
@@ -71,29 +71,40 @@ def test_ssd_equals_greedy_all_tokens(big, s):
     set_s(model, W.s)
 
 
-def test_sampled_prefix_matches_oracle(big):
+@pytest.mark.parametrize("s", [0.05, 0.2])
+def test_sampled_prefix_matches_oracle(big, s):
+    """The first 8 SSD steps against the fp64 oracle: tokens, the full-model logits of every emitted
+    token, the drafting stage's logits g(I(x_k)), and the per-step accept lengths and draft counts
+    (bit-exact).  s = 0.05 accepts most drafts, so verification rows with accepted drafts are
+    exercised; s = 0.2 is the headline setting."""
     model, bits, vis, prompt, v, p = big
-    set_s(model, W.s)
+    set_s(model, s)
+    steps = 8
     logits = torch.zeros((W.max_new, W.shape.vocab), device="cuda")
+    dlog = torch.zeros((steps, lib.SSD_MAX_GAMMA, W.shape.vocab), device="cuda")
+    model.set_draft_logits_capture(dlog)
     toks, st = decode(model, v, p, W.gamma, logits)
+    acc, dr = model.step_log()
     model.set_logits_capture(None)
-    m = oracle.model_from_bits(W, bits, synth.bf16_to_f64)
-    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, W.max_new, W.gamma, max_steps=3)
+    model.set_draft_logits_capture(None)
+    w = W.replace(s=s)
+    m = oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, W.max_new, W.gamma, max_steps=steps,
+                              keep_draft_logits=True)
+    assert len(ref.accept_lengths) == steps
     n_ref = len(ref.tokens)
     agree = common_prefix(toks[:n_ref], ref.tokens, ref.logits)
     lg = logits.cpu().numpy()
     for t in range(min(agree + 1, n_ref)):
         assert_logits_close(lg[t], ref.logits[t], f"7B logits of token {t}")
     k = steps_before(ref.accept_lengths, agree)
-    assert k >= 1 or agree < 2
-    # the GPU's first k steps accepted exactly what the oracle's did: re-run them step by step
-    _, _, _ = None, None, None
-    first = torch.zeros(1, dtype=torch.int32, device="cuda")
-    model.prefill(v, p, first)
-    ne = torch.zeros(1, dtype=torch.int32, device="cuda")
-    for step in range(k):
-        model.draft(W.gamma)
-        model.verify(W.gamma, ne)
-        model.sync()
-        assert int(ne.item()) == ref.accept_lengths[step] + 1
-    assert int(first.item()) == ref.tokens[0]
+    assert acc[:k] == ref.accept_lengths[:k]
+    assert dr[:k] == [len(d) for d in ref.draft_tokens[:k]]
+    rows = assert_draft_logits(dlog.cpu().numpy(), ref, k)
+    # the compared prefix may end early only at an oracle near-tie (common_prefix checks the
+    # margin); with these seeds the first 8 steps agree at both settings
+    assert k == steps and agree == n_ref, (k, agree, n_ref)
+    assert rows >= steps
+    if s == 0.05:
+        assert sum(ref.accept_lengths) >= steps  # verification rows with accepted drafts occur
+    set_s(model, W.s)

@@ -14,7 +14,7 @@ import oracle
 import paper_2510_22641_gb300 as lib
 import synth
 from tests.gpu_util import device_inputs, make_model
-from tests.parity import assert_logits_close, common_prefix, steps_before
+from tests.parity import assert_draft_logits, assert_logits_close, assert_step_log, common_prefix, steps_before
 
 pytestmark = pytest.mark.gpu
 
@@ -24,14 +24,19 @@ def run_oracle(w, bits, gamma=None, greedy=False):
     vis, prompt = synth.make_inputs(w)
     if greedy:
         return oracle.greedy_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, max_seq=w.max_seq())
-    return oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma or w.gamma)
+    return oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma or w.gamma,
+                               keep_draft_logits=True)
 
 
 def gpu_decode(model, w, gamma, capture=True):
-    """prefill + decode through the device-buffer entry points; returns tokens, logits, stats."""
+    """prefill + decode through the device-buffer entry points; returns tokens, logits, stats (with
+    capture, stats["draft_logits"] holds the drafting stage's logits [step][j][vocab])."""
     _, _, v, p = device_inputs(w)
     logits = torch.full((w.max_new, w.shape.vocab), float("nan"), device="cuda") if capture else None
+    dlog = (torch.full((w.max_new, model.cfg["gamma_max"], w.shape.vocab), float("nan"), device="cuda")
+            if capture and gamma > 0 else None)
     model.set_logits_capture(logits)
+    model.set_draft_logits_capture(dlog)
     out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
     n = torch.zeros(1, dtype=torch.int32, device="cuda")
     model.prefill(v, p)
@@ -41,23 +46,39 @@ def gpu_decode(model, w, gamma, capture=True):
         model.greedy_decode(w.max_new, out, n)
     model.sync()
     toks = out[: int(n.item())].cpu().tolist()
-    return toks, (logits.cpu().numpy() if capture else None), model.stats()
+    stats = model.stats()
+    stats["accepted_log"], stats["drafted_log"] = model.step_log()
+    if dlog is not None:
+        stats["draft_logits"] = dlog.cpu().numpy()
+    model.set_draft_logits_capture(None)
+    return toks, (logits.cpu().numpy() if capture else None), stats
 
 
 def check_against_oracle(toks, logits, stats, ref, gamma):
+    """Tokens up to an excused near-tie, full-model logits of every agreeing token, and for SSD the
+    per-step accept lengths and draft counts (bit-exact), the counters, and the draft logits."""
     agree = common_prefix(toks, ref.tokens, ref.logits)
     for t in range(min(agree + 1, len(ref.tokens))):
         assert_logits_close(logits[t], ref.logits[t], f"logits of token {t}")
     if gamma > 0:
-        k = steps_before(ref.accept_lengths, agree)
-        hist = np.bincount(ref.accept_lengths[:k], minlength=synth.LLAVA7B.gamma + 4)
+        k = assert_step_log(stats["accepted_log"], stats["drafted_log"], ref, agree)
         if agree == len(ref.tokens):
             assert stats["steps"] == len(ref.accept_lengths)
             assert stats["accepted"] == sum(ref.accept_lengths)
             assert stats["kv_len"] == ref.kv_len
             assert stats["accept_hist"][: gamma + 1] == np.bincount(ref.accept_lengths, minlength=gamma + 1).tolist()
-        assert k <= stats["steps"] and hist.sum() == k
+        assert k <= stats["steps"]
+        if "draft_logits" in stats and ref.draft_logits:
+            # at least the first draft row of every compared step that drafted anything
+            assert assert_draft_logits(stats["draft_logits"], ref, k) >= sum(1 for d in ref.draft_tokens[:k] if d)
     return agree
+
+
+def assert_accept_sequence(model, ref, toks):
+    """The device's per-step record against the oracle's, over the steps before the streams part
+    (toks may be a prefix of the oracle's stream)."""
+    acc, dr = model.step_log()
+    assert_step_log(acc, dr, ref, common_prefix(toks, ref.tokens[: len(toks)], ref.logits))
 
 
 @pytest.fixture(scope="module")
@@ -104,25 +125,41 @@ def test_ssd_matches_oracle_and_gpu_greedy(tiny_model, tiny_bits, s, gamma):
     assert stats["steps"] + stats["accepted"] + 1 == w.max_new
 
 
+@pytest.fixture(scope="module")
+def tiny_model_host_loop(tiny_bits):
+    """The same context driven from the host, one plain graph per step (SSD_OPT_HOST_LOOP)."""
+    w = synth.TINY.replace(norm_gain="perturbed", gamma=8)
+    model, _, dev = make_model(w, tiny_bits, gamma_max=8, max_seq=w.max_seq(), options=lib.SSD_OPT_HOST_LOOP)
+    yield model, dev
+    model.close()
+
+
+@pytest.mark.parametrize("host", [False, True], ids=["device_loop", "host_loop"])
 @pytest.mark.parametrize("s,cap,n_max", [(0.05, 8, 120), (0.2, 6, 90), (1.0, 8, 40)])
-def test_dynamic_draft_length_matches_oracle(tiny_model, tiny_bits, s, cap, n_max):
+def test_dynamic_draft_length_matches_oracle(request, tiny_bits, s, cap, n_max, host):
     """Sec. "Choice of d": each step drafts min(d(kv_len + 2), cap) tokens; tokens, logits, steps,
     accept lengths and kv_len match the oracle's dynamic run, and the tokens equal greedy decoding."""
-    model, _ = tiny_model
+    model, _ = request.getfixturevalue("tiny_model_host_loop" if host else "tiny_model")
     w = synth.TINY.replace(norm_gain="perturbed", s=s)
     set_scale(model, w)
     _, _, v, p = device_inputs(w)
     logits = torch.full((w.max_new, w.shape.vocab), float("nan"), device="cuda")
+    dlog = torch.full((w.max_new, 8, w.shape.vocab), float("nan"), device="cuda")
     model.set_logits_capture(logits)
+    model.set_draft_logits_capture(dlog)
     out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
     n = torch.zeros(1, dtype=torch.int32, device="cuda")
     model.prefill(v, p)
     model.decode_dynamic(w.max_new, 5, n_max, cap, out, n)
     model.sync()
     toks, stats = out[: int(n.item())].cpu().tolist(), model.stats()
+    stats["accepted_log"], stats["drafted_log"] = model.step_log()
+    stats["draft_logits"] = dlog.cpu().numpy()
+    model.set_draft_logits_capture(None)
     m = oracle.model_from_bits(w, tiny_bits, synth.bf16_to_f64)
     vis, prompt = synth.make_inputs(w)
-    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, cap, dynamic=(5, n_max))
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, cap, dynamic=(5, n_max),
+                              keep_draft_logits=True)
     _, dec = model.launch_counts()
     check_against_oracle(toks, logits.cpu().numpy(), stats, ref, cap)
     assert stats["drafted"] == sum(len(d) for d in ref.draft_tokens)
@@ -131,9 +168,7 @@ def test_dynamic_draft_length_matches_oracle(tiny_model, tiny_bits, s, cap, n_ma
     # launches: setup, loop test at entry, copy-out; per step the branch for gamma_t plus its
     # selection (and, in the device loop, the loop test)
     L, k = w.shape.n_layers, w.draft_exit_k
-    fwd = os.environ.get("SSD_DECODE") == "fwd"
-    host = os.environ.get("SSD_HOST_LOOP", "0") not in ("", "0")
-    body = lambda g: 3 if fwd else g * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
+    body = lambda g: g * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
     p_, expect = w.prompt_len, 0
     for kv in ref.kv_lens:
         g_t = min(oracle.draft_length(p_ + 2, 5, n_max), cap)
@@ -214,6 +249,7 @@ def test_standalone_draft_and_verify_steps(tiny_model, tiny_bits):
         toks += em[:n].cpu().tolist()
     common_prefix(toks, ref.tokens[: len(toks)], ref.logits)
     assert len(toks) > 4
+    assert_accept_sequence(model, ref, toks)
 
 
 @pytest.mark.parametrize("case", ["ragged_prefill", "vocab_tail", "no_visual", "head128", "narrow_in",
@@ -304,12 +340,7 @@ def test_launch_counts(tiny_model):
     _, _, st = gpu_decode(model, w, 4, capture=False)
     pre, dec = model.launch_counts()
     L, k = w.shape.n_layers, w.draft_exit_k
-    if os.environ.get("SSD_DECODE") == "fwd":
-        # one persistent forward launch for the gamma = 4 drafting passes, one for the
-        # verification pass, and the acceptance kernel
-        body = 3
-    else:
-        body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
+    body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
     # + decode setup, loop begin and copy-out
     assert dec == 3 + st["steps"] * body
     # prefill: begin + input rows, per layer 4 activation splits + 4 tensor-core GEMMs + attention, head + finish
@@ -339,16 +370,15 @@ def test_lm_head_op_matches_oracle(tiny_model, tiny_bits, rows):
 
 
 @pytest.mark.parametrize("case", ["tiny", "ragged"])
-def test_tensor_core_prefill_matches_row_prefill_and_oracle(case, monkeypatch):
+def test_tensor_core_prefill_matches_row_prefill_and_oracle(case):
     """The tcgen05 prefill (hi/lo bf16 split, fp32 accumulation) against the row-chunked decode-kernel prefill."""
     w = synth.TINY.replace(norm_gain="perturbed", max_new=2)
     if case == "ragged":
         w = w.replace(n_vis=131, n_prompt=14)              # P = 145: a partial 128-row tile and 64-query block
     bits = synth.make_weights(w)
     caches = []
-    for mode in ("rows", "tc"):
-        monkeypatch.setenv("SSD_PREFILL", mode)
-        model, _, _ = make_model(w, bits)
+    for options in (lib.SSD_OPT_PREFILL_ROWS, 0):
+        model, _, _ = make_model(w, bits, options=options)
         toks, _, _ = gpu_decode(model, w, 0, capture=False)
         k, v, n = model.kv()
         P = w.prompt_len
@@ -425,14 +455,11 @@ def test_in_block_imitation_matches_oracle(block_model, block_bits, s, gamma):
     model = block_model
     w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=s)
     set_scale(model, w)
-    if os.environ.get("SSD_DECODE") == "fwd":
-        with pytest.raises(lib.SSDError, match="UNSUPPORTED"):
-            gpu_decode(model, w, gamma)
-        return
     toks, logits, stats = gpu_decode(model, w, gamma)
     m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
     vis, prompt = synth.make_inputs(w)
-    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma, keep_cache=True)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, gamma, keep_cache=True,
+                              keep_draft_logits=True)
     agree = check_against_oracle(toks, logits, stats, ref, gamma)
     K, V, n = model.kv()
     L = w.shape.n_layers
@@ -454,16 +481,13 @@ def test_in_block_with_dynamic_draft_length_matches_oracle(block_model, block_bi
     n = torch.zeros(1, dtype=torch.int32, device="cuda")
     model.set_logits_capture(None)
     model.prefill(v, p)
-    if os.environ.get("SSD_DECODE") == "fwd":
-        with pytest.raises(lib.SSDError, match="UNSUPPORTED"):
-            model.decode_dynamic(w.max_new, 5, 120, 8, out, n)
-        return
     model.decode_dynamic(w.max_new, 5, 120, 8, out, n)
     model.sync()
     toks, stats = out[: int(n.item())].cpu().tolist(), model.stats()
     m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
     vis, prompt = synth.make_inputs(w)
     ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 8, dynamic=(5, 120))
+    assert_accept_sequence(model, ref, toks)
     agree = common_prefix(toks, ref.tokens, ref.logits)
     if agree == len(ref.tokens):
         assert stats["steps"] == len(ref.accept_lengths)
@@ -474,15 +498,13 @@ def test_in_block_with_dynamic_draft_length_matches_oracle(block_model, block_bi
 def test_in_block_draft_exit_at_last_layer(block_bits):
     """k = L: the block's prompt rows come from the final x_L rows (after the last layer), and the
     verification pass has no deep layers; tokens and stats match the oracle."""
-    if os.environ.get("SSD_DECODE") == "fwd":
-        pytest.skip("the persistent forward kernel path has no imitation-block program")
     w = synth.TINY_BLOCK.replace(norm_gain="perturbed", s=0.2, draft_exit_k=4, gamma=4)
     model, _, _ = make_model(w, block_bits, gamma_max=4, max_seq=w.max_seq())
     try:
         toks, logits, stats = gpu_decode(model, w, 4)
         m = oracle.model_from_bits(w, block_bits, synth.bf16_to_f64)
         vis, prompt = synth.make_inputs(w)
-        ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 4)
+        ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 4, keep_draft_logits=True)
         check_against_oracle(toks, logits, stats, ref, 4)
     finally:
         model.close()
