@@ -45,7 +45,7 @@ METRIC = "tokens/s and speedup vs full-model greedy decode (7B shape, bs1); HBM 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up GEMV
 # launch from an ncu capture, valid only for the kernel source it was taken on.
-GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "8dbe91b28c5a66ff", "bytes": 182_967_552}
+GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "d5bddf15d880f543", "bytes": 183_015_168}
 UNIT = "tokens/s"
 S_VALUES = synth.LLAVA7B_S_VALUES
 
