@@ -68,9 +68,17 @@ def algorithmic_bytes(w: synth.Workload) -> dict:
     head = 2 * sh.vocab * sh.d_model
     imit = 2 * 2 * sh.d_model * w.in_hidden if w.in_kind == synth.IN_MLP2 else 0
     kv_pos = 2 * sh.n_heads * sh.head_dim * 2
-    return {"layer": layer, "head": head, "imit": imit, "kv_pos_layer": kv_pos,
+    return {"layer": layer, "head": head, "imit": imit, "kv_pos_layer": kv_pos, "kv_pos_layer_f32": 2 * kv_pos,
             "draft_token": w.draft_exit_k * layer + imit + head,
             "verify": sh.n_layers * layer + head, "greedy_token": sh.n_layers * layer + head}
+
+
+def measured_peak(key: str, fallback: float = 6800.0) -> float:
+    """A roofline denominator from MEASURED_PEAKS.json (the machine's measured copy / GEMM peaks)."""
+    try:
+        return float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))[key])
+    except (OSError, KeyError, ValueError):
+        return fallback
 
 
 KERNEL_ROWS = (("qkv", "ssd_wstream_kernel<M, QKV> (q/k/v + RoPE + KV write)"),
@@ -417,6 +425,178 @@ def run_encdec(args) -> None:
           flush=True)
 
 
+BATCH_KERNEL_ROWS = (("qkv", "ssd_wstream_mid_kernel<QKV> (q/k/v + RoPE + KV write)"),
+                     ("o", "ssd_wstream_mid_kernel<RESID> (o_proj)"),
+                     ("gateup", "ssd_wstream_mid_kernel<GATE_SILU> (gate/up)"),
+                     ("down", "ssd_wstream_mid_kernel<RESID> (down)"),
+                     ("head", "ssd_wstream_mid_kernel<ARGMAX> (LM head)"))
+
+
+def batch_algorithmic_bytes(w: synth.Workload, prompts, accept_logs, gamma: int) -> dict:
+    """Bytes a batched decode must move: per step the drafting stage's weights gamma times, the
+    verification pass's weights once, and the K/V of every active request read once per drafting
+    row and once per verification pass (positions up to the row; fp32 K and V)."""
+    ab = algorithmic_bytes(w)
+    sh = w.shape
+    L, k = sh.n_layers, w.draft_exit_k
+    steps = max(len(a) for a in accept_logs)
+    weights = kv = 0
+    kv_len = list(prompts)
+    for s in range(steps):
+        weights += gamma * ab["draft_token"] + ab["verify"] if gamma > 0 else ab["greedy_token"]
+        for b, acc in enumerate(accept_logs):
+            if s >= len(acc):
+                continue
+            if gamma > 0:
+                kv += sum(k * (kv_len[b] + j + 1) for j in range(gamma)) * ab["kv_pos_layer_f32"]
+                kv += L * (kv_len[b] + gamma + 1) * ab["kv_pos_layer_f32"]
+            else:
+                kv += L * (kv_len[b] + 1) * ab["kv_pos_layer_f32"]
+            kv_len[b] += acc[s] + 1
+    return {"weights": weights, "kv": kv, "total": weights + kv, "steps": steps}
+
+
+def run_batch16(args) -> None:
+    """Batched requests (BASELINE configs[4]): 16 requests on the LLaVA-1.5-13B shape (40 layers,
+    d = 5120, 40 x 128 heads, SwiGLU 13824, V = 32000), each with 576 visual rows and a prompt of
+    U[32, 256] ids, k = 10, gamma = 6, s = 0.2, 256 new tokens per request, decoded in lockstep
+    (ragged positions and accept lengths): batched SSD and batched greedy decode tokens/s over all
+    requests, the speedup, accept lengths, the decode's HBM bytes per second, the verification
+    projections at 112 rows through the medium-M tensor-core kernel timed alone, and the fp64
+    oracle's rate on the host cores.  One JSON line."""
+    import torch
+
+    import paper_2510_22641_gb300 as lib
+    lib.build()
+    bw = synth.LLAVA13B_B16.replace(base=synth.LLAVA13B.replace(s=args.s))
+    w = bw.base
+    up = lib.bf16_bits_to_device
+    bits = synth.make_weights(w, with_layers=False)
+    dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm", "in_norm", "in_w1", "in_w2")}
+    dev["layers"] = []
+    for l in range(w.shape.n_layers):   # one layer at a time: 634 MB of bf16 each
+        dev["layers"].append({n: up(a) for n, a in synth.make_layer_weights(w, l).items()})
+    ins = synth.make_batch_inputs(bw)
+    nv = [v.shape[0] for v, _ in ins]
+    npr = [len(p) for _, p in ins]
+    prompts = [a + b for a, b in zip(nv, npr)]
+    dv = up(np.concatenate([v for v, _ in ins]))
+    dp = torch.from_numpy(np.concatenate([p for _, p in ins]).astype(np.int32)).cuda()
+    rs = torch.tensor(w.resid_scale(), device="cuda")
+    ins_t = torch.tensor([w.in_scale()], device="cuda")
+    cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, w.gamma, bw.max_seq(),
+                          options=lib.SSD_OPT_HOST_LOOP if args.host_loop else 0, max_batch=bw.batch)
+    model = lib.SSDModel(cfg, dev, rs, ins_t)
+    B, T = bw.batch, w.max_new
+    out = torch.zeros(B, T, dtype=torch.int32, device="cuda")
+    n_out = torch.zeros(B, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+    hbm_peak = measured_peak("hbm_gbs")
+
+    def run(gamma):
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+        torch.cuda.synchronize()
+        ev[0].record(stream)
+        model.prefill_batch(dv, nv, dp, npr)
+        ev[1].record(stream)
+        if gamma > 0:
+            model.decode_batch(T, gamma, out, n_out)
+        else:
+            model.greedy_decode_batch(T, out, n_out)
+        ev[2].record(stream)
+        torch.cuda.synchronize()
+        model.sync()
+        assert all(int(x) == T for x in n_out.cpu()), n_out
+        return ev[0].elapsed_time(ev[1]), ev[1].elapsed_time(ev[2])
+
+    def set_s(s_val):
+        ws = w.replace(s=s_val)
+        rs.copy_(torch.tensor(ws.resid_scale(), device="cuda"))
+        ins_t.copy_(torch.tensor([ws.in_scale()], device="cuda"))
+
+    run(w.gamma)   # warm-up: builds the graphs
+    run(0)
+    clocks = ClockSampler(torch.cuda.current_device())
+    rows = []
+    greedy_ms = run(0)[1]
+    greedy_tokens = B * (T - 1)
+    gb = batch_algorithmic_bytes(w, prompts, [[0] * (T - 1)] * B, 0)
+    for s_val in (args.s, 0.05, 1.0):
+        set_s(s_val)
+        pre_ms, dec_ms = run(w.gamma)
+        logs = [model.batch_step_log(b)[0] for b in range(B)]
+        ab = batch_algorithmic_bytes(w, prompts, logs, w.gamma)
+        acc = [a for lg in logs for a in lg]
+        rows.append({"s": s_val, "ssd_decode_tok_s": B * (T - 1) / (dec_ms / 1e3),
+                     "speedup": greedy_ms / dec_ms, "mean_accept": sum(acc) / max(len(acc), 1),
+                     "batch_steps": ab["steps"], "decode_ms": dec_ms, "prefill_ms": pre_ms,
+                     "decode_hbm_gbs": ab["total"] / (dec_ms / 1e3) / 1e9,
+                     "decode_hbm_frac": ab["total"] / (dec_ms / 1e3) / 1e9 / hbm_peak,
+                     "weight_gb": ab["weights"] / 1e9, "kv_gb": ab["kv"] / 1e9})
+    set_s(args.s)
+    clk = clocks.stop()
+    head = rows[0]
+
+    # the verification projections at B * (gamma + 1) rows, each kernel timed alone
+    vrows = B * (w.gamma + 1)
+    kernels = []
+    flops_total = 0.0
+    for name, label in BATCH_KERNEL_ROWS:
+        model.profile_projection(name, layer=w.draft_exit_k, rows=vrows, reps=3)
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = 20
+        torch.cuda.synchronize()
+        a.record(stream)
+        nbytes = model.profile_projection(name, layer=w.draft_exit_k, rows=vrows, reps=reps)
+        b.record(stream)
+        torch.cuda.synchronize()
+        us = a.elapsed_time(b) / reps * 1e3
+        sh = w.shape
+        n_out_rows = {"qkv": 3 * sh.qdim, "o": sh.d_model, "gateup": 2 * sh.d_ff, "down": sh.d_model,
+                      "head": sh.vocab}[name]
+        k_in = {"qkv": sh.d_model, "o": sh.qdim, "gateup": sh.d_model, "down": sh.d_ff, "head": sh.d_model}[name]
+        flops = 2.0 * vrows * n_out_rows * k_in * 2   # bf16 hi + lo parts
+        kernels.append({"kernel": label + " + split", "rows": vrows, "bytes": nbytes, "us": round(us, 2),
+                        "gbs": round(nbytes / us / 1e3, 1), "frac": round(nbytes / us / 1e3 / hbm_peak, 3),
+                        "tflops_issued": round(flops / us / 1e6, 1)})
+    cpu = None
+    if not args.no_cpu_baseline:
+        cpu = oracle_batch_sample(w, ins[0], max_steps=1)
+    model.close()
+    line = {"metric": "batched decode tokens/s (16 requests, 13B shape) and speedup vs batched greedy",
+            "value": head["ssd_decode_tok_s"], "unit": UNIT, "n_gpus": 1, "higher_is_better": True,
+            "dtype": "bf16 weights, fp32 activations / KV / accumulation", "data": "synthetic",
+            "config": {"workload": f"{w.name} x {B} requests: L={w.shape.n_layers} d={w.shape.d_model} "
+                                   f"H={w.shape.n_heads}x{w.shape.head_dim} ff={w.shape.d_ff} V={w.shape.vocab}, "
+                                   f"576 visual + prompts U[{bw.prompt_min},{bw.prompt_max}] "
+                                   f"({min(npr)}..{max(npr)}), {T} new tokens each, k={w.draft_exit_k}, "
+                                   f"gamma={w.gamma}, s={args.s}", "batch": B, "prompt_rows": prompts},
+            "greedy_decode_tok_s": greedy_tokens / (greedy_ms / 1e3),
+            "greedy_decode_hbm_frac": gb["total"] / (greedy_ms / 1e3) / 1e9 / hbm_peak,
+            "per_s": rows, "verify_kernels": kernels, "clocks": clk,
+            "cpu_baseline": cpu}
+    print(json.dumps(line), flush=True)
+
+
+def oracle_batch_sample(w: synth.Workload, request, max_steps: int) -> dict:
+    """The fp64 oracle on one request of the batch (it decodes requests one after another, so the
+    batch's oracle rate is one request's): its prefill and `max_steps` SSD steps, weights widened
+    from bf16 to fp64 (about 8 bytes per parameter of host memory)."""
+    import oracle
+    bits = synth.make_weights(w)
+    vis, prompt = request
+    m = oracle.model_from_bits(w, bits, synth.bf16_to_f64)
+    del bits
+    r = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, w.gamma, max_steps=max_steps)
+    acc = r.accept_lengths
+    tps = (sum(acc) + len(acc)) / max(len(acc), 1)
+    step = sum(r.step_s) / max(len(r.step_s), 1)
+    return {"value": tps / step if step > 0 else None, "unit": "decode tokens/s", "cores": os.cpu_count(),
+            "kind": "oracle", "prefill_s": r.prefill_s, "step_s": step,
+            "sample": f"fp64 numpy oracle, request 0 of the batch ({vis.shape[0] + len(prompt)} prompt rows): "
+                      f"its prefill and {len(acc)} SSD step(s); the oracle runs requests one at a time"}
+
+
 def run_sweep(args) -> None:
     """Sweep k x gamma x s on the 7B shape (256 new tokens): accept length, tokens/s, speedup
     over greedy, draft and verify HBM GB/s.  One JSON line per point."""
@@ -575,6 +755,8 @@ def main() -> None:
                     help="the 7B workload with the imitation module as one decoder block (one JSON line)")
     ap.add_argument("--encdec", action="store_true",
                     help="the BLIP-2 FlanT5-xl-shaped encoder-decoder workload (one JSON line)")
+    ap.add_argument("--batch16", action="store_true",
+                    help="16 batched ragged requests on the 13B shape (one JSON line)")
     ap.add_argument("--profile", choices=["greedy", "ssd", "prefill", "proj"],
                     help="a profiler window around one phase instead of the bench (see run_profile)")
     ap.add_argument("--layers", type=int, default=32, help="--profile: layers of the model")
@@ -589,6 +771,9 @@ def main() -> None:
         return
     if args.encdec:
         run_encdec(args)
+        return
+    if args.batch16:
+        run_batch16(args)
         return
     if args.sweep:
         run_sweep(args)

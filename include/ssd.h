@@ -116,6 +116,9 @@ typedef struct {
   int rel_max_distance; /* T5: offsets at or beyond this share the last bucket */
   int start_token;   /* T5: the decoder's first input id */
   int options;       /* SSD_OPT_* bits, 0 = the default path */
+  int max_batch;     /* requests one batched decode may carry (0 or 1: single requests only; at most
+                      * SSD_MAX_ROWS, with max_batch * (gamma_max + 1) <= 128; SSD_ARCH_LLAMA with
+                      * SSD_IN_IDENTITY or SSD_IN_MLP2).  The KV cache holds max_batch request slots. */
 } ssd_config;
 
 /* Extra weights of SSD_ARCH_T5, device bf16, [out][in], borrowed.  The
@@ -189,7 +192,7 @@ typedef struct {
 } ssd_stats;
 
 /* Create a context: checks the shape, builds TMA descriptors for the borrowed
- * weights, allocates the KV cache [L][H][max_seq][head_dim] fp32 (K and V),
+ * weights, allocates the KV cache [L][max_batch][H][max_seq][head_dim] fp32 (K and V),
  * activations and workspaces on the current device.  cuda_stream is a
  * cudaStream_t (NULL = legacy default stream).  sync. */
 SSD_API ssd_status ssd_create(const ssd_config* cfg, const ssd_weights* w, void* cuda_stream, ssd_ctx** out);
@@ -310,15 +313,69 @@ SSD_API ssd_status ssd_set_draft_logits_capture(ssd_ctx* ctx, float* buf, int ma
  * NULL) and sets *n_steps to the number of steps.  sync. */
 SSD_API ssd_status ssd_get_step_log(ssd_ctx* ctx, int32_t* accepted, int32_t* drafted, int cap, int* n_steps);
 
-/* Device pointers to the KV cache, layout [L][n_heads][max_seq][head_dim]
- * fp32 (with SSD_IN_BLOCK, [L + 1]: slot L is the imitation block's), and the
- * current valid length (sync read).  Positions >= kv_len hold stale rows of
- * rejected drafts. */
+/* Device pointers to the KV cache, layout [L][max_batch][n_heads][max_seq][head_dim]
+ * fp32 (with SSD_IN_BLOCK, [L + 1]: slot L is the imitation block's; the
+ * single-request calls use request slot 0), and the single request's current
+ * valid length (sync read).  Positions >= kv_len hold stale rows of rejected
+ * drafts. */
 SSD_API ssd_status ssd_get_kv(ssd_ctx* ctx, const void** k_cache, const void** v_cache, int* kv_len);
 
 /* Number of kernel launches the last ssd_decode / ssd_greedy_decode /
  * ssd_prefill performed (from the device step counter).  sync. */
 SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches, int64_t* decode_launches);
+
+/* ---- Batched requests: the serving form of Algorithm 1 ----
+ * B <= max_batch independent requests, each with its own visual rows, prompt
+ * length, positions, cache slot and accept lengths, decode in lockstep: each
+ * step drafts gamma tokens for every request (layers 0..k-1 and the imitation
+ * network over B rows per token), verifies all B * (gamma + 1) rows in one
+ * full-depth pass (the medium-M tensor-core kernel beyond 16 rows), and
+ * accepts / rolls back each request on its own.  A request that is done (max_new
+ * tokens or eos) keeps its tokens; its rows ride along unused until every request
+ * is done.  Every request's tokens and accept lengths are those of the same
+ * request decoded alone.  The single-request calls (ssd_prefill .. ssd_verify)
+ * and the batched calls share the cache: a prefill of one kind invalidates the
+ * other kind's decode state. */
+
+/* Prefill of B requests (each as ssd_prefill: rows [vis_b; embed(prompt_b)] at
+ * positions 0..P_b-1 into request b's cache slot, first token from the last row).
+ *   vis_emb:   device bf16 [sum_b n_vis[b]][d_model], request b's rows after those of 0..b-1
+ *   n_vis, n_prompt: host int32 [B]
+ *   prompt:    device int32 [sum_b n_prompt[b]], concatenated the same way
+ *   first_tok: device int32 [B] (may be NULL)
+ * 1 <= B <= max_batch; n_vis[b] + n_prompt[b] + 1 <= max_seq.  async. */
+SSD_API ssd_status ssd_prefill_batch(ssd_ctx* ctx, int batch, const void* vis_emb, const int32_t* n_vis,
+                                     const int32_t* prompt, const int32_t* n_prompt, int32_t* first_tok);
+
+/* SSD decode of the prefilled batch, one CUDA-graph launch (a WHILE node over
+ * draft + verify + accept of every request until all are done).  Request b
+ * stops after max_new tokens (the prefill's included) or an eos; in its last
+ * steps it accepts at most max_new - n_out - 1 drafts.  Capacity: for every
+ * request P_b + max_new + gamma + 1 <= max_seq.
+ *   out_tok: device int32 [B][max_new];  n_out: device int32 [B]
+ * async. */
+SSD_API ssd_status ssd_decode_batch(ssd_ctx* ctx, int max_new, int gamma, int32_t* out_tok, int32_t* n_out);
+
+/* Baseline: greedy decoding of every request of the prefilled batch with the
+ * full model (all L layers over B rows per token).  Same buffers.  async. */
+SSD_API ssd_status ssd_greedy_decode_batch(ssd_ctx* ctx, int max_new, int32_t* out_tok, int32_t* n_out);
+
+/* End-to-end batched call with HOST buffers: copies the inputs (laid out as for
+ * ssd_prefill_batch) to the device, prefill, SSD decode (gamma >= 1) or greedy
+ * decode (gamma == 0), copies the tokens back.  out: host int32 [B][max_new];
+ * n_out: host int32 [B].  sync. */
+SSD_API ssd_status ssd_generate_batch(ssd_ctx* ctx, int batch, const void* vis_emb, const int32_t* n_vis,
+                                      const int32_t* prompt, const int32_t* n_prompt, int max_new, int gamma,
+                                      int32_t* out, int32_t* n_out);
+
+/* Counters (see ssd_stats) and per-step record (see ssd_get_step_log) of
+ * request b of the last batched decode.  sync.  With a batch prefilled, the
+ * logits captures address request b's rows at buf + b * max_rows * vocab
+ * (ssd_set_logits_capture) and buf + b * max_steps * gamma_max * vocab
+ * (ssd_set_draft_logits_capture). */
+SSD_API ssd_status ssd_get_batch_stats(ssd_ctx* ctx, int b, ssd_stats* stats);
+SSD_API ssd_status ssd_get_batch_step_log(ssd_ctx* ctx, int b, int32_t* accepted, int32_t* drafted, int cap,
+                                          int* n_steps);
 
 /* The LM head alone (Sec. "SSD Setup for VLMs": o = g(x), greedy argmax):
  * logits = W_lm RMSNorm_f(x) and the argmax of each row (lowest index on ties)
@@ -355,8 +412,9 @@ SSD_API ssd_status ssd_lm_head_static(const void* lm_head, const void* final_nor
 
 /* Diagnostic for timing one kernel alone: enqueue `reps` back-to-back launches
  * of one weight-streaming projection (the GEMV kernel with its fused
- * epilogue) over `rows` activation rows, with whatever activations the ctx
- * holds.  which: 0 QKV, 1 o_proj, 2 gate/up, 3 down (of `layer`), 4 LM head,
+ * epilogue; beyond 16 rows, in a ctx with max_batch > 1, the activation split
+ * + the medium-M kernel) over `rows` activation rows (at most 16, or 128 and
+ * max_seq), with whatever activations the ctx holds.  which: 0 QKV, 1 o_proj, 2 gate/up, 3 down (of `layer`), 4 LM head,
  * 5 imitation FC1, 6 imitation FC2, 7 the split-KV attention of `layer` for
  * query rows kv_len .. kv_len+rows-1 over the cache as it stands (waits for
  * the stream once to read kv_len).  *bytes receives the algorithmic bytes one

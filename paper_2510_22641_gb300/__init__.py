@@ -22,14 +22,14 @@ def __getattr__(name):
 
 
 def config_dict(shape, draft_exit_k: int, in_kind: int, in_hidden: int, gamma_max: int, max_seq: int,
-                eos_id: int = -1, options: int = 0) -> dict:
+                eos_id: int = -1, options: int = 0, max_batch: int = 1) -> dict:
     """ssd_config fields from a model shape (anything with n_layers, d_model, ... attributes)."""
     return {"n_layers": shape.n_layers, "d_model": shape.d_model, "n_heads": shape.n_heads,
             "head_dim": shape.head_dim, "d_ff": shape.d_ff, "vocab": shape.vocab, "draft_exit_k": draft_exit_k,
             "in_kind": in_kind, "in_hidden": in_hidden, "gamma_max": gamma_max, "max_seq": max_seq,
             "rms_eps": shape.rms_eps, "rope_theta": shape.rope_theta, "eos_id": eos_id, "arch": SSD_ARCH_LLAMA,
             "n_enc_layers": 0, "max_enc": 0, "rel_buckets": 0, "rel_max_distance": 0, "start_token": 0,
-            "options": options}
+            "options": options, "max_batch": max_batch}
 
 
 def t5_config_dict(shape, draft_exit_k: int, in_kind: int, in_hidden: int, gamma_max: int, max_seq: int,

@@ -28,9 +28,10 @@ STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_C
 EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify", "ssd_decode", "ssd_decode_dynamic",
             "ssd_draft_length", "ssd_rel_bucket",
             "ssd_greedy_decode", "ssd_generate", "ssd_greedy_generate", "ssd_sync", "ssd_get_stats",
-            "ssd_set_logits_capture", "ssd_set_draft_logits_capture", "ssd_get_step_log", "ssd_get_kv", "ssd_last_launch_count", "ssd_lm_head", "ssd_lm_head_static", "ssd_profile_projection",
-            "ssd_status_string",
-            "ssd_last_error")
+            "ssd_set_logits_capture", "ssd_set_draft_logits_capture", "ssd_get_step_log", "ssd_get_kv",
+            "ssd_last_launch_count", "ssd_prefill_batch", "ssd_decode_batch", "ssd_greedy_decode_batch",
+            "ssd_generate_batch", "ssd_get_batch_stats", "ssd_get_batch_step_log", "ssd_lm_head",
+            "ssd_lm_head_static", "ssd_profile_projection", "ssd_status_string", "ssd_last_error")
 
 
 class SSDConfig(ctypes.Structure):
@@ -40,7 +41,8 @@ class SSDConfig(ctypes.Structure):
                 ("gamma_max", ctypes.c_int), ("max_seq", ctypes.c_int), ("rms_eps", ctypes.c_float),
                 ("rope_theta", ctypes.c_float), ("eos_id", ctypes.c_int), ("arch", ctypes.c_int),
                 ("n_enc_layers", ctypes.c_int), ("max_enc", ctypes.c_int), ("rel_buckets", ctypes.c_int),
-                ("rel_max_distance", ctypes.c_int), ("start_token", ctypes.c_int), ("options", ctypes.c_int)]
+                ("rel_max_distance", ctypes.c_int), ("start_token", ctypes.c_int), ("options", ctypes.c_int),
+                ("max_batch", ctypes.c_int)]
 
 
 _PP = ctypes.POINTER(ctypes.c_void_p)
@@ -104,6 +106,12 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_get_kv": [vp, ctypes.POINTER(vp), ctypes.POINTER(vp), ctypes.POINTER(i32)],
         "ssd_last_launch_count": [vp, ctypes.POINTER(ctypes.c_int64), ctypes.POINTER(ctypes.c_int64)],
         "ssd_profile_projection": [vp, i32, i32, i32, i32, ctypes.POINTER(ctypes.c_int64)],
+        "ssd_prefill_batch": [vp, i32, vp, vp, vp, vp, pi32],
+        "ssd_decode_batch": [vp, i32, i32, pi32, pi32],
+        "ssd_greedy_decode_batch": [vp, i32, pi32, pi32],
+        "ssd_generate_batch": [vp, i32, vp, vp, vp, vp, i32, i32, vp, vp],
+        "ssd_get_batch_stats": [vp, i32, ctypes.POINTER(SSDStats)],
+        "ssd_get_batch_step_log": [vp, i32, vp, vp, i32, ctypes.POINTER(i32)],
         "ssd_lm_head": [vp, vp, i32, vp, vp],
         "ssd_lm_head_static": [vp, vp, vp, i32, i32, i32, ctypes.c_float, vp, vp, vp],
     }

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libssd.so")
-SOURCES = ["engine.cu", "gemv_qkv.cu", "gemv_gate.cu", "gemv_silu.cu", "gemv_resid.cu", "gemv_head.cu",
+SOURCES = ["engine.cu", "gemv_qkv.cu", "gemv_gate.cu", "gemv_silu.cu", "gemv_resid.cu", "gemv_head.cu", "gemv_mid.cu",
            "static_head.cu", "prefill.cu"]
 FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-lineinfo", "-std=c++17",
          "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]
@@ -65,7 +65,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
     with concurrent.futures.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB + f".{os.getpid()}.tmp"
-    r = subprocess.run([nvcc, "-shared", "-o", tmp, *objs], capture_output=True, text=True)
+    r = subprocess.run([nvcc, "-shared", "-Xlinker", "-z", "-Xlinker", "defs", "-o", tmp, *objs], capture_output=True,
+                       text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stderr}")
     os.replace(tmp, LIB)

@@ -23,6 +23,11 @@
 // assignment and every summation order depend only on key positions, never on
 // M, so each row's output equals the single-row (M = 1) result bitwise.
 //
+// Batched requests (batch_rows > 0) add a grid dimension: blockIdx.z is the
+// request z, whose M rows are rows z*M .. z*M+M-1 of q and o, whose keys are
+// its own cache rows (k_cache / v_cache + z * req_kv) and whose base is
+// req_st[z].kv_len + pos_off; requests never share a CTA, a state or a ticket.
+//
 // With prefetch_old set, the launch before this one triggered its dependents
 // only after its own upstream grid had completed, so everything older than that
 // launch is complete here: the chunks holding only keys below base (written by
@@ -53,8 +58,8 @@ struct AttnParams {
   int n_heads, max_seq;
   float scale;       // 1/sqrt(Dh)
   int prefetch_old;  // the previous launch triggered after its own upstream completed (see above)
-  float* part;        // [n_heads][kAttnSplit][kAttnMaxRows][Dh + 2] CTA states (output, max, sum)
-  unsigned* tickets;  // [n_heads], zero between launches
+  float* part;        // [requests][n_heads][kAttnSplit][kAttnMaxRows][Dh + 2] CTA states (output, max, sum)
+  unsigned* tickets;  // [requests][n_heads], zero between launches
   // Non-causal key sets and relative-position bias (encoder-decoder models; read only by the EXT
   // instantiations, so the causal kernels compile without them):
   int fixed_keys;     // 1: keys 0 .. st->enc_len - 1, every one visible to every row (cross-attention,
@@ -62,6 +67,10 @@ struct AttnParams {
   int abs_pos;        // row m sits at position pos_off + m (st->kv_len ignored): the encoder's rows
   const float* bias;  // null, or [n_heads][bias_stride]: score(row at i, key j) += bias[h][j - i + bias_zero]
   int bias_stride, bias_zero;
+  // Batched requests (0: one request; else the rows per request, = M): see the header.
+  int batch_rows;
+  const DevState* req_st;
+  long long req_kv;
 };
 
 template <int DH>
@@ -109,6 +118,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
   const int tid = threadIdx.x, w = tid >> 5, lane = tid & 31;
   const int rank = blockIdx.x;
   const int h = blockIdx.y;
+  const int z = blockIdx.z;  // request (0 for one request)
+  const float* k_cache = p.k_cache + z * p.req_kv;
+  const float* v_cache = p.v_cache + z * p.req_kv;
+  const float* q_rows = p.q + static_cast<size_t>(z) * M * p.q_stride;
+  float* o_rows = p.o + static_cast<size_t>(z) * M * p.o_stride;
 
   pdl_trigger();
   if (tid == 0) {
@@ -124,7 +138,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
   int base = 0, n_keys = 0, my_chunks = 0;
   bool bad = false;
   auto geometry = [&]() {
-    base = ((EXT && p.abs_pos) ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
+    base = ((EXT && p.abs_pos) ? 0 : __ldcg(p.batch_rows ? &p.req_st[z].kv_len : &p.st->kv_len)) + p.pos_off;
     if (EXT && p.fixed_keys) {
       const int ne = __ldcg(&p.st->enc_len);
       bad = base < 0 || ne < 1 || ne > p.max_seq;
@@ -142,8 +156,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
     const uint32_t kv_bytes = static_cast<uint32_t>(nk * DH * 4);
     mbar_arrive_expect_tx(&bar[buf], 2 * kv_bytes);
     const size_t off = (static_cast<size_t>(h) * p.max_seq + j0) * DH;
-    bulk_load(b, p.k_cache + off, kv_bytes, &bar[buf]);
-    bulk_load(b + S::kKV, p.v_cache + off, kv_bytes, &bar[buf]);
+    bulk_load(b, k_cache + off, kv_bytes, &bar[buf]);
+    bulk_load(b + S::kKV, v_cache + off, kv_bytes, &bar[buf]);
   };
   int issued = 0;  // thread 0: chunks of the first group already requested
   if (p.prefetch_old) {
@@ -163,7 +177,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
     mbar_arrive_expect_tx(&bar[kAttnBufs], M * DH * 4);
 #pragma unroll
     for (int m = 0; m < M; ++m)
-      bulk_load(Qs + m * DH, p.q + static_cast<size_t>(m) * p.q_stride + h * DH, DH * 4, &bar[kAttnBufs]);
+      bulk_load(Qs + m * DH, q_rows + static_cast<size_t>(m) * p.q_stride + h * DH, DH * 4, &bar[kAttnBufs]);
     for (; issued < kAttnBufs && issued < my_chunks; ++issued) issue(issued, rank + issued * kAttnSplit);
   }
 
@@ -343,7 +357,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
     for (int e = 0; e < DPL; ++e) ws[(w * M + m) * DH + lane * DPL + e] = acc[m][e];
   __syncthreads();
   constexpr int kSlot = kAttnMaxRows * E;  // one CTA state in part
-  float* head_part = p.part + static_cast<size_t>(h) * kAttnSplit * kSlot;
+  const int zh = z * p.n_heads + h;  // this request's head
+  float* head_part = p.part + static_cast<size_t>(zh) * kAttnSplit * kSlot;
   float* mine = head_part + rank * kSlot;
   for (int idx = tid; idx < M * DH; idx += kAttnThreads) {
     const int m = idx / DH, d = idx - m * DH;
@@ -358,7 +373,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
   }
   int* last = reinterpret_cast<int*>(smem + S::kFlag);
   __syncthreads();
-  if (tid == 0) *last = atom_add_acq_rel_gpu(&p.tickets[h], 1u) == static_cast<unsigned>(kAttnSplit - 1);
+  if (tid == 0) *last = atom_add_acq_rel_gpu(&p.tickets[zh], 1u) == static_cast<unsigned>(kAttnSplit - 1);
   __syncthreads();
   if (*last) {
     if (!bad && !timed_out) {
@@ -402,10 +417,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
 #pragma unroll
         for (int q = 0; q < kAttnSplit; ++q) O = fmaf(wq[m * kAttnSplit + q], v[e][q], O);
         const float L = wq[M * kAttnSplit + m];
-        p.o[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
+        o_rows[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
       }
     }
-    if (tid == 0) p.tickets[h] = 0u;
+    if (tid == 0) p.tickets[zh] = 0u;
   }
 }
 

@@ -13,6 +13,7 @@
 namespace ssd {
 
 constexpr int kMaxRows = SSD_MAX_ROWS;
+constexpr int kMaxMidRows = 128;  // rows of one medium-M projection (the verification of batched requests)
 
 // Device error bits (DevState::error).
 enum : int { DERR_TOKEN = 1, DERR_TIMEOUT = 2, DERR_POS = 4 };
@@ -40,7 +41,7 @@ struct DevState {
   int tok_in[kMaxRows];          // verify rows t_0 = y, t_j = d_j
   int full_tok[kMaxRows];        // f_i = full-model argmax of row i
   int last_emitted[kMaxRows];
-  unsigned long long am_key[kMaxRows];  // packed argmax accumulators (LM head)
+  unsigned long long am_key[kMaxMidRows];  // packed argmax accumulators of the LM head's rows
   unsigned int am_count;                // LM-head row tiles finished
 };
 

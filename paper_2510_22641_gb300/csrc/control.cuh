@@ -74,7 +74,7 @@ __global__ void ssd_prefill_begin_kernel(DevState* st, int P, int eos_id, int en
   st->eos_id = eos_id;
   st->steps = st->drafted = st->accepted = 0;
   for (int i = 0; i <= SSD_MAX_GAMMA; ++i) st->hist[i] = 0;
-  for (int i = 0; i < kMaxRows; ++i) st->am_key[i] = 0ull;
+  for (int i = 0; i < kMaxMidRows; ++i) st->am_key[i] = 0ull;
   st->am_count = 0u;
 }
 
@@ -227,6 +227,137 @@ __global__ void ssd_copy_emitted_kernel(const DevState* st, int* n_emitted, int*
 __global__ void ssd_first_token_kernel(const DevState* st, int* first_tok) {
   pdl_wait();
   if (threadIdx.x == 0) *first_tok = st->cur_tok;
+}
+
+// ------------------------------------------------------------------ batched requests
+// B independent requests decode in lockstep (Algorithm 1 per request): req[b] is request b's
+// state; st (the launch state of the projections) holds the error word, the argmax keys and the
+// batch's done flag and step count.  Request b's tokens go to out + b * out_cap, its step record
+// to step_log + b * log_cap.
+
+// Row b of x (stride x_stride) = E[req[b].tok_in[j]]: the embedding of request b's j-th input.
+__global__ void ssd_batch_embed_kernel(const __nv_bfloat16* __restrict__ E, const DevState* req, int j, float* x,
+                                       int x_stride, int d, int vocab, DevState* st) {
+  pdl_trigger();
+  pdl_wait();
+  const int b = blockIdx.x;
+  int t = __ldcg(&req[b].tok_in[j]);
+  if (t < 0 || t >= vocab) {
+    if (threadIdx.x == 0) set_error(st, DERR_TOKEN);
+    t = 0;
+  }
+  const uint4* src = reinterpret_cast<const uint4*>(E + static_cast<size_t>(t) * d);
+  float4* dst = reinterpret_cast<float4*>(x + static_cast<size_t>(b) * x_stride);
+  for (int i = threadIdx.x; i < d / 8; i += blockDim.x) {
+    const uint4 v = __ldg(src + i);
+    const float2 a = bf16x2_to_float2(v.x), c = bf16x2_to_float2(v.y), e = bf16x2_to_float2(v.z),
+                 f = bf16x2_to_float2(v.w);
+    dst[2 * i] = make_float4(a.x, a.y, c.x, c.y);
+    dst[2 * i + 1] = make_float4(e.x, e.y, f.x, f.y);
+  }
+}
+
+// Start of a batched decode: every request's limits and counters; st->done once all are done.
+__global__ void ssd_batch_setup_kernel(DevState* st, DevState* req, int B, int max_new, int gamma) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ int all_done;
+  if (threadIdx.x == 0) all_done = 1;
+  __syncthreads();
+  const bool err = __ldcg(&st->error) != 0;
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    DevState* r = req + b;
+    r->max_new = max_new;
+    r->gamma = gamma;
+    r->steps = r->drafted = r->accepted = 0;
+    for (int i = 0; i <= SSD_MAX_GAMMA; ++i) r->hist[i] = 0;
+    if (r->n_out >= max_new || r->error || err) r->done = 1;
+    if (!r->done) atomicAnd(&all_done, 0);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    st->done = all_done;
+    st->steps = 0;
+    st->max_new = max_new;
+    st->gamma = gamma;
+  }
+}
+
+// One request's acceptance (the rule of ssd_accept_kernel on state r), g_max drafts per step.
+__device__ __forceinline__ void accept_one(DevState* r, int gamma, int* out, int out_cap, int2* log, int log_cap,
+                                           bool err) {
+  if (r->done) {
+    r->last_n = 0;
+    return;
+  }
+  const int remaining = r->max_new - r->n_out;
+  const int g_eff = min(gamma, remaining - 1);
+  int a = 0;
+  while (a < g_eff && r->tok_in[a + 1] == r->full_tok[a]) ++a;
+  int cnt = a + 1;
+  bool eos = false;
+  for (int i = 0; i < a + 1; ++i) {
+    const int t = (i < a) ? r->tok_in[i + 1] : r->full_tok[a];
+    r->last_emitted[i] = t;
+    const int o = r->n_out + i;
+    if (o < out_cap) out[o] = t;
+    if (r->eos_id >= 0 && t == r->eos_id) {
+      cnt = i + 1;
+      eos = true;
+      break;
+    }
+  }
+  r->last_n = cnt;
+  r->n_out += cnt;
+  r->kv_len += a + 1;
+  if (r->steps < log_cap) log[r->steps] = make_int2(a, g_eff);
+  const int y = r->full_tok[a];
+  r->cur_tok = y;
+  r->tok_in[0] = y;
+  r->steps += 1;
+  r->drafted += g_eff;
+  r->accepted += a;
+  r->hist[a] += 1;
+  if (eos || r->n_out >= r->max_new || err) r->done = 1;
+}
+
+// Algorithm 1's acceptance for every request of the batch (gamma = 0: a greedy step, f_0
+// emitted); st->done (and the WHILE condition) once every request is done.
+__global__ void ssd_batch_accept_kernel(DevState* st, DevState* req, int B, int gamma, int* out, int out_cap,
+                                        int2* step_log, int log_cap, cudaGraphConditionalHandle cond, int has_cond) {
+  pdl_trigger();
+  pdl_wait();
+  __shared__ int all_done;
+  if (threadIdx.x == 0) all_done = 1;
+  __syncthreads();
+  const bool err = __ldcg(&st->error) != 0;
+  for (int b = threadIdx.x; b < B; b += blockDim.x) {
+    accept_one(req + b, gamma, out + static_cast<size_t>(b) * out_cap, out_cap,
+               step_log + static_cast<size_t>(b) * log_cap, log_cap, err);
+    if (!req[b].done) atomicAnd(&all_done, 0);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    st->done = all_done;
+    st->steps += 1;
+    if (has_cond) cudaGraphSetConditional(cond, all_done ? 0u : 1u);
+  }
+}
+
+// First tokens (after a batched prefill) and tokens out of a batched decode.
+__global__ void ssd_batch_first_tokens_kernel(const DevState* req, int B, int* first) {
+  pdl_wait();
+  for (int b = threadIdx.x; b < B; b += blockDim.x) first[b] = req[b].cur_tok;
+}
+
+__global__ void ssd_batch_copy_out_kernel(const DevState* req, const int* out_int, int out_cap, int* user_out,
+                                          int* user_n, int max_new) {
+  pdl_wait();
+  const int b = blockIdx.x;
+  const int n = min(req[b].n_out, max_new);
+  for (int i = threadIdx.x; i < n; i += blockDim.x)
+    if (user_out) user_out[static_cast<size_t>(b) * max_new + i] = out_int[static_cast<size_t>(b) * out_cap + i];
+  if (threadIdx.x == 0 && user_n) user_n[b] = n;
 }
 
 // cos/sin of pos * theta^(-2j/head_dim), computed in fp64 and rounded to fp32.

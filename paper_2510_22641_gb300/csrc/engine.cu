@@ -44,6 +44,12 @@ cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bf
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
                                 float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
                                 cudaStream_t s, bool pdl);
+cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
+                       int grid, cudaStream_t s, bool pdl);
+cudaError_t mid_attrs();
+cudaError_t split_act_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
+                             __nv_bfloat16* hi, __nv_bfloat16* lo, int ld, float* rs, int rows, cudaStream_t s,
+                             bool pdl);
 }  // namespace ssd
 
 using namespace ssd;
@@ -51,7 +57,8 @@ using namespace ssd;
 namespace {
 
 constexpr int kPrefillChunk = 8;  // prefill rows per pass through the layers
-constexpr int kMaxVerifyRows = 9; // gemv / attention instantiations cover M = 1..9
+constexpr int kMaxVerifyRows = 9; // rows of one request's verification pass (gamma_max + 1)
+constexpr int kMidMinRows = kMaxRows + 1;  // projections over more rows use the medium-M kernel
 
 struct Site {  // one projection: up to three weight matrices with a common K
   CUtensorMap maps[3];
@@ -101,8 +108,26 @@ struct ssd_ctx {
   int* out_int = nullptr;  // [max_seq] emitted tokens
   int2* step_log = nullptr;  // [max_seq] (accepted drafts a, gamma_eff) per step since the prefill
   float *xv = nullptr, *qb = nullptr, *ob = nullptr, *hb = nullptr, *hin = nullptr, *xt = nullptr;
-  float *kc = nullptr, *vc = nullptr;  // KV cache [L][H][max_seq][Dh], fp32
-  size_t layer_kv = 0;  // elements per layer in kc / vc
+  float *kc = nullptr, *vc = nullptr;  // KV cache [L][max_batch][H][max_seq][Dh], fp32
+  size_t req_kv = 0;    // elements per request and layer in kc / vc
+  size_t layer_kv = 0;  // elements per layer (max_batch * req_kv)
+  size_t kv_slot = 0;   // request slot the single-request enqueue functions address (b * req_kv)
+  // batched requests (the serving form of Algorithm 1; max_batch > 1)
+  int max_batch = 1;
+  int batch = 0;                 // requests of the last ssd_prefill_batch
+  DevState* req = nullptr;       // [max_batch] per-request decode state
+  int* bout = nullptr;           // [max_batch][max_seq] emitted tokens per request
+  int2* blog = nullptr;          // [max_batch][max_seq] per-step (a, gamma_eff) per request
+  __nv_bfloat16 *act_hi = nullptr, *act_lo = nullptr;  // split activations [kMaxMidRows][act_ld] (medium-M)
+  float* act_rs = nullptr;       // [kMaxMidRows] RMSNorm scales of the split rows
+  int act_ld = 0;
+  float* mid_partials = nullptr;  // [2 * grid][kMaxMidRows][kTileN]
+  std::map<std::pair<int, int>, std::pair<CUtensorMap, CUtensorMap>> act_maps;  // (K, NP) -> hi, lo
+  std::map<int, cudaGraphExec_t> batch_graphs;  // decode loops by gamma (0: greedy), for batch_graph_b requests
+  std::map<int, int64_t> batch_body_launches;
+  int batch_graph_b = 0;
+  __nv_bfloat16* bvis = nullptr;  // batched prefill inputs: [max_batch * max_seq][d_model] rows, ids
+  int* bprompt = nullptr;
   float2* rope = nullptr;
   float* partials = nullptr;
   unsigned* counters = nullptr;
@@ -137,7 +162,8 @@ struct ssd_ctx {
   int drafted_gamma = 0;
   int prompt_len = 0;
   int64_t kv_upper = 0;  // upper bound on the device kv_len
-  int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy, 3 ssd with the dynamic draft length
+  int last_decode_kind = 0;  // 0 none, 1 ssd, 2 greedy, 3 ssd with the dynamic draft length, 4 batched
+  std::vector<int> batch_prompt;  // P_b of the prefilled batch
   int last_gamma = 0;
   std::pair<int, int> last_prefill_shape{0, 0};
   // encoder-decoder model (SSD_ARCH_T5)
@@ -163,6 +189,10 @@ struct ssd_ctx {
 };
 
 // ------------------------------------------------------------------ helpers
+
+// Layer l's K / V cache of the request slot the single-request path addresses.
+static float* kv_k(ssd_ctx* c, int l) { return c->kc + l * c->layer_kv + c->kv_slot; }
+static float* kv_v(ssd_ctx* c, int l) { return c->vc + l * c->layer_kv + c->kv_slot; }
 
 static ssd_status fail(ssd_ctx* c, ssd_status s, const char* fmt, ...) {
   if (c) {
@@ -286,8 +316,8 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
 
 // EXT: fixed key sets / absolute positions / relative-position bias (the encoder-decoder model).
 template <int M>
-static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a) {
-  const dim3 grid(kAttnSplit, c->cfg.n_heads);
+static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a, int nreq) {
+  const dim3 grid(kAttnSplit, c->cfg.n_heads, nreq);
   const bool ext = a.fixed_keys || a.abs_pos || a.bias;
   if (c->cfg.head_dim == 128)
     return ext ? launch_k(c, ssd_splitkv_attn_kernel<M, 128, true>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a)
@@ -325,23 +355,24 @@ static cudaError_t attn_attrs() {
   return attn_attr_m<9>();
 }
 
-// One split-KV attention launch over M query rows (the ctx's scratch, state and head count filled in).
-static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a) {
+// One split-KV attention launch over M query rows per request for nreq requests (the ctx's
+// scratch, state and head count filled in).
+static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a, int nreq = 1) {
   a.part = c->attn_part;
   a.tickets = c->attn_tickets;
   a.st = c->st;
   a.n_heads = c->cfg.n_heads;
   cudaError_t r;
   switch (M) {
-    case 1: r = attn_launch_m<1>(c, a); break;
-    case 2: r = attn_launch_m<2>(c, a); break;
-    case 3: r = attn_launch_m<3>(c, a); break;
-    case 4: r = attn_launch_m<4>(c, a); break;
-    case 5: r = attn_launch_m<5>(c, a); break;
-    case 6: r = attn_launch_m<6>(c, a); break;
-    case 7: r = attn_launch_m<7>(c, a); break;
-    case 8: r = attn_launch_m<8>(c, a); break;
-    case 9: r = attn_launch_m<9>(c, a); break;
+    case 1: r = attn_launch_m<1>(c, a, nreq); break;
+    case 2: r = attn_launch_m<2>(c, a, nreq); break;
+    case 3: r = attn_launch_m<3>(c, a, nreq); break;
+    case 4: r = attn_launch_m<4>(c, a, nreq); break;
+    case 5: r = attn_launch_m<5>(c, a, nreq); break;
+    case 6: r = attn_launch_m<6>(c, a, nreq); break;
+    case 7: r = attn_launch_m<7>(c, a, nreq); break;
+    case 8: r = attn_launch_m<8>(c, a, nreq); break;
+    case 9: r = attn_launch_m<9>(c, a, nreq); break;
     default: return fail(c, SSD_ERR_INVALID_ARG, "attention rows %d out of range", M);
   }
   CK(r);
@@ -356,8 +387,8 @@ static ssd_status attention(ssd_ctx* c, int l, int M, int pos_off, bool prefetch
   a.prefetch_old = prefetch_old ? 1 : 0;
   a.q = c->qb;
   a.q_stride = c->qp;
-  a.k_cache = c->kc + l * c->layer_kv;
-  a.v_cache = c->vc + l * c->layer_kv;
+  a.k_cache = kv_k(c, l);
+  a.v_cache = kv_v(c, l);
   a.o = c->ob;
   a.o_stride = c->qp;
   a.pos_off = pos_off;
@@ -402,8 +433,8 @@ static ssd_status enqueue_qkv_only(ssd_ctx* c, int l, const float* x, int M, int
   p.pos_off = pos_off;
   p.q_out = c->qb;
   p.q_stride = c->qp;
-  p.k_cache = c->kc + l * c->layer_kv;
-  p.v_cache = c->vc + l * c->layer_kv;
+  p.k_cache = kv_k(c, l);
+  p.v_cache = kv_v(c, l);
   p.head_dim = c->cfg.head_dim;
   p.max_seq = c->cfg.max_seq;
   p.rope_cs = c->rope;
@@ -430,8 +461,8 @@ static ssd_status enqueue_t5_layer(ssd_ctx* c, int l, float* x, int M, int pos_o
   p.pos_off = pos_off;
   p.q_out = c->qb;
   p.q_stride = c->qp;
-  p.k_cache = c->kc + l * c->layer_kv;
-  p.v_cache = c->vc + l * c->layer_kv;
+  p.k_cache = kv_k(c, l);
+  p.v_cache = kv_v(c, l);
   p.head_dim = c->cfg.head_dim;
   p.max_seq = c->cfg.max_seq;
   p.late_trigger = 1;
@@ -483,8 +514,8 @@ static ssd_status enqueue_layer_x(ssd_ctx* c, int l, float* x, int M, int pos_of
   p.pos_off = pos_off;
   p.q_out = c->qb;
   p.q_stride = c->qp;
-  p.k_cache = c->kc + l * c->layer_kv;
-  p.v_cache = c->vc + l * c->layer_kv;
+  p.k_cache = kv_k(c, l);
+  p.v_cache = kv_v(c, l);
   p.head_dim = c->cfg.head_dim;
   p.max_seq = c->cfg.max_seq;
   p.rope_cs = c->rope;
@@ -627,7 +658,7 @@ static ssd_status enqueue_prefill(ssd_ctx* c, int n_vis, int n_prompt) {
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   // tickets of the split-row reductions start from zero (a previous aborted run may have left some)
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
-  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->max_batch * c->cfg.n_heads, c->cs));
   CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
   int r0 = 0;
   for (; r0 < P; r0 += kPrefillChunk) {
@@ -657,7 +688,7 @@ static ssd_status enqueue_prefill_t5(ssd_ctx* c, int n_vis, int n_prompt) {
   const int P = n_vis + n_prompt, dp = c->dp, qp = c->qp;
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
-  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->max_batch * c->cfg.n_heads, c->cs));
   CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 1, c->cfg.eos_id, P));
   CK(launch_k(c, ssd_prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_enc, dp, c->cfg.d_model,
@@ -765,7 +796,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   const int P = n_vis + n_prompt, dp = c->dp;
   int* full_tok = st_field(c, offsetof(DevState, full_tok));
   CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
-  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->cfg.n_heads, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->max_batch * c->cfg.n_heads, c->cs));
   CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, P, c->cfg.eos_id, 0));
   CK(launch_k(c, ssd_prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
               static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_pre, dp, c->cfg.d_model,
@@ -777,8 +808,8 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     p.pos0 = 0;
     p.q_out = c->q_pre;
     p.q_stride = c->qp;
-    p.k_cache = c->kc + b * c->layer_kv;
-    p.v_cache = c->vc + b * c->layer_kv;
+    p.k_cache = kv_k(c, b);
+    p.v_cache = kv_v(c, b);
     p.head_dim = c->cfg.head_dim;
     p.max_seq = c->cfg.max_seq;
     p.rope_cs = c->rope;
@@ -792,15 +823,15 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     p.pos0 = 0;
     p.q_out = c->q_pre;
     p.q_stride = c->qp;
-    p.k_cache = c->kc + l * c->layer_kv;
-    p.v_cache = c->vc + l * c->layer_kv;
+    p.k_cache = kv_k(c, l);
+    p.v_cache = kv_v(c, l);
     p.head_dim = c->cfg.head_dim;
     p.max_seq = c->cfg.max_seq;
     p.rope_cs = c->rope;
     CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->attn_norm[l], P));
     CKS(tc_gemm(c, Epi::QKV, 0, tl.qkv, P, p));
     ++c->launch_counter;
-    CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, c->kc + l * c->layer_kv, c->vc + l * c->layer_kv,
+    CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, kv_k(c, l), kv_v(c, l),
                            c->o_pre, c->qp, P, c->cfg.n_heads, c->cfg.max_seq,
                            1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->cs, c->use_pdl));
     CKS(split(c, c->o_pre, c->qp, c->qdim, nullptr, P));
@@ -831,6 +862,240 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   return SSD_OK;
 }
 
+// ------------------------------------------------------------------ batched requests
+// The serving form of Algorithm 1: B requests, each with its own prompt, positions, cache slot
+// and accept lengths, decode in lockstep.  Request b's row i (i = 0..g) of a step lives in row
+// b * (g + 1) + i of xv, so drafting step j's rows (a stride of g + 1 rows) are exactly where the
+// verification pass needs x_k (option B).  Every launch carries all B requests, finished ones
+// too (their rows are computed and never used), so a step has one shape and one graph.
+
+// The split activations' tensor maps for K columns and NP rows (built once per shape).
+static ssd_status act_maps_for(ssd_ctx* c, int K, int NP, const CUtensorMap** out) {
+  auto key = std::make_pair(K, NP);
+  auto it = c->act_maps.find(key);
+  if (it == c->act_maps.end()) {
+    std::pair<CUtensorMap, CUtensorMap> m;
+    CKS(encode_map_sw128(c, &m.first, c->act_hi, kMaxMidRows, K, NP));
+    CKS(encode_map_sw128(c, &m.second, c->act_lo, kMaxMidRows, K, NP));
+    it = c->act_maps.emplace(key, m).first;
+  }
+  *out = &it->second.first;  // hi, then lo (adjacent in the pair)
+  return SSD_OK;
+}
+
+// One projection over M > kMaxRows rows: the rows are split into bf16 hi / lo parts with their
+// RMSNorm scales (gain folded in), then the medium-M tensor-core kernel streams the weights once.
+static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
+  if (M > kMaxMidRows || !c->act_hi) return fail(c, SSD_ERR_INVALID_ARG, "%d rows exceed the medium-M kernel", M);
+  ++c->launch_counter;
+  CK(split_act_launch(p.x, p.x_stride, s.K, p.gain, c->cfg.rms_eps, c->act_hi, c->act_lo, s.K, c->act_rs, M, c->cs,
+                      c->use_pdl));
+  CUtensorMap amaps[2];
+  const CUtensorMap* am = nullptr;
+  CKS(act_maps_for(c, s.K, (M + 15) & ~15, &am));
+  amaps[0] = am[0];
+  amaps[1] = am[1];
+  p.K = s.K;
+  p.n_kt = s.n_kt;
+  p.n_rt = s.n_rt;
+  p.units = s.units;
+  p.N = s.N;
+  p.seg_rows = s.seg_rows;
+  p.partials = c->mid_partials;
+  p.counters = c->counters;
+  p.st = c->st;
+  p.eps = c->cfg.rms_eps;
+  p.rs_in = c->act_rs;
+  ++c->launch_counter;
+  CK(mid_launch(e, s.maps, amaps, p, M, s.grid, c->cs, c->use_pdl));
+  return SSD_OK;
+}
+
+// A projection over M rows of the batch: the GEMV up to kMaxRows rows, the medium-M kernel beyond.
+static ssd_status proj_rows(ssd_ctx* c, Epi e, int M, const Site& s, const GemvParams& p) {
+  return M <= kMaxRows ? gemv(c, e, M, s, p) : mid_gemm(c, e, M, s, p);
+}
+
+static void set_batch_rows(ssd_ctx* c, GemvParams& p, int R) {
+  p.batch_rows = R;
+  p.req_st = c->req;
+  p.req_kv = static_cast<long long>(c->req_kv);
+  p.tok_stride = static_cast<int>(sizeof(DevState) / sizeof(int));
+}
+
+// Decoder layer l on M = B * R rows x (row stride x_stride): request b's rows b * R .. b * R + R - 1
+// at positions req[b].kv_len + pos_off + i, in place.
+static ssd_status enqueue_layer_batch(ssd_ctx* c, int l, float* x, int x_stride, int M, int R, int pos_off) {
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = x_stride;
+  p.gain = c->attn_norm[l];
+  p.pos_off = pos_off;
+  p.q_out = c->qb;
+  p.q_stride = c->qp;
+  p.k_cache = c->kc + l * c->layer_kv;
+  p.v_cache = c->vc + l * c->layer_kv;
+  p.head_dim = c->cfg.head_dim;
+  p.max_seq = c->cfg.max_seq;
+  p.rope_cs = c->rope;
+  p.late_trigger = 1;
+  set_batch_rows(c, p, R);
+  CKS(proj_rows(c, Epi::QKV, M, c->layers[l].qkv, p));
+  AttnParams a{};
+  a.prefetch_old = 1;
+  a.q = c->qb;
+  a.q_stride = c->qp;
+  a.k_cache = c->kc + l * c->layer_kv;
+  a.v_cache = c->vc + l * c->layer_kv;
+  a.o = c->ob;
+  a.o_stride = c->qp;
+  a.pos_off = pos_off;
+  a.max_seq = c->cfg.max_seq;
+  a.scale = 1.0f / sqrtf(static_cast<float>(c->cfg.head_dim));
+  a.batch_rows = R;
+  a.req_st = c->req;
+  a.req_kv = static_cast<long long>(c->req_kv);
+  CKS(attn_run(c, R, a, M / R));
+  p = GemvParams{};
+  p.x = c->ob;
+  p.x_stride = c->qp;
+  p.base = x;
+  p.base_stride = x_stride;
+  p.dst = x;
+  p.dst_stride = x_stride;
+  p.scale = resid_scale_of(c, l);
+  CKS(proj_rows(c, Epi::RESID, M, c->layers[l].o, p));
+  p = GemvParams{};
+  p.x = x;
+  p.x_stride = x_stride;
+  p.gain = c->ffn_norm[l];
+  p.h_out = c->hb;
+  p.h_stride = c->fp;
+  CKS(proj_rows(c, Epi::GATE_SILU, M, c->layers[l].gateup, p));
+  p = GemvParams{};
+  p.x = c->hb;
+  p.x_stride = c->fp;
+  p.base = x;
+  p.base_stride = x_stride;
+  p.dst = x;
+  p.dst_stride = x_stride;
+  p.scale = resid_scale_of(c, l);
+  return proj_rows(c, Epi::RESID, M, c->layers[l].down, p);
+}
+
+// LM head + argmax over M = B * R rows x: row (b, i) writes its token to tok0[b][i] (tok0 a field of
+// req[0], indexed across requests by the DevState stride); draft heads (draft = true) capture their
+// logits by (request, step, j = pos_off), full-model heads by (request, predicted token index).
+static ssd_status enqueue_head_batch(ssd_ctx* c, const float* x, int x_stride, int M, int R, int pos_off, int* tok0,
+                                     bool draft) {
+  GemvParams p{};
+  p.x = x;
+  p.x_stride = x_stride;
+  p.gain = c->final_norm;
+  p.pos_off = pos_off;
+  p.tok_dst = tok0;
+  set_batch_rows(c, p, R);
+  if (draft) {
+    p.logits = c->draft_logits_buf;
+    p.logits_rows = c->draft_logits_buf ? c->draft_logits_steps * c->cfg.gamma_max : 0;
+    p.logits_step_rows = c->cfg.gamma_max;
+  } else {
+    p.logits = c->logits_buf;
+    p.logits_rows = c->logits_buf ? c->logits_rows : 0;
+  }
+  return proj_rows(c, Epi::ARGMAX, M, c->head, p);
+}
+
+// Drafting stage of every request (gamma tokens each): layers 0..k-1 and the imitation network at
+// M = B rows per token.
+static ssd_status enqueue_draft_batch(ssd_ctx* c, int gamma) {
+  const int B = c->batch, d = c->dp, rs = (gamma + 1) * c->dp;
+  for (int j = 0; j < gamma; ++j) {
+    float* xj = c->xv + static_cast<size_t>(j) * d;
+    CK(launch_k(c, ssd_batch_embed_kernel, dim3(B), dim3(256), 0, c->embed, static_cast<const DevState*>(c->req), j,
+                xj, rs, c->cfg.d_model, c->cfg.vocab, c->st));
+    for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer_batch(c, l, xj, rs, B, 1, j));
+    const float* hx = xj;
+    int hx_stride = rs;
+    if (c->cfg.in_kind == SSD_IN_MLP2) {
+      GemvParams p{};
+      p.x = xj;
+      p.x_stride = rs;
+      p.gain = c->in_norm;
+      p.h_out = c->hin;
+      p.h_stride = c->ip;
+      CKS(gemv(c, Epi::SILU, B, c->in1, p));
+      p = GemvParams{};
+      p.x = c->hin;
+      p.x_stride = c->ip;
+      p.base = xj;
+      p.base_stride = rs;
+      p.dst = c->xt;
+      p.dst_stride = d;
+      p.scale = c->in_scale;
+      CKS(gemv(c, Epi::RESID, B, c->in2, p));
+      hx = c->xt;
+      hx_stride = d;
+    }
+    CKS(enqueue_head_batch(c, hx, hx_stride, B, 1, j, &c->req[0].tok_in[j + 1], true));
+  }
+  return SSD_OK;
+}
+
+// Verification of every request's gamma + 1 rows and the acceptance: row gamma of each request
+// through layers 0..k-1 (M = B), all B * (gamma + 1) rows through layers k..L-1 and the head.
+static ssd_status enqueue_verify_batch(ssd_ctx* c, int gamma, cudaGraphConditionalHandle cond, int has_cond) {
+  const int B = c->batch, d = c->dp, R = gamma + 1, rs = R * c->dp;
+  float* xg = c->xv + static_cast<size_t>(gamma) * d;
+  CK(launch_k(c, ssd_batch_embed_kernel, dim3(B), dim3(256), 0, c->embed, static_cast<const DevState*>(c->req),
+              gamma, xg, rs, c->cfg.d_model, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer_batch(c, l, xg, rs, B, 1, gamma));
+  for (int l = c->cfg.draft_exit_k; l < c->cfg.n_layers; ++l) CKS(enqueue_layer_batch(c, l, c->xv, d, B * R, R, 0));
+  CKS(enqueue_head_batch(c, c->xv, d, B * R, R, 0, &c->req[0].full_tok[0], false));
+  CK(launch_k(c, ssd_batch_accept_kernel, dim3(1), dim3(32 * ((B + 31) / 32)), 0, c->st, c->req, B, gamma, c->bout,
+              c->cfg.max_seq, c->blog, c->cfg.max_seq, cond, has_cond));
+  return SSD_OK;
+}
+
+// One greedy step of every request (the batched baseline): all L layers at M = B rows.
+static ssd_status enqueue_greedy_batch(ssd_ctx* c, cudaGraphConditionalHandle cond, int has_cond) {
+  const int B = c->batch, d = c->dp;
+  CK(launch_k(c, ssd_batch_embed_kernel, dim3(B), dim3(256), 0, c->embed, static_cast<const DevState*>(c->req), 0,
+              c->xv, d, c->cfg.d_model, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer_batch(c, l, c->xv, d, B, 1, 0));
+  CKS(enqueue_head_batch(c, c->xv, d, B, 1, 0, &c->req[0].full_tok[0], false));
+  CK(launch_k(c, ssd_batch_accept_kernel, dim3(1), dim3(32 * ((B + 31) / 32)), 0, c->st, c->req, B, 0, c->bout,
+              c->cfg.max_seq, c->blog, c->cfg.max_seq, cond, has_cond));
+  return SSD_OK;
+}
+
+static ssd_status enqueue_prefill_any(ssd_ctx* c, int n_vis, int n_prompt);
+
+// Prefill of request b: the single-request prefill with its state, token row, inputs and cache
+// slot swapped in (launched directly; every request has its own prompt length).
+static ssd_status enqueue_prefill_slot(ssd_ctx* c, int b, const __nv_bfloat16* vis, const int* prompt, int n_vis,
+                                       int n_prompt) {
+  DevState* st = c->st;
+  int* out = c->out_int;
+  __nv_bfloat16* iv = c->in_vis;
+  int* ip = c->in_prompt;
+  c->st = c->req + b;
+  c->out_int = c->bout + static_cast<size_t>(b) * c->cfg.max_seq;
+  c->in_vis = const_cast<__nv_bfloat16*>(vis);
+  c->in_prompt = const_cast<int*>(prompt);
+  c->kv_slot = static_cast<size_t>(b) * c->req_kv;
+  float* lg = c->logits_buf;  // request b's captured logits start at its own block of rows
+  if (lg) c->logits_buf = lg + static_cast<size_t>(b) * c->logits_rows * c->cfg.vocab;
+  const ssd_status r = enqueue_prefill_any(c, n_vis, n_prompt);
+  c->logits_buf = lg;
+  c->st = st;
+  c->out_int = out;
+  c->in_vis = iv;
+  c->in_prompt = ip;
+  c->kv_slot = 0;
+  return r;
+}
+
 // ------------------------------------------------------------------ graphs
 
 static ssd_status begin_capture(ssd_ctx* c, cudaGraph_t g) {
@@ -848,8 +1113,9 @@ static ssd_status end_capture(ssd_ctx* c, cudaGraph_t g, ssd_status inner) {
 }
 
 // Graph = [loop_begin] -> WHILE(cond) { body }.  body is draft+verify+accept
-// (gamma > 0) or one greedy step (gamma == 0).
-static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec, int64_t* body_launches) {
+// (gamma > 0) or one greedy step (gamma == 0), of one request or (batched) of every request.
+static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec, int64_t* body_launches,
+                                   bool batched = false) {
   cudaGraph_t g = nullptr;
   CK(cudaGraphCreate(&g, 0));
   cudaGraphConditionalHandle cond;
@@ -887,8 +1153,14 @@ static ssd_status build_loop_graph(ssd_ctx* c, int gamma, cudaGraphExec_t* exec,
     s = begin_capture(c, body);
     if (s == SSD_OK) {
       const int64_t l0 = c->launch_counter;
-      ssd_status inner = gamma > 0 ? enqueue_draft(c, gamma) : SSD_OK;
-      if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify(c, gamma, cond, 1) : enqueue_greedy_step(c, cond, 1);
+      ssd_status inner = SSD_OK;
+      if (batched) {
+        inner = gamma > 0 ? enqueue_draft_batch(c, gamma) : SSD_OK;
+        if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify_batch(c, gamma, cond, 1) : enqueue_greedy_batch(c, cond, 1);
+      } else {
+        inner = gamma > 0 ? enqueue_draft(c, gamma) : SSD_OK;
+        if (inner == SSD_OK) inner = gamma > 0 ? enqueue_verify(c, gamma, cond, 1) : enqueue_greedy_step(c, cond, 1);
+      }
       *body_launches = c->launch_counter - l0;
       s = end_capture(c, body, inner);
     }
@@ -1025,6 +1297,7 @@ static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) {
   if (c->t5) return enqueue_prefill_t5(c, a, b);
   return c->prefill_rows ? enqueue_prefill(c, a, b) : enqueue_prefill_tc(c, a, b);
 }
+static ssd_status enqueue_prefill_any(ssd_ctx* c, int n_vis, int n_prompt) { return enq_prefill_fn(c, n_vis, n_prompt); }
 static ssd_status enq_draft_fn(ssd_ctx* c, int g, int) { return enqueue_draft(c, g); }
 static ssd_status enq_verify_fn(ssd_ctx* c, int g, int) { return enqueue_verify(c, g, 0, 0); }
 // One decode step without a conditional node (host-driven loop, used for profiling).
@@ -1044,6 +1317,8 @@ static void drop_graphs(ssd_ctx* c) {
   for (auto& kv : c->dyn_graphs) cudaGraphExecDestroy(kv.second);
   c->dyn_graphs.clear();
   if (c->greedy_graph) cudaGraphExecDestroy(c->greedy_graph);
+  for (auto& kv : c->batch_graphs) cudaGraphExecDestroy(kv.second);
+  c->batch_graphs.clear();
   c->decode_graphs.clear();
   c->draft_graphs.clear();
   c->verify_graphs.clear();
@@ -1067,6 +1342,12 @@ static ssd_status read_device_error(ssd_ctx* c) {
   int errw = 0;
   CK(cudaMemcpy(&errw, reinterpret_cast<char*>(c->st) + offsetof(DevState, error), sizeof(int),
                 cudaMemcpyDeviceToHost));
+  for (int b = 0; b < c->batch; ++b) {  // a batched prefill records faults in the request's state
+    int e = 0;
+    CK(cudaMemcpy(&e, reinterpret_cast<char*>(c->req + b) + offsetof(DevState, error), sizeof(int),
+                  cudaMemcpyDeviceToHost));
+    errw |= e;
+  }
   if (errw & DERR_TIMEOUT) return fail(c, SSD_ERR_TIMEOUT, "a bounded device wait ran out (error word %d)", errw);
   if (errw) return fail(c, SSD_ERR_DEVICE, "device error word %d (1 = bad token id, 4 = position out of range)", errw);
   return SSD_OK;
@@ -1111,7 +1392,8 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->step_log, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
                   c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt,
                   c->x_enc, c->enc_q, c->enc_o, c->enc_k, c->enc_v, c->ckc, c->cvc, c->dec_bias, c->enc_bias, c->one,
-                  c->start_tok};
+                  c->start_tok, c->req, c->bout, c->blog, c->bvis, c->bprompt, c->act_hi, c->act_lo, c->act_rs,
+                  c->mid_partials};
   for (void* b : bufs)
     if (b) cudaFree(b);
   if (c->ev_in) cudaEventDestroy(c->ev_in);
@@ -1182,6 +1464,15 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   if (k.gamma_max < 1 || k.gamma_max > SSD_MAX_GAMMA || k.gamma_max + 1 > kMaxVerifyRows)
     return fail(c, SSD_ERR_INVALID_ARG, "gamma_max must be in [1, %d]", SSD_MAX_GAMMA);
   if (k.max_seq < 2) return fail(c, SSD_ERR_INVALID_ARG, "max_seq");
+  const int max_batch = k.max_batch < 1 ? 1 : k.max_batch;
+  if (max_batch > kMaxRows) return fail(c, SSD_ERR_INVALID_ARG, "max_batch %d > %d", k.max_batch, kMaxRows);
+  if (max_batch > 1) {
+    if (t5 || k.in_kind == SSD_IN_BLOCK)
+      return fail(c, SSD_ERR_INVALID_ARG, "batched requests need SSD_ARCH_LLAMA with SSD_IN_IDENTITY or SSD_IN_MLP2");
+    if (max_batch * (k.gamma_max + 1) > kMaxMidRows)
+      return fail(c, SSD_ERR_INVALID_ARG, "max_batch * (gamma_max + 1) = %d > %d", max_batch * (k.gamma_max + 1),
+                  kMaxMidRows);
+  }
   if (!w || !w->embed || !w->lm_head || !w->final_norm || !w->wq || !w->wk || !w->wv || !w->wo || !w->w_gate ||
       !w->w_up || !w->w_down || !w->attn_norm || !w->ffn_norm || !w->resid_scale)
     return fail(c, SSD_ERR_INVALID_ARG, "null weight pointer");
@@ -1241,8 +1532,10 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_head());
   CK(attn_attrs());
   CK(prefill_attrs());
+  CK(mid_attrs());
 
   c->cfg = k;
+  c->max_batch = max_batch;
   c->qdim = qdim;
   c->t5 = t5;
   c->max_enc = t5 ? k.max_enc : 0;
@@ -1331,8 +1624,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     t.down.tiles_n = (k.d_model + kTcN - 1) / kTcN;
   }
 
-  // owned memory
-  const int R = kMaxRows;
+  // owned memory (activation rows: one request's passes, or every request's verification rows)
+  const int R = std::max(kMaxRows, max_batch * (k.gamma_max + 1));
   const size_t d = k.d_model;
   CKS(alloc(c, reinterpret_cast<void**>(&c->st), sizeof(DevState)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->op_st), sizeof(DevState)));
@@ -1376,7 +1669,8 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     c->enc_final = copy_gain(slot++, ed->enc_final);
     if (!c->enc_final) return fail(c, SSD_ERR_CUDA, "copying norm gains failed");
   }
-  c->layer_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
+  c->req_kv = static_cast<size_t>(k.n_heads) * k.max_seq * k.head_dim;
+  c->layer_kv = c->req_kv * max_batch;
   CKS(alloc(c, reinterpret_cast<void**>(&c->kc), sizeof(float) * c->layer_kv * n_blocks));
   CKS(alloc(c, reinterpret_cast<void**>(&c->vc), sizeof(float) * c->layer_kv * n_blocks));
   CKS(alloc(c, reinterpret_cast<void**>(&c->rope), sizeof(float2) * k.max_seq * (k.head_dim / 2)));
@@ -1410,8 +1704,25 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_part),
-            sizeof(float) * k.n_heads * kAttnSplit * kAttnMaxRows * (k.head_dim + 2)));
-  CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * k.n_heads));
+            sizeof(float) * max_batch * k.n_heads * kAttnSplit * kAttnMaxRows * (k.head_dim + 2)));
+  CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * max_batch * k.n_heads));
+  if (max_batch > 1) {
+    const size_t S = k.max_seq;
+    CKS(alloc(c, reinterpret_cast<void**>(&c->req), sizeof(DevState) * max_batch));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->bout), sizeof(int) * max_batch * S));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->blog), sizeof(int2) * max_batch * S));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->bvis), sizeof(__nv_bfloat16) * max_batch * S * d));
+    CKS(alloc(c, reinterpret_cast<void**>(&c->bprompt), sizeof(int) * max_batch * S));
+    if (R > kMaxRows) {  // verification rows beyond the GEMV: the medium-M kernel's buffers
+      const size_t kmax = std::max(std::max(static_cast<size_t>(k.d_model), static_cast<size_t>(qdim)),
+                                   static_cast<size_t>(k.d_ff));
+      CKS(alloc(c, reinterpret_cast<void**>(&c->act_hi), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
+      CKS(alloc(c, reinterpret_cast<void**>(&c->act_lo), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
+      CKS(alloc(c, reinterpret_cast<void**>(&c->act_rs), sizeof(float) * kMaxMidRows));
+      CKS(alloc(c, reinterpret_cast<void**>(&c->mid_partials),
+                sizeof(float) * 2 * kGemvCtasPerSm * c->num_sms * kMaxMidRows * kTileN));
+    }
+  }
   CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_table), sizeof(int) * (k.max_seq + 1)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_launch), sizeof(int) * SSD_MAX_GAMMA));
   const size_t in_rows = std::max(static_cast<size_t>(k.max_seq), static_cast<size_t>(c->max_enc));
@@ -1479,6 +1790,7 @@ static ssd_status prefill_impl(ssd_ctx* c, int n_vis, int n_prompt) {
   }
   CK(cudaGraphLaunch(it->second, c->cs));
   c->prefilled = true;
+  c->batch = 0;  // slot 0 now holds this request: a batched decode needs a new batched prefill
   c->drafted_gamma = 0;
   c->prompt_len = c->t5 ? 1 : P;  // decoder positions before the first new token
   c->kv_upper = c->prompt_len;
@@ -1817,6 +2129,7 @@ ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t*
     int64_t body = 0;
     if (c->last_decode_kind == 1) body = c->decode_body_launches[c->last_gamma];
     if (c->last_decode_kind == 2) body = c->greedy_body_launches;
+    if (c->last_decode_kind == 4) body = c->batch_body_launches[c->last_gamma];
     // setup + loop_begin + steps x body + copy-out
     *decode_launches = c->last_decode_kind ? 2 + static_cast<int64_t>(h.steps) * body + 1 : 0;
     // dynamic draft length: setup + loop_begin + per step (select + branch + loop test) + copy-out,
@@ -1824,6 +2137,196 @@ ssd_status ssd_last_launch_count(ssd_ctx* c, int64_t* prefill_launches, int64_t*
     if (c->last_decode_kind == 3)
       *decode_launches = c->host_loop ? 2 + c->dyn_host_launches : 3 + static_cast<int64_t>(h.dyn_launches);
   }
+  return SSD_OK;
+}
+
+// ------------------------------------------------------------------ batched requests
+
+static ssd_status check_batch_args(ssd_ctx* c, int B, const void* vis, const int32_t* n_vis, const int32_t* prompt,
+                                   const int32_t* n_prompt) {
+  if (c->max_batch < 2) return fail(c, SSD_ERR_INVALID_ARG, "batched calls need a ctx created with max_batch >= 2");
+  if (B < 1 || B > c->max_batch) return fail(c, SSD_ERR_INVALID_ARG, "batch %d not in [1, %d]", B, c->max_batch);
+  if (!n_vis || !n_prompt) return fail(c, SSD_ERR_INVALID_ARG, "n_vis / n_prompt is null");
+  int64_t tv = 0, tp = 0;
+  for (int b = 0; b < B; ++b) {
+    if (n_vis[b] < 0 || n_prompt[b] < 0 || n_vis[b] + n_prompt[b] < 1)
+      return fail(c, SSD_ERR_INVALID_ARG, "request %d has an empty prompt", b);
+    if (n_vis[b] + n_prompt[b] + 1 > c->cfg.max_seq)
+      return fail(c, SSD_ERR_CAPACITY, "request %d: prompt longer than max_seq", b);
+    tv += n_vis[b];
+    tp += n_prompt[b];
+  }
+  if (tv > 0 && !vis) return fail(c, SSD_ERR_INVALID_ARG, "vis_emb is null");
+  if (tp > 0 && !prompt) return fail(c, SSD_ERR_INVALID_ARG, "prompt is null");
+  return SSD_OK;
+}
+
+static ssd_status prefill_batch_impl(ssd_ctx* c, int B, const int32_t* n_vis, const int32_t* n_prompt) {
+  size_t vo = 0, po = 0;
+  c->batch = 0;  // the request errors are read only once the batch is complete
+  for (int b = 0; b < B; ++b) {
+    CKS(enqueue_prefill_slot(c, b, c->bvis + vo * c->cfg.d_model, c->bprompt + po, n_vis[b], n_prompt[b]));
+    vo += n_vis[b];
+    po += n_prompt[b];
+  }
+  // the batch's own launch state (error word, argmax keys, tickets) starts clean
+  CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 0, c->cfg.eos_id, 0));
+  c->batch = B;
+  c->batch_prompt.assign(B, 0);
+  for (int b = 0; b < B; ++b) c->batch_prompt[b] = n_vis[b] + n_prompt[b];
+  c->prefilled = false;  // slot 0 now holds request 0 of the batch
+  if (c->batch_graph_b != B) {
+    for (auto& kv : c->batch_graphs) cudaGraphExecDestroy(kv.second);
+    c->batch_graphs.clear();
+    c->batch_graph_b = B;
+  }
+  return SSD_OK;
+}
+
+ssd_status ssd_prefill_batch(ssd_ctx* c, int B, const void* vis, const int32_t* n_vis, const int32_t* prompt,
+                             const int32_t* n_prompt, int32_t* first_tok) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CKS(check_batch_args(c, B, vis, n_vis, prompt, n_prompt));
+  CKS(enter(c));
+  int64_t tv = 0, tp = 0;
+  for (int b = 0; b < B; ++b) {
+    tv += n_vis[b];
+    tp += n_prompt[b];
+  }
+  if (tv > 0)
+    CK(cudaMemcpyAsync(c->bvis, vis, sizeof(__nv_bfloat16) * tv * c->cfg.d_model, cudaMemcpyDeviceToDevice, c->cs));
+  if (tp > 0) CK(cudaMemcpyAsync(c->bprompt, prompt, sizeof(int) * tp, cudaMemcpyDeviceToDevice, c->cs));
+  CKS(prefill_batch_impl(c, B, n_vis, n_prompt));
+  if (first_tok) ssd_batch_first_tokens_kernel<<<1, 32 * ((B + 31) / 32), 0, c->cs>>>(c->req, B, first_tok);
+  CK(cudaGetLastError());
+  return leave(c);
+}
+
+static ssd_status enq_batch_step_fn(ssd_ctx* c, int g, int) {
+  if (g == 0) return enqueue_greedy_batch(c, 0, 0);
+  CKS(enqueue_draft_batch(c, g));
+  return enqueue_verify_batch(c, g, 0, 0);
+}
+
+static ssd_status decode_batch_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_tok, int32_t* n_out) {
+  const int B = c->batch;
+  if (B < 1) return fail(c, SSD_ERR_STATE, "batched decode before ssd_prefill_batch");
+  if (max_new < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_new must be >= 1");
+  if (gamma < 0 || gamma > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma %d", gamma);
+  for (int b = 0; b < B; ++b)
+    if (static_cast<int64_t>(c->batch_prompt[b]) + max_new + gamma + 1 > c->cfg.max_seq)
+      return fail(c, SSD_ERR_CAPACITY, "request %d: prompt + max_new + gamma + 1 = %d > max_seq = %d", b,
+                  c->batch_prompt[b] + max_new + gamma + 1, c->cfg.max_seq);
+  auto it = c->batch_graphs.find(gamma);
+  if (it == c->batch_graphs.end()) {
+    cudaGraphExec_t ge;
+    int64_t nb = 0;
+    if (c->host_loop) CKS(build_plain_graph(c, enq_batch_step_fn, gamma, 0, &ge, &nb));
+    else CKS(build_loop_graph(c, gamma, &ge, &nb, true));
+    it = c->batch_graphs.emplace(gamma, ge).first;
+    c->batch_body_launches[gamma] = nb;
+  }
+  ssd_batch_setup_kernel<<<1, 32 * ((B + 31) / 32), 0, c->cs>>>(c->st, c->req, B, max_new, gamma);
+  CK(cudaGetLastError());
+  if (c->host_loop) {  // one plain graph per step; the host reads the batch's done flag
+    for (int i = 0; i < max_new; ++i) {
+      int done = 0;
+      CK(cudaMemcpyAsync(&done, reinterpret_cast<char*>(c->st) + offsetof(DevState, done), sizeof(int),
+                         cudaMemcpyDeviceToHost, c->cs));
+      CK(cudaStreamSynchronize(c->cs));
+      if (done) break;
+      CK(cudaGraphLaunch(it->second, c->cs));
+    }
+  } else {
+    CK(cudaGraphLaunch(it->second, c->cs));
+  }
+  if (out_tok || n_out)
+    ssd_batch_copy_out_kernel<<<B, 256, 0, c->cs>>>(c->req, c->bout, c->cfg.max_seq, out_tok, n_out, max_new);
+  CK(cudaGetLastError());
+  c->last_decode_kind = 4;
+  c->last_gamma = gamma;
+  return SSD_OK;
+}
+
+ssd_status ssd_decode_batch(ssd_ctx* c, int max_new, int gamma, int32_t* out_tok, int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (gamma < 1) return fail(c, SSD_ERR_INVALID_ARG, "gamma must be >= 1");
+  CKS(enter(c));
+  CKS(decode_batch_impl(c, max_new, gamma, out_tok, n_out));
+  return leave(c);
+}
+
+ssd_status ssd_greedy_decode_batch(ssd_ctx* c, int max_new, int32_t* out_tok, int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  CKS(enter(c));
+  CKS(decode_batch_impl(c, max_new, 0, out_tok, n_out));
+  return leave(c);
+}
+
+ssd_status ssd_generate_batch(ssd_ctx* c, int B, const void* vis, const int32_t* n_vis, const int32_t* prompt,
+                              const int32_t* n_prompt, int max_new, int gamma, int32_t* out, int32_t* n_out) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (!out || !n_out) return fail(c, SSD_ERR_INVALID_ARG, "out / n_out is null");
+  CKS(check_batch_args(c, B, vis, n_vis, prompt, n_prompt));
+  if (max_new < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_new must be >= 1");
+  int64_t tv = 0, tp = 0;
+  for (int b = 0; b < B; ++b) {
+    tv += n_vis[b];
+    tp += n_prompt[b];
+    if (static_cast<int64_t>(n_vis[b]) + n_prompt[b] + max_new + gamma + 1 > c->cfg.max_seq)
+      return fail(c, SSD_ERR_CAPACITY, "request %d: prompt + max_new + gamma + 1 > max_seq", b);
+  }
+  CKS(enter(c));
+  if (tv > 0)
+    CK(cudaMemcpyAsync(c->bvis, vis, sizeof(__nv_bfloat16) * tv * c->cfg.d_model, cudaMemcpyHostToDevice, c->cs));
+  if (tp > 0) CK(cudaMemcpyAsync(c->bprompt, prompt, sizeof(int) * tp, cudaMemcpyHostToDevice, c->cs));
+  CKS(prefill_batch_impl(c, B, n_vis, n_prompt));
+  CKS(decode_batch_impl(c, max_new, gamma, nullptr, nullptr));
+  CK(cudaMemcpy2DAsync(out, sizeof(int) * max_new, c->bout, sizeof(int) * c->cfg.max_seq, sizeof(int) * max_new, B,
+                       cudaMemcpyDeviceToHost, c->cs));
+  std::vector<DevState> h(B);
+  CK(cudaMemcpyAsync(h.data(), c->req, sizeof(DevState) * B, cudaMemcpyDeviceToHost, c->cs));
+  CK(cudaStreamSynchronize(c->cs));
+  CKS(read_device_error(c));
+  for (int b = 0; b < B; ++b) n_out[b] = h[b].n_out < max_new ? h[b].n_out : max_new;
+  return leave(c);
+}
+
+ssd_status ssd_get_batch_stats(ssd_ctx* c, int b, ssd_stats* out) {
+  if (!c || !out) return SSD_ERR_INVALID_ARG;
+  if (b < 0 || b >= c->batch) return fail(c, SSD_ERR_INVALID_ARG, "request %d of a batch of %d", b, c->batch);
+  CK(cudaStreamSynchronize(c->cs));
+  DevState h;
+  CK(cudaMemcpy(&h, c->req + b, sizeof(DevState), cudaMemcpyDeviceToHost));
+  memset(out, 0, sizeof(*out));
+  out->steps = h.steps;
+  out->drafted = h.drafted;
+  out->accepted = h.accepted;
+  out->emitted = h.n_out;
+  for (int i = 0; i <= SSD_MAX_GAMMA; ++i) out->accept_hist[i] = h.hist[i];
+  out->kv_len = h.kv_len;
+  return SSD_OK;
+}
+
+ssd_status ssd_get_batch_step_log(ssd_ctx* c, int b, int32_t* accepted, int32_t* drafted, int cap, int* n_steps) {
+  if (!c || !n_steps || cap < 0 || (cap > 0 && !accepted && !drafted)) return SSD_ERR_INVALID_ARG;
+  if (b < 0 || b >= c->batch) return fail(c, SSD_ERR_INVALID_ARG, "request %d of a batch of %d", b, c->batch);
+  CK(cudaStreamSynchronize(c->cs));
+  int steps = 0;
+  CK(cudaMemcpy(&steps, reinterpret_cast<char*>(c->req + b) + offsetof(DevState, steps), sizeof(int),
+                cudaMemcpyDeviceToHost));
+  steps = std::min(steps, c->cfg.max_seq);
+  const int n = std::min(steps, cap);
+  if (n > 0) {
+    std::vector<int2> h(n);
+    CK(cudaMemcpy(h.data(), c->blog + static_cast<size_t>(b) * c->cfg.max_seq, sizeof(int2) * n,
+                  cudaMemcpyDeviceToHost));
+    for (int i = 0; i < n; ++i) {
+      if (accepted) accepted[i] = h[i].x;
+      if (drafted) drafted[i] = h[i].y;
+    }
+  }
+  *n_steps = steps;
   return SSD_OK;
 }
 
@@ -1866,7 +2369,10 @@ ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float
 
 ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, int reps, int64_t* bytes) {
   if (!c) return SSD_ERR_INVALID_ARG;
-  if (rows < 1 || rows > kMaxVerifyRows || reps < 1) return fail(c, SSD_ERR_INVALID_ARG, "rows / reps");
+  // projections: up to kMaxRows rows through the GEMV, beyond that (a ctx with batched verification
+  // rows) through the medium-M kernel; attention up to one request's verification rows
+  const int max_rows = which == 7 ? kMaxVerifyRows : (c->act_hi ? std::min(kMaxMidRows, c->cfg.max_seq) : kMaxRows);
+  if (rows < 1 || rows > max_rows || reps < 1) return fail(c, SSD_ERR_INVALID_ARG, "rows / reps");
   if (which < 0 || which > 7 || layer < 0 || layer >= c->cfg.n_layers)
     return fail(c, SSD_ERR_INVALID_ARG, "which / layer");
   if (which == 7) {  // split-KV attention of `layer` for rows kv_len .. kv_len+rows-1
@@ -1882,8 +2388,8 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     c->prefilled = false;
     return leave(c);
   }
-  if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows != 1))
-    return fail(c, SSD_ERR_INVALID_ARG, "imitation projections need SSD_IN_MLP2 and rows == 1");
+  if ((which == 5 || which == 6) && (c->cfg.in_kind != SSD_IN_MLP2 || rows > kMaxRows))
+    return fail(c, SSD_ERR_INVALID_ARG, "imitation projections need SSD_IN_MLP2 and rows <= %d", kMaxRows);
   const int d = c->dp;
   const Site* site = nullptr;
   Epi e = Epi::RESID;
@@ -1897,8 +2403,8 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       p.gain = c->attn_norm[layer];
       p.q_out = c->qb;
       p.q_stride = c->qp;
-      p.k_cache = c->kc + layer * c->layer_kv;
-      p.v_cache = c->vc + layer * c->layer_kv;
+      p.k_cache = kv_k(c, layer);
+      p.v_cache = kv_v(c, layer);
       p.head_dim = c->cfg.head_dim;
       p.max_seq = c->cfg.max_seq;
       p.rope_cs = c->t5 ? nullptr : c->rope;
@@ -1925,7 +2431,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
       site = &c->head;
       e = Epi::ARGMAX;
       p.gain = c->final_norm;
-      p.tok_dst = st_field(c, offsetof(DevState, full_tok));
+      p.tok_dst = rows <= kMaxRows ? st_field(c, offsetof(DevState, full_tok)) : c->out_int;
       break;
     case 5:
       site = &c->in1;
@@ -1952,8 +2458,9 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     *bytes = N * site->K * 2 + static_cast<int64_t>(rows) * site->K * 4 + (p.gain ? site->K * 2 : 0) + out_bytes +
              (e == Epi::RESID ? static_cast<int64_t>(rows) * site->N * 4 : 0);
   CKS(enter(c));
-  for (int r = 0; r < reps; ++r) CKS(gemv(c, e, rows, *site, p));
+  for (int r = 0; r < reps; ++r) CKS(proj_rows(c, e, rows, *site, p));
   c->prefilled = false;
+  c->batch = 0;
   return leave(c);
 }
 

@@ -1,4 +1,4 @@
-// Weight-streaming skinny GEMM ("GEMV" for M = 1..9 activation rows) on the
+// Weight-streaming skinny GEMM ("GEMV" for M = 1..16 activation rows) on the
 // 5th-generation tensor cores.
 //
 //   out[m][n] = sum_k W[n][k] * a[m][k],   W bf16 [N][K] (nn.Linear layout), a fp32
@@ -97,12 +97,27 @@ struct GemvParams {
   // before its own wait.
   int late_trigger;
   int seg_base;  // QKV: segment of the site's first matrix (0 = q; 1 = k, for a [k; v] site)
+  // Batched requests (batch_rows = 0: one request, whose state is st).  With batch_rows = R > 0,
+  // row m belongs to request b = m / R at offset i = pos_off + m % R within the request's rows:
+  // it sits at position req_st[b].kv_len + i, its K/V rows are at k_cache / v_cache + b * req_kv,
+  // its argmax goes to tok_dst[b * tok_stride + m % R], and a logits capture writes
+  // logits[b][row][N] (full-model rows by the index of the predicted token within the request,
+  // draft rows by req_st[b].steps * logits_step_rows + i).  st still holds the error word and the
+  // argmax keys of the launch.
+  int batch_rows;
+  DevState* req_st;
+  long long req_kv;
+  int tok_stride;
+  // Medium-M kernel only: the rows' RMSNorm scales 1/rms(x_m), computed by the split kernel
+  // (the gain is folded into its bf16 hi/lo parts).
+  const float* rs_in;
   int abs_pos;   // row m sits at position pos_off + m, st->kv_len ignored (the encoder's rows)
   int act;       // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up (gated GELU)
 };
 
 template <int M>
 struct GemvSmem {
+  static constexpr int kPreRows = M <= 9 ? M : 0;  // epilogue inputs fetched early (rows up to 9)
   static constexpr int kActBytes = M * kTileK * 4;
   static constexpr int kW = 0;                                  // [stages][16 KB] weight units (1024-aligned)
   static constexpr int kB = kW + kStages * kWTileBytes;         // [stages][hi | lo] B operands (1024-aligned)
@@ -110,7 +125,8 @@ struct GemvSmem {
   static constexpr int kG = kA + kStages * kActBytes;           // [stages][64] bf16 gain slices
   static constexpr int kOut = kG + kStages * kTileK * 2;        // drained row tile [M][128]
   static constexpr int kPre = kOut + M * kTileN * 4;             // epilogue inputs fetched early: [2][M][128] fp32
-  static constexpr int kRs = kPre + 2 * M * kTileN * 4;
+  static constexpr int kRowPos = kPre + 2 * kPreRows * kTileN * 4;  // batched rows: position, request [2][kMaxRows]
+  static constexpr int kRs = kRowPos + 2 * kMaxRows * 4;
   static constexpr int kRed = kRs + kMaxRows * 4;               // [4][kMaxRows]
   static constexpr int kFlag = kRed + 4 * kMaxRows * 4;
   static constexpr int kBar = (kFlag + 16 + 7) & ~7;            // full, empty, bready [stages]; afull, aempty [2]
@@ -185,18 +201,27 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 lo, __nv_bfloat16 
 }
 
 // ------------------------------------------------------------------ epilogues
-// Run on the 128 drain threads with the finished row tile in out ([M][kTileN],
-// fp32, before the RMSNorm scale) and rs[m] (1 if no norm).  pre: inputs fetched
-// into shared memory after the upstream wait, or null -- QKV: the rotation table
-// rows of the M positions ([M][head_dim / 2] float2); RESID: the tile's base rows
-// ([M][kTileN]).  base_pos: position of row 0 (st->kv_len + pos_off, or pos_off with abs_pos; read
-// once per CTA).
+// Run on the 128 drain threads with a finished row tile in out ([MT][kTileN],
+// fp32, before the RMSNorm scale) and rs[m] (1 if no norm) for the mc <= MT
+// rows m0 .. m0 + mc - 1 of the launch (local row m is launch row m0 + m).
+// pre: inputs fetched into shared memory after the upstream wait, or null --
+// QKV: the rotation table rows of the rows' positions ([mc][head_dim / 2]
+// float2); RESID: the tile's base rows ([mc][kTileN]).  base_pos: position of
+// launch row 0 (st->kv_len + pos_off, or pos_off with abs_pos; read once per
+// CTA) for one request; with batch_rows, rpos[m] / rreq[m] hold the position
+// and the request of launch row m instead (rpos is null for one request).
 
 __device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
 
-template <int M, Epi EPI>
+// Launch row mg's request and offset within the request's rows (batch_rows > 0).
+__device__ __forceinline__ int batch_offset(const GemvParams& p, int mg, int b) {
+  return p.pos_off + mg - b * p.batch_rows;
+}
+
+template <int MT, Epi EPI>
 __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const float* out, const float* rs,
-                                              const float* pre, int base_pos, int tid) {
+                                              const float* pre, int base_pos, const int* rpos, const int* rreq,
+                                              int tid, int m0, int mc) {
   if constexpr (EPI == Epi::QKV) {
     const int r0 = rt * kTileN;
     const int seg = r0 / p.seg_rows;       // source matrix of this row tile within the site
@@ -204,11 +229,11 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     const int local0 = r0 - seg * p.seg_rows;
     const int Dh = p.head_dim, half = Dh >> 1;
     if (mat < 2) {
-      for (int idx = tid; idx < M * (kTileN / 2); idx += kDrainThreads) {
-        const int m = idx / (kTileN / 2), pr = idx - m * (kTileN / 2);
+      for (int idx = tid; idx < mc * (kTileN / 2); idx += kDrainThreads) {
+        const int m = idx / (kTileN / 2), pr = idx - m * (kTileN / 2), mg = m0 + m;
         const int hh = pr / half, j = pr - hh * half;
         const int ra = hh * Dh + j, rb = ra + half;
-        const int pos = base_pos + m;
+        const int pos = rpos ? rpos[mg] : base_pos + mg;
         if (pos < 0 || pos >= p.max_seq) {
           set_error(p.st, DERR_POS);
           continue;
@@ -223,42 +248,43 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
           vb = a * cs.y + b * cs.x;
         }
         if (mat == 0) {
-          p.q_out[m * p.q_stride + local0 + ra] = va;
-          p.q_out[m * p.q_stride + local0 + rb] = vb;
+          p.q_out[mg * p.q_stride + local0 + ra] = va;
+          p.q_out[mg * p.q_stride + local0 + rb] = vb;
         } else {
           const int h = local0 / Dh + hh;
-          float* kr = p.k_cache + (static_cast<size_t>(h) * p.max_seq + pos) * Dh;
+          float* kr = p.k_cache + (rreq ? rreq[mg] * p.req_kv : 0ll) + (static_cast<size_t>(h) * p.max_seq + pos) * Dh;
           kr[j] = va;
           kr[j + half] = vb;
         }
       }
     } else {
-      for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
-        const int m = idx / kTileN, i = idx - m * kTileN;
-        const int pos = base_pos + m;
+      for (int idx = tid; idx < mc * kTileN; idx += kDrainThreads) {
+        const int m = idx / kTileN, i = idx - m * kTileN, mg = m0 + m;
+        const int pos = rpos ? rpos[mg] : base_pos + mg;
         if (pos < 0 || pos >= p.max_seq) {
           set_error(p.st, DERR_POS);
           continue;
         }
         const int row = local0 + i, h = row / Dh, d = row - h * Dh;
-        p.v_cache[(static_cast<size_t>(h) * p.max_seq + pos) * Dh + d] = out[idx] * rs[m];
+        p.v_cache[(rreq ? rreq[mg] * p.req_kv : 0ll) + (static_cast<size_t>(h) * p.max_seq + pos) * Dh + d] =
+            out[idx] * rs[m];
       }
     }
   } else if constexpr (EPI == Epi::GATE_SILU) {
-    for (int idx = tid; idx < M * kHalfN; idx += kDrainThreads) {
+    for (int idx = tid; idx < mc * kHalfN; idx += kDrainThreads) {
       const int m = idx / kHalfN, j = idx - m * kHalfN;
       const int n = rt * kHalfN + j;
       if (n >= p.N) continue;
       const float g = out[m * kTileN + j] * rs[m];
       const float u = out[m * kTileN + kHalfN + j] * rs[m];
-      p.h_out[m * p.h_stride + n] = (p.act ? gelu_tanh_f(g) : silu_f(g)) * u;
+      p.h_out[(m0 + m) * p.h_stride + n] = (p.act ? gelu_tanh_f(g) : silu_f(g)) * u;
     }
   } else if constexpr (EPI == Epi::SILU) {
-    for (int idx = tid; idx < M * kTileN; idx += kDrainThreads) {
+    for (int idx = tid; idx < mc * kTileN; idx += kDrainThreads) {
       const int m = idx / kTileN, i = idx - m * kTileN;
       const int n = rt * kTileN + i;
       if (n >= p.N) continue;
-      p.h_out[m * p.h_stride + n] = silu_f(out[idx] * rs[m]);
+      p.h_out[(m0 + m) * p.h_stride + n] = silu_f(out[idx] * rs[m]);
     }
   } else if constexpr (EPI == Epi::RESID) {
     // thread tid owns column tid of every row; the base rows are loaded before any store
@@ -267,25 +293,38 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     const float s = __ldg(p.scale);
     const int n = rt * kTileN + tid;
     if (n < p.N) {
-      float bv[M];
+      float bv[MT];
 #pragma unroll
-      for (int m = 0; m < M; ++m) bv[m] = pre ? pre[m * kTileN + tid] : __ldcg(p.base + m * p.base_stride + n);
+      for (int m = 0; m < MT; ++m)
+        if (m < mc) bv[m] = pre ? pre[m * kTileN + tid] : __ldcg(p.base + (m0 + m) * p.base_stride + n);
 #pragma unroll
-      for (int m = 0; m < M; ++m) p.dst[m * p.dst_stride + n] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
+      for (int m = 0; m < MT; ++m)
+        if (m < mc) p.dst[(m0 + m) * p.dst_stride + n] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
     }
-  } else {  // ARGMAX (LM head): argmax over the vocabulary, lowest index on ties
+  } else {  // ARGMAX (LM head): this tile's keys of the rows; gemv_argmax_finish turns them into tokens
     const int lane = tid & 31;
-    const int row0 = p.logits == nullptr ? 0
+    const int row0 = (p.logits == nullptr || rpos) ? 0
                      : p.logits_step_rows > 0 ? __ldcg(&p.st->steps) * p.logits_step_rows + p.pos_off
                                               : base_pos + 1 - __ldcg(&p.st->prompt_len);
     const int n = rt * kTileN + tid;  // thread per tile row
     const bool valid = n < p.N;
 #pragma unroll
-    for (int m = 0; m < M; ++m) {
+    for (int m = 0; m < MT; ++m) {
+      if (m >= mc) break;
+      const int mg = m0 + m;
       const float logit = out[m * kTileN + tid] * rs[m];
       if (p.logits != nullptr && valid) {
-        const int row = row0 + m;
-        if (row >= 0 && row < p.logits_rows) p.logits[static_cast<size_t>(row) * p.N + n] = logit;
+        if (rpos) {  // batched: rows [request][logits_rows]
+          const int b = rreq[mg];
+          const int row = p.logits_step_rows > 0
+                              ? __ldcg(&p.req_st[b].steps) * p.logits_step_rows + batch_offset(p, mg, b)
+                              : rpos[mg] + 1 - __ldcg(&p.req_st[b].prompt_len);
+          if (row >= 0 && row < p.logits_rows)
+            p.logits[(static_cast<size_t>(b) * p.logits_rows + row) * p.N + n] = logit;
+        } else {
+          const int row = row0 + mg;
+          if (row >= 0 && row < p.logits_rows) p.logits[static_cast<size_t>(row) * p.N + n] = logit;
+        }
       }
       unsigned long long key = valid ? argmax_key(logit, static_cast<uint32_t>(n)) : 0ull;
 #pragma unroll
@@ -293,22 +332,33 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
         const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
         key = o > key ? o : key;
       }
-      if (lane == 0) atomicMax(&p.st->am_key[m], key);
+      if (lane == 0) atomicMax(&p.st->am_key[mg], key);
     }
-    // the tile's maxima are released by one acq_rel ticket after the CTA barrier; the tile
-    // that completes the count reads and resets the M keys, one thread per row
-    __shared__ int am_last;
-    drain_sync();
-    if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(p.n_rt - 1);
-    drain_sync();
-    if (am_last) {
-      if (tid < M) {  // -1 once a bounded wait anywhere has given up: the keys may miss tiles
-        const unsigned long long key = atomicExch(&p.st->am_key[tid], 0ull);
-        const bool stopped = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
-        p.tok_dst[tid] = stopped ? -1 : static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
+  }
+}
+
+// LM head, after a row tile's keys of all M launch rows are in: the tile's maxima are released
+// by one acq_rel ticket after the CTA barrier; the tile that completes the count reads and resets
+// the M keys, one thread per row, and writes the tokens (-1 once a bounded wait anywhere has
+// given up: the keys may miss tiles).
+__device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, int M, const int* rreq, int tid) {
+  __shared__ int am_last;
+  drain_sync();
+  if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(p.n_rt - 1);
+  drain_sync();
+  if (am_last) {
+    const bool stopped = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
+    for (int r = tid; r < M; r += kDrainThreads) {
+      const unsigned long long key = atomicExch(&p.st->am_key[r], 0ull);
+      const int tok = stopped ? -1 : static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
+      if (rreq) {
+        const int b = rreq[r];
+        p.tok_dst[b * p.tok_stride + (r - b * p.batch_rows)] = tok;
+      } else {
+        p.tok_dst[r * (p.tok_stride ? p.tok_stride : 1)] = tok;
       }
-      if (tid == 0) atomicExch(&p.st->am_count, 0u);
     }
+    if (tid == 0) atomicExch(&p.st->am_count, 0u);
   }
 }
 
@@ -535,18 +585,27 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
     // the base rows of this CTA's first and last row tiles (RESID; every contributor of a split
     // tile fetches them, whichever ends up owning it, before its ticket)
     const int rt_first = u0 / p.n_kt, rt_last = (u1 - 1) / p.n_kt;
-    const int base_pos = (p.abs_pos ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
+    const int base_pos = (p.abs_pos || p.batch_rows ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
     float* pre = reinterpret_cast<float*>(smem + S::kPre);
+    // batched rows: each row's position and request, once per CTA
+    int* rpos = p.batch_rows ? reinterpret_cast<int*>(smem + S::kRowPos) : nullptr;
+    int* rreq = p.batch_rows ? rpos + kMaxRows : nullptr;
+    if (rpos && dt < M) {
+      const int b = dt / p.batch_rows;
+      rreq[dt] = b;
+      rpos[dt] = __ldcg(&p.req_st[b].kv_len) + batch_offset(p, dt, b);
+    }
     bool pre_rope = false;
-    if constexpr (EPI == Epi::QKV) {
+    if constexpr (EPI == Epi::QKV && S::kPreRows > 0) {
       const int half = p.head_dim >> 1;
-      pre_rope = p.rope_cs != nullptr && base_pos >= 0 && base_pos + M <= p.max_seq && half <= kTileN;
+      pre_rope = p.rope_cs != nullptr && !p.batch_rows && base_pos >= 0 && base_pos + M <= p.max_seq &&
+                 half <= kTileN;
       if (pre_rope)
         for (int idx = dt; idx < M * half; idx += kDrainThreads) {
           const int m = idx / half, j = idx - m * half;
           reinterpret_cast<float2*>(pre)[idx] = p.rope_cs[static_cast<size_t>(base_pos + m) * half + j];
         }
-    } else if constexpr (EPI == Epi::RESID) {
+    } else if constexpr (EPI == Epi::RESID && S::kPreRows > 0) {
       const int nb = rt_last == rt_first ? 1 : 2;
       for (int idx = dt; idx < nb * M * kTileN; idx += kDrainThreads) {
         const int b = idx / (M * kTileN), r = idx - b * (M * kTileN), m = r / kTileN, i = r - m * kTileN;
@@ -557,7 +616,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
     drain_sync();
     auto pre_of = [&](int rt) -> const float* {
       if constexpr (EPI == Epi::QKV) return pre_rope ? pre : nullptr;
-      if constexpr (EPI == Epi::RESID) {
+      if constexpr (EPI == Epi::RESID && S::kPreRows > 0) {
         if (rt == rt_first) return pre;
         if (rt == rt_last) return pre + M * kTileN;
       }
@@ -585,7 +644,8 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       drain_sync();
       const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
       if (whole) {
-        gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, dt);
+        gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
+        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
       } else {
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
@@ -661,7 +721,8 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
             }
           }
           drain_sync();
-          gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, dt);
+          gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
+          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
           if (dt == 0) p.counters[rt] = 0u;
         }
       }

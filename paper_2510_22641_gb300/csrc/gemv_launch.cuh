@@ -29,21 +29,22 @@ cudaError_t gemv_attr_m() {
 
 }  // namespace ssd
 
-// Defines gemv_launch_<name>(M, ...) and gemv_attrs_<name>() for M = 1..MAXM.
+// Defines gemv_launch_<name>(M, ...) and gemv_attrs_<name>() for M = 1..16.
 #define SSD_GEMV_CASE(M_, EPI_) \
   case M_:                      \
     return gemv_launch_m<M_, EPI_>(maps, p, grid, s, pdl);
 #define SSD_GEMV_ATTR(M_, EPI_)               \
   if ((e = gemv_attr_m<M_, EPI_>()) != cudaSuccess) return e;
 
-#define SSD_DEFINE_GEMV_9(NAME, EPI_)                                                                         \
+#define SSD_DEFINE_GEMV_16(NAME, EPI_)                                                                        \
   namespace ssd {                                                                                           \
   cudaError_t gemv_launch_##NAME(int M, const CUtensorMap* maps, const GemvParams& p, int grid, cudaStream_t s, \
                                  bool pdl) {                                                                \
     switch (M) {                                                                                            \
       SSD_GEMV_CASE(1, EPI_) SSD_GEMV_CASE(2, EPI_) SSD_GEMV_CASE(3, EPI_) SSD_GEMV_CASE(4, EPI_)            \
       SSD_GEMV_CASE(5, EPI_) SSD_GEMV_CASE(6, EPI_) SSD_GEMV_CASE(7, EPI_) SSD_GEMV_CASE(8, EPI_)            \
-      SSD_GEMV_CASE(9, EPI_)                                                                                \
+      SSD_GEMV_CASE(9, EPI_) SSD_GEMV_CASE(10, EPI_) SSD_GEMV_CASE(11, EPI_) SSD_GEMV_CASE(12, EPI_)         \
+      SSD_GEMV_CASE(13, EPI_) SSD_GEMV_CASE(14, EPI_) SSD_GEMV_CASE(15, EPI_) SSD_GEMV_CASE(16, EPI_)        \
       default:                                                                                              \
         return cudaErrorInvalidValue;                                                                       \
     }                                                                                                       \
@@ -52,24 +53,8 @@ cudaError_t gemv_attr_m() {
     cudaError_t e;                                                                                          \
     SSD_GEMV_ATTR(1, EPI_) SSD_GEMV_ATTR(2, EPI_) SSD_GEMV_ATTR(3, EPI_) SSD_GEMV_ATTR(4, EPI_)              \
     SSD_GEMV_ATTR(5, EPI_) SSD_GEMV_ATTR(6, EPI_) SSD_GEMV_ATTR(7, EPI_) SSD_GEMV_ATTR(8, EPI_)              \
-    SSD_GEMV_ATTR(9, EPI_)                                                                                  \
-    return cudaSuccess;                                                                                     \
-  }                                                                                                         \
-  }
-
-#define SSD_DEFINE_GEMV_1(NAME, EPI_)                                                                         \
-  namespace ssd {                                                                                           \
-  cudaError_t gemv_launch_##NAME(int M, const CUtensorMap* maps, const GemvParams& p, int grid, cudaStream_t s, \
-                                 bool pdl) {                                                                \
-    switch (M) {                                                                                            \
-      SSD_GEMV_CASE(1, EPI_)                                                                                \
-      default:                                                                                              \
-        return cudaErrorInvalidValue;                                                                       \
-    }                                                                                                       \
-  }                                                                                                         \
-  cudaError_t gemv_attrs_##NAME() {                                                                         \
-    cudaError_t e;                                                                                          \
-    SSD_GEMV_ATTR(1, EPI_)                                                                                  \
+    SSD_GEMV_ATTR(9, EPI_) SSD_GEMV_ATTR(10, EPI_) SSD_GEMV_ATTR(11, EPI_) SSD_GEMV_ATTR(12, EPI_)           \
+    SSD_GEMV_ATTR(13, EPI_) SSD_GEMV_ATTR(14, EPI_) SSD_GEMV_ATTR(15, EPI_) SSD_GEMV_ATTR(16, EPI_)          \
     return cudaSuccess;                                                                                     \
   }                                                                                                         \
   }

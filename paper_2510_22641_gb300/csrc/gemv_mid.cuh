@@ -1,0 +1,377 @@
+// Medium-M weight-streaming GEMM on the 5th-generation tensor cores: the
+// verification pass of batched requests, M = 17..128 activation rows.
+//
+//   out[m][n] = sum_k W[n][k] * a[m][k],   W bf16 [N][K] (nn.Linear layout), a fp32
+//
+// In the serving form of Algorithm 1 every request of a batch verifies its
+// gamma + 1 rows in the same full-depth pass, so one projection carries
+// B * (gamma + 1) rows (112 for 16 requests at gamma = 6).  Each weight byte now
+// meets up to 128 rows: a real dense contraction, still bound by the weight
+// stream.  The kernel keeps ssd_wstream_kernel's stream-K unit partition (units of
+// 128 weight rows x 64 columns, contiguous CTA ranges, split row tiles summed in
+// CTA order by the CTA that takes the tile's last ticket), its MMA orientation
+// (the weight unit is A, M = 128; the activations are B) and its fused epilogues,
+// and changes what the row count makes expensive:
+//  * the B operand is no longer converted inside every CTA: ssd_split_act_kernel
+//    turns the M rows into bf16 hi + lo parts once per projection (RMSNorm gain
+//    folded in, exactly as the GEMV's converter warps do) and computes the rows'
+//    RMSNorm scales; warp 0 TMA-loads the parts as 128-byte swizzled [NP][64]
+//    tiles beside each weight unit (NP = M rounded up to 16 is the MMA's N);
+//  * 2 stages of 16 KB weights + 2 x NP x 128 B per CTA and 2 CTAs per SM;
+//  * a row tile's accumulator is NP TMEM columns (two 128-column buffers), read
+//    back 16 columns -- 16 activation rows -- at a time by warps 2..5, which run
+//    the GEMV epilogues on each 16-row chunk.
+// The per-element arithmetic is the GEMV's: a = hi + lo, 4 K slices x (hi, lo)
+// MMAs per unit accumulating in fp32, the RMSNorm scale applied after the
+// products, and the split-tile sums in CTA order.
+#pragma once
+
+#include "gemv.cuh"
+
+namespace ssd {
+
+constexpr int kMidStages = 2;
+constexpr int kMidThreads = 192;    // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 drain
+constexpr int kMidTmemCols = 256;   // two 128-column accumulators
+constexpr uint32_t kMidBBytes = kMaxMidRows * kTileK * 2;  // one B part (hi or lo) of up to 128 rows: 16 KB
+constexpr int kMidSlot = kMaxMidRows * kTileN;             // floats of one partial row tile, [m][128]
+
+struct MidSmem {
+  static constexpr int kW = 0;                                  // [stages][16 KB] weight units
+  static constexpr int kBh = kW + kMidStages * kWTileBytes;     // [stages][NP][64] bf16 hi
+  static constexpr int kBl = kBh + kMidStages * kMidBBytes;     // [stages][NP][64] bf16 lo
+  static constexpr int kOut = kBl + kMidStages * kMidBBytes;    // one drained 16-row chunk [16][128] fp32
+  static constexpr int kRs = kOut + kNPad * kTileN * 4;         // [128] RMSNorm scales
+  static constexpr int kRowPos = kRs + kMaxMidRows * 4;         // [2][128] positions, requests
+  static constexpr int kFlag = kRowPos + 2 * kMaxMidRows * 4;
+  static constexpr int kBar = (kFlag + 16 + 7) & ~7;            // full, empty [stages]; afull, aempty [2]
+  static constexpr int kTmemSlot = kBar + (2 * kMidStages + 4) * 8;
+  static constexpr int kTotal = kTmemSlot + 16 + 1024;          // + slack for the 1024-byte alignment
+};
+
+// ------------------------------------------------------------------ activation split
+// Row r of hi / lo (bf16 [rows][ld]) = the split of x[r] * gain (gain null: x[r]): v = x * g,
+// hi = bf16(v), lo = bf16(v - hi); rs[r] = 1/sqrt(mean(x[r]^2) + eps) with gain, 1 without.
+// 128 threads per row and the same summation order as the GEMV's drain warps, so the scale is
+// bitwise the one the GEMV computes for the row.
+__global__ void __launch_bounds__(kDrainThreads) ssd_split_act_kernel(const float* __restrict__ x, int x_stride,
+                                                                      int K, const __nv_bfloat16* __restrict__ gain,
+                                                                      float eps, __nv_bfloat16* __restrict__ hi,
+                                                                      __nv_bfloat16* __restrict__ lo, int ld,
+                                                                      float* __restrict__ rs) {
+  __shared__ float red[4];
+  pdl_trigger();
+  pdl_wait();
+  const int r = blockIdx.x, t = threadIdx.x, lane = t & 31;
+  const float* xr = x + static_cast<size_t>(r) * x_stride;
+  if (gain) {
+    float ss = 0.f;
+    for (int i = t; i < (K >> 2); i += kDrainThreads) {
+      const float4 v = __ldcg(reinterpret_cast<const float4*>(xr) + i);
+      ss = fmaf(v.x, v.x, ss);
+      ss = fmaf(v.y, v.y, ss);
+      ss = fmaf(v.z, v.z, ss);
+      ss = fmaf(v.w, v.w, ss);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    if (lane == 0) red[t >> 5] = ss;
+    __syncthreads();
+    if (t == 0) {
+      float s = 0.f;
+      for (int w = 0; w < 4; ++w) s += red[w];
+      rs[r] = rsqrtf(s / static_cast<float>(K) + eps);
+    }
+  } else if (t == 0) {
+    rs[r] = 1.0f;
+  }
+  __nv_bfloat16* hr = hi + static_cast<size_t>(r) * ld;
+  __nv_bfloat16* lr = lo + static_cast<size_t>(r) * ld;
+  for (int i = t; i < (K >> 3); i += kDrainThreads) {
+    const float4 a0 = __ldcg(reinterpret_cast<const float4*>(xr) + 2 * i);
+    const float4 a1 = __ldcg(reinterpret_cast<const float4*>(xr) + 2 * i + 1);
+    float v[8] = {a0.x, a0.y, a0.z, a0.w, a1.x, a1.y, a1.z, a1.w};
+    if (gain) {
+      const uint4 gv = __ldg(reinterpret_cast<const uint4*>(gain) + i);
+      const float2 g0 = bf16x2_to_float2(gv.x), g1 = bf16x2_to_float2(gv.y), g2 = bf16x2_to_float2(gv.z),
+                   g3 = bf16x2_to_float2(gv.w);
+      v[0] *= g0.x; v[1] *= g0.y; v[2] *= g1.x; v[3] *= g1.y;
+      v[4] *= g2.x; v[5] *= g2.y; v[6] *= g3.x; v[7] *= g3.y;
+    }
+    uint32_t hw[4], lw[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]), h1 = __float2bfloat16_rn(v[2 * e + 1]);
+      const __nv_bfloat16 l0 = __float2bfloat16_rn(v[2 * e] - __bfloat162float(h0));
+      const __nv_bfloat16 l1 = __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1));
+      hw[e] = pack_bf16x2(h0, h1);
+      lw[e] = pack_bf16x2(l0, l1);
+    }
+    reinterpret_cast<uint4*>(hr)[i] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    reinterpret_cast<uint4*>(lr)[i] = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+  }
+}
+
+// ------------------------------------------------------------------ kernel
+// map0..2: the site's weight matrices (as for ssd_wstream_kernel); map_hi / map_lo: the split
+// activations [128][K] with [NP][64] boxes.  M rows, NP = M rounded up to 16.
+template <Epi EPI>
+__global__ void __launch_bounds__(kMidThreads, 2)
+    ssd_wstream_mid_kernel(const __grid_constant__ CUtensorMap map0, const __grid_constant__ CUtensorMap map1,
+                           const __grid_constant__ CUtensorMap map2, const __grid_constant__ CUtensorMap map_hi,
+                           const __grid_constant__ CUtensorMap map_lo, const GemvParams p, int M) {
+  using S = MidSmem;
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  uint64_t* empty = full + kMidStages;
+  uint64_t* afull = empty + kMidStages;
+  uint64_t* aempty = afull + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
+  float* outb = reinterpret_cast<float*>(smem + S::kOut);
+  float* rs = reinterpret_cast<float*>(smem + S::kRs);
+  int* flag = reinterpret_cast<int*>(smem + S::kFlag);
+
+  const int G = gridDim.x, c = blockIdx.x;
+  const int u0 = unit_begin(c, p.units, G), u1 = unit_begin(c + 1, p.units, G);
+  const int n_units = u1 - u0;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int NP = (M + 15) & ~15;
+  const uint32_t bbytes = static_cast<uint32_t>(NP) * kTileK * 2;
+  const uint32_t tx = kWTileBytes + 2 * bbytes;
+
+  if (!p.late_trigger) pdl_trigger();
+  if (*reinterpret_cast<volatile int*>(&p.st->error) & DERR_TIMEOUT) return;
+
+  if (tid == 0) {
+    for (int s = 0; s < kMidStages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&afull[b], 1);
+      mbar_init(&aempty[b], 4);
+    }
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kMidTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  tmem_fence_before();
+  __syncthreads();
+  tmem_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      auto issue_weights = [&](int s, int u) {
+        const int rt = u / p.n_kt, kt = u - rt * p.n_kt;
+        uint8_t* wdst = smem + S::kW + s * kWTileBytes;
+        const int x = kt * kTileK;
+        if constexpr (EPI == Epi::GATE_SILU) {
+          tma_load_2d(wdst, &map0, &full[s], x, rt * kHalfN);
+          tma_load_2d(wdst + kWTileBytes / 2, &map1, &full[s], x, rt * kHalfN);
+        } else if constexpr (EPI == Epi::QKV) {
+          const int r0 = rt * kTileN, mat = r0 / p.seg_rows;
+          tma_load_2d(wdst, mat == 0 ? &map0 : (mat == 1 ? &map1 : &map2), &full[s], x, r0 - mat * p.seg_rows);
+        } else {
+          tma_load_2d(wdst, &map0, &full[s], x, rt * kTileN);
+        }
+      };
+      auto issue_acts = [&](int s, int u) {
+        const int x = (u % p.n_kt) * kTileK;
+        tma_load_2d(smem + S::kBh + s * kMidBBytes, &map_hi, &full[s], x, 0);
+        tma_load_2d(smem + S::kBl + s * kMidBBytes, &map_lo, &full[s], x, 0);
+      };
+      prefetch_tensormap(&map0);
+      const int npre = n_units < kMidStages ? n_units : kMidStages;
+      for (int i = 0; i < npre; ++i) {
+        mbar_arrive_expect_tx(&full[i], tx);
+        issue_weights(i, u0 + i);  // weights do not depend on the previous kernel
+      }
+      pdl_wait();
+      if (p.late_trigger) pdl_trigger();
+      for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
+      for (int i = npre; i < n_units; ++i) {
+        const int s = i % kMidStages;
+        if (!mbar_wait(&empty[s], static_cast<uint32_t>((i / kMidStages) - 1) & 1u)) {
+          set_error(p.st, DERR_TIMEOUT);
+          break;
+        }
+        mbar_arrive_expect_tx(&full[s], tx);
+        issue_weights(s, u0 + i);
+        issue_acts(s, u0 + i);
+      }
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      const uint32_t idesc = umma_idesc_bf16(kTileN, NP);
+      int sg = 0;
+      bool seg_open = false;
+      uint32_t d = tmem;
+      for (int i = 0; i < n_units; ++i) {
+        const int u = u0 + i, kt = u % p.n_kt, s = i % kMidStages;
+        if (!seg_open) {  // a new row-tile segment: take a free accumulator
+          const int b = sg & 1;
+          if (!mbar_wait(&aempty[b], static_cast<uint32_t>(((sg >> 1) & 1) ^ 1))) {
+            set_error(p.st, DERR_TIMEOUT);
+            break;
+          }
+          tmem_fence_after();
+          d = tmem + static_cast<uint32_t>(b * kMaxMidRows);
+        }
+        if (!mbar_wait(&full[s], static_cast<uint32_t>(i / kMidStages) & 1u)) {
+          set_error(p.st, DERR_TIMEOUT);
+          break;
+        }
+        tmem_fence_after();
+        const uint64_t adesc = umma_desc_sw128(smem_u32(smem + S::kW + s * kWTileBytes));
+        const uint64_t hdesc = umma_desc_sw128(smem_u32(smem + S::kBh + s * kMidBBytes));
+        const uint64_t ldesc = umma_desc_sw128(smem_u32(smem + S::kBl + s * kMidBBytes));
+#pragma unroll
+        for (int kk = 0; kk < kTileK / 16; ++kk) {
+          // +32 bytes (2 descriptor units) per 16-element K slice inside the swizzled row
+          umma_f16(d, adesc + 2 * kk, hdesc + 2 * kk, idesc, (seg_open || kk > 0) ? 1u : 0u);
+          umma_f16(d, adesc + 2 * kk, ldesc + 2 * kk, idesc, 1u);
+          seg_open = true;
+        }
+        umma_commit(&empty[s]);  // stage s may be refilled once these MMAs have read it
+        if (kt == p.n_kt - 1 || i == n_units - 1) {
+          umma_commit(&afull[sg & 1]);  // the row tile's accumulator is complete
+          ++sg;
+          seg_open = false;
+        }
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- drain + epilogues (warps 2..5)
+    const int dt = tid - 64;  // 0..127
+    const int q = warp & 3;   // TMEM lane quadrant: tile rows 32q .. 32q+31
+    pdl_wait();
+    for (int m = dt; m < M; m += kDrainThreads) rs[m] = p.rs_in ? __ldcg(p.rs_in + m) : 1.0f;
+    const int base_pos = (p.abs_pos || p.batch_rows ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
+    int* rpos = p.batch_rows ? reinterpret_cast<int*>(smem + S::kRowPos) : nullptr;
+    int* rreq = p.batch_rows ? rpos + kMaxMidRows : nullptr;
+    if (rpos)
+      for (int m = dt; m < M; m += kDrainThreads) {
+        const int b = m / p.batch_rows;
+        rreq[m] = b;
+        rpos[m] = __ldcg(&p.req_st[b].kv_len) + batch_offset(p, m, b);
+      }
+    drain_sync();
+    const int rt_first = u0 / p.n_kt;
+    const int n_ch = (M + kNPad - 1) / kNPad;
+    int seg_kt0 = u0 - rt_first * p.n_kt;
+    int sg = 0;
+    bool ok = true;
+    for (int i = 0; ok && i < n_units; ++i) {
+      const int u = u0 + i, rt = u / p.n_kt, kt = u - rt * p.n_kt;
+      if (!(kt == p.n_kt - 1 || i == n_units - 1)) continue;
+      const int b = sg & 1;
+      if (!mbar_wait(&afull[b], static_cast<uint32_t>((sg >> 1) & 1))) {
+        set_error(p.st, DERR_TIMEOUT);
+        break;
+      }
+      tmem_fence_after();
+      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kMaxMidRows);
+      const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
+      if (whole) {
+        for (int ch = 0; ch < n_ch; ++ch) {
+          float v[kNPad];
+          tmem_ld16(tbase + ch * kNPad, v);
+#pragma unroll
+          for (int m = 0; m < kNPad; ++m) outb[m * kTileN + q * 32 + lane] = v[m];
+          drain_sync();
+          const int m0 = ch * kNPad, mc = min(kNPad, M - m0);
+          gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
+          drain_sync();
+        }
+        tmem_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&aempty[b]);  // the MMA warp may reuse accumulator b
+        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
+      } else {
+        const int slot = 2 * c + (rt == rt_first ? 0 : 1);
+        float* dstp = p.partials + static_cast<size_t>(slot) * kMidSlot;
+        for (int ch = 0; ch < n_ch; ++ch) {
+          float v[kNPad];
+          tmem_ld16(tbase + ch * kNPad, v);
+#pragma unroll
+          for (int m = 0; m < kNPad; ++m)
+            if (ch * kNPad + m < M) __stcg(dstp + (ch * kNPad + m) * kTileN + q * 32 + lane, v[m]);
+        }
+        tmem_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&aempty[b]);
+        // the tile's ticket releases this CTA's partial (CTA barrier, then one acq_rel atomic)
+        drain_sync();
+        const int c_first = unit_owner(rt * p.n_kt, p.units, G);
+        const int c_last = unit_owner(rt * p.n_kt + p.n_kt - 1, p.units, G);
+        if (dt == 0) {
+          const unsigned prev = atom_add_acq_rel_gpu(&p.counters[rt], 1u);
+          flag[0] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
+        }
+        drain_sync();
+        if (flag[0]) {
+          // sum the contributors' partials in CTA order, one 16-row chunk at a time
+          const int nsp = c_last - c_first + 1;
+          const int slot0 = 2 * c_first + (unit_begin(c_first, p.units, G) / p.n_kt == rt ? 0 : 1);
+          const float4* part = reinterpret_cast<const float4*>(p.partials);
+          constexpr int kSlotF4 = kMidSlot / 4;
+          for (int ch = 0; ch < n_ch; ++ch) {
+            const int m0 = ch * kNPad, mc = min(kNPad, M - m0);
+            const int f0 = m0 * (kTileN / 4), nf = mc * (kTileN / 4);
+            for (int f = dt; f < nf; f += kDrainThreads) {
+              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+              for (int k0 = 0; k0 < nsp; k0 += 8) {
+                float4 pv[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                  const int k = k0 + j;
+                  const int sl = k == 0 ? slot0 : 2 * (c_first + k);
+                  pv[j] = k < nsp ? __ldcg(part + static_cast<size_t>(sl) * kSlotF4 + f0 + f)
+                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                  if (k0 + j >= nsp) continue;
+                  if (k0 + j == 0) {
+                    sum = pv[j];
+                  } else {
+                    sum.x += pv[j].x;
+                    sum.y += pv[j].y;
+                    sum.z += pv[j].z;
+                    sum.w += pv[j].w;
+                  }
+                }
+              }
+              reinterpret_cast<float4*>(outb)[f] = sum;
+            }
+            drain_sync();
+            gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
+            drain_sync();
+          }
+          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
+          if (dt == 0) p.counters[rt] = 0u;
+        }
+      }
+      drain_sync();
+      seg_kt0 = 0;
+      ++sg;
+    }
+  }
+  tmem_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tmem_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kMidTmemCols) : "memory");
+  }
+}
+
+}  // namespace ssd

@@ -1,3 +1,3 @@
-// ssd_wstream_kernel instantiations with the RESID epilogue, M = 1..9 rows.
+// ssd_wstream_kernel instantiations with the RESID epilogue, M = 1..16 rows.
 #include "gemv_launch.cuh"
-SSD_DEFINE_GEMV_9(resid, ssd::Epi::RESID)
+SSD_DEFINE_GEMV_16(resid, ssd::Epi::RESID)

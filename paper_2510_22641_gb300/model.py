@@ -193,11 +193,13 @@ class SSDModel:
         return st.as_dict()
 
     def set_logits_capture(self, buf: torch.Tensor | None):
-        self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
+        """buf: device fp32 [max_rows][vocab], or [batch][max_rows][vocab] for batched requests."""
+        self._call("ssd_set_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[-2])
 
     def set_draft_logits_capture(self, buf: torch.Tensor | None):
-        """buf: device fp32 [max_steps][gamma_max][vocab]; draft j of step s writes buf[s][j]."""
-        self._call("ssd_set_draft_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[0])
+        """buf: device fp32 [max_steps][gamma_max][vocab] (draft j of step s writes buf[s][j]), or
+        [batch][max_steps][gamma_max][vocab] for batched requests."""
+        self._call("ssd_set_draft_logits_capture", _ptr(buf), 0 if buf is None else buf.shape[-3])
 
     def step_log(self, cap: int = 4096) -> tuple[list, list]:
         """(accepted a, drafted gamma_eff) of every step since the last prefill."""
@@ -210,12 +212,15 @@ class SSDModel:
 
     def kv(self):
         """(K, V, kv_len): zero-copy torch views [L][H][max_seq][Dh] (fp32) of the library's cache
-        ([L + 1] with the block imitation network, whose rows are slot L)."""
+        ([L + 1] with the block imitation network, whose rows are slot L; [L][max_batch][H][max_seq][Dh]
+        for a ctx with max_batch > 1)."""
         k, v, n = ctypes.c_void_p(), ctypes.c_void_p(), ctypes.c_int()
         self._call("ssd_get_kv", ctypes.byref(k), ctypes.byref(v), ctypes.byref(n))
         c = self.cfg
         slots = c["n_layers"] + (1 if c["in_kind"] == B.SSD_IN_BLOCK else 0)
         shape = (slots, c["n_heads"], c["max_seq"], c["head_dim"])
+        if c.get("max_batch", 1) > 1:
+            shape = (slots, c["max_batch"], c["n_heads"], c["max_seq"], c["head_dim"])
         return _device_view(k.value, shape), _device_view(v.value, shape), n.value
 
     def lm_head(self, x: torch.Tensor, tok: torch.Tensor, logits: torch.Tensor | None = None):
@@ -229,6 +234,52 @@ class SSDModel:
         b = ctypes.c_int64()
         self._call("ssd_profile_projection", self.PROJECTIONS[which], layer, rows, reps, ctypes.byref(b))
         return b.value
+
+    # ------------------------------------------------------------------ batched requests
+    def prefill_batch(self, vis: torch.Tensor | None, n_vis, prompt: torch.Tensor, n_prompt,
+                      first_tok: torch.Tensor | None = None):
+        """ssd_prefill_batch: vis bf16 [sum n_vis][d] and prompt int32 [sum n_prompt] on the device, the
+        requests' rows concatenated in order; n_vis / n_prompt: per-request counts (host)."""
+        nv = np.ascontiguousarray(n_vis, dtype=np.int32)
+        npr = np.ascontiguousarray(n_prompt, dtype=np.int32)
+        self._call("ssd_prefill_batch", len(nv), _ptr(vis), nv.ctypes.data, _ptr(prompt), npr.ctypes.data,
+                   _ptr(first_tok))
+
+    def decode_batch(self, max_new: int, gamma: int, out_tok: torch.Tensor | None = None,
+                     n_out: torch.Tensor | None = None):
+        """ssd_decode_batch: out_tok int32 [B][max_new], n_out int32 [B] on the device."""
+        self._call("ssd_decode_batch", max_new, gamma, _ptr(out_tok), _ptr(n_out))
+
+    def greedy_decode_batch(self, max_new: int, out_tok: torch.Tensor | None = None,
+                            n_out: torch.Tensor | None = None):
+        self._call("ssd_greedy_decode_batch", max_new, _ptr(out_tok), _ptr(n_out))
+
+    def generate_batch(self, vis: np.ndarray | None, n_vis, prompt: np.ndarray, n_prompt, max_new: int,
+                       gamma: int) -> list:
+        """ssd_generate_batch with host buffers (vis: bf16 bit patterns [sum n_vis][d], prompt int32);
+        gamma = 0 decodes greedily.  Returns each request's tokens."""
+        nv = np.ascontiguousarray(n_vis, dtype=np.int32)
+        npr = np.ascontiguousarray(n_prompt, dtype=np.int32)
+        pr = np.ascontiguousarray(prompt, dtype=np.int32)
+        vp = None if vis is None else np.ascontiguousarray(vis)
+        out = np.zeros((len(nv), max_new), dtype=np.int32)
+        n = np.zeros(len(nv), dtype=np.int32)
+        self._call("ssd_generate_batch", len(nv), None if vp is None else vp.ctypes.data, nv.ctypes.data,
+                   pr.ctypes.data, npr.ctypes.data, max_new, gamma, out.ctypes.data, n.ctypes.data)
+        return [out[b, :n[b]].tolist() for b in range(len(nv))]
+
+    def batch_stats(self, b: int) -> dict:
+        st = B.SSDStats()
+        self._call("ssd_get_batch_stats", b, ctypes.byref(st))
+        return st.as_dict()
+
+    def batch_step_log(self, b: int, cap: int = 4096) -> tuple[list, list]:
+        acc = np.zeros(cap, dtype=np.int32)
+        dr = np.zeros(cap, dtype=np.int32)
+        n = ctypes.c_int(0)
+        self._call("ssd_get_batch_step_log", b, acc.ctypes.data, dr.ctypes.data, cap, ctypes.byref(n))
+        m = min(n.value, cap)
+        return acc[:m].tolist(), dr[:m].tolist()
 
     def launch_counts(self) -> tuple[int, int]:
         a, b = ctypes.c_int64(), ctypes.c_int64()

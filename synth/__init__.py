@@ -245,12 +245,24 @@ def _gain(w: Workload, kind: str, layer: int, n: int) -> np.ndarray:
     return normal_bf16(w.weight_seed, stream_id(kind, layer), (n,), mean=1.0, std=0.1)
 
 
-def make_weights(w: Workload) -> dict:
+def make_layer_weights(w: Workload, l: int) -> dict:
+    """Decoder layer l's weights (l = IN_BLOCK_LAYER: the imitation block's) as bf16 bit arrays."""
+    lw = {}
+    for name, shp in layer_shapes(w.shape).items():
+        if name.endswith("norm"):
+            lw[name] = _gain(w, name, l, shp[0])
+        else:
+            lw[name] = normal_bf16(w.weight_seed, stream_id(name, l), shp, std=w.weight_std)
+    return lw
+
+
+def make_weights(w: Workload, with_layers: bool = True) -> dict:
     """All weights of the workload as bf16 bit arrays, nn.Linear layout [out][in].
 
     Returns {"embed", "lm_head", "final_norm", "layers": [ {wq, ...}, ... ],
              "in_norm", "in_w1", "in_w2"} (IN_MLP2) or "in_block": {wq, ...} (IN_BLOCK);
-    no IN entries for IN_IDENTITY.
+    no IN entries for IN_IDENTITY.  with_layers=False leaves "layers" empty (large models build
+    them one at a time with make_layer_weights).
     """
     sh = w.shape
     d, V = sh.d_model, sh.vocab
@@ -261,19 +273,11 @@ def make_weights(w: Workload) -> dict:
         "final_norm": _gain(w, "final_norm", 0, d),
         "layers": [],
     }
-    def block(l: int) -> dict:
-        lw = {}
-        for name, shp in layer_shapes(sh).items():
-            if name.endswith("norm"):
-                lw[name] = _gain(w, name, l, shp[0])
-            else:
-                lw[name] = normal_bf16(w.weight_seed, stream_id(name, l), shp, std=std)
-        return lw
-
-    for l in range(sh.n_layers):
-        out["layers"].append(block(l))
+    if with_layers:
+        for l in range(sh.n_layers):
+            out["layers"].append(make_layer_weights(w, l))
     if w.in_kind == IN_BLOCK:
-        out["in_block"] = block(IN_BLOCK_LAYER)
+        out["in_block"] = make_layer_weights(w, IN_BLOCK_LAYER)
     if w.in_kind == IN_MLP2:
         out["in_norm"] = _gain(w, "in_norm", 0, d)
         out["in_w1"] = normal_bf16(w.weight_seed, stream_id("in_w1"), (w.in_hidden, d), std=std)
