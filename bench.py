@@ -683,7 +683,9 @@ def run_sweep(args) -> None:
 def run_profile(args) -> None:
     """A profiler window around one phase (run under `ncu --profile-from-start off`): the 7B layer
     shape with --layers layers (fewer layers keep a capture to a few GB on the device while every
-    weight matrix keeps its full size), or with --encdec the FlanT5-xl layer shape.  Decode phases
+    weight matrix keeps its full size), with --encdec the FlanT5-xl layer shape, or with --batch16
+    the 13B layer shape and 16 batched ragged requests (proj at --rows up to 112 then runs the
+    medium-M kernel).  Decode phases
     run the host-driven loop (SSD_OPT_HOST_LOOP), since profilers do not see kernels inside
     conditional graph nodes.  Phases: greedy / ssd (--tokens new tokens), prefill, proj (reps
     launches of one kernel alone: --proj qkv, o, gateup, down, head, in1, in2 or attn at --rows)."""
@@ -703,6 +705,21 @@ def run_profile(args) -> None:
                                  w.max_new + lib.SSD_MAX_GAMMA + 2, w.enc_len, options=lib.SSD_OPT_HOST_LOOP)
         rs = torch.tensor(w.dec_scale(), device="cuda")
         vis, prompt = synth.make_t5_inputs(w)
+    elif args.batch16:   # the 13B layer shape, 16 ragged requests (batched calls)
+        bw = synth.LLAVA13B_B16
+        shape = synth.ModelShape(args.layers, 5120, 40, 128, 13824, 32000)
+        w = bw.base.replace(shape=shape, draft_exit_k=min(bw.base.draft_exit_k, args.layers), s=args.s)
+        bw = bw.replace(base=w)
+        bits = synth.make_weights(w)
+        dev = {k: up(bits[k]) for k in ("embed", "lm_head", "final_norm", "in_norm", "in_w1", "in_w2")}
+        dev["layers"] = [{n: up(a) for n, a in lw.items()} for lw in bits["layers"]]
+        cfg = lib.config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, w.gamma, bw.max_seq(),
+                              options=lib.SSD_OPT_HOST_LOOP, max_batch=bw.batch)
+        rs = torch.tensor(w.resid_scale(), device="cuda")
+        ins = synth.make_batch_inputs(bw)
+        vis = np.concatenate([v for v, _ in ins])
+        prompt = np.concatenate([p for _, p in ins])
+        counts = ([v.shape[0] for v, _ in ins], [len(p) for _, p in ins])
     else:
         base = synth.LLAVA7B
         shape = synth.ModelShape(args.layers, 4096, 32, 128, 11008, 32000)
@@ -719,19 +736,25 @@ def run_profile(args) -> None:
     p = torch.from_numpy(prompt.astype(np.int32)).cuda()
     n = 1 + args.tokens
 
-    def phase():
-        if args.profile == "greedy":
-            model.greedy_decode(n)
-        elif args.profile == "ssd":
-            model.decode(n, w.gamma)
-        elif args.profile == "proj":
-            model.profile_projection(args.proj, 0, args.rows, 3)
+    def prefill():
+        if args.batch16:
+            model.prefill_batch(v, counts[0], p, counts[1])
         else:
             model.prefill(v, p)
 
-    model.prefill(v, p)
+    def phase():
+        if args.profile == "greedy":
+            (model.greedy_decode_batch if args.batch16 else model.greedy_decode)(n)
+        elif args.profile == "ssd":
+            (model.decode_batch if args.batch16 else model.decode)(n, w.gamma)
+        elif args.profile == "proj":
+            model.profile_projection(args.proj, 0, args.rows, 3)
+        else:
+            prefill()
+
+    prefill()
     phase()                     # builds the graphs, warms up
-    model.prefill(v, p)
+    prefill()
     model.sync()
     torch.cuda.profiler.start()
     phase()

@@ -423,6 +423,25 @@ SSD_API ssd_status ssd_lm_head_static(const void* lm_head, const void* final_nor
  * ssd_prefill before decoding again.  async. */
 SSD_API ssd_status ssd_profile_projection(ssd_ctx* ctx, int which, int layer, int rows, int reps, int64_t* bytes);
 
+/* ---- Failure-path diagnostics (for tests of callers' error handling; no GPU fault is made) ---- */
+
+/* Host-side fault injection: after this call, the countdown-th device allocation
+ * (kind SSD_FAULT_ALLOC: reported as SSD_ERR_OOM) or the countdown-th kernel launch
+ * through the library's launch wrappers (kind SSD_FAULT_LAUNCH: reported as
+ * SSD_ERR_CUDA, the kernel is not launched) of any ctx fails once, without
+ * reaching the GPU.  kind SSD_FAULT_NONE or countdown <= 0 disarms.  Process-wide;
+ * not thread-safe against concurrent ssd_* calls. */
+enum { SSD_FAULT_NONE = 0, SSD_FAULT_ALLOC = 1, SSD_FAULT_LAUNCH = 2 };
+SSD_API void ssd_set_fault_injection(int kind, int countdown);
+
+/* Runs out one bounded device wait on purpose: a kernel waits, with the same
+ * bounded-wait helper every pipeline stage uses, on an mbarrier phase that never
+ * completes, for limit_ns (0 .. 2e9) nanoseconds, then records the timeout in the
+ * ctx's error word like any stage that gives up.  The next ssd_sync returns
+ * SSD_ERR_TIMEOUT; decode kernels enqueued meanwhile skip their work; the next
+ * ssd_prefill / ssd_prefill_batch clears the word and the ctx is usable again.  async. */
+SSD_API ssd_status ssd_probe_bounded_wait(ssd_ctx* ctx, int64_t limit_ns);
+
 SSD_API const char* ssd_status_string(ssd_status s);
 SSD_API const char* ssd_last_error(const ssd_ctx* ctx);
 

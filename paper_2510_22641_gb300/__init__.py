@@ -4,13 +4,20 @@ The compute lives in libssd.so (hand-written CUDA, C ABI in include/ssd.h);
 this package only builds it and marshals arguments.
 """
 from . import _binding
-from ._binding import (SSD_ARCH_LLAMA, SSD_ARCH_T5, SSD_IN_IDENTITY, SSD_IN_MLP2, SSD_MAX_GAMMA, SSD_OPT_HOST_LOOP,
-                       SSD_OPT_PREFILL_ROWS, SSDError, load)
+from ._binding import (SSD_ARCH_LLAMA, SSD_ARCH_T5, SSD_FAULT_ALLOC, SSD_FAULT_LAUNCH, SSD_FAULT_NONE, SSD_IN_IDENTITY,
+                       SSD_IN_MLP2, SSD_MAX_GAMMA, SSD_OPT_HOST_LOOP, SSD_OPT_PREFILL_ROWS, SSDError, load)
 from .build import build
 
 __all__ = ["build", "load", "SSDError", "SSD_ARCH_LLAMA", "SSD_ARCH_T5", "SSD_IN_IDENTITY", "SSD_IN_MLP2",
-           "SSD_MAX_GAMMA", "SSD_OPT_HOST_LOOP", "SSD_OPT_PREFILL_ROWS", "SSDModel", "bf16_bits_to_device", "encdec_device_weights", "config_dict",
-           "t5_config_dict"]
+           "SSD_MAX_GAMMA", "SSD_OPT_HOST_LOOP", "SSD_OPT_PREFILL_ROWS", "SSD_FAULT_NONE", "SSD_FAULT_ALLOC",
+           "SSD_FAULT_LAUNCH", "SSDModel", "bf16_bits_to_device", "encdec_device_weights", "config_dict",
+           "t5_config_dict", "set_fault_injection"]
+
+
+def set_fault_injection(kind: int, countdown: int) -> None:
+    """ssd_set_fault_injection: the countdown-th allocation or launch after this call fails once on
+    the host (tests of the error paths; no GPU fault)."""
+    load().ssd_set_fault_injection(kind, countdown)
 
 
 def __getattr__(name):

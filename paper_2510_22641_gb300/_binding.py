@@ -21,6 +21,9 @@ SSD_ARCH_LLAMA = 0
 SSD_ARCH_T5 = 1
 SSD_OPT_HOST_LOOP = 1
 SSD_OPT_PREFILL_ROWS = 2
+SSD_FAULT_NONE = 0
+SSD_FAULT_ALLOC = 1
+SSD_FAULT_LAUNCH = 2
 
 STATUS = {0: "SSD_OK", 1: "SSD_ERR_INVALID_ARG", 2: "SSD_ERR_OOM", 3: "SSD_ERR_CUDA", 4: "SSD_ERR_CAPACITY",
           5: "SSD_ERR_STATE", 6: "SSD_ERR_TIMEOUT", 7: "SSD_ERR_DEVICE", 8: "SSD_ERR_UNSUPPORTED"}
@@ -31,7 +34,8 @@ EXPORTED = ("ssd_create", "ssd_destroy", "ssd_prefill", "ssd_draft", "ssd_verify
             "ssd_set_logits_capture", "ssd_set_draft_logits_capture", "ssd_get_step_log", "ssd_get_kv",
             "ssd_last_launch_count", "ssd_prefill_batch", "ssd_decode_batch", "ssd_greedy_decode_batch",
             "ssd_generate_batch", "ssd_get_batch_stats", "ssd_get_batch_step_log", "ssd_lm_head",
-            "ssd_lm_head_static", "ssd_profile_projection", "ssd_status_string", "ssd_last_error")
+            "ssd_lm_head_static", "ssd_profile_projection", "ssd_set_fault_injection", "ssd_probe_bounded_wait",
+            "ssd_status_string", "ssd_last_error")
 
 
 class SSDConfig(ctypes.Structure):
@@ -113,12 +117,15 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_get_batch_stats": [vp, i32, ctypes.POINTER(SSDStats)],
         "ssd_get_batch_step_log": [vp, i32, vp, vp, i32, ctypes.POINTER(i32)],
         "ssd_lm_head": [vp, vp, i32, vp, vp],
+        "ssd_probe_bounded_wait": [vp, ctypes.c_int64],
         "ssd_lm_head_static": [vp, vp, vp, i32, i32, i32, ctypes.c_float, vp, vp, vp],
     }
     for name, args in sig.items():
         f = getattr(lib, name)
         f.argtypes = args
         f.restype = ctypes.c_int
+    lib.ssd_set_fault_injection.argtypes = [ctypes.c_int, ctypes.c_int]
+    lib.ssd_set_fault_injection.restype = None
     lib.ssd_draft_length.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int]
     lib.ssd_draft_length.restype = ctypes.c_int
     lib.ssd_rel_bucket.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int]

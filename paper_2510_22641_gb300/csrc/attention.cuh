@@ -27,6 +27,7 @@
 // request z, whose M rows are rows z*M .. z*M+M-1 of q and o, whose keys are
 // its own cache rows (k_cache / v_cache + z * req_kv) and whose base is
 // req_st[z].kv_len + pos_off; requests never share a CTA, a state or a ticket.
+// A request that is done reads no keys (its output rows are zero and unused).
 //
 // With prefetch_old set, the launch before this one triggered its dependents
 // only after its own upstream grid had completed, so everything older than that
@@ -139,6 +140,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const
   bool bad = false;
   auto geometry = [&]() {
     base = ((EXT && p.abs_pos) ? 0 : __ldcg(p.batch_rows ? &p.req_st[z].kv_len : &p.st->kv_len)) + p.pos_off;
+    if (p.batch_rows && __ldcg(&p.req_st[z].done)) {  // a finished request's rows are never used
+      n_keys = my_chunks = 0;
+      return;
+    }
     if (EXT && p.fixed_keys) {
       const int ne = __ldcg(&p.st->enc_len);
       bad = base < 0 || ne < 1 || ne > p.max_seq;

@@ -84,14 +84,19 @@ __device__ __forceinline__ uint64_t globaltimer_ns() {
   return t;
 }
 
-// Waits for the phase with the given parity; gives up after ~2 s and returns false.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+// Waits for the phase with the given parity; gives up after limit_ns and returns false.
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, uint64_t limit_ns) {
   if (mbar_try_wait(bar, parity)) return true;
   const uint64_t t0 = globaltimer_ns();
   for (uint32_t i = 1;; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
-    if ((i & 255u) == 0u && globaltimer_ns() - t0 > 2000000000ull) return false;
+    if ((i & 255u) == 0u && globaltimer_ns() - t0 > limit_ns) return false;
   }
+}
+
+// The library's bounded wait: gives up after ~2 s.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  return mbar_wait_for(bar, parity, 2000000000ull);
 }
 
 // 2D tiled TMA load of one box into shared memory, completing on `bar`.

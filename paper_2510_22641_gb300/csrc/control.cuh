@@ -360,6 +360,19 @@ __global__ void ssd_batch_copy_out_kernel(const DevState* req, const int* out_in
   if (threadIdx.x == 0 && user_n) user_n[b] = n;
 }
 
+// Diagnostic of the failure path: one thread waits, with the kernels' bounded-wait helper and a
+// limit of limit_ns, on the first phase of a fresh mbarrier that nothing ever completes, so the wait
+// runs out and records DERR_TIMEOUT exactly as a stalled pipeline stage would.  No copy is in flight
+// and no other thread waits.
+__global__ void ssd_wait_probe_kernel(DevState* st, unsigned long long limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+    if (!mbar_wait_for(&bar, 0u, limit_ns)) set_error(st, DERR_TIMEOUT);
+  }
+}
+
 // cos/sin of pos * theta^(-2j/head_dim), computed in fp64 and rounded to fp32.
 __global__ void ssd_rope_table_kernel(float2* cs, int max_seq, int head_dim, double theta) {
   const int half = head_dim / 2;

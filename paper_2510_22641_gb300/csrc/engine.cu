@@ -13,6 +13,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <algorithm>
+#include <atomic>
 #include <cstdlib>
 #include <cstring>
 #include <map>
@@ -45,7 +46,7 @@ cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, cons
                                 float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
                                 cudaStream_t s, bool pdl);
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
-                       int grid, cudaStream_t s, bool pdl);
+                       int num_sms, cudaStream_t s, bool pdl);
 cudaError_t mid_attrs();
 cudaError_t split_act_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                              __nv_bfloat16* hi, __nv_bfloat16* lo, int ld, float* rs, int rows, cudaStream_t s,
@@ -81,6 +82,18 @@ struct TcLayer {
 };
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+
+// Host-side fault injection for tests of the error paths (ssd_set_fault_injection): the countdown-th
+// device allocation or kernel launch after arming fails without reaching the GPU.
+std::atomic<int> g_fault_kind{0};
+std::atomic<int> g_fault_countdown{0};
+
+bool injected_fault(int kind) {
+  if (g_fault_kind.load() != kind) return false;
+  if (g_fault_countdown.fetch_sub(1) != 1) return false;
+  g_fault_kind.store(0);
+  return true;
+}
 
 }  // namespace
 
@@ -190,6 +203,14 @@ struct ssd_ctx {
 
 // ------------------------------------------------------------------ helpers
 
+// The kernel launches of launch_k and of the projection, attention and prefill wrappers go through
+// here first: it counts the launch and reports an injected launch failure (the kernel is then not
+// launched).
+static cudaError_t count_launch(ssd_ctx* c) {
+  ++c->launch_counter;
+  return injected_fault(SSD_FAULT_LAUNCH) ? cudaErrorLaunchFailure : cudaSuccess;
+}
+
 // Layer l's K / V cache of the request slot the single-request path addresses.
 static float* kv_k(ssd_ctx* c, int l) { return c->kc + l * c->layer_kv + c->kv_slot; }
 static float* kv_v(ssd_ctx* c, int l) { return c->vc + l * c->layer_kv + c->kv_slot; }
@@ -233,7 +254,7 @@ static cudaError_t launch_k(ssd_ctx* c, Kern kern, dim3 grid, dim3 block, size_t
   at[0].val.programmaticStreamSerializationAllowed = c->use_pdl ? 1 : 0;
   cfg.attrs = at;
   cfg.numAttrs = 1;
-  ++c->launch_counter;
+  if (cudaError_t e = count_launch(c)) return e;
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
@@ -302,7 +323,7 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
   cudaError_t r;
-  ++c->launch_counter;
+  CK(count_launch(c));
   switch (e) {
     case Epi::QKV: r = gemv_launch_qkv(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
     case Epi::GATE_SILU: r = gemv_launch_gate(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
@@ -781,13 +802,13 @@ static ssd_status tc_gemm(ssd_ctx* c, Epi e, int kidx, const TcSite& site, int P
   p.seg_rows = site.seg_rows;
   p.st = c->st;
   const int tiles = p.tiles_m * p.tiles_n;
-  ++c->launch_counter;
+  CK(count_launch(c));
   CK(tc_gemm_launch(e, c->a_maps[kidx], site.maps, p, tiles < c->num_sms ? tiles : c->num_sms, c->cs, c->use_pdl));
   return SSD_OK;
 }
 
 static ssd_status split(ssd_ctx* c, const float* x, int x_stride, int K, const __nv_bfloat16* gain, int P) {
-  ++c->launch_counter;
+  CK(count_launch(c));
   CK(split_rows_launch(x, x_stride, K, gain, c->cfg.rms_eps, c->a_hi, c->a_lo, P, c->cs, c->use_pdl));
   return SSD_OK;
 }
@@ -830,7 +851,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     p.rope_cs = c->rope;
     CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->attn_norm[l], P));
     CKS(tc_gemm(c, Epi::QKV, 0, tl.qkv, P, p));
-    ++c->launch_counter;
+    CK(count_launch(c));
     CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, kv_k(c, l), kv_v(c, l),
                            c->o_pre, c->qp, P, c->cfg.n_heads, c->cfg.max_seq,
                            1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->cs, c->use_pdl));
@@ -887,7 +908,7 @@ static ssd_status act_maps_for(ssd_ctx* c, int K, int NP, const CUtensorMap** ou
 // RMSNorm scales (gain folded in), then the medium-M tensor-core kernel streams the weights once.
 static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   if (M > kMaxMidRows || !c->act_hi) return fail(c, SSD_ERR_INVALID_ARG, "%d rows exceed the medium-M kernel", M);
-  ++c->launch_counter;
+  CK(count_launch(c));
   CK(split_act_launch(p.x, p.x_stride, s.K, p.gain, c->cfg.rms_eps, c->act_hi, c->act_lo, s.K, c->act_rs, M, c->cs,
                       c->use_pdl));
   CUtensorMap amaps[2];
@@ -906,8 +927,8 @@ static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
   p.rs_in = c->act_rs;
-  ++c->launch_counter;
-  CK(mid_launch(e, s.maps, amaps, p, M, s.grid, c->cs, c->use_pdl));
+  CK(count_launch(c));
+  CK(mid_launch(e, s.maps, amaps, p, M, c->num_sms, c->cs, c->use_pdl));
   return SSD_OK;
 }
 
@@ -1208,7 +1229,7 @@ static cudaError_t launch_plain(ssd_ctx* c, Kern kern, Args... args) {
   cfg.gridDim = dim3(1);
   cfg.blockDim = dim3(32);
   cfg.stream = c->cs;
-  ++c->launch_counter;
+  if (cudaError_t e = count_launch(c)) return e;
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
@@ -1375,7 +1396,7 @@ const char* ssd_status_string(ssd_status s) {
 const char* ssd_last_error(const ssd_ctx* c) { return c ? c->err.c_str() : "null context"; }
 
 static ssd_status alloc(ssd_ctx* c, void** p, size_t bytes) {
-  cudaError_t e = cudaMalloc(p, bytes);
+  cudaError_t e = injected_fault(SSD_FAULT_ALLOC) ? cudaErrorMemoryAllocation : cudaMalloc(p, bytes);
   if (e != cudaSuccess) {
     *p = nullptr;
     return fail(c, SSD_ERR_OOM, "cudaMalloc(%zu) failed: %s", bytes, cudaGetErrorString(e));
@@ -2330,6 +2351,23 @@ ssd_status ssd_get_batch_step_log(ssd_ctx* c, int b, int32_t* accepted, int32_t*
   return SSD_OK;
 }
 
+void ssd_set_fault_injection(int kind, int countdown) {
+  g_fault_kind.store(0);
+  g_fault_countdown.store(countdown > 0 ? countdown : 0);
+  if (countdown > 0 && (kind == SSD_FAULT_ALLOC || kind == SSD_FAULT_LAUNCH)) g_fault_kind.store(kind);
+}
+
+ssd_status ssd_probe_bounded_wait(ssd_ctx* c, int64_t limit_ns) {
+  if (!c) return SSD_ERR_INVALID_ARG;
+  if (limit_ns < 0 || limit_ns > 2000000000ll) return fail(c, SSD_ERR_INVALID_ARG, "limit_ns %lld", (long long)limit_ns);
+  CKS(enter(c));
+  ssd_wait_probe_kernel<<<1, 32, 0, c->cs>>>(c->st, static_cast<unsigned long long>(limit_ns));
+  CK(cudaGetLastError());
+  c->prefilled = false;  // later kernels skip their work until the next prefill clears the error
+  c->batch = 0;
+  return leave(c);
+}
+
 ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float* logits) {
   if (!c) return SSD_ERR_INVALID_ARG;
   if (!x || !tok || rows < 1 || rows > kMaxVerifyRows) return fail(c, SSD_ERR_INVALID_ARG, "x / tok / rows");
@@ -2359,7 +2397,7 @@ ssd_status ssd_lm_head(ssd_ctx* c, const float* x, int rows, int32_t* tok, float
   p.counters = c->counters;
   p.st = c->op_st;
   p.eps = c->cfg.rms_eps;
-  ++c->launch_counter;
+  CK(count_launch(c));
   CK(gemv_launch_head(rows, c->head.maps, p, c->head.grid, c->cs, false));
   CKS(leave(c));
   // the host-side DevState must outlive the async copy

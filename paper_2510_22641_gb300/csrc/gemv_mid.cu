@@ -9,7 +9,7 @@ template <Epi EPI>
 cudaError_t mid_launch_e(const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M, int grid,
                          cudaStream_t s, bool pdl) {
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(grid);
+  cfg.gridDim = dim3(grid);  // persistent: min(units, kMidCtasPerSm x #SMs)
   cfg.blockDim = dim3(kMidThreads);
   cfg.dynamicSmemBytes = MidSmem::kTotal;
   cfg.stream = s;
@@ -28,10 +28,12 @@ cudaError_t mid_attr_e() {
 }
 }  // namespace
 
-// M in 1..kMaxMidRows; amaps: the split activations' hi and lo tensor maps ([NP][64] boxes).
+// M in 1..kMaxMidRows; amaps: the split activations' hi and lo tensor maps ([NP][64] boxes); the
+// grid is min(units, kMidCtasPerSm x num_sms).
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
-                       int grid, cudaStream_t s, bool pdl) {
+                       int num_sms, cudaStream_t s, bool pdl) {
   if (M < 1 || M > kMaxMidRows) return cudaErrorInvalidValue;
+  const int grid = p.units < kMidCtasPerSm * num_sms ? p.units : kMidCtasPerSm * num_sms;
   switch (e) {
     case Epi::QKV: return mid_launch_e<Epi::QKV>(wmaps, amaps, p, M, grid, s, pdl);
     case Epi::GATE_SILU: return mid_launch_e<Epi::GATE_SILU>(wmaps, amaps, p, M, grid, s, pdl);

@@ -17,7 +17,7 @@
 //    folded in, exactly as the GEMV's converter warps do) and computes the rows'
 //    RMSNorm scales; warp 0 TMA-loads the parts as 128-byte swizzled [NP][64]
 //    tiles beside each weight unit (NP = M rounded up to 16 is the MMA's N);
-//  * 2 stages of 16 KB weights + 2 x NP x 128 B per CTA and 2 CTAs per SM;
+//  * one CTA per SM with a 4-stage ring of 16 KB weights + 2 x NP x 128 B;
 //  * a row tile's accumulator is NP TMEM columns (two 128-column buffers), read
 //    back 16 columns -- 16 activation rows -- at a time by warps 2..5, which run
 //    the GEMV epilogues on each 16-row chunk.
@@ -30,7 +30,8 @@
 
 namespace ssd {
 
-constexpr int kMidStages = 2;
+constexpr int kMidStages = 4;
+constexpr int kMidCtasPerSm = 1;
 constexpr int kMidThreads = 192;    // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 drain
 constexpr int kMidTmemCols = 256;   // two 128-column accumulators
 constexpr uint32_t kMidBBytes = kMaxMidRows * kTileK * 2;  // one B part (hi or lo) of up to 128 rows: 16 KB
@@ -116,7 +117,7 @@ __global__ void __launch_bounds__(kDrainThreads) ssd_split_act_kernel(const floa
 // map0..2: the site's weight matrices (as for ssd_wstream_kernel); map_hi / map_lo: the split
 // activations [128][K] with [NP][64] boxes.  M rows, NP = M rounded up to 16.
 template <Epi EPI>
-__global__ void __launch_bounds__(kMidThreads, 2)
+__global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
     ssd_wstream_mid_kernel(const __grid_constant__ CUtensorMap map0, const __grid_constant__ CUtensorMap map1,
                            const __grid_constant__ CUtensorMap map2, const __grid_constant__ CUtensorMap map_hi,
                            const __grid_constant__ CUtensorMap map_lo, const GemvParams p, int M) {
@@ -319,43 +320,93 @@ __global__ void __launch_bounds__(kMidThreads, 2)
         }
         drain_sync();
         if (flag[0]) {
-          // sum the contributors' partials in CTA order, one 16-row chunk at a time
+          // Sum the contributors' partials in CTA order, one 16-row chunk at a time.  When this is
+          // the CTA's last segment its ring is idle (every MMA has completed), so each chunk of
+          // every contributor lands there by 16-byte asynchronous copies, the next chunk's copies
+          // in flight while this one is summed; otherwise up to 16 loads per thread are in flight.
           const int nsp = c_last - c_first + 1;
           const int slot0 = 2 * c_first + (unit_begin(c_first, p.units, G) / p.n_kt == rt ? 0 : 1);
           const float4* part = reinterpret_cast<const float4*>(p.partials);
           constexpr int kSlotF4 = kMidSlot / 4;
-          for (int ch = 0; ch < n_ch; ++ch) {
-            const int m0 = ch * kNPad, mc = min(kNPad, M - m0);
-            const int f0 = m0 * (kTileN / 4), nf = mc * (kTileN / 4);
-            for (int f = dt; f < nf; f += kDrainThreads) {
-              float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
-              for (int k0 = 0; k0 < nsp; k0 += 8) {
-                float4 pv[8];
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  const int k = k0 + j;
-                  const int sl = k == 0 ? slot0 : 2 * (c_first + k);
-                  pv[j] = k < nsp ? __ldcg(part + static_cast<size_t>(sl) * kSlotF4 + f0 + f)
-                                  : make_float4(0.f, 0.f, 0.f, 0.f);
+          constexpr int kChF4 = kNPad * kTileN / 4;  // float4s of one full chunk (512)
+          auto slot_of = [&](int k) { return k == 0 ? slot0 : 2 * (c_first + k); };
+          if (i == n_units - 1 && 2 * nsp * kChF4 * 16 <= S::kOut) {
+            float4* land = reinterpret_cast<float4*>(smem + S::kW);  // [2][nsp][kChF4]
+            auto issue = [&](int ch) {
+              const int nf = min(kNPad, M - ch * kNPad) * (kTileN / 4), f0 = ch * kChF4;
+              float4* dstb = land + (ch & 1) * nsp * kChF4;
+              for (int t = dt; t < nsp * nf; t += kDrainThreads) {
+                const int k = t / nf, f = t - k * nf;
+                cp_async16(dstb + k * kChF4 + f, part + static_cast<size_t>(slot_of(k)) * kSlotF4 + f0 + f);
+              }
+              cp_async_commit();
+            };
+            issue(0);
+            for (int ch = 0; ch < n_ch; ++ch) {
+              const int m0 = ch * kNPad, mc = min(kNPad, M - m0), nf = mc * (kTileN / 4);
+              if (ch + 1 < n_ch) {
+                issue(ch + 1);
+                cp_async_wait_group<1>();
+              } else {
+                cp_async_wait_all();
+              }
+              drain_sync();
+              const float4* src = land + (ch & 1) * nsp * kChF4;
+              for (int f = dt; f < nf; f += kDrainThreads) {
+                float4 sum = src[f];
+                for (int k = 1; k < nsp; ++k) {
+                  const float4 v = src[k * kChF4 + f];
+                  sum.x += v.x;
+                  sum.y += v.y;
+                  sum.z += v.z;
+                  sum.w += v.w;
                 }
+                reinterpret_cast<float4*>(outb)[f] = sum;
+              }
+              drain_sync();
+              gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
+              drain_sync();
+            }
+          } else {
+            for (int ch = 0; ch < n_ch; ++ch) {
+              const int m0 = ch * kNPad, mc = min(kNPad, M - m0), nf = mc * (kTileN / 4), f0 = ch * kChF4;
+              float4 acc[4];
+              for (int k0 = 0; k0 < nsp; k0 += 4) {
+                float4 pv[4][4];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                  if (k0 + j >= nsp) continue;
-                  if (k0 + j == 0) {
-                    sum = pv[j];
-                  } else {
-                    sum.x += pv[j].x;
-                    sum.y += pv[j].y;
-                    sum.z += pv[j].z;
-                    sum.w += pv[j].w;
+                for (int kk = 0; kk < 4; ++kk)
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    const int f = dt + e * kDrainThreads;
+                    pv[kk][e] = (k0 + kk < nsp && f < nf)
+                                    ? __ldcg(part + static_cast<size_t>(slot_of(k0 + kk)) * kSlotF4 + f0 + f)
+                                    : make_float4(0.f, 0.f, 0.f, 0.f);
+                  }
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) {
+                  if (k0 + kk >= nsp) break;
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    if (k0 + kk == 0) {
+                      acc[e] = pv[kk][e];
+                    } else {
+                      acc[e].x += pv[kk][e].x;
+                      acc[e].y += pv[kk][e].y;
+                      acc[e].z += pv[kk][e].z;
+                      acc[e].w += pv[kk][e].w;
+                    }
                   }
                 }
               }
-              reinterpret_cast<float4*>(outb)[f] = sum;
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int f = dt + e * kDrainThreads;
+                if (f < nf) reinterpret_cast<float4*>(outb)[f] = acc[e];
+              }
+              drain_sync();
+              gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
+              drain_sync();
             }
-            drain_sync();
-            gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
-            drain_sync();
           }
           if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
           if (dt == 0) p.counters[rt] = 0u;

@@ -281,6 +281,10 @@ class SSDModel:
         m = min(n.value, cap)
         return acc[:m].tolist(), dr[:m].tolist()
 
+    def probe_bounded_wait(self, limit_ns: int):
+        """ssd_probe_bounded_wait: one device wait runs out after limit_ns; the next sync reports it."""
+        self._call("ssd_probe_bounded_wait", limit_ns)
+
     def launch_counts(self) -> tuple[int, int]:
         a, b = ctypes.c_int64(), ctypes.c_int64()
         self._call("ssd_last_launch_count", ctypes.byref(a), ctypes.byref(b))
