@@ -8,11 +8,22 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 
+def pytest_addoption(parser):
+    parser.addoption("--runslow", action="store_true", default=False,
+                     help="also run tests marked slow (minutes of CPU work at full model widths)")
+
+
 def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (GB300, sm_103a) and the built library")
+    config.addinivalue_line("markers", "slow: minutes of CPU work; runs only with --runslow")
 
 
 def pytest_collection_modifyitems(config, items):
+    if not config.getoption("--runslow"):
+        skip_slow = pytest.mark.skip(reason="slow: needs --runslow")
+        for it in items:
+            if "slow" in it.keywords:
+                it.add_marker(skip_slow)
     # A gpu-marked test never silently passes on a machine without a GPU.
     try:
         import torch
