@@ -48,6 +48,7 @@ cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, cons
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
                        int num_sms, cudaStream_t s, bool pdl);
 cudaError_t mid_attrs();
+int mid_max_ctas(int num_sms);
 cudaError_t split_act_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                              __nv_bfloat16* hi, __nv_bfloat16* lo, int ld, float* rs, int rows, cudaStream_t s,
                              bool pdl);
@@ -927,7 +928,8 @@ static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
   p.rs_in = c->act_rs;
-  CK(count_launch(c));
+  CK(count_launch(c));  // the stream
+  CK(count_launch(c));  // the reduction + epilogue
   CK(mid_launch(e, s.maps, amaps, p, M, c->num_sms, c->cs, c->use_pdl));
   return SSD_OK;
 }
@@ -1724,6 +1726,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
       max_rt = s->n_rt > max_rt ? s->n_rt : max_rt;
   c->n_counters = max_rt;
   CKS(alloc(c, reinterpret_cast<void**>(&c->counters), sizeof(unsigned) * max_rt));
+
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_part),
             sizeof(float) * max_batch * k.n_heads * kAttnSplit * kAttnMaxRows * (k.head_dim + 2)));
   CKS(alloc(c, reinterpret_cast<void**>(&c->attn_tickets), sizeof(unsigned) * max_batch * k.n_heads));
@@ -1740,8 +1743,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_hi), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_lo), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_rs), sizeof(float) * kMaxMidRows));
+      // partials: one slot per (streaming CTA, row tile) pair, c + rt
       CKS(alloc(c, reinterpret_cast<void**>(&c->mid_partials),
-                sizeof(float) * 2 * kGemvCtasPerSm * c->num_sms * kMaxMidRows * kTileN));
+                sizeof(float) * (mid_max_ctas(c->num_sms) + c->n_counters) * kMaxMidRows * kTileN));
     }
   }
   CKS(alloc(c, reinterpret_cast<void**>(&c->dyn_table), sizeof(int) * (k.max_seq + 1)));

@@ -111,6 +111,7 @@ struct GemvParams {
   // Medium-M kernel only: the rows' RMSNorm scales 1/rms(x_m), computed by the split kernel
   // (the gain is folded into its bf16 hi/lo parts).
   const float* rs_in;
+  int grid_ctas;  // medium-M reduction: the CTAs of the streaming launch
   int abs_pos;   // row m sits at position pos_off + m, st->kv_len ignored (the encoder's rows)
   int act;       // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up (gated GELU)
 };
@@ -229,32 +230,52 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     const int local0 = r0 - seg * p.seg_rows;
     const int Dh = p.head_dim, half = Dh >> 1;
     if (mat < 2) {
-      for (int idx = tid; idx < mc * (kTileN / 2); idx += kDrainThreads) {
-        const int m = idx / (kTileN / 2), pr = idx - m * (kTileN / 2), mg = m0 + m;
-        const int hh = pr / half, j = pr - hh * half;
-        const int ra = hh * Dh + j, rb = ra + half;
-        const int pos = rpos ? rpos[mg] : base_pos + mg;
-        if (pos < 0 || pos >= p.max_seq) {
-          set_error(p.st, DERR_POS);
-          continue;
+      // four (row, pair) items per thread at a time: their rotation coefficients are fetched
+      // first (from shared memory, or from the table in global memory), then rotated and stored
+      constexpr int kPairs = kTileN / 2;
+      const int n_items = mc * kPairs;
+      for (int i0 = tid; i0 < n_items; i0 += 4 * kDrainThreads) {
+        float2 cs[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int idx = i0 + u * kDrainThreads;
+          cs[u] = make_float2(1.f, 0.f);
+          if (idx < n_items && p.rope_cs) {
+            const int m = idx / kPairs, pr = idx - m * kPairs, mg = m0 + m;
+            const int j = pr - (pr / half) * half;
+            const int pos = rpos ? rpos[mg] : base_pos + mg;
+            if (pre) cs[u] = reinterpret_cast<const float2*>(pre)[m * half + j];
+            else if (pos >= 0 && pos < p.max_seq) cs[u] = __ldg(p.rope_cs + static_cast<size_t>(pos) * half + j);
+          }
         }
-        const float a = out[m * kTileN + ra] * rs[m];
-        const float b = out[m * kTileN + rb] * rs[m];
-        float va = a, vb = b;  // no rotation without a table (relative-position-bias models)
-        if (p.rope_cs) {
-          const float2 cs = pre ? reinterpret_cast<const float2*>(pre)[m * half + j]
-                                : p.rope_cs[static_cast<size_t>(pos) * half + j];
-          va = a * cs.x - b * cs.y;
-          vb = a * cs.y + b * cs.x;
-        }
-        if (mat == 0) {
-          p.q_out[mg * p.q_stride + local0 + ra] = va;
-          p.q_out[mg * p.q_stride + local0 + rb] = vb;
-        } else {
-          const int h = local0 / Dh + hh;
-          float* kr = p.k_cache + (rreq ? rreq[mg] * p.req_kv : 0ll) + (static_cast<size_t>(h) * p.max_seq + pos) * Dh;
-          kr[j] = va;
-          kr[j + half] = vb;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int idx = i0 + u * kDrainThreads;
+          if (idx >= n_items) break;
+          const int m = idx / kPairs, pr = idx - m * kPairs, mg = m0 + m;
+          const int hh = pr / half, j = pr - hh * half;
+          const int ra = hh * Dh + j, rb = ra + half;
+          const int pos = rpos ? rpos[mg] : base_pos + mg;
+          if (pos < 0 || pos >= p.max_seq) {
+            set_error(p.st, DERR_POS);
+            continue;
+          }
+          const float a = out[m * kTileN + ra] * rs[m];
+          const float b = out[m * kTileN + rb] * rs[m];
+          float va = a, vb = b;  // no rotation without a table (relative-position-bias models)
+          if (p.rope_cs) {
+            va = a * cs[u].x - b * cs[u].y;
+            vb = a * cs[u].y + b * cs[u].x;
+          }
+          if (mat == 0) {
+            p.q_out[mg * p.q_stride + local0 + ra] = va;
+            p.q_out[mg * p.q_stride + local0 + rb] = vb;
+          } else {
+            const int h = local0 / Dh + hh;
+            float* kr = p.k_cache + (rreq ? rreq[mg] * p.req_kv : 0ll) + (static_cast<size_t>(h) * p.max_seq + pos) * Dh;
+            kr[j] = va;
+            kr[j + half] = vb;
+          }
         }
       }
     } else {
@@ -337,14 +358,15 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
   }
 }
 
-// LM head, after a row tile's keys of all M launch rows are in: the tile's maxima are released
-// by one acq_rel ticket after the CTA barrier; the tile that completes the count reads and resets
+// LM head, after a row tile's keys of all M launch rows are in (or one chunk's rows, `tiles`
+// counting every tile x chunk): the maxima are released by one acq_rel ticket after the CTA
+// barrier; the tile that completes the count reads and resets
 // the M keys, one thread per row, and writes the tokens (-1 once a bounded wait anywhere has
 // given up: the keys may miss tiles).
-__device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, int M, const int* rreq, int tid) {
+__device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, int M, const int* rreq, int tid, int tiles) {
   __shared__ int am_last;
   drain_sync();
-  if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(p.n_rt - 1);
+  if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(tiles - 1);
   drain_sync();
   if (am_last) {
     const bool stopped = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
@@ -645,7 +667,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
       if (whole) {
         gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
-        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
+        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt, p.n_rt);
       } else {
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
@@ -722,7 +744,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
           }
           drain_sync();
           gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
-          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
+          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt, p.n_rt);
           if (dt == 0) p.counters[rt] = 0u;
         }
       }

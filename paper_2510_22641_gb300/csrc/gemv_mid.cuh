@@ -17,10 +17,18 @@
 //    folded in, exactly as the GEMV's converter warps do) and computes the rows'
 //    RMSNorm scales; warp 0 TMA-loads the parts as 128-byte swizzled [NP][64]
 //    tiles beside each weight unit (NP = M rounded up to 16 is the MMA's N);
-//  * one CTA per SM with a 4-stage ring of 16 KB weights + 2 x NP x 128 B;
+//  * one CTA per SM; the weight units stream through an 8-stage ring of 16 KB fed by warp 0
+//    (issued ahead of the upstream wait), the B tiles through a 3-stage ring of
+//    2 x NP x 128 B fed by warp 6, so the weight stream keeps 8 units in flight
+//    whatever the B ring holds;
 //  * a row tile's accumulator is NP TMEM columns (two 128-column buffers), read
-//    back 16 columns -- 16 activation rows -- at a time by warps 2..5, which run
-//    the GEMV epilogues on each 16-row chunk.
+//    back 16 columns -- 16 activation rows -- at a time by warps 2..5 and stored
+//    as the CTA's partial of that tile;
+//  * the reduction and the fused epilogue run in a second kernel,
+//    ssd_mid_reduce_kernel, one CTA per (row tile, 16-row chunk): a tile's 112
+//    rows are finished by 7 CTAs at once instead of one CTA's 128 threads after
+//    the stream (measured: about 3 us per 16-row chunk, which made the serial
+//    tail as long as the stream itself).
 // The per-element arithmetic is the GEMV's: a = hi + lo, 4 K slices x (hi, lo)
 // MMAs per unit accumulating in fp32, the RMSNorm scale applied after the
 // products, and the split-tile sums in CTA order.
@@ -30,23 +38,20 @@
 
 namespace ssd {
 
-constexpr int kMidStages = 4;
+constexpr int kMidWStages = 8;      // weight ring
+constexpr int kMidBStages = 3;      // activation (B) ring
 constexpr int kMidCtasPerSm = 1;
-constexpr int kMidThreads = 192;    // warp 0 TMA, warp 1 MMA + TMEM, warps 2..5 drain
+constexpr int kMidThreads = 224;    // warp 0 weight TMA, warp 1 MMA + TMEM, warps 2..5 drain, warp 6 B TMA
 constexpr int kMidTmemCols = 256;   // two 128-column accumulators
 constexpr uint32_t kMidBBytes = kMaxMidRows * kTileK * 2;  // one B part (hi or lo) of up to 128 rows: 16 KB
 constexpr int kMidSlot = kMaxMidRows * kTileN;             // floats of one partial row tile, [m][128]
 
 struct MidSmem {
-  static constexpr int kW = 0;                                  // [stages][16 KB] weight units
-  static constexpr int kBh = kW + kMidStages * kWTileBytes;     // [stages][NP][64] bf16 hi
-  static constexpr int kBl = kBh + kMidStages * kMidBBytes;     // [stages][NP][64] bf16 lo
-  static constexpr int kOut = kBl + kMidStages * kMidBBytes;    // one drained 16-row chunk [16][128] fp32
-  static constexpr int kRs = kOut + kNPad * kTileN * 4;         // [128] RMSNorm scales
-  static constexpr int kRowPos = kRs + kMaxMidRows * 4;         // [2][128] positions, requests
-  static constexpr int kFlag = kRowPos + 2 * kMaxMidRows * 4;
-  static constexpr int kBar = (kFlag + 16 + 7) & ~7;            // full, empty [stages]; afull, aempty [2]
-  static constexpr int kTmemSlot = kBar + (2 * kMidStages + 4) * 8;
+  static constexpr int kW = 0;                                  // [wstages][16 KB] weight units
+  static constexpr int kBh = kW + kMidWStages * kWTileBytes;    // [bstages][NP][64] bf16 hi
+  static constexpr int kBl = kBh + kMidBStages * kMidBBytes;    // [bstages][NP][64] bf16 lo
+  static constexpr int kBar = kBl + kMidBStages * kMidBBytes;  // wfull, wempty [wstages]; bfull, bempty [bstages]; afull, aempty [2]
+  static constexpr int kTmemSlot = kBar + (2 * kMidWStages + 2 * kMidBStages + 4) * 8;
   static constexpr int kTotal = kTmemSlot + 16 + 1024;          // + slack for the 1024-byte alignment
 };
 
@@ -125,30 +130,31 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + S::kBar);
-  uint64_t* empty = full + kMidStages;
-  uint64_t* afull = empty + kMidStages;
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  uint64_t* wempty = wfull + kMidWStages;
+  uint64_t* bfull = wempty + kMidWStages;
+  uint64_t* bempty = bfull + kMidBStages;
+  uint64_t* afull = bempty + kMidBStages;
   uint64_t* aempty = afull + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
-  float* outb = reinterpret_cast<float*>(smem + S::kOut);
-  float* rs = reinterpret_cast<float*>(smem + S::kRs);
-  int* flag = reinterpret_cast<int*>(smem + S::kFlag);
 
   const int G = gridDim.x, c = blockIdx.x;
   const int u0 = unit_begin(c, p.units, G), u1 = unit_begin(c + 1, p.units, G);
   const int n_units = u1 - u0;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int NP = (M + 15) & ~15;
-  const uint32_t bbytes = static_cast<uint32_t>(NP) * kTileK * 2;
-  const uint32_t tx = kWTileBytes + 2 * bbytes;
 
   if (!p.late_trigger) pdl_trigger();
   if (*reinterpret_cast<volatile int*>(&p.st->error) & DERR_TIMEOUT) return;
 
   if (tid == 0) {
-    for (int s = 0; s < kMidStages; ++s) {
-      mbar_init(&full[s], 1);
-      mbar_init(&empty[s], 1);
+    for (int s = 0; s < kMidWStages; ++s) {
+      mbar_init(&wfull[s], 1);
+      mbar_init(&wempty[s], 1);
+    }
+    for (int s = 0; s < kMidBStages; ++s) {
+      mbar_init(&bfull[s], 1);
+      mbar_init(&bempty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&afull[b], 1);
@@ -168,45 +174,32 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
   const uint32_t tmem = *tmem_slot;
 
   if (warp == 0) {
-    // ---------------------------------------------------------------- TMA producer
+    // ---------------------------------------------------------------- weight TMA producer
     if (lane == 0) {
       auto issue_weights = [&](int s, int u) {
         const int rt = u / p.n_kt, kt = u - rt * p.n_kt;
         uint8_t* wdst = smem + S::kW + s * kWTileBytes;
         const int x = kt * kTileK;
+        mbar_arrive_expect_tx(&wfull[s], kWTileBytes);
         if constexpr (EPI == Epi::GATE_SILU) {
-          tma_load_2d(wdst, &map0, &full[s], x, rt * kHalfN);
-          tma_load_2d(wdst + kWTileBytes / 2, &map1, &full[s], x, rt * kHalfN);
+          tma_load_2d(wdst, &map0, &wfull[s], x, rt * kHalfN);
+          tma_load_2d(wdst + kWTileBytes / 2, &map1, &wfull[s], x, rt * kHalfN);
         } else if constexpr (EPI == Epi::QKV) {
           const int r0 = rt * kTileN, mat = r0 / p.seg_rows;
-          tma_load_2d(wdst, mat == 0 ? &map0 : (mat == 1 ? &map1 : &map2), &full[s], x, r0 - mat * p.seg_rows);
+          tma_load_2d(wdst, mat == 0 ? &map0 : (mat == 1 ? &map1 : &map2), &wfull[s], x, r0 - mat * p.seg_rows);
         } else {
-          tma_load_2d(wdst, &map0, &full[s], x, rt * kTileN);
+          tma_load_2d(wdst, &map0, &wfull[s], x, rt * kTileN);
         }
       };
-      auto issue_acts = [&](int s, int u) {
-        const int x = (u % p.n_kt) * kTileK;
-        tma_load_2d(smem + S::kBh + s * kMidBBytes, &map_hi, &full[s], x, 0);
-        tma_load_2d(smem + S::kBl + s * kMidBBytes, &map_lo, &full[s], x, 0);
-      };
       prefetch_tensormap(&map0);
-      const int npre = n_units < kMidStages ? n_units : kMidStages;
-      for (int i = 0; i < npre; ++i) {
-        mbar_arrive_expect_tx(&full[i], tx);
-        issue_weights(i, u0 + i);  // weights do not depend on the previous kernel
-      }
-      pdl_wait();
-      if (p.late_trigger) pdl_trigger();
-      for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
-      for (int i = npre; i < n_units; ++i) {
-        const int s = i % kMidStages;
-        if (!mbar_wait(&empty[s], static_cast<uint32_t>((i / kMidStages) - 1) & 1u)) {
+      // weights do not depend on the previous kernel: the first stages go out before its end
+      for (int i = 0; i < n_units; ++i) {
+        const int s = i % kMidWStages;
+        if (i >= kMidWStages && !mbar_wait(&wempty[s], static_cast<uint32_t>((i / kMidWStages) - 1) & 1u)) {
           set_error(p.st, DERR_TIMEOUT);
           break;
         }
-        mbar_arrive_expect_tx(&full[s], tx);
         issue_weights(s, u0 + i);
-        issue_acts(s, u0 + i);
       }
     }
   } else if (warp == 1) {
@@ -217,7 +210,7 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
       bool seg_open = false;
       uint32_t d = tmem;
       for (int i = 0; i < n_units; ++i) {
-        const int u = u0 + i, kt = u % p.n_kt, s = i % kMidStages;
+        const int u = u0 + i, kt = u % p.n_kt, s = i % kMidWStages, sb = i % kMidBStages;
         if (!seg_open) {  // a new row-tile segment: take a free accumulator
           const int b = sg & 1;
           if (!mbar_wait(&aempty[b], static_cast<uint32_t>(((sg >> 1) & 1) ^ 1))) {
@@ -227,14 +220,15 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
           tmem_fence_after();
           d = tmem + static_cast<uint32_t>(b * kMaxMidRows);
         }
-        if (!mbar_wait(&full[s], static_cast<uint32_t>(i / kMidStages) & 1u)) {
+        if (!mbar_wait(&wfull[s], static_cast<uint32_t>(i / kMidWStages) & 1u) ||
+            !mbar_wait(&bfull[sb], static_cast<uint32_t>(i / kMidBStages) & 1u)) {
           set_error(p.st, DERR_TIMEOUT);
           break;
         }
         tmem_fence_after();
         const uint64_t adesc = umma_desc_sw128(smem_u32(smem + S::kW + s * kWTileBytes));
-        const uint64_t hdesc = umma_desc_sw128(smem_u32(smem + S::kBh + s * kMidBBytes));
-        const uint64_t ldesc = umma_desc_sw128(smem_u32(smem + S::kBl + s * kMidBBytes));
+        const uint64_t hdesc = umma_desc_sw128(smem_u32(smem + S::kBh + sb * kMidBBytes));
+        const uint64_t ldesc = umma_desc_sw128(smem_u32(smem + S::kBl + sb * kMidBBytes));
 #pragma unroll
         for (int kk = 0; kk < kTileK / 16; ++kk) {
           // +32 bytes (2 descriptor units) per 16-element K slice inside the swizzled row
@@ -242,7 +236,8 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
           umma_f16(d, adesc + 2 * kk, ldesc + 2 * kk, idesc, 1u);
           seg_open = true;
         }
-        umma_commit(&empty[s]);  // stage s may be refilled once these MMAs have read it
+        umma_commit(&wempty[s]);  // the stages may be refilled once these MMAs have read them
+        umma_commit(&bempty[sb]);
         if (kt == p.n_kt - 1 || i == n_units - 1) {
           umma_commit(&afull[sg & 1]);  // the row tile's accumulator is complete
           ++sg;
@@ -250,28 +245,34 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         }
       }
     }
-  } else {
-    // ---------------------------------------------------------------- drain + epilogues (warps 2..5)
-    const int dt = tid - 64;  // 0..127
-    const int q = warp & 3;   // TMEM lane quadrant: tile rows 32q .. 32q+31
-    pdl_wait();
-    for (int m = dt; m < M; m += kDrainThreads) rs[m] = p.rs_in ? __ldcg(p.rs_in + m) : 1.0f;
-    const int base_pos = (p.abs_pos || p.batch_rows ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
-    int* rpos = p.batch_rows ? reinterpret_cast<int*>(smem + S::kRowPos) : nullptr;
-    int* rreq = p.batch_rows ? rpos + kMaxMidRows : nullptr;
-    if (rpos)
-      for (int m = dt; m < M; m += kDrainThreads) {
-        const int b = m / p.batch_rows;
-        rreq[m] = b;
-        rpos[m] = __ldcg(&p.req_st[b].kv_len) + batch_offset(p, m, b);
+  } else if (warp == 6) {
+    // ---------------------------------------------------------------- B TMA producer (split activations)
+    if (lane == 0) {
+      const uint32_t bbytes = static_cast<uint32_t>(NP) * kTileK * 2;
+      pdl_wait();  // the split kernel's rows
+      if (p.late_trigger) pdl_trigger();
+      for (int i = 0; i < n_units; ++i) {
+        const int sb = i % kMidBStages;
+        if (i >= kMidBStages && !mbar_wait(&bempty[sb], static_cast<uint32_t>((i / kMidBStages) - 1) & 1u)) {
+          set_error(p.st, DERR_TIMEOUT);
+          break;
+        }
+        const int x = ((u0 + i) % p.n_kt) * kTileK;
+        mbar_arrive_expect_tx(&bfull[sb], 2 * bbytes);
+        tma_load_2d(smem + S::kBh + sb * kMidBBytes, &map_hi, &bfull[sb], x, 0);
+        tma_load_2d(smem + S::kBl + sb * kMidBBytes, &map_lo, &bfull[sb], x, 0);
       }
-    drain_sync();
-    const int rt_first = u0 / p.n_kt;
+    }
+  } else {
+    // ---------------------------------------------------------------- drain (warps 2..5)
+    // Every finished accumulator -- row tile rt's share of this CTA's unit range -- goes to
+    // partial slot c + rt, 16 columns (activation rows) at a time, [m][128] fp32.  Along the
+    // partition the pairs (CTA, tile) never decrease in either index, so c + rt is unique;
+    // ssd_mid_reduce_kernel sums each tile's slots in CTA order and runs the epilogue.
+    const int q = warp & 3;  // TMEM lane quadrant: tile rows 32q .. 32q+31
     const int n_ch = (M + kNPad - 1) / kNPad;
-    int seg_kt0 = u0 - rt_first * p.n_kt;
     int sg = 0;
-    bool ok = true;
-    for (int i = 0; ok && i < n_units; ++i) {
+    for (int i = 0; i < n_units; ++i) {
       const int u = u0 + i, rt = u / p.n_kt, kt = u - rt * p.n_kt;
       if (!(kt == p.n_kt - 1 || i == n_units - 1)) continue;
       const int b = sg & 1;
@@ -281,139 +282,17 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
       }
       tmem_fence_after();
       const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kMaxMidRows);
-      const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
-      if (whole) {
-        for (int ch = 0; ch < n_ch; ++ch) {
-          float v[kNPad];
-          tmem_ld16(tbase + ch * kNPad, v);
+      float* dstp = p.partials + static_cast<size_t>(c + rt) * kMidSlot;
+      for (int ch = 0; ch < n_ch; ++ch) {
+        float v[kNPad];
+        tmem_ld16(tbase + ch * kNPad, v);
 #pragma unroll
-          for (int m = 0; m < kNPad; ++m) outb[m * kTileN + q * 32 + lane] = v[m];
-          drain_sync();
-          const int m0 = ch * kNPad, mc = min(kNPad, M - m0);
-          gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
-          drain_sync();
-        }
-        tmem_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&aempty[b]);  // the MMA warp may reuse accumulator b
-        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
-      } else {
-        const int slot = 2 * c + (rt == rt_first ? 0 : 1);
-        float* dstp = p.partials + static_cast<size_t>(slot) * kMidSlot;
-        for (int ch = 0; ch < n_ch; ++ch) {
-          float v[kNPad];
-          tmem_ld16(tbase + ch * kNPad, v);
-#pragma unroll
-          for (int m = 0; m < kNPad; ++m)
-            if (ch * kNPad + m < M) __stcg(dstp + (ch * kNPad + m) * kTileN + q * 32 + lane, v[m]);
-        }
-        tmem_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&aempty[b]);
-        // the tile's ticket releases this CTA's partial (CTA barrier, then one acq_rel atomic)
-        drain_sync();
-        const int c_first = unit_owner(rt * p.n_kt, p.units, G);
-        const int c_last = unit_owner(rt * p.n_kt + p.n_kt - 1, p.units, G);
-        if (dt == 0) {
-          const unsigned prev = atom_add_acq_rel_gpu(&p.counters[rt], 1u);
-          flag[0] = (prev == static_cast<unsigned>(c_last - c_first)) ? 1 : 0;
-        }
-        drain_sync();
-        if (flag[0]) {
-          // Sum the contributors' partials in CTA order, one 16-row chunk at a time.  When this is
-          // the CTA's last segment its ring is idle (every MMA has completed), so each chunk of
-          // every contributor lands there by 16-byte asynchronous copies, the next chunk's copies
-          // in flight while this one is summed; otherwise up to 16 loads per thread are in flight.
-          const int nsp = c_last - c_first + 1;
-          const int slot0 = 2 * c_first + (unit_begin(c_first, p.units, G) / p.n_kt == rt ? 0 : 1);
-          const float4* part = reinterpret_cast<const float4*>(p.partials);
-          constexpr int kSlotF4 = kMidSlot / 4;
-          constexpr int kChF4 = kNPad * kTileN / 4;  // float4s of one full chunk (512)
-          auto slot_of = [&](int k) { return k == 0 ? slot0 : 2 * (c_first + k); };
-          if (i == n_units - 1 && 2 * nsp * kChF4 * 16 <= S::kOut) {
-            float4* land = reinterpret_cast<float4*>(smem + S::kW);  // [2][nsp][kChF4]
-            auto issue = [&](int ch) {
-              const int nf = min(kNPad, M - ch * kNPad) * (kTileN / 4), f0 = ch * kChF4;
-              float4* dstb = land + (ch & 1) * nsp * kChF4;
-              for (int t = dt; t < nsp * nf; t += kDrainThreads) {
-                const int k = t / nf, f = t - k * nf;
-                cp_async16(dstb + k * kChF4 + f, part + static_cast<size_t>(slot_of(k)) * kSlotF4 + f0 + f);
-              }
-              cp_async_commit();
-            };
-            issue(0);
-            for (int ch = 0; ch < n_ch; ++ch) {
-              const int m0 = ch * kNPad, mc = min(kNPad, M - m0), nf = mc * (kTileN / 4);
-              if (ch + 1 < n_ch) {
-                issue(ch + 1);
-                cp_async_wait_group<1>();
-              } else {
-                cp_async_wait_all();
-              }
-              drain_sync();
-              const float4* src = land + (ch & 1) * nsp * kChF4;
-              for (int f = dt; f < nf; f += kDrainThreads) {
-                float4 sum = src[f];
-                for (int k = 1; k < nsp; ++k) {
-                  const float4 v = src[k * kChF4 + f];
-                  sum.x += v.x;
-                  sum.y += v.y;
-                  sum.z += v.z;
-                  sum.w += v.w;
-                }
-                reinterpret_cast<float4*>(outb)[f] = sum;
-              }
-              drain_sync();
-              gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
-              drain_sync();
-            }
-          } else {
-            for (int ch = 0; ch < n_ch; ++ch) {
-              const int m0 = ch * kNPad, mc = min(kNPad, M - m0), nf = mc * (kTileN / 4), f0 = ch * kChF4;
-              float4 acc[4];
-              for (int k0 = 0; k0 < nsp; k0 += 4) {
-                float4 pv[4][4];
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-#pragma unroll
-                  for (int e = 0; e < 4; ++e) {
-                    const int f = dt + e * kDrainThreads;
-                    pv[kk][e] = (k0 + kk < nsp && f < nf)
-                                    ? __ldcg(part + static_cast<size_t>(slot_of(k0 + kk)) * kSlotF4 + f0 + f)
-                                    : make_float4(0.f, 0.f, 0.f, 0.f);
-                  }
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) {
-                  if (k0 + kk >= nsp) break;
-#pragma unroll
-                  for (int e = 0; e < 4; ++e) {
-                    if (k0 + kk == 0) {
-                      acc[e] = pv[kk][e];
-                    } else {
-                      acc[e].x += pv[kk][e].x;
-                      acc[e].y += pv[kk][e].y;
-                      acc[e].z += pv[kk][e].z;
-                      acc[e].w += pv[kk][e].w;
-                    }
-                  }
-                }
-              }
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const int f = dt + e * kDrainThreads;
-                if (f < nf) reinterpret_cast<float4*>(outb)[f] = acc[e];
-              }
-              drain_sync();
-              gemv_epilogue<kNPad, EPI>(p, rt, outb, rs + m0, nullptr, base_pos, rpos, rreq, dt, m0, mc);
-              drain_sync();
-            }
-          }
-          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt);
-          if (dt == 0) p.counters[rt] = 0u;
-        }
+        for (int m = 0; m < kNPad; ++m)
+          if (ch * kNPad + m < M) __stcg(dstp + (ch * kNPad + m) * kTileN + q * 32 + lane, v[m]);
       }
-      drain_sync();
-      seg_kt0 = 0;
+      tmem_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&aempty[b]);  // the MMA warp may reuse accumulator b
       ++sg;
     }
   }
@@ -423,6 +302,90 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
     tmem_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kMidTmemCols) : "memory");
   }
+}
+
+// ------------------------------------------------------------------ reduction + epilogue
+// One CTA per (16-row chunk ch = blockIdx.x, row tile rt = blockIdx.y) of a medium-M projection
+// streamed by `G = p.grid_ctas` CTAs: sums the tile's partials (slots c + rt for the CTAs c that
+// held its units) in CTA order, then applies the RMSNorm scale and the fused epilogue to rows
+// 16 ch .. 16 ch + 15 -- the GEMV's epilogue code, with its inputs (rotation table rows, residual
+// base rows) loaded up front.  The LM head's argmax keys are finished by the last of all
+// n_rt x chunks CTAs.
+template <Epi EPI>
+__global__ void __launch_bounds__(kDrainThreads) ssd_mid_reduce_kernel(const GemvParams p, int M) {
+  __shared__ __align__(16) float outb[kNPad * kTileN];
+  __shared__ __align__(16) float pre[kNPad * kTileN];  // QKV: [16][head_dim / 2] float2; RESID: [16][128]
+  __shared__ float rs[kNPad];
+  __shared__ int rmap[2 * kMaxMidRows];                // positions, requests of all M rows
+  const int ch = blockIdx.x, rt = blockIdx.y, tid = threadIdx.x;
+  const int m0 = ch * kNPad, mc = min(kNPad, M - m0);
+  const int G = p.grid_ctas;
+  pdl_trigger();
+  pdl_wait();
+  if (__ldcg(&p.st->error) & DERR_TIMEOUT) return;  // the stream gave up: partials are incomplete
+  const int base_pos = (p.abs_pos || p.batch_rows ? 0 : __ldcg(&p.st->kv_len)) + p.pos_off;
+  int* rpos = p.batch_rows ? rmap : nullptr;
+  int* rreq = p.batch_rows ? rmap + kMaxMidRows : nullptr;
+  if (rpos)
+    for (int m = tid; m < M; m += kDrainThreads) {
+      const int b = m / p.batch_rows;
+      rreq[m] = b;
+      rpos[m] = __ldcg(&p.req_st[b].kv_len) + batch_offset(p, m, b);
+    }
+  if (tid < mc) rs[tid] = p.rs_in ? __ldcg(p.rs_in + m0 + tid) : 1.0f;
+  __syncthreads();
+  // epilogue inputs, all loads independent
+  bool use_pre = false;
+  if constexpr (EPI == Epi::QKV) {
+    const int half = p.head_dim >> 1;
+    use_pre = p.rope_cs != nullptr && (rt * kTileN) / p.seg_rows + p.seg_base < 2;
+    if (use_pre)
+      for (int t = tid; t < mc * half; t += kDrainThreads) {
+        const int m = t / half, j = t - m * half;
+        const int pos = rpos ? rpos[m0 + m] : base_pos + m0 + m;
+        reinterpret_cast<float2*>(pre)[t] =
+            (pos >= 0 && pos < p.max_seq) ? __ldg(p.rope_cs + static_cast<size_t>(pos) * half + j) : make_float2(1.f, 0.f);
+      }
+  } else if constexpr (EPI == Epi::RESID) {
+    use_pre = true;
+    for (int t = tid; t < mc * kTileN; t += kDrainThreads) {
+      const int m = t / kTileN, n = rt * kTileN + (t - m * kTileN);
+      pre[t] = n < p.N ? __ldcg(p.base + static_cast<size_t>(m0 + m) * p.base_stride + n) : 0.f;
+    }
+  }
+  // the tile's partials in CTA order, four contributors' loads in flight per row slice
+  const int c_first = unit_owner(rt * p.n_kt, p.units, G);
+  const int c_last = unit_owner(rt * p.n_kt + p.n_kt - 1, p.units, G);
+  const int nsp = c_last - c_first + 1;
+  const float4* part = reinterpret_cast<const float4*>(p.partials);
+  constexpr int kSlotF4 = kMidSlot / 4;
+  const int nf = mc * (kTileN / 4), f0 = m0 * (kTileN / 4);
+  for (int f = tid; f < nf; f += kDrainThreads) {
+    float4 sum = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int k0 = 0; k0 < nsp; k0 += 4) {
+      float4 pv[4];
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk)
+        pv[kk] = k0 + kk < nsp ? __ldcg(part + static_cast<size_t>(c_first + k0 + kk + rt) * kSlotF4 + f0 + f)
+                               : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int kk = 0; kk < 4; ++kk) {
+        if (k0 + kk >= nsp) break;
+        if (k0 + kk == 0) {
+          sum = pv[kk];
+        } else {
+          sum.x += pv[kk].x;
+          sum.y += pv[kk].y;
+          sum.z += pv[kk].z;
+          sum.w += pv[kk].w;
+        }
+      }
+    }
+    reinterpret_cast<float4*>(outb)[f] = sum;
+  }
+  __syncthreads();
+  gemv_epilogue<kNPad, EPI>(p, rt, outb, rs, use_pre ? pre : nullptr, base_pos, rpos, rreq, tid, m0, mc);
+  if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, tid, p.n_rt * gridDim.x);
 }
 
 }  // namespace ssd
