@@ -12,7 +12,8 @@ Printed as one JSON line (rank 0):
   roofline       the dominant kernel (weight-streaming GEMV, gate/up, 1 row)
                  timed alone with CUDA events, against the measured HBM copy peak
   per_s          decode tokens/s of SSD and of greedy decoding (same kernels), and of SSD with the
-                 dynamic draft length d(t) (d0 = 5, N = the context's max_seq, capped at gamma_max)
+                 dynamic draft length d(t) (d0 = 5, capped at gamma_max = 15; t over the context with
+                 N = the context's max_seq, and t over the generated tokens with N = max_new)
                  and their ratio for s in {0.05, 0.2, 1.0}
   cpu_baseline   the fp64 oracle on the host cores over a bounded sample
 
@@ -847,8 +848,10 @@ def main() -> None:
         model.prefill(v, p)
         if ev is not None:
             ev.record(stream)
-        if gamma < 0:   # dynamic draft length d(t), d0 = 5, capped at gamma_max
+        if gamma == -1:   # dynamic draft length d(t), d0 = 5, capped at gamma_max; t over the context
             model.decode_dynamic(w.max_new, 5, dyn_n, lib.SSD_MAX_GAMMA, out, n_out)
+        elif gamma == -2:  # the same with t over the generated tokens and N = max_new
+            model.decode_dynamic(w.max_new, 5, w.max_new, lib.SSD_MAX_GAMMA, out, n_out, t_from=lib.SSD_DLEN_GENERATED)
         elif gamma > 0:
             model.decode(w.max_new, gamma, out, n_out)
         else:
@@ -904,7 +907,7 @@ def main() -> None:
         rs.copy_(torch.tensor(ws.resid_scale(), device="cuda"))
         ins.copy_(torch.tensor([ws.in_scale()], device="cuda"))
         row = {"s": s}
-        for name, gamma in (("ssd", w.gamma), ("greedy", 0), ("ssd_dynamic", -1)):
+        for name, gamma in (("ssd", w.gamma), ("greedy", 0), ("ssd_dynamic", -1), ("ssd_dynamic_gen", -2)):
             ts = []
             for _ in range(2):
                 a, b, c = (torch.cuda.Event(enable_timing=True) for _ in range(3))
@@ -918,12 +921,16 @@ def main() -> None:
                 sst = model.stats()
                 row["mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
                 row["steps"] = sst["steps"]
-            if name == "ssd_dynamic":
+            if name.startswith("ssd_dynamic"):
                 sst = model.stats()
-                row["dynamic_mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
-                row["dynamic_mean_gamma"] = sst["drafted"] / max(sst["steps"], 1)
+                acc, dr = model.step_log()
+                tag = name[len("ssd_"):]
+                row[f"{tag}_mean_accept"] = sst["accepted"] / max(sst["steps"], 1)
+                row[f"{tag}_mean_gamma"] = sst["drafted"] / max(sst["steps"], 1)
+                row[f"{tag}_gamma_first_max"] = [dr[0], max(dr)] if dr else None   # the schedule grows with t
         row["speedup"] = row["ssd_decode_tok_s"] / row["greedy_decode_tok_s"]
         row["dynamic_speedup"] = row["ssd_dynamic_decode_tok_s"] / row["greedy_decode_tok_s"]
+        row["dynamic_gen_speedup"] = row["ssd_dynamic_gen_decode_tok_s"] / row["greedy_decode_tok_s"]
         per_s.append(row)
     rs.copy_(torch.tensor(w.resid_scale(), device="cuda"))
     ins.copy_(torch.tensor([w.in_scale()], device="cuda"))

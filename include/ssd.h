@@ -85,7 +85,7 @@ enum {
 #define SSD_OPT_PREFILL_ROWS 2  /* prefill through the decode kernels in 8-row chunks instead of the
                                  * tensor-core GEMMs */
 
-#define SSD_MAX_GAMMA 8
+#define SSD_MAX_GAMMA 15  /* the paper's d0 + 10 for d0 = 5 (Sec. "Choice of d") */
 #define SSD_MAX_ROWS 16   /* rows one decode pass may carry (gamma + 1, prefill chunk) */
 
 typedef struct ssd_ctx ssd_ctx;
@@ -243,15 +243,20 @@ SSD_API ssd_status ssd_decode(ssd_ctx* ctx, int max_new, int gamma, int32_t* out
 
 /* SSD decode with the dynamic draft length of Sec. "Choice of d":
  *   d(t) = d0 + floor(10 / (1 + exp(-0.01 (t - n_max / 2))))   (fp64, host)
- * where the t-th token is generated from t - 1 tokens of context, so a step
- * whose last emitted token sits at position kv_len uses t = kv_len + 2.  Each
- * step drafts min(d(t), gamma_cap) tokens (gamma_cap <= gamma_max; the paper's
+ * with t counted one of two ways (the paper does not say which):
+ *   t_from = SSD_DLEN_CONTEXT:   over the whole context -- the t-th token is generated
+ *     from t - 1 tokens, so a step whose last emitted token sits at position kv_len
+ *     uses t = kv_len + 2 (n_max: the longest sequence, e.g. max_seq);
+ *   t_from = SSD_DLEN_GENERATED: over the generated tokens -- t = tokens emitted so far
+ *     + 1, the index of the next new token (n_max: the generation length, max_new).
+ * Each step drafts min(d(t), gamma_cap) tokens (gamma_cap <= gamma_max; the paper's
  * range is d0 .. d0 + 10) and, in the last steps, accepts at most remaining - 1.
  * One CUDA-graph launch: a WHILE node whose body selects the step's branch of a
  * SWITCH node (one draft + verify + accept branch per gamma) from a device
- * table of d(kv_len + 2).  Same buffers, capacity rule (with gamma_cap) and
+ * table of d indexed by kv_len.  Same buffers, capacity rule (with gamma_cap) and
  * errors as ssd_decode.  async. */
-SSD_API ssd_status ssd_decode_dynamic(ssd_ctx* ctx, int max_new, int d0, int n_max, int gamma_cap,
+enum { SSD_DLEN_CONTEXT = 0, SSD_DLEN_GENERATED = 1 };
+SSD_API ssd_status ssd_decode_dynamic(ssd_ctx* ctx, int max_new, int d0, int n_max, int t_from, int gamma_cap,
                                       int32_t* out_tok, int32_t* n_out);
 
 /* d(t) of Sec. "Choice of d", the value ssd_decode_dynamic tabulates (host

@@ -305,7 +305,7 @@ class _SSDRun:
     step per call to step() (see ssd_generate)."""
 
     def __init__(self, m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int, max_seq: int | None,
-                 reuse_draft_rows: bool, keep_draft_logits: bool, dynamic: tuple[int, int] | None):
+                 reuse_draft_rows: bool, keep_draft_logits: bool, dynamic: tuple | None):
         c = m.cfg
         self.m, self.max_new, self.gamma = m, max_new, gamma
         self.reuse, self.keep_dlog, self.dynamic = reuse_draft_rows, keep_draft_logits, dynamic
@@ -324,7 +324,15 @@ class _SSDRun:
     def gamma_eff(self) -> int:
         """Drafts of the next step: min(gamma or d(t), remaining - 1)."""
         remaining = self.max_new - len(self.res.tokens)
-        g_step = self.gamma if self.dynamic is None else min(self.gamma, draft_length(self.p + 2, *self.dynamic))
+        g_step = self.gamma
+        if self.dynamic is not None:
+            d0, n_max = self.dynamic[0], self.dynamic[1]
+            over = self.dynamic[2] if len(self.dynamic) > 2 else "context"
+            # t: the index of the token this step's verification will emit first, counted over the
+            # whole context (a token at position q is the (q + 1)-th; the next one sits at p + 1) or
+            # over the generated tokens (the next new token is number len(tokens) + 1)
+            t = self.p + 2 if over == "context" else len(self.res.tokens) + 1
+            g_step = min(self.gamma, draft_length(t, d0, n_max))
         return min(g_step, remaining - 1)
 
     def step(self) -> None:
@@ -372,7 +380,7 @@ class _SSDRun:
 def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
                  max_seq: int | None = None, reuse_draft_rows: bool = True,
                  keep_cache: bool = False, keep_draft_logits: bool = False,
-                 max_steps: int | None = None, dynamic: tuple[int, int] | None = None) -> Result:
+                 max_steps: int | None = None, dynamic: tuple | None = None) -> Result:
     """Algorithm 1 (greedy self-speculative decoding with the imitation network).
 
     Per step, with y the last emitted token at position p = kv_len:
@@ -383,8 +391,9 @@ def ssd_generate(m: Model, vis: np.ndarray, prompt, max_new: int, gamma: int,
       accepting: a = largest i <= gamma_eff with d_1..d_i = f_0..f_{i-1};
                  emit d_1..d_a and f_a; kv_len = p + a + 1; y = f_a.
     max_steps (timing samples only) stops after that many steps.
-    dynamic = (d0, N): each step drafts min(d(t), gamma, remaining - 1) tokens with
-    t = kv_len + 2 (Sec. "Choice of d"); gamma is then the cap.
+    dynamic = (d0, N) or (d0, N, "generated"): each step drafts min(d(t), gamma, remaining - 1)
+    tokens (Sec. "Choice of d"); gamma is then the cap.  t = kv_len + 2 counts the whole context;
+    with "generated", t = tokens emitted so far + 1 counts the new tokens only.
     """
     run = _SSDRun(m, vis, prompt, max_new, gamma, max_seq, reuse_draft_rows, keep_draft_logits, dynamic)
     while not run.finished and (max_steps is None or len(run.res.step_s) < max_steps):

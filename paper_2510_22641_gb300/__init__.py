@@ -4,12 +4,13 @@ The compute lives in libssd.so (hand-written CUDA, C ABI in include/ssd.h);
 this package only builds it and marshals arguments.
 """
 from . import _binding
-from ._binding import (SSD_ARCH_LLAMA, SSD_ARCH_T5, SSD_FAULT_ALLOC, SSD_FAULT_LAUNCH, SSD_FAULT_NONE, SSD_IN_IDENTITY,
+from ._binding import (SSD_ARCH_LLAMA, SSD_ARCH_T5, SSD_DLEN_CONTEXT, SSD_DLEN_GENERATED, SSD_FAULT_ALLOC, SSD_FAULT_LAUNCH, SSD_FAULT_NONE, SSD_IN_IDENTITY,
                        SSD_IN_MLP2, SSD_MAX_GAMMA, SSD_OPT_HOST_LOOP, SSD_OPT_PREFILL_ROWS, SSDError, load)
 from .build import build
 
 __all__ = ["build", "load", "SSDError", "SSD_ARCH_LLAMA", "SSD_ARCH_T5", "SSD_IN_IDENTITY", "SSD_IN_MLP2",
-           "SSD_MAX_GAMMA", "SSD_OPT_HOST_LOOP", "SSD_OPT_PREFILL_ROWS", "SSD_FAULT_NONE", "SSD_FAULT_ALLOC",
+           "SSD_MAX_GAMMA", "SSD_OPT_HOST_LOOP", "SSD_OPT_PREFILL_ROWS", "SSD_DLEN_CONTEXT", "SSD_DLEN_GENERATED",
+           "SSD_FAULT_NONE", "SSD_FAULT_ALLOC",
            "SSD_FAULT_LAUNCH", "SSDModel", "bf16_bits_to_device", "encdec_device_weights", "config_dict",
            "t5_config_dict", "set_fault_injection"]
 

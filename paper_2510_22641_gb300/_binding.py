@@ -12,7 +12,7 @@ import os
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "libssd.so")
 
-SSD_MAX_GAMMA = 8
+SSD_MAX_GAMMA = 15
 SSD_MAX_ROWS = 16
 SSD_IN_IDENTITY = 0
 SSD_IN_MLP2 = 1
@@ -21,6 +21,8 @@ SSD_ARCH_LLAMA = 0
 SSD_ARCH_T5 = 1
 SSD_OPT_HOST_LOOP = 1
 SSD_OPT_PREFILL_ROWS = 2
+SSD_DLEN_CONTEXT = 0
+SSD_DLEN_GENERATED = 1
 SSD_FAULT_NONE = 0
 SSD_FAULT_ALLOC = 1
 SSD_FAULT_LAUNCH = 2
@@ -98,7 +100,7 @@ def load(path: str = LIB_PATH) -> ctypes.CDLL:
         "ssd_draft": [vp, i32, pi32],
         "ssd_verify": [vp, i32, pi32, pi32],
         "ssd_decode": [vp, i32, i32, pi32, pi32],
-        "ssd_decode_dynamic": [vp, i32, i32, i32, i32, pi32, pi32],
+        "ssd_decode_dynamic": [vp, i32, i32, i32, i32, i32, pi32, pi32],
         "ssd_greedy_decode": [vp, i32, pi32, pi32],
         "ssd_generate": [vp, vp, i32, vp, i32, i32, i32, vp, ctypes.POINTER(i32), ctypes.POINTER(SSDStats)],
         "ssd_greedy_generate": [vp, vp, i32, vp, i32, i32, vp, ctypes.POINTER(i32), ctypes.POINTER(SSDStats)],

@@ -40,7 +40,7 @@
 
 namespace ssd {
 
-constexpr int kAttnMaxRows = 9;           // query rows of one call (gamma_max + 1)
+constexpr int kAttnMaxRows = SSD_MAX_GAMMA + 1;  // query rows per request of one call (gamma_max + 1)
 constexpr int kAttnChunkBytes = 16384;    // one K (or V) chunk: 32 keys of head_dim 128, 64 of 64
 constexpr int kAttnWarps = 8;
 constexpr int kAttnThreads = 32 * kAttnWarps;
@@ -103,8 +103,9 @@ struct AttnSmem {
   static constexpr int kTotal = kBar + (kAttnBufs + 1) * 8;
 };
 
+// Up to 9 rows two CTAs share an SM; beyond that one CTA holds the larger q rows and accumulators.
 template <int M, int DH, bool EXT>
-__global__ void __launch_bounds__(kAttnThreads, 2) ssd_splitkv_attn_kernel(const AttnParams p) {
+__global__ void __launch_bounds__(kAttnThreads, M <= 9 ? 2 : 1) ssd_splitkv_attn_kernel(const AttnParams p) {
   using S = AttnSmem<M, DH>;
   using G = AttnGeo<DH>;
   constexpr int KPC = G::KPC, KPW = G::KPW, TPK = G::TPK, DPP = G::DPP, NF = G::NF, DPL = G::DPL;

@@ -19,8 +19,10 @@ constexpr int kMaxMidRows = 128;  // rows of one medium-M projection (the verifi
 enum : int { DERR_TOKEN = 1, DERR_TIMEOUT = 2, DERR_POS = 4 };
 
 // Decode state kept in device memory so that a captured graph replays the
-// whole draft/verify/accept loop without host round trips.
-struct DevState {
+// whole draft/verify/accept loop without host round trips.  16-byte aligned, so
+// that whatever follows a DevState (an array of them, a scratch struct) keeps
+// 16-byte alignment for vector and bulk copies.
+struct alignas(16) DevState {
   int kv_len;      // valid cache length p == position of the current token y
   int cur_tok;     // y: last emitted token, not yet in the cache
   int n_out;       // tokens emitted so far (the prefill's first token included)

@@ -48,6 +48,8 @@ cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, cons
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
                        int num_sms, cudaStream_t s, bool pdl);
 cudaError_t mid_attrs();
+cudaError_t attn_launch(int M, int head_dim, const AttnParams& a, int nreq, cudaStream_t s, bool pdl);
+cudaError_t attn_attrs();
 int mid_max_ctas(int num_sms);
 cudaError_t split_act_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                              __nv_bfloat16* hi, __nv_bfloat16* lo, int ld, float* rs, int rows, cudaStream_t s,
@@ -59,7 +61,7 @@ using namespace ssd;
 namespace {
 
 constexpr int kPrefillChunk = 8;  // prefill rows per pass through the layers
-constexpr int kMaxVerifyRows = 9; // rows of one request's verification pass (gamma_max + 1)
+constexpr int kMaxVerifyRows = SSD_MAX_GAMMA + 1;  // rows of one request's verification pass
 constexpr int kMidMinRows = kMaxRows + 1;  // projections over more rows use the medium-M kernel
 
 struct Site {  // one projection: up to three weight matrices with a common K
@@ -159,7 +161,7 @@ struct ssd_ctx {
   int* dyn_table = nullptr;   // device [max_seq + 1]
   int* dyn_launch = nullptr;  // device [SSD_MAX_GAMMA]: kernel launches of the step branch for gamma
   std::vector<int> dyn_table_h;
-  int dyn_d0 = -1, dyn_n = -1;
+  int dyn_d0 = -1, dyn_n = -1, dyn_origin = -1;  // the tabulated schedule: d0, N, t's origin
   std::map<int, cudaGraphExec_t> dyn_graphs;
   int64_t dyn_host_launches = 0;
   // Diagnostic: drive the decode loop from the host with one plain graph per
@@ -336,47 +338,6 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
   return SSD_OK;
 }
 
-// EXT: fixed key sets / absolute positions / relative-position bias (the encoder-decoder model).
-template <int M>
-static cudaError_t attn_launch_m(ssd_ctx* c, const AttnParams& a, int nreq) {
-  const dim3 grid(kAttnSplit, c->cfg.n_heads, nreq);
-  const bool ext = a.fixed_keys || a.abs_pos || a.bias;
-  if (c->cfg.head_dim == 128)
-    return ext ? launch_k(c, ssd_splitkv_attn_kernel<M, 128, true>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a)
-               : launch_k(c, ssd_splitkv_attn_kernel<M, 128, false>, grid, dim3(kAttnThreads), AttnSmem<M, 128>::kTotal, a);
-  return ext ? launch_k(c, ssd_splitkv_attn_kernel<M, 64, true>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a)
-             : launch_k(c, ssd_splitkv_attn_kernel<M, 64, false>, grid, dim3(kAttnThreads), AttnSmem<M, 64>::kTotal, a);
-}
-
-template <int M, int DH>
-static cudaError_t attn_attr_md() {
-  cudaError_t e = cudaFuncSetAttribute(ssd_splitkv_attn_kernel<M, DH, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       AttnSmem<M, DH>::kTotal);
-  if (e != cudaSuccess) return e;
-  return cudaFuncSetAttribute(ssd_splitkv_attn_kernel<M, DH, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              AttnSmem<M, DH>::kTotal);
-}
-
-template <int M>
-static cudaError_t attn_attr_m() {
-  cudaError_t e = attn_attr_md<M, 128>();
-  if (e != cudaSuccess) return e;
-  return attn_attr_md<M, 64>();
-}
-
-static cudaError_t attn_attrs() {
-  cudaError_t e;
-  if ((e = attn_attr_m<1>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<2>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<3>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<4>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<5>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<6>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<7>()) != cudaSuccess) return e;
-  if ((e = attn_attr_m<8>()) != cudaSuccess) return e;
-  return attn_attr_m<9>();
-}
-
 // One split-KV attention launch over M query rows per request for nreq requests (the ctx's
 // scratch, state and head count filled in).
 static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a, int nreq = 1) {
@@ -384,20 +345,9 @@ static ssd_status attn_run(ssd_ctx* c, int M, AttnParams a, int nreq = 1) {
   a.tickets = c->attn_tickets;
   a.st = c->st;
   a.n_heads = c->cfg.n_heads;
-  cudaError_t r;
-  switch (M) {
-    case 1: r = attn_launch_m<1>(c, a, nreq); break;
-    case 2: r = attn_launch_m<2>(c, a, nreq); break;
-    case 3: r = attn_launch_m<3>(c, a, nreq); break;
-    case 4: r = attn_launch_m<4>(c, a, nreq); break;
-    case 5: r = attn_launch_m<5>(c, a, nreq); break;
-    case 6: r = attn_launch_m<6>(c, a, nreq); break;
-    case 7: r = attn_launch_m<7>(c, a, nreq); break;
-    case 8: r = attn_launch_m<8>(c, a, nreq); break;
-    case 9: r = attn_launch_m<9>(c, a, nreq); break;
-    default: return fail(c, SSD_ERR_INVALID_ARG, "attention rows %d out of range", M);
-  }
-  CK(r);
+  if (M < 1 || M > kAttnMaxRows) return fail(c, SSD_ERR_INVALID_ARG, "attention rows %d out of range", M);
+  CK(count_launch(c));
+  CK(attn_launch(M, c->cfg.head_dim, a, nreq, c->cs, c->use_pdl));
   return SSD_OK;
 }
 
@@ -1948,22 +1898,28 @@ static ssd_status decode_impl(ssd_ctx* c, int max_new, int gamma, int32_t* out_t
   return SSD_OK;
 }
 
-static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, int cap, int32_t* out_tok,
-                                  int32_t* n_out) {
+static ssd_status decode_dyn_impl(ssd_ctx* c, int max_new, int d0, int n_max, int t_from, int cap,
+                                  int32_t* out_tok, int32_t* n_out) {
   if (!c->prefilled) return fail(c, SSD_ERR_STATE, "decode before ssd_prefill");
   if (max_new < 1) return fail(c, SSD_ERR_INVALID_ARG, "max_new must be >= 1");
   if (cap < 1 || cap > c->cfg.gamma_max) return fail(c, SSD_ERR_INVALID_ARG, "gamma cap %d", cap);
   if (d0 < 1 || n_max < 1) return fail(c, SSD_ERR_INVALID_ARG, "d0 %d, n_max %d", d0, n_max);
+  if (t_from != SSD_DLEN_CONTEXT && t_from != SSD_DLEN_GENERATED)
+    return fail(c, SSD_ERR_INVALID_ARG, "t_from %d", t_from);
+  // t of the step whose last emitted token sits at position p: p + 2 over the whole context, or
+  // p - P + 2 (= tokens emitted so far + 1) over the generated tokens
+  const int origin = t_from == SSD_DLEN_CONTEXT ? 0 : c->prompt_len;
   if (static_cast<int64_t>(c->prompt_len) + max_new + cap + 1 > c->cfg.max_seq)
     return fail(c, SSD_ERR_CAPACITY, "n_vis + n_prompt + max_new + cap + 1 = %d > max_seq = %d",
                 c->prompt_len + max_new + cap + 1, c->cfg.max_seq);
-  if (d0 != c->dyn_d0 || n_max != c->dyn_n) {  // the table of the previous schedule may still be read
+  if (d0 != c->dyn_d0 || n_max != c->dyn_n || origin != c->dyn_origin) {  // the old table may still be read
     CK(cudaStreamSynchronize(c->cs));
     c->dyn_table_h.resize(c->cfg.max_seq + 1);
-    for (int p = 0; p <= c->cfg.max_seq; ++p) c->dyn_table_h[p] = draft_length_fp64(p + 2, d0, n_max);
+    for (int p = 0; p <= c->cfg.max_seq; ++p) c->dyn_table_h[p] = draft_length_fp64(p - origin + 2, d0, n_max);
     CK(cudaMemcpy(c->dyn_table, c->dyn_table_h.data(), sizeof(int) * (c->cfg.max_seq + 1), cudaMemcpyHostToDevice));
     c->dyn_d0 = d0;
     c->dyn_n = n_max;
+    c->dyn_origin = origin;
   }
   ssd_decode_setup_kernel<<<1, 32, 0, c->cs>>>(c->st, max_new, cap);
   CK(cudaGetLastError());
@@ -2011,11 +1967,11 @@ int ssd_rel_bucket(int delta, int bidirectional, int n_buckets, int max_distance
   return rel_bucket_host(delta, bidirectional != 0, n_buckets, max_distance);
 }
 
-ssd_status ssd_decode_dynamic(ssd_ctx* c, int max_new, int d0, int n_max, int gamma_cap, int32_t* out_tok,
+ssd_status ssd_decode_dynamic(ssd_ctx* c, int max_new, int d0, int n_max, int t_from, int gamma_cap, int32_t* out_tok,
                               int32_t* n_out) {
   if (!c) return SSD_ERR_INVALID_ARG;
   CKS(enter(c));
-  CKS(decode_dyn_impl(c, max_new, d0, n_max, gamma_cap, out_tok, n_out));
+  CKS(decode_dyn_impl(c, max_new, d0, n_max, t_from, gamma_cap, out_tok, n_out));
   return leave(c);
 }
 

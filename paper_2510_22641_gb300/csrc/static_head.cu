@@ -31,7 +31,8 @@ constexpr int kStaticMaxDevices = 64;
 struct StaticScratch {
   DevState st;                                             // argmax accumulators, error word
   unsigned counters[kStaticMaxTiles];                      // tickets of split row tiles
-  float partials[2 * kStaticMaxCtas * kMaxRows * kTileN];  // partial sums of split row tiles
+  // partial sums of split row tiles, read 16 bytes at a time
+  alignas(16) float partials[2 * kStaticMaxCtas * kMaxRows * kTileN];
 };
 
 // About 5.3 MB of device memory per GPU, held from library load until exit.

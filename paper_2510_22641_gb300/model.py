@@ -154,9 +154,10 @@ class SSDModel:
         self._call("ssd_decode", max_new, gamma, _ptr(out_tok), _ptr(n_out))
 
     def decode_dynamic(self, max_new: int, d0: int, n_max: int, gamma_cap: int, out_tok: torch.Tensor | None = None,
-                       n_out: torch.Tensor | None = None):
-        """SSD with the dynamic draft length d(t) (Sec. "Choice of d"), capped at gamma_cap."""
-        self._call("ssd_decode_dynamic", max_new, d0, n_max, gamma_cap, _ptr(out_tok), _ptr(n_out))
+                       n_out: torch.Tensor | None = None, t_from: int = B.SSD_DLEN_CONTEXT):
+        """SSD with the dynamic draft length d(t) (Sec. "Choice of d"), capped at gamma_cap; t counted
+        over the whole context (SSD_DLEN_CONTEXT) or over the generated tokens (SSD_DLEN_GENERATED)."""
+        self._call("ssd_decode_dynamic", max_new, d0, n_max, t_from, gamma_cap, _ptr(out_tok), _ptr(n_out))
 
     def greedy_decode(self, max_new: int, out_tok: torch.Tensor | None = None, n_out: torch.Tensor | None = None):
         self._call("ssd_greedy_decode", max_new, _ptr(out_tok), _ptr(n_out))

@@ -177,6 +177,46 @@ def test_dynamic_draft_length_matches_oracle(request, tiny_bits, s, cap, n_max, 
     assert dec == expect + (2 if host else 3)
 
 
+@pytest.fixture(scope="module")
+def tiny_model_g15(tiny_bits):
+    """gamma_max = 15 (d0 + 10 for d0 = 5): verification passes of up to 16 rows."""
+    w = synth.TINY.replace(norm_gain="perturbed", gamma=15)
+    model, _, dev = make_model(w, tiny_bits, gamma_max=15, max_seq=w.max_seq())
+    yield model, dev
+    model.close()
+
+
+@pytest.mark.parametrize("s,n_max", [(0.05, 32), (0.2, 200)])
+def test_dynamic_draft_length_over_generated_tokens(tiny_model_g15, tiny_bits, s, n_max):
+    """d(t) with t = the index of the next new token and N the generation length, capped at 15:
+    tokens, logits, draft logits, per-step accept lengths and draft counts match the oracle's run
+    under the same reading; the steps draft up to 15 tokens (16-row verification passes)."""
+    model, _ = tiny_model_g15
+    w = synth.TINY.replace(norm_gain="perturbed", s=s)
+    set_scale(model, w)
+    _, _, v, p = device_inputs(w)
+    logits = torch.full((w.max_new, w.shape.vocab), float("nan"), device="cuda")
+    dlog = torch.full((w.max_new, 15, w.shape.vocab), float("nan"), device="cuda")
+    model.set_logits_capture(logits)
+    model.set_draft_logits_capture(dlog)
+    out = torch.zeros(w.max_new, dtype=torch.int32, device="cuda")
+    n = torch.zeros(1, dtype=torch.int32, device="cuda")
+    model.prefill(v, p)
+    model.decode_dynamic(w.max_new, 5, n_max, 15, out, n, t_from=lib.SSD_DLEN_GENERATED)
+    model.sync()
+    toks, stats = out[: int(n.item())].cpu().tolist(), model.stats()
+    stats["accepted_log"], stats["drafted_log"] = model.step_log()
+    stats["draft_logits"] = dlog.cpu().numpy()
+    model.set_draft_logits_capture(None)
+    m = oracle.model_from_bits(w, tiny_bits, synth.bf16_to_f64)
+    vis, prompt = synth.make_inputs(w)
+    ref = oracle.ssd_generate(m, synth.bf16_to_f64(vis), prompt, w.max_new, 15, dynamic=(5, n_max, "generated"),
+                              keep_draft_logits=True)
+    check_against_oracle(toks, logits.cpu().numpy(), stats, ref, 15)
+    assert stats["drafted"] == sum(len(d) for d in ref.draft_tokens)
+    assert max(len(d) for d in ref.draft_tokens) >= 7
+
+
 def test_kv_cache_after_rollback_equals_greedy_cache(tiny_model):
     model, _ = tiny_model
     w = synth.TINY.replace(norm_gain="perturbed", s=0.2)

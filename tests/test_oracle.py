@@ -320,6 +320,29 @@ def test_ssd_dynamic_draft_length_equals_greedy(tiny_bits, s, cap, n_max):
     assert p == r.kv_len == g.kv_len
 
 
+@pytest.mark.parametrize("s,n_max", [(0.05, 32), (0.2, 200)])
+def test_ssd_dynamic_draft_length_over_generated_tokens(tiny_bits, s, n_max):
+    """The other reading of t: the index of the next new token.  Per step the schedule follows the
+    count of emitted tokens (not the cache length), so the first step drafts d(2) whatever the
+    prompt's length; with N = 200 over 32 tokens the drafts grow with t; SSD still equals greedy."""
+    cap = 15
+    w = tiny(s=s, gamma=cap)
+    m, vis, prompt = build(w, tiny_bits)
+    g = oracle.greedy_generate(m, vis, prompt, w.max_new)
+    r = oracle.ssd_generate(m, vis, prompt, w.max_new, cap, dynamic=(5, n_max, "generated"))
+    assert r.tokens == g.tokens
+    n = 1
+    for drafts, a in zip(r.draft_tokens, r.accept_lengths):
+        t = n + 1                                                 # the next new token's index
+        g_t = min(oracle.draft_length(t, 5, n_max), cap, w.max_new - n - 1)
+        assert len(drafts) == g_t and 0 <= a <= g_t
+        n += a + 1
+    assert len(r.draft_tokens[0]) == min(oracle.draft_length(2, 5, n_max), cap)
+    if n_max == 200:  # d(t) = 5 + floor(10 sigmoid(0.01 (t - 100))): 7 at t = 2, 8 from t = 16 on
+        assert oracle.draft_length(2, 5, 200) == 7 and oracle.draft_length(16, 5, 200) == 8
+        assert len(r.draft_tokens[0]) == 7
+
+
 # --------------------------------------------------------------------------- IN_BLOCK imitation (one decoder block)
 
 def torch_block_rows(m: oracle.Model, vis: np.ndarray, tokens):
