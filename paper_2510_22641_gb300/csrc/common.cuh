@@ -14,6 +14,9 @@ namespace ssd {
 
 constexpr int kMaxRows = SSD_MAX_ROWS;
 constexpr int kMaxMidRows = 128;  // rows of one medium-M projection (the verification of batched requests)
+constexpr int kAmKeyStride = 16;    // 64-bit argmax keys per LM-head row slot (128 bytes)
+constexpr int kAmChunks = kMaxMidRows / 16;  // 16-row chunks of a medium-M LM head
+constexpr int kAmCountStride = 32;  // 32-bit tickets per chunk slot (128 bytes)
 
 // Device error bits (DevState::error).
 enum : int { DERR_TOKEN = 1, DERR_TIMEOUT = 2, DERR_POS = 4 };
@@ -43,8 +46,11 @@ struct alignas(16) DevState {
   int tok_in[kMaxRows];          // verify rows t_0 = y, t_j = d_j
   int full_tok[kMaxRows];        // f_i = full-model argmax of row i
   int last_emitted[kMaxRows];
-  unsigned long long am_key[kMaxMidRows];  // packed argmax accumulators of the LM head's rows
-  unsigned int am_count;                // LM-head row tiles finished
+  // packed argmax accumulators of the LM head's rows, row r at am_key[r * kAmKeyStride] (one
+  // 128-byte line per row: the tiles' atomics on different rows do not share a line)
+  unsigned long long am_key[kMaxMidRows * kAmKeyStride];
+  // LM-head row tiles finished, per 16-row chunk ch at am_count[ch * kAmCountStride]
+  unsigned int am_count[kAmChunks * kAmCountStride];
 };
 
 // ------------------------------------------------------------------ PTX wrappers

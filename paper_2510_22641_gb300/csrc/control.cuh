@@ -74,8 +74,8 @@ __global__ void ssd_prefill_begin_kernel(DevState* st, int P, int eos_id, int en
   st->eos_id = eos_id;
   st->steps = st->drafted = st->accepted = 0;
   for (int i = 0; i <= SSD_MAX_GAMMA; ++i) st->hist[i] = 0;
-  for (int i = 0; i < kMaxMidRows; ++i) st->am_key[i] = 0ull;
-  st->am_count = 0u;
+  for (int i = 0; i < kMaxMidRows; ++i) st->am_key[i * kAmKeyStride] = 0ull;
+  for (int i = 0; i < kAmChunks; ++i) st->am_count[i * kAmCountStride] = 0u;
 }
 
 // The last prompt row's greedy token is the first new token; the cache now holds positions 0..P-1.

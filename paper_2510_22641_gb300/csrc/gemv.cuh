@@ -214,6 +214,12 @@ __device__ __forceinline__ uint32_t pack_bf16x2(__nv_bfloat16 lo, __nv_bfloat16 
 
 __device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
 
+// The LM head epilogue's per-warp argmax keys of a tile's rows, [drain warp][row] (16 rows).
+__device__ __forceinline__ unsigned long long* argmax_warp_keys() {
+  __shared__ unsigned long long keys[(kDrainThreads / 32) * kNPad];
+  return keys;
+}
+
 // Launch row mg's request and offset within the request's rows (batch_rows > 0).
 __device__ __forceinline__ int batch_offset(const GemvParams& p, int mg, int b) {
   return p.pos_off + mg - b * p.batch_rows;
@@ -353,25 +359,36 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
         const unsigned long long o = __shfl_xor_sync(0xffffffffu, key, off);
         key = o > key ? o : key;
       }
-      if (lane == 0) atomicMax(&p.st->am_key[mg], key);
+      if (lane == 0) argmax_warp_keys()[(tid >> 5) * kNPad + m] = key;
     }
   }
 }
 
-// LM head, after a row tile's keys of all M launch rows are in (or one chunk's rows, `tiles`
-// counting every tile x chunk): the maxima are released by one acq_rel ticket after the CTA
-// barrier; the tile that completes the count reads and resets
-// the M keys, one thread per row, and writes the tokens (-1 once a bounded wait anywhere has
-// given up: the keys may miss tiles).
-__device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, int M, const int* rreq, int tid, int tiles) {
+// LM head, after the epilogue of a row tile: each drain warp left its maxima of the tile's rows
+// m0 .. m0 + mc - 1 in shared memory; thread r folds the four warps' keys of row m0 + r into the
+// row's global key with one atomic (rows on separate 128-byte lines).  The maxima are released
+// by one acq_rel ticket of the rows' 16-row chunk after the CTA barrier; the tile that completes
+// the chunk's count of `tiles` reads and resets the chunk's keys, one thread per row, and writes
+// the tokens (-1 once a bounded wait anywhere has given up: the keys may miss tiles).
+__device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, const int* rreq, int tid, int tiles,
+                                                   int m0, int mc) {
   __shared__ int am_last;
+  const unsigned long long* wk = argmax_warp_keys();
+  unsigned int* count = &p.st->am_count[(m0 / kNPad) * kAmCountStride];
   drain_sync();
-  if (tid == 0) am_last = atom_add_acq_rel_gpu(&p.st->am_count, 1u) == static_cast<unsigned>(tiles - 1);
+  if (tid < mc) {
+    unsigned long long key = wk[tid];
+#pragma unroll
+    for (int w = 1; w < kDrainThreads / 32; ++w) key = max(key, wk[w * kNPad + tid]);
+    atomicMax(&p.st->am_key[(m0 + tid) * kAmKeyStride], key);
+  }
+  drain_sync();
+  if (tid == 0) am_last = atom_add_acq_rel_gpu(count, 1u) == static_cast<unsigned>(tiles - 1);
   drain_sync();
   if (am_last) {
     const bool stopped = (__ldcg(&p.st->error) & DERR_TIMEOUT) != 0;
-    for (int r = tid; r < M; r += kDrainThreads) {
-      const unsigned long long key = atomicExch(&p.st->am_key[r], 0ull);
+    for (int r = m0 + tid; r < m0 + mc; r += kDrainThreads) {
+      const unsigned long long key = atomicExch(&p.st->am_key[r * kAmKeyStride], 0ull);
       const int tok = stopped ? -1 : static_cast<int>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFull));
       if (rreq) {
         const int b = rreq[r];
@@ -380,7 +397,7 @@ __device__ __forceinline__ void gemv_argmax_finish(const GemvParams& p, int M, c
         p.tok_dst[r * (p.tok_stride ? p.tok_stride : 1)] = tok;
       }
     }
-    if (tid == 0) atomicExch(&p.st->am_count, 0u);
+    if (tid == 0) atomicExch(count, 0u);
   }
 }
 
@@ -667,7 +684,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       const bool whole = (seg_kt0 == 0) && (kt == p.n_kt - 1);
       if (whole) {
         gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
-        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt, p.n_rt);
+        if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, rreq, dt, p.n_rt, 0, M);
       } else {
         const int slot = 2 * c + (rt == rt_first ? 0 : 1);
         float* dstp = p.partials + static_cast<size_t>(slot) * (kMaxRows * kTileN);
@@ -744,7 +761,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
           }
           drain_sync();
           gemv_epilogue<M, EPI>(p, rt, outb, rs, pre_of(rt), base_pos, rpos, rreq, dt, 0, M);
-          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, dt, p.n_rt);
+          if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, rreq, dt, p.n_rt, 0, M);
           if (dt == 0) p.counters[rt] = 0u;
         }
       }

@@ -309,8 +309,8 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
 // streamed by `G = p.grid_ctas` CTAs: sums the tile's partials (slots c + rt for the CTAs c that
 // held its units) in CTA order, then applies the RMSNorm scale and the fused epilogue to rows
 // 16 ch .. 16 ch + 15 -- the GEMV's epilogue code, with its inputs (rotation table rows, residual
-// base rows) loaded up front.  The LM head's argmax keys are finished by the last of all
-// n_rt x chunks CTAs.
+// base rows) loaded up front.  The LM head's argmax keys of a chunk are finished by the last of
+// the chunk's n_rt CTAs.
 template <Epi EPI>
 __global__ void __launch_bounds__(kDrainThreads) ssd_mid_reduce_kernel(const GemvParams p, int M) {
   __shared__ __align__(16) float outb[kNPad * kTileN];
@@ -385,7 +385,7 @@ __global__ void __launch_bounds__(kDrainThreads) ssd_mid_reduce_kernel(const Gem
   }
   __syncthreads();
   gemv_epilogue<kNPad, EPI>(p, rt, outb, rs, use_pre ? pre : nullptr, base_pos, rpos, rreq, tid, m0, mc);
-  if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, M, rreq, tid, p.n_rt * gridDim.x);
+  if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, rreq, tid, p.n_rt, m0, mc);
 }
 
 }  // namespace ssd
