@@ -23,61 +23,6 @@
 
 namespace ssd {
 
-// ------------------------------------------------------------------ tcgen05 helpers
-
-// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
-// groups 1024 bytes apart (the layout TMA writes with SWIZZLE_128B).
-__device__ __forceinline__ uint64_t tc_smem_desc(uint32_t saddr) {
-  uint64_t d = 0;
-  d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);        // start address
-  d |= static_cast<uint64_t>(1u) << 16;                       // leading byte offset (unused for swizzled K-major)
-  d |= static_cast<uint64_t>(1024u >> 4) << 32;               // stride byte offset: 8 rows x 128 B
-  d |= static_cast<uint64_t>(1u) << 46;                       // descriptor version
-  d |= static_cast<uint64_t>(2u) << 61;                       // swizzle: 128 B
-  return d;
-}
-
-// Instruction descriptor, kind::f16: bf16 x bf16 -> fp32, both K-major, M x N.
-__host__ __device__ constexpr uint32_t tc_idesc(int m, int n) {
-  return (1u << 4)                                  // D format: fp32
-         | (1u << 7)                                // A format: bf16
-         | (1u << 10)                               // B format: bf16
-         | (static_cast<uint32_t>(n >> 3) << 17)    // N / 8
-         | (static_cast<uint32_t>(m >> 4) << 24);   // M / 16
-}
-
-__device__ __forceinline__ void tc_mma(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                       uint32_t accumulate) {
-  asm volatile(
-      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
-      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-__device__ __forceinline__ void tc_commit(uint64_t* bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
-               : "memory");
-}
-
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-
-// 32 consecutive fp32 columns of this warp's 32 TMEM lanes (one lane per thread).
-__device__ __forceinline__ void tc_ld32(uint32_t taddr, float* v) {
-  uint32_t r[32];
-  asm volatile(
-      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
-      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
-      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
-        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
-        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
-      : "r"(taddr));
-  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
-#pragma unroll
-  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-}
 
 // ------------------------------------------------------------------ activation split
 
@@ -219,9 +164,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
-  tc_fence_before();
+  tmem_fence_before();
   __syncthreads();
-  tc_fence_after();
+  tmem_fence_after();
   const uint32_t tmem = *tmem_slot;
   pdl_wait();
 
@@ -259,7 +204,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = tc_idesc(kTcM, kTcN);
+      constexpr uint32_t idesc = umma_idesc_bf16(kTcM, kTcN);
       int g = 0, it = 0;
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
         const int b = it & 1;
@@ -268,7 +213,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           *reinterpret_cast<volatile int*>(abort_flag) = 1;
           break;
         }
-        tc_fence_after();
+        tmem_fence_after();
         const uint32_t d = tmem + b * kTcN;
         bool ok = true;
         for (int ks = 0; ks < p.k_steps; ++ks, ++g) {
@@ -279,20 +224,20 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             ok = false;
             break;
           }
-          tc_fence_after();
+          tmem_fence_after();
           const uint32_t sa = smem_u32(smem + s * kTcStage);
-          const uint64_t ahi = tc_smem_desc(sa), alo = tc_smem_desc(sa + kTcATile),
-                         bw = tc_smem_desc(sa + 2 * kTcATile);
+          const uint64_t ahi = umma_desc_sw128(sa), alo = umma_desc_sw128(sa + kTcATile),
+                         bw = umma_desc_sw128(sa + 2 * kTcATile);
 #pragma unroll
           for (int kk = 0; kk < kTcK / 16; ++kk) {
             // +32 bytes per 16-element K slice inside the 128-byte swizzled row
-            tc_mma(d, ahi + 2 * kk, bw + 2 * kk, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
-            tc_mma(d, alo + 2 * kk, bw + 2 * kk, idesc, 1u);
+            umma_f16(d, ahi + 2 * kk, bw + 2 * kk, idesc, (ks > 0 || kk > 0) ? 1u : 0u);
+            umma_f16(d, alo + 2 * kk, bw + 2 * kk, idesc, 1u);
           }
-          tc_commit(&empty[s]);  // stage s is free once these MMAs have read it
+          umma_commit(&empty[s]);  // stage s is free once these MMAs have read it
         }
         if (!ok) break;
-        tc_commit(&tfull[b]);    // accumulator b is complete
+        umma_commit(&tfull[b]);    // accumulator b is complete
       }
     }
   } else {
@@ -306,22 +251,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         set_error(p.st, DERR_TIMEOUT);
         break;
       }
-      tc_fence_after();
+      tmem_fence_after();
       float acc[kTcN];
       const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + b * kTcN;
 #pragma unroll
-      for (int c = 0; c < kTcN / 32; ++c) tc_ld32(base + c * 32, acc + c * 32);
-      tc_fence_before();
+      for (int c = 0; c < kTcN / 32; ++c) tmem_ld32(base + c * 32, acc + c * 32);
+      tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[b]);  // accumulator b may be overwritten
       const int r = m_t * kTcM + q * 32 + lane;
       if (r < p.M) tc_epilogue_row<EPI>(p, n_t, r, acc);
     }
   }
-  tc_fence_before();
+  tmem_fence_before();
   __syncthreads();
   if (warp == 1) {
-    tc_fence_after();
+    tmem_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
   }
 }
