@@ -114,6 +114,8 @@ struct ssd_ctx {
   Site in1, in2, head;
   // prefill (tcgen05) state
   std::vector<TcLayer> tc_layers;
+  std::vector<TcLayer> enc_tc_layers;  // encoder-decoder model: the encoder's layers
+  std::vector<TcSite> cross_kv_tc;     // and every decoder layer's [ck; cv]
   CUtensorMap a_maps[3][2];  // activation splits (hi, lo) for K = d_model, n_heads*head_dim, d_ff
   __nv_bfloat16 *a_hi = nullptr, *a_lo = nullptr;
   float *x_pre = nullptr, *q_pre = nullptr, *o_pre = nullptr, *h_pre = nullptr;
@@ -311,6 +313,37 @@ static ssd_status make_pair_site(ssd_ctx* c, Site* s, const void* gate, const vo
   s->n_kt = (K + kTileK - 1) / kTileK;
   s->units = s->n_rt * s->n_kt;
   s->grid = s->units < c->num_sms * kGemvCtasPerSm ? s->units : c->num_sms * kGemvCtasPerSm;
+  return SSD_OK;
+}
+
+// One decoder (or encoder) layer's projections for the prefill GEMM: 128-row boxes (2 x 64 rows for
+// the gate/up pair) of 64 columns.
+static ssd_status make_tc_layer(ssd_ctx* c, TcLayer* t, const void* const qkv[3], const void* wo, const void* wg,
+                                const void* wu, const void* wd, int qdim, int d_model, int d_ff) {
+  for (int i = 0; i < 3; ++i) CKS(encode_map_sw128(c, &t->qkv.maps[i], qkv[i], qdim, d_model, kTcN));
+  t->qkv.N = 3 * qdim;
+  t->qkv.K = d_model;
+  t->qkv.seg_rows = qdim;
+  t->qkv.tiles_n = 3 * qdim / kTcN;
+  CKS(encode_map_sw128(c, &t->o.maps[0], wo, d_model, qdim, kTcN));
+  t->o.maps[1] = t->o.maps[2] = t->o.maps[0];
+  t->o.N = d_model;
+  t->o.K = qdim;
+  t->o.seg_rows = d_model;
+  t->o.tiles_n = (d_model + kTcN - 1) / kTcN;
+  CKS(encode_map_sw128(c, &t->gateup.maps[0], wg, d_ff, d_model, kTcN / 2));
+  CKS(encode_map_sw128(c, &t->gateup.maps[1], wu, d_ff, d_model, kTcN / 2));
+  t->gateup.maps[2] = t->gateup.maps[0];
+  t->gateup.N = d_ff;
+  t->gateup.K = d_model;
+  t->gateup.seg_rows = d_ff;
+  t->gateup.tiles_n = (d_ff + kTcN / 2 - 1) / (kTcN / 2);
+  CKS(encode_map_sw128(c, &t->down.maps[0], wd, d_model, d_ff, kTcN));
+  t->down.maps[1] = t->down.maps[2] = t->down.maps[0];
+  t->down.N = d_model;
+  t->down.K = d_ff;
+  t->down.seg_rows = d_model;
+  t->down.tiles_n = (d_model + kTcN - 1) / kTcN;
   return SSD_OK;
 }
 
@@ -834,6 +867,94 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
   return SSD_OK;
 }
 
+// Prefill of the encoder-decoder model through the tensor-core GEMM (the same steps as
+// enqueue_prefill_t5): each encoder projection runs once over all P rows -- activation split,
+// tcgen05 GEMM with the fused epilogue (q/k/v without rotation into the encoder's K/V, scaled
+// residual adds, gated GELU) -- the bidirectional attention with the encoder's relative-position
+// bias in 16-row launches, then every decoder layer's cross K/V from one split of the encoder's
+// normed output, and the decoder on start_token.
+static ssd_status enqueue_prefill_t5_tc(ssd_ctx* c, int n_vis, int n_prompt) {
+  const int P = n_vis + n_prompt, dp = c->dp, qp = c->qp;
+  int* full_tok = st_field(c, offsetof(DevState, full_tok));
+  CK(cudaMemsetAsync(c->counters, 0, sizeof(unsigned) * c->n_counters, c->cs));
+  CK(cudaMemsetAsync(c->attn_tickets, 0, sizeof(unsigned) * c->max_batch * c->cfg.n_heads, c->cs));
+  CK(launch_k(c, ssd_prefill_begin_kernel, dim3(1), dim3(32), 0, c->st, 1, c->cfg.eos_id, P));
+  CK(launch_k(c, ssd_prefill_rows_kernel, dim3(P), dim3(256), 0, static_cast<const __nv_bfloat16*>(c->in_vis),
+              static_cast<const int*>(c->in_prompt), n_vis, 0, c->embed, c->cfg.vocab, c->x_enc, dp, c->cfg.d_model,
+              c->st));
+  for (int e = 0; e < c->cfg.n_enc_layers; ++e) {
+    const TcLayer& tl = c->enc_tc_layers[e];
+    TcParams p{};
+    p.pos0 = 0;
+    p.q_out = c->enc_q;
+    p.q_stride = qp;
+    p.k_cache = c->enc_k;
+    p.v_cache = c->enc_v;
+    p.head_dim = c->cfg.head_dim;
+    p.max_seq = c->max_enc;
+    CKS(split(c, c->x_enc, dp, c->cfg.d_model, c->enc_attn_norm[e], P));
+    CKS(tc_gemm(c, Epi::QKV, 0, tl.qkv, P, p));
+    for (int r0 = 0; r0 < P; r0 += kAttnMaxRows) {
+      const int Mc = std::min(kAttnMaxRows, P - r0);
+      AttnParams a{};
+      a.q = c->enc_q + static_cast<size_t>(r0) * qp;
+      a.q_stride = qp;
+      a.k_cache = c->enc_k;
+      a.v_cache = c->enc_v;
+      a.o = c->enc_o + static_cast<size_t>(r0) * qp;
+      a.o_stride = qp;
+      a.pos_off = r0;
+      a.abs_pos = 1;
+      a.fixed_keys = 1;
+      a.max_seq = c->max_enc;
+      a.scale = 1.0f;
+      a.bias = c->enc_bias;
+      a.bias_stride = 2 * c->max_enc - 1;
+      a.bias_zero = c->max_enc - 1;
+      CKS(attn_run(c, Mc, a));
+    }
+    CKS(split(c, c->enc_o, qp, c->qdim, nullptr, P));
+    p = TcParams{};
+    p.base = c->x_enc;
+    p.base_stride = dp;
+    p.dst = c->x_enc;
+    p.dst_stride = dp;
+    p.scale = c->one;
+    CKS(tc_gemm(c, Epi::RESID, 1, tl.o, P, p));
+    CKS(split(c, c->x_enc, dp, c->cfg.d_model, c->enc_ffn_norm[e], P));
+    p = TcParams{};
+    p.h_out = c->h_pre;
+    p.h_stride = c->fp;
+    p.act = 1;
+    CKS(tc_gemm(c, Epi::GATE_SILU, 0, tl.gateup, P, p));
+    CKS(split(c, c->h_pre, c->fp, c->cfg.d_ff, nullptr, P));
+    p = TcParams{};
+    p.base = c->x_enc;
+    p.base_stride = dp;
+    p.dst = c->x_enc;
+    p.dst_stride = dp;
+    p.scale = c->one;
+    CKS(tc_gemm(c, Epi::RESID, 2, tl.down, P, p));
+  }
+  CKS(split(c, c->x_enc, dp, c->cfg.d_model, c->enc_final, P));  // cross K/V read the encoder's normed output
+  for (int l = 0; l < c->cfg.n_layers; ++l) {
+    TcParams p{};
+    p.pos0 = 0;
+    p.seg_base = 1;  // the [ck; cv] site's segments are k and v
+    p.k_cache = c->ckc + l * c->cross_layer_kv;
+    p.v_cache = c->cvc + l * c->cross_layer_kv;
+    p.head_dim = c->cfg.head_dim;
+    p.max_seq = c->max_enc;
+    CKS(tc_gemm(c, Epi::QKV, 0, c->cross_kv_tc[l], P, p));
+  }
+  CK(launch_k(c, ssd_embed_kernel, dim3(1), dim3(256), 0, c->embed, static_cast<const int*>(c->start_tok), c->xv, dp,
+              c->cfg.d_model, c->cfg.vocab, c->st));
+  for (int l = 0; l < c->cfg.n_layers; ++l) CKS(enqueue_layer(c, l, 0, 1, 0));
+  CKS(enqueue_head(c, c->xv, 1, 0, full_tok, true));
+  CK(launch_k(c, ssd_prefill_finish_kernel, dim3(1), dim3(32), 0, c->st, c->out_int, 1));
+  return SSD_OK;
+}
+
 // ------------------------------------------------------------------ batched requests
 // The serving form of Algorithm 1: B requests, each with its own prompt, positions, cache slot
 // and accept lengths, decode in lockstep.  Request b's row i (i = 0..g) of a step lives in row
@@ -1267,7 +1388,7 @@ static ssd_status build_dyn_graph(ssd_ctx* c, int cap, cudaGraphExec_t* exec) {
 }
 
 static ssd_status enq_prefill_fn(ssd_ctx* c, int a, int b) {
-  if (c->t5) return enqueue_prefill_t5(c, a, b);
+  if (c->t5) return c->prefill_rows ? enqueue_prefill_t5(c, a, b) : enqueue_prefill_t5_tc(c, a, b);
   return c->prefill_rows ? enqueue_prefill(c, a, b) : enqueue_prefill_tc(c, a, b);
 }
 static ssd_status enqueue_prefill_any(ssd_ctx* c, int n_vis, int n_prompt) { return enq_prefill_fn(c, n_vis, n_prompt); }
@@ -1569,32 +1690,27 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   }
   c->tc_layers.resize(n_blocks);
   for (int l = 0; l < n_blocks; ++l) {
-    TcLayer& t = c->tc_layers[l];
     const void* qkv[3] = {wt(l, 0), wt(l, 1), wt(l, 2)};
-    for (int i = 0; i < 3; ++i) CKS(encode_map_sw128(c, &t.qkv.maps[i], qkv[i], qdim, k.d_model, kTcN));
-    t.qkv.N = 3 * qdim;
-    t.qkv.K = k.d_model;
-    t.qkv.seg_rows = qdim;
-    t.qkv.tiles_n = 3 * qdim / kTcN;
-    CKS(encode_map_sw128(c, &t.o.maps[0], wt(l, 3), k.d_model, qdim, kTcN));
-    t.o.maps[1] = t.o.maps[2] = t.o.maps[0];
-    t.o.N = k.d_model;
-    t.o.K = qdim;
-    t.o.seg_rows = k.d_model;
-    t.o.tiles_n = (k.d_model + kTcN - 1) / kTcN;
-    CKS(encode_map_sw128(c, &t.gateup.maps[0], wt(l, 4), k.d_ff, k.d_model, kTcN / 2));
-    CKS(encode_map_sw128(c, &t.gateup.maps[1], wt(l, 5), k.d_ff, k.d_model, kTcN / 2));
-    t.gateup.maps[2] = t.gateup.maps[0];
-    t.gateup.N = k.d_ff;
-    t.gateup.K = k.d_model;
-    t.gateup.seg_rows = k.d_ff;
-    t.gateup.tiles_n = (k.d_ff + kTcN / 2 - 1) / (kTcN / 2);
-    CKS(encode_map_sw128(c, &t.down.maps[0], wt(l, 6), k.d_model, k.d_ff, kTcN));
-    t.down.maps[1] = t.down.maps[2] = t.down.maps[0];
-    t.down.N = k.d_model;
-    t.down.K = k.d_ff;
-    t.down.seg_rows = k.d_model;
-    t.down.tiles_n = (k.d_model + kTcN - 1) / kTcN;
+    CKS(make_tc_layer(c, &c->tc_layers[l], qkv, wt(l, 3), wt(l, 4), wt(l, 5), wt(l, 6), qdim, k.d_model, k.d_ff));
+  }
+  if (t5) {  // the encoder's projections and every decoder layer's [ck; cv] for the prefill GEMM
+    c->enc_tc_layers.resize(k.n_enc_layers);
+    for (int e = 0; e < k.n_enc_layers; ++e) {
+      const void* qkv[3] = {ed->enc_wq[e], ed->enc_wk[e], ed->enc_wv[e]};
+      CKS(make_tc_layer(c, &c->enc_tc_layers[e], qkv, ed->enc_wo[e], ed->enc_wi0[e], ed->enc_wi1[e], ed->enc_wff[e],
+                        qdim, k.d_model, k.d_ff));
+    }
+    c->cross_kv_tc.resize(k.n_layers);
+    for (int l = 0; l < k.n_layers; ++l) {
+      TcSite& t = c->cross_kv_tc[l];
+      CKS(encode_map_sw128(c, &t.maps[0], ed->ck[l], qdim, k.d_model, kTcN));
+      CKS(encode_map_sw128(c, &t.maps[1], ed->cv[l], qdim, k.d_model, kTcN));
+      t.maps[2] = t.maps[0];
+      t.N = 2 * qdim;
+      t.K = k.d_model;
+      t.seg_rows = qdim;
+      t.tiles_n = 2 * qdim / kTcN;
+    }
   }
 
   // owned memory (activation rows: one request's passes, or every request's verification rows)
@@ -1703,7 +1819,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   const size_t in_rows = std::max(static_cast<size_t>(k.max_seq), static_cast<size_t>(c->max_enc));
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_vis), sizeof(__nv_bfloat16) * in_rows * d));
   {
-    const size_t Pm = k.max_seq;
+    const size_t Pm = std::max(k.max_seq, c->max_enc);
     const size_t kmax = std::max(std::max(static_cast<size_t>(k.d_model), static_cast<size_t>(qdim)),
                                  static_cast<size_t>(k.d_ff));
     CKS(alloc(c, reinterpret_cast<void**>(&c->a_hi), sizeof(__nv_bfloat16) * Pm * kmax));

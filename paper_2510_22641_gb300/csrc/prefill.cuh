@@ -79,7 +79,7 @@ __device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int 
   // acc: the 128 fp32 outputs of token row r in output tile n_t (columns of the tile)
   const int pos = p.pos0 + r;
   if constexpr (EPI == Epi::QKV) {
-    const int c0 = n_t * kTcN, mat = c0 / p.seg_rows, local0 = c0 - mat * p.seg_rows;
+    const int c0 = n_t * kTcN, seg = c0 / p.seg_rows, mat = seg + p.seg_base, local0 = c0 - seg * p.seg_rows;
     const int Dh = p.head_dim, half = Dh >> 1;
     if (pos < 0 || pos >= p.max_seq) {
       set_error(p.st, DERR_POS);
@@ -92,9 +92,12 @@ __device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int 
         float* qr = mat == 0 ? p.q_out + static_cast<size_t>(r) * p.q_stride + h * Dh : nullptr;
         for (int j = 0; j < half; ++j) {
           const float a = acc[hh * Dh + j], b = acc[hh * Dh + j + half];
-          const float2 cs = p.rope_cs[static_cast<size_t>(pos) * half + j];
-          const float va = a * cs.x - b * cs.y;
-          const float vb = a * cs.y + b * cs.x;
+          float va = a, vb = b;
+          if (p.rope_cs) {
+            const float2 cs = p.rope_cs[static_cast<size_t>(pos) * half + j];
+            va = a * cs.x - b * cs.y;
+            vb = a * cs.y + b * cs.x;
+          }
           if (mat == 0) {
             qr[j] = va;
             qr[j + half] = vb;
@@ -114,7 +117,7 @@ __device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int 
     float* hr = p.h_out + static_cast<size_t>(r) * p.h_stride + n_t * (kTcN / 2);
     for (int j = 0; j < kTcN / 2; ++j) {
       if (n_t * (kTcN / 2) + j >= p.N) break;
-      hr[j] = silu_f(acc[j]) * acc[kTcN / 2 + j];
+      hr[j] = (p.act ? gelu_tanh_f(acc[j]) : silu_f(acc[j])) * acc[kTcN / 2 + j];
     }
   } else {  // RESID
     const float s = __ldg(p.scale);

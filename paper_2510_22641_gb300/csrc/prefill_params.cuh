@@ -21,6 +21,7 @@ struct TcParams {
   int M, N, K;          // rows (tokens), output columns, reduction
   int tiles_m, tiles_n, k_steps;
   int seg_rows;         // QKV: rows per source matrix
+  int seg_base;         // QKV: segment of the site's first matrix (0 = q; 1 = k, for a [k; v] site)
   int pos0;             // position of row 0
   DevState* st;
   // epilogues (same meaning as GemvParams)
@@ -29,9 +30,10 @@ struct TcParams {
   float* k_cache;
   float* v_cache;
   int head_dim, max_seq;
-  const float2* rope_cs;
+  const float2* rope_cs;  // null: no rotation (the encoder-decoder model)
   float* h_out;
   int h_stride;
+  int act;                // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up
   const float* base;
   int base_stride;
   float* dst;

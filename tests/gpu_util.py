@@ -55,11 +55,12 @@ def t5_device_weights(bits: dict) -> dict:
 
 
 def make_t5_model(w: synth.T5Workload, bits: dict | None = None, dev: dict | None = None,
-                  gamma_max: int | None = None, max_seq: int | None = None, max_enc: int | None = None):
+                  gamma_max: int | None = None, max_seq: int | None = None, max_enc: int | None = None,
+                  options: int = 0):
     bits = bits if bits is not None else synth.make_t5_weights(w)
     dev = dev if dev is not None else t5_device_weights(bits)
     cfg = lib.t5_config_dict(w.shape, w.draft_exit_k, w.in_kind, w.in_hidden, gamma_max or max(w.gamma, 1),
-                             max_seq or (w.max_dec() + 1), max_enc or w.enc_len, w.eos_id)
+                             max_seq or (w.max_dec() + 1), max_enc or w.enc_len, w.eos_id, options=options)
     rs = torch.tensor(w.dec_scale(), dtype=torch.float32, device="cuda")
     ins = torch.tensor([w.in_scale()], dtype=torch.float32, device="cuda")
     return lib.SSDModel(cfg, dev, rs, ins), bits, dev

@@ -1,9 +1,11 @@
 """Encoder-decoder (BLIP-2 FlanT5-shaped) CUDA path vs the fp64 encoder-decoder oracle, through the C ABI.
 
-Tiny workload: 2 encoder + 4 decoder layers, d=256, 4 heads x 64, V=2048.  The default 48 encoder
-rows give 6 prefill chunks of 8 rows; a long case (130 encoder rows, 150 new tokens) spans three
-64-key attention chunks on both the encoder and the decoder side, a ragged last prefill chunk
-(130 = 16 x 8 + 2) and relative offsets beyond max_distance / 2 in both bucket schemes.  The
+Tiny workload: 2 encoder + 4 decoder layers, d=256, 4 heads x 64, V=2048.  The encoder runs through
+the tensor-core prefill GEMM (one 128-row tile for the default 48 encoder rows); a long case (130
+encoder rows, 150 new tokens) spans two row tiles (the second holds 2 rows), three 64-key attention
+chunks on both the encoder and the decoder side, and relative offsets beyond max_distance / 2 in
+both bucket schemes.  The row prefill (the decode kernels in 8-row chunks) is checked against the
+tensor-core one and the oracle.  The
 FlanT5-xl-shaped case (24 + 24 layers, d=2048, V=32128) compares the oracle's prefill and first SSD
 steps with the GPU's and checks SSD == greedy over all 30 tokens.
 """
@@ -103,6 +105,28 @@ def test_t5_ssd_matches_oracle_and_gpu_greedy(tiny_model, tiny_bits, s, gamma):
     assert toks == gtoks  # batch invariance: the verify rows reproduce greedy decoding bitwise
     np.testing.assert_array_equal(logits, glogits)
     assert st["steps"] + st["accepted"] + 1 == w.max_new
+
+
+def test_t5_tensor_core_prefill_matches_row_prefill(tiny_model, tiny_bits):
+    """The encoder through the tcgen05 prefill GEMM and through the decode kernels in 8-row chunks
+    give the same greedy stream within the oracle's tolerance; both match the oracle."""
+    w = tiny(s=0.3, n_query=100, n_prompt=30, max_new=40)
+    set_s(tiny_model, w)
+    toks, logits, st = gpu_decode(tiny_model, w, 0)
+    rows_model, _, _ = make_t5_model(w, tiny_bits, gamma_max=GAMMA_MAX, max_seq=200, max_enc=160,
+                                     options=lib.SSD_OPT_PREFILL_ROWS)
+    try:
+        set_s(rows_model, w)
+        rtoks, rlogits, _ = gpu_decode(rows_model, w, 0)
+    finally:
+        rows_model.close()
+    ref = oracle_run(w, tiny_bits, 0)
+    agree = check(toks, logits, st, ref, 0)
+    assert agree >= 16
+    ragree = common_prefix(rtoks, ref.tokens, ref.logits)
+    assert ragree >= 16
+    for t in range(min(agree + 1, ragree + 1, w.max_new)):
+        assert_logits_close(logits[t], rlogits[t], f"tensor-core vs row prefill, logits of token {t}")
 
 
 def test_t5_long_encoder_and_decoder(tiny_model, tiny_bits):
