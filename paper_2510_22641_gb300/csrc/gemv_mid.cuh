@@ -31,7 +31,10 @@
 //    tail as long as the stream itself).
 // The per-element arithmetic is the GEMV's: a = hi + lo, 4 K slices x (hi, lo)
 // MMAs per unit accumulating in fp32, the RMSNorm scale applied after the
-// products, and the split-tile sums in CTA order.
+// products, and the split-tile sums in CTA order.  The grid is its own (one CTA
+// per SM), so the split points differ from the GEMV's: a row through this kernel
+// equals the same row through the GEMV up to rounding, and every row is still
+// independent of the launch's other rows.
 #pragma once
 
 #include "gemv.cuh"
