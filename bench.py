@@ -45,8 +45,8 @@ import synth  # noqa: E402
 METRIC = "tokens/s and speedup vs full-model greedy decode (7B shape, bs1); HBM GB/s"
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one gate/up GEMV
-# launch from an ncu capture, valid only for the kernel source it was taken on.
-GEMV_TRAFFIC = {"gemv_cuh_sha256_prefix": "d5bddf15d880f543", "bytes": 183_015_168}
+# launch from an ncu capture, valid only for the kernel sources it was taken on.
+GEMV_TRAFFIC = {"gemv_sources_sha256_prefix": "6d1ad7b9f4622fc1", "bytes": 183_197_696}
 UNIT = "tokens/s"
 S_VALUES = synth.LLAVA7B_S_VALUES
 
@@ -133,14 +133,16 @@ def kernel_table(model, w, v, p, stream, hbm_peak, reps=50, rows_table=KERNEL_RO
 
 
 def gemv_traffic_bytes():
-    """Measured bytes per launch if gemv.cuh is the captured version, else None."""
+    """Measured bytes per launch if the GEMV's sources (gemv.cuh, tcgen05.cuh, common.cuh) are the
+    captured version, else None."""
     import hashlib
-    src = os.path.join(ROOT, "paper_2510_22641_gb300", "csrc", "gemv.cuh")
+    h = hashlib.sha256()
     try:
-        digest = hashlib.sha256(open(src, "rb").read()).hexdigest()
+        for name in ("gemv.cuh", "tcgen05.cuh", "common.cuh"):
+            h.update(open(os.path.join(ROOT, "paper_2510_22641_gb300", "csrc", name), "rb").read())
     except OSError:
         return None
-    return GEMV_TRAFFIC["bytes"] if digest.startswith(GEMV_TRAFFIC["gemv_cuh_sha256_prefix"]) else None
+    return GEMV_TRAFFIC["bytes"] if h.hexdigest().startswith(GEMV_TRAFFIC["gemv_sources_sha256_prefix"]) else None
 
 
 def prefill_flops(w: synth.Workload) -> float:
