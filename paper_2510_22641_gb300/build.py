@@ -16,7 +16,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libssd.so")
-SOURCES = ["engine.cu", "gemv_qkv.cu", "gemv_gate.cu", "gemv_silu.cu", "gemv_resid.cu", "gemv_head.cu", "gemv_mid.cu", "attention.cu",
+SOURCES = ["engine.cu", "gemv_qkv.cu", "gemv_gate.cu", "gemv_silu.cu", "gemv_resid.cu", "gemv_head.cu", "gemv_xattn.cu", "gemv_mid.cu", "attention.cu",
            "static_head.cu", "prefill.cu"]
 FLAGS = ["-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-lineinfo", "-std=c++17",
          "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]

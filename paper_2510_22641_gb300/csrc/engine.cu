@@ -32,11 +32,13 @@ cudaError_t gemv_launch_gate(int M, const CUtensorMap*, const GemvParams&, int, 
 cudaError_t gemv_launch_silu(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
 cudaError_t gemv_launch_resid(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
 cudaError_t gemv_launch_head(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
+cudaError_t gemv_launch_xattn(int M, const CUtensorMap*, const GemvParams&, int, cudaStream_t, bool);
 cudaError_t gemv_attrs_qkv();
 cudaError_t gemv_attrs_gate();
 cudaError_t gemv_attrs_silu();
 cudaError_t gemv_attrs_resid();
 cudaError_t gemv_attrs_head();
+cudaError_t gemv_attrs_xattn();
 cudaError_t prefill_attrs();
 cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
                            cudaStream_t s, bool pdl);
@@ -365,6 +367,7 @@ static ssd_status gemv(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
     case Epi::GATE_SILU: r = gemv_launch_gate(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
     case Epi::SILU: r = gemv_launch_silu(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
     case Epi::RESID: r = gemv_launch_resid(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
+    case Epi::XATTN: r = gemv_launch_xattn(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
     default: r = gemv_launch_head(M, s.maps, p, s.grid, c->cs, c->use_pdl); break;
   }
   CK(r);
@@ -483,19 +486,29 @@ static ssd_status enqueue_t5_layer(ssd_ctx* c, int l, float* x, int M, int pos_o
   p.q_stride = c->qp;
   p.head_dim = c->cfg.head_dim;
   p.max_seq = c->cfg.max_seq;
-  CKS(gemv(c, Epi::QKV, M, c->cross_q[l], p));  // a one-matrix site: q only
-  AttnParams a{};
-  a.q = c->qb;
-  a.q_stride = c->qp;
-  a.k_cache = c->ckc + l * c->cross_layer_kv;
-  a.v_cache = c->cvc + l * c->cross_layer_kv;
-  a.o = c->ob;
-  a.o_stride = c->qp;
-  a.pos_off = pos_off;
-  a.max_seq = c->max_enc;
-  a.scale = 1.0f;
-  a.fixed_keys = 1;
-  CKS(attn_run(c, M, a));
+  if (c->max_enc <= kXattnKeys) {  // the cross-attention runs in the cross-q projection's epilogue
+    p.xk = c->ckc + l * c->cross_layer_kv;
+    p.xv = c->cvc + l * c->cross_layer_kv;
+    p.x_max = c->max_enc;
+    p.x_scale = 1.0f;
+    p.xo = c->ob;
+    p.xo_stride = c->qp;
+    CKS(gemv(c, Epi::XATTN, M, c->cross_q[l], p));
+  } else {
+    CKS(gemv(c, Epi::QKV, M, c->cross_q[l], p));  // a one-matrix site: q only
+    AttnParams a{};
+    a.q = c->qb;
+    a.q_stride = c->qp;
+    a.k_cache = c->ckc + l * c->cross_layer_kv;
+    a.v_cache = c->cvc + l * c->cross_layer_kv;
+    a.o = c->ob;
+    a.o_stride = c->qp;
+    a.pos_off = pos_off;
+    a.max_seq = c->max_enc;
+    a.scale = 1.0f;
+    a.fixed_keys = 1;
+    CKS(attn_run(c, M, a));
+  }
   CKS(resid_gemv(c, M, c->cross_o[l], c->ob, c->qp, x, s_l));
   p = GemvParams{};
   p.x = x;
@@ -1624,6 +1637,7 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
   CK(gemv_attrs_silu());
   CK(gemv_attrs_resid());
   CK(gemv_attrs_head());
+  CK(gemv_attrs_xattn());
   CK(attn_attrs());
   CK(prefill_attrs());
   CK(mid_attrs());

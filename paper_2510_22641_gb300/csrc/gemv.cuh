@@ -55,7 +55,7 @@ constexpr int kTmemCols = 32;        // two 16-column accumulators
 constexpr uint32_t kWTileBytes = kTileN * kTileK * 2;   // 16 KB
 constexpr uint32_t kBOpBytes = kNPad * kTileK * 2;      // 2 KB (hi or lo)
 
-enum class Epi : int { QKV = 0, GATE_SILU = 1, SILU = 2, RESID = 3, ARGMAX = 4 };
+enum class Epi : int { QKV = 0, GATE_SILU = 1, SILU = 2, RESID = 3, ARGMAX = 4, XATTN = 5 };
 
 struct GemvParams {
   int K, n_kt, n_rt, units;
@@ -115,7 +115,19 @@ struct GemvParams {
   int grid_ctas;  // medium-M reduction: the CTAs of the streaming launch
   int abs_pos;   // row m sits at position pos_off + m, st->kv_len ignored (the encoder's rows)
   int act;       // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up (gated GELU)
+  // XATTN (a q-only site: the encoder-decoder model's cross-attention query): instead of writing
+  // q, the tile's owner attends with it over the st->enc_len <= kXattnKeys cross keys xk / xv
+  // ([H][x_max][head_dim] fp32, every key visible, scores times x_scale) and writes the attention
+  // output rows to xo (row stride xo_stride).
+  const float* xk;
+  const float* xv;
+  int x_max;
+  float x_scale;
+  float* xo;
+  int xo_stride;
 };
+
+constexpr int kXattnKeys = 128;  // cross keys the folded cross-attention takes
 
 template <int M>
 struct GemvSmem {
@@ -168,11 +180,94 @@ __device__ __forceinline__ int batch_offset(const GemvParams& p, int mg, int b) 
   return p.pos_off + mg - b * p.batch_rows;
 }
 
+// Cross-attention folded into the cross-q projection's epilogue (see GemvParams::xk): for the
+// tile's heads (128 / head_dim of them) and rows m0 .. m0 + mc - 1, with q = out * rs,
+//   s_j = x_scale * q . K_j,  p_j = exp(s_j - max_j s),  o = (sum_j p_j V_j) / (sum_j p_j),
+// keys in order, each row on its own (the result does not depend on the launch's other rows).
+template <int MT>
+__device__ __forceinline__ void gemv_cross_attention(const GemvParams& p, int rt, const float* out, const float* rs,
+                                                     int tid, int m0, int mc) {
+  __shared__ float xs[kNPad * 2 * kXattnKeys];  // [row][head of the tile][key] scores, then exponentials
+  __shared__ float xl[kNPad * 2];               // [row][head] sums
+  const int Dh = p.head_dim, hpt = kTileN / Dh, h0 = (rt * kTileN) / Dh;
+  const int nk = min(__ldcg(&p.st->enc_len), kXattnKeys);
+  // 1. scores: one (head, key) item per thread, its key row read once for all rows
+  for (int it = tid; it < hpt * nk; it += kDrainThreads) {
+    const int hh = it / nk, j = it - hh * nk;
+    const float4* kr = reinterpret_cast<const float4*>(p.xk + (static_cast<size_t>(h0 + hh) * p.x_max + j) * Dh);
+    float a[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) a[m] = 0.f;
+    for (int d4 = 0; d4 < (Dh >> 2); ++d4) {
+      const float4 k4 = __ldg(kr + d4);
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m >= mc) break;
+        const float* q = out + m * kTileN + hh * Dh + 4 * d4;
+        a[m] = fmaf(q[0], k4.x, a[m]);
+        a[m] = fmaf(q[1], k4.y, a[m]);
+        a[m] = fmaf(q[2], k4.z, a[m]);
+        a[m] = fmaf(q[3], k4.w, a[m]);
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      if (m >= mc) break;
+      xs[(m * 2 + hh) * kXattnKeys + j] = (a[m] * rs[m]) * p.x_scale;
+    }
+  }
+  drain_sync();
+  // 2. per (row, head), one warp: max, exponentials in place, their sum
+  const int lane = tid & 31, w = tid >> 5;
+  for (int r = w; r < mc * hpt; r += kDrainThreads / 32) {
+    const int m = r / hpt, hh = r - m * hpt;
+    float* sr = xs + (m * 2 + hh) * kXattnKeys;
+    float mx = -INFINITY;
+    for (int j = lane; j < nk; j += 32) mx = fmaxf(mx, sr[j]);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    float sum = 0.f;
+    for (int j = lane; j < nk; j += 32) {
+      const float e = expf(sr[j] - mx);
+      sr[j] = e;
+      sum += e;
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+    if (lane == 0) xl[m * 2 + hh] = sum;
+  }
+  drain_sync();
+  // 3. P.V: one (head, dimension) item per thread, the keys in order
+  for (int it = tid; it < hpt * Dh; it += kDrainThreads) {
+    const int hh = it / Dh, d = it - hh * Dh;
+    const float* vc = p.xv + static_cast<size_t>(h0 + hh) * p.x_max * Dh + d;
+    float o[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) o[m] = 0.f;
+    for (int j = 0; j < nk; ++j) {
+      const float v = __ldg(vc + static_cast<size_t>(j) * Dh);
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        if (m >= mc) break;
+        o[m] = fmaf(xs[(m * 2 + hh) * kXattnKeys + j], v, o[m]);
+      }
+    }
+#pragma unroll
+    for (int m = 0; m < MT; ++m) {
+      if (m >= mc) break;
+      const float L = xl[m * 2 + hh];
+      p.xo[(m0 + m) * p.xo_stride + (h0 + hh) * Dh + d] = L > 0.f ? o[m] / L : 0.f;
+    }
+  }
+}
+
 template <int MT, Epi EPI>
 __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const float* out, const float* rs,
                                               const float* pre, int base_pos, const int* rpos, const int* rreq,
                                               int tid, int m0, int mc) {
-  if constexpr (EPI == Epi::QKV) {
+  if constexpr (EPI == Epi::XATTN) {
+    gemv_cross_attention<MT>(p, rt, out, rs, tid, m0, mc);
+  } else if constexpr (EPI == Epi::QKV) {
     const int r0 = rt * kTileN;
     const int seg = r0 / p.seg_rows;       // source matrix of this row tile within the site
     const int mat = seg + p.seg_base;      // 0 = q, 1 = k, 2 = v

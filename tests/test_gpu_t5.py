@@ -5,7 +5,8 @@ the tensor-core prefill GEMM (one 128-row tile for the default 48 encoder rows);
 encoder rows, 150 new tokens) spans two row tiles (the second holds 2 rows), three 64-key attention
 chunks on both the encoder and the decoder side, and relative offsets beyond max_distance / 2 in
 both bucket schemes.  The row prefill (the decode kernels in 8-row chunks) is checked against the
-tensor-core one and the oracle.  The
+tensor-core one and the oracle, and a model with max_enc = 64 runs the cross-attention folded into
+the cross-q projection's epilogue (the fixture's max_enc = 160 keeps the separate kernel).  The
 FlanT5-xl-shaped case (24 + 24 layers, d=2048, V=32128) compares the oracle's prefill and first SSD
 steps with the GPU's and checks SSD == greedy over all 30 tokens.
 """
@@ -127,6 +128,30 @@ def test_t5_tensor_core_prefill_matches_row_prefill(tiny_model, tiny_bits):
     assert ragree >= 16
     for t in range(min(agree + 1, ragree + 1, w.max_new)):
         assert_logits_close(logits[t], rlogits[t], f"tensor-core vs row prefill, logits of token {t}")
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.3, 3)])
+def test_t5_folded_cross_attention(tiny_model, tiny_bits, s, gamma):
+    """With max_enc <= 128 the cross-attention runs in the cross-q projection's epilogue: greedy and
+    SSD against the oracle, SSD == greedy bitwise, logits within tolerance of the separate
+    cross-attention kernel's (the fixture's max_enc = 160 keeps that path)."""
+    w = tiny(s=s)
+    fold, _, _ = make_t5_model(w, tiny_bits, gamma_max=GAMMA_MAX, max_seq=200, max_enc=64)
+    try:
+        set_s(fold, w)
+        gtoks, glogits, gst = gpu_decode(fold, w, 0)
+        toks, logits, st = gpu_decode(fold, w, gamma)
+    finally:
+        fold.close()
+    assert check(gtoks, glogits, gst, oracle_run(w, tiny_bits, 0), 0) >= 8
+    check(toks, logits, st, oracle_run(w, tiny_bits, gamma), gamma)
+    assert toks == gtoks
+    np.testing.assert_array_equal(logits, glogits)
+    set_s(tiny_model, w)
+    ktoks, klogits, _ = gpu_decode(tiny_model, w, 0)
+    n = common_prefix(gtoks, ktoks, klogits)
+    for t in range(min(n + 1, w.max_new)):
+        assert_logits_close(glogits[t], klogits[t], f"folded vs separate cross-attention, logits of token {t}")
 
 
 def test_t5_long_encoder_and_decoder(tiny_model, tiny_bits):
