@@ -45,7 +45,7 @@ cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, co
 cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                               __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl);
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
-                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
+                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale, DevState* st,
                                 cudaStream_t s, bool pdl);
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
                        int num_sms, cudaStream_t s, bool pdl);
@@ -851,7 +851,7 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     CK(count_launch(c));
     CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, kv_k(c, l), kv_v(c, l),
                            c->o_pre, c->qp, P, c->cfg.n_heads, c->cfg.max_seq,
-                           1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->cs, c->use_pdl));
+                           1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->st, c->cs, c->use_pdl));
     CKS(split(c, c->o_pre, c->qp, c->qdim, nullptr, P));
     p = TcParams{};
     p.base = c->x_pre;

@@ -29,10 +29,10 @@ cudaError_t prefill_attrs() {
   if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
     return e;
   if ((e = cudaFuncSetAttribute(ssd_prefill_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                PaSmem<128>::kTotal)))
+                                FaSmem<128>::kTotal)))
     return e;
   return cudaFuncSetAttribute(ssd_prefill_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              PaSmem<64>::kTotal);
+                              FaSmem<64>::kTotal);
 }
 
 cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
@@ -56,14 +56,14 @@ cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bf
 }
 
 cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
-                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale,
+                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale, DevState* st,
                                 cudaStream_t s, bool pdl) {
-  const dim3 grid((P + kPaQ - 1) / kPaQ, n_heads);
+  const dim3 grid((P + kFaQ - 1) / kFaQ, n_heads);
   if (head_dim == 128)
-    return launch_pdl(ssd_prefill_attn_kernel<128>, grid, dim3(256), PaSmem<128>::kTotal, s, pdl, q, q_stride, kc, vc,
-                      o, o_stride, P, max_seq, scale);
-  return launch_pdl(ssd_prefill_attn_kernel<64>, grid, dim3(256), PaSmem<64>::kTotal, s, pdl, q, q_stride, kc, vc, o,
-                    o_stride, P, max_seq, scale);
+    return launch_pdl(ssd_prefill_attn_kernel<128>, grid, dim3(kFaThreads), FaSmem<128>::kTotal, s, pdl, q, q_stride,
+                      kc, vc, o, o_stride, P, max_seq, scale, st);
+  return launch_pdl(ssd_prefill_attn_kernel<64>, grid, dim3(kFaThreads), FaSmem<64>::kTotal, s, pdl, q, q_stride, kc,
+                    vc, o, o_stride, P, max_seq, scale, st);
 }
 
 }  // namespace ssd

@@ -279,181 +279,299 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 namespace ssd {
 
 // ------------------------------------------------------------------ causal prefill attention
-// One CTA per (64-query block, head), the blocks with the most key blocks launched
-// first: keys in blocks of 64 up to the query block (causal), brought into shared
-// memory with 16-byte asynchronous copies, double-buffered (block kb + 1 loads while
-// block kb is computed).  Scores 4 rows x 4 keys per thread in fp32 (keys tc, tc + 16,
-// tc + 32, tc + 48: with K rows padded to Dh + 4 floats, the 16-byte K reads of a
-// quarter warp hit 8 different bank groups), online softmax per row (a row's 64
-// scores live on 16 consecutive lanes), O += P V with 4 rows x Dh/16 dims per thread.
-// q: [P][q_stride] rotated queries; K, V: the fp32 cache.
-constexpr int kPaQ = 64;
-constexpr int kPaK = 64;
-constexpr int kPaPad = 68;  // Q^T and P rows: 64 + 4 floats
+// One CTA per (128-query block, head), the blocks with the most key blocks launched first.
+// Both products run on the 5th-generation tensor cores with fp32-class accuracy: every fp32
+// operand x is split into bf16 parts x = hi + lo, and a product a.b is taken as
+// hi(a) hi(b) + hi(a) lo(b) + lo(a) hi(b) in fp32 (the lo lo term is below fp32 rounding).
+//   * Q block (128 rows x Dh) -> bf16 hi / lo, 128-byte swizzled K-major (rows = queries), once;
+//   * per 64-key block (causal: up to the query block): thread 0 bulk-copies the block's fp32 K and
+//     V rows into a staging buffer one block ahead; all threads turn them into bf16 hi / lo K
+//     (rows = keys) and V^T (rows = head dimensions, keys along K);
+//   * S = Q K^T: 3 x Dh/16 tcgen05.mma (M = 128 queries, N = 64 keys) into TMEM columns 0..63;
+//   * warps 0..3, one thread per query row (its TMEM lane): scale, causal mask, online softmax
+//     (running max and sum in registers), P = exp(S - max) -> bf16 hi / lo, 128-byte swizzled
+//     (rows = queries, keys along K);
+//   * O_blk = P V: 3 x 4 tcgen05.mma (M = 128, N = Dh, K = 64 keys) into TMEM columns 64..64+Dh;
+//     the same threads fold it into their row's fp32 output registers, O = O * alpha + O_blk.
+// Every step of a row depends on the keys' positions only; rows are independent.
+// q: [P][q_stride] rotated queries; K, V: the fp32 cache [H][max_seq][Dh]; o: [P][o_stride].
+constexpr int kFaQ = 128;       // query rows per CTA (the MMA's M)
+constexpr int kFaK = 64;        // keys per block (the S MMA's N, the P.V MMA's K)
+constexpr int kFaThreads = 256;
+constexpr int kFaTmemCols = 256;  // S: 64 columns, O block: Dh columns
 
 template <int DH>
-struct PaSmem {
-  static constexpr int kKs = DH + 4;                            // padded K row
-  static constexpr int kQt = 0;                                 // [DH][kPaPad]
-  static constexpr int kK = kQt + DH * kPaPad * 4;              // [2][64][DH + 4]
-  static constexpr int kV = kK + 2 * kPaK * kKs * 4;            // [2][64][DH]
-  static constexpr int kP = kV + 2 * kPaK * DH * 4;             // [64][kPaPad]
-  static constexpr int kTotal = kP + kPaQ * kPaPad * 4;
+struct FaSmem {
+  static constexpr int kNA = DH / 64;                    // 64-column atoms along the head dimension
+  static constexpr int kQAtom = kFaQ * 128;              // one atom of the Q block (hi or lo)
+  static constexpr int kKAtom = kFaK * 128;              // one atom of the K block
+  static constexpr int kQh = 0;                          // [kNA][128 rows][128 B]
+  static constexpr int kQl = kQh + kNA * kQAtom;
+  static constexpr int kKh = kQl + kNA * kQAtom;         // [kNA][64 keys][128 B]
+  static constexpr int kKl = kKh + kNA * kKAtom;
+  static constexpr int kVh = kKl + kNA * kKAtom;         // V^T: [Dh rows][64 keys x 2 B]
+  static constexpr int kVl = kVh + DH * 128;
+  static constexpr int kPh = kVl + DH * 128;             // P: [128 rows][64 keys x 2 B]
+  static constexpr int kPl = kPh + kFaQ * 128;
+  static constexpr int kStK = kPl + kFaQ * 128;          // fp32 staging of one block: K [64][Dh]
+  static constexpr int kStV = kStK + kFaK * DH * 4;      //                            V [64][Dh]
+  static constexpr int kBar = kStV + kFaK * DH * 4;      // staging full, MMA done
+  static constexpr int kTmemSlot = kBar + 16;
+  static constexpr int kTotal = kTmemSlot + 16 + 1024;   // + slack for the 1024-byte alignment
 };
 
+// 8 fp32 values -> bf16 hi and lo parts, packed two per word.
+__device__ __forceinline__ void split8_bf16(const float* v, uint4& hi, uint4& lo) {
+  uint32_t hw[4], lw[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(v[2 * e]), h1 = __float2bfloat16_rn(v[2 * e + 1]);
+    hw[e] = pack_bf16x2(h0, h1);
+    lw[e] = pack_bf16x2(__float2bfloat16_rn(v[2 * e] - __bfloat162float(h0)),
+                        __float2bfloat16_rn(v[2 * e + 1] - __bfloat162float(h1)));
+  }
+  hi = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+  lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
+}
+
+// Byte offset of 16-byte chunk ch of row r in a 128-byte swizzled atom.
+__device__ __forceinline__ int sw128_off(int r, int ch) { return r * 128 + ((ch ^ (r & 7)) << 4); }
+
 template <int DH>
-__global__ void __launch_bounds__(256) ssd_prefill_attn_kernel(const float* __restrict__ q, int q_stride,
-                                                           const float* __restrict__ k_cache,
-                                                           const float* __restrict__ v_cache, float* __restrict__ o,
-                                                           int o_stride, int P, int max_seq, float scale) {
-  using S = PaSmem<DH>;
-  constexpr int DPT = DH / 16;  // output dims per thread
-  constexpr int KS = S::kKs;
-  extern __shared__ __align__(128) uint8_t pa_smem[];
-  float* Qt = reinterpret_cast<float*>(pa_smem + S::kQt);
-  float* Kb = reinterpret_cast<float*>(pa_smem + S::kK);
-  float* Vb = reinterpret_cast<float*>(pa_smem + S::kV);
-  float* Ps = reinterpret_cast<float*>(pa_smem + S::kP);
-  const int nqb = gridDim.x, qb = nqb - 1 - static_cast<int>(blockIdx.x), h = blockIdx.y, tid = threadIdx.x;
-  const int q0 = qb * kPaQ;
-  const int tr = tid >> 4, tc = tid & 15;  // rows 4tr..4tr+3; score keys tc + 16b; output dims tc*DPT..
+__global__ void __launch_bounds__(kFaThreads, 1)
+    ssd_prefill_attn_kernel(const float* __restrict__ q, int q_stride, const float* __restrict__ k_cache,
+                            const float* __restrict__ v_cache, float* __restrict__ o, int o_stride, int P,
+                            int max_seq, float scale, DevState* st) {
+  using S = FaSmem<DH>;
+  extern __shared__ __align__(1024) uint8_t fa_raw[];
+  const uint32_t raw = smem_u32(fa_raw);
+  uint8_t* smem = fa_raw + (((raw + 1023u) & ~1023u) - raw);
+  uint64_t* bar_ld = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  uint64_t* bar_mma = bar_ld + 1;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
+  const float* stk = reinterpret_cast<const float*>(smem + S::kStK);
+  const float* stv = reinterpret_cast<const float*>(smem + S::kStV);
+  const int nqb = gridDim.x, qb = nqb - 1 - static_cast<int>(blockIdx.x), h = blockIdx.y;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int q0 = qb * kFaQ;
+  const int n_keys = min(q0 + kFaQ, P);  // keys 0 .. n_keys - 1 reach some row of the block
+  const int n_kb = (n_keys + kFaK - 1) / kFaK;
   const float* kh = k_cache + static_cast<size_t>(h) * max_seq * DH;
   const float* vh = v_cache + static_cast<size_t>(h) * max_seq * DH;
-  const int n_kb = min(qb + 1, (P + kPaK - 1) / kPaK);
-  // key block kb -> buffer kb & 1; rows at or past P are zero-filled (nothing read)
-  auto issue = [&](int kb) {
-    const int j0 = kb * kPaK;
-    float* kd = Kb + (kb & 1) * kPaK * KS;
-    float* vd = Vb + (kb & 1) * kPaK * DH;
-    for (int c = tid; c < kPaK * (DH / 4); c += 256) {
-      const int j = c / (DH / 4), d4 = (c - j * (DH / 4)) * 4;
-      const bool in = j0 + j < P;
-      const size_t off = in ? static_cast<size_t>(j0 + j) * DH + d4 : 0;
-      cp_async16_fill(kd + j * KS + d4, kh + off, in ? 16u : 0u);
-      cp_async16_fill(vd + j * DH + d4, vh + off, in ? 16u : 0u);
-    }
-    cp_async_commit();
-  };
-  pdl_trigger();
-  pdl_wait();
-  issue(0);
-  if (n_kb > 1) issue(1);
-  else cp_async_commit();  // keep one group per block for the waits below
 
-  // Q block, transposed: Qt[d][i] = q[q0 + i][h*DH + d] (rows past P read as 0)
-  for (int idx = tid; idx < kPaQ * DH; idx += 256) {
-    const int i = idx / DH, d = idx - i * DH;
-    Qt[d * kPaPad + i] = (q0 + i < P) ? __ldcg(q + static_cast<size_t>(q0 + i) * q_stride + h * DH + d) : 0.f;
+  pdl_trigger();
+  if (tid == 0) {
+    mbar_init(bar_ld, 1);
+    mbar_init(bar_mma, 1);
+    fence_mbar_init();
   }
-  float m_run[4], l_run[4], acc[4][DPT];
-#pragma unroll
-  for (int a = 0; a < 4; ++a) {
-    m_run[a] = -INFINITY;
-    l_run[a] = 0.f;
-#pragma unroll
-    for (int e = 0; e < DPT; ++e) acc[a][e] = 0.f;
+  if (warp == 0) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
+                 "r"(kFaTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
+  tmem_fence_before();
+  __syncthreads();
+  tmem_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  pdl_wait();  // q, K and V come from the upstream projection
+
+  // block kb's K and V rows (the keys below P) into the staging buffer
+  auto issue = [&](int kb) {
+    const int j0 = kb * kFaK, nk = min(kFaK, n_keys - j0);
+    const uint32_t bytes = static_cast<uint32_t>(nk * DH * 4);
+    mbar_arrive_expect_tx(bar_ld, 2 * bytes);
+    bulk_load(smem + S::kStK, kh + static_cast<size_t>(j0) * DH, bytes, bar_ld);
+    bulk_load(smem + S::kStV, vh + static_cast<size_t>(j0) * DH, bytes, bar_ld);
+  };
+  int pending = -1;  // thread 0: the block whose staging copy has not been waited for
+  if (tid == 0) {
+    issue(0);
+    pending = 0;
+  }
+
+  // Q block -> hi / lo (rows past P are zero)
+  for (int t = tid; t < kFaQ * (DH / 8); t += kFaThreads) {
+    const int r = t / (DH / 8), c8 = t - r * (DH / 8);
+    float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+    if (q0 + r < P) {
+      const float4* src = reinterpret_cast<const float4*>(q + static_cast<size_t>(q0 + r) * q_stride + h * DH + c8 * 8);
+      const float4 a = __ldcg(src), b = __ldcg(src + 1);
+      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    }
+    uint4 hi, lo;
+    split8_bf16(v, hi, lo);
+    const int off = (c8 >> 3) * S::kQAtom + sw128_off(r, c8 & 7);
+    *reinterpret_cast<uint4*>(smem + S::kQh + off) = hi;
+    *reinterpret_cast<uint4*>(smem + S::kQl + off) = lo;
+  }
+
+  const int row = (warp & 3) * 32 + lane;  // softmax threads (warps 0..3): query row = TMEM lane
+  const int qi = q0 + row;
+  float m_run = -INFINITY, l_run = 0.f;
+  float acc[DH];
+#pragma unroll
+  for (int d = 0; d < DH; ++d) acc[d] = 0.f;
+  bool ok = true;
+  uint32_t mma_phase = 0;
+  constexpr uint32_t idesc_s = umma_idesc_bf16(kFaQ, kFaK);
+  constexpr uint32_t idesc_o = umma_idesc_bf16(kFaQ, DH);
+
   for (int kb = 0; kb < n_kb; ++kb) {
-    const int j0 = kb * kPaK;
-    const float* Ks = Kb + (kb & 1) * kPaK * KS;
-    const float* Vs = Vb + (kb & 1) * kPaK * DH;
-    cp_async_wait_group<1>();  // block kb has landed (block kb + 1 may still be in flight)
-    __syncthreads();
-    // scores s[a][b] = q_{4tr+a} . k_{tc+16b}
-    float s[4][4];
+    const int j0 = kb * kFaK, nk = min(kFaK, n_keys - j0);
+    // ---- the block's K and V: staging -> bf16 hi / lo operands (keys past nk are zero)
+    if (ok && !mbar_wait(bar_ld, static_cast<uint32_t>(kb) & 1u)) ok = false;
+    if (ok && tid == 0) pending = -1;
+    for (int t = tid; t < kFaK * (DH / 8); t += kFaThreads) {  // K: rows = keys
+      const int j = t / (DH / 8), c8 = t - j * (DH / 8);
+      float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+      if (j < nk) {
+        const float4 a = *reinterpret_cast<const float4*>(stk + j * DH + c8 * 8);
+        const float4 b = *reinterpret_cast<const float4*>(stk + j * DH + c8 * 8 + 4);
+        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+      }
+      uint4 hi, lo;
+      split8_bf16(v, hi, lo);
+      const int off = (c8 >> 3) * S::kKAtom + sw128_off(j, c8 & 7);
+      *reinterpret_cast<uint4*>(smem + S::kKh + off) = hi;
+      *reinterpret_cast<uint4*>(smem + S::kKl + off) = lo;
+    }
+    for (int t = tid; t < DH * (kFaK / 8); t += kFaThreads) {  // V^T: rows = dimensions, keys along K
+      const int c8 = t / DH, d = t - c8 * DH;
+      float v[8];
 #pragma unroll
-    for (int a = 0; a < 4; ++a)
+      for (int e = 0; e < 8; ++e) v[e] = (c8 * 8 + e < nk) ? stv[(c8 * 8 + e) * DH + d] : 0.f;
+      uint4 hi, lo;
+      split8_bf16(v, hi, lo);
+      const int off = sw128_off(d, c8);
+      *reinterpret_cast<uint4*>(smem + S::kVh + off) = hi;
+      *reinterpret_cast<uint4*>(smem + S::kVl + off) = lo;
+    }
+    fence_proxy_async_smem();
+    if (!__syncthreads_and(ok)) {
+      ok = false;
+      break;
+    }
+    if (tid == 0) {
+      if (kb + 1 < n_kb) {  // the staging buffer is free: the next block's rows go out now
+        issue(kb + 1);
+        pending = kb + 1;
+      }
+      // ---- S = Q K^T
+      tmem_fence_after();
 #pragma unroll
-      for (int b = 0; b < 4; ++b) s[a][b] = 0.f;
-#pragma unroll 2
-    for (int d = 0; d < DH; d += 4) {
-      float4 qv[4], kv[4];
+      for (int kk = 0; kk < DH / 16; ++kk) {
+        const int at = kk >> 2, sub = 2 * (kk & 3);
+        const uint64_t qh = umma_desc_sw128(smem_u32(smem + S::kQh + at * S::kQAtom)) + sub;
+        const uint64_t ql = umma_desc_sw128(smem_u32(smem + S::kQl + at * S::kQAtom)) + sub;
+        const uint64_t kh_ = umma_desc_sw128(smem_u32(smem + S::kKh + at * S::kKAtom)) + sub;
+        const uint64_t kl_ = umma_desc_sw128(smem_u32(smem + S::kKl + at * S::kKAtom)) + sub;
+        umma_f16(tmem, qh, kh_, idesc_s, kk > 0 ? 1u : 0u);
+        umma_f16(tmem, qh, kl_, idesc_s, 1u);
+        umma_f16(tmem, ql, kh_, idesc_s, 1u);
+      }
+      umma_commit(bar_mma);
+    }
+    // ---- softmax of the block's scores, one row per thread of warps 0..3
+    if (ok && !mbar_wait(bar_mma, mma_phase)) ok = false;
+    mma_phase ^= 1u;
+    tmem_fence_after();
+    float alpha = 1.f;
+    if (warp < 4) {
+      const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+      float sv[32];
+      float bm = -INFINITY;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) qv[e] = *reinterpret_cast<const float4*>(Qt + (d + e) * kPaPad + 4 * tr);
+      for (int half = 0; half < 2; ++half) {
+        tmem_ld32(trow + half * 32, sv);
 #pragma unroll
-      for (int b = 0; b < 4; ++b) kv[b] = *reinterpret_cast<const float4*>(Ks + (tc + 16 * b) * KS + d);
+        for (int c = 0; c < 32; ++c) {
+          const int kj = j0 + half * 32 + c;
+          if (kj <= qi && kj < P) bm = fmaxf(bm, sv[c] * scale);
+        }
+      }
+      const float m_new = fmaxf(m_run, bm);
+      alpha = m_run == -INFINITY ? 0.f : expf(m_run - m_new);
+      float ls = 0.f;
 #pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        s[0][b] = fmaf(qv[0].x, kv[b].x, s[0][b]);
-        s[1][b] = fmaf(qv[0].y, kv[b].x, s[1][b]);
-        s[2][b] = fmaf(qv[0].z, kv[b].x, s[2][b]);
-        s[3][b] = fmaf(qv[0].w, kv[b].x, s[3][b]);
-        s[0][b] = fmaf(qv[1].x, kv[b].y, s[0][b]);
-        s[1][b] = fmaf(qv[1].y, kv[b].y, s[1][b]);
-        s[2][b] = fmaf(qv[1].z, kv[b].y, s[2][b]);
-        s[3][b] = fmaf(qv[1].w, kv[b].y, s[3][b]);
-        s[0][b] = fmaf(qv[2].x, kv[b].z, s[0][b]);
-        s[1][b] = fmaf(qv[2].y, kv[b].z, s[1][b]);
-        s[2][b] = fmaf(qv[2].z, kv[b].z, s[2][b]);
-        s[3][b] = fmaf(qv[2].w, kv[b].z, s[3][b]);
-        s[0][b] = fmaf(qv[3].x, kv[b].w, s[0][b]);
-        s[1][b] = fmaf(qv[3].y, kv[b].w, s[1][b]);
-        s[2][b] = fmaf(qv[3].z, kv[b].w, s[2][b]);
-        s[3][b] = fmaf(qv[3].w, kv[b].w, s[3][b]);
+      for (int half = 0; half < 2; ++half) {
+        tmem_ld32(trow + half * 32, sv);
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const int kj = j0 + half * 32 + c;
+          sv[c] = (kj <= qi && kj < P) ? expf(sv[c] * scale - m_new) : 0.f;
+          ls += sv[c];
+        }
+#pragma unroll
+        for (int c8 = 0; c8 < 4; ++c8) {
+          uint4 hi, lo;
+          split8_bf16(sv + 8 * c8, hi, lo);
+          const int off = sw128_off(row, half * 4 + c8);
+          *reinterpret_cast<uint4*>(smem + S::kPh + off) = hi;
+          *reinterpret_cast<uint4*>(smem + S::kPl + off) = lo;
+        }
+      }
+      l_run = l_run * alpha + ls;
+      m_run = m_new;
+    }
+    tmem_fence_before();
+    fence_proxy_async_smem();
+    if (!__syncthreads_and(ok)) {
+      ok = false;
+      break;
+    }
+    if (tid == 0) {
+      // ---- O_blk = P V
+      tmem_fence_after();
+#pragma unroll
+      for (int kk = 0; kk < kFaK / 16; ++kk) {
+        const uint64_t ph = umma_desc_sw128(smem_u32(smem + S::kPh)) + 2 * kk;
+        const uint64_t pl = umma_desc_sw128(smem_u32(smem + S::kPl)) + 2 * kk;
+        const uint64_t vh_ = umma_desc_sw128(smem_u32(smem + S::kVh)) + 2 * kk;
+        const uint64_t vl_ = umma_desc_sw128(smem_u32(smem + S::kVl)) + 2 * kk;
+        umma_f16(tmem + kFaK, ph, vh_, idesc_o, kk > 0 ? 1u : 0u);
+        umma_f16(tmem + kFaK, ph, vl_, idesc_o, 1u);
+        umma_f16(tmem + kFaK, pl, vh_, idesc_o, 1u);
+      }
+      umma_commit(bar_mma);
+    }
+    if (ok && !mbar_wait(bar_mma, mma_phase)) ok = false;
+    mma_phase ^= 1u;
+    tmem_fence_after();
+    if (warp < 4) {
+      const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16) + kFaK;
+#pragma unroll
+      for (int c = 0; c < DH / 32; ++c) {
+        float ov[32];
+        tmem_ld32(trow + c * 32, ov);
+#pragma unroll
+        for (int e = 0; e < 32; ++e) acc[c * 32 + e] = fmaf(acc[c * 32 + e], alpha, ov[e]);
       }
     }
-    // online softmax per row over this key block (16 lanes share a row)
-#pragma unroll
-    for (int a = 0; a < 4; ++a) {
-      const int qi = q0 + 4 * tr + a;
-      float mx = -INFINITY;
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const int kj = j0 + tc + 16 * b;
-        s[a][b] = (kj <= qi && kj < P) ? s[a][b] * scale : -INFINITY;
-        mx = fmaxf(mx, s[a][b]);
-      }
-#pragma unroll
-      for (int off = 8; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      const float m_new = fmaxf(m_run[a], mx);
-      float rsum = 0.f;
-#pragma unroll
-      for (int b = 0; b < 4; ++b) {
-        const float e = (m_new == -INFINITY || s[a][b] == -INFINITY) ? 0.f : expf(s[a][b] - m_new);
-        Ps[(4 * tr + a) * kPaPad + tc + 16 * b] = e;
-        rsum += e;
-      }
-#pragma unroll
-      for (int off = 8; off > 0; off >>= 1) rsum += __shfl_xor_sync(0xffffffffu, rsum, off);
-      const float corr = (m_run[a] == -INFINITY) ? 0.f : expf(m_run[a] - m_new);
-      l_run[a] = l_run[a] * corr + rsum;
-#pragma unroll
-      for (int e = 0; e < DPT; ++e) acc[a][e] *= corr;
-      m_run[a] = m_new;
+    tmem_fence_before();
+    if (!__syncthreads_and(ok)) {  // the operands and the accumulators are free for the next block
+      ok = false;
+      break;
     }
-    __syncthreads();
-    // O += P V
-    const int kn = min(kPaK, P - j0);
-    for (int j = 0; j < kn; ++j) {
-      float vv[DPT];
-#pragma unroll
-      for (int e = 0; e < DPT; e += 4) {
-        const float4 t = *reinterpret_cast<const float4*>(Vs + j * DH + tc * DPT + e);
-        vv[e] = t.x;
-        vv[e + 1] = t.y;
-        vv[e + 2] = t.z;
-        vv[e + 3] = t.w;
-      }
-#pragma unroll
-      for (int a = 0; a < 4; ++a) {
-        const float pj = Ps[(4 * tr + a) * kPaPad + j];
-#pragma unroll
-        for (int e = 0; e < DPT; ++e) acc[a][e] = fmaf(pj, vv[e], acc[a][e]);
-      }
-    }
-    __syncthreads();  // buffer kb & 1 and Ps are free again
-    if (kb + 2 < n_kb) issue(kb + 2);
-    else cp_async_commit();
   }
-  cp_async_wait_all();
+  if (!ok && tid == 0) {
+    set_error(st, DERR_TIMEOUT);
+    if (pending >= 0)  // a staging copy may still be landing: a bounded wait before the CTA leaves
+      mbar_wait_for(bar_ld, static_cast<uint32_t>(pending) & 1u, 100000000ull);
+  }
+  if (warp < 4 && qi < P && ok) {
+    const float inv = 1.0f / l_run;
+    float4* orow = reinterpret_cast<float4*>(o + static_cast<size_t>(qi) * o_stride + h * DH);
 #pragma unroll
-  for (int a = 0; a < 4; ++a) {
-    const int qi = q0 + 4 * tr + a;
-    if (qi >= P) continue;
-    const float inv = 1.0f / l_run[a];
-    float* orow = o + static_cast<size_t>(qi) * o_stride + h * DH + tc * DPT;
-#pragma unroll
-    for (int e = 0; e < DPT; ++e) orow[e] = acc[a][e] * inv;
+    for (int d4 = 0; d4 < DH / 4; ++d4)
+      orow[d4] = make_float4(acc[4 * d4] * inv, acc[4 * d4 + 1] * inv, acc[4 * d4 + 2] * inv, acc[4 * d4 + 3] * inv);
+  }
+  tmem_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tmem_fence_after();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kFaTmemCols) : "memory");
   }
 }
 
