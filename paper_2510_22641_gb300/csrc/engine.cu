@@ -44,9 +44,11 @@ cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, co
                            cudaStream_t s, bool pdl);
 cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                               __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl);
-cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
-                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale, DevState* st,
-                                cudaStream_t s, bool pdl);
+cudaError_t prefill_attn_launch(int head_dim, const CUtensorMap* maps, float* o, int o_stride, int P, int n_heads,
+                                int s_pad, float scale, DevState* st, cudaStream_t s, bool pdl);
+cudaError_t attn_parts_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc, int max_seq,
+                              int P, int n_heads, __nv_bfloat16* parts, size_t q_elems, size_t kv_elems, int qs_stride,
+                              int s_pad, cudaStream_t s, bool pdl);
 cudaError_t mid_launch(Epi e, const CUtensorMap* wmaps, const CUtensorMap* amaps, const GemvParams& p, int M,
                        int num_sms, cudaStream_t s, bool pdl);
 cudaError_t mid_attrs();
@@ -121,6 +123,12 @@ struct ssd_ctx {
   CUtensorMap a_maps[3][2];  // activation splits (hi, lo) for K = d_model, n_heads*head_dim, d_ff
   __nv_bfloat16 *a_hi = nullptr, *a_lo = nullptr;
   float *x_pre = nullptr, *q_pre = nullptr, *o_pre = nullptr, *h_pre = nullptr;
+  // the prefill attention's bf16 hi / lo operands, written by ssd_attn_parts_kernel: q rows
+  // [Pm][qdim] x 2, K [H][fa_spad][Dh] x 2, V transposed [H][Dh][fa_spad] x 2; their tensor maps
+  __nv_bfloat16* fa_parts = nullptr;
+  CUtensorMap fa_maps[6];
+  int fa_spad = 0;
+  size_t fa_q_elems = 0, fa_kv_elems = 0;  // elements of one q part and of one K (or V^T) part
   bool prefill_rows = false;  // SSD_OPT_PREFILL_ROWS: prefill through the decode kernels in 8-row chunks
   // owned device memory
   DevState* st = nullptr;
@@ -849,8 +857,10 @@ static ssd_status enqueue_prefill_tc(ssd_ctx* c, int n_vis, int n_prompt) {
     CKS(split(c, c->x_pre, dp, c->cfg.d_model, c->attn_norm[l], P));
     CKS(tc_gemm(c, Epi::QKV, 0, tl.qkv, P, p));
     CK(count_launch(c));
-    CK(prefill_attn_launch(c->cfg.head_dim, c->q_pre, c->qp, kv_k(c, l), kv_v(c, l),
-                           c->o_pre, c->qp, P, c->cfg.n_heads, c->cfg.max_seq,
+    CK(attn_parts_launch(c->cfg.head_dim, c->q_pre, c->qp, kv_k(c, l), kv_v(c, l), c->cfg.max_seq, P, c->cfg.n_heads,
+                         c->fa_parts, c->fa_q_elems, c->fa_kv_elems, c->qdim, c->fa_spad, c->cs, c->use_pdl));
+    CK(count_launch(c));
+    CK(prefill_attn_launch(c->cfg.head_dim, c->fa_maps, c->o_pre, c->qp, P, c->cfg.n_heads, c->fa_spad,
                            1.0f / sqrtf(static_cast<float>(c->cfg.head_dim)), c->st, c->cs, c->use_pdl));
     CKS(split(c, c->o_pre, c->qp, c->qdim, nullptr, P));
     p = TcParams{};
@@ -1496,7 +1506,7 @@ ssd_status ssd_destroy(ssd_ctx* c) {
   if (!c) return SSD_OK;
   if (c->cs) cudaStreamSynchronize(c->cs);
   drop_graphs(c);
-  void* bufs[] = {c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->step_log, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
+  void* bufs[] = {c->fa_parts, c->a_hi, c->a_lo, c->x_pre, c->q_pre, c->o_pre, c->h_pre, c->st, c->op_st, c->out_int, c->step_log, c->xv, c->qb, c->ob, c->hb, c->hin, c->xt, c->kc, c->vc, c->rope, c->gains,
                   c->partials, c->counters, c->attn_part, c->attn_tickets, c->dyn_table, c->dyn_launch, c->in_vis, c->in_prompt,
                   c->x_enc, c->enc_q, c->enc_o, c->enc_k, c->enc_v, c->ckc, c->cvc, c->dec_bias, c->enc_bias, c->one,
                   c->start_tok, c->req, c->bout, c->blog, c->bvis, c->bprompt, c->act_hi, c->act_lo, c->act_rs,
@@ -1846,6 +1856,23 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
     for (int i = 0; i < 3; ++i) {
       CKS(encode_map_sw128(c, &c->a_maps[i][0], c->a_hi, Pm, ks[i], kTcM));
       CKS(encode_map_sw128(c, &c->a_maps[i][1], c->a_lo, Pm, ks[i], kTcM));
+    }
+    if (!t5) {  // the prefill attention's operand parts (zeroed once: rows past a prompt stay finite)
+      const int H = k.n_heads, Dh = k.head_dim;
+      c->fa_spad = (k.max_seq + kFaK - 1) / kFaK * kFaK;
+      c->fa_q_elems = Pm * static_cast<size_t>(qdim);
+      c->fa_kv_elems = static_cast<size_t>(H) * c->fa_spad * Dh;
+      const size_t n = 2 * c->fa_q_elems + 4 * c->fa_kv_elems;
+      CKS(alloc(c, reinterpret_cast<void**>(&c->fa_parts), sizeof(__nv_bfloat16) * n));
+      CK(cudaMemset(c->fa_parts, 0, sizeof(__nv_bfloat16) * n));
+      __nv_bfloat16* base = c->fa_parts;
+      const size_t qn = c->fa_q_elems, kn = c->fa_kv_elems;
+      CKS(encode_map_sw128(c, &c->fa_maps[0], base, Pm, qdim, kFaQ));
+      CKS(encode_map_sw128(c, &c->fa_maps[1], base + qn, Pm, qdim, kFaQ));
+      CKS(encode_map_sw128(c, &c->fa_maps[2], base + 2 * qn, static_cast<uint64_t>(H) * c->fa_spad, Dh, kFaK));
+      CKS(encode_map_sw128(c, &c->fa_maps[3], base + 2 * qn + kn, static_cast<uint64_t>(H) * c->fa_spad, Dh, kFaK));
+      CKS(encode_map_sw128(c, &c->fa_maps[4], base + 2 * qn + 2 * kn, static_cast<uint64_t>(H) * Dh, c->fa_spad, Dh));
+      CKS(encode_map_sw128(c, &c->fa_maps[5], base + 2 * qn + 3 * kn, static_cast<uint64_t>(H) * Dh, c->fa_spad, Dh));
     }
   }
   CKS(alloc(c, reinterpret_cast<void**>(&c->in_prompt), sizeof(int) * in_rows));

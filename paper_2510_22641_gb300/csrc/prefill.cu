@@ -55,15 +55,27 @@ cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bf
   return launch_pdl(ssd_split_rows_kernel, dim3(rows), dim3(256), 0, s, pdl, x, x_stride, K, gain, eps, hi, lo);
 }
 
-cudaError_t prefill_attn_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc,
-                                float* o, int o_stride, int P, int n_heads, int max_seq, float scale, DevState* st,
-                                cudaStream_t s, bool pdl) {
+cudaError_t attn_parts_launch(int head_dim, const float* q, int q_stride, const float* kc, const float* vc, int max_seq,
+                              int P, int n_heads, __nv_bfloat16* parts, size_t q_elems, size_t kv_elems, int qs_stride,
+                              int s_pad, cudaStream_t s, bool pdl) {
+  const dim3 grid((P + 63) / 64, n_heads);
+  __nv_bfloat16 *qh = parts, *ql = parts + q_elems, *kh = parts + 2 * q_elems, *kl = kh + kv_elems,
+                *vh = kh + 2 * kv_elems, *vl = kh + 3 * kv_elems;
+  if (head_dim == 128)
+    return launch_pdl(ssd_attn_parts_kernel<128>, grid, dim3(256), 0, s, pdl, q, q_stride, kc, vc, max_seq, P, qh, ql,
+                      qs_stride, kh, kl, vh, vl, s_pad);
+  return launch_pdl(ssd_attn_parts_kernel<64>, grid, dim3(256), 0, s, pdl, q, q_stride, kc, vc, max_seq, P, qh, ql,
+                    qs_stride, kh, kl, vh, vl, s_pad);
+}
+
+cudaError_t prefill_attn_launch(int head_dim, const CUtensorMap* maps, float* o, int o_stride, int P, int n_heads,
+                                int s_pad, float scale, DevState* st, cudaStream_t s, bool pdl) {
   const dim3 grid((P + kFaQ - 1) / kFaQ, n_heads);
   if (head_dim == 128)
-    return launch_pdl(ssd_prefill_attn_kernel<128>, grid, dim3(kFaThreads), FaSmem<128>::kTotal, s, pdl, q, q_stride,
-                      kc, vc, o, o_stride, P, max_seq, scale, st);
-  return launch_pdl(ssd_prefill_attn_kernel<64>, grid, dim3(kFaThreads), FaSmem<64>::kTotal, s, pdl, q, q_stride, kc,
-                    vc, o, o_stride, P, max_seq, scale, st);
+    return launch_pdl(ssd_prefill_attn_kernel<128>, grid, dim3(kFaThreads), FaSmem<128>::kTotal, s, pdl, maps[0],
+                      maps[1], maps[2], maps[3], maps[4], maps[5], o, o_stride, P, s_pad, scale, st);
+  return launch_pdl(ssd_prefill_attn_kernel<64>, grid, dim3(kFaThreads), FaSmem<64>::kTotal, s, pdl, maps[0], maps[1],
+                    maps[2], maps[3], maps[4], maps[5], o, o_stride, P, s_pad, scale, st);
 }
 
 }  // namespace ssd

@@ -281,43 +281,37 @@ namespace ssd {
 // ------------------------------------------------------------------ causal prefill attention
 // One CTA per (128-query block, head), the blocks with the most key blocks launched first.
 // Both products run on the 5th-generation tensor cores with fp32-class accuracy: every fp32
-// operand x is split into bf16 parts x = hi + lo, and a product a.b is taken as
+// operand x is split into bf16 parts x = hi + lo and a product a.b is taken as
 // hi(a) hi(b) + hi(a) lo(b) + lo(a) hi(b) in fp32 (the lo lo term is below fp32 rounding).
-//   * Q block (128 rows x Dh) -> bf16 hi / lo, 128-byte swizzled K-major (rows = queries), once;
-//   * per 64-key block (causal: up to the query block): thread 0 bulk-copies the block's fp32 K and
-//     V rows into a staging buffer one block ahead; all threads turn them into bf16 hi / lo K
-//     (rows = keys) and V^T (rows = head dimensions, keys along K);
-//   * S = Q K^T: 3 x Dh/16 tcgen05.mma (M = 128 queries, N = 64 keys) into TMEM columns 0..63;
-//   * warps 0..3, one thread per query row (its TMEM lane): scale, causal mask, online softmax
-//     (running max and sum in registers), P = exp(S - max) -> bf16 hi / lo, 128-byte swizzled
-//     (rows = queries, keys along K);
-//   * O_blk = P V: 3 x 4 tcgen05.mma (M = 128, N = Dh, K = 64 keys) into TMEM columns 64..64+Dh;
-//     the same threads fold it into their row's fp32 output registers, O = O * alpha + O_blk.
+// ssd_attn_parts_kernel writes the parts once per layer (q rows, K rows, V transposed), so here
+// every operand arrives by TMA in the 128-byte swizzled layout the MMA reads:
+//   * warp 0 (one thread): the Q block, then each 64-key block's K and V^T parts into a 2-stage ring;
+//   * warp 1 (one thread): S_j = Q K_j^T, 3 x Dh/16 MMAs (M = 128 queries, N = 64 keys) into one of
+//     two TMEM score buffers, issued while the softmax works on the previous block; then
+//     O_j = P_j V_j, 3 x 4 MMAs (N = Dh) into the TMEM output block;
+//   * warps 2..5, one thread per query row (its TMEM lane): causal mask, online softmax in
+//     registers (exp2 of the scores times scale * log2 e), P_j as bf16 parts into shared memory,
+//     and O = O * alpha + O_j folded into the row's fp32 registers.
 // Every step of a row depends on the keys' positions only; rows are independent.
-// q: [P][q_stride] rotated queries; K, V: the fp32 cache [H][max_seq][Dh]; o: [P][o_stride].
-constexpr int kFaQ = 128;       // query rows per CTA (the MMA's M)
-constexpr int kFaK = 64;        // keys per block (the S MMA's N, the P.V MMA's K)
-constexpr int kFaThreads = 256;
-constexpr int kFaTmemCols = 256;  // S: 64 columns, O block: Dh columns
+constexpr int kFaThreads = 192;
+constexpr int kFaTmemCols = 256;  // S: 2 x 64 columns, O block: Dh columns
 
 template <int DH>
 struct FaSmem {
   static constexpr int kNA = DH / 64;                    // 64-column atoms along the head dimension
   static constexpr int kQAtom = kFaQ * 128;              // one atom of the Q block (hi or lo)
-  static constexpr int kKAtom = kFaK * 128;              // one atom of the K block
+  static constexpr int kKAtom = kFaK * 128;              // one atom of a K block
   static constexpr int kQh = 0;                          // [kNA][128 rows][128 B]
   static constexpr int kQl = kQh + kNA * kQAtom;
-  static constexpr int kKh = kQl + kNA * kQAtom;         // [kNA][64 keys][128 B]
-  static constexpr int kKl = kKh + kNA * kKAtom;
-  static constexpr int kVh = kKl + kNA * kKAtom;         // V^T: [Dh rows][64 keys x 2 B]
-  static constexpr int kVl = kVh + DH * 128;
-  static constexpr int kPh = kVl + DH * 128;             // P: [128 rows][64 keys x 2 B]
+  static constexpr int kStage = 2 * kNA * kKAtom + 2 * DH * 128;  // K hi, K lo, V^T hi, V^T lo
+  static constexpr int kKV = kQl + kNA * kQAtom;         // [2 stages]
+  static constexpr int kPh = kKV + 2 * kStage;           // P: [128 rows][64 keys x 2 B]
   static constexpr int kPl = kPh + kFaQ * 128;
-  static constexpr int kStK = kPl + kFaQ * 128;          // fp32 staging of one block: K [64][Dh]
-  static constexpr int kStV = kStK + kFaK * DH * 4;      //                            V [64][Dh]
-  static constexpr int kBar = kStV + kFaK * DH * 4;      // staging full, MMA done
-  static constexpr int kTmemSlot = kBar + 16;
+  static constexpr int kBar = kPl + kFaQ * 128;          // q_full, kv_full[2], kv_empty[2], s_full[2], p_full, o_full, o_empty
+  static constexpr int kTmemSlot = kBar + 10 * 8;
   static constexpr int kTotal = kTmemSlot + 16 + 1024;   // + slack for the 1024-byte alignment
+  // within a stage
+  static constexpr int kKh = 0, kKl = kNA * kKAtom, kVh = 2 * kNA * kKAtom, kVl = kVh + DH * 128;
 };
 
 // 8 fp32 values -> bf16 hi and lo parts, packed two per word.
@@ -334,38 +328,107 @@ __device__ __forceinline__ void split8_bf16(const float* v, uint4& hi, uint4& lo
   lo = make_uint4(lw[0], lw[1], lw[2], lw[3]);
 }
 
-// Byte offset of 16-byte chunk ch of row r in a 128-byte swizzled atom.
+// Byte offset of 16-byte chunk ch of row r in a 128-byte swizzled tile.
 __device__ __forceinline__ int sw128_off(int r, int ch) { return r * 128 + ((ch ^ (r & 7)) << 4); }
 
+// The attention's operand parts of one layer, once per prefill: for the 64 positions
+// r0 .. r0 + 63 of head h, the q rows and the cache's K rows as bf16 hi / lo rows
+// (qs [rows][qs_stride], ks [H][s_pad][Dh]) and the V rows transposed through shared memory
+// (vt [H][Dh][s_pad], positions at or past P written as zeros), all with 16-byte stores.
+template <int DH>
+__global__ void __launch_bounds__(256) ssd_attn_parts_kernel(const float* __restrict__ q, int q_stride,
+                                                            const float* __restrict__ k_cache,
+                                                            const float* __restrict__ v_cache, int max_seq, int P,
+                                                            __nv_bfloat16* qs_hi, __nv_bfloat16* qs_lo, int qs_stride,
+                                                            __nv_bfloat16* ks_hi, __nv_bfloat16* ks_lo,
+                                                            __nv_bfloat16* vt_hi, __nv_bfloat16* vt_lo, int s_pad) {
+  __shared__ float vt[DH][65];
+  const int r0 = blockIdx.x * 64, h = blockIdx.y, tid = threadIdx.x;
+  pdl_trigger();
+  pdl_wait();
+  for (int t = tid; t < 64 * (DH / 8); t += 256) {
+    const int r = t / (DH / 8), c8 = t - r * (DH / 8), pos = r0 + r;
+    if (pos >= P) {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) vt[c8 * 8 + e][r] = 0.f;
+      continue;
+    }
+    uint4 hi, lo;
+    float v[8];
+    const float4* qr = reinterpret_cast<const float4*>(q + static_cast<size_t>(pos) * q_stride + h * DH + c8 * 8);
+    float4 a = __ldcg(qr), b = __ldcg(qr + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    split8_bf16(v, hi, lo);
+    const size_t qo = static_cast<size_t>(pos) * qs_stride + h * DH + c8 * 8;
+    *reinterpret_cast<uint4*>(qs_hi + qo) = hi;
+    *reinterpret_cast<uint4*>(qs_lo + qo) = lo;
+    const size_t ko = (static_cast<size_t>(h) * max_seq + pos) * DH + c8 * 8;
+    a = __ldcg(reinterpret_cast<const float4*>(k_cache + ko));
+    b = __ldcg(reinterpret_cast<const float4*>(k_cache + ko) + 1);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+    split8_bf16(v, hi, lo);
+    const size_t kso = (static_cast<size_t>(h) * s_pad + pos) * DH + c8 * 8;
+    *reinterpret_cast<uint4*>(ks_hi + kso) = hi;
+    *reinterpret_cast<uint4*>(ks_lo + kso) = lo;
+    a = __ldcg(reinterpret_cast<const float4*>(v_cache + ko));
+    b = __ldcg(reinterpret_cast<const float4*>(v_cache + ko) + 1);
+    vt[c8 * 8 + 0][r] = a.x; vt[c8 * 8 + 1][r] = a.y; vt[c8 * 8 + 2][r] = a.z; vt[c8 * 8 + 3][r] = a.w;
+    vt[c8 * 8 + 4][r] = b.x; vt[c8 * 8 + 5][r] = b.y; vt[c8 * 8 + 6][r] = b.z; vt[c8 * 8 + 7][r] = b.w;
+  }
+  __syncthreads();
+  for (int t = tid; t < DH * 8; t += 256) {
+    const int d = t >> 3, p8 = t & 7;
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = vt[d][p8 * 8 + e];
+    uint4 hi, lo;
+    split8_bf16(v, hi, lo);
+    const size_t o = (static_cast<size_t>(h) * DH + d) * s_pad + r0 + p8 * 8;
+    *reinterpret_cast<uint4*>(vt_hi + o) = hi;
+    *reinterpret_cast<uint4*>(vt_lo + o) = lo;
+  }
+}
+
+// maps: q hi, q lo ([rows][H*Dh], 128-row boxes), k hi, k lo ([H*s_pad][Dh], 64-row boxes),
+// v^T hi, v^T lo ([H*Dh][s_pad], Dh-row boxes), all with 64-column boxes.
 template <int DH>
 __global__ void __launch_bounds__(kFaThreads, 1)
-    ssd_prefill_attn_kernel(const float* __restrict__ q, int q_stride, const float* __restrict__ k_cache,
-                            const float* __restrict__ v_cache, float* __restrict__ o, int o_stride, int P,
-                            int max_seq, float scale, DevState* st) {
+    ssd_prefill_attn_kernel(const __grid_constant__ CUtensorMap mqh, const __grid_constant__ CUtensorMap mql,
+                            const __grid_constant__ CUtensorMap mkh, const __grid_constant__ CUtensorMap mkl,
+                            const __grid_constant__ CUtensorMap mvh, const __grid_constant__ CUtensorMap mvl,
+                            float* __restrict__ o, int o_stride, int P, int s_pad, float scale, DevState* st) {
   using S = FaSmem<DH>;
   extern __shared__ __align__(1024) uint8_t fa_raw[];
   const uint32_t raw = smem_u32(fa_raw);
   uint8_t* smem = fa_raw + (((raw + 1023u) & ~1023u) - raw);
-  uint64_t* bar_ld = reinterpret_cast<uint64_t*>(smem + S::kBar);
-  uint64_t* bar_mma = bar_ld + 1;
+  uint64_t* q_full = reinterpret_cast<uint64_t*>(smem + S::kBar);
+  uint64_t* kv_full = q_full + 1;
+  uint64_t* kv_empty = kv_full + 2;
+  uint64_t* s_full = kv_empty + 2;
+  uint64_t* p_full = s_full + 2;
+  uint64_t* o_full = p_full + 1;
+  uint64_t* o_empty = o_full + 1;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + S::kTmemSlot);
-  const float* stk = reinterpret_cast<const float*>(smem + S::kStK);
-  const float* stv = reinterpret_cast<const float*>(smem + S::kStV);
   const int nqb = gridDim.x, qb = nqb - 1 - static_cast<int>(blockIdx.x), h = blockIdx.y;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int q0 = qb * kFaQ;
   const int n_keys = min(q0 + kFaQ, P);  // keys 0 .. n_keys - 1 reach some row of the block
   const int n_kb = (n_keys + kFaK - 1) / kFaK;
-  const float* kh = k_cache + static_cast<size_t>(h) * max_seq * DH;
-  const float* vh = v_cache + static_cast<size_t>(h) * max_seq * DH;
 
   pdl_trigger();
   if (tid == 0) {
-    mbar_init(bar_ld, 1);
-    mbar_init(bar_mma, 1);
+    mbar_init(q_full, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&kv_full[b], 1);
+      mbar_init(&kv_empty[b], 1);
+      mbar_init(&s_full[b], 1);
+    }
+    mbar_init(p_full, 4);
+    mbar_init(o_full, 1);
+    mbar_init(o_empty, 4);
     fence_mbar_init();
   }
-  if (warp == 0) {
+  if (warp == 1) {
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
                  "r"(kFaTmemCols)
                  : "memory");
@@ -375,201 +438,182 @@ __global__ void __launch_bounds__(kFaThreads, 1)
   __syncthreads();
   tmem_fence_after();
   const uint32_t tmem = *tmem_slot;
-  pdl_wait();  // q, K and V come from the upstream projection
 
-  // block kb's K and V rows (the keys below P) into the staging buffer
-  auto issue = [&](int kb) {
-    const int j0 = kb * kFaK, nk = min(kFaK, n_keys - j0);
-    const uint32_t bytes = static_cast<uint32_t>(nk * DH * 4);
-    mbar_arrive_expect_tx(bar_ld, 2 * bytes);
-    bulk_load(smem + S::kStK, kh + static_cast<size_t>(j0) * DH, bytes, bar_ld);
-    bulk_load(smem + S::kStV, vh + static_cast<size_t>(j0) * DH, bytes, bar_ld);
-  };
-  int pending = -1;  // thread 0: the block whose staging copy has not been waited for
-  if (tid == 0) {
-    issue(0);
-    pending = 0;
-  }
-
-  // Q block -> hi / lo (rows past P are zero)
-  for (int t = tid; t < kFaQ * (DH / 8); t += kFaThreads) {
-    const int r = t / (DH / 8), c8 = t - r * (DH / 8);
-    float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-    if (q0 + r < P) {
-      const float4* src = reinterpret_cast<const float4*>(q + static_cast<size_t>(q0 + r) * q_stride + h * DH + c8 * 8);
-      const float4 a = __ldcg(src), b = __ldcg(src + 1);
-      v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-    }
-    uint4 hi, lo;
-    split8_bf16(v, hi, lo);
-    const int off = (c8 >> 3) * S::kQAtom + sw128_off(r, c8 & 7);
-    *reinterpret_cast<uint4*>(smem + S::kQh + off) = hi;
-    *reinterpret_cast<uint4*>(smem + S::kQl + off) = lo;
-  }
-
-  const int row = (warp & 3) * 32 + lane;  // softmax threads (warps 0..3): query row = TMEM lane
-  const int qi = q0 + row;
-  float m_run = -INFINITY, l_run = 0.f;
-  float acc[DH];
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    if (lane == 0) {
+      prefetch_tensormap(&mkh);
+      pdl_wait();  // the parts come from the upstream QKV projection
+      mbar_arrive_expect_tx(q_full, 2 * S::kNA * S::kQAtom);
 #pragma unroll
-  for (int d = 0; d < DH; ++d) acc[d] = 0.f;
-  bool ok = true;
-  uint32_t mma_phase = 0;
-  constexpr uint32_t idesc_s = umma_idesc_bf16(kFaQ, kFaK);
-  constexpr uint32_t idesc_o = umma_idesc_bf16(kFaQ, DH);
-
-  for (int kb = 0; kb < n_kb; ++kb) {
-    const int j0 = kb * kFaK, nk = min(kFaK, n_keys - j0);
-    // ---- the block's K and V: staging -> bf16 hi / lo operands (keys past nk are zero)
-    if (ok && !mbar_wait(bar_ld, static_cast<uint32_t>(kb) & 1u)) ok = false;
-    if (ok && tid == 0) pending = -1;
-    for (int t = tid; t < kFaK * (DH / 8); t += kFaThreads) {  // K: rows = keys
-      const int j = t / (DH / 8), c8 = t - j * (DH / 8);
-      float v[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
-      if (j < nk) {
-        const float4 a = *reinterpret_cast<const float4*>(stk + j * DH + c8 * 8);
-        const float4 b = *reinterpret_cast<const float4*>(stk + j * DH + c8 * 8 + 4);
-        v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+      for (int a = 0; a < S::kNA; ++a) {
+        tma_load_2d(smem + S::kQh + a * S::kQAtom, &mqh, q_full, h * DH + a * 64, q0);
+        tma_load_2d(smem + S::kQl + a * S::kQAtom, &mql, q_full, h * DH + a * 64, q0);
       }
-      uint4 hi, lo;
-      split8_bf16(v, hi, lo);
-      const int off = (c8 >> 3) * S::kKAtom + sw128_off(j, c8 & 7);
-      *reinterpret_cast<uint4*>(smem + S::kKh + off) = hi;
-      *reinterpret_cast<uint4*>(smem + S::kKl + off) = lo;
-    }
-    for (int t = tid; t < DH * (kFaK / 8); t += kFaThreads) {  // V^T: rows = dimensions, keys along K
-      const int c8 = t / DH, d = t - c8 * DH;
-      float v[8];
+      for (int j = 0; j < n_kb; ++j) {
+        const int b = j & 1;
+        if (j >= 2 && !mbar_wait(&kv_empty[b], static_cast<uint32_t>((j - 2) >> 1) & 1u)) {
+          set_error(st, DERR_TIMEOUT);
+          break;
+        }
+        uint8_t* sb = smem + S::kKV + b * S::kStage;
+        mbar_arrive_expect_tx(&kv_full[b], S::kStage);
 #pragma unroll
-      for (int e = 0; e < 8; ++e) v[e] = (c8 * 8 + e < nk) ? stv[(c8 * 8 + e) * DH + d] : 0.f;
-      uint4 hi, lo;
-      split8_bf16(v, hi, lo);
-      const int off = sw128_off(d, c8);
-      *reinterpret_cast<uint4*>(smem + S::kVh + off) = hi;
-      *reinterpret_cast<uint4*>(smem + S::kVl + off) = lo;
-    }
-    fence_proxy_async_smem();
-    if (!__syncthreads_and(ok)) {
-      ok = false;
-      break;
-    }
-    if (tid == 0) {
-      if (kb + 1 < n_kb) {  // the staging buffer is free: the next block's rows go out now
-        issue(kb + 1);
-        pending = kb + 1;
+        for (int a = 0; a < S::kNA; ++a) {
+          tma_load_2d(sb + S::kKh + a * S::kKAtom, &mkh, &kv_full[b], a * 64, h * s_pad + j * kFaK);
+          tma_load_2d(sb + S::kKl + a * S::kKAtom, &mkl, &kv_full[b], a * 64, h * s_pad + j * kFaK);
+        }
+        tma_load_2d(sb + S::kVh, &mvh, &kv_full[b], j * kFaK, h * DH);
+        tma_load_2d(sb + S::kVl, &mvl, &kv_full[b], j * kFaK, h * DH);
       }
-      // ---- S = Q K^T
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc_s = umma_idesc_bf16(kFaQ, kFaK);
+      constexpr uint32_t idesc_o = umma_idesc_bf16(kFaQ, DH);
+      auto issue_s = [&](int j) {  // S_j into score buffer j & 1
+        const int b = j & 1;
+        const uint8_t* sb = smem + S::kKV + b * S::kStage;
+        const uint32_t d = tmem + static_cast<uint32_t>(b * kFaK);
+        tmem_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < DH / 16; ++kk) {
+          const int at = kk >> 2, sub = 2 * (kk & 3);
+          const uint64_t qh = umma_desc_sw128(smem_u32(smem + S::kQh + at * S::kQAtom)) + sub;
+          const uint64_t ql = umma_desc_sw128(smem_u32(smem + S::kQl + at * S::kQAtom)) + sub;
+          const uint64_t kh = umma_desc_sw128(smem_u32(sb + S::kKh + at * S::kKAtom)) + sub;
+          const uint64_t kl = umma_desc_sw128(smem_u32(sb + S::kKl + at * S::kKAtom)) + sub;
+          umma_f16(d, qh, kh, idesc_s, kk > 0 ? 1u : 0u);
+          umma_f16(d, qh, kl, idesc_s, 1u);
+          umma_f16(d, ql, kh, idesc_s, 1u);
+        }
+        umma_commit(&s_full[b]);
+      };
+      auto issue_o = [&](int j) {  // O_j = P_j V_j; frees stage j & 1
+        const uint8_t* sb = smem + S::kKV + (j & 1) * S::kStage;
+        const uint32_t d = tmem + static_cast<uint32_t>(2 * kFaK);
+        tmem_fence_after();
+#pragma unroll
+        for (int kk = 0; kk < kFaK / 16; ++kk) {
+          const uint64_t ph = umma_desc_sw128(smem_u32(smem + S::kPh)) + 2 * kk;
+          const uint64_t pl = umma_desc_sw128(smem_u32(smem + S::kPl)) + 2 * kk;
+          const uint64_t vh = umma_desc_sw128(smem_u32(sb + S::kVh)) + 2 * kk;
+          const uint64_t vl = umma_desc_sw128(smem_u32(sb + S::kVl)) + 2 * kk;
+          umma_f16(d, ph, vh, idesc_o, kk > 0 ? 1u : 0u);
+          umma_f16(d, ph, vl, idesc_o, 1u);
+          umma_f16(d, pl, vh, idesc_o, 1u);
+        }
+        umma_commit(o_full);
+        umma_commit(&kv_empty[j & 1]);
+      };
+      bool ok = n_kb > 0 && mbar_wait(q_full, 0) && mbar_wait(&kv_full[0], 0);
+      if (ok) issue_s(0);
+      for (int j = 0; ok && j < n_kb; ++j) {
+        if (j + 1 < n_kb) {  // S_{j+1} runs while the softmax works on S_j: its score buffer held S_{j-1},
+                             // which the softmax read before it released P_{j-1} (waited for below, last round)
+          if (!mbar_wait(&kv_full[(j + 1) & 1], static_cast<uint32_t>((j + 1) >> 1) & 1u)) {
+            ok = false;
+            break;
+          }
+          issue_s(j + 1);
+        }
+        // O_j once P_j is written and O_{j-1} has been folded
+        if (!mbar_wait(p_full, static_cast<uint32_t>(j) & 1u) ||
+            (j >= 1 && !mbar_wait(o_empty, static_cast<uint32_t>(j - 1) & 1u))) {
+          ok = false;
+          break;
+        }
+        issue_o(j);
+      }
+      if (!ok && n_kb > 0) set_error(st, DERR_TIMEOUT);
+    }
+  } else {
+    // ---------------------------------------------------------------- softmax (warps 2..5)
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane, qi = q0 + row;
+    const float sl2 = scale * 1.4426950408889634f;  // scores in log2 units: exp(x) = exp2(x log2 e)
+    const uint32_t tl = tmem + (static_cast<uint32_t>(quad * 32) << 16);
+    float m_run = -INFINITY, l_run = 0.f, alpha_prev = 0.f;
+    float acc[DH];
+#pragma unroll
+    for (int d = 0; d < DH; ++d) acc[d] = 0.f;
+    bool ok = true;
+    auto fold = [&](int j) {  // acc = acc * alpha_j + O_j
+      if (ok && !mbar_wait(o_full, static_cast<uint32_t>(j) & 1u)) ok = false;
       tmem_fence_after();
-#pragma unroll
-      for (int kk = 0; kk < DH / 16; ++kk) {
-        const int at = kk >> 2, sub = 2 * (kk & 3);
-        const uint64_t qh = umma_desc_sw128(smem_u32(smem + S::kQh + at * S::kQAtom)) + sub;
-        const uint64_t ql = umma_desc_sw128(smem_u32(smem + S::kQl + at * S::kQAtom)) + sub;
-        const uint64_t kh_ = umma_desc_sw128(smem_u32(smem + S::kKh + at * S::kKAtom)) + sub;
-        const uint64_t kl_ = umma_desc_sw128(smem_u32(smem + S::kKl + at * S::kKAtom)) + sub;
-        umma_f16(tmem, qh, kh_, idesc_s, kk > 0 ? 1u : 0u);
-        umma_f16(tmem, qh, kl_, idesc_s, 1u);
-        umma_f16(tmem, ql, kh_, idesc_s, 1u);
-      }
-      umma_commit(bar_mma);
-    }
-    // ---- softmax of the block's scores, one row per thread of warps 0..3
-    if (ok && !mbar_wait(bar_mma, mma_phase)) ok = false;
-    mma_phase ^= 1u;
-    tmem_fence_after();
-    float alpha = 1.f;
-    if (warp < 4) {
-      const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-      float sv[32];
-      float bm = -INFINITY;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        tmem_ld32(trow + half * 32, sv);
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const int kj = j0 + half * 32 + c;
-          if (kj <= qi && kj < P) bm = fmaxf(bm, sv[c] * scale);
-        }
-      }
-      const float m_new = fmaxf(m_run, bm);
-      alpha = m_run == -INFINITY ? 0.f : expf(m_run - m_new);
-      float ls = 0.f;
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        tmem_ld32(trow + half * 32, sv);
-#pragma unroll
-        for (int c = 0; c < 32; ++c) {
-          const int kj = j0 + half * 32 + c;
-          sv[c] = (kj <= qi && kj < P) ? expf(sv[c] * scale - m_new) : 0.f;
-          ls += sv[c];
-        }
-#pragma unroll
-        for (int c8 = 0; c8 < 4; ++c8) {
-          uint4 hi, lo;
-          split8_bf16(sv + 8 * c8, hi, lo);
-          const int off = sw128_off(row, half * 4 + c8);
-          *reinterpret_cast<uint4*>(smem + S::kPh + off) = hi;
-          *reinterpret_cast<uint4*>(smem + S::kPl + off) = lo;
-        }
-      }
-      l_run = l_run * alpha + ls;
-      m_run = m_new;
-    }
-    tmem_fence_before();
-    fence_proxy_async_smem();
-    if (!__syncthreads_and(ok)) {
-      ok = false;
-      break;
-    }
-    if (tid == 0) {
-      // ---- O_blk = P V
-      tmem_fence_after();
-#pragma unroll
-      for (int kk = 0; kk < kFaK / 16; ++kk) {
-        const uint64_t ph = umma_desc_sw128(smem_u32(smem + S::kPh)) + 2 * kk;
-        const uint64_t pl = umma_desc_sw128(smem_u32(smem + S::kPl)) + 2 * kk;
-        const uint64_t vh_ = umma_desc_sw128(smem_u32(smem + S::kVh)) + 2 * kk;
-        const uint64_t vl_ = umma_desc_sw128(smem_u32(smem + S::kVl)) + 2 * kk;
-        umma_f16(tmem + kFaK, ph, vh_, idesc_o, kk > 0 ? 1u : 0u);
-        umma_f16(tmem + kFaK, ph, vl_, idesc_o, 1u);
-        umma_f16(tmem + kFaK, pl, vh_, idesc_o, 1u);
-      }
-      umma_commit(bar_mma);
-    }
-    if (ok && !mbar_wait(bar_mma, mma_phase)) ok = false;
-    mma_phase ^= 1u;
-    tmem_fence_after();
-    if (warp < 4) {
-      const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16) + kFaK;
 #pragma unroll
       for (int c = 0; c < DH / 32; ++c) {
         float ov[32];
-        tmem_ld32(trow + c * 32, ov);
+        tmem_ld32(tl + static_cast<uint32_t>(2 * kFaK + c * 32), ov);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) acc[c * 32 + e] = fmaf(acc[c * 32 + e], alpha, ov[e]);
+        for (int e = 0; e < 32; ++e) acc[c * 32 + e] = fmaf(acc[c * 32 + e], alpha_prev, ov[e]);
       }
-    }
-    tmem_fence_before();
-    if (!__syncthreads_and(ok)) {  // the operands and the accumulators are free for the next block
-      ok = false;
-      break;
-    }
-  }
-  if (!ok && tid == 0) {
-    set_error(st, DERR_TIMEOUT);
-    if (pending >= 0)  // a staging copy may still be landing: a bounded wait before the CTA leaves
-      mbar_wait_for(bar_ld, static_cast<uint32_t>(pending) & 1u, 100000000ull);
-  }
-  if (warp < 4 && qi < P && ok) {
-    const float inv = 1.0f / l_run;
-    float4* orow = reinterpret_cast<float4*>(o + static_cast<size_t>(qi) * o_stride + h * DH);
+      tmem_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(o_empty);
+    };
+    for (int j = 0; j < n_kb; ++j) {
+      const int j0 = j * kFaK;
+      const bool full = j0 + kFaK - 1 <= q0 && j0 + kFaK <= P;  // every key visible to every row
+      if (ok && !mbar_wait(&s_full[j & 1], static_cast<uint32_t>(j >> 1) & 1u)) ok = false;
+      tmem_fence_after();
+      const uint32_t ts = tl + static_cast<uint32_t>((j & 1) * kFaK);
+      float sv[2][32];
+      tmem_ld32(ts, sv[0]);
+      tmem_ld32(ts + 32, sv[1]);
+      float bm = -INFINITY;
 #pragma unroll
-    for (int d4 = 0; d4 < DH / 4; ++d4)
-      orow[d4] = make_float4(acc[4 * d4] * inv, acc[4 * d4 + 1] * inv, acc[4 * d4 + 2] * inv, acc[4 * d4 + 3] * inv);
+      for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const int kj = j0 + hf * 32 + c;
+          if (!full && (kj > qi || kj >= P)) sv[hf][c] = -INFINITY;
+          bm = fmaxf(bm, sv[hf][c]);
+        }
+      const float m_new = fmaxf(m_run, bm * sl2);  // scale > 0: the max commutes with it
+      const float alpha = m_run == -INFINITY ? 0.f : exp2f(m_run - m_new);
+      float ls = 0.f;
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+        for (int c = 0; c < 32; ++c) {
+          const float e = sv[hf][c] == -INFINITY ? 0.f : exp2f(fmaf(sv[hf][c], sl2, -m_new));
+          sv[hf][c] = e;
+          ls += e;
+        }
+      tmem_fence_before();
+      if (j >= 1) fold(j - 1);  // O_{j-1} is done, so P_{j-1} has been read: P_j may be written
+#pragma unroll
+      for (int hf = 0; hf < 2; ++hf)
+#pragma unroll
+        for (int c8 = 0; c8 < 4; ++c8) {
+          uint4 hi, lo;
+          split8_bf16(sv[hf] + 8 * c8, hi, lo);
+          const int off = sw128_off(row, hf * 4 + c8);
+          *reinterpret_cast<uint4*>(smem + S::kPh + off) = hi;
+          *reinterpret_cast<uint4*>(smem + S::kPl + off) = lo;
+        }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(p_full);
+      l_run = l_run * alpha + ls;
+      m_run = m_new;
+      alpha_prev = alpha;
+    }
+    if (n_kb > 0) fold(n_kb - 1);
+    if (!ok) set_error(st, DERR_TIMEOUT);
+    if (qi < P && ok) {
+      const float inv = 1.0f / l_run;
+      float4* orow = reinterpret_cast<float4*>(o + static_cast<size_t>(qi) * o_stride + h * DH);
+#pragma unroll
+      for (int d4 = 0; d4 < DH / 4; ++d4)
+        orow[d4] = make_float4(acc[4 * d4] * inv, acc[4 * d4 + 1] * inv, acc[4 * d4 + 2] * inv, acc[4 * d4 + 3] * inv);
+    }
   }
   tmem_fence_before();
   __syncthreads();
-  if (warp == 0) {
+  if (warp == 1) {
     tmem_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kFaTmemCols) : "memory");
   }

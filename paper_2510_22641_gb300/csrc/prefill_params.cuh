@@ -16,6 +16,8 @@ constexpr uint32_t kTcBTile = kTcN * kTcK * 2;             // 16 KB
 constexpr uint32_t kTcStage = 2 * kTcATile + kTcBTile;     // 48 KB
 constexpr int kTcTmemCols = 2 * kTcN;                      // double-buffered fp32 accumulator
 constexpr int kTcSmem = kTcStages * kTcStage + 1024 + 256;  // + alignment slack + barriers
+constexpr int kFaQ = 128;  // prefill attention: query rows per CTA (the MMA's M)
+constexpr int kFaK = 64;   // prefill attention: keys per block (the S MMA's N, the P.V MMA's K)
 
 struct TcParams {
   int M, N, K;          // rows (tokens), output columns, reduction

@@ -383,8 +383,9 @@ def test_launch_counts(tiny_model):
     body = 4 * (1 + 5 * k + 2 + 1) + (1 + 5 * L + 1 + 1)
     # + decode setup, loop begin and copy-out
     assert dec == 3 + st["steps"] * body
-    # prefill: begin + input rows, per layer 4 activation splits + 4 tensor-core GEMMs + attention, head + finish
-    assert pre == 2 + 9 * L + 2
+    # prefill: begin + input rows, per layer 4 activation splits + 4 tensor-core GEMMs + the attention's
+    # operand split + attention, head + finish
+    assert pre == 2 + 10 * L + 2
 
 
 @pytest.mark.parametrize("rows", [1, 5, 9])
