@@ -40,7 +40,7 @@ cudaError_t gemv_attrs_resid();
 cudaError_t gemv_attrs_head();
 cudaError_t gemv_attrs_xattn();
 cudaError_t prefill_attrs();
-cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
+cudaError_t tc_gemm_launch(Epi e, int nt, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
                            cudaStream_t s, bool pdl);
 cudaError_t split_rows_launch(const float* x, int x_stride, int K, const __nv_bfloat16* gain, float eps,
                               __nv_bfloat16* hi, __nv_bfloat16* lo, int rows, cudaStream_t s, bool pdl);
@@ -806,9 +806,14 @@ static ssd_status tc_gemm(ssd_ctx* c, Epi e, int kidx, const TcSite& site, int P
   p.k_steps = site.K / kTcK;
   p.seg_rows = site.seg_rows;
   p.st = c->st;
-  const int tiles = p.tiles_m * p.tiles_n;
+  // 256-column tiles (each A slice feeds two 128-column weight tiles, halving the A traffic per flop)
+  // where they still give every SM a tile
+  const int wide_tiles = p.tiles_m * ((p.tiles_n + 1) / 2);
+  const int nt = (e == Epi::QKV || e == Epi::GATE_SILU) && wide_tiles >= c->num_sms ? 256 : 128;
+  const int tiles = nt == 256 ? wide_tiles : p.tiles_m * p.tiles_n;
   CK(count_launch(c));
-  CK(tc_gemm_launch(e, c->a_maps[kidx], site.maps, p, tiles < c->num_sms ? tiles : c->num_sms, c->cs, c->use_pdl));
+  CK(tc_gemm_launch(e, nt, c->a_maps[kidx], site.maps, p, tiles < c->num_sms ? tiles : c->num_sms, c->cs,
+                    c->use_pdl));
   return SSD_OK;
 }
 

@@ -19,14 +19,16 @@ static cudaError_t launch_pdl(Kern kern, dim3 grid, dim3 block, size_t smem, cud
   return cudaLaunchKernelEx(&cfg, kern, args...);
 }
 
+template <Epi EPI, int NT>
+static cudaError_t tc_attr() {
+  return cudaFuncSetAttribute(ssd_prefill_tc_kernel<EPI, NT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              TcShape<NT>::kSmem);
+}
+
 cudaError_t prefill_attrs() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::QKV>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
-    return e;
-  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::GATE_SILU>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                kTcSmem)))
-    return e;
-  if ((e = cudaFuncSetAttribute(ssd_prefill_tc_kernel<Epi::RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcSmem)))
+  if ((e = tc_attr<Epi::QKV, 128>()) || (e = tc_attr<Epi::QKV, 256>()) || (e = tc_attr<Epi::GATE_SILU, 128>()) ||
+      (e = tc_attr<Epi::GATE_SILU, 256>()) || (e = tc_attr<Epi::RESID, 128>()))
     return e;
   if ((e = cudaFuncSetAttribute(ssd_prefill_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 FaSmem<128>::kTotal)))
@@ -35,16 +37,24 @@ cudaError_t prefill_attrs() {
                               FaSmem<64>::kTotal);
 }
 
-cudaError_t tc_gemm_launch(Epi e, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
+// nt: output tile width, 128 or 256 (QKV and gate/up only).
+cudaError_t tc_gemm_launch(Epi e, int nt, const CUtensorMap* a, const CUtensorMap* b, const TcParams& p, int grid,
                            cudaStream_t s, bool pdl) {
   const dim3 g(grid), blk(kTcThreads);
   switch (e) {
     case Epi::QKV:
-      return launch_pdl(ssd_prefill_tc_kernel<Epi::QKV>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return nt == 256 ? launch_pdl(ssd_prefill_tc_kernel<Epi::QKV, 256>, g, blk, TcShape<256>::kSmem, s, pdl, a[0],
+                                    a[1], b[0], b[1], b[2], p)
+                       : launch_pdl(ssd_prefill_tc_kernel<Epi::QKV, 128>, g, blk, TcShape<128>::kSmem, s, pdl, a[0],
+                                    a[1], b[0], b[1], b[2], p);
     case Epi::GATE_SILU:
-      return launch_pdl(ssd_prefill_tc_kernel<Epi::GATE_SILU>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return nt == 256 ? launch_pdl(ssd_prefill_tc_kernel<Epi::GATE_SILU, 256>, g, blk, TcShape<256>::kSmem, s, pdl,
+                                    a[0], a[1], b[0], b[1], b[2], p)
+                       : launch_pdl(ssd_prefill_tc_kernel<Epi::GATE_SILU, 128>, g, blk, TcShape<128>::kSmem, s, pdl,
+                                    a[0], a[1], b[0], b[1], b[2], p);
     case Epi::RESID:
-      return launch_pdl(ssd_prefill_tc_kernel<Epi::RESID>, g, blk, kTcSmem, s, pdl, a[0], a[1], b[0], b[1], b[2], p);
+      return launch_pdl(ssd_prefill_tc_kernel<Epi::RESID, 128>, g, blk, TcShape<128>::kSmem, s, pdl, a[0], a[1], b[0],
+                        b[1], b[2], p);
     default:
       return cudaErrorInvalidValue;
   }

@@ -130,27 +130,33 @@ __device__ __forceinline__ void tc_epilogue_row(const TcParams& p, int n_t, int 
   }
 }
 
-template <Epi EPI>
+// p.tiles_n counts 128-column sub-tiles; a CTA tile is NT columns (kSub sub-tiles, the last one of a
+// row of tiles possibly past the end, then neither loaded nor stored).
+template <Epi EPI, int NT>
 __global__ void __launch_bounds__(kTcThreads, 1)
     ssd_prefill_tc_kernel(const __grid_constant__ CUtensorMap map_ahi, const __grid_constant__ CUtensorMap map_alo,
                    const __grid_constant__ CUtensorMap map_b0, const __grid_constant__ CUtensorMap map_b1,
                    const __grid_constant__ CUtensorMap map_b2, const TcParams p) {
+  using TS = TcShape<NT>;
+  constexpr int kStagesT = TS::kStages;
+  constexpr uint32_t kStageT = TS::kStage;
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   // 1024-byte aligned base for the swizzled tiles
   const uint32_t raw = smem_u32(smem_raw);
   uint8_t* smem = smem_raw + (((raw + 1023u) & ~1023u) - raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kTcStages * kTcStage);
-  uint64_t* empty = full + kTcStages;
-  uint64_t* tfull = empty + kTcStages;   // [2]
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + kStagesT * kStageT);
+  uint64_t* empty = full + kStagesT;
+  uint64_t* tfull = empty + kStagesT;     // [2]
   uint64_t* tempty = tfull + 2;          // [2]
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tempty + 2);
   int* abort_flag = reinterpret_cast<int*>(tmem_slot + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n_tiles = p.tiles_m * p.tiles_n;
+  const int tiles_nt = (p.tiles_n + TS::kSub - 1) / TS::kSub;  // NT-column tiles
+  const int n_tiles = p.tiles_m * tiles_nt;
 
   pdl_trigger();
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kTcStages; ++s) {
+    for (int s = 0; s < kStagesT; ++s) {
       mbar_init(&full[s], 1);
       mbar_init(&empty[s], 1);
     }
@@ -161,9 +167,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 1) {  // TMEM: 2 x 128 fp32 columns
+  if (warp == 1) {  // TMEM: 2 x NT fp32 columns
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(tmem_slot)),
-                 "r"(kTcTmemCols)
+                 "r"(TS::kTmemCols)
                  : "memory");
     asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
   }
@@ -178,28 +184,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     if (lane == 0) {
       int g = 0;
       for (int t = blockIdx.x; t < n_tiles && !*reinterpret_cast<volatile int*>(abort_flag); t += gridDim.x) {
-        const int m_t = t % p.tiles_m, n_t = t / p.tiles_m;
+        const int m_t = t % p.tiles_m, n_t0 = (t / p.tiles_m) * TS::kSub;
+        const int n_sub = min(TS::kSub, p.tiles_n - n_t0);  // sub-tiles inside the matrix
         for (int ks = 0; ks < p.k_steps; ++ks, ++g) {
-          const int s = g % kTcStages;
-          if (!mbar_wait(&empty[s], ((g / kTcStages) & 1) ^ 1)) {
+          const int s = g % kStagesT;
+          if (!mbar_wait(&empty[s], ((g / kStagesT) & 1) ^ 1)) {
             set_error(p.st, DERR_TIMEOUT);
             *reinterpret_cast<volatile int*>(abort_flag) = 1;
             break;
           }
-          uint8_t* st = smem + s * kTcStage;
-          mbar_arrive_expect_tx(&full[s], kTcStage);
+          uint8_t* st = smem + s * kStageT;
+          mbar_arrive_expect_tx(&full[s], 2 * kTcATile + n_sub * kTcBTile);
           const int kx = ks * kTcK;
           tma_load_2d(st, &map_ahi, &full[s], kx, m_t * kTcM);
           tma_load_2d(st + kTcATile, &map_alo, &full[s], kx, m_t * kTcM);
-          uint8_t* bs = st + 2 * kTcATile;
-          if constexpr (EPI == Epi::GATE_SILU) {
-            tma_load_2d(bs, &map_b0, &full[s], kx, n_t * (kTcN / 2));
-            tma_load_2d(bs + kTcBTile / 2, &map_b1, &full[s], kx, n_t * (kTcN / 2));
-          } else if constexpr (EPI == Epi::QKV) {
-            const int r0 = n_t * kTcN, mat = r0 / p.seg_rows;
-            tma_load_2d(bs, mat == 0 ? &map_b0 : (mat == 1 ? &map_b1 : &map_b2), &full[s], kx, r0 - mat * p.seg_rows);
-          } else {
-            tma_load_2d(bs, &map_b0, &full[s], kx, n_t * kTcN);
+          for (int sub = 0; sub < n_sub; ++sub) {
+            const int n_t = n_t0 + sub;
+            uint8_t* bs = st + 2 * kTcATile + sub * kTcBTile;
+            if constexpr (EPI == Epi::GATE_SILU) {
+              tma_load_2d(bs, &map_b0, &full[s], kx, n_t * (kTcN / 2));
+              tma_load_2d(bs + kTcBTile / 2, &map_b1, &full[s], kx, n_t * (kTcN / 2));
+            } else if constexpr (EPI == Epi::QKV) {
+              const int r0 = n_t * kTcN, mat = r0 / p.seg_rows;
+              tma_load_2d(bs, mat == 0 ? &map_b0 : (mat == 1 ? &map_b1 : &map_b2), &full[s], kx, r0 - mat * p.seg_rows);
+            } else {
+              tma_load_2d(bs, &map_b0, &full[s], kx, n_t * kTcN);
+            }
           }
         }
       }
@@ -207,7 +217,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = umma_idesc_bf16(kTcM, kTcN);
+      constexpr uint32_t idesc = umma_idesc_bf16(kTcM, NT);
       int g = 0, it = 0;
       for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
         const int b = it & 1;
@@ -217,18 +227,18 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           break;
         }
         tmem_fence_after();
-        const uint32_t d = tmem + b * kTcN;
+        const uint32_t d = tmem + b * NT;
         bool ok = true;
         for (int ks = 0; ks < p.k_steps; ++ks, ++g) {
-          const int s = g % kTcStages;
-          if (!mbar_wait(&full[s], (g / kTcStages) & 1)) {
+          const int s = g % kStagesT;
+          if (!mbar_wait(&full[s], (g / kStagesT) & 1)) {
             set_error(p.st, DERR_TIMEOUT);
             *reinterpret_cast<volatile int*>(abort_flag) = 1;
             ok = false;
             break;
           }
           tmem_fence_after();
-          const uint32_t sa = smem_u32(smem + s * kTcStage);
+          const uint32_t sa = smem_u32(smem + s * kStageT);
           const uint64_t ahi = umma_desc_sw128(sa), alo = umma_desc_sw128(sa + kTcATile),
                          bw = umma_desc_sw128(sa + 2 * kTcATile);
 #pragma unroll
@@ -249,28 +259,32 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     int it = 0;
     for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++it) {
       const int b = it & 1;
-      const int m_t = t % p.tiles_m, n_t = t / p.tiles_m;
+      const int m_t = t % p.tiles_m, n_t0 = (t / p.tiles_m) * TS::kSub;
       if (!mbar_wait(&tfull[b], (it >> 1) & 1)) {
         set_error(p.st, DERR_TIMEOUT);
         break;
       }
       tmem_fence_after();
-      float acc[kTcN];
-      const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + b * kTcN;
+      const int r = m_t * kTcM + q * 32 + lane;
+#pragma unroll 1
+      for (int sub = 0; sub < TS::kSub; ++sub) {
+        if (n_t0 + sub >= p.tiles_n) break;
+        float acc[kTcN];
+        const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + b * NT + sub * kTcN;
 #pragma unroll
-      for (int c = 0; c < kTcN / 32; ++c) tmem_ld32(base + c * 32, acc + c * 32);
+        for (int c = 0; c < kTcN / 32; ++c) tmem_ld32(base + c * 32, acc + c * 32);
+        if (r < p.M) tc_epilogue_row<EPI>(p, n_t0 + sub, r, acc);
+      }
       tmem_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty[b]);  // accumulator b may be overwritten
-      const int r = m_t * kTcM + q * 32 + lane;
-      if (r < p.M) tc_epilogue_row<EPI>(p, n_t, r, acc);
     }
   }
   tmem_fence_before();
   __syncthreads();
   if (warp == 1) {
     tmem_fence_after();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTcTmemCols) : "memory");
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(TS::kTmemCols) : "memory");
   }
 }
 

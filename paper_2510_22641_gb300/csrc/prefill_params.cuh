@@ -16,6 +16,17 @@ constexpr uint32_t kTcBTile = kTcN * kTcK * 2;             // 16 KB
 constexpr uint32_t kTcStage = 2 * kTcATile + kTcBTile;     // 48 KB
 constexpr int kTcTmemCols = 2 * kTcN;                      // double-buffered fp32 accumulator
 constexpr int kTcSmem = kTcStages * kTcStage + 1024 + 256;  // + alignment slack + barriers
+
+// The GEMM templated on its output tile width NT (128, or 256 = two 128-column sub-tiles sharing each
+// A slice): ring stages, stage bytes, TMEM columns (double-buffered accumulator) and shared memory.
+template <int NT>
+struct TcShape {
+  static constexpr int kSub = NT / kTcN;                              // 128-column sub-tiles
+  static constexpr int kStages = NT == kTcN ? kTcStages : 3;
+  static constexpr uint32_t kStage = 2 * kTcATile + kSub * kTcBTile;  // A hi, A lo, the sub-tiles' W
+  static constexpr int kTmemCols = 2 * NT;
+  static constexpr int kSmem = kStages * kStage + 1024 + 256;
+};
 constexpr int kFaQ = 128;  // prefill attention: query rows per CTA (the MMA's M)
 constexpr int kFaK = 64;   // prefill attention: keys per block (the S MMA's N, the P.V MMA's K)
 
