@@ -18,7 +18,11 @@
 // accumulators summed in warp order.  Each CTA stores its state and takes the
 // head's ticket (one acq_rel atomic after a CTA barrier); the CTA that completes
 // the count merges the kAttnSplit states in CTA order and writes the head's
-// output, so the other CTAs leave without waiting for each other.  The chunk
+// output, so the other CTAs leave without waiting for each other.  When all of
+// a head's keys fit one chunk (short caches: the encoder-decoder's decoder,
+// early positions) CTA 0 holds the whole state and writes the output itself,
+// with no state store, ticket or merge: the merge would return that state's
+// O / L unchanged, so the result is the same bits.  The chunk
 // grid, the grouping, the key -> (CTA, warp)
 // assignment and every summation order depend only on key positions, never on
 // M, so each row's output equals the single-row (M = 1) result bitwise.
@@ -72,6 +76,11 @@ struct AttnParams {
   int batch_rows;
   const DevState* req_st;
   long long req_kv;
+  // Null, or the merged output rows also go out as bf16 hi / lo parts, [request * M + row][xo_ld]
+  // (the medium-M o projection's operand, so it needs no split launch of its own).
+  __nv_bfloat16* xo_hi;
+  __nv_bfloat16* xo_lo;
+  int xo_ld;
 };
 
 template <int DH>
@@ -362,6 +371,31 @@ __global__ void __launch_bounds__(kAttnThreads, M <= 9 ? 2 : 1) ssd_splitkv_attn
 #pragma unroll
     for (int e = 0; e < DPL; ++e) ws[(w * M + m) * DH + lane * DPL + e] = acc[m][e];
   __syncthreads();
+  // one output element of row m, with its bf16 parts for a medium-M o projection when asked
+  auto put = [&](int m, int d, float ov) {
+    o_rows[m * p.o_stride + h * DH + d] = ov;
+    if (p.xo_hi) {
+      const size_t i = (static_cast<size_t>(z) * M + m) * p.xo_ld + h * DH + d;
+      const __nv_bfloat16 oh = __float2bfloat16_rn(ov);
+      p.xo_hi[i] = oh;
+      p.xo_lo[i] = __float2bfloat16_rn(ov - __bfloat162float(oh));
+    }
+  };
+  if (n_keys <= KPC) {
+    // At most one chunk, CTA 0's: its state is the head's and the merge would return it unchanged
+    // (weight exp(0) = 1 on it, 0 on the empty states), so CTA 0 writes O / L itself and no CTA
+    // takes the ticket.
+    if (rank == 0 && ok && !bad && !timed_out)
+      for (int idx = tid; idx < M * DH; idx += kAttnThreads) {
+        const int m = idx / DH, d = idx - m * DH;
+        float O = 0.f;
+#pragma unroll
+        for (int q = 0; q < kAttnWarps; ++q) O += ws[(q * M + m) * DH + d];
+        const float L = rowst[4 * m + 1];
+        put(m, d, L > 0.f ? O / L : 0.f);
+      }
+    return;
+  }
   constexpr int kSlot = kAttnMaxRows * E;  // one CTA state in part
   const int zh = z * p.n_heads + h;  // this request's head
   float* head_part = p.part + static_cast<size_t>(zh) * kAttnSplit * kSlot;
@@ -423,7 +457,7 @@ __global__ void __launch_bounds__(kAttnThreads, M <= 9 ? 2 : 1) ssd_splitkv_attn
 #pragma unroll
         for (int q = 0; q < kAttnSplit; ++q) O = fmaf(wq[m * kAttnSplit + q], v[e][q], O);
         const float L = wq[M * kAttnSplit + m];
-        o_rows[m * p.o_stride + h * DH + d] = L > 0.f ? O / L : 0.f;
+        put(m, d, L > 0.f ? O / L : 0.f);
       }
     }
     if (tid == 0) p.tickets[zh] = 0u;

@@ -102,6 +102,13 @@ __device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, ui
   }
 }
 
+// After a wait gave up: the copies a ring's producer issued for its last `issued` fills (stage
+// i % stages, phase i / stages) may still be landing; a bounded wait for each before the CTA leaves.
+__device__ __forceinline__ void drain_ring(uint64_t* full, int stages, int issued) {
+  for (int i = issued > stages ? issued - stages : 0; i < issued; ++i)
+    mbar_wait_for(&full[i % stages], static_cast<uint32_t>(i / stages) & 1u, 100000000ull);
+}
+
 // The library's bounded wait: gives up after ~2 s.
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
   return mbar_wait_for(bar, parity, 2000000000ull);

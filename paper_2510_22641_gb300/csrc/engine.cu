@@ -149,6 +149,16 @@ struct ssd_ctx {
   __nv_bfloat16 *act_hi = nullptr, *act_lo = nullptr;  // split activations [kMaxMidRows][act_ld] (medium-M)
   float* act_rs = nullptr;       // [kMaxMidRows] RMSNorm scales of the split rows
   int act_ld = 0;
+  // The next medium-M projection's operand as its producer left it in act_hi / act_lo (the attention
+  // merge, or a medium-M reduction's epilogue), so that projection needs no split launch: valid
+  // while act_ready, for the rows act_x (act_m of them), act_k columns, RMSNorm gain act_gain, with
+  // the rows' sums of squares per producer tile in act_ssq[row][act_parts] (act_parts 0: none).
+  float* act_ssq = nullptr;
+  int act_ssq_ld = 0;
+  bool act_ready = false;
+  const float* act_x = nullptr;
+  int act_m = 0, act_k = 0, act_parts = 0;
+  const __nv_bfloat16* act_gain = nullptr;
   float* mid_partials = nullptr;  // [2 * grid][kMaxMidRows][kTileN]
   std::map<std::pair<int, int>, std::pair<CUtensorMap, CUtensorMap>> act_maps;  // (K, NP) -> hi, lo
   std::map<int, cudaGraphExec_t> batch_graphs;  // decode loops by gamma (0: greedy), for batch_graph_b requests
@@ -1004,13 +1014,52 @@ static ssd_status act_maps_for(ssd_ctx* c, int K, int NP, const CUtensorMap** ou
   return SSD_OK;
 }
 
+// The medium-M projection that reads the output of the one being enqueued: its rows x, columns K and
+// RMSNorm gain, and whether it needs the rows' sums of squares (it has a gain).
+struct NextSplit {
+  const float* x;
+  int K;
+  const __nv_bfloat16* gain;
+};
+
+// Records that act_hi / act_lo now hold the operand of the projection nx describes over M rows.
+static void set_act_ready(ssd_ctx* c, const NextSplit& nx, int M, int parts) {
+  c->act_ready = true;
+  c->act_x = nx.x;
+  c->act_m = M;
+  c->act_k = nx.K;
+  c->act_gain = nx.gain;
+  c->act_parts = parts;
+}
+
 // One projection over M > kMaxRows rows: the rows are split into bf16 hi / lo parts with their
 // RMSNorm scales (gain folded in), then the medium-M tensor-core kernel streams the weights once.
-static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p) {
+// The split launch is skipped when the producing kernel already wrote this projection's parts
+// (act_ready for the same rows, width and gain); with nx, this projection's reduction writes the
+// next one's parts (and, when that one has a gain, the rows' sums of squares per output tile).
+static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p, const NextSplit* nx = nullptr) {
   if (M > kMaxMidRows || !c->act_hi) return fail(c, SSD_ERR_INVALID_ARG, "%d rows exceed the medium-M kernel", M);
-  CK(count_launch(c));
-  CK(split_act_launch(p.x, p.x_stride, s.K, p.gain, c->cfg.rms_eps, c->act_hi, c->act_lo, s.K, c->act_rs, M, c->cs,
-                      c->use_pdl));
+  const bool fused = c->act_ready && c->act_x == p.x && c->act_m == M && c->act_k == s.K && c->act_gain == p.gain &&
+                     (p.gain == nullptr || c->act_parts > 0);
+  c->act_ready = false;
+  if (fused) {
+    p.rs_parts = p.gain ? c->act_ssq : nullptr;
+    p.rs_nparts = p.gain ? c->act_parts : 0;
+  } else {
+    CK(count_launch(c));
+    CK(split_act_launch(p.x, p.x_stride, s.K, p.gain, c->cfg.rms_eps, c->act_hi, c->act_lo, s.K, c->act_rs, M, c->cs,
+                        c->use_pdl));
+    p.rs_in = c->act_rs;
+  }
+  if (nx) {
+    if (nx->K > c->act_ld || (nx->gain && (e != Epi::RESID || s.n_rt > c->act_ssq_ld || p.rs_parts)))
+      return fail(c, SSD_ERR_INVALID_ARG, "no fused split for this projection pair");
+    p.nx_hi = c->act_hi;
+    p.nx_lo = c->act_lo;
+    p.nx_ld = nx->K;
+    p.nx_gain = nx->gain;
+    p.nx_ssq = nx->gain ? c->act_ssq : nullptr;
+  }
   CUtensorMap amaps[2];
   const CUtensorMap* am = nullptr;
   CKS(act_maps_for(c, s.K, (M + 15) & ~15, &am));
@@ -1026,16 +1075,21 @@ static ssd_status mid_gemm(ssd_ctx* c, Epi e, int M, const Site& s, GemvParams p
   p.counters = c->counters;
   p.st = c->st;
   p.eps = c->cfg.rms_eps;
-  p.rs_in = c->act_rs;
   CK(count_launch(c));  // the stream
   CK(count_launch(c));  // the reduction + epilogue
   CK(mid_launch(e, s.maps, amaps, p, M, c->num_sms, c->cs, c->use_pdl));
+  if (nx) set_act_ready(c, *nx, M, nx->gain ? s.n_rt : 0);
   return SSD_OK;
 }
 
 // A projection over M rows of the batch: the GEMV up to kMaxRows rows, the medium-M kernel beyond.
-static ssd_status proj_rows(ssd_ctx* c, Epi e, int M, const Site& s, const GemvParams& p) {
-  return M <= kMaxRows ? gemv(c, e, M, s, p) : mid_gemm(c, e, M, s, p);
+static ssd_status proj_rows(ssd_ctx* c, Epi e, int M, const Site& s, const GemvParams& p,
+                            const NextSplit* nx = nullptr) {
+  if (M <= kMaxRows) {
+    c->act_ready = false;
+    return gemv(c, e, M, s, p);
+  }
+  return mid_gemm(c, e, M, s, p, nx);
 }
 
 static void set_batch_rows(ssd_ctx* c, GemvParams& p, int R) {
@@ -1077,7 +1131,23 @@ static ssd_status enqueue_layer_batch(ssd_ctx* c, int l, float* x, int x_stride,
   a.batch_rows = R;
   a.req_st = c->req;
   a.req_kv = static_cast<long long>(c->req_kv);
+  // Medium-M rows: each kernel also writes the next projection's bf16 operand parts, so only the
+  // first projection of a pass runs the split launch (o reads the attention's parts, gate/up the
+  // o reduction's, down the gate/up reduction's, the next layer's q/k/v or the head the down's).
+  const bool mid = M > kMaxRows && c->act_hi;
+  const NextSplit o_in{c->ob, c->layers[l].o.K, nullptr};
+  if (mid) {
+    a.xo_hi = c->act_hi;
+    a.xo_lo = c->act_lo;
+    a.xo_ld = o_in.K;
+  }
+  c->act_ready = false;
   CKS(attn_run(c, R, a, M / R));
+  if (mid) set_act_ready(c, o_in, M, 0);
+  const NextSplit gate_in{x, c->layers[l].gateup.K, c->ffn_norm[l]};
+  const NextSplit down_in{c->hb, c->layers[l].down.K, nullptr};
+  const bool last = l + 1 >= c->cfg.n_layers;
+  const NextSplit next_in{x, last ? c->head.K : c->layers[l + 1].qkv.K, last ? c->final_norm : c->attn_norm[l + 1]};
   p = GemvParams{};
   p.x = c->ob;
   p.x_stride = c->qp;
@@ -1086,14 +1156,14 @@ static ssd_status enqueue_layer_batch(ssd_ctx* c, int l, float* x, int x_stride,
   p.dst = x;
   p.dst_stride = x_stride;
   p.scale = resid_scale_of(c, l);
-  CKS(proj_rows(c, Epi::RESID, M, c->layers[l].o, p));
+  CKS(proj_rows(c, Epi::RESID, M, c->layers[l].o, p, &gate_in));
   p = GemvParams{};
   p.x = x;
   p.x_stride = x_stride;
   p.gain = c->ffn_norm[l];
   p.h_out = c->hb;
   p.h_stride = c->fp;
-  CKS(proj_rows(c, Epi::GATE_SILU, M, c->layers[l].gateup, p));
+  CKS(proj_rows(c, Epi::GATE_SILU, M, c->layers[l].gateup, p, &down_in));
   p = GemvParams{};
   p.x = c->hb;
   p.x_stride = c->fp;
@@ -1102,7 +1172,7 @@ static ssd_status enqueue_layer_batch(ssd_ctx* c, int l, float* x, int x_stride,
   p.dst = x;
   p.dst_stride = x_stride;
   p.scale = resid_scale_of(c, l);
-  return proj_rows(c, Epi::RESID, M, c->layers[l].down, p);
+  return proj_rows(c, Epi::RESID, M, c->layers[l].down, p, &next_in);
 }
 
 // LM head + argmax over M = B * R rows x: row (b, i) writes its token to tok0[b][i] (tok0 a field of
@@ -1169,6 +1239,7 @@ static ssd_status enqueue_draft_batch(ssd_ctx* c, int gamma) {
 static ssd_status enqueue_verify_batch(ssd_ctx* c, int gamma, cudaGraphConditionalHandle cond, int has_cond) {
   const int B = c->batch, d = c->dp, R = gamma + 1, rs = R * c->dp;
   float* xg = c->xv + static_cast<size_t>(gamma) * d;
+  c->act_ready = false;
   CK(launch_k(c, ssd_batch_embed_kernel, dim3(B), dim3(256), 0, c->embed, static_cast<const DevState*>(c->req),
               gamma, xg, rs, c->cfg.d_model, c->cfg.vocab, c->st));
   for (int l = 0; l < c->cfg.draft_exit_k; ++l) CKS(enqueue_layer_batch(c, l, xg, rs, B, 1, gamma));
@@ -1838,6 +1909,9 @@ static ssd_status create_impl(ssd_ctx* c, const ssd_config* cfg, const ssd_weigh
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_hi), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_lo), sizeof(__nv_bfloat16) * kMaxMidRows * kmax));
       CKS(alloc(c, reinterpret_cast<void**>(&c->act_rs), sizeof(float) * kMaxMidRows));
+      c->act_ld = static_cast<int>(kmax);
+      c->act_ssq_ld = static_cast<int>((kmax + kTileN - 1) / kTileN);
+      CKS(alloc(c, reinterpret_cast<void**>(&c->act_ssq), sizeof(float) * kMaxMidRows * c->act_ssq_ld));
       // partials: one slot per (streaming CTA, row tile) pair, c + rt
       CKS(alloc(c, reinterpret_cast<void**>(&c->mid_partials),
                 sizeof(float) * (mid_max_ctas(c->num_sms) + c->n_counters) * kMaxMidRows * kTileN));
@@ -2618,6 +2692,7 @@ ssd_status ssd_profile_projection(ssd_ctx* c, int which, int layer, int rows, in
     *bytes = N * site->K * 2 + static_cast<int64_t>(rows) * site->K * 4 + (p.gain ? site->K * 2 : 0) + out_bytes +
              (e == Epi::RESID ? static_cast<int64_t>(rows) * site->N * 4 : 0);
   CKS(enter(c));
+  c->act_ready = false;
   for (int r = 0; r < reps; ++r) CKS(proj_rows(c, e, rows, *site, p));
   c->prefilled = false;
   c->batch = 0;

@@ -112,6 +112,18 @@ struct GemvParams {
   // Medium-M kernel only: the rows' RMSNorm scales 1/rms(x_m), computed by the split kernel
   // (the gain is folded into its bf16 hi/lo parts).
   const float* rs_in;
+  // Medium-M, when the producing kernel has already split this launch's rows: their sums of squares
+  // per 128-column tile of the producer, [row][rs_nparts], summed here in tile order for 1/rms.
+  const float* rs_parts;
+  int rs_nparts;
+  // Medium-M reduction as the producer of the next medium-M projection's input (nx_hi null: none):
+  // the RESID / GATE_SILU outputs also go out as bf16 parts of value * nx_gain[n] (no gain: value),
+  // [row][nx_ld], and RESID rows' sums of squares per tile to nx_ssq[row][n_rt].
+  __nv_bfloat16* nx_hi;
+  __nv_bfloat16* nx_lo;
+  int nx_ld;
+  const __nv_bfloat16* nx_gain;
+  float* nx_ssq;
   int grid_ctas;  // medium-M reduction: the CTAs of the streaming launch
   int abs_pos;   // row m sits at position pos_off + m, st->kv_len ignored (the encoder's rows)
   int act;       // GATE_SILU: 0 = SiLU(gate) * up, 1 = GELU_tanh(gate) * up (gated GELU)
@@ -168,6 +180,12 @@ __device__ __forceinline__ int unit_begin(int c, int units, int G) {
 // and the request of launch row m instead (rpos is null for one request).
 
 __device__ __forceinline__ void drain_sync() { named_bar_sync(1, kDrainThreads); }
+
+// The medium-M RESID epilogue's per-warp sums of squares of a tile's rows, [drain warp][row].
+__device__ __forceinline__ float* argmax_warp_ssq() {
+  __shared__ float sq[(kDrainThreads / 32) * kNPad];
+  return sq;
+}
 
 // The LM head epilogue's per-warp argmax keys of a tile's rows, [drain warp][row] (16 rows).
 __device__ __forceinline__ unsigned long long* argmax_warp_keys() {
@@ -261,7 +279,9 @@ __device__ __forceinline__ void gemv_cross_attention(const GemvParams& p, int rt
   }
 }
 
-template <int MT, Epi EPI>
+// NX: the medium-M reduction's instance, which may also write the next projection's operand parts
+// (GemvParams nx_*); the GEMV's instances compile without that code.
+template <int MT, Epi EPI, bool NX = false>
 __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const float* out, const float* rs,
                                               const float* pre, int base_pos, const int* rpos, const int* rreq,
                                               int tid, int m0, int mc) {
@@ -342,7 +362,13 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
       if (n >= p.N) continue;
       const float g = out[m * kTileN + j] * rs[m];
       const float u = out[m * kTileN + kHalfN + j] * rs[m];
-      p.h_out[(m0 + m) * p.h_stride + n] = (p.act ? gelu_tanh_f(g) : silu_f(g)) * u;
+      const float hv = (p.act ? gelu_tanh_f(g) : silu_f(g)) * u;
+      p.h_out[(m0 + m) * p.h_stride + n] = hv;
+      if (NX && p.nx_hi) {
+        const __nv_bfloat16 hh = __float2bfloat16_rn(hv);
+        p.nx_hi[(m0 + m) * p.nx_ld + n] = hh;
+        p.nx_lo[(m0 + m) * p.nx_ld + n] = __float2bfloat16_rn(hv - __bfloat162float(hh));
+      }
     }
   } else if constexpr (EPI == Epi::SILU) {
     for (int idx = tid; idx < mc * kTileN; idx += kDrainThreads) {
@@ -357,6 +383,9 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
     static_assert(kDrainThreads == kTileN, "one thread per tile column");
     const float s = __ldg(p.scale);
     const int n = rt * kTileN + tid;
+    float xv[MT];
+#pragma unroll
+    for (int m = 0; m < MT; ++m) xv[m] = 0.f;
     if (n < p.N) {
       float bv[MT];
 #pragma unroll
@@ -364,7 +393,36 @@ __device__ __forceinline__ void gemv_epilogue(const GemvParams& p, int rt, const
         if (m < mc) bv[m] = pre ? pre[m * kTileN + tid] : __ldcg(p.base + (m0 + m) * p.base_stride + n);
 #pragma unroll
       for (int m = 0; m < MT; ++m)
-        if (m < mc) p.dst[(m0 + m) * p.dst_stride + n] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
+        if (m < mc) {
+          xv[m] = bv[m] + s * (out[m * kTileN + tid] * rs[m]);
+          p.dst[(m0 + m) * p.dst_stride + n] = xv[m];
+        }
+      if (NX && p.nx_hi) {  // the next projection's input parts: x * gain
+        const float gn = p.nx_gain ? __bfloat162float(p.nx_gain[n]) : 1.0f;
+#pragma unroll
+        for (int m = 0; m < MT; ++m)
+          if (m < mc) {
+            const float v = xv[m] * gn;
+            const __nv_bfloat16 hh = __float2bfloat16_rn(v);
+            p.nx_hi[(m0 + m) * p.nx_ld + n] = hh;
+            p.nx_lo[(m0 + m) * p.nx_ld + n] = __float2bfloat16_rn(v - __bfloat162float(hh));
+          }
+      }
+    }
+    if (NX && p.nx_ssq) {  // the rows' sums of squares over this tile: warps, then the 4 warps in order
+      float* red = argmax_warp_ssq();
+      const int lane = tid & 31, w = tid >> 5;
+#pragma unroll
+      for (int m = 0; m < MT; ++m) {
+        float q = xv[m] * xv[m];
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) q += __shfl_xor_sync(0xffffffffu, q, off);
+        if (lane == 0) red[w * kNPad + m] = q;
+      }
+      drain_sync();
+      if (tid < mc)
+        p.nx_ssq[(m0 + tid) * p.n_rt + rt] = ((red[tid] + red[kNPad + tid]) + red[2 * kNPad + tid]) + red[3 * kNPad + tid];
+      drain_sync();
     }
   } else {  // ARGMAX (LM head): this tile's keys of the rows; gemv_argmax_finish turns them into tokens
     const int lane = tid & 31;
@@ -534,7 +592,8 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
       pdl_wait();
       if (p.late_trigger) pdl_trigger();
       for (int i = 0; i < npre; ++i) issue_acts(i, u0 + i);
-      for (int i = npre; i < n_units; ++i) {
+      int issued = npre;
+      for (int i = npre; i < n_units; ++i, ++issued) {
         const int s = i % kStages;
         if (!mbar_wait(&empty[s], static_cast<uint32_t>((i / kStages) - 1) & 1u)) {
           set_error(p.st, DERR_TIMEOUT);
@@ -544,6 +603,7 @@ __global__ void __launch_bounds__(kGemvThreads, 2)
         issue_weights(s, u0 + i);
         issue_acts(s, u0 + i);
       }
+      if (__ldcg(&p.st->error) & DERR_TIMEOUT) drain_ring(full, kStages, issued);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer

@@ -196,7 +196,8 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
       };
       prefetch_tensormap(&map0);
       // weights do not depend on the previous kernel: the first stages go out before its end
-      for (int i = 0; i < n_units; ++i) {
+      int issued = 0;
+      for (int i = 0; i < n_units; ++i, ++issued) {
         const int s = i % kMidWStages;
         if (i >= kMidWStages && !mbar_wait(&wempty[s], static_cast<uint32_t>((i / kMidWStages) - 1) & 1u)) {
           set_error(p.st, DERR_TIMEOUT);
@@ -204,6 +205,7 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         }
         issue_weights(s, u0 + i);
       }
+      if (__ldcg(&p.st->error) & DERR_TIMEOUT) drain_ring(wfull, kMidWStages, issued);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -254,7 +256,8 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
       const uint32_t bbytes = static_cast<uint32_t>(NP) * kTileK * 2;
       pdl_wait();  // the split kernel's rows
       if (p.late_trigger) pdl_trigger();
-      for (int i = 0; i < n_units; ++i) {
+      int issued = 0;
+      for (int i = 0; i < n_units; ++i, ++issued) {
         const int sb = i % kMidBStages;
         if (i >= kMidBStages && !mbar_wait(&bempty[sb], static_cast<uint32_t>((i / kMidBStages) - 1) & 1u)) {
           set_error(p.st, DERR_TIMEOUT);
@@ -265,6 +268,7 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         tma_load_2d(smem + S::kBh + sb * kMidBBytes, &map_hi, &bfull[sb], x, 0);
         tma_load_2d(smem + S::kBl + sb * kMidBBytes, &map_lo, &bfull[sb], x, 0);
       }
+      if (__ldcg(&p.st->error) & DERR_TIMEOUT) drain_ring(bfull, kMidBStages, issued);
     }
   } else {
     // ---------------------------------------------------------------- drain (warps 2..5)
@@ -335,7 +339,27 @@ __global__ void __launch_bounds__(kDrainThreads) ssd_mid_reduce_kernel(const Gem
       rreq[m] = b;
       rpos[m] = __ldcg(&p.req_st[b].kv_len) + batch_offset(p, m, b);
     }
-  if (tid < mc) rs[tid] = p.rs_in ? __ldcg(p.rs_in + m0 + tid) : 1.0f;
+  if (p.rs_parts) {
+    // 1/rms from the producer's per-tile sums of squares: 8 lanes per row, lane l summing tiles
+    // l, l + 8, ... (loads issued together), then a fixed xor tree over the 8 lanes
+    static_assert(kDrainThreads == 8 * kNPad, "8 lanes per row");
+    const int r = tid >> 3, l = tid & 7;
+    const float* src = p.rs_parts + (m0 + r) * p.rs_nparts;
+    float t = 0.f;
+    if (r < mc)
+      for (int i0 = l; i0 < p.rs_nparts; i0 += 64) {
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = i0 + 8 * k < p.rs_nparts ? __ldcg(src + i0 + 8 * k) : 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t += v[k];
+      }
+#pragma unroll
+    for (int off = 4; off > 0; off >>= 1) t += __shfl_xor_sync(0xffffffffu, t, off);
+    if (r < mc && l == 0) rs[r] = rsqrtf(t / static_cast<float>(p.K) + p.eps);
+  } else if (tid < mc) {
+    rs[tid] = p.rs_in ? __ldcg(p.rs_in + m0 + tid) : 1.0f;
+  }
   __syncthreads();
   // epilogue inputs, all loads independent
   bool use_pre = false;
@@ -387,7 +411,7 @@ __global__ void __launch_bounds__(kDrainThreads) ssd_mid_reduce_kernel(const Gem
     reinterpret_cast<float4*>(outb)[f] = sum;
   }
   __syncthreads();
-  gemv_epilogue<kNPad, EPI>(p, rt, outb, rs, use_pre ? pre : nullptr, base_pos, rpos, rreq, tid, m0, mc);
+  gemv_epilogue<kNPad, EPI, true>(p, rt, outb, rs, use_pre ? pre : nullptr, base_pos, rpos, rreq, tid, m0, mc);
   if constexpr (EPI == Epi::ARGMAX) gemv_argmax_finish(p, rreq, tid, p.n_rt, m0, mc);
 }
 

@@ -213,6 +213,7 @@ __global__ void __launch_bounds__(kTcThreads, 1)
           }
         }
       }
+      if (*reinterpret_cast<volatile int*>(abort_flag)) drain_ring(full, kStagesT, g);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -464,6 +465,7 @@ __global__ void __launch_bounds__(kFaThreads, 1)
         tma_load_2d(smem + S::kQh + a * S::kQAtom, &mqh, q_full, h * DH + a * 64, q0);
         tma_load_2d(smem + S::kQl + a * S::kQAtom, &mql, q_full, h * DH + a * 64, q0);
       }
+      int issued = 0;
       for (int j = 0; j < n_kb; ++j) {
         const int b = j & 1;
         if (j >= 2 && !mbar_wait(&kv_empty[b], static_cast<uint32_t>((j - 2) >> 1) & 1u)) {
@@ -479,6 +481,11 @@ __global__ void __launch_bounds__(kFaThreads, 1)
         }
         tma_load_2d(sb + S::kVh, &mvh, &kv_full[b], j * kFaK, h * DH);
         tma_load_2d(sb + S::kVl, &mvl, &kv_full[b], j * kFaK, h * DH);
+        issued = j + 1;
+      }
+      if (__ldcg(&st->error) & DERR_TIMEOUT) {  // a wait gave up somewhere: bounded waits for the copies
+        mbar_wait_for(q_full, 0u, 100000000ull);
+        drain_ring(kv_full, 2, issued);
       }
     }
   } else if (warp == 1) {
