@@ -21,20 +21,24 @@
 //    (issued ahead of the upstream wait), the B tiles through a 3-stage ring of
 //    2 x NP x 128 B fed by warp 6, so the weight stream keeps 8 units in flight
 //    whatever the B ring holds;
-//  * a row tile's accumulator is NP TMEM columns (two 128-column buffers), read
-//    back 16 columns -- 16 activation rows -- at a time by warps 2..5 and stored
-//    as the CTA's partial of that tile;
+//  * one MMA of N = 2 NP per 16-column K slice takes a stage's hi rows and the
+//    lo rows stored right after them, so a row tile's accumulator is 2 NP TMEM
+//    columns (two buffers of up to 256), the hi products in the first NP and the
+//    lo products in the last NP; warps 2..5 read back 16 columns -- 16
+//    activation rows -- of each half at a time and store their sum as the CTA's
+//    partial of that tile;
 //  * the reduction and the fused epilogue run in a second kernel,
 //    ssd_mid_reduce_kernel, one CTA per (row tile, 16-row chunk): a tile's 112
 //    rows are finished by 7 CTAs at once instead of one CTA's 128 threads after
 //    the stream (measured: about 3 us per 16-row chunk, which made the serial
 //    tail as long as the stream itself).
-// The per-element arithmetic is the GEMV's: a = hi + lo, 4 K slices x (hi, lo)
-// MMAs per unit accumulating in fp32, the RMSNorm scale applied after the
-// products, and the split-tile sums in CTA order.  The grid is its own (one CTA
-// per SM), so the split points differ from the GEMV's: a row through this kernel
-// equals the same row through the GEMV up to rounding, and every row is still
-// independent of the launch's other rows.
+// The per-element arithmetic is the GEMV's up to rounding order: a = hi + lo,
+// fp32 accumulation, the RMSNorm scale applied after the products, and the
+// split-tile sums in CTA order; the hi and lo products accumulate separately
+// over a CTA's K range and are added at the drain.  The grid is its own (one CTA
+// per SM), so the split points differ from the GEMV's too: a row through this
+// kernel equals the same row through the GEMV up to rounding, and every row is
+// still independent of the launch's other rows.
 #pragma once
 
 #include "gemv.cuh"
@@ -45,15 +49,16 @@ constexpr int kMidWStages = 8;      // weight ring
 constexpr int kMidBStages = 3;      // activation (B) ring
 constexpr int kMidCtasPerSm = 1;
 constexpr int kMidThreads = 224;    // warp 0 weight TMA, warp 1 MMA + TMEM, warps 2..5 drain, warp 6 B TMA
-constexpr int kMidTmemCols = 256;   // two 128-column accumulators
+constexpr int kMidTmemCols = 512;   // two accumulators of up to 256 columns (hi rows, then lo rows)
 constexpr uint32_t kMidBBytes = kMaxMidRows * kTileK * 2;  // one B part (hi or lo) of up to 128 rows: 16 KB
 constexpr int kMidSlot = kMaxMidRows * kTileN;             // floats of one partial row tile, [m][128]
 
 struct MidSmem {
   static constexpr int kW = 0;                                  // [wstages][16 KB] weight units
-  static constexpr int kBh = kW + kMidWStages * kWTileBytes;    // [bstages][NP][64] bf16 hi
-  static constexpr int kBl = kBh + kMidBStages * kMidBBytes;    // [bstages][NP][64] bf16 lo
-  static constexpr int kBar = kBl + kMidBStages * kMidBBytes;  // wfull, wempty [wstages]; bfull, bempty [bstages]; afull, aempty [2]
+  // [bstages][2 NP][64] bf16: a stage holds the NP hi rows, then the NP lo rows right after them,
+  // so one MMA of N = 2 NP takes both parts
+  static constexpr int kB = kW + kMidWStages * kWTileBytes;
+  static constexpr int kBar = kB + kMidBStages * 2 * kMidBBytes;  // wfull, wempty [wstages]; bfull, bempty [bstages]; afull, aempty [2]
   static constexpr int kTmemSlot = kBar + (2 * kMidWStages + 2 * kMidBStages + 4) * 8;
   static constexpr int kTotal = kTmemSlot + 16 + 1024;          // + slack for the 1024-byte alignment
 };
@@ -210,7 +215,7 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
     if (lane == 0) {
-      const uint32_t idesc = umma_idesc_bf16(kTileN, NP);
+      const uint32_t idesc = umma_idesc_bf16(kTileN, 2 * NP);
       int sg = 0;
       bool seg_open = false;
       uint32_t d = tmem;
@@ -223,7 +228,7 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
             break;
           }
           tmem_fence_after();
-          d = tmem + static_cast<uint32_t>(b * kMaxMidRows);
+          d = tmem + static_cast<uint32_t>(b * 2 * kMaxMidRows);
         }
         if (!mbar_wait(&wfull[s], static_cast<uint32_t>(i / kMidWStages) & 1u) ||
             !mbar_wait(&bfull[sb], static_cast<uint32_t>(i / kMidBStages) & 1u)) {
@@ -232,13 +237,12 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         }
         tmem_fence_after();
         const uint64_t adesc = umma_desc_sw128(smem_u32(smem + S::kW + s * kWTileBytes));
-        const uint64_t hdesc = umma_desc_sw128(smem_u32(smem + S::kBh + sb * kMidBBytes));
-        const uint64_t ldesc = umma_desc_sw128(smem_u32(smem + S::kBl + sb * kMidBBytes));
+        const uint64_t bdesc = umma_desc_sw128(smem_u32(smem + S::kB + sb * 2 * kMidBBytes));
 #pragma unroll
         for (int kk = 0; kk < kTileK / 16; ++kk) {
-          // +32 bytes (2 descriptor units) per 16-element K slice inside the swizzled row
-          umma_f16(d, adesc + 2 * kk, hdesc + 2 * kk, idesc, (seg_open || kk > 0) ? 1u : 0u);
-          umma_f16(d, adesc + 2 * kk, ldesc + 2 * kk, idesc, 1u);
+          // +32 bytes (2 descriptor units) per 16-element K slice inside the swizzled row; columns
+          // 0..NP-1 of the accumulator take the hi products, NP..2NP-1 the lo products
+          umma_f16(d, adesc + 2 * kk, bdesc + 2 * kk, idesc, (seg_open || kk > 0) ? 1u : 0u);
           seg_open = true;
         }
         umma_commit(&wempty[s]);  // the stages may be refilled once these MMAs have read them
@@ -265,8 +269,9 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         }
         const int x = ((u0 + i) % p.n_kt) * kTileK;
         mbar_arrive_expect_tx(&bfull[sb], 2 * bbytes);
-        tma_load_2d(smem + S::kBh + sb * kMidBBytes, &map_hi, &bfull[sb], x, 0);
-        tma_load_2d(smem + S::kBl + sb * kMidBBytes, &map_lo, &bfull[sb], x, 0);
+        uint8_t* bdst = smem + S::kB + sb * 2 * kMidBBytes;
+        tma_load_2d(bdst, &map_hi, &bfull[sb], x, 0);
+        tma_load_2d(bdst + bbytes, &map_lo, &bfull[sb], x, 0);
       }
       if (__ldcg(&p.st->error) & DERR_TIMEOUT) drain_ring(bfull, kMidBStages, issued);
     }
@@ -288,14 +293,16 @@ __global__ void __launch_bounds__(kMidThreads, kMidCtasPerSm)
         break;
       }
       tmem_fence_after();
-      const uint32_t tbase = tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * kMaxMidRows);
+      const uint32_t tbase =
+          tmem + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(b * 2 * kMaxMidRows);
       float* dstp = p.partials + static_cast<size_t>(c + rt) * kMidSlot;
       for (int ch = 0; ch < n_ch; ++ch) {
-        float v[kNPad];
+        float v[kNPad], vl[kNPad];
         tmem_ld16(tbase + ch * kNPad, v);
+        tmem_ld16(tbase + NP + ch * kNPad, vl);
 #pragma unroll
         for (int m = 0; m < kNPad; ++m)
-          if (ch * kNPad + m < M) __stcg(dstp + (ch * kNPad + m) * kTileN + q * 32 + lane, v[m]);
+          if (ch * kNPad + m < M) __stcg(dstp + (ch * kNPad + m) * kTileN + q * 32 + lane, v[m] + vl[m]);
       }
       tmem_fence_before();
       __syncwarp();
