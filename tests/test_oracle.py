@@ -103,6 +103,61 @@ def test_imitation_network_matches_torch(tiny_bits):
     np.testing.assert_allclose(oracle.imitation(m, x), ref.numpy(), rtol=1e-12, atol=1e-12)
 
 
+def torch_xk_rows(m: oracle.Model, vis: np.ndarray, tokens, k: int) -> torch.Tensor:
+    """No-cache torch forward of rows [z; embed(tokens)] through layers 0..k-1: x_k of every row."""
+    c, W = m.cfg, m.w
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    H, Dh, half = c.n_heads, c.head_dim, c.head_dim // 2
+    X = torch.cat([t(vis), t(W["embed"])[torch.as_tensor(np.asarray(tokens, dtype=np.int64))]], 0)
+    P = X.shape[0]
+    inv = c.rope_theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / Dh)
+    rot = torch.polar(torch.ones(P, half, dtype=torch.float64), torch.arange(P, dtype=torch.float64)[:, None] * inv)
+
+    def rope_c(Z):
+        z = torch.complex(Z[..., :half], Z[..., half:]) * rot[:, None, :]
+        return torch.cat([z.real, z.imag], -1)
+
+    for l in range(k):
+        lw = {n: t(v) for n, v in W["layers"][l].items()}
+        N = F.rms_norm(X, (c.d_model,), lw["attn_norm"], c.rms_eps)
+        Q = rope_c((N @ lw["wq"].T).view(P, H, Dh)).transpose(0, 1)
+        K = rope_c((N @ lw["wk"].T).view(P, H, Dh)).transpose(0, 1)
+        V = (N @ lw["wv"].T).view(P, H, Dh).transpose(0, 1)
+        O = F.scaled_dot_product_attention(Q[None], K[None], V[None], is_causal=True)[0]
+        X = X + m.s[l] * (O.transpose(0, 1).reshape(P, H * Dh) @ lw["wo"].T)
+        U = F.rms_norm(X, (c.d_model,), lw["ffn_norm"], c.rms_eps)
+        X = X + m.s[l] * ((F.silu(U @ lw["w_gate"].T) * (U @ lw["w_up"].T)) @ lw["w_down"].T)
+    return X
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.2, 3)])
+def test_mlp2_draft_logits_match_torch_no_cache_forward(tiny_bits, s, gamma):
+    """Every draft row of every SSD step, g(I(x_k)) with the MLP2 imitation at k < L, equals a no-cache
+    torch forward of the sequence as it stands at that step (the emitted tokens, then the step's own
+    drafts): the cached shallow layers, the row and position each draft reads, and the rollback of
+    rejected drafts' cache rows all show up in it."""
+    w = tiny(s=s, gamma=gamma, max_new=14)
+    m, vis, prompt = build(w, tiny_bits)
+    c = m.cfg
+    assert c.draft_exit_k < c.n_layers
+    r = oracle.ssd_generate(m, vis, prompt, w.max_new, gamma, keep_draft_logits=True)
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    n_vis, emitted = vis.shape[0], 1
+    for step, (drafts, dlog) in enumerate(zip(r.draft_tokens, r.draft_logits)):
+        seq = list(prompt) + r.tokens[:emitted] + list(drafts[:-1])
+        X = torch_xk_rows(m, vis, seq, c.draft_exit_k)
+        row0 = n_vis + len(prompt) + emitted - 1          # the last emitted token's row
+        for j in range(len(drafts)):
+            x = X[row0 + j]
+            n = F.rms_norm(x, (c.d_model,), t(m.w["in_norm"]), c.rms_eps)
+            xi = x + m.s_in * (t(m.w["in_w2"]) @ F.silu(t(m.w["in_w1"]) @ n))
+            ref = t(m.w["lm_head"]) @ F.rms_norm(xi, (c.d_model,), t(m.w["final_norm"]), c.rms_eps)
+            np.testing.assert_allclose(dlog[j], ref.numpy(), rtol=1e-9, atol=1e-9, err_msg=f"step {step} row {j}")
+            assert drafts[j] == int(np.argmax(dlog[j]))
+        emitted += r.accept_lengths[step] + 1
+    assert len(r.draft_tokens) >= 3 and sum(r.accept_lengths) > 0 if s < 0.1 else True
+
+
 # --------------------------------------------------------------------------- closed forms
 
 def test_rope_position_zero_is_identity_and_norm_preserving():
