@@ -292,8 +292,8 @@ def test_standalone_draft_and_verify_steps(tiny_model, tiny_bits):
     assert_accept_sequence(model, ref, toks)
 
 
-@pytest.mark.parametrize("case", ["ragged_prefill", "vocab_tail", "no_visual", "head128", "narrow_in",
-                                  "max_new_1", "max_new_2"])
+@pytest.mark.parametrize("case", ["ragged_prefill", "vocab_tail", "no_visual", "head128", "head128_short",
+                                  "narrow_in", "max_new_1", "max_new_2"])
 def test_edge_shapes(case):
     base = synth.TINY.replace(norm_gain="perturbed", s=0.2)
     w = {
@@ -301,6 +301,10 @@ def test_edge_shapes(case):
         "vocab_tail": base.replace(shape=synth.ModelShape(4, 256, 4, 64, 1024, 2000)),
         "no_visual": base.replace(n_vis=0, n_prompt=21),
         "head128": base.replace(shape=synth.ModelShape(3, 256, 2, 128, 512, 1024), draft_exit_k=1),
+        # 5 prompt rows: the first decode steps see at most one 32-key chunk (CTA 0 finishes the
+        # head alone), later ones several (the split-KV merge), within one SSD step too
+        "head128_short": base.replace(shape=synth.ModelShape(3, 256, 2, 128, 512, 1024), draft_exit_k=1,
+                                      n_vis=0, n_prompt=5),
         "narrow_in": base.replace(in_hidden=192),
         "max_new_1": base.replace(max_new=1),
         "max_new_2": base.replace(max_new=2),
