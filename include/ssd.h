@@ -337,8 +337,11 @@ SSD_API ssd_status ssd_last_launch_count(ssd_ctx* ctx, int64_t* prefill_launches
  * full-depth pass (the medium-M tensor-core kernel beyond 16 rows), and
  * accepts / rolls back each request on its own.  A request that is done (max_new
  * tokens or eos) keeps its tokens; its rows ride along unused until every request
- * is done.  Every request's tokens and accept lengths are those of the same
- * request decoded alone.  The single-request calls (ssd_prefill .. ssd_verify)
+ * is done.  Every request's rows are computed independently of the other
+ * requests', so its tokens and accept lengths are those of the same request
+ * decoded alone; beyond 16 verification rows the medium-M kernel's own split
+ * points round differently from the GEMV's, so there they agree up to logits
+ * that tie within rounding.  The single-request calls (ssd_prefill .. ssd_verify)
  * and the batched calls share the cache: a prefill of one kind invalidates the
  * other kind's decode state. */
 
