@@ -130,19 +130,15 @@ def torch_xk_rows(m: oracle.Model, vis: np.ndarray, tokens, k: int) -> torch.Ten
     return X
 
 
-@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.2, 3)])
-def test_mlp2_draft_logits_match_torch_no_cache_forward(tiny_bits, s, gamma):
-    """Every draft row of every SSD step, g(I(x_k)) with the MLP2 imitation at k < L, equals a no-cache
-    torch forward of the sequence as it stands at that step (the emitted tokens, then the step's own
-    drafts): the cached shallow layers, the row and position each draft reads, and the rollback of
-    rejected drafts' cache rows all show up in it."""
-    w = tiny(s=s, gamma=gamma, max_new=14)
-    m, vis, prompt = build(w, tiny_bits)
+def mlp2_draft_path_error(m: oracle.Model, vis: np.ndarray, prompt, max_new: int, gamma: int) -> tuple[float, int]:
+    """Runs ssd_generate and compares every draft row g(I(x_k)) of every step with a no-cache torch
+    forward of the sequence as it stands at that step (the emitted tokens, then the step's own
+    drafts) through layers 0..k-1, the MLP2 imitation and the head.  Returns the largest absolute
+    difference relative to the row's scale, and the number of rows compared."""
     c = m.cfg
-    assert c.draft_exit_k < c.n_layers
-    r = oracle.ssd_generate(m, vis, prompt, w.max_new, gamma, keep_draft_logits=True)
+    r = oracle.ssd_generate(m, vis, prompt, max_new, gamma, keep_draft_logits=True)
     t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
-    n_vis, emitted = vis.shape[0], 1
+    n_vis, emitted, worst, rows = vis.shape[0], 1, 0.0, 0
     for step, (drafts, dlog) in enumerate(zip(r.draft_tokens, r.draft_logits)):
         seq = list(prompt) + r.tokens[:emitted] + list(drafts[:-1])
         X = torch_xk_rows(m, vis, seq, c.draft_exit_k)
@@ -151,11 +147,25 @@ def test_mlp2_draft_logits_match_torch_no_cache_forward(tiny_bits, s, gamma):
             x = X[row0 + j]
             n = F.rms_norm(x, (c.d_model,), t(m.w["in_norm"]), c.rms_eps)
             xi = x + m.s_in * (t(m.w["in_w2"]) @ F.silu(t(m.w["in_w1"]) @ n))
-            ref = t(m.w["lm_head"]) @ F.rms_norm(xi, (c.d_model,), t(m.w["final_norm"]), c.rms_eps)
-            np.testing.assert_allclose(dlog[j], ref.numpy(), rtol=1e-9, atol=1e-9, err_msg=f"step {step} row {j}")
+            ref = (t(m.w["lm_head"]) @ F.rms_norm(xi, (c.d_model,), t(m.w["final_norm"]), c.rms_eps)).numpy()
+            worst = max(worst, float(np.max(np.abs(dlog[j] - ref)) / max(1.0, float(np.max(np.abs(ref))))))
             assert drafts[j] == int(np.argmax(dlog[j]))
+            rows += 1
         emitted += r.accept_lengths[step] + 1
-    assert len(r.draft_tokens) >= 3 and sum(r.accept_lengths) > 0 if s < 0.1 else True
+    return worst, rows
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.2, 3)])
+def test_mlp2_draft_logits_match_torch_no_cache_forward(tiny_bits, s, gamma):
+    """Every draft row of every SSD step, g(I(x_k)) with the MLP2 imitation at k < L, equals a no-cache
+    torch forward of the sequence at that step: the cached shallow layers, the row and position each
+    draft reads, and the rollback of rejected drafts' cache rows all show up in it.  (SSD == greedy
+    cannot see a wrong draft: drafts only change how many tokens a step accepts.)"""
+    w = tiny(s=s, gamma=gamma, max_new=14)
+    m, vis, prompt = build(w, tiny_bits)
+    assert m.cfg.draft_exit_k < m.cfg.n_layers
+    err, rows = mlp2_draft_path_error(m, vis, prompt, w.max_new, gamma)
+    assert rows >= 12 and err < 1e-9, (err, rows)
 
 
 # --------------------------------------------------------------------------- closed forms

@@ -11,7 +11,7 @@ import pytest
 import oracle
 import oracle.ssd_oracle as so
 import synth
-from tests.test_oracle import build, tiny, torch_logits_all_rows
+from tests.test_oracle import build, mlp2_draft_path_error, tiny, torch_logits_all_rows
 
 
 def _rope_wrong_sign(v, pos, theta):
@@ -127,3 +127,22 @@ def test_encoder_decoder_cross_cache_from_unnormed_output_is_caught(monkeypatch)
     got = [T.lm_head(m, T.dec_forward_row(m, m.w["embed"][y].copy(), pos, cache, range(m.cfg.n_dec)))
            for pos, y in enumerate([m.cfg.start_token] + toks)]
     assert not np.allclose(np.stack(got), ref, rtol=1e-6, atol=1e-6)
+
+
+def _imitation_no_residual(m, x, *rest):
+    n = so.rms_norm(x, m.w["in_norm"], m.cfg.rms_eps)
+    return m.s_in * (m.w["in_w2"] @ so.silu(m.w["in_w1"] @ n))
+
+
+def test_draft_path_mistake_passes_ssd_equals_greedy_but_not_the_draft_pin(monkeypatch):
+    """An imitation network without its residual still gives SSD == greedy (the verification corrects
+    every draft), so only the draft-path pin can catch it."""
+    w = tiny(s=0.05, gamma=4, max_new=14)
+    m, vis, prompt = build(w)
+    g = so.greedy_generate(m, vis, prompt, w.max_new)
+    err, _ = mlp2_draft_path_error(m, vis, prompt, w.max_new, w.gamma)
+    assert err < 1e-9
+    monkeypatch.setattr(so, "imitation", _imitation_no_residual)
+    assert so.ssd_generate(m, vis, prompt, w.max_new, w.gamma).tokens == g.tokens
+    err, _ = mlp2_draft_path_error(m, vis, prompt, w.max_new, w.gamma)
+    assert err > 1e-3
