@@ -87,8 +87,9 @@ def _torch_bias(table: torch.Tensor, n_q: int, n_k: int, bidirectional: bool) ->
     return table[bucket].permute(2, 0, 1)
 
 
-def torch_forward(m: T.T5Model, z: np.ndarray, prompt, dec_tokens) -> np.ndarray:
-    """Logits of every decoder row for decoder inputs [start; dec_tokens] (no cache)."""
+def torch_forward(m: T.T5Model, z: np.ndarray, prompt, dec_tokens, n_dec: int | None = None):
+    """Logits of every decoder row for decoder inputs [start; dec_tokens] (no cache); with n_dec, the
+    hidden rows after decoder layers 0..n_dec-1 instead."""
     c, W = m.cfg, m.w
     t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
     H, Dh, d = c.n_heads, c.head_dim, c.d_model
@@ -117,7 +118,7 @@ def torch_forward(m: T.T5Model, z: np.ndarray, prompt, dec_tokens) -> np.ndarray
     S = Y.shape[0]
     causal = torch.triu(torch.full((S, S), float("-inf"), dtype=torch.float64), 1)
     db = (_torch_bias(t(W["dec_rel"]), S, S, False) + causal)[None]
-    for l in range(c.n_dec):
+    for l in range(c.n_dec if n_dec is None else n_dec):
         lw = {k: t(v) for k, v in W["dec"][l].items()}
         s = m.s[l]
         N = F.rms_norm(Y, (d,), lw["self_norm"], c.eps)
@@ -129,6 +130,8 @@ def torch_forward(m: T.T5Model, z: np.ndarray, prompt, dec_tokens) -> np.ndarray
                                            scale=1.0)[0]
         Y = Y + s * (O.transpose(0, 1).reshape(S, H * Dh) @ lw["co"].T)
         Y = Y + s * mlp(lw, Y)
+    if n_dec is not None:
+        return Y
     Yn = F.rms_norm(Y, (d,), t(W["dec_final"]), c.eps)
     return (Yn @ t(W["lm_head"]).T).numpy()
 
@@ -144,6 +147,34 @@ def test_greedy_logits_match_torch_no_cache_forward(tiny_model):
     ref = torch_forward(m, z, prompt, r.tokens[:-1])
     np.testing.assert_allclose(np.stack(r.logits), ref, rtol=1e-9, atol=1e-9)
     assert r.tokens == [int(np.argmax(row)) for row in ref]
+
+
+@pytest.mark.parametrize("s,gamma", [(0.05, 4), (0.3, 3)])
+def test_draft_tokens_match_torch_no_cache_forward(s, gamma):
+    """Every drafted token of every SSD step is the argmax of g(I(x_k)) for x_k from a no-cache torch
+    forward through decoder layers 0..k-1 of the sequence at that step (the emitted tokens, then the
+    step's own drafts), the MLP2 imitation and the head: the draft path's cache rows, positions and
+    rollback, which SSD == greedy cannot see.  Rows whose top two logits are within 1e-9 are skipped."""
+    w = tiny(s=s, max_new=16)
+    m, z, prompt = build(w)
+    c = m.cfg
+    assert 0 < c.draft_exit_k < c.n_dec
+    r = T.ssd_generate(m, z, prompt, w.max_new, gamma)
+    t = lambda a: torch.from_numpy(np.asarray(a, dtype=np.float64))
+    p, checked = 1, 0
+    for step, drafts in enumerate(r.draft_tokens):
+        Y = torch_forward(m, z, prompt, r.tokens[:p] + list(drafts[:-1]), n_dec=c.draft_exit_k)
+        for j, d in enumerate(drafts):
+            x = Y[p + j]
+            n = F.rms_norm(x, (c.d_model,), t(m.w["in_norm"]), c.eps)
+            xi = x + m.s_in * (t(m.w["in_w2"]) @ F.silu(t(m.w["in_w1"]) @ n))
+            o = (t(m.w["lm_head"]) @ F.rms_norm(xi, (c.d_model,), t(m.w["dec_final"]), c.eps)).numpy()
+            top = np.sort(o)[-2:]
+            if top[1] - top[0] > 1e-9:
+                assert d == int(np.argmax(o)), (step, j)
+                checked += 1
+        p = r.kv_lens[step]
+    assert checked >= 8
 
 
 def test_encoder_is_bidirectional_and_decoder_causal(tiny_model):
@@ -263,3 +294,18 @@ def test_ssd_dynamic_draft_length_equals_greedy(s, cap, n_max):
         assert len(r.draft_tokens[step]) == g and 0 <= a <= g
         p += a + 1
         n += a + 1
+
+
+def test_draft_pin_catches_an_imitation_without_residual(monkeypatch):
+    """Planted on the CPU: SSD == greedy still holds with a broken imitation network (verification
+    corrects every draft), the draft-token pin does not."""
+    def no_residual(m, x):
+        n = T.rms_norm(x, m.w["in_norm"], m.cfg.eps)
+        return m.s_in * (m.w["in_w2"] @ T.silu(m.w["in_w1"] @ n))
+    w = tiny(s=0.05, max_new=16)
+    m, z, prompt = build(w)
+    g = T.greedy_generate(m, z, prompt, w.max_new)
+    monkeypatch.setattr(T, "imitation", no_residual)
+    assert T.ssd_generate(m, z, prompt, w.max_new, 4).tokens == g.tokens
+    with pytest.raises(AssertionError):
+        test_draft_tokens_match_torch_no_cache_forward(0.05, 4)
